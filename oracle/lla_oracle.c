@@ -1,0 +1,277 @@
+/*
+ * lla_oracle.c -- plain, slow CPU float64 oracle for Looped Latent Attention (LLA).
+ *
+ * TEST INFRASTRUCTURE ONLY.  The tests, the smoke check and the CPU-baseline leg of the
+ * benchmark are the only callers.  The CUDA library never calls, links or includes this
+ * file, and this file knows nothing about the CUDA library (no paged layout, no absorbed
+ * form, no tiling).
+ *
+ * What it computes, in the paper's notation (Sec. 3, "Looped Latent Attention"):
+ *   stacked loop vector   x = [x_1; ...; x_T] in R^{T d}          ("Teacher cache")
+ *   encode                c = (x - mu) W_down,  W_down in R^{Td x r}      (Eq. encode)
+ *   per-loop decode       xhat_t = c W_up,t^T + mu_t,  W_up,t in R^{d x r} (Eq. decode)
+ *   compression ratio     rho = 2 T d / (r_k + r_v)                       (Eq. ratio)
+ * and softmax attention over the explicitly reconstructed keys and values:
+ *   s_i = scale * q . Khat_t[i],  a = softmax(s),  o = sum_i a_i Vhat_t[i].
+ *
+ * Decode follows the two-pass cached reconstruction decoder (App. A, "Decoding and
+ * caching"): in pass 1 the current token's stacked vector is not complete yet, so at loop t
+ * it attends with its own exact loop-t key and value; in pass 2 the current token has been
+ * encoded and is read back through Eq. decode like every other cached token.
+ *
+ * Everything is double precision with plain loops in the order the equations are written.
+ * Inputs that the GPU side stores in bf16 are passed here already widened (exactly) to
+ * double.  No fused or reordered arithmetic beyond what the equations state; OpenMP only
+ * runs independent (sequence, head, loop) problems side by side.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Eq. ratio: rho = 2 T H d / ((r_k + r_v) H) = 2 T d / (r_k + r_v). */
+double lla_oracle_ratio(int T, int d_head, int r_k, int r_v)
+{
+    return 2.0 * (double)T * (double)d_head / (double)(r_k + r_v);
+}
+
+/* "Teacher cache": 2 T H d scalars per token per layer (K and V of every loop and head). */
+double lla_oracle_teacher_cache_bytes_per_token(int T, int H, int d_head, int D, int elem_bytes)
+{
+    return 2.0 * T * H * (double)d_head * D * elem_bytes;
+}
+
+/* Eq. ratio, numerator of the compressed side: (r_k + r_v) H scalars per token per layer. */
+double lla_oracle_latent_cache_bytes_per_token(int H, int D, int r_k, int r_v, int elem_bytes)
+{
+    return (double)(r_k + r_v) * H * D * elem_bytes;
+}
+
+/*
+ * Eq. encode for N tokens of one (layer, head, axis).
+ *   x      [T][N][d]   x[t][n] is the loop-t vector of token n (loops counted from 0)
+ *   mu     [T*d]       calibration mean of the stacked vector, or NULL for mu = 0
+ *   w_down [T*d][r]
+ *   c      [N][r]      output latents
+ */
+void lla_oracle_encode(int T, int d, int r, int64_t N, const double *x, const double *mu,
+                       const double *w_down, double *c)
+{
+    const int Td = T * d;
+    double *xs = (double *)malloc(sizeof(double) * (size_t)Td);
+    for (int64_t n = 0; n < N; ++n) {
+        /* stack the loop vectors: x = [x_1; ...; x_T] */
+        for (int t = 0; t < T; ++t)
+            for (int e = 0; e < d; ++e)
+                xs[t * d + e] = x[((int64_t)t * N + n) * d + e];
+        /* centre: x - mu */
+        if (mu)
+            for (int k = 0; k < Td; ++k)
+                xs[k] = xs[k] - mu[k];
+        /* project: c = (x - mu) W_down */
+        for (int j = 0; j < r; ++j) {
+            double acc = 0.0;
+            for (int k = 0; k < Td; ++k)
+                acc += xs[k] * w_down[(int64_t)k * r + j];
+            c[n * r + j] = acc;
+        }
+    }
+    free(xs);
+}
+
+/*
+ * Eq. decode for N latents at one loop t.
+ *   c      [N][r]
+ *   w_up_t [d][r]   W_up,t
+ *   mu_t   [d]      loop-t slice of mu, or NULL
+ *   xhat   [N][d]   xhat_t = c W_up,t^T + mu_t
+ */
+void lla_oracle_reconstruct(int d, int r, int64_t N, const double *c, const double *w_up_t,
+                            const double *mu_t, double *xhat)
+{
+    for (int64_t n = 0; n < N; ++n) {
+        for (int e = 0; e < d; ++e) {
+            double acc = 0.0;
+            for (int j = 0; j < r; ++j)
+                acc += c[n * r + j] * w_up_t[(int64_t)e * r + j];
+            xhat[n * d + e] = acc + (mu_t ? mu_t[e] : 0.0);
+        }
+    }
+}
+
+/*
+ * Plain softmax attention of one query over L >= 1 keys and values.
+ *   s_i = scale * q . K[i];  a_i = exp(s_i - max s) / sum_j exp(s_j - max s);  o = sum_i a_i V[i]
+ * Returns 0, or -1 when L < 1.
+ */
+int lla_oracle_attention(int d, int64_t L, const double *q, const double *K, const double *V,
+                         double scale, double *o)
+{
+    if (L < 1)
+        return -1;
+    double *s = (double *)malloc(sizeof(double) * (size_t)L);
+    double m = -INFINITY;
+    for (int64_t i = 0; i < L; ++i) {
+        double dot = 0.0;
+        for (int e = 0; e < d; ++e)
+            dot += q[e] * K[i * d + e];
+        s[i] = scale * dot;
+        if (s[i] > m)
+            m = s[i];
+    }
+    double z = 0.0;
+    for (int64_t i = 0; i < L; ++i) {
+        s[i] = exp(s[i] - m);
+        z += s[i];
+    }
+    for (int64_t i = 0; i < L; ++i)
+        s[i] = s[i] / z; /* a_i */
+    for (int e = 0; e < d; ++e) {
+        double acc = 0.0;
+        for (int64_t i = 0; i < L; ++i)
+            acc += s[i] * V[i * d + e];
+        o[e] = acc;
+    }
+    free(s);
+    return 0;
+}
+
+/*
+ * One decode call for one (sequence, head) at loop t (0-based) of one layer.
+ *   c_k [L][r_k], c_v [L][r_v]       latents of the L cached tokens
+ *   w_up_k [T][d][r_k], w_up_v [T][d][r_v]
+ *   mu_k, mu_v [T*d] or NULL
+ *   q [d]                            loop-t query of the current token
+ *   cur_k, cur_v [d] or NULL         pass 1: the current token's exact loop-t key/value
+ *                                    pass 2 (NULL): the current token is one of the L cached
+ *   out [d]
+ * Returns 0, or -1 on bad arguments (pass 2 needs L >= 1).
+ */
+int lla_oracle_decode(int T, int d, int r_k, int r_v, int t, int64_t L, const double *c_k,
+                      const double *c_v, const double *w_up_k, const double *w_up_v,
+                      const double *mu_k, const double *mu_v, const double *q,
+                      const double *cur_k, const double *cur_v, double scale, double *out)
+{
+    if (t < 0 || t >= T || L < 0)
+        return -1;
+    if ((cur_k == NULL) != (cur_v == NULL))
+        return -1;
+    const int pass1 = cur_k != NULL;
+    if (!pass1 && L < 1)
+        return -1;
+    const int64_t n = L + (pass1 ? 1 : 0);
+    double *K = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    double *V = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    /* Eq. decode, loop t, for every cached token */
+    lla_oracle_reconstruct(d, r_k, L, c_k, w_up_k + (int64_t)t * d * r_k,
+                           mu_k ? mu_k + (int64_t)t * d : NULL, K);
+    lla_oracle_reconstruct(d, r_v, L, c_v, w_up_v + (int64_t)t * d * r_v,
+                           mu_v ? mu_v + (int64_t)t * d : NULL, V);
+    /* pass 1: the current token joins with its exact loop-t key and value */
+    if (pass1) {
+        memcpy(K + L * d, cur_k, sizeof(double) * (size_t)d);
+        memcpy(V + L * d, cur_v, sizeof(double) * (size_t)d);
+    }
+    int rc = lla_oracle_attention(d, n, q, K, V, scale, out);
+    free(K);
+    free(V);
+    return rc;
+}
+
+/*
+ * Causal prefill at loop t for one (sequence, head): the N prompt tokens are all cached as
+ * latents (pass 2 of the two-pass prefill, App. A and App. J "Eviction and long-context
+ * prefill"); query i attends to keys j <= i through Eq. decode.
+ *   q [N][d], out [N][d]
+ */
+int lla_oracle_prefill(int T, int d, int r_k, int r_v, int t, int64_t N, const double *c_k,
+                       const double *c_v, const double *w_up_k, const double *w_up_v,
+                       const double *mu_k, const double *mu_v, const double *q, double scale,
+                       double *out)
+{
+    if (t < 0 || t >= T || N < 0)
+        return -1;
+    double *K = (double *)malloc(sizeof(double) * (size_t)(N * d + 1));
+    double *V = (double *)malloc(sizeof(double) * (size_t)(N * d + 1));
+    lla_oracle_reconstruct(d, r_k, N, c_k, w_up_k + (int64_t)t * d * r_k,
+                           mu_k ? mu_k + (int64_t)t * d : NULL, K);
+    lla_oracle_reconstruct(d, r_v, N, c_v, w_up_v + (int64_t)t * d * r_v,
+                           mu_v ? mu_v + (int64_t)t * d : NULL, V);
+    int rc = 0;
+    for (int64_t i = 0; i < N && rc == 0; ++i)
+        rc = lla_oracle_attention(d, i + 1, q + i * d, K, V, scale, out + i * d);
+    free(K);
+    free(V);
+    return rc;
+}
+
+/* One independent decode problem for lla_oracle_decode_batch. */
+typedef struct {
+    int32_t t;
+    int32_t pad_;
+    int64_t L;
+    const double *c_k, *c_v, *w_up_k, *w_up_v, *mu_k, *mu_v;
+    const double *q, *cur_k, *cur_v;
+    double *out;
+} lla_oracle_decode_item;
+
+/* Runs n_items independent decode problems, n_threads at a time (<= 0: the OpenMP default).
+ * Returns 0, or the first nonzero item status. */
+int lla_oracle_decode_batch(int T, int d, int r_k, int r_v, double scale, int64_t n_items,
+                            const lla_oracle_decode_item *items, int n_threads)
+{
+    int err = 0;
+#ifdef _OPENMP
+    if (n_threads <= 0)
+        n_threads = omp_get_max_threads();
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads)
+#endif
+    for (int64_t i = 0; i < n_items; ++i) {
+        const lla_oracle_decode_item *it = &items[i];
+        int rc = lla_oracle_decode(T, d, r_k, r_v, it->t, it->L, it->c_k, it->c_v, it->w_up_k,
+                                   it->w_up_v, it->mu_k, it->mu_v, it->q, it->cur_k, it->cur_v,
+                                   scale, it->out);
+        if (rc != 0) {
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+            err = rc;
+        }
+    }
+    return err;
+}
+
+/* One (head, axis) encode problem for lla_oracle_encode_batch. */
+typedef struct {
+    int32_t r;
+    int32_t pad_;
+    const double *x, *mu, *w_down;
+    double *c;
+} lla_oracle_encode_item;
+
+int lla_oracle_encode_batch(int T, int d, int64_t N, int64_t n_items,
+                            const lla_oracle_encode_item *items, int n_threads)
+{
+#ifdef _OPENMP
+    if (n_threads <= 0)
+        n_threads = omp_get_max_threads();
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads)
+#endif
+    for (int64_t i = 0; i < n_items; ++i)
+        lla_oracle_encode(T, d, items[i].r, N, items[i].x, items[i].mu, items[i].w_down,
+                          items[i].c);
+    return 0;
+}
+
+/* Threads an unrestricted batch call would use. */
+int lla_oracle_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}

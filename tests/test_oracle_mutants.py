@@ -1,0 +1,61 @@
+"""The pins in test_oracle_pins.py must catch plausible mistakes in the oracle.
+
+Each case plants one mistake in a private copy of oracle/lla_oracle.c (compiled on the CPU
+into a temporary directory), runs the pin tests against that copy, and expects them to fail.
+The committed oracle is never modified.
+"""
+import os
+import subprocess
+import sys
+import tempfile
+from concurrent.futures import ThreadPoolExecutor
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "lla_oracle.c")
+
+# (name, exact text in the oracle, planted replacement)
+MUTANTS = [
+    ("ratio_drops_factor_2", "return 2.0 * (double)T * (double)d_head",
+     "return (double)T * (double)d_head"),
+    ("encode_wrong_stacking", "xs[t * d + e] = x[((int64_t)t * N + n) * d + e];",
+     "xs[e * T + t] = x[((int64_t)t * N + n) * d + e];"),
+    ("encode_mu_sign", "xs[k] = xs[k] - mu[k];", "xs[k] = xs[k] + mu[k];"),
+    ("decode_transposed_w_up", "acc += c[n * r + j] * w_up_t[(int64_t)e * r + j];",
+     "acc += c[n * r + j] * w_up_t[(int64_t)j * d + e];"),
+    ("decode_drops_mu_t", "xhat[n * d + e] = acc + (mu_t ? mu_t[e] : 0.0);",
+     "xhat[n * d + e] = acc;"),
+    ("decode_wrong_loop_slice",
+     "lla_oracle_reconstruct(d, r_k, L, c_k, w_up_k + (int64_t)t * d * r_k,",
+     "lla_oracle_reconstruct(d, r_k, L, c_k, w_up_k,"),
+    ("attention_drops_scale", "s[i] = scale * dot;", "s[i] = dot;"),
+    ("attention_no_max_subtraction", "s[i] = exp(s[i] - m);", "s[i] = exp(s[i]);"),
+    ("pass1_value_is_key", "memcpy(V + L * d, cur_v,", "memcpy(V + L * d, cur_k,"),
+    ("prefill_not_causal", "rc = lla_oracle_attention(d, i + 1, q + i * d, K, V, scale, out + i * d);",
+     "rc = lla_oracle_attention(d, N, q + i * d, K, V, scale, out + i * d);"),
+]
+
+
+def _run_mutant(name, old, new, tmp):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"{name}: anchor text not found exactly once"
+    path_c = os.path.join(tmp, f"{name}.c")
+    path_so = os.path.join(tmp, f"lib{name}.so")
+    with open(path_c, "w") as f:
+        f.write(src.replace(old, new))
+    subprocess.run(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-fopenmp", path_c, "-o",
+                    path_so, "-lm"], check=True)
+    env = dict(os.environ, LLA_ORACLE_LIB=path_so)
+    res = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                          os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                         cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    return name, res.returncode
+
+
+def test_pins_catch_every_planted_mistake():
+    with tempfile.TemporaryDirectory() as tmp:
+        with ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 2)) as ex:
+            results = list(ex.map(lambda m: _run_mutant(*m, tmp), MUTANTS))
+    survivors = [name for name, rc in results if rc == 0]
+    assert not survivors, f"pins did not catch: {survivors}"

@@ -1,0 +1,348 @@
+"""Pins the CPU oracle to what the paper and the mathematics fix (no GPU needed).
+
+Each test names the passage it follows.  None of them re-types the oracle's own code:
+they check it against printed values (tests/golden), closed forms, library routines that
+compute the textbook definition (torch SDPA in float64, numpy SVD), an independently
+written absorbed formulation (App. J), hand-expanded tiny cases and invariances.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import oracle
+
+GOLD = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _gold(name):
+    with open(os.path.join(GOLD, name)) as f:
+        return json.load(f)
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _orthogonal(n, seed):
+    q, r = np.linalg.qr(_rng(seed).standard_normal((n, n)))
+    return q * np.sign(np.diag(r))
+
+
+def _sdpa(q, K, V, scale, causal=False):
+    """torch's float64 scaled-dot-product attention (textbook softmax attention)."""
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float64))
+    qq = t(q).reshape(1, 1, -1, K.shape[1])
+    out = F.scaled_dot_product_attention(qq, t(K)[None, None], t(V)[None, None],
+                                         is_causal=causal, scale=scale)
+    return out[0, 0].numpy()
+
+
+def _random_codec(T, d, r_k, r_v, seed, with_mu=True):
+    g = _rng(seed)
+    return dict(
+        w_up_k=g.standard_normal((T, d, r_k)) / math.sqrt(r_k),
+        w_up_v=g.standard_normal((T, d, r_v)) / math.sqrt(r_v),
+        mu_k=g.standard_normal(T * d) if with_mu else None,
+        mu_v=g.standard_normal(T * d) if with_mu else None,
+    )
+
+
+# ------------------------------------------------------------------ Eq. ratio (Sec. 3)
+
+@pytest.mark.parametrize("table", ["tier4", "huginn", "isocache"])
+def test_ratio_matches_printed_values(table):
+    g = _gold("ratios.json")[table]
+    for r_k, r_v, printed in g["rows"]:
+        rho = oracle.ratio(g["T"], g["d_head"], r_k, r_v)
+        # printed to two decimals (Huginn: integers, exact)
+        tol = 1e-12 if table == "huginn" else 0.005 + 1e-12
+        assert abs(rho - printed) <= tol, (r_k, r_v, rho, printed)
+
+
+def test_cache_bytes_match_table_memory():
+    g = _gold("cache_bytes.json")
+    for row in g["per_token_kib"]:
+        teacher = oracle.teacher_cache_bytes_per_token(4, 16, 128, row["D"], 2) / 1024
+        lla4 = oracle.latent_cache_bytes_per_token(16, row["D"], 96, 160, 2) / 1024
+        lla21 = oracle.latent_cache_bytes_per_token(16, row["D"], 18, 30, 2) / 1024
+        assert (teacher, lla4, lla21) == (row["teacher"], row["lla4"], row["lla21"])
+        # the ratio of the two cache sizes is Eq. ratio exactly
+        assert teacher / lla4 == oracle.ratio(4, 128, 96, 160)
+        assert abs(teacher / lla21 - oracle.ratio(4, 128, 18, 30)) < 1e-12
+    m = g["at_1m_context_gib"]
+    gib = lambda b: b * m["tokens"] / 2**30
+    assert gib(oracle.teacher_cache_bytes_per_token(4, 16, 128, m["D"], 2)) == m["teacher"]
+    assert gib(oracle.latent_cache_bytes_per_token(16, m["D"], 96, 160, 2)) == m["lla4"]
+    assert gib(oracle.latent_cache_bytes_per_token(16, m["D"], 18, 30, 2)) == m["lla21"]
+
+
+# ------------------------------------------------------------------ Eqs. encode / decode
+
+def test_full_rank_orthogonal_codec_is_lossless():
+    """r = T d with W_down = Q orthogonal and W_up,t = the loop-t row block of Q:
+    Eq. decode(Eq. encode(x)) = x for every loop (Sec. 3)."""
+    T, d, N = 4, 128, 24
+    g = _rng(1)
+    Q = _orthogonal(T * d, 2)
+    x = g.standard_normal((T, N, d))
+    mu = g.standard_normal(T * d)
+    c = oracle.encode(x, mu, Q)
+    assert c.shape == (N, T * d)
+    for t in range(T):
+        xhat = oracle.reconstruct(c, Q[t * d:(t + 1) * d, :], mu[t * d:(t + 1) * d])
+        np.testing.assert_allclose(xhat, x[t], rtol=0, atol=1e-12)
+
+
+def test_encode_matches_stacked_projection_definition():
+    """Eq. encode with the stacking of the "Teacher cache" paragraph: the latent of token n
+    is the centred stacked vector [x_1; ...; x_T] times W_down (numpy matmul)."""
+    T, d, N, r = 4, 16, 9, 7
+    g = _rng(3)
+    x = g.standard_normal((T, N, d))
+    mu = g.standard_normal(T * d)
+    w = g.standard_normal((T * d, r))
+    stacked = np.concatenate([x[t] for t in range(T)], axis=1)  # [N][T d]
+    np.testing.assert_allclose(oracle.encode(x, mu, w), (stacked - mu) @ w, rtol=1e-13,
+                               atol=1e-12)
+    np.testing.assert_allclose(oracle.encode(x, None, w), stacked @ w, rtol=1e-13, atol=1e-12)
+
+
+def test_svd_initialised_codec_meets_eckart_young():
+    """SVD initialisation (Sec. 3, "Initialization and conversion"; App. A): centre per loop,
+    W_down = top-r right singular vectors of the stacked-loop matrix, W_up,t = its loop
+    slices.  The total squared reconstruction error is then the sum of the trailing
+    squared singular values."""
+    T, d, N, r = 4, 16, 300, 10
+    g = _rng(4)
+    spectrum = np.exp(-np.arange(T * d) / 6.0)
+    X = (g.standard_normal((N, T * d)) * spectrum) @ _orthogonal(T * d, 5)
+    mu = X.mean(axis=0)
+    _, S, Vt = np.linalg.svd(X - mu, full_matrices=False)
+    w_down = Vt[:r].T  # [T d][r]
+    x = np.stack([X[:, t * d:(t + 1) * d] for t in range(T)])  # [T][N][d]
+    c = oracle.encode(x, mu, w_down)
+    err = 0.0
+    for t in range(T):
+        xhat = oracle.reconstruct(c, w_down[t * d:(t + 1) * d, :], mu[t * d:(t + 1) * d])
+        err += np.sum((x[t] - xhat) ** 2)
+    expect = np.sum(S[r:] ** 2)
+    assert abs(err - expect) <= 1e-10 * expect
+
+
+# ------------------------------------------------------------------ attention
+
+def test_attention_matches_torch_sdpa():
+    g = _rng(6)
+    d, L = 128, 37
+    q, K, V = g.standard_normal(d), g.standard_normal((L, d)), g.standard_normal((L, d))
+    scale = 1 / math.sqrt(d)
+    np.testing.assert_allclose(oracle.attention(q, K, V, scale), _sdpa(q, K, V, scale)[0],
+                               rtol=0, atol=1e-13)
+
+
+def test_attention_large_scores_are_stable():
+    """Softmax with max subtraction: huge equal scores still give the mean."""
+    d = 4
+    q = np.full(d, 1e3)
+    K = np.ones((3, d))
+    V = np.arange(12.0).reshape(3, d)
+    np.testing.assert_allclose(oracle.attention(q, K, V, 1.0), V.mean(axis=0), atol=1e-12)
+
+
+def test_decode_tiny_case_expanded_by_hand():
+    """T=2, d=2, r_k=r_v=1, L=2 at loop t=1, with mu; softmax expanded with math.exp."""
+    w_up_k = np.array([[[1.0], [0.0]], [[2.0], [0.0]]])    # [T][d][r_k]
+    w_up_v = np.array([[[5.0], [5.0]], [[1.0], [2.0]]])    # [T][d][r_v]
+    mu_k = None
+    mu_v = np.array([7.0, 7.0, 10.0, 0.0])                 # loop-1 slice = [10, 0]
+    c_k = np.array([[1.0], [2.0]])
+    c_v = np.array([[1.0], [-1.0]])
+    q = np.array([1.0, 3.0])
+    # loop 1: Khat = [2 c_k, 0] -> s = [2, 4];  Vhat = [c_v + 10, 2 c_v]
+    v0, v1 = np.array([11.0, 2.0]), np.array([9.0, -2.0])
+    e2, e4 = math.exp(2.0), math.exp(4.0)
+    expect2 = (e2 * v0 + e4 * v1) / (e2 + e4)
+    out2 = oracle.decode(1, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, None, None, 1.0)
+    np.testing.assert_allclose(out2, expect2, rtol=0, atol=1e-14)
+    # pass 1: exact current key [0.5, 0.5] (score 2) and value [3, -3]
+    cur_k, cur_v = np.array([0.5, 0.5]), np.array([3.0, -3.0])
+    expect1 = (e2 * v0 + e4 * v1 + e2 * cur_v) / (e2 + e4 + e2)
+    out1 = oracle.decode(1, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, cur_k, cur_v, 1.0)
+    np.testing.assert_allclose(out1, expect1, rtol=0, atol=1e-14)
+
+
+def _absorbed(t, c_k, c_v, cod, q, cur_k, cur_v, scale):
+    """App. J "Absorbed attention", written independently of the oracle: the K up-projection
+    moves to the query (q~ = W_up,t^T q) and the V up-projection leaves the softmax sum."""
+    d = q.shape[0]
+    Wk, Wv = cod["w_up_k"][t], cod["w_up_v"][t]
+    mk = np.zeros(d) if cod["mu_k"] is None else cod["mu_k"][t * d:(t + 1) * d]
+    mv = np.zeros(d) if cod["mu_v"] is None else cod["mu_v"][t * d:(t + 1) * d]
+    q_lat = Wk.T @ q
+    s = scale * (c_k @ q_lat + q @ mk)
+    if cur_k is not None:
+        s = np.append(s, scale * (q @ cur_k))
+    p = np.exp(s - s.max())
+    L = c_k.shape[0]
+    o_lat = p[:L] @ c_v
+    o = Wv @ o_lat + p[:L].sum() * mv
+    if cur_k is not None:
+        o = o + p[L] * cur_v
+    return o / p.sum()
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+@pytest.mark.parametrize("with_mu", [False, True])
+def test_decode_equals_absorbed_formulation(pass1, with_mu):
+    T, d, r_k, r_v, L = 4, 128, 96, 160, 70
+    g = _rng(7)
+    cod = _random_codec(T, d, r_k, r_v, 8, with_mu)
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    q = g.standard_normal(d)
+    cur_k = g.standard_normal(d) if pass1 else None
+    cur_v = g.standard_normal(d) if pass1 else None
+    scale = 1 / math.sqrt(d)
+    for t in range(T):
+        out = oracle.decode(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], cod["mu_k"],
+                            cod["mu_v"], q, cur_k, cur_v, scale)
+        ref = _absorbed(t, c_k, c_v, cod, q, cur_k, cur_v, scale)
+        np.testing.assert_allclose(out, ref, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+def test_full_rank_decode_equals_uncompressed_attention(pass1):
+    """With the lossless full-rank codec, LLA decode is exactly uncompressed loop-t attention
+    (Sec. 3 "Teacher cache"), computed here by torch SDPA on the raw per-loop K/V."""
+    T, d, L = 4, 128, 33
+    g = _rng(9)
+    Qk, Qv = _orthogonal(T * d, 10), _orthogonal(T * d, 11)
+    xk, xv = g.standard_normal((T, L + 1, d)), g.standard_normal((T, L + 1, d))
+    mu_k, mu_v = g.standard_normal(T * d), g.standard_normal(T * d)
+    n_cached = L if pass1 else L + 1
+    c_k = oracle.encode(xk[:, :n_cached], mu_k, Qk)
+    c_v = oracle.encode(xv[:, :n_cached], mu_v, Qv)
+    w_up_k = np.stack([Qk[t * d:(t + 1) * d] for t in range(T)])
+    w_up_v = np.stack([Qv[t * d:(t + 1) * d] for t in range(T)])
+    scale = 1 / math.sqrt(d)
+    for t in range(T):
+        q = g.standard_normal(d)
+        cur_k = xk[t, L] if pass1 else None
+        cur_v = xv[t, L] if pass1 else None
+        out = oracle.decode(t, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, cur_k, cur_v, scale)
+        ref = _sdpa(q, xk[t], xv[t], scale)[0]
+        np.testing.assert_allclose(out, ref, rtol=0, atol=1e-12)
+
+
+def test_decode_special_cases():
+    T, d, r_k, r_v = 4, 128, 96, 160
+    g = _rng(12)
+    cod = _random_codec(T, d, r_k, r_v, 13)
+    scale = 1 / math.sqrt(d)
+    t = 2
+    # one cached token, pass 2: the output is that token's reconstructed value
+    c_k, c_v = g.standard_normal((1, r_k)), g.standard_normal((1, r_v))
+    q = g.standard_normal(d)
+    out = oracle.decode(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], cod["mu_k"], cod["mu_v"],
+                        q, None, None, scale)
+    vhat = oracle.reconstruct(c_v, cod["w_up_v"][t], cod["mu_v"][t * d:(t + 1) * d])[0]
+    np.testing.assert_allclose(out, vhat, rtol=0, atol=1e-12)
+    # zero query: uniform weights, the mean of the reconstructed values
+    L = 50
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    out = oracle.decode(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], cod["mu_k"], cod["mu_v"],
+                        np.zeros(d), None, None, scale)
+    vhat = oracle.reconstruct(c_v, cod["w_up_v"][t], cod["mu_v"][t * d:(t + 1) * d])
+    np.testing.assert_allclose(out, vhat.mean(axis=0), rtol=0, atol=1e-12)
+    # pass 1 with an empty cache: the current token's own value
+    cur_k, cur_v = g.standard_normal(d), g.standard_normal(d)
+    out = oracle.decode(t, np.zeros((0, r_k)), np.zeros((0, r_v)), cod["w_up_k"],
+                        cod["w_up_v"], cod["mu_k"], cod["mu_v"], q, cur_k, cur_v, scale)
+    np.testing.assert_array_equal(out, cur_v)
+    # pass 2 with an empty cache is not defined
+    with pytest.raises(ValueError):
+        oracle.decode(t, np.zeros((0, r_k)), np.zeros((0, r_v)), cod["w_up_k"],
+                      cod["w_up_v"], None, None, q, None, None, scale)
+
+
+def test_mu_shift_invariances():
+    """Shifting mu^K by delta moves every reconstructed key by delta_t: pass-2 scores all
+    shift by one constant and the output is unchanged; pass 1's exact current key does
+    not move, so there the output changes.  Shifting mu^V by delta moves every
+    reconstructed value by delta_t: the pass-2 output moves by delta_t exactly, the pass-1
+    output by (1 - a_cur) delta_t."""
+    T, d, r_k, r_v, L = 4, 128, 96, 160, 40
+    g = _rng(14)
+    cod = _random_codec(T, d, r_k, r_v, 15)
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    q, cur_k, cur_v = g.standard_normal(d), g.standard_normal(d), g.standard_normal(d)
+    delta = g.standard_normal(T * d)
+    scale = 1 / math.sqrt(d)
+    t = 1
+    dec = lambda mk, mv, ck, cv: oracle.decode(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], mk,
+                                               mv, q, ck, cv, scale)
+    base2 = dec(cod["mu_k"], cod["mu_v"], None, None)
+    np.testing.assert_allclose(dec(cod["mu_k"] + delta, cod["mu_v"], None, None), base2,
+                               rtol=0, atol=1e-12)
+    base1 = dec(cod["mu_k"], cod["mu_v"], cur_k, cur_v)
+    assert np.abs(dec(cod["mu_k"] + 3 * delta, cod["mu_v"], cur_k, cur_v) - base1).max() > 1e-3
+    dt = delta[t * d:(t + 1) * d]
+    np.testing.assert_allclose(dec(cod["mu_k"], cod["mu_v"] + delta, None, None), base2 + dt,
+                               rtol=0, atol=1e-12)
+    # pass-1 weight of the current token, from the definition of the softmax
+    Khat = oracle.reconstruct(c_k, cod["w_up_k"][t], cod["mu_k"][t * d:(t + 1) * d])
+    s = scale * np.append(Khat @ q, q @ cur_k)
+    a_cur = np.exp(s[-1] - s.max()) / np.exp(s - s.max()).sum()
+    np.testing.assert_allclose(dec(cod["mu_k"], cod["mu_v"] + delta, cur_k, cur_v),
+                               base1 + (1 - a_cur) * dt, rtol=0, atol=1e-12)
+
+
+# ------------------------------------------------------------------ prefill
+
+def test_prefill_matches_causal_sdpa_and_decode():
+    T, d, r_k, r_v, N = 4, 128, 96, 160, 45
+    g = _rng(16)
+    cod = _random_codec(T, d, r_k, r_v, 17)
+    c_k, c_v = g.standard_normal((N, r_k)), g.standard_normal((N, r_v))
+    q = g.standard_normal((N, d))
+    scale = 1 / math.sqrt(d)
+    t = 3
+    out = oracle.prefill(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], cod["mu_k"], cod["mu_v"],
+                         q, scale)
+    K = oracle.reconstruct(c_k, cod["w_up_k"][t], cod["mu_k"][t * d:(t + 1) * d])
+    V = oracle.reconstruct(c_v, cod["w_up_v"][t], cod["mu_v"][t * d:(t + 1) * d])
+    np.testing.assert_allclose(out, _sdpa(q, K, V, scale, causal=True), rtol=0, atol=1e-12)
+    for i in (0, 1, 17, N - 1):
+        row = oracle.decode(t, c_k[:i + 1], c_v[:i + 1], cod["w_up_k"], cod["w_up_v"],
+                            cod["mu_k"], cod["mu_v"], q[i], None, None, scale)
+        np.testing.assert_allclose(out[i], row, rtol=0, atol=1e-12)
+
+
+# ------------------------------------------------------------------ batched drivers
+
+def test_batched_drivers_equal_single_calls():
+    T, d, r_k, r_v = 4, 32, 12, 20
+    g = _rng(18)
+    cod = _random_codec(T, d, r_k, r_v, 19)
+    scale = 0.3
+    items = []
+    for k in range(9):
+        L = int(g.integers(0, 20))
+        pass1 = L == 0 or k % 2 == 0
+        items.append(dict(t=k % T, c_k=g.standard_normal((L, r_k)),
+                          c_v=g.standard_normal((L, r_v)), q=g.standard_normal(d),
+                          cur_k=g.standard_normal(d) if pass1 else None,
+                          cur_v=g.standard_normal(d) if pass1 else None, **cod))
+    outs = oracle.decode_batch(T, d, r_k, r_v, scale, items, n_threads=3)
+    for it, o in zip(items, outs):
+        ref = oracle.decode(it["t"], it["c_k"], it["c_v"], cod["w_up_k"], cod["w_up_v"],
+                            cod["mu_k"], cod["mu_v"], it["q"], it["cur_k"], it["cur_v"], scale)
+        np.testing.assert_array_equal(o, ref)
+    enc_items = [dict(x=g.standard_normal((T, 5, d)), mu=g.standard_normal(T * d),
+                      w_down=g.standard_normal((T * d, r))) for r in (3, 8)]
+    for it, c in zip(enc_items, oracle.encode_batch(T, d, enc_items, n_threads=2)):
+        np.testing.assert_array_equal(c, oracle.encode(it["x"], it["mu"], it["w_down"]))
