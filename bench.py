@@ -1,0 +1,511 @@
+#!/usr/bin/env python
+"""Benchmark of the LLA decode hot path on GB300.
+
+One step = one decode step of the Ouro-shaped workload: pass 1 of the cached reconstruction
+decoder over every (loop, layer) call (T*D calls of lla_decode_attn, the current token attending
+with its exact loop-t K/V), then lla_encode of the B completed tokens in every layer (D calls).
+Inputs (latent cache, codec, queries, current K/V) are resident in HBM when the timed region
+starts; the latent cache (9.7 GB for ouro14_rho4) is far larger than L2, so no flush is needed.
+
+Prints one JSON line (rank 0).  `value` is tokens/s over all ranks (each rank decodes its own
+batch: weak scaling, no collective on the data path).  `roofline` is for the decode kernel:
+algorithmic bytes per launch over its average launch time, measured with CUDA events around the
+decode calls of every timed step.  `e2e` repeats the step through the C ABI with the step's
+inputs copied from pinned host memory and the outputs copied back inside the timed region.
+`cpu_baseline` (and `--impl reference`) time the CPU float64 oracle on a bounded sample.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "LLA decode-attn tokens/s, Ouro-1.4B shape, rho=4; HBM GB/s as % of peak"
+FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="ouro14_rho4")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0,
+                   help="target CPU time of the oracle sample")
+    return p.parse_args()
+
+
+# ------------------------------------------------------------------------------------ helpers
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def decode_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in ("paper_2607_15456_gb300/csrc/lla_decode.cu", "paper_2607_15456_gb300/csrc/lla_device.cuh"):
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload: str):
+    """DRAM bytes per decode launch from the committed ncu summary, if it was taken on the
+    current kernel source and on this workload (else None)."""
+    path = os.path.join(ROOT, "profiles", "decode_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        ent = d.get(workload)
+        if ent and ent.get("kernel_src_sha") == decode_source_hash():
+            return float(ent["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        time.sleep(0.3)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append((time.time(), line.strip()))
+
+    def mark(self, begin: bool):
+        if begin:
+            self.t0 = time.time()
+        else:
+            self.t1 = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return {"samples": 0, "note": "nvidia-smi unavailable"}
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        inside = [r for t, r in self.rows if self.t0 is not None and self.t0 <= t <= (self.t1 or t)]
+        use = inside or [r for _, r in self.rows[-3:]]
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in use:
+            parts = [x.strip() for x in r.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        out = {"sm_mhz": statistics.median(sm) if sm else None,
+               "sm_max_mhz": max(smax) if smax else None,
+               "reasons": sorted(reasons), "samples": len(sm),
+               "samples_inside_timed_region": len(inside)}
+        return out
+
+
+# ------------------------------------------------------------------------------- our arm
+
+class DecodeBench:
+    def __init__(self, wname: str, device):
+        import torch
+        from paper_2607_15456_gb300 import lla
+        from paper_2607_15456_gb300 import workloads as W
+
+        self.torch, self.lla, self.W = torch, lla, W
+        w = W.WORKLOADS[wname]
+        self.w = w
+        self.device = device
+        self.geom = lla.Geometry(w.T, w.H, w.d, w.r_k, w.r_v, w.storage)
+        self.lens = W.context_lengths(w)
+        self.B = len(self.lens)
+        # one page table for all layers (the next token's page is allocated too)
+        self.pt = W.page_table(self.lens, w.seed, extra_tokens=1)
+        self.table = self.pt.block_table.to(device)
+        bb = lla.lla_cache_block_bytes(self.geom)
+        self.codecs, self.caches, self.pools = [], [], []
+        slots_all = torch.cat([self.pt.slots(b, range(L)) for b, L in enumerate(self.lens)])
+        seq_of_tok = torch.cat([torch.full((L,), b) for b, L in enumerate(self.lens)])
+        chunk = 1 << 17
+        N = slots_all.numel()
+        for l in range(w.D):
+            cod = W.codec_tensors(w.T, w.H, w.d, w.r_k, w.r_v, w.seed, l, dtype=torch.bfloat16,
+                                  device=device)
+            codec = lla.Codec(**cod)
+            pool = torch.empty(self.pt.num_blocks * bb, dtype=torch.uint8, device=device)
+            cache = lla.Cache(pool, self.pt.num_blocks, self.table, self.pt.max_blocks)
+            for ci, n0 in enumerate(range(0, N, chunk)):
+                n1 = min(N, n0 + chunk)
+                xk = W.normal((w.T, n1 - n0, w.H, w.d), w.seed, 100, l, ci, device=device)
+                xv = W.normal((w.T, n1 - n0, w.H, w.d), w.seed, 101, l, ci, device=device)
+                lla.lla_encode(self.geom, codec, cache, xk, xv, slots_all[n0:n1].to(device))
+                del xk, xv
+            self.codecs.append(codec)
+            self.caches.append(cache)
+            self.pools.append(pool)
+        shape = (w.D, w.T, self.B, w.H, w.d)
+        self.q = W.normal(shape, w.seed, 200, device=device)
+        self.cur_k = W.normal(shape, w.seed, 201, device=device)
+        self.cur_v = W.normal(shape, w.seed, 202, device=device)
+        self.out = torch.empty(shape, dtype=torch.bfloat16, device=device)
+        self.next_slots = torch.stack([self.pt.slots(b, [L])[0] for b, L in enumerate(self.lens)]).to(device)
+        self.ctx = torch.tensor(self.lens, dtype=torch.int32, device=device)
+        self.max_ctx = max(self.lens)
+        self.ws = torch.zeros(lla.lla_decode_workspace_size(self.geom, self.B), dtype=torch.uint8,
+                              device=device)
+        torch.cuda.synchronize()
+        lla.lla_clear_device_error()
+
+    def decode_calls(self):
+        w, lla = self.w, self.lla
+        for t in range(w.T):
+            for l in range(w.D):
+                lla.lla_decode_attn(self.geom, self.codecs[l], self.caches[l], self.ctx,
+                                    self.max_ctx, t, self.q[l, t], self.cur_k[l, t],
+                                    self.cur_v[l, t], self.out[l, t], self.ws)
+
+    def encode_calls(self):
+        # the completed token of every sequence: its stacked loop-t keys / values
+        for l in range(self.w.D):
+            self.lla.lla_encode(self.geom, self.codecs[l], self.caches[l], self.cur_k[l],
+                                self.cur_v[l], self.next_slots)
+
+    def step(self):
+        self.decode_calls()
+        self.encode_calls()
+
+    # algorithmic bytes of one decode launch: latents of every cached token of every head,
+    # this loop's W_up^K and W_up^V, and q, k_cur, v_cur, out
+    def decode_bytes_per_launch(self) -> int:
+        w = self.w
+        es = 2
+        lat = sum(self.lens) * w.H * (w.r_k + w.r_v) * es
+        wup = w.H * w.d * (w.r_k + w.r_v) * es
+        io = 4 * self.B * w.H * w.d * 2
+        return lat + wup + io
+
+    def encode_bytes_per_launch(self) -> int:
+        w = self.w
+        return (w.H * w.T * w.d * (w.r_k + w.r_v) * 2 + 2 * w.T * self.B * w.H * w.d * 2
+                + self.B * w.H * (w.r_k + w.r_v) * 2)
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    from __graft_entry__ import build
+    if rank == 0:
+        build()
+    if world > 1:
+        dist.barrier()
+    build()
+    bench = DecodeBench(args.workload, device)
+    w = bench.w
+    lla = bench.lla
+    stream = torch.cuda.current_stream()
+
+    for _ in range(args.warmup):
+        bench.step()
+    torch.cuda.synchronize()
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error during warm-up")
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(device.index if device.index is not None else 0)
+    sampler.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.mark(True)
+    t_start.record(stream)
+    for k in range(K):
+        ev[k][0].record(stream)
+        bench.decode_calls()
+        ev[k][1].record(stream)
+        bench.encode_calls()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    sampler.mark(False)
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    dec_ms = sum(a.elapsed_time(b) for a, b in ev)
+    if world > 1:
+        t = torch.tensor([total_ms, dec_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, dec_ms = float(t[0]), float(t[1])
+    err = lla.lla_get_device_error()
+    if err != 0:
+        raise RuntimeError(f"device error word {err:#x} after the timed region")
+
+    ms_per_step = total_ms / K
+    value = world * bench.B / (ms_per_step / 1e3)
+    launches_dec = w.D * w.T
+    dec_launch_s = dec_ms / 1e3 / (K * launches_dec)
+    bytes_launch = bench.decode_bytes_per_launch()
+    achieved = bytes_launch / dec_launch_s / 1e9
+    peak, peak_kind = measured_peaks()
+    step_bytes = launches_dec * bytes_launch + w.D * bench.encode_bytes_per_launch()
+
+    result = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {
+            "workload": w.name, "D": w.D, "H": w.H, "d_head": w.d, "T": w.T, "r_k": w.r_k,
+            "r_v": w.r_v, "rho": round(w.rho, 4), "batch_per_gpu": bench.B,
+            "context": list(w.lens), "sum_context": sum(bench.lens), "block_tokens": 64,
+            "storage": "bf16 latents and codec weights, fp32 accumulation",
+            "step": f"{w.T}x{w.D} pass-1 lla_decode_attn calls + {w.D} lla_encode calls of the "
+                    f"{bench.B} completed tokens",
+            "l2": "no flush: latent cache (%.1f GB) far larger than L2" %
+                  (len(bench.pools) * bench.pools[0].numel() / 1e9),
+            "parallelism": f"replicas x{world} (independent batches)",
+        },
+        "roofline": {
+            "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+            "frac": achieved / peak, "traffic": ncu_traffic(w.name),
+            "kernel": "decode_kernel (lla_decode_attn)",
+            "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
+                           if peak_kind == "measured" else "fallback 6.8 TB/s",
+            "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
+            "bytes_per_launch": bytes_launch,
+            "avg_launch_us": dec_launch_s * 1e6,
+        },
+        "step_hbm_gbs": step_bytes / (ms_per_step / 1e3) / 1e9,
+        "gpu_launches": K * (launches_dec + w.D),
+        "clocks": clocks,
+    }
+
+    if not args.no_e2e:
+        result["e2e"] = run_e2e(bench, args, world)
+    if not args.no_cpu_baseline and rank == 0 and world == 1:
+        result["cpu_baseline"] = cpu_baseline(bench.w, bench.lens, args.cpu_seconds)
+    return result
+
+
+def run_e2e(bench, args, world):
+    """Same step with the step's inputs (q, k_cur, v_cur of every call) copied from pinned
+    host memory and the outputs copied back, inside the timed region."""
+    import torch
+    import torch.distributed as dist
+
+    q_h = bench.q.cpu().pin_memory()
+    k_h = bench.cur_k.cpu().pin_memory()
+    v_h = bench.cur_v.cpu().pin_memory()
+    o_h = torch.empty(bench.out.shape, dtype=bench.out.dtype).pin_memory()
+    stream = torch.cuda.current_stream()
+    K = max(1, args.steps)
+
+    def one():
+        bench.q.copy_(q_h, non_blocking=True)
+        bench.cur_k.copy_(k_h, non_blocking=True)
+        bench.cur_v.copy_(v_h, non_blocking=True)
+        bench.step()
+        o_h.copy_(bench.out, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        one()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(K):
+        one()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b)
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=bench.device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t[0])
+    nbytes = lambda t: t.numel() * t.element_size()
+    return {"value": world * bench.B / (ms / K / 1e3), "unit": "tokens/s",
+            "h2d_bytes_per_step": nbytes(q_h) + nbytes(k_h) + nbytes(v_h),
+            "d2h_bytes_per_step": nbytes(o_h), "ms_per_step": ms / K}
+
+
+# ----------------------------------------------------------------- oracle (CPU) timing
+
+def oracle_step_time(w, lens, target_s: float):
+    """Times the CPU oracle on a bounded sample of one decode step and extrapolates to the
+    whole step.  The sample is layer 0: pass-1 decode items (loop, sequence, head) in order
+    until about target_s of work, plus the encode of the B completed tokens of layer 0.  The
+    oracle's time depends on shapes only, so latents and activations are N(0,1) draws.
+    Returns (seconds per full step, sample description, threads)."""
+    import numpy as np
+
+    import oracle
+
+    rng = np.random.default_rng(w.seed)
+    T, H, d, rk, rv = w.T, w.H, w.d, w.r_k, w.r_v
+    w_up_k = rng.standard_normal((T, d, rk)) / math.sqrt(rk)
+    w_up_v = rng.standard_normal((T, d, rv)) / math.sqrt(rv)
+    scale = 1 / math.sqrt(d)
+    threads = oracle.max_threads()
+    lat = {}
+
+    def item(t, b):
+        if b not in lat:
+            lat[b] = (rng.standard_normal((lens[b], rk)), rng.standard_normal((lens[b], rv)))
+        return dict(t=t, c_k=lat[b][0], c_v=lat[b][1], w_up_k=w_up_k, w_up_v=w_up_v, mu_k=None,
+                    mu_v=None, q=rng.standard_normal(d), cur_k=rng.standard_normal(d),
+                    cur_v=rng.standard_normal(d))
+
+    order = [(t, b, h) for t in range(T) for b in range(len(lens)) for h in range(H)]
+    work = lambda b: lens[b] + 1  # reconstruction cost per item is proportional to L + 1
+    total_work = w.D * H * T * sum(lens[b] + 1 for b in range(len(lens)))
+    # calibration batch: one item per thread
+    done_work, secs, i = 0, 0.0, 0
+    while i < len(order) and secs < target_s:
+        n = threads if i == 0 else max(threads, int(threads * 4))
+        batch = order[i:i + n]
+        items = [item(t, b) for t, b, h in batch]
+        t0 = time.perf_counter()
+        oracle.decode_batch(T, d, rk, rv, scale, items, n_threads=threads)
+        secs += time.perf_counter() - t0
+        done_work += sum(work(b) for _, b, _ in batch)
+        i += n
+    # encode of the completed tokens of layer 0 (all heads, both axes)
+    enc_items = [dict(x=rng.standard_normal((T, len(lens), d)), mu=None,
+                      w_down=rng.standard_normal((T * d, r)) / math.sqrt(T * d))
+                 for _ in range(H) for r in (rk, rv)]
+    t0 = time.perf_counter()
+    oracle.encode_batch(T, d, enc_items, n_threads=threads)
+    enc_s = time.perf_counter() - t0
+    step_s = secs * total_work / done_work + enc_s * w.D
+    sample = (f"layer 0 of {w.D}: {i if i < len(order) else len(order)} of {len(order)} pass-1 "
+              f"decode items (loop, sequence, head) = {done_work / (total_work / w.D):.1%} of the "
+              f"layer's decode work, plus the layer's encode of {len(lens)} tokens; extrapolated "
+              f"linearly to the full step (work is linear in context length x heads x loops x "
+              f"layers)")
+    return step_s, sample, threads
+
+
+def cpu_baseline(w, lens, target_s):
+    step_s, sample, threads = oracle_step_time(w, lens, target_s)
+    return {"value": len(lens) / step_s, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": sample, "seconds_per_step": step_s}
+
+
+def run_reference(args, rank, world):
+    from paper_2607_15456_gb300 import workloads as W
+    w = W.WORKLOADS[args.workload]
+    lens = W.context_lengths(w)
+    per_step = max(2.0, min(args.cpu_seconds, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        oracle_step_time(w, lens, per_step)
+    times, sample, threads = [], "", 1
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        s, sample, threads = oracle_step_time(w, lens, per_step)
+        times.append(s)
+    wall = time.perf_counter() - t0
+    step_s = statistics.mean(times)
+    value = len(lens) / step_s
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "D": w.D, "H": w.H, "d_head": w.d, "T": w.T,
+                   "r_k": w.r_k, "r_v": w.r_v, "batch_per_gpu": len(lens)},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "wall_seconds": wall,
+    }
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", init_method="env://")
+    result = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

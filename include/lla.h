@@ -1,0 +1,200 @@
+/*
+ * lla.h -- C ABI of liblla: the hot path of Looped Latent Attention (LLA) on GB300 (sm_103a).
+ *
+ * A looped transformer runs its D-layer stack T times, and every loop writes its own key and
+ * value per layer, head and token ("Teacher cache", Sec. 3).  LLA stores instead one latent
+ * pair per (token, layer, head): c = (x - mu) W_down over the stacked loop vector
+ * x = [x_1; ...; x_T] (Eq. encode), and rebuilds loop t on demand as
+ * xhat_t = c W_up,t^T + mu_t (Eq. decode).  This library implements:
+ *
+ *   lla_encode           Eq. encode for newly completed tokens, written into a paged cache
+ *   lla_decode_attn      one decode call (one layer, one loop) over the paged latent cache,
+ *                        for a batch of sequences of different lengths (App. A, "Decoding and
+ *                        caching": pass 1 and pass 2 of the cached reconstruction decoder)
+ *   lla_prefill_attn     causal pass-2 prefill attention over the latents of a prompt
+ *   lla_dense_*          the uncompressed loop-t KV decode in the same kernel style (the
+ *                        "teacher" column of Table absorbed_latency, App. J), for comparison
+ *
+ * Attention reads the latents directly (App. J, "Absorbed attention"): the score is bilinear,
+ * q . (W_up,t c) = (W_up,t^T q) . c, and the value path satisfies
+ * sum_i a_i W_up,t c_i = W_up,t sum_i a_i c_i.  Reconstructed keys and values are never
+ * written to memory.
+ *
+ * Conventions that hold for every call:
+ *   - All pointers named "device" are CUDA device pointers of the current device.  The caller
+ *     owns every buffer (weights, cache pool, tables, workspace, inputs, outputs).  No call
+ *     allocates memory.
+ *   - Work is enqueued on `stream` (a cudaStream_t passed as void*, NULL = legacy default
+ *     stream) and is asynchronous.  Argument checks that need no device data are synchronous
+ *     and return LLA_ERR_INVALID_ARG or LLA_ERR_UNSUPPORTED before anything is enqueued.
+ *   - Checks that need device data (block ids, context lengths) and bounded waits inside the
+ *     kernels never fault or hang: a failed check sets a sticky per-device error word, the
+ *     affected outputs are undefined, and the host reads the word with lla_get_device_error.
+ *   - No call throws; every call returns an lla_status.
+ *
+ * Cache layout (one layer).  Tokens are grouped in blocks of LLA_BLOCK_TOKENS = 64.  With es =
+ * element size of `storage` (2 for bf16, 4 for fp32):
+ *   pool      [num_blocks][H][K-plane | V-plane]          (one "head page" per block and head)
+ *   K-plane   64 x r_k latents in granules of gk bytes, gk = 16 if (r_k*es) % 16 == 0 else 4:
+ *             the byte offset of element (token i, column j) is
+ *             ((j*es) / gk) * (64*gk) + i*gk + (j*es) % gk
+ *   V-plane   64 x r_v latents, row-major: element (i, j) at byte offset (i*r_v + j)*es
+ *   head page = 64*(r_k + r_v)*es bytes; block = H head pages.
+ * Token p of sequence b lives in block block_table[b*max_blocks_per_seq + p/64], row p%64.
+ * A slot is block_id*64 + row.  The pool must be 16-byte aligned.
+ */
+#ifndef LLA_H_
+#define LLA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LLA_BLOCK_TOKENS 64
+#define LLA_MAX_BATCH 1024
+
+typedef enum {
+    LLA_OK = 0,
+    LLA_ERR_INVALID_ARG = 1,  /* a NULL pointer, a bad size or a bad alignment */
+    LLA_ERR_UNSUPPORTED = 2,  /* a valid geometry this build has no kernel for */
+    LLA_ERR_CUDA = 3,         /* a CUDA runtime call failed (launch, attribute, memcpy) */
+    LLA_ERR_TIMEOUT = 4,      /* device error word: a bounded wait inside a kernel expired */
+    LLA_ERR_DEVICE_CHECK = 5, /* device error word: a block id or length was out of range */
+    LLA_ERR_WORKSPACE = 6     /* the workspace is smaller than the *_workspace_size answer */
+} lla_status;
+
+typedef enum { LLA_BF16 = 0, LLA_F32 = 1 } lla_dtype;
+
+/* Bits of the device error word. */
+#define LLA_DEVERR_BLOCK_ID 0x1u    /* a block id outside [0, num_blocks) */
+#define LLA_DEVERR_CONTEXT 0x2u     /* a context length < 0, > max_ctx or > table capacity */
+#define LLA_DEVERR_EMPTY_PASS2 0x4u /* pass 2 with an empty sequence (nothing to attend to) */
+#define LLA_DEVERR_TIMEOUT 0x8u     /* a bounded wait expired */
+#define LLA_DEVERR_SLOT 0x10u       /* an encode slot outside the pool */
+
+/* Shape of the codec and the cache (Sec. 3; App. A "Models"). */
+typedef struct {
+    int32_t T;          /* loops (recurrence steps), 1..16 */
+    int32_t H;          /* attention heads, >= 1 */
+    int32_t d;          /* head width d_head: a multiple of 8, 8..256 */
+    int32_t r_k, r_v;   /* latent ranks, 2..512; even for bf16 storage */
+    int32_t block_size; /* tokens per cache block: must be LLA_BLOCK_TOKENS */
+    lla_dtype storage;  /* dtype of the latents and of the codec weights */
+    float scale;        /* softmax scale applied to q . k (e.g. 1/sqrt(d)) */
+} lla_geometry;
+
+/* Codec of one layer (Eqs. encode and decode), for all H heads; device pointers. */
+typedef struct {
+    const void *w_down_k; /* [H][T*d][r_k] storage dtype: W_down of the K axis */
+    const void *w_down_v; /* [H][T*d][r_v] storage dtype */
+    const void *w_up_k;   /* [H][T][d][r_k] storage dtype: W_up,t of the K axis */
+    const void *w_up_v;   /* [H][T][d][r_v] storage dtype */
+    const float *mu_k;    /* [H][T*d] fp32 calibration mean, or NULL for mu = 0 */
+    const float *mu_v;    /* [H][T*d] fp32, or NULL */
+} lla_codec;
+
+/* Paged cache of one layer; device pointers. */
+typedef struct {
+    void *pool;                 /* [num_blocks][H][head page], layout above, 16-byte aligned */
+    int64_t num_blocks;
+    const int32_t *block_table; /* [B][max_blocks_per_seq] block ids (unused by lla_encode) */
+    int32_t max_blocks_per_seq;
+} lla_cache;
+
+/* Static description of a status. */
+const char *lla_status_string(lla_status status);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int32_t lla_version(void);
+
+/* Bytes of one cache block (H head pages) for geometry `g`.  Host only. */
+lla_status lla_cache_block_bytes(const lla_geometry *g, size_t *bytes);
+
+/*
+ * Eq. encode (Sec. 3) for N newly completed tokens of one layer, written into the cache.
+ *   x_k, x_v      device [T][N][H][d] in x_dtype: the pre-RoPE loop-t keys / values of each
+ *                 token (Sec. 3 "RoPE and reconstruction"; App. A "LLA codec and conversion")
+ *   slot_mapping  device [N] int64: destination slot of each token; a negative slot skips
+ *                 the token.  A slot beyond the pool sets LLA_DEVERR_SLOT.
+ * Latents are computed with fp32 accumulation and rounded to `storage` (round to nearest
+ * even for bf16).  N may be 0.
+ */
+lla_status lla_encode(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                      const void *x_k, const void *x_v, lla_dtype x_dtype,
+                      const int64_t *slot_mapping, int32_t N, void *stream);
+
+/* Workspace bytes lla_decode_attn needs for a batch of B sequences on the current device. */
+lla_status lla_decode_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes);
+
+/* Zero-fills a decode workspace (needed once before first use and after a device error). */
+lla_status lla_decode_workspace_init(void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * One decode call: layer given by `codec` and `cache`, loop `loop` (0-based), B sequences.
+ * App. A "Decoding and caching" (two-pass cached reconstruction decoder) and App. J
+ * "Absorbed attention".
+ *   context_lens  device [B] int32: tokens of sequence b already in the cache (0..max_ctx)
+ *   max_ctx       host upper bound of every context length (<= 64*max_blocks_per_seq)
+ *   q             device [B][H][d] io_dtype: the loop-t query of the current token
+ *   cur_k, cur_v  device [B][H][d] io_dtype, pass 1: the current token's exact loop-t key and
+ *                 value, attended beside the cached tokens (its stacked vector is not complete
+ *                 before loop T).  Both NULL selects pass 2: the current token was encoded
+ *                 and is one of the context_lens cached tokens (then every length must be >= 1).
+ *   out           device [B][H][d] io_dtype: softmax(scale q.Khat_t) Vhat_t, Khat/Vhat by Eq.
+ *                 decode, without materialising them
+ *   workspace     device, >= lla_decode_workspace_size bytes, zero-filled before first use;
+ *                 every completed call leaves it zero-filled again.  Calls that share a
+ *                 workspace must be ordered (one stream).
+ * B may be 0.  B <= LLA_MAX_BATCH.
+ */
+lla_status lla_decode_attn(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                           const int32_t *context_lens, int32_t B, int32_t max_ctx, int32_t loop,
+                           const void *q, const void *cur_k, const void *cur_v,
+                           lla_dtype io_dtype, void *out, void *workspace,
+                           size_t workspace_bytes, void *stream);
+
+/*
+ * Causal pass-2 prefill attention at loop `loop` over latents already written by lla_encode
+ * (App. A "Decoding and caching": the capacity decoder's two-pass prefill; App. J).
+ *   cu_seqlens  device [B+1] int32 prefix sums of prompt lengths (cu_seqlens[0] = 0); the
+ *               prompt of sequence b occupies cache positions 0..len_b-1 of block-table row b
+ *   max_len     host upper bound of every prompt length (<= 64*max_blocks_per_seq)
+ *   q, out      device [cu_seqlens[B]][H][d] io_dtype; query i of sequence b attends to
+ *               cache positions 0..i of that sequence
+ */
+lla_status lla_prefill_attn(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                            const int32_t *cu_seqlens, int32_t B, int32_t max_len, int32_t loop,
+                            const void *q, lla_dtype io_dtype, void *out, void *stream);
+
+/*
+ * Comparator: the uncompressed loop-indexed cache ("Teacher cache", Sec. 3) decoded by the same
+ * kernel without the codec.  `g` must have r_k = r_v = d; `cache` then holds the plain loop-t
+ * keys and values of one layer in the layout above (K-plane = keys, V-plane = values).
+ */
+lla_status lla_dense_store(const lla_geometry *g, const lla_cache *cache, const void *k,
+                           const void *v, lla_dtype x_dtype, const int64_t *slot_mapping,
+                           int32_t N, void *stream); /* k, v device [N][H][d] */
+lla_status lla_dense_decode_attn(const lla_geometry *g, const lla_cache *cache,
+                                 const int32_t *context_lens, int32_t B, int32_t max_ctx,
+                                 const void *q, const void *cur_k, const void *cur_v,
+                                 lla_dtype io_dtype, void *out, void *workspace,
+                                 size_t workspace_bytes, void *stream);
+
+/*
+ * Reads the sticky device error word of the current device after synchronising `stream`.
+ * *word receives the LLA_DEVERR_* bits; the status is LLA_OK when it is 0, LLA_ERR_TIMEOUT
+ * when the timeout bit is set, LLA_ERR_DEVICE_CHECK otherwise.
+ */
+lla_status lla_get_device_error(void *stream, uint32_t *word);
+
+/* Clears the device error word of the current device (enqueued on `stream`). */
+lla_status lla_clear_device_error(void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LLA_H_ */

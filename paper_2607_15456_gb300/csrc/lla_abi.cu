@@ -1,0 +1,292 @@
+// lla_abi.cu -- the extern "C" entry points of liblla: argument checks, the per-device error
+// word, and dispatch to the kernel files.  Checks that need no device data run before anything
+// is enqueued; nothing here allocates device memory.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "lla_internal.h"
+
+namespace lla {
+
+namespace {
+
+__device__ unsigned g_error_word;  // sticky LLA_DEVERR_* bits of this device
+
+constexpr int kMaxDevices = 64;
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int elem_size(lla_dtype t) { return t == LLA_BF16 ? 2 : 4; }
+
+bool valid_dtype(lla_dtype t) { return t == LLA_BF16 || t == LLA_F32; }
+
+lla_status check_geometry(const lla_geometry *g) {
+    if (!g) return LLA_ERR_INVALID_ARG;
+    if (g->T < 1 || g->T > 16 || g->H < 1 || g->H > 4096) return LLA_ERR_INVALID_ARG;
+    if (g->d < 8 || g->d > 256 || (g->d % 8) != 0) return LLA_ERR_INVALID_ARG;
+    if (g->r_k < 2 || g->r_v < 2 || g->r_k > 512 || g->r_v > 512) return LLA_ERR_INVALID_ARG;
+    if ((g->r_k % 2) != 0 || (g->r_v % 2) != 0) return LLA_ERR_INVALID_ARG;
+    if (g->block_size != LLA_BLOCK_TOKENS) return LLA_ERR_UNSUPPORTED;
+    if (!valid_dtype(g->storage)) return LLA_ERR_INVALID_ARG;
+    if (!isfinite(g->scale)) return LLA_ERR_INVALID_ARG;
+    return LLA_OK;
+}
+
+lla_status check_cache(const lla_cache *c, bool need_table) {
+    if (!c || !c->pool || c->num_blocks < 1) return LLA_ERR_INVALID_ARG;
+    if (!aligned(c->pool, 16)) return LLA_ERR_INVALID_ARG;
+    if (need_table && (!c->block_table || c->max_blocks_per_seq < 1)) return LLA_ERR_INVALID_ARG;
+    return LLA_OK;
+}
+
+}  // namespace
+
+unsigned *device_error_word(lla_status *st) {
+    static unsigned *addr[kMaxDevices] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev >= kMaxDevices) {
+        *st = LLA_ERR_CUDA;
+        return nullptr;
+    }
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) {
+            *st = LLA_ERR_CUDA;
+            return nullptr;
+        }
+        addr[dev] = static_cast<unsigned *>(p);
+    }
+    *st = LLA_OK;
+    return addr[dev];
+}
+
+int num_sms() {
+    static int cached[kMaxDevices] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev >= kMaxDevices) return 0;
+    if (!cached[dev]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+        cached[dev] = n;
+    }
+    return cached[dev];
+}
+
+}  // namespace lla
+
+using namespace lla;
+
+extern "C" {
+
+const char *lla_status_string(lla_status s) {
+    switch (s) {
+        case LLA_OK: return "ok";
+        case LLA_ERR_INVALID_ARG: return "invalid argument";
+        case LLA_ERR_UNSUPPORTED: return "unsupported geometry";
+        case LLA_ERR_CUDA: return "CUDA runtime error";
+        case LLA_ERR_TIMEOUT: return "device wait timed out";
+        case LLA_ERR_DEVICE_CHECK: return "device-side check failed";
+        case LLA_ERR_WORKSPACE: return "workspace too small";
+    }
+    return "unknown status";
+}
+
+int32_t lla_version(void) { return 100; /* 0.1.0 */ }
+
+lla_status lla_cache_block_bytes(const lla_geometry *g, size_t *bytes) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!bytes) return LLA_ERR_INVALID_ARG;
+    *bytes = head_page_bytes(g->r_k, g->r_v, elem_size(g->storage)) * g->H;
+    return LLA_OK;
+}
+
+lla_status lla_encode(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                      const void *x_k, const void *x_v, lla_dtype x_dtype,
+                      const int64_t *slot_mapping, int32_t N, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!codec || !codec->w_down_k || !codec->w_down_v) return LLA_ERR_INVALID_ARG;
+    if ((st = check_cache(cache, false)) != LLA_OK) return st;
+    if (!valid_dtype(x_dtype) || N < 0) return LLA_ERR_INVALID_ARG;
+    if (N > 0 && (!x_k || !x_v || !slot_mapping)) return LLA_ERR_INVALID_ARG;
+    const int es = elem_size(g->storage);
+    if (!aligned(codec->w_down_k, 2 * es) || !aligned(codec->w_down_v, 2 * es))
+        return LLA_ERR_INVALID_ARG;
+    if (N == 0) return LLA_OK;
+    EncodeArgs a = {};
+    a.T = g->T; a.H = g->H; a.d = g->d; a.r_k = g->r_k; a.r_v = g->r_v;
+    a.storage_bf16 = g->storage == LLA_BF16;
+    a.x_bf16 = x_dtype == LLA_BF16;
+    a.w_down_k = codec->w_down_k; a.w_down_v = codec->w_down_v;
+    a.mu_k = codec->mu_k; a.mu_v = codec->mu_v;
+    a.x_k = x_k; a.x_v = x_v;
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.slot_mapping = slot_mapping; a.N = N;
+    a.dense = 0;
+    return launch_encode(a, static_cast<cudaStream_t>(stream));
+}
+
+lla_status lla_decode_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
+    const int sms = num_sms();
+    if (sms <= 0) return LLA_ERR_CUDA;
+    *bytes = decode_workspace_bytes(g->r_v, B, g->H, sms);
+    return LLA_OK;
+}
+
+lla_status lla_decode_workspace_init(void *workspace, size_t workspace_bytes, void *stream) {
+    if (!workspace || workspace_bytes == 0) return LLA_ERR_INVALID_ARG;
+    if (cudaMemsetAsync(workspace, 0, workspace_bytes, static_cast<cudaStream_t>(stream)) !=
+        cudaSuccess)
+        return LLA_ERR_CUDA;
+    return LLA_OK;
+}
+
+namespace {
+
+lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                         const int32_t *context_lens, int32_t B, int32_t max_ctx, int32_t loop,
+                         const void *q, const void *cur_k, const void *cur_v, lla_dtype io_dtype,
+                         void *out, void *workspace, size_t workspace_bytes, void *stream,
+                         bool absorbed) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if ((st = check_cache(cache, true)) != LLA_OK) return st;
+    const int es = elem_size(g->storage);
+    if (absorbed) {
+        if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;
+        if (!aligned(codec->w_up_k, 2 * es) || !aligned(codec->w_up_v, 2 * es))
+            return LLA_ERR_INVALID_ARG;
+        if (loop < 0 || loop >= g->T) return LLA_ERR_INVALID_ARG;
+    } else if (g->r_k != g->d || g->r_v != g->d) {
+        return LLA_ERR_INVALID_ARG;
+    }
+    if (B < 0 || B > LLA_MAX_BATCH || !valid_dtype(io_dtype)) return LLA_ERR_INVALID_ARG;
+    if (max_ctx < 0 || static_cast<int64_t>(max_ctx) >
+                           static_cast<int64_t>(cache->max_blocks_per_seq) * LLA_BLOCK_TOKENS)
+        return LLA_ERR_INVALID_ARG;
+    if ((cur_k == nullptr) != (cur_v == nullptr)) return LLA_ERR_INVALID_ARG;
+    if (B > 0 && (!context_lens || !q || !out)) return LLA_ERR_INVALID_ARG;
+    if ((st = decode_fits(g->r_k, g->r_v, es, g->d)) != LLA_OK) return st;
+    if (B == 0) return LLA_OK;
+    if (!workspace) return LLA_ERR_INVALID_ARG;
+    DecodeArgs a = {};
+    a.T = g->T; a.H = g->H; a.d = g->d; a.r_k = g->r_k; a.r_v = g->r_v;
+    a.loop = absorbed ? loop : 0;
+    a.absorbed = absorbed ? 1 : 0;
+    a.storage_bf16 = g->storage == LLA_BF16;
+    a.io_bf16 = io_dtype == LLA_BF16;
+    a.scale = g->scale;
+    if (absorbed) {
+        a.w_up_k = codec->w_up_k; a.w_up_v = codec->w_up_v;
+        a.mu_k = codec->mu_k; a.mu_v = codec->mu_v;
+    }
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.block_table = cache->block_table; a.max_blocks = cache->max_blocks_per_seq;
+    a.context_lens = context_lens; a.B = B; a.max_ctx = max_ctx;
+    a.q = q; a.cur_k = cur_k; a.cur_v = cur_v; a.out = out;
+    a.workspace = workspace; a.workspace_bytes = workspace_bytes;
+    return launch_decode(a, static_cast<cudaStream_t>(stream));
+}
+
+}  // namespace
+
+lla_status lla_decode_attn(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                           const int32_t *context_lens, int32_t B, int32_t max_ctx, int32_t loop,
+                           const void *q, const void *cur_k, const void *cur_v,
+                           lla_dtype io_dtype, void *out, void *workspace,
+                           size_t workspace_bytes, void *stream) {
+    return decode_common(g, codec, cache, context_lens, B, max_ctx, loop, q, cur_k, cur_v,
+                         io_dtype, out, workspace, workspace_bytes, stream, true);
+}
+
+lla_status lla_dense_decode_attn(const lla_geometry *g, const lla_cache *cache,
+                                 const int32_t *context_lens, int32_t B, int32_t max_ctx,
+                                 const void *q, const void *cur_k, const void *cur_v,
+                                 lla_dtype io_dtype, void *out, void *workspace,
+                                 size_t workspace_bytes, void *stream) {
+    return decode_common(g, nullptr, cache, context_lens, B, max_ctx, 0, q, cur_k, cur_v,
+                         io_dtype, out, workspace, workspace_bytes, stream, false);
+}
+
+lla_status lla_dense_store(const lla_geometry *g, const lla_cache *cache, const void *k,
+                           const void *v, lla_dtype x_dtype, const int64_t *slot_mapping,
+                           int32_t N, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (g->r_k != g->d || g->r_v != g->d) return LLA_ERR_INVALID_ARG;
+    if ((st = check_cache(cache, false)) != LLA_OK) return st;
+    if (!valid_dtype(x_dtype) || N < 0) return LLA_ERR_INVALID_ARG;
+    if (N > 0 && (!k || !v || !slot_mapping)) return LLA_ERR_INVALID_ARG;
+    if (N == 0) return LLA_OK;
+    EncodeArgs a = {};
+    a.T = 1; a.H = g->H; a.d = g->d; a.r_k = g->d; a.r_v = g->d;
+    a.storage_bf16 = g->storage == LLA_BF16;
+    a.x_bf16 = x_dtype == LLA_BF16;
+    a.x_k = k; a.x_v = v;
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.slot_mapping = slot_mapping; a.N = N;
+    a.dense = 1;
+    return launch_encode(a, static_cast<cudaStream_t>(stream));
+}
+
+lla_status lla_prefill_attn(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                            const int32_t *cu_seqlens, int32_t B, int32_t max_len, int32_t loop,
+                            const void *q, lla_dtype io_dtype, void *out, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if ((st = check_cache(cache, true)) != LLA_OK) return st;
+    if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;
+    const int es = elem_size(g->storage);
+    if (!aligned(codec->w_up_k, 2 * es) || !aligned(codec->w_up_v, 2 * es))
+        return LLA_ERR_INVALID_ARG;
+    if (loop < 0 || loop >= g->T || B < 0 || B > LLA_MAX_BATCH || !valid_dtype(io_dtype))
+        return LLA_ERR_INVALID_ARG;
+    if (max_len < 0 || static_cast<int64_t>(max_len) >
+                           static_cast<int64_t>(cache->max_blocks_per_seq) * LLA_BLOCK_TOKENS)
+        return LLA_ERR_INVALID_ARG;
+    if (B > 0 && (!cu_seqlens || !q || !out)) return LLA_ERR_INVALID_ARG;
+    if (B == 0 || max_len == 0) return LLA_OK;
+    PrefillArgs a = {};
+    a.T = g->T; a.H = g->H; a.d = g->d; a.r_k = g->r_k; a.r_v = g->r_v; a.loop = loop;
+    a.storage_bf16 = g->storage == LLA_BF16;
+    a.io_bf16 = io_dtype == LLA_BF16;
+    a.scale = g->scale;
+    a.w_up_k = codec->w_up_k; a.w_up_v = codec->w_up_v;
+    a.mu_k = codec->mu_k; a.mu_v = codec->mu_v;
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.block_table = cache->block_table; a.max_blocks = cache->max_blocks_per_seq;
+    a.cu_seqlens = cu_seqlens; a.B = B; a.max_len = max_len;
+    a.q = q; a.out = out;
+    return launch_prefill(a, static_cast<cudaStream_t>(stream));
+}
+
+lla_status lla_get_device_error(void *stream, uint32_t *word) {
+    if (!word) return LLA_ERR_INVALID_ARG;
+    lla_status st = LLA_OK;
+    unsigned *addr = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    unsigned host = 0;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(&host, addr, sizeof(unsigned), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return LLA_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return LLA_ERR_CUDA;
+    *word = host;
+    if (host == 0) return LLA_OK;
+    return (host & LLA_DEVERR_TIMEOUT) ? LLA_ERR_TIMEOUT : LLA_ERR_DEVICE_CHECK;
+}
+
+lla_status lla_clear_device_error(void *stream) {
+    lla_status st = LLA_OK;
+    unsigned *addr = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    if (cudaMemsetAsync(addr, 0, sizeof(unsigned), static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return LLA_ERR_CUDA;
+    return LLA_OK;
+}
+
+}  // extern "C"

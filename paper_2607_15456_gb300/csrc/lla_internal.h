@@ -1,0 +1,79 @@
+// lla_internal.h -- host-side interface between the C ABI (lla_abi.cu) and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/lla.h"
+
+namespace lla {
+
+// Everything one decode launch needs (one layer, one loop, B sequences).
+struct DecodeArgs {
+    int T, H, d, r_k, r_v, loop;
+    int absorbed;  // 1: latent cache with codec; 0: dense comparator (r_k = r_v = d, no codec)
+    int storage_bf16, io_bf16;
+    float scale;
+    const void *w_up_k, *w_up_v;  // [H][T][d][r] storage dtype (absorbed only)
+    const float *mu_k, *mu_v;     // [H][T*d] or NULL
+    const void *pool;
+    int64_t num_blocks;
+    const int32_t *block_table;
+    int max_blocks;
+    const int32_t *context_lens;
+    int B, max_ctx;
+    const void *q, *cur_k, *cur_v;
+    void *out;
+    void *workspace;
+    size_t workspace_bytes;
+};
+
+struct EncodeArgs {
+    int T, H, d, r_k, r_v;
+    int storage_bf16, x_bf16;
+    const void *w_down_k, *w_down_v;  // [H][T*d][r]
+    const float *mu_k, *mu_v;         // [H][T*d] or NULL
+    const void *x_k, *x_v;            // [T][N][H][d]
+    void *pool;
+    int64_t num_blocks;
+    const int64_t *slot_mapping;
+    int N;
+    int dense;  // 1: store x_k / x_v ([N][H][d]) as plain K/V pages (r_k = r_v = d, T = 1)
+};
+
+struct PrefillArgs {
+    int T, H, d, r_k, r_v, loop;
+    int storage_bf16, io_bf16;
+    float scale;
+    const void *w_up_k, *w_up_v;
+    const float *mu_k, *mu_v;
+    const void *pool;
+    int64_t num_blocks;
+    const int32_t *block_table;
+    int max_blocks;
+    const int32_t *cu_seqlens;
+    int B, max_len;
+    const void *q;
+    void *out;
+};
+
+// Per-device address of the sticky error word (owned by lla_abi.cu).
+unsigned *device_error_word(lla_status *st);
+
+// Bytes of one head page (K-plane + V-plane) and of one block.
+inline size_t head_page_bytes(int r_k, int r_v, int es) {
+    return static_cast<size_t>(LLA_BLOCK_TOKENS) * (r_k + r_v) * es;
+}
+
+// Decode: workspace bytes for `grid` CTAs and B sequences; launch.
+size_t decode_workspace_bytes(int r_v, int B, int H, int grid);
+lla_status decode_fits(int r_k, int r_v, int es, int d);  // UNSUPPORTED if no kernel shape fits
+lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream);
+
+lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream);
+lla_status launch_prefill(const PrefillArgs &a, cudaStream_t stream);
+
+int num_sms();  // SM count of the current device (cached), 0 on failure
+
+}  // namespace lla

@@ -1,0 +1,262 @@
+"""Thin Python binding of liblla (include/lla.h): argument marshalling only.
+
+Every function here has the name of the C entry point it calls and does nothing but turn
+torch tensors into device pointers, fill the ABI structs and raise ``LLAError`` on a non-zero
+status.  All computation happens in the CUDA kernels of liblla.so; there is no fallback: if
+the library is missing or a call fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+from .build import LIB
+
+LLA_BLOCK_TOKENS = 64
+LLA_MAX_BATCH = 1024
+LLA_BF16, LLA_F32 = 0, 1
+LLA_DEVERR_BLOCK_ID = 0x1
+LLA_DEVERR_CONTEXT = 0x2
+LLA_DEVERR_EMPTY_PASS2 = 0x4
+LLA_DEVERR_TIMEOUT = 0x8
+LLA_DEVERR_SLOT = 0x10
+
+_STATUS = {0: "LLA_OK", 1: "LLA_ERR_INVALID_ARG", 2: "LLA_ERR_UNSUPPORTED", 3: "LLA_ERR_CUDA",
+           4: "LLA_ERR_TIMEOUT", 5: "LLA_ERR_DEVICE_CHECK", 6: "LLA_ERR_WORKSPACE"}
+
+
+class LLAError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} returned {_STATUS.get(status, status)}")
+
+
+class lla_geometry(ctypes.Structure):
+    _fields_ = [("T", ctypes.c_int32), ("H", ctypes.c_int32), ("d", ctypes.c_int32),
+                ("r_k", ctypes.c_int32), ("r_v", ctypes.c_int32), ("block_size", ctypes.c_int32),
+                ("storage", ctypes.c_int32), ("scale", ctypes.c_float)]
+
+
+class lla_codec(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in
+                ("w_down_k", "w_down_v", "w_up_k", "w_up_v", "mu_k", "mu_v")]
+
+
+class lla_cache(ctypes.Structure):
+    _fields_ = [("pool", ctypes.c_void_p), ("num_blocks", ctypes.c_int64),
+                ("block_table", ctypes.c_void_p), ("max_blocks_per_seq", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def library() -> ctypes.CDLL:
+    """Loads liblla.so from the package directory (built by ``__graft_entry__.build()``)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB):
+            raise RuntimeError(f"liblla.so not found at {LIB}: build it first "
+                               "(python -c 'import __graft_entry__ as g; g.build()')")
+        lib = ctypes.CDLL(LIB)
+        P, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+        sig = {
+            "lla_status_string": (ctypes.c_char_p, [I32]),
+            "lla_version": (I32, []),
+            "lla_cache_block_bytes": (I32, [P, P]),
+            "lla_encode": (I32, [P, P, P, P, P, I32, P, I32, P]),
+            "lla_decode_workspace_size": (I32, [P, I32, P]),
+            "lla_decode_workspace_init": (I32, [P, SZ, P]),
+            "lla_decode_attn": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ, P]),
+            "lla_prefill_attn": (I32, [P, P, P, P, I32, I32, I32, P, I32, P, P]),
+            "lla_dense_store": (I32, [P, P, P, P, I32, P, I32, P]),
+            "lla_dense_decode_attn": (I32, [P, P, P, I32, I32, P, P, P, I32, P, P, SZ, P]),
+            "lla_get_device_error": (I32, [P, P]),
+            "lla_clear_device_error": (I32, [P]),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(lib, name)
+            fn.restype, fn.argtypes = res, args
+        _lib = lib
+    return _lib
+
+
+def _check(fn: str, status: int):
+    if status != 0:
+        raise LLAError(fn, status)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to liblla must be contiguous")
+    return t.data_ptr()
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return LLA_BF16
+    if t.dtype == torch.float32:
+        return LLA_F32
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+@dataclass
+class Geometry:
+    T: int
+    H: int
+    d: int
+    r_k: int
+    r_v: int
+    storage: str = "bf16"
+    scale: Optional[float] = None
+
+    def c(self) -> lla_geometry:
+        scale = self.scale if self.scale is not None else 1.0 / math.sqrt(self.d)
+        return lla_geometry(self.T, self.H, self.d, self.r_k, self.r_v, LLA_BLOCK_TOKENS,
+                            LLA_BF16 if self.storage == "bf16" else LLA_F32, scale)
+
+    @property
+    def torch_dtype(self):
+        return torch.bfloat16 if self.storage == "bf16" else torch.float32
+
+
+@dataclass
+class Codec:
+    """Codec of one layer: w_down_* [H][T*d][r], w_up_* [H][T][d][r], mu_* [H][T*d] fp32."""
+    w_down_k: torch.Tensor
+    w_down_v: torch.Tensor
+    w_up_k: torch.Tensor
+    w_up_v: torch.Tensor
+    mu_k: Optional[torch.Tensor] = None
+    mu_v: Optional[torch.Tensor] = None
+
+    def c(self) -> lla_codec:
+        return lla_codec(*(_ptr(t) for t in (self.w_down_k, self.w_down_v, self.w_up_k,
+                                             self.w_up_v, self.mu_k, self.mu_v)))
+
+
+@dataclass
+class Cache:
+    """Paged cache of one layer: pool (uint8 or any dtype, 16-byte aligned), block table
+    [B][max_blocks_per_seq] int32."""
+    pool: torch.Tensor
+    num_blocks: int
+    block_table: Optional[torch.Tensor]
+    max_blocks_per_seq: int
+
+    def c(self) -> lla_cache:
+        return lla_cache(_ptr(self.pool), self.num_blocks, _ptr(self.block_table),
+                         self.max_blocks_per_seq)
+
+
+def lla_status_string(status: int) -> str:
+    return library().lla_status_string(status).decode()
+
+
+def lla_version() -> int:
+    return library().lla_version()
+
+
+def lla_cache_block_bytes(geom: Geometry) -> int:
+    out = ctypes.c_size_t(0)
+    g = geom.c()
+    _check("lla_cache_block_bytes",
+           library().lla_cache_block_bytes(ctypes.byref(g), ctypes.byref(out)))
+    return out.value
+
+
+def lla_encode(geom: Geometry, codec: Codec, cache: Cache, x_k: torch.Tensor, x_v: torch.Tensor,
+               slot_mapping: torch.Tensor, stream=None) -> None:
+    """x_k, x_v [T][N][H][d] (bf16 or fp32); slot_mapping [N] int64."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    N = x_k.shape[1] if x_k.dim() == 4 else 0
+    _check("lla_encode", library().lla_encode(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(x_k), _ptr(x_v),
+        _dtype_code(x_k), _ptr(slot_mapping), N, _stream(stream)))
+
+
+def lla_decode_workspace_size(geom: Geometry, B: int) -> int:
+    out = ctypes.c_size_t(0)
+    g = geom.c()
+    _check("lla_decode_workspace_size",
+           library().lla_decode_workspace_size(ctypes.byref(g), B, ctypes.byref(out)))
+    return out.value
+
+
+def lla_decode_workspace_init(workspace: torch.Tensor, stream=None) -> None:
+    nbytes = workspace.numel() * workspace.element_size()
+    _check("lla_decode_workspace_init",
+           library().lla_decode_workspace_init(_ptr(workspace), nbytes, _stream(stream)))
+
+
+def lla_decode_attn(geom: Geometry, codec: Codec, cache: Cache, context_lens: torch.Tensor,
+                    max_ctx: int, loop: int, q: torch.Tensor, cur_k: Optional[torch.Tensor],
+                    cur_v: Optional[torch.Tensor], out: torch.Tensor, workspace: torch.Tensor,
+                    stream=None) -> None:
+    """q, cur_k, cur_v, out [B][H][d]; cur_k = cur_v = None selects pass 2."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    B = q.shape[0]
+    _check("lla_decode_attn", library().lla_decode_attn(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(context_lens), B, max_ctx,
+        loop, _ptr(q), _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def lla_prefill_attn(geom: Geometry, codec: Codec, cache: Cache, cu_seqlens: torch.Tensor,
+                     max_len: int, loop: int, q: torch.Tensor, out: torch.Tensor,
+                     stream=None) -> None:
+    """q, out [Ntok][H][d]; cu_seqlens [B+1] int32."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    B = cu_seqlens.shape[0] - 1
+    _check("lla_prefill_attn", library().lla_prefill_attn(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(cu_seqlens), B, max_len, loop,
+        _ptr(q), _dtype_code(q), _ptr(out), _stream(stream)))
+
+
+def lla_dense_store(geom: Geometry, cache: Cache, k: torch.Tensor, v: torch.Tensor,
+                    slot_mapping: torch.Tensor, stream=None) -> None:
+    """k, v [N][H][d]: plain loop-t keys and values for the uncompressed comparator."""
+    g, ch = geom.c(), cache.c()
+    _check("lla_dense_store", library().lla_dense_store(
+        ctypes.byref(g), ctypes.byref(ch), _ptr(k), _ptr(v), _dtype_code(k), _ptr(slot_mapping),
+        k.shape[0], _stream(stream)))
+
+
+def lla_dense_decode_attn(geom: Geometry, cache: Cache, context_lens: torch.Tensor, max_ctx: int,
+                          q: torch.Tensor, cur_k: Optional[torch.Tensor],
+                          cur_v: Optional[torch.Tensor], out: torch.Tensor,
+                          workspace: torch.Tensor, stream=None) -> None:
+    g, ch = geom.c(), cache.c()
+    _check("lla_dense_decode_attn", library().lla_dense_decode_attn(
+        ctypes.byref(g), ctypes.byref(ch), _ptr(context_lens), q.shape[0], max_ctx, _ptr(q),
+        _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def lla_get_device_error(stream=None) -> int:
+    """Returns the device error word (0 = no error) without raising."""
+    word = ctypes.c_uint32(0)
+    st = library().lla_get_device_error(_stream(stream), ctypes.byref(word))
+    if st not in (0, 4, 5):
+        raise LLAError("lla_get_device_error", st)
+    return word.value
+
+
+def lla_clear_device_error(stream=None) -> None:
+    _check("lla_clear_device_error", library().lla_clear_device_error(_stream(stream)))

@@ -1,0 +1,172 @@
+"""Host-side checks of the C ABI (no GPU): the library loads, exports every entry point that
+include/lla.h declares, and rejects bad arguments synchronously, before touching CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from helpers import ensure_library
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "lla.h")
+
+OK, INVALID, UNSUPPORTED, CUDA_ERR, TIMEOUT, DEVCHECK, WORKSPACE = range(7)
+FAKE = 0x10000  # a non-NULL, 16-byte aligned "device pointer" that validation never touches
+
+
+@pytest.fixture(scope="module")
+def lib():
+    ensure_library()
+    from paper_2607_15456_gb300 import lla
+    return lla
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(lla_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    for must in ("lla_encode", "lla_decode_attn", "lla_prefill_attn", "lla_decode_workspace_size",
+                 "lla_dense_decode_attn", "lla_get_device_error", "lla_status_string"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    so = lib.library()
+    missing = [n for n in declared_functions() if not hasattr(so, n)]
+    assert not missing, missing
+
+
+def test_status_strings_and_version(lib):
+    assert lib.lla_version() >= 100
+    assert lib.lla_status_string(0) == "ok"
+    assert lib.lla_status_string(6) == "workspace too small"
+
+
+def test_block_bytes_follow_the_documented_layout(lib):
+    for T, H, d, rk, rv, st, es in ((4, 16, 128, 96, 160, "bf16", 2), (4, 16, 128, 18, 30, "bf16", 2),
+                                    (4, 4, 128, 96, 160, "fp32", 4)):
+        g = lib.Geometry(T, H, d, rk, rv, st)
+        assert lib.lla_cache_block_bytes(g) == H * 64 * (rk + rv) * es
+
+
+def _g(lib, **kw):
+    base = dict(T=4, H=16, d=128, r_k=96, r_v=160, storage="bf16")
+    base.update(kw)
+    return lib.Geometry(**base).c()
+
+
+def _codec(lib, **kw):
+    c = lib.lla_codec(FAKE, FAKE, FAKE, FAKE, None, None)
+    for k, v in kw.items():
+        setattr(c, k, v)
+    return c
+
+
+def _cache(lib, pool=FAKE, table=FAKE, nb=10, mb=4):
+    return lib.lla_cache(pool, nb, table, mb)
+
+
+@pytest.mark.parametrize("bad", [dict(T=0), dict(T=17), dict(H=0), dict(d=12), dict(d=512),
+                                 dict(r_k=1), dict(r_v=513), dict(r_k=95), dict(storage="x")])
+def test_bad_geometry_is_rejected(lib, bad):
+    kw = dict(T=4, H=16, d=128, r_k=96, r_v=160, storage="bf16")
+    kw.update(bad)
+    g = lib.Geometry(**{k: v for k, v in kw.items() if k != "storage"}).c()
+    if "storage" in bad:
+        g.storage = 7
+    so = lib.library()
+    out = ctypes.c_size_t()
+    assert so.lla_cache_block_bytes(ctypes.byref(g), ctypes.byref(out)) == INVALID
+
+
+def test_block_size_other_than_64_is_unsupported(lib):
+    g = _g(lib)
+    g.block_size = 32
+    out = ctypes.c_size_t()
+    assert lib.library().lla_cache_block_bytes(ctypes.byref(g), ctypes.byref(out)) == UNSUPPORTED
+
+
+def _decode(lib, g=None, codec=None, cache=None, lens=FAKE, B=4, max_ctx=128, loop=0, q=FAKE,
+            ck=FAKE, cv=FAKE, io=0, out=FAKE, ws=FAKE, ws_bytes=1 << 20):
+    so = lib.library()
+    g = g or _g(lib)
+    codec = codec or _codec(lib)
+    cache = cache or _cache(lib)
+    return so.lla_decode_attn(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache), lens, B,
+                              max_ctx, loop, q, ck, cv, io, out, ws, ws_bytes, None)
+
+
+def test_decode_argument_checks(lib):
+    assert _decode(lib, ck=None) == INVALID                      # cur_k without cur_v
+    assert _decode(lib, loop=4) == INVALID                       # loop outside [0, T)
+    assert _decode(lib, loop=-1) == INVALID
+    assert _decode(lib, B=-1) == INVALID
+    assert _decode(lib, B=1025) == INVALID                       # above LLA_MAX_BATCH
+    assert _decode(lib, max_ctx=4 * 64 + 1) == INVALID           # beyond the table capacity
+    assert _decode(lib, q=None) == INVALID
+    assert _decode(lib, lens=None) == INVALID
+    assert _decode(lib, out=None) == INVALID
+    assert _decode(lib, ws=None) == INVALID
+    assert _decode(lib, io=3) == INVALID
+    assert _decode(lib, codec=_codec(lib, w_up_k=None)) == INVALID
+    assert _decode(lib, codec=_codec(lib, w_up_v=FAKE + 2)) == INVALID   # misaligned bf16 pairs
+    assert _decode(lib, cache=_cache(lib, pool=FAKE + 8)) == INVALID     # pool not 16-B aligned
+    assert _decode(lib, cache=_cache(lib, table=None)) == INVALID
+    assert _decode(lib, cache=_cache(lib, nb=0)) == INVALID
+    # an empty batch is a valid no-op that never touches the device
+    assert _decode(lib, B=0, lens=None, q=None, out=None, ws=None) == OK
+
+
+def test_decode_rejects_geometries_without_a_kernel_shape(lib):
+    # fp32 latents with r_k + r_v = 1024 do not leave room for two pipeline stages
+    g = _g(lib, r_k=512, r_v=512, storage="fp32")
+    assert _decode(lib, g=g) == UNSUPPORTED
+
+
+def test_encode_argument_checks(lib):
+    so = lib.library()
+    g, cache = _g(lib), _cache(lib)
+
+    def enc(codec=None, xk=FAKE, xv=FAKE, slots=FAKE, N=8, xd=0):
+        codec = codec or _codec(lib)
+        return so.lla_encode(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache), xk, xv,
+                             xd, slots, N, None)
+
+    assert enc(codec=_codec(lib, w_down_k=None)) == INVALID
+    assert enc(xk=None) == INVALID
+    assert enc(slots=None) == INVALID
+    assert enc(N=-1) == INVALID
+    assert enc(xd=5) == INVALID
+    assert enc(N=0, xk=None, xv=None, slots=None) == OK
+
+
+def test_dense_comparator_needs_r_equal_d(lib):
+    so = lib.library()
+    g, cache = _g(lib), _cache(lib)  # r_k = 96 != d
+    assert so.lla_dense_decode_attn(ctypes.byref(g), ctypes.byref(cache), FAKE, 4, 64, FAKE, None,
+                                    None, 0, FAKE, FAKE, 1 << 20, None) == INVALID
+    assert so.lla_dense_store(ctypes.byref(g), ctypes.byref(cache), FAKE, FAKE, 0, FAKE, 4,
+                              None) == INVALID
+
+
+def test_prefill_argument_checks(lib):
+    so = lib.library()
+    g, codec, cache = _g(lib), _codec(lib), _cache(lib)
+
+    def pre(cu=FAKE, B=2, max_len=64, loop=0, q=FAKE, out=FAKE):
+        return so.lla_prefill_attn(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache), cu,
+                                   B, max_len, loop, q, 0, out, None)
+
+    assert pre(cu=None) == INVALID
+    assert pre(loop=4) == INVALID
+    assert pre(max_len=10**6) == INVALID
+    assert pre(B=0, cu=None, q=None, out=None) == OK
+
+
+def test_workspace_init_rejects_null(lib):
+    assert lib.library().lla_decode_workspace_init(None, 16, None) == INVALID

@@ -1,0 +1,312 @@
+"""GPU parity of lla_encode and lla_decode_attn against the CPU float64 oracle.
+
+Inputs come from the seeded generators (paper_2607_15456_gb300.workloads) and go unchanged to
+both sides; the oracle reconstructs every loop's K/V explicitly (Eq. decode) and runs plain
+softmax attention, the GPU reads latents directly (App. J absorbed form).  Tolerances: bf16
+storage with fp32 accumulation, max abs <= 2e-2 and relative L2 <= 5e-3; fp32 mode, relative
+L2 <= 1e-5.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import assert_parity, ensure_library, f64, rel_l2, unpack_head
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module")
+def lla():
+    ensure_library()
+    from paper_2607_15456_gb300 import lla as m
+    m.lla_clear_device_error()
+    return m
+
+
+def _dt(name):
+    return torch.bfloat16 if name == "bf16" else torch.float32
+
+
+class Scene:
+    """One layer's codec, a paged cache filled by lla_encode, and the oracle's latents."""
+
+    def __init__(self, lla, T=4, H=4, d=128, r_k=96, r_v=160, storage="bf16", io="fp32",
+                 lens=(256,), seed=0, with_mu=False, extra_tokens=1):
+        from paper_2607_15456_gb300 import workloads as W
+        self.lla, self.W = lla, W
+        self.T, self.H, self.d, self.r_k, self.r_v = T, H, d, r_k, r_v
+        self.storage, self.io, self.lens, self.seed = storage, io, list(lens), seed
+        self.geom = lla.Geometry(T, H, d, r_k, r_v, storage)
+        self.scale = 1.0 / math.sqrt(d)
+        cod = W.codec_tensors(T, H, d, r_k, r_v, seed, 0, dtype=_dt(storage), device=DEV,
+                              with_mu=with_mu)
+        self.cod = cod
+        self.codec = lla.Codec(**cod)
+        self.pt = W.page_table(self.lens, seed, extra_tokens=extra_tokens)
+        bb = lla.lla_cache_block_bytes(self.geom)
+        # poison the pool (all-ones bytes are NaN in bf16 and fp32) so that any read of a row
+        # that was never written shows up as a non-finite output
+        self.pool = torch.full((self.pt.num_blocks * bb,), 0xFF, dtype=torch.uint8, device=DEV)
+        self.table = self.pt.block_table.to(DEV)
+        self.cache = lla.Cache(self.pool, self.pt.num_blocks, self.table, self.pt.max_blocks)
+        self.B = len(self.lens)
+        N = sum(self.lens)
+        self.x_k = W.normal((T, N, H, d), seed, 10, dtype=_dt(io), device=DEV)
+        self.x_v = W.normal((T, N, H, d), seed, 11, dtype=_dt(io), device=DEV)
+        slots = [self.pt.slots(b, range(L)) for b, L in enumerate(self.lens)]
+        self.slots = torch.cat(slots).to(DEV) if N else torch.zeros(0, dtype=torch.int64, device=DEV)
+        if N:
+            lla.lla_encode(self.geom, self.codec, self.cache, self.x_k, self.x_v, self.slots)
+        # oracle latents, per (sequence, head)
+        self.w64 = {k: (None if v is None else f64(v)) for k, v in cod.items()}
+        xk, xv = f64(self.x_k), f64(self.x_v)
+        self.ck, self.cv = {}, {}
+        off = 0
+        for b, L in enumerate(self.lens):
+            for h in range(H):
+                mk = None if self.w64["mu_k"] is None else self.w64["mu_k"][h]
+                mv = None if self.w64["mu_v"] is None else self.w64["mu_v"][h]
+                self.ck[b, h] = oracle.encode(xk[:, off:off + L, h, :], mk, self.w64["w_down_k"][h])
+                self.cv[b, h] = oracle.encode(xv[:, off:off + L, h, :], mv, self.w64["w_down_v"][h])
+            off += L
+        size = lla.lla_decode_workspace_size(self.geom, self.B)
+        self.ws = torch.zeros(size, dtype=torch.uint8, device=DEV)
+
+    def gpu_latents(self, b, h, L=None):
+        L = self.lens[b] if L is None else L
+        return unpack_head(self.pool.cpu(), self.H, self.r_k, self.r_v, self.storage,
+                           self.pt.block_table[b], L, h)
+
+    def append_token(self, seed_key=20):
+        """Encodes one new token per sequence at position L_b (its stacked loop vectors are the
+        new token's per-loop K/V) and grows every context by one."""
+        W = self.W
+        xk = W.normal((self.T, self.B, self.H, self.d), self.seed, seed_key, dtype=_dt(self.io), device=DEV)
+        xv = W.normal((self.T, self.B, self.H, self.d), self.seed, seed_key + 1, dtype=_dt(self.io), device=DEV)
+        slots = torch.stack([self.pt.slots(b, [L])[0] for b, L in enumerate(self.lens)]).to(DEV)
+        self.lla.lla_encode(self.geom, self.codec, self.cache, xk, xv, slots)
+        xk64, xv64 = f64(xk), f64(xv)
+        for b in range(self.B):
+            for h in range(self.H):
+                mk = None if self.w64["mu_k"] is None else self.w64["mu_k"][h]
+                mv = None if self.w64["mu_v"] is None else self.w64["mu_v"][h]
+                ck = oracle.encode(xk64[:, b:b + 1, h, :], mk, self.w64["w_down_k"][h])
+                cv = oracle.encode(xv64[:, b:b + 1, h, :], mv, self.w64["w_down_v"][h])
+                self.ck[b, h] = np.concatenate([self.ck[b, h], ck])
+                self.cv[b, h] = np.concatenate([self.cv[b, h], cv])
+        self.lens = [L + 1 for L in self.lens]
+        return xk, xv
+
+    def decode(self, loop, pass1, key=30):
+        W = self.W
+        shape = (self.B, self.H, self.d)
+        q = W.normal(shape, self.seed, key, loop, dtype=_dt(self.io), device=DEV)
+        ck = W.normal(shape, self.seed, key + 1, loop, dtype=_dt(self.io), device=DEV) if pass1 else None
+        cv = W.normal(shape, self.seed, key + 2, loop, dtype=_dt(self.io), device=DEV) if pass1 else None
+        out = torch.empty(shape, dtype=_dt(self.io), device=DEV)
+        lens = torch.tensor(self.lens, dtype=torch.int32, device=DEV)
+        self.lla.lla_decode_attn(self.geom, self.codec, self.cache, lens, max(self.lens + [0]),
+                                 loop, q, ck, cv, out, self.ws)
+        torch.cuda.synchronize()
+        return q, ck, cv, out
+
+    def oracle_decode(self, loop, q, ck, cv, b, h, latents=None):
+        c_k, c_v = latents if latents is not None else (self.ck[b, h], self.cv[b, h])
+        w = self.w64
+        return oracle.decode(loop, c_k, c_v, w["w_up_k"][h], w["w_up_v"][h],
+                             None if w["mu_k"] is None else w["mu_k"][h],
+                             None if w["mu_v"] is None else w["mu_v"][h],
+                             f64(q[b, h]), None if ck is None else f64(ck[b, h]),
+                             None if cv is None else f64(cv[b, h]), self.scale)
+
+
+def _check_decode(sc, loop, pass1, tight=False):
+    q, ck, cv, out = sc.decode(loop, pass1)
+    got = f64(out)
+    ref = np.zeros_like(got)
+    for b in range(sc.B):
+        for h in range(sc.H):
+            ref[b, h] = sc.oracle_decode(loop, q, ck, cv, b, h)
+    assert_parity(got, ref, sc.storage, f"decode loop {loop} pass{1 if pass1 else 2}", io=sc.io)
+    if tight:
+        # the oracle fed the latents the GPU stored: only accumulation order differs
+        ref2 = np.zeros_like(got)
+        for b in range(sc.B):
+            for h in range(sc.H):
+                ref2[b, h] = sc.oracle_decode(loop, q, ck, cv, b, h,
+                                              latents=sc.gpu_latents(b, h))
+        bound = 1e-4 if sc.io == "fp32" else 5e-3
+        assert rel_l2(got, ref2) <= bound, rel_l2(got, ref2)
+    return got
+
+
+@pytest.mark.parametrize("storage", ["bf16", "fp32"])
+@pytest.mark.parametrize("with_mu", [False, True])
+def test_tiny_workload_encode_then_two_pass_decode(lla, storage, with_mu):
+    """T=4, H=4, (96,160), one sequence of 256 cached tokens: encode, pass 1 over all four
+    loops, encode of the completed token, pass 2 over all four loops (App. A)."""
+    sc = Scene(lla, storage=storage, io="fp32", with_mu=with_mu, seed=0)
+    for h in range(sc.H):
+        gk, gv = sc.gpu_latents(0, h)
+        assert_parity(gk, sc.ck[0, h], storage, "K latents")
+        assert_parity(gv, sc.cv[0, h], storage, "V latents")
+    for t in range(sc.T):
+        _check_decode(sc, t, pass1=True, tight=True)
+    sc.append_token()
+    for t in range(sc.T):
+        _check_decode(sc, t, pass1=False, tight=True)
+    assert lla.lla_get_device_error() == 0
+
+
+@pytest.mark.parametrize("rk,rv", [(96, 160), (192, 320), (72, 120), (18, 30)])
+@pytest.mark.parametrize("storage", ["bf16", "fp32"])
+def test_ragged_batch_all_rank_shapes(lla, rk, rv, storage):
+    """Mixed lengths: empty (pass 1 only), one token, page-aligned, ragged tails, several pages."""
+    lens = [0, 1, 63, 64, 65, 200, 513]
+    if storage == "fp32" and rk + rv > 400:
+        # an fp32 head page of 64 x 512 latents (128 KiB) leaves no room for two pipeline
+        # stages in shared memory: documented as unsupported
+        with pytest.raises(lla.LLAError) as e:
+            Scene(lla, r_k=rk, r_v=rv, storage=storage, io="bf16", lens=[5], seed=5).decode(0, True)
+        assert e.value.status == 2
+        return
+    sc = Scene(lla, r_k=rk, r_v=rv, storage=storage, io="bf16", lens=lens, seed=5)
+    for b in (1, 4, 6):
+        gk, gv = sc.gpu_latents(b, 2)
+        assert_parity(gk, sc.ck[b, 2], storage, "K latents")
+        assert_parity(gv, sc.cv[b, 2], storage, "V latents")
+    for t in (0, 3):
+        _check_decode(sc, t, pass1=True)
+    sc.append_token()
+    _check_decode(sc, 1, pass1=False)
+    assert lla.lla_get_device_error() == 0
+
+
+def test_pass1_empty_cache_returns_current_value(lla):
+    sc = Scene(lla, lens=[0, 0, 0], io="fp32", seed=6)
+    q, ck, cv, out = sc.decode(2, pass1=True)
+    torch.testing.assert_close(out, cv, rtol=0, atol=0)
+
+
+def test_long_sequences_split_across_many_ctas(lla):
+    """A few long sequences and H=16: every (sequence, head) is split over several CTAs, so
+    the partial merge and the last-arriver epilogue are exercised."""
+    sc = Scene(lla, H=16, lens=[4000, 3100, 2049], io="bf16", seed=7)
+    for t in (0, 2):
+        _check_decode(sc, t, pass1=True)
+    sc.append_token()
+    _check_decode(sc, 3, pass1=False)
+
+
+def test_many_short_sequences(lla):
+    """Batch of 300 with lengths 1..140: many (sequence, head) ranges finish inside one CTA."""
+    g = torch.Generator().manual_seed(8)
+    lens = [int(v) for v in torch.randint(1, 141, (300,), generator=g)]
+    sc = Scene(lla, H=2, lens=lens, io="bf16", seed=8)
+    _check_decode(sc, 1, pass1=True)
+
+
+def test_decode_is_deterministic(lla):
+    sc = Scene(lla, H=8, lens=[700, 1500, 90], io="bf16", seed=9)
+    a = sc.decode(0, pass1=True)[3].clone()
+    b = sc.decode(0, pass1=True)[3]
+    assert torch.equal(a, b)
+
+
+def test_workspace_stays_zero_after_calls(lla):
+    sc = Scene(lla, H=16, lens=[3000, 2500], io="bf16", seed=10)
+    sc.decode(0, pass1=True)
+    sc.decode(1, pass1=True)
+    torch.cuda.synchronize()
+    # counters sit after the partial records; a completed call leaves every counter at zero
+    from paper_2607_15456_gb300 import lla as m
+    size = m.lla_decode_workspace_size(sc.geom, sc.B)
+    counters = sc.ws[size - sc.B * sc.H * 4:size].view(torch.int32)
+    assert int(counters.abs().sum()) == 0
+
+
+def test_device_checks_flag_bad_tables_and_lengths(lla):
+    sc = Scene(lla, lens=[100, 200], io="bf16", seed=11)
+    lla.lla_clear_device_error()
+    bad = sc.table.clone()
+    bad[1, 1] = sc.pt.num_blocks + 5  # a block id beyond the pool
+    cache = lla.Cache(sc.pool, sc.pt.num_blocks, bad, sc.pt.max_blocks)
+    shape = (sc.B, sc.H, sc.d)
+    q = torch.randn(shape, device=DEV).to(torch.bfloat16)
+    out = torch.empty_like(q)
+    lens = torch.tensor(sc.lens, dtype=torch.int32, device=DEV)
+    lla.lla_decode_attn(sc.geom, sc.codec, cache, lens, 200, 0, q, q, q, out, sc.ws)
+    assert lla.lla_get_device_error() & lla.LLA_DEVERR_BLOCK_ID
+    lla.lla_clear_device_error()
+    lla.lla_decode_workspace_init(sc.ws)
+    # a context length beyond max_ctx
+    lla.lla_decode_attn(sc.geom, sc.codec, sc.cache, lens, 150, 0, q, q, q, out, sc.ws)
+    assert lla.lla_get_device_error() & lla.LLA_DEVERR_CONTEXT
+    lla.lla_clear_device_error()
+    lla.lla_decode_workspace_init(sc.ws)
+    # pass 2 over an empty sequence
+    zl = torch.tensor([0, 5], dtype=torch.int32, device=DEV)
+    lla.lla_decode_attn(sc.geom, sc.codec, sc.cache, zl, 200, 0, q, None, None, out, sc.ws)
+    assert lla.lla_get_device_error() & lla.LLA_DEVERR_EMPTY_PASS2
+    lla.lla_clear_device_error()
+    # an encode slot beyond the pool
+    xk = torch.zeros((4, 1, sc.H, sc.d), device=DEV)
+    slot = torch.tensor([(sc.pt.num_blocks + 1) * 64], dtype=torch.int64, device=DEV)
+    lla.lla_encode(sc.geom, sc.codec, sc.cache, xk, xk, slot)
+    assert lla.lla_get_device_error() & lla.LLA_DEVERR_SLOT
+    lla.lla_clear_device_error()
+    assert lla.lla_get_device_error() == 0
+
+
+def test_workspace_too_small_is_rejected(lla):
+    sc = Scene(lla, lens=[10], io="bf16", seed=12)
+    small = torch.zeros(16, dtype=torch.uint8, device=DEV)
+    q = torch.zeros((1, sc.H, sc.d), dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(lla.LLAError) as e:
+        lla.lla_decode_attn(sc.geom, sc.codec, sc.cache,
+                            torch.tensor([10], dtype=torch.int32, device=DEV), 10, 0, q, None,
+                            None, q.clone(), small)
+    assert e.value.status == 6
+
+
+@pytest.mark.parametrize("storage", ["bf16", "fp32"])
+def test_dense_comparator_matches_uncompressed_attention(lla, storage):
+    """The uncompressed loop-t decode (same kernel, no codec) against plain attention on the
+    raw keys and values (oracle.attention)."""
+    from paper_2607_15456_gb300 import workloads as W
+    H, d = 4, 128
+    lens = [1, 64, 130, 1000]
+    geom = lla.Geometry(1, H, d, d, d, storage)
+    pt = W.page_table(lens, 13, extra_tokens=1)
+    pool = torch.full((pt.num_blocks * lla.lla_cache_block_bytes(geom),), 0xFF, dtype=torch.uint8, device=DEV)
+    cache = lla.Cache(pool, pt.num_blocks, pt.block_table.to(DEV), pt.max_blocks)
+    N = sum(lens)
+    k = W.normal((N, H, d), 13, 1, dtype=torch.bfloat16, device=DEV)
+    v = W.normal((N, H, d), 13, 2, dtype=torch.bfloat16, device=DEV)
+    slots = torch.cat([pt.slots(b, range(L)) for b, L in enumerate(lens)]).to(DEV)
+    lla.lla_dense_store(geom, cache, k, v, slots)
+    B = len(lens)
+    q = W.normal((B, H, d), 13, 3, dtype=torch.bfloat16, device=DEV)
+    ck = W.normal((B, H, d), 13, 4, dtype=torch.bfloat16, device=DEV)
+    cv = W.normal((B, H, d), 13, 5, dtype=torch.bfloat16, device=DEV)
+    out = torch.empty_like(q)
+    ws = torch.zeros(lla.lla_decode_workspace_size(geom, B), dtype=torch.uint8, device=DEV)
+    lens_t = torch.tensor(lens, dtype=torch.int32, device=DEV)
+    lla.lla_dense_decode_attn(geom, cache, lens_t, max(lens), q, ck, cv, out, ws)
+    torch.cuda.synchronize()
+    k64, v64 = f64(k), f64(v)
+    ref = np.zeros((B, H, d))
+    off = 0
+    for b, L in enumerate(lens):
+        for h in range(H):
+            K = np.concatenate([k64[off:off + L, h], f64(ck[b, h])[None]])
+            V = np.concatenate([v64[off:off + L, h], f64(cv[b, h])[None]])
+            ref[b, h] = oracle.attention(f64(q[b, h]), K, V, 1 / math.sqrt(d))
+        off += L
+    assert_parity(f64(out), ref, "bf16", "dense decode")
+    assert lla.lla_get_device_error() == 0
