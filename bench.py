@@ -156,13 +156,16 @@ class ClockSampler:
 # ------------------------------------------------------------------------------- our arm
 
 class DecodeBench:
-    def __init__(self, wname: str, device):
+    def __init__(self, wname: str, device, layers=None):
         import torch
         from paper_2607_15456_gb300 import lla
         from paper_2607_15456_gb300 import workloads as W
 
         self.torch, self.lla, self.W = torch, lla, W
         w = W.WORKLOADS[wname]
+        if layers is not None:  # a shallower model with the same per-launch shape (profiling)
+            from dataclasses import replace
+            w = replace(w, D=layers)
         self.w = w
         self.device = device
         self.geom = lla.Geometry(w.T, w.H, w.d, w.r_k, w.r_v, w.storage)
@@ -174,7 +177,6 @@ class DecodeBench:
         bb = lla.lla_cache_block_bytes(self.geom)
         self.codecs, self.caches, self.pools = [], [], []
         slots_all = torch.cat([self.pt.slots(b, range(L)) for b, L in enumerate(self.lens)])
-        seq_of_tok = torch.cat([torch.full((L,), b) for b, L in enumerate(self.lens)])
         chunk = 1 << 17
         N = slots_all.numel()
         for l in range(w.D):
