@@ -157,6 +157,26 @@ lla_status lla_decode_attn(const lla_geometry *g, const lla_codec *codec, const 
                            size_t workspace_bytes, void *stream);
 
 /*
+ * lla_decode_attn for callers that cannot allocate device memory (for example a plug-in inside a
+ * host application that owns all device memory and offers it no allocator, or a latency-critical
+ * loop that cannot afford cudaMalloc's device-wide synchronisation).  Same arguments and result
+ * as lla_decode_attn, without the workspace: the scratch lives in a 1 MiB device array of this
+ * library, held on every GPU that loads it until the process exits.  The paper has no
+ * counterpart; this is a deployment convenience.
+ *   - Returns LLA_ERR_WORKSPACE (and enqueues nothing) when lla_decode_workspace_size for this
+ *     geometry and B exceeds 1 MiB.
+ *   - Every call shares the array and clears the part it uses (cudaMemsetAsync on `stream`);
+ *     calls that can overlap on the GPU race on it: order them on one stream.
+ *   - The first call on a device looks up the array's address with that device current; make
+ *     that first call before any stream capture.
+ *   - Allocates nothing (no cudaMalloc, no cudaFree).
+ */
+lla_status lla_decode_attn_noalloc(const lla_geometry *g, const lla_codec *codec,
+                                   const lla_cache *cache, const int32_t *context_lens, int32_t B,
+                                   int32_t max_ctx, int32_t loop, const void *q, const void *cur_k,
+                                   const void *cur_v, lla_dtype io_dtype, void *out, void *stream);
+
+/*
  * Causal pass-2 prefill attention at loop `loop` over latents already written by lla_encode
  * (App. A "Decoding and caching": the capacity decoder's two-pass prefill; App. J).
  *   cu_seqlens  device [B+1] int32 prefix sums of prompt lengths (cu_seqlens[0] = 0); the

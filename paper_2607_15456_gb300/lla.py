@@ -72,6 +72,7 @@ def library() -> ctypes.CDLL:
             "lla_decode_workspace_size": (I32, [P, I32, P]),
             "lla_decode_workspace_init": (I32, [P, SZ, P]),
             "lla_decode_attn": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ, P]),
+            "lla_decode_attn_noalloc": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P]),
             "lla_prefill_attn": (I32, [P, P, P, P, I32, I32, I32, P, I32, P, P]),
             "lla_dense_store": (I32, [P, P, P, P, I32, P, I32, P]),
             "lla_dense_decode_attn": (I32, [P, P, P, I32, I32, P, P, P, I32, P, P, SZ, P]),
@@ -216,6 +217,20 @@ def lla_decode_attn(geom: Geometry, codec: Codec, cache: Cache, context_lens: to
         ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(context_lens), B, max_ctx,
         loop, _ptr(q), _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def lla_decode_attn_noalloc(geom: Geometry, codec: Codec, cache: Cache,
+                            context_lens: torch.Tensor, max_ctx: int, loop: int,
+                            q: torch.Tensor, cur_k: Optional[torch.Tensor],
+                            cur_v: Optional[torch.Tensor], out: torch.Tensor,
+                            stream=None) -> None:
+    """lla_decode_attn with the library's own 1 MiB device scratch instead of a caller
+    workspace, for callers that cannot allocate device memory (see include/lla.h)."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    _check("lla_decode_attn_noalloc", library().lla_decode_attn_noalloc(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(context_lens), q.shape[0],
+        max_ctx, loop, _ptr(q), _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out),
+        _stream(stream)))
 
 
 def lla_prefill_attn(geom: Geometry, codec: Codec, cache: Cache, cu_seqlens: torch.Tensor,
