@@ -7,9 +7,11 @@
 // slot: the K latent into the granule-interleaved K-plane, the V latent into the row-major
 // V-plane of its block's head page.
 //
-// One CTA takes a tile of tokens of one head and one axis: the centred stacked vectors of the
-// tile are staged in shared memory (fp32), each thread owns a pair of latent columns for a
-// subset of the tile's tokens and streams W_down once per tile (coalesced along the columns).
+// One CTA takes (a tile of up to 16 tokens, a tile of 32 latent columns of one axis, one head).
+// The tile's centred stacked vectors are staged in shared memory (fp32); 256 threads are 16
+// column pairs x 16 slices of the T*d reduction axis, each streaming its slice of W_down with
+// several loads in flight, and the 16 partial sums per output meet in shared memory.  At a decode
+// step (N = batch) this spreads the weight-bound work over H x (r_k + r_v)/32 CTAs.
 #include <cuda_runtime.h>
 
 #include "lla_device.cuh"
@@ -19,8 +21,11 @@ namespace lla {
 namespace {
 
 constexpr int kThreads = 256;
+constexpr int kColTile = 32;          // latent columns per CTA
+constexpr int kPairs = kColTile / 2;  // column pairs per CTA
+constexpr int kSlices = kThreads / kPairs;  // slices of the reduction axis
 constexpr int kMaxTileTokens = 16;
-constexpr int kSmemLimit = 200 * 1024;
+constexpr int kXsBudget = 96 * 1024;  // shared bytes for the staged token tile
 
 struct EncParams {
     int T, H, d, r_k, r_v, x_bf16;
@@ -31,7 +36,7 @@ struct EncParams {
     int64_t num_blocks, block_bytes;
     int head_page_bytes, kplane_bytes;
     const int64_t *slot_mapping;
-    int N, tile;
+    int N, tile, ctiles_k;
     unsigned *err;
 };
 
@@ -49,11 +54,16 @@ __device__ __forceinline__ void store_latent(char *dst, float v) {
 
 template <int ES>
 __global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
-    extern __shared__ __align__(16) float xs[];  // [tile][T*d] centred stacked vectors
-    const int axis = blockIdx.z, h = blockIdx.y;
+    extern __shared__ __align__(16) float smem_f[];
+    const int Td = p.T * p.d;
+    float *xs = smem_f;                          // [tile][Td] centred stacked vectors
+    float *red = smem_f + p.tile * Td;           // [kSlices][tile][kColTile] partial sums
+    const int ct = blockIdx.y;
+    const int axis = ct < p.ctiles_k ? 0 : 1;
+    const int col0 = (axis ? ct - p.ctiles_k : ct) * kColTile;
+    const int h = blockIdx.z;
     const int n0 = blockIdx.x * p.tile;
     const int nt = min(p.tile, p.N - n0);
-    const int Td = p.T * p.d;
     const int r = axis ? p.r_v : p.r_k;
     const void *W = axis ? p.w_down_v : p.w_down_k;
     const float *mu = axis ? p.mu_v : p.mu_k;
@@ -72,33 +82,63 @@ __global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
     }
     __syncthreads();
 
-    // c = (x - mu) W_down: thread owns columns (2 jp, 2 jp + 1) for tokens ng, ng + NG, ...
-    const int njp = r >> 1;
-    const int ng_count = kThreads / njp;
-    const int jp = tid % njp, ng = tid / njp;
-    if (ng >= ng_count || ng >= nt) return;
-    const int cnt = (nt - ng + ng_count - 1) / ng_count;
+    // c = (x - mu) W_down over this thread's slice of the reduction axis
+    const int jp = tid % kPairs, sl = tid / kPairs;
+    const int col = col0 + 2 * jp;
+    const bool active = col < r;
     float2 acc[kMaxTileTokens];
 #pragma unroll
     for (int i = 0; i < kMaxTileTokens; ++i) acc[i] = make_float2(0.f, 0.f);
-    const int64_t wbase = static_cast<int64_t>(h) * Td * r + 2 * jp;
-    for (int k = 0; k < Td; ++k) {
-        const float2 w = load_pair<ES>(W, wbase + static_cast<int64_t>(k) * r);
+    if (active) {
+        const int64_t wbase = static_cast<int64_t>(h) * Td * r + col;
+        int k = sl;
+        for (; k + 3 * kSlices < Td; k += 4 * kSlices) {
+            float2 w[4];
 #pragma unroll
-        for (int i = 0; i < kMaxTileTokens; ++i) {
-            if (i < cnt) {
-                const float xv = xs[(ng + i * ng_count) * Td + k];
-                acc[i].x = fmaf(xv, w.x, acc[i].x);
-                acc[i].y = fmaf(xv, w.y, acc[i].y);
+            for (int u = 0; u < 4; ++u)
+                w[u] = load_pair<ES>(W, wbase + static_cast<int64_t>(k + u * kSlices) * r);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+#pragma unroll
+                for (int i = 0; i < kMaxTileTokens; ++i) {
+                    if (i < nt) {
+                        const float xv = xs[i * Td + k + u * kSlices];
+                        acc[i].x = fmaf(xv, w[u].x, acc[i].x);
+                        acc[i].y = fmaf(xv, w[u].y, acc[i].y);
+                    }
+                }
+            }
+        }
+        for (; k < Td; k += kSlices) {
+            const float2 w = load_pair<ES>(W, wbase + static_cast<int64_t>(k) * r);
+#pragma unroll
+            for (int i = 0; i < kMaxTileTokens; ++i) {
+                if (i < nt) {
+                    const float xv = xs[i * Td + k];
+                    acc[i].x = fmaf(xv, w.x, acc[i].x);
+                    acc[i].y = fmaf(xv, w.y, acc[i].y);
+                }
             }
         }
     }
-    const int gk = granule_bytes(p.r_k, ES);
 #pragma unroll
     for (int i = 0; i < kMaxTileTokens; ++i) {
-        if (i >= cnt) break;
-        const int n = n0 + ng + i * ng_count;
-        const int64_t slot = p.slot_mapping[n];
+        if (i < nt) {
+            red[(sl * p.tile + i) * kColTile + 2 * jp] = acc[i].x;
+            red[(sl * p.tile + i) * kColTile + 2 * jp + 1] = acc[i].y;
+        }
+    }
+    __syncthreads();
+
+    // sum the slices, round to the storage dtype and scatter to each token's slot
+    const int gk = granule_bytes(p.r_k, ES);
+    for (int o = tid; o < nt * kColTile; o += kThreads) {
+        const int i = o / kColTile, c = o % kColTile;
+        const int j = col0 + c;
+        if (j >= r) continue;
+        float v = 0.f;
+        for (int s2 = 0; s2 < kSlices; ++s2) v += red[(s2 * p.tile + i) * kColTile + c];
+        const int64_t slot = p.slot_mapping[n0 + i];
         if (slot < 0) continue;
         const int64_t blk = slot / kBlockTokens;
         const int row = static_cast<int>(slot % kBlockTokens);
@@ -107,15 +147,10 @@ __global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
             continue;
         }
         char *page = p.pool + blk * p.block_bytes + static_cast<int64_t>(h) * p.head_page_bytes;
-        const int j = 2 * jp;
-        if (axis == 0) {
-            store_latent<ES>(page + kplane_offset(row, j, ES, gk), acc[i].x);
-            store_latent<ES>(page + kplane_offset(row, j + 1, ES, gk), acc[i].y);
-        } else {
-            char *vrow = page + p.kplane_bytes + static_cast<int64_t>(row) * p.r_v * ES;
-            store_latent<ES>(vrow + j * ES, acc[i].x);
-            store_latent<ES>(vrow + (j + 1) * ES, acc[i].y);
-        }
+        if (axis == 0)
+            store_latent<ES>(page + kplane_offset(row, j, ES, gk), v);
+        else
+            store_latent<ES>(page + p.kplane_bytes + (static_cast<int64_t>(row) * p.r_v + j) * ES, v);
     }
 }
 
@@ -164,7 +199,7 @@ lla_status set_smem(int dev) {
     static bool configured[64] = {};
     if (dev < 64 && configured[dev]) return LLA_OK;
     if (cudaFuncSetAttribute(encode_kernel<ES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kSmemLimit) != cudaSuccess)
+                             kXsBudget + kSlices * kMaxTileTokens * kColTile * 4) != cudaSuccess)
         return LLA_ERR_CUDA;
     if (dev < 64) configured[dev] = true;
     return LLA_OK;
@@ -196,16 +231,19 @@ lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream) {
                        : launch(dense_store_kernel<4>, grid, block, 0, stream, p);
     }
     const int Td = a.T * a.d;
-    int tile = kSmemLimit / (Td * 4);
+    int tile = kXsBudget / (Td * 4);
     if (tile > kMaxTileTokens) tile = kMaxTileTokens;
     if (tile < 1) return LLA_ERR_UNSUPPORTED;
     p.tile = tile;
-    const int smem = tile * Td * 4;
+    p.ctiles_k = (a.r_k + kColTile - 1) / kColTile;
+    const int ctiles_v = (a.r_v + kColTile - 1) / kColTile;
+    const int smem = (tile * Td + kSlices * tile * kColTile) * 4;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     st = es == 2 ? set_smem<2>(dev) : set_smem<4>(dev);
     if (st != LLA_OK) return st;
-    const dim3 grid((a.N + tile - 1) / tile, a.H, 2), block(kThreads);
+    if (a.H > 65535) return LLA_ERR_UNSUPPORTED;
+    const dim3 grid((a.N + tile - 1) / tile, p.ctiles_k + ctiles_v, a.H), block(kThreads);
     return es == 2 ? launch(encode_kernel<2>, grid, block, smem, stream, p)
                    : launch(encode_kernel<4>, grid, block, smem, stream, p);
 }

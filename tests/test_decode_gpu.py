@@ -163,10 +163,13 @@ def test_tiny_workload_encode_then_two_pass_decode(lla, storage, with_mu):
     assert lla.lla_get_device_error() == 0
 
 
-@pytest.mark.parametrize("rk,rv", [(96, 160), (192, 320), (72, 120), (18, 30)])
+@pytest.mark.parametrize("rk,rv", [(96, 160), (192, 320), (72, 120), (18, 30),
+                                   (120, 200), (20, 36)])
 @pytest.mark.parametrize("storage", ["bf16", "fp32"])
 def test_ragged_batch_all_rank_shapes(lla, rk, rv, storage):
-    """Mixed lengths: empty (pass 1 only), one token, page-aligned, ragged tails, several pages."""
+    """Mixed lengths: empty (pass 1 only), one token, page-aligned, ragged tails, several pages.
+    The first four rank shapes run the shape-specialised decode kernel, (120, 200) (Table tier4,
+    rho = 3.20) and (20, 36) the generic one."""
     lens = [0, 1, 63, 64, 65, 200, 513]
     if storage == "fp32" and rk + rv > 400:
         # an fp32 head page of 64 x 512 latents (128 KiB) leaves no room for two pipeline
