@@ -134,7 +134,7 @@ lla_status lla_decode_workspace_size(const lla_geometry *g, int32_t B, size_t *b
     if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
     const int sms = num_sms();
     if (sms <= 0) return LLA_ERR_CUDA;
-    *bytes = decode_workspace_bytes(g->r_v, B, g->H, sms);
+    *bytes = decode_workspace_bytes(g->r_v, B, g->H, 2 * sms);  // up to two CTAs per SM
     return LLA_OK;
 }
 

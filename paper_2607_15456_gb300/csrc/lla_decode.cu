@@ -19,7 +19,11 @@
 //     (cp.async.bulk + mbarrier transaction counts), evict-first in L2.
 //   * Eight consumer warps compute scores from the K-plane (granule-interleaved so that
 //     consecutive lanes read consecutive 16-byte words), an exact online softmax (warp-shuffle
-//     max, exp2), and accumulate sum_i p_i c_v,i in latent space from the V-plane.
+//     max, exp2), and accumulate sum_i p_i c_v,i in latent space from the V-plane.  For the rank
+//     shapes of the Ouro workloads a shape-specialised kernel splits them into score warps
+//     (one token per thread, q~ held in registers, softmax) and value warps, which run one or
+//     two steps apart through a two-slot ring of softmax weights in shared memory; any other
+//     shape runs the generic kernel, where all eight warps take each phase in turn.
 //   * A range that covers a (sequence, head) completely finishes it in place; ranges that split
 //     one write (m, l, o_latent) partials, and the last CTA to arrive (atomic counter) merges
 //     them by log-sum-exp, adds the current token and applies W_up,t^V, mu^V_t and 1/l.
@@ -37,9 +41,10 @@ constexpr int kComputeThreads = kComputeWarps * 32;
 constexpr int kThreads = kComputeThreads + 32;  // + one producer warp
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
+constexpr int kHalfSmem = 113 * 1024;  // per CTA when two CTAs share an SM
 constexpr int kStepTargetBytes = 32 * 1024;
-constexpr int kBarAll = 1;   // named barrier over the 256 consumer threads
-constexpr int kBarTok = 2;   // named barrier over the score-owning threads
+constexpr int kBarAll = 1;  // named barrier over the 256 consumer threads
+constexpr int kBarTok = 2;  // named barrier over the score threads
 
 struct Params {
     int T, H, d, r_k, r_v, loop, absorbed, io_bf16;
@@ -62,8 +67,8 @@ struct Params {
 };
 
 struct Layout {
-    int ring, full, empty, prefix, lens, qlat, qfull, spart, psm, tmp, red, lred, ovec, misc,
-        total;
+    int ring, full, empty, pfull, pempty, prefix, lens, qlat, qfull, spart, psm, tmp, red, lred,
+        ovec, misc, total;
 };
 
 __host__ __device__ inline int up16(int x) { return (x + 15) & ~15; }
@@ -78,6 +83,10 @@ __host__ __device__ inline Layout make_layout(int stages, int stage_bytes, int B
     o += stages * 8;
     L.empty = o;
     o += stages * 8;
+    L.pfull = o;
+    o += 2 * 8;
+    L.pempty = o;
+    o += 2 * 8;
     L.prefix = o;
     o += up16((B + 1) * 8);
     L.lens = o;
@@ -89,7 +98,7 @@ __host__ __device__ inline Layout make_layout(int stages, int stage_bytes, int B
     L.spart = o;
     o += kComputeThreads * 4;
     L.psm = o;
-    o += kComputeThreads * 4;
+    o += 2 * kComputeThreads * 4;
     L.tmp = o;
     o += 2 * kComputeThreads * 4;
     L.red = o;
@@ -99,14 +108,49 @@ __host__ __device__ inline Layout make_layout(int stages, int stage_bytes, int B
     L.ovec = o;
     o += up16((r_v > d ? r_v : d) * 4);
     L.misc = o;
-    o += 32 * 4;
+    o += 64 * 4;
     L.total = o;
     return L;
 }
 
 // misc slots
 constexpr int kMiscAlpha = 0, kMiscM = 1, kMiscL = 2, kMiscBeta = 3, kMiscScur = 4,
-              kMiscWmax = 8, kMiscAbort = 16, kMiscLast = 17;
+              kMiscPAlpha = 5 /* 5, 6 */, kMiscWmax = 16 /* [2][8] */, kMiscAbort = 32,
+              kMiscLast = 33;
+
+struct Smem {
+    char *ring;
+    uint64_t *full, *empty, *pfull, *pempty;
+    int64_t *prefix;
+    int *lens;
+    float *qlat, *qfull, *spart, *psm, *tmp, *red, *lred, *ovec, *misc;
+    volatile int *abort_flag;
+    int *last_flag;
+};
+
+__device__ __forceinline__ Smem carve(char *smem, const Params &p) {
+    const Layout L = make_layout(p.stages, p.stage_bytes, p.B, p.r_k, p.r_v, p.d);
+    Smem s;
+    s.ring = smem + L.ring;
+    s.full = reinterpret_cast<uint64_t *>(smem + L.full);
+    s.empty = reinterpret_cast<uint64_t *>(smem + L.empty);
+    s.pfull = reinterpret_cast<uint64_t *>(smem + L.pfull);
+    s.pempty = reinterpret_cast<uint64_t *>(smem + L.pempty);
+    s.prefix = reinterpret_cast<int64_t *>(smem + L.prefix);
+    s.lens = reinterpret_cast<int *>(smem + L.lens);
+    s.qlat = reinterpret_cast<float *>(smem + L.qlat);
+    s.qfull = reinterpret_cast<float *>(smem + L.qfull);
+    s.spart = reinterpret_cast<float *>(smem + L.spart);
+    s.psm = reinterpret_cast<float *>(smem + L.psm);
+    s.tmp = reinterpret_cast<float *>(smem + L.tmp);
+    s.red = reinterpret_cast<float *>(smem + L.red);
+    s.lred = reinterpret_cast<float *>(smem + L.lred);
+    s.ovec = reinterpret_cast<float *>(smem + L.ovec);
+    s.misc = reinterpret_cast<float *>(smem + L.misc);
+    s.abort_flag = reinterpret_cast<volatile int *>(s.misc + kMiscAbort);
+    s.last_flag = reinterpret_cast<int *>(s.misc + kMiscLast);
+    return s;
+}
 
 template <int ES, int GB>
 __device__ __forceinline__ void load_gran(const char *p, float (&v)[GB / ES]) {
@@ -157,14 +201,149 @@ __device__ __forceinline__ int64_t range_start(int c, int64_t U, int Geff) {
     return static_cast<int64_t>(c) * U / Geff;
 }
 
+struct Range {
+    int64_t U, A0, A1;
+    int Geff;
+};
+
+// Barrier set-up and the per-sequence unit prefix (H heads x pages), with device-side length
+// checks.  All threads of the CTA; ends with __syncthreads.
+__device__ Range prologue(const Params &p, const Smem &s, uint32_t pfull_count,
+                          uint32_t pempty_count) {
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (tid == 0) {
+        for (int i = 0; i < p.stages; ++i) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], kComputeWarps);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s.pfull[i], pfull_count);
+            mbar_init(&s.pempty[i], pempty_count);
+        }
+        *s.abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        const int cap = min(p.max_ctx, p.max_blocks * kBlockTokens);
+        int64_t run = 0;
+        for (int b0 = 0; b0 < p.B; b0 += 32) {
+            const int b = b0 + lane;
+            int np = 0;
+            if (b < p.B) {
+                int Lb = p.context_lens[b];
+                if (Lb < 0 || Lb > cap) {
+                    if (blockIdx.x == 0) atomicOr(p.err, LLA_DEVERR_CONTEXT);
+                    Lb = max(0, min(Lb, cap));
+                }
+                s.lens[b] = Lb;
+                np = (Lb + kBlockTokens - 1) / kBlockTokens;
+            }
+            int v = np;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int n = __shfl_up_sync(0xffffffffu, v, o);
+                if (lane >= o) v += n;
+            }
+            if (b < p.B) s.prefix[b] = run + static_cast<int64_t>(v - np) * p.H;
+            run += static_cast<int64_t>(__shfl_sync(0xffffffffu, v, 31)) * p.H;
+        }
+        if (lane == 0) s.prefix[p.B] = run;
+    }
+    __syncthreads();
+    Range r;
+    r.U = s.prefix[p.B];
+    r.Geff = static_cast<int>(r.U < gridDim.x ? r.U : gridDim.x);
+    r.A0 = r.A1 = 0;
+    if (static_cast<int>(blockIdx.x) < r.Geff) {
+        r.A0 = range_start(blockIdx.x, r.U, r.Geff);
+        r.A1 = range_start(blockIdx.x + 1, r.U, r.Geff);
+    }
+    return r;
+}
+
+// One run: the part of a (sequence, head) inside this CTA's range.
+struct Run {
+    int b, h, Lb, pg0, npages;
+    int64_t seg_start, seg_end, run_end;
+};
+
+__device__ __forceinline__ Run locate_run(const Params &p, const Smem &s, int64_t u, int64_t A1) {
+    Run R;
+    R.b = seq_of_unit(s.prefix, p.B, u);
+    R.Lb = s.lens[R.b];
+    const int np = static_cast<int>((s.prefix[R.b + 1] - s.prefix[R.b]) / p.H);
+    const int64_t off = u - s.prefix[R.b];
+    R.h = static_cast<int>(off / np);
+    R.pg0 = static_cast<int>(off % np);
+    R.seg_start = s.prefix[R.b] + static_cast<int64_t>(R.h) * np;
+    R.seg_end = R.seg_start + np;
+    R.run_end = R.seg_end < A1 ? R.seg_end : A1;
+    R.npages = static_cast<int>(R.run_end - u);
+    return R;
+}
+
+// Producer: the whole warp walks the CTA's range.  Block ids are fetched 32 pages at a time
+// (one per lane) so the copies of consecutive steps are issued back to back instead of each
+// waiting for its own block-table load; lane 0 issues the bulk copies.
+__device__ void producer(const Params &p, const Smem &s, const Range &rg) {
+    const int lane = threadIdx.x & 31;
+    const int hpb = p.head_page_bytes;
+    const uint64_t pol = policy_evict_first();
+    int it = 0;
+    for (int64_t u = rg.A0; u < rg.A1;) {
+        const Run R = locate_run(p, s, u, rg.A1);
+        const int32_t *bt = p.block_table + static_cast<int64_t>(R.b) * p.max_blocks + R.pg0;
+        for (int k0 = 0; k0 < R.npages; k0 += 32) {
+            const int32_t blk_lane = (k0 + lane < R.npages) ? bt[k0 + lane] : -1;
+            const int kend = min(R.npages, k0 + 32);
+            for (int k = k0; k < kend; k += p.pps, ++it) {
+                int32_t blk[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    blk[i] = __shfl_sync(0xffffffffu, blk_lane, (k - k0 + i) & 31);
+                if (lane == 0) {
+                    const int stage = it % p.stages;
+                    const uint32_t ph = (it / p.stages) & 1;
+                    mbar_wait(&s.empty[stage], ph ^ 1u, s.abort_flag, p.err);
+                    const int n = min(p.pps, R.npages - k);
+                    uint32_t bytes = 0;
+                    for (int i = 0; i < n; ++i) {
+                        if (blk[i] < 0 || blk[i] >= p.num_blocks) {
+                            atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                            blk[i] = -1;
+                        } else {
+                            bytes += hpb;
+                        }
+                    }
+                    mbar_arrive_expect_tx(&s.full[stage], bytes);
+                    char *dst = s.ring + stage * p.stage_bytes;
+                    for (int i = 0; i < n; ++i)
+                        if (blk[i] >= 0)
+                            bulk_g2s(dst + i * hpb,
+                                     p.pool + blk[i] * p.block_bytes + static_cast<int64_t>(R.h) * hpb,
+                                     hpb, &s.full[stage], pol);
+                }
+                __syncwarp();
+            }
+        }
+        u = R.run_end;
+    }
+    if (lane == 0 && *s.abort_flag) {
+        // let the copies still in flight land before the CTA exits
+        volatile int never = 0;
+        const int first = it > p.stages ? it - p.stages : 0;
+        for (int j = first; j < it; ++j)
+            mbar_wait(&s.full[j % p.stages], (j / p.stages) & 1, &never, p.err);
+    }
+}
+
 // Query set-up of one (sequence, head): q in d-space, q~ = W_up,t^K^T q (or q itself for the
 // dense comparator) and beta = q . mu^K_t.  All consumer threads.
 template <int ES>
-__device__ void setup_query(const Params &p, int b, int h, float *qfull, float *qlat, float *tmp,
-                            float *misc) {
+__device__ void setup_query(const Params &p, const Smem &s, int b, int h) {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int64_t qoff = (static_cast<int64_t>(b) * p.H + h) * p.d;
-    for (int e = tid; e < p.d; e += kComputeThreads) qfull[e] = load_elem(p.q, qoff + e, p.io_bf16);
+    for (int e = tid; e < p.d; e += kComputeThreads) s.qfull[e] = load_elem(p.q, qoff + e, p.io_bf16);
     named_bar_sync(kBarAll, kComputeThreads);
     if (p.absorbed) {
         const int njp = p.r_k >> 1;
@@ -175,32 +354,31 @@ __device__ void setup_query(const Params &p, int b, int h, float *qfull, float *
             float a0 = 0.f, a1 = 0.f;
             for (int e = eg; e < p.d; e += neg) {
                 const float2 w = load_pair<ES>(p.w_up_k, w0 + static_cast<int64_t>(e) * p.r_k + 2 * jp);
-                const float qe = qfull[e];
+                const float qe = s.qfull[e];
                 a0 = fmaf(w.x, qe, a0);
                 a1 = fmaf(w.y, qe, a1);
             }
-            tmp[eg * p.r_k + 2 * jp] = a0;
-            tmp[eg * p.r_k + 2 * jp + 1] = a1;
+            s.tmp[eg * p.r_k + 2 * jp] = a0;
+            s.tmp[eg * p.r_k + 2 * jp + 1] = a1;
         }
         if (warp == kComputeWarps - 1) {
             float bsum = 0.f;
             if (p.mu_k) {
                 const float *mu = p.mu_k + (static_cast<int64_t>(h) * p.T + p.loop) * p.d;
-                for (int e = lane; e < p.d; e += 32) bsum = fmaf(qfull[e], mu[e], bsum);
+                for (int e = lane; e < p.d; e += 32) bsum = fmaf(s.qfull[e], mu[e], bsum);
             }
             bsum = warp_sum(bsum);
-            // written after the partial sums of this warp; read after the next barrier
-            if (lane == 0) misc[kMiscBeta] = bsum;
+            if (lane == 0) s.misc[kMiscBeta] = bsum;
         }
         named_bar_sync(kBarAll, kComputeThreads);
         for (int j = tid; j < p.r_k; j += kComputeThreads) {
-            float s = 0.f;
-            for (int g = 0; g < neg; ++g) s += tmp[g * p.r_k + j];
-            qlat[j] = s;
+            float acc = 0.f;
+            for (int g = 0; g < neg; ++g) acc += s.tmp[g * p.r_k + j];
+            s.qlat[j] = acc;
         }
     } else {
-        for (int e = tid; e < p.d; e += kComputeThreads) qlat[e] = qfull[e];
-        if (tid == 0) misc[kMiscBeta] = 0.f;
+        for (int e = tid; e < p.d; e += kComputeThreads) s.qlat[e] = s.qfull[e];
+        if (tid == 0) s.misc[kMiscBeta] = 0.f;
     }
     named_bar_sync(kBarAll, kComputeThreads);
 }
@@ -208,21 +386,21 @@ __device__ void setup_query(const Params &p, int b, int h, float *qfull, float *
 // Final output of one (sequence, head) from its cached softmax state: maximum m (log2 units),
 // mass l and latent value sum ovec (all relative to m).  All consumer threads.
 template <int ES>
-__device__ void finish_output(const Params &p, int b, int h, float m, float l, const float *ovec,
-                              const float *qfull, float *misc) {
+__device__ void finish_output(const Params &p, const Smem &s, int b, int h, float m, float l) {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool pass1 = p.cur_k != nullptr;
     const int64_t row = (static_cast<int64_t>(b) * p.H + h) * p.d;
     if (pass1 && warp == 0) {
-        float s = 0.f;
-        for (int e = lane; e < p.d; e += 32) s = fmaf(qfull[e], load_elem(p.cur_k, row + e, p.io_bf16), s);
-        s = warp_sum(s);
-        if (lane == 0) misc[kMiscScur] = s * p.scale_log2;
+        float acc = 0.f;
+        for (int e = lane; e < p.d; e += 32)
+            acc = fmaf(s.qfull[e], load_elem(p.cur_k, row + e, p.io_bf16), acc);
+        acc = warp_sum(acc);
+        if (lane == 0) s.misc[kMiscScur] = acc * p.scale_log2;
     }
     named_bar_sync(kBarAll, kComputeThreads);
     float M = m, pc = 0.f;
     if (pass1) {
-        const float sc = misc[kMiscScur];
+        const float sc = s.misc[kMiscScur];
         M = fmaxf(m, sc);
         pc = exp2f(sc - M);
     }
@@ -237,8 +415,8 @@ __device__ void finish_output(const Params &p, int b, int h, float m, float l, c
             float acc = 0.f;
             for (int jp = lane; jp < njp; jp += 32) {
                 const float2 w = load_pair<ES>(p.w_up_v, w0 + static_cast<int64_t>(e) * p.r_v + 2 * jp);
-                acc = fmaf(w.x, ovec[2 * jp], acc);
-                acc = fmaf(w.y, ovec[2 * jp + 1], acc);
+                acc = fmaf(w.x, s.ovec[2 * jp], acc);
+                acc = fmaf(w.y, s.ovec[2 * jp + 1], acc);
             }
             acc = warp_sum(acc);
             if (lane == 0) {
@@ -250,7 +428,7 @@ __device__ void finish_output(const Params &p, int b, int h, float m, float l, c
         }
     } else {
         for (int e = tid; e < p.d; e += kComputeThreads) {
-            float o = ovec[e] * wl;
+            float o = s.ovec[e] * wl;
             if (pass1) o = fmaf(pc, load_elem(p.cur_v, row + e, p.io_bf16), o);
             store_elem(p.out, row + e, o * inv, p.io_bf16);
         }
@@ -258,132 +436,118 @@ __device__ void finish_output(const Params &p, int b, int h, float m, float l, c
     named_bar_sync(kBarAll, kComputeThreads);
 }
 
+// After a run, with misc[kMiscM], misc[kMiscL] and ovec holding its softmax state: finish the
+// (sequence, head) in place when the run covers it, else leave a partial and, if this CTA is
+// the last to arrive, merge all partials by log-sum-exp and finish.  All consumer threads.
+template <class Finish>
+__device__ void finish_run(const Params &p, const Smem &s, const Run &R, int64_t u,
+                           const Range &rg) {
+    const int tid = threadIdx.x;
+    if (u == R.seg_start && R.run_end == R.seg_end) {
+        Finish::run(p, s, R.b, R.h, s.misc[kMiscM], s.misc[kMiscL]);
+        return;
+    }
+    // partial of a (sequence, head) split across CTAs: slot 0 if this is the CTA's first run,
+    // slot 1 if its last
+    const int c = blockIdx.x;
+    const int slot = (R.seg_start <= rg.A0) ? 0 : 1;
+    float *rec = p.partials + (static_cast<int64_t>(c) * 2 + slot) * (p.r_v + 2);
+    if (tid == 0) {
+        rec[0] = s.misc[kMiscM];
+        rec[1] = s.misc[kMiscL];
+    }
+    for (int j = tid; j < p.r_v; j += kComputeThreads) rec[2 + j] = s.ovec[j];
+    __threadfence();
+    named_bar_sync(kBarAll, kComputeThreads);
+    const int c_first = owner_of(R.seg_start, rg.U, rg.Geff);
+    const int c_last = owner_of(R.seg_end - 1, rg.U, rg.Geff);
+    int *counter = &p.counters[R.b * p.H + R.h];
+    if (tid == 0) {
+        const int prev = atomicAdd(counter, 1);
+        *s.last_flag = (prev == c_last - c_first);
+    }
+    named_bar_sync(kBarAll, kComputeThreads);
+    if (!*s.last_flag) return;
+    __threadfence();
+    auto record = [&](int cc) {
+        const int sl = (R.seg_start <= range_start(cc, rg.U, rg.Geff)) ? 0 : 1;
+        return p.partials + (static_cast<int64_t>(cc) * 2 + sl) * (p.r_v + 2);
+    };
+    // every part's (m, l) into shared memory (tmp: 2 x 256 floats), then the maximum
+    const int nparts = c_last - c_first + 1;
+    float M = -INFINITY, lsum = 0.f;
+    for (int c0 = 0; c0 < nparts; c0 += kComputeThreads) {
+        const int np = min(kComputeThreads, nparts - c0);
+        if (tid < np) {
+            const float *r = record(c_first + c0 + tid);
+            s.tmp[tid] = __ldcg(r);
+            s.tmp[kComputeThreads + tid] = __ldcg(r + 1);
+        }
+        named_bar_sync(kBarAll, kComputeThreads);
+        float Mc = M;
+        for (int i = 0; i < np; ++i) Mc = fmaxf(Mc, s.tmp[i]);
+        lsum *= exp2f(M - Mc);
+        for (int i = 0; i < np; ++i) lsum = fmaf(s.tmp[kComputeThreads + i], exp2f(s.tmp[i] - Mc), lsum);
+        M = Mc;
+        named_bar_sync(kBarAll, kComputeThreads);
+    }
+    for (int j = tid; j < p.r_v; j += kComputeThreads) {
+        float acc = 0.f;
+#pragma unroll 4
+        for (int cc = c_first; cc <= c_last; ++cc) {
+            const float *r = record(cc);
+            acc = fmaf(__ldcg(r + 2 + j), exp2f(__ldcg(r) - M), acc);
+        }
+        s.ovec[j] = acc;
+    }
+    named_bar_sync(kBarAll, kComputeThreads);
+    Finish::run(p, s, R.b, R.h, M, lsum);
+    if (tid == 0) atomicExch(counter, 0);
+}
+
+// Finisher of the generic kernel.
+template <int ES>
+struct GenericFinish {
+    __device__ static void run(const Params &p, const Smem &s, int b, int h, float m, float l) {
+        finish_output<ES>(p, s, b, h, m, l);
+    }
+};
+
+// Sequences with no cached token: pass 1 attends to the current token only.  Consumers.
+__device__ void empty_sequences(const Params &p, const Smem &s) {
+    const int tid = threadIdx.x;
+    const bool pass1 = p.cur_k != nullptr;
+    for (int b = 0; b < p.B; ++b) {
+        if (s.lens[b] != 0) continue;
+        for (int h = 0; h < p.H; ++h) {
+            if ((b * p.H + h) % gridDim.x != blockIdx.x) continue;
+            const int64_t row = (static_cast<int64_t>(b) * p.H + h) * p.d;
+            if (!pass1 && tid == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
+            for (int e = tid; e < p.d; e += kComputeThreads)
+                store_elem(p.out, row + e, pass1 ? load_elem(p.cur_v, row + e, p.io_bf16) : 0.f,
+                           p.io_bf16);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ generic kernel (any shape)
+
 template <int ES, int GK, int VB>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
     extern __shared__ __align__(128) char smem[];
-    const Layout L = make_layout(p.stages, p.stage_bytes, p.B, p.r_k, p.r_v, p.d);
-    char *ring = smem + L.ring;
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + L.full);
-    uint64_t *empty = reinterpret_cast<uint64_t *>(smem + L.empty);
-    int64_t *prefix = reinterpret_cast<int64_t *>(smem + L.prefix);
-    int *lens = reinterpret_cast<int *>(smem + L.lens);
-    float *qlat = reinterpret_cast<float *>(smem + L.qlat);
-    float *qfull = reinterpret_cast<float *>(smem + L.qfull);
-    float *spart = reinterpret_cast<float *>(smem + L.spart);
-    float *psm = reinterpret_cast<float *>(smem + L.psm);
-    float *tmp = reinterpret_cast<float *>(smem + L.tmp);
-    float *red = reinterpret_cast<float *>(smem + L.red);
-    float *lred = reinterpret_cast<float *>(smem + L.lred);
-    float *ovec = reinterpret_cast<float *>(smem + L.ovec);
-    float *misc = reinterpret_cast<float *>(smem + L.misc);
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + kMiscAbort);
-    int *last_flag = reinterpret_cast<int *>(misc + kMiscLast);
-
+    const Smem s = carve(smem, p);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int c = blockIdx.x;
     const int hpb = p.head_page_bytes;
 
-    // Inputs may come from the previous kernel in the stream.
-    pdl_wait();
-
-    if (tid == 0) {
-        for (int s = 0; s < p.stages; ++s) {
-            mbar_init(&full[s], 1);
-            mbar_init(&empty[s], kComputeWarps);
-        }
-        *abort_flag = 0;
-        fence_mbar_init();
-    }
-    // Units per sequence (H heads x pages), exclusive prefix; lengths checked on the device.
-    if (warp == 0) {
-        const int cap = min(p.max_ctx, p.max_blocks * kBlockTokens);
-        int64_t run = 0;
-        for (int b0 = 0; b0 < p.B; b0 += 32) {
-            const int b = b0 + lane;
-            int np = 0;
-            if (b < p.B) {
-                int Lb = p.context_lens[b];
-                if (Lb < 0 || Lb > cap) {
-                    if (c == 0) atomicOr(p.err, LLA_DEVERR_CONTEXT);
-                    Lb = max(0, min(Lb, cap));
-                }
-                lens[b] = Lb;
-                np = (Lb + kBlockTokens - 1) / kBlockTokens;
-            }
-            int v = np;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int n = __shfl_up_sync(0xffffffffu, v, o);
-                if (lane >= o) v += n;
-            }
-            if (b < p.B) prefix[b] = run + static_cast<int64_t>(v - np) * p.H;
-            run += static_cast<int64_t>(__shfl_sync(0xffffffffu, v, 31)) * p.H;
-        }
-        if (lane == 0) prefix[p.B] = run;
-    }
-    __syncthreads();
+    pdl_wait();  // inputs may come from the previous kernel in the stream
+    const Range rg = prologue(p, s, 1, 1);
     pdl_trigger();
 
-    const int64_t U = prefix[p.B];
-    const int Geff = static_cast<int>(U < gridDim.x ? U : gridDim.x);
-    int64_t A0 = 0, A1 = 0;
-    if (c < Geff) {
-        A0 = range_start(c, U, Geff);
-        A1 = range_start(c + 1, U, Geff);
-    }
-
     if (warp == kComputeWarps) {
-        // ------------------------------------------------------------------ producer warp
-        if (lane == 0) {
-            const uint64_t pol = policy_evict_first();
-            int it = 0;
-            for (int64_t u = A0; u < A1;) {
-                const int b = seq_of_unit(prefix, p.B, u);
-                const int np = static_cast<int>((prefix[b + 1] - prefix[b]) / p.H);
-                const int64_t off = u - prefix[b];
-                const int h = static_cast<int>(off / np);
-                const int pg0 = static_cast<int>(off % np);
-                const int64_t seg_end = prefix[b] + static_cast<int64_t>(h + 1) * np;
-                const int64_t run_end = seg_end < A1 ? seg_end : A1;
-                const int npages = static_cast<int>(run_end - u);
-                const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks + pg0;
-                for (int k = 0; k < npages; k += p.pps, ++it) {
-                    const int stage = it % p.stages;
-                    const uint32_t ph = (it / p.stages) & 1;
-                    mbar_wait(&empty[stage], ph ^ 1u, abort_flag, p.err);
-                    const int n = min(p.pps, npages - k);
-                    int32_t blk[4];
-                    uint32_t bytes = 0;
-                    for (int i = 0; i < n; ++i) {
-                        blk[i] = bt[k + i];
-                        if (blk[i] < 0 || blk[i] >= p.num_blocks) {
-                            atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
-                            blk[i] = -1;
-                        } else {
-                            bytes += hpb;
-                        }
-                    }
-                    mbar_arrive_expect_tx(&full[stage], bytes);
-                    char *dst = ring + stage * p.stage_bytes;
-                    for (int i = 0; i < n; ++i)
-                        if (blk[i] >= 0)
-                            bulk_g2s(dst + i * hpb, p.pool + blk[i] * p.block_bytes + static_cast<int64_t>(h) * hpb,
-                                     hpb, &full[stage], pol);
-                }
-                u = run_end;
-            }
-            if (*abort_flag) {
-                // let the copies still in flight land before the CTA exits
-                volatile int never = 0;
-                const int first = it > p.stages ? it - p.stages : 0;
-                for (int j = first; j < it; ++j)
-                    mbar_wait(&full[j % p.stages], (j / p.stages) & 1, &never, p.err);
-            }
-        }
+        producer(p, s, rg);
         return;
     }
 
-    // ---------------------------------------------------------------------- consumer warps
     constexpr int KE = GK / ES;  // elements per K granule
     constexpr int VE = VB / ES;  // elements per V unit
     const int TOK = p.pps * kBlockTokens;
@@ -393,37 +557,26 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
     const int NTG = kComputeThreads / NVU;
     const int vu = tid % NVU, tg = tid / NVU;
     const bool vthread = tg < NTG;
-    const bool pass1 = p.cur_k != nullptr;
 
     int it = 0;
-    for (int64_t u = A0; u < A1;) {
-        const int b = seq_of_unit(prefix, p.B, u);
-        const int Lb = lens[b];
-        const int np = static_cast<int>((prefix[b + 1] - prefix[b]) / p.H);
-        const int64_t off = u - prefix[b];
-        const int h = static_cast<int>(off / np);
-        const int pg0 = static_cast<int>(off % np);
-        const int64_t seg_start = prefix[b] + static_cast<int64_t>(h) * np;
-        const int64_t seg_end = seg_start + np;
-        const int64_t run_end = seg_end < A1 ? seg_end : A1;
-        const int npages = static_cast<int>(run_end - u);
-
-        setup_query<ES>(p, b, h, qfull, qlat, tmp, misc);
-        const float beta = misc[kMiscBeta];
+    for (int64_t u = rg.A0; u < rg.A1;) {
+        const Run R = locate_run(p, s, u, rg.A1);
+        setup_query<ES>(p, s, R.b, R.h);
+        const float beta = s.misc[kMiscBeta];
 
         float m_run = -INFINITY, l_part = 0.f;
         float accv[VE];
 #pragma unroll
         for (int k = 0; k < VE; ++k) accv[k] = 0.f;
 
-        for (int k = 0; k < npages; k += p.pps, ++it) {
+        for (int k = 0; k < R.npages; k += p.pps, ++it) {
             const int stage = it % p.stages;
             const uint32_t ph = (it / p.stages) & 1;
-            mbar_wait(&full[stage], ph, abort_flag, p.err);
-            const char *sb = ring + stage * p.stage_bytes;
-            const int n = min(p.pps, npages - k);
-            const int tok0 = (pg0 + k) * kBlockTokens;  // sequence position of the step's row 0
-            const int nvalid = min(n * kBlockTokens, Lb - tok0);
+            mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+            const char *sb = s.ring + stage * p.stage_bytes;
+            const int n = min(p.pps, R.npages - k);
+            const int tok0 = (R.pg0 + k) * kBlockTokens;  // sequence position of row 0
+            const int nvalid = min(n * kBlockTokens, R.Lb - tok0);
 
             // scores: partial dot products of q~ with the K-plane rows
             {
@@ -435,42 +588,42 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
                     for (int g = sp; g < NGK; g += SPLIT) {
                         float v[KE];
                         load_gran<ES, GK>(kp + g * (kBlockTokens * GK), v);
-                        const float *qq = qlat + g * KE;
+                        const float *qq = s.qlat + g * KE;
 #pragma unroll
                         for (int e = 0; e < KE; ++e) acc = fmaf(v[e], qq[e], acc);
                     }
                 }
-                spart[sp * TOK + tk] = acc;
+                s.spart[sp * TOK + tk] = acc;
             }
             named_bar_sync(kBarAll, kComputeThreads);
             // online softmax over the step's tokens (threads that own a token)
             if (tid < TOK) {
-                float s = 0.f;
-                for (int sp = 0; sp < SPLIT; ++sp) s += spart[sp * TOK + tid];
+                float sc = 0.f;
+                for (int sp = 0; sp < SPLIT; ++sp) sc += s.spart[sp * TOK + tid];
                 const bool valid = tid < nvalid;
-                const float x = valid ? (s + beta) * p.scale_log2 : -INFINITY;
+                const float x = valid ? (sc + beta) * p.scale_log2 : -INFINITY;
                 const float wm = warp_max(x);
-                if (lane == 0) misc[kMiscWmax + warp] = wm;
+                if (lane == 0) s.misc[kMiscWmax + warp] = wm;
                 named_bar_sync(kBarTok, TOK);
-                float ms = misc[kMiscWmax];
-                for (int w = 1; w < (TOK >> 5); ++w) ms = fmaxf(ms, misc[kMiscWmax + w]);
+                float ms = s.misc[kMiscWmax];
+                for (int w = 1; w < (TOK >> 5); ++w) ms = fmaxf(ms, s.misc[kMiscWmax + w]);
                 const float m_new = fmaxf(m_run, ms);
                 const float alpha = exp2f(m_run - m_new);
                 const float pv = valid ? exp2f(x - m_new) : 0.f;
                 l_part = fmaf(l_part, alpha, pv);
-                psm[tid] = pv;
-                if (tid == 0) misc[kMiscAlpha] = alpha;
+                s.psm[tid] = pv;
+                if (tid == 0) s.misc[kMiscAlpha] = alpha;
                 m_run = m_new;
             }
             named_bar_sync(kBarAll, kComputeThreads);
             // latent value accumulation: sum_i p_i c_v,i
             if (vthread) {
-                const float alpha = misc[kMiscAlpha];
+                const float alpha = s.misc[kMiscAlpha];
 #pragma unroll
                 for (int e = 0; e < VE; ++e) accv[e] *= alpha;
                 const char *vp = sb + p.kplane_bytes + vu * VB;
                 for (int tk = tg; tk < nvalid; tk += NTG) {
-                    const float pv = psm[tk];
+                    const float pv = s.psm[tk];
                     float v[VE];
                     load_gran<ES, VB>(vp + (tk >> 6) * hpb + (tk & 63) * (p.r_v * ES), v);
 #pragma unroll
@@ -478,100 +631,469 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
                 }
             }
             __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[stage]);
+            if (lane == 0) mbar_arrive(&s.empty[stage]);
         }
 
         // reduce the run's softmax state across threads
-        if (tid < TOK) lred[tid] = l_part;
+        if (tid < TOK) s.lred[tid] = l_part;
         if (vthread) {
 #pragma unroll
-            for (int e = 0; e < VE; ++e) red[tg * p.r_v + vu * VE + e] = accv[e];
+            for (int e = 0; e < VE; ++e) s.red[tg * p.r_v + vu * VE + e] = accv[e];
         }
-        if (tid == 0) misc[kMiscM] = m_run;
+        if (tid == 0) s.misc[kMiscM] = m_run;
         named_bar_sync(kBarAll, kComputeThreads);
         for (int j = tid; j < p.r_v; j += kComputeThreads) {
-            float s = 0.f;
-            for (int g = 0; g < NTG; ++g) s += red[g * p.r_v + j];
-            ovec[j] = s;
+            float acc = 0.f;
+            for (int g = 0; g < NTG; ++g) acc += s.red[g * p.r_v + j];
+            s.ovec[j] = acc;
         }
         if (warp == 0) {
-            float s = 0.f;
-            for (int i = lane; i < TOK; i += 32) s += lred[i];
-            s = warp_sum(s);
-            if (lane == 0) misc[kMiscL] = s;
+            float acc = 0.f;
+            for (int i = lane; i < TOK; i += 32) acc += s.lred[i];
+            acc = warp_sum(acc);
+            if (lane == 0) s.misc[kMiscL] = acc;
         }
         named_bar_sync(kBarAll, kComputeThreads);
-
-        if (u == seg_start && run_end == seg_end) {
-            finish_output<ES>(p, b, h, misc[kMiscM], misc[kMiscL], ovec, qfull, misc);
-        } else {
-            // partial of a (sequence, head) split across CTAs: slot 0 if this is the CTA's first
-            // run, slot 1 if its last
-            const int slot = (seg_start <= A0) ? 0 : 1;
-            float *rec = p.partials + (static_cast<int64_t>(c) * 2 + slot) * (p.r_v + 2);
-            if (tid == 0) {
-                rec[0] = misc[kMiscM];
-                rec[1] = misc[kMiscL];
-            }
-            for (int j = tid; j < p.r_v; j += kComputeThreads) rec[2 + j] = ovec[j];
-            __threadfence();
-            named_bar_sync(kBarAll, kComputeThreads);
-            const int c_first = owner_of(seg_start, U, Geff);
-            const int c_last = owner_of(seg_end - 1, U, Geff);
-            if (tid == 0) {
-                const int prev = atomicAdd(&p.counters[b * p.H + h], 1);
-                *last_flag = (prev == c_last - c_first);
-            }
-            named_bar_sync(kBarAll, kComputeThreads);
-            if (*last_flag) {
-                __threadfence();
-                float M = -INFINITY;
-                for (int cc = c_first; cc <= c_last; ++cc) {
-                    const int sl = (seg_start <= range_start(cc, U, Geff)) ? 0 : 1;
-                    M = fmaxf(M, __ldcg(p.partials + (static_cast<int64_t>(cc) * 2 + sl) * (p.r_v + 2)));
-                }
-                float lsum = 0.f;
-                for (int cc = c_first; cc <= c_last; ++cc) {
-                    const int sl = (seg_start <= range_start(cc, U, Geff)) ? 0 : 1;
-                    const float *r = p.partials + (static_cast<int64_t>(cc) * 2 + sl) * (p.r_v + 2);
-                    lsum += __ldcg(r + 1) * exp2f(__ldcg(r) - M);
-                }
-                named_bar_sync(kBarAll, kComputeThreads);  // ovec is rewritten below
-                for (int j = tid; j < p.r_v; j += kComputeThreads) {
-                    float s = 0.f;
-                    for (int cc = c_first; cc <= c_last; ++cc) {
-                        const int sl = (seg_start <= range_start(cc, U, Geff)) ? 0 : 1;
-                        const float *r = p.partials + (static_cast<int64_t>(cc) * 2 + sl) * (p.r_v + 2);
-                        s = fmaf(__ldcg(r + 2 + j), exp2f(__ldcg(r) - M), s);
-                    }
-                    ovec[j] = s;
-                }
-                named_bar_sync(kBarAll, kComputeThreads);
-                finish_output<ES>(p, b, h, M, lsum, ovec, qfull, misc);
-                if (tid == 0) atomicExch(&p.counters[b * p.H + h], 0);
-            }
-        }
-        u = run_end;
+        finish_run<GenericFinish<ES>>(p, s, R, u, rg);
+        u = R.run_end;
     }
+    empty_sequences(p, s);
+}
 
-    // sequences with no cached token: pass 1 attends to the current token only
-    for (int b = 0; b < p.B; ++b) {
-        if (lens[b] != 0) continue;
-        for (int h = 0; h < p.H; ++h) {
-            if ((b * p.H + h) % gridDim.x != c) continue;
-            const int64_t row = (static_cast<int64_t>(b) * p.H + h) * p.d;
-            if (!pass1 && tid == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
-            for (int e = tid; e < p.d; e += kComputeThreads)
-                store_elem(p.out, row + e, pass1 ? load_elem(p.cur_v, row + e, p.io_bf16) : 0.f,
-                           p.io_bf16);
-        }
+// --------------------------------------------- shape-specialised kernel (Ouro rank shapes)
+
+template <int ES, int RK, int RV>
+struct Fast {
+    static constexpr int HPB = kBlockTokens * (RK + RV) * ES;  // head page bytes
+    static constexpr int PPS = (4 * HPB <= kStepTargetBytes) ? 4 : (2 * HPB <= kStepTargetBytes) ? 2 : 1;
+    static constexpr int TOK = PPS * kBlockTokens;             // tokens per pipeline step
+    static constexpr int GK = ((RK * ES) % 16 == 0) ? 16 : 4;  // K granule bytes
+    static constexpr int KE = GK / ES;                         // elements per K granule
+    static constexpr int NGK = RK * ES / GK;                   // K granules per token
+    // Score threads: TT threads per k-split, each owning TPT tokens; KSPLIT groups share a
+    // token's granules so that the score role has up to four warps.
+    static constexpr int TPT = TOK > 128 ? TOK / 128 : 1;
+    static constexpr int TT = TOK / TPT;
+    static constexpr int KSPLIT = (TT <= 64 && NGK > 6) ? 2 : 1;
+    static constexpr int NGT = (NGK + KSPLIT - 1) / KSPLIT;    // granules per k-split
+    static constexpr int S_THREADS = TT * KSPLIT;
+    static constexpr int S_WARPS = S_THREADS / 32;
+    static constexpr int V_WARPS = kComputeWarps - S_WARPS;
+    static constexpr int V_THREADS = V_WARPS * 32;
+    static constexpr int VB = ((RV * ES) % 16 == 0) ? 16 : 4;  // V unit bytes
+    static constexpr int VE = VB / ES;                         // elements per V unit
+    static constexpr int VU = RV * ES / VB;                    // V units per row
+    static constexpr int NTG = V_THREADS / VU;                 // token groups of value threads
+    // Two CTAs share an SM when two pipeline stages each fit in half of its shared memory: one
+    // CTA's run set-up and merge then overlap the other's streaming.
+    static constexpr int CTAS = (2 * PPS * HPB + 24 * 1024 <= kHalfSmem) ? 2 : 1;
+    static_assert(S_THREADS % 32 == 0 && S_WARPS >= 1 && V_WARPS >= 1, "role split");
+    static_assert(NTG >= 1 && TT * TPT == TOK, "every token has a score thread");
+    static_assert(KE % 4 == 0 || KE <= 2, "q~ vector loads");
+    static_assert(TT % 32 == 0, "score-owning threads are whole warps");
+};
+
+// Bytes of the widest aligned load that splits `bytes` evenly (16, 8 or 4).
+__host__ __device__ constexpr int chunk_bytes(int bytes) {
+    return (bytes % 16 == 0) ? 16 : (bytes % 8 == 0) ? 8 : 4;
+}
+
+// Raw (packed) chunk of CB bytes, and its conversion to CB/ES floats.
+template <int CB> struct RawChunk;
+template <> struct RawChunk<16> { using T = uint4; };
+template <> struct RawChunk<8> { using T = uint2; };
+template <> struct RawChunk<4> { using T = uint32_t; };
+
+template <int CB>
+__device__ __forceinline__ typename RawChunk<CB>::T load_raw(const char *p) {
+    return *reinterpret_cast<const typename RawChunk<CB>::T *>(p);
+}
+
+template <int ES>
+__device__ __forceinline__ void unpack_word(uint32_t u, float *v) {
+    if constexpr (ES == 2) {
+        const float2 a = bf2_to_f2(u);
+        v[0] = a.x;
+        v[1] = a.y;
+    } else {
+        v[0] = __uint_as_float(u);
     }
 }
 
-template <int ES, int GK, int VB>
-lla_status launch_t(const Params &prm, int grid, int smem, cudaStream_t stream) {
-    auto kern = decode_kernel<ES, GK, VB>;
-    static bool configured[64] = {};
+template <int ES>
+__device__ __forceinline__ void unpack(const uint4 &u, float *v) {
+    constexpr int W = 4 / ES;  // elements per 32-bit word
+    unpack_word<ES>(u.x, v); unpack_word<ES>(u.y, v + W); unpack_word<ES>(u.z, v + 2 * W);
+    unpack_word<ES>(u.w, v + 3 * W);
+}
+template <int ES>
+__device__ __forceinline__ void unpack(const uint2 &u, float *v) {
+    constexpr int W = 4 / ES;
+    unpack_word<ES>(u.x, v); unpack_word<ES>(u.y, v + W);
+}
+template <int ES>
+__device__ __forceinline__ void unpack(const uint32_t &u, float *v) { unpack_word<ES>(u, v); }
+
+constexpr int kMaxChunksInFlight = 10;  // per thread and round trip
+
+// Query set-up with compile-time shapes: every thread issues its W_up,t^K loads (at most
+// kMaxChunksInFlight per round trip) before using any.  q~[j] = sum_e W[e][j] q[e].
+template <int ES, int RK, int D>
+__device__ void fast_setup_query(const Params &p, const Smem &s, int b, int h) {
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int64_t qoff = (static_cast<int64_t>(b) * p.H + h) * D;
+    for (int e = tid; e < D; e += kComputeThreads) s.qfull[e] = load_elem(p.q, qoff + e, p.io_bf16);
+    if (!p.absorbed) {
+        named_bar_sync(kBarAll, kComputeThreads);
+        for (int e = tid; e < D; e += kComputeThreads) s.qlat[e] = s.qfull[e];
+        if (tid == 0) s.misc[kMiscBeta] = 0.f;
+        named_bar_sync(kBarAll, kComputeThreads);
+        return;
+    }
+    constexpr int CB = chunk_bytes(RK * ES);  // load width along a row of W
+    constexpr int CE = CB / ES;
+    constexpr int CPR = RK * ES / CB;          // chunks per row
+    constexpr int RG = kComputeThreads / CPR;  // row groups
+    constexpr int ROWS = (D + RG - 1) / RG;    // rows per thread
+    constexpr int BATCH = ROWS < kMaxChunksInFlight ? ROWS : kMaxChunksInFlight;
+    static_assert(RG * RK <= 8 * kComputeThreads, "partial sums fit the reduction buffer");
+    using Raw = typename RawChunk<CB>::T;
+    const int cg = tid % CPR, rg = tid / CPR;
+    const char *W = static_cast<const char *>(p.w_up_k) +
+                    ((static_cast<int64_t>(h) * p.T + p.loop) * D * RK + cg * CE) * ES;
+    Raw w[BATCH];
+    if (rg < RG) {
+#pragma unroll
+        for (int k = 0; k < BATCH; ++k) {
+            const int e = rg + k * RG;
+            if (e < D) w[k] = load_raw<CB>(W + static_cast<int64_t>(e) * RK * ES);
+        }
+    }
+    named_bar_sync(kBarAll, kComputeThreads);  // qfull ready
+    if (warp == kComputeWarps - 1) {
+        float bsum = 0.f;
+        if (p.mu_k) {
+            const float *mu = p.mu_k + (static_cast<int64_t>(h) * p.T + p.loop) * D;
+            for (int e = lane; e < D; e += 32) bsum = fmaf(s.qfull[e], mu[e], bsum);
+        }
+        bsum = warp_sum(bsum);
+        if (lane == 0) s.misc[kMiscBeta] = bsum;
+    }
+    if (rg < RG) {
+        float acc[CE];
+#pragma unroll
+        for (int i = 0; i < CE; ++i) acc[i] = 0.f;
+#pragma unroll
+        for (int k0 = 0; k0 < ROWS; k0 += BATCH) {
+            if (k0 > 0) {
+#pragma unroll
+                for (int k = 0; k < BATCH; ++k) {
+                    const int e = rg + (k0 + k) * RG;
+                    if (k0 + k < ROWS && e < D) w[k] = load_raw<CB>(W + static_cast<int64_t>(e) * RK * ES);
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < BATCH; ++k) {
+                const int e = rg + (k0 + k) * RG;
+                if (k0 + k < ROWS && e < D) {
+                    float v[CE];
+                    unpack<ES>(w[k], v);
+                    const float qe = s.qfull[e];
+#pragma unroll
+                    for (int i = 0; i < CE; ++i) acc[i] = fmaf(v[i], qe, acc[i]);
+                }
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < CE; ++i) s.red[rg * RK + cg * CE + i] = acc[i];
+    }
+    named_bar_sync(kBarAll, kComputeThreads);
+    for (int j = tid; j < RK; j += kComputeThreads) {
+        float acc = 0.f;
+#pragma unroll 4
+        for (int g = 0; g < RG; ++g) acc += s.red[g * RK + j];
+        s.qlat[j] = acc;
+    }
+    named_bar_sync(kBarAll, kComputeThreads);
+}
+
+// Output with compile-time shapes: TPR threads per output row, each issuing its W_up,t^V
+// loads (at most kMaxChunksInFlight per round trip) before using any.
+// o = (W ovec wl + lc mu^V_t + p_cur v_cur) / (lc + p_cur).
+template <int ES, int RV, int D>
+struct FastFinish {
+    static constexpr int TPR = ((RV / 2) % 2 == 0 && D * 2 <= kComputeThreads) ? 2 : 1;
+    static constexpr int COLS = RV / TPR;      // columns per thread
+    static constexpr int CB = chunk_bytes(COLS * ES);
+    static constexpr int CE = CB / ES;
+    static constexpr int NCH = COLS / CE;      // chunks per thread
+    static constexpr int BATCH = NCH < kMaxChunksInFlight ? NCH : kMaxChunksInFlight;
+    static_assert(D * TPR <= kComputeThreads, "one pass over the rows");
+    using Raw = typename RawChunk<CB>::T;
+
+    __device__ static void run(const Params &p, const Smem &s, int b, int h, float m, float l) {
+        const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+        const bool pass1 = p.cur_k != nullptr;
+        const int64_t row = (static_cast<int64_t>(b) * p.H + h) * D;
+        if (!p.absorbed) {
+            finish_output<ES>(p, s, b, h, m, l);
+            return;
+        }
+        const int e = tid / TPR, half = tid % TPR;
+        const bool active = e < D;
+        const char *W = static_cast<const char *>(p.w_up_v) +
+                        ((static_cast<int64_t>(h) * p.T + p.loop) * D * RV +
+                         static_cast<int64_t>(e) * RV + half * COLS) * ES;
+        Raw w[BATCH];
+        if (active) {
+#pragma unroll
+            for (int k = 0; k < BATCH; ++k) w[k] = load_raw<CB>(W + k * CB);
+        }
+        float vcur = 0.f, muv = 0.f;
+        if (active && half == 0) {
+            if (pass1) vcur = load_elem(p.cur_v, row + e, p.io_bf16);
+            if (p.mu_v) muv = p.mu_v[(static_cast<int64_t>(h) * p.T + p.loop) * D + e];
+        }
+        if (pass1 && warp == 0) {
+            float acc = 0.f;
+            for (int i = lane; i < D; i += 32)
+                acc = fmaf(s.qfull[i], load_elem(p.cur_k, row + i, p.io_bf16), acc);
+            acc = warp_sum(acc);
+            if (lane == 0) s.misc[kMiscScur] = acc * p.scale_log2;
+        }
+        named_bar_sync(kBarAll, kComputeThreads);
+        float M = m, pc = 0.f;
+        if (pass1) {
+            const float sc = s.misc[kMiscScur];
+            M = fmaxf(m, sc);
+            pc = exp2f(sc - M);
+        }
+        const float wl = exp2f(m - M);
+        const float lc = l * wl;
+        const float inv = 1.f / (lc + pc);
+        float acc = 0.f;
+        if (active) {
+            const float *ov = s.ovec + half * COLS;
+#pragma unroll
+            for (int k0 = 0; k0 < NCH; k0 += BATCH) {
+                if (k0 > 0) {
+#pragma unroll
+                    for (int k = 0; k < BATCH; ++k)
+                        if (k0 + k < NCH) w[k] = load_raw<CB>(W + (k0 + k) * CB);
+                }
+#pragma unroll
+                for (int k = 0; k < BATCH; ++k) {
+                    if (k0 + k < NCH) {
+                        float v[CE];
+                        unpack<ES>(w[k], v);
+#pragma unroll
+                        for (int i = 0; i < CE; ++i) acc = fmaf(v[i], ov[(k0 + k) * CE + i], acc);
+                    }
+                }
+            }
+        }
+        if constexpr (TPR == 2) acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+        if (active && half == 0) {
+            float o = acc * wl;
+            if (p.mu_v) o = fmaf(lc, muv, o);
+            if (pass1) o = fmaf(pc, vcur, o);
+            store_elem(p.out, row + e, o * inv, p.io_bf16);
+        }
+        named_bar_sync(kBarAll, kComputeThreads);
+    }
+};
+
+// KE consecutive floats of q~ from shared memory (16-byte aligned at every granule start).
+template <int KE>
+__device__ __forceinline__ void load_qvec(const float *q, float (&v)[KE]) {
+    if constexpr (KE % 4 == 0) {
+#pragma unroll
+        for (int i = 0; i < KE; i += 4) {
+            const float4 t = *reinterpret_cast<const float4 *>(q + i);
+            v[i] = t.x; v[i + 1] = t.y; v[i + 2] = t.z; v[i + 3] = t.w;
+        }
+    } else if constexpr (KE == 2) {
+        const float2 t = *reinterpret_cast<const float2 *>(q);
+        v[0] = t.x; v[1] = t.y;
+    } else {
+#pragma unroll
+        for (int i = 0; i < KE; ++i) v[i] = q[i];
+    }
+}
+
+template <int ES, int RK, int RV, int D>
+__global__ void __launch_bounds__(kThreads, Fast<ES, RK, RV>::CTAS) decode_fast_kernel(const Params p) {
+    using F = Fast<ES, RK, RV>;
+    extern __shared__ __align__(128) char smem[];
+    const Smem s = carve(smem, p);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    pdl_wait();  // inputs may come from the previous kernel in the stream
+    const Range rg = prologue(p, s, F::S_THREADS, F::V_THREADS);
+    pdl_trigger();
+
+    if (warp == kComputeWarps) {
+        producer(p, s, rg);
+        return;
+    }
+
+    const bool is_s = warp < F::S_WARPS;
+    // score threads: k-split ks, token thread tt (tokens tt + i*TT)
+    const int ks = tid / F::TT, tt = tid % F::TT;
+    // value threads: column unit vu, token group tg (tokens tg + i*NTG)
+    const int vt = tid - F::S_THREADS;
+    const int vu = vt % F::VU, tg = vt / F::VU;
+    const bool vwork = !is_s && tg < F::NTG;
+
+    int it = 0;
+    for (int64_t u = rg.A0; u < rg.A1;) {
+        const Run R = locate_run(p, s, u, rg.A1);
+        fast_setup_query<ES, RK, D>(p, s, R.b, R.h);
+        const float beta = s.misc[kMiscBeta];
+
+        float m_run = -INFINITY, l_part = 0.f;
+        float accv[F::VE];
+#pragma unroll
+        for (int e = 0; e < F::VE; ++e) accv[e] = 0.f;
+        const float *qq = s.qlat + ks * F::NGT * F::KE;  // this k-split's part of q~
+
+        for (int k = 0; k < R.npages; k += F::PPS, ++it) {
+            const int stage = it % p.stages;
+            const uint32_t ph = (it / p.stages) & 1;
+            const int slot = it & 1;
+            const uint32_t pph = (it >> 1) & 1;
+            const char *sb = s.ring + stage * p.stage_bytes;
+            const int n = min(F::PPS, R.npages - k);
+            const int tok0 = (R.pg0 + k) * kBlockTokens;
+            const int nvalid = min(n * kBlockTokens, R.Lb - tok0);
+            float *pring = s.psm + slot * kComputeThreads;
+
+            if (is_s) {
+                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+                float sc[F::TPT];
+#pragma unroll
+                for (int i = 0; i < F::TPT; ++i) {
+                    const int tok = tt + i * F::TT;
+                    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+                    if (tok < nvalid) {
+                        const char *kp = sb + (tok >> 6) * F::HPB + (tok & 63) * F::GK +
+                                         ks * F::NGT * (kBlockTokens * F::GK);
+#pragma unroll 4
+                        for (int g = 0; g < F::NGT; ++g) {
+                            if (F::NGK % F::KSPLIT != 0 && ks * F::NGT + g >= F::NGK) break;
+                            float v[F::KE], qv[F::KE];
+                            load_gran<ES, F::GK>(kp + g * (kBlockTokens * F::GK), v);
+                            load_qvec<F::KE>(qq + g * F::KE, qv);  // broadcast read
+#pragma unroll
+                            for (int e = 0; e < F::KE; ++e) {
+                                if ((e & 3) == 0) a0 = fmaf(v[e], qv[e], a0);
+                                else if ((e & 3) == 1) a1 = fmaf(v[e], qv[e], a1);
+                                else if ((e & 3) == 2) a2 = fmaf(v[e], qv[e], a2);
+                                else a3 = fmaf(v[e], qv[e], a3);
+                            }
+                        }
+                    }
+                    sc[i] = (a0 + a1) + (a2 + a3);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s.empty[stage]);  // K-plane read
+                if constexpr (F::KSPLIT == 2) {
+                    if (ks == 1) {
+#pragma unroll
+                        for (int i = 0; i < F::TPT; ++i) s.spart[tt + i * F::TT] = sc[i];
+                    }
+                    named_bar_sync(kBarTok, F::S_THREADS);
+                    if (ks == 0) {
+#pragma unroll
+                        for (int i = 0; i < F::TPT; ++i) sc[i] += s.spart[tt + i * F::TT];
+                    }
+                }
+                float x[F::TPT];
+                float lm = -INFINITY;
+#pragma unroll
+                for (int i = 0; i < F::TPT; ++i) {
+                    const bool valid = tt + i * F::TT < nvalid;
+                    x[i] = valid ? (sc[i] + beta) * p.scale_log2 : -INFINITY;
+                    lm = fmaxf(lm, x[i]);
+                }
+                float *wmax = s.misc + kMiscWmax + (it & 1) * 8;
+                if (ks == 0) {
+                    lm = warp_max(lm);
+                    if (lane == 0) wmax[warp] = lm;
+                }
+                named_bar_sync(kBarTok, F::S_THREADS);
+                float ms = wmax[0];
+#pragma unroll
+                for (int w = 1; w < F::TT / 32; ++w) ms = fmaxf(ms, wmax[w]);
+                const float m_new = fmaxf(m_run, ms);
+                const float alpha = exp2f(m_run - m_new);
+                m_run = m_new;
+                if (ks == 0) {
+                    mbar_wait(&s.pempty[slot], pph ^ 1u, s.abort_flag, p.err);
+                    float lsum = 0.f;
+#pragma unroll
+                    for (int i = 0; i < F::TPT; ++i) {
+                        const float pv = (tt + i * F::TT < nvalid) ? exp2f(x[i] - m_new) : 0.f;
+                        pring[tt + i * F::TT] = pv;
+                        lsum += pv;
+                    }
+                    l_part = fmaf(l_part, alpha, lsum);
+                    if (tid == 0) s.misc[kMiscPAlpha + slot] = alpha;
+                }
+                mbar_arrive(&s.pfull[slot]);
+            } else {
+                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+                mbar_wait(&s.pfull[slot], pph, s.abort_flag, p.err);
+                if (vwork) {
+                    const float alpha = s.misc[kMiscPAlpha + slot];
+#pragma unroll
+                    for (int e = 0; e < F::VE; ++e) accv[e] *= alpha;
+                    const char *vp = sb + kBlockTokens * RK * ES + vu * F::VB;
+#pragma unroll 4
+                    for (int tk = tg; tk < nvalid; tk += F::NTG) {
+                        const float pv = pring[tk];
+                        float v[F::VE];
+                        load_gran<ES, F::VB>(vp + (tk >> 6) * F::HPB + (tk & 63) * (RV * ES), v);
+#pragma unroll
+                        for (int e = 0; e < F::VE; ++e) accv[e] = fmaf(pv, v[e], accv[e]);
+                    }
+                }
+                mbar_arrive(&s.pempty[slot]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s.empty[stage]);  // V-plane read
+            }
+        }
+
+        // reduce the run's softmax state across threads
+        if (is_s && ks == 0) s.lred[tt] = l_part;
+        if (vwork) {
+#pragma unroll
+            for (int e = 0; e < F::VE; ++e) s.red[tg * RV + vu * F::VE + e] = accv[e];
+        }
+        if (tid == 0) s.misc[kMiscM] = m_run;
+        named_bar_sync(kBarAll, kComputeThreads);
+        for (int j = tid; j < RV; j += kComputeThreads) {
+            float acc = 0.f;
+#pragma unroll 4
+            for (int g = 0; g < F::NTG; ++g) acc += s.red[g * RV + j];
+            s.ovec[j] = acc;
+        }
+        if (warp == 0) {
+            float acc = 0.f;
+            for (int i = lane; i < F::TT; i += 32) acc += s.lred[i];
+            acc = warp_sum(acc);
+            if (lane == 0) s.misc[kMiscL] = acc;
+        }
+        named_bar_sync(kBarAll, kComputeThreads);
+        finish_run<FastFinish<ES, RV, D>>(p, s, R, u, rg);
+        u = R.run_end;
+    }
+    empty_sequences(p, s);
+}
+
+template <typename Kern>
+lla_status launch_kernel(Kern kern, bool *configured, const Params &prm, int grid, int smem,
+                         cudaStream_t stream) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     if (dev < 64 && !configured[dev]) {
@@ -594,6 +1116,48 @@ lla_status launch_t(const Params &prm, int grid, int smem, cudaStream_t stream) 
     return LLA_OK;
 }
 
+template <int ES, int GK, int VB>
+lla_status launch_generic(const Params &prm, int grid, int smem, cudaStream_t stream) {
+    static bool configured[64] = {};
+    return launch_kernel(decode_kernel<ES, GK, VB>, configured, prm, grid, smem, stream);
+}
+
+template <int ES, int RK, int RV>
+lla_status launch_fast(const Params &prm, int grid, int smem, cudaStream_t stream) {
+    static bool configured[64] = {};
+    return launch_kernel(decode_fast_kernel<ES, RK, RV, 128>, configured, prm, grid, smem, stream);
+}
+
+// Pages per pipeline step: small head pages are grouped so one step moves about 32 KiB.
+int pages_per_step(int hpb) {
+    if (4 * hpb <= kStepTargetBytes) return 4;
+    if (2 * hpb <= kStepTargetBytes) return 2;
+    return 1;
+}
+
+// Shape-specialised kernel for (es, r_k, r_v): its launcher and CTAs per SM (launcher null when
+// the shape has none).
+using FastLauncher = lla_status (*)(const Params &, int, int, cudaStream_t);
+struct FastEntry {
+    FastLauncher launch;
+    int ctas;
+};
+FastEntry fast_entry(int es, int r_k, int r_v) {
+#define LLA_FAST(E, K, V) \
+    if (es == E && r_k == K && r_v == V) return FastEntry{launch_fast<E, K, V>, Fast<E, K, V>::CTAS};
+    LLA_FAST(2, 96, 160)
+    LLA_FAST(2, 192, 320)
+    LLA_FAST(2, 72, 120)
+    LLA_FAST(2, 18, 30)
+    LLA_FAST(2, 128, 128)
+    LLA_FAST(4, 96, 160)
+    LLA_FAST(4, 72, 120)
+    LLA_FAST(4, 18, 30)
+    LLA_FAST(4, 128, 128)
+#undef LLA_FAST
+    return FastEntry{nullptr, 1};
+}
+
 }  // namespace
 
 size_t decode_workspace_bytes(int r_v, int B, int H, int grid) {
@@ -604,9 +1168,7 @@ size_t decode_workspace_bytes(int r_v, int B, int H, int grid) {
 
 lla_status decode_fits(int r_k, int r_v, int es, int d) {
     const int hpb = static_cast<int>(head_page_bytes(r_k, r_v, es));
-    int pps = 1;
-    if (4 * hpb <= kStepTargetBytes) pps = 4;
-    else if (2 * hpb <= kStepTargetBytes) pps = 2;
+    const int pps = pages_per_step(hpb);
     const Layout base = make_layout(0, pps * hpb, LLA_MAX_BATCH, r_k, r_v, d);
     if ((kSmemLimit - base.total) / (pps * hpb) < 2) return LLA_ERR_UNSUPPORTED;
     if (r_v * es / granule_bytes(r_v, es) > kComputeThreads) return LLA_ERR_UNSUPPORTED;
@@ -616,17 +1178,19 @@ lla_status decode_fits(int r_k, int r_v, int es, int d) {
 lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream) {
     const int es = a.storage_bf16 ? 2 : 4;
     const int hpb = static_cast<int>(head_page_bytes(a.r_k, a.r_v, es));
-    int pps = 1;
-    if (4 * hpb <= kStepTargetBytes) pps = 4;
-    else if (2 * hpb <= kStepTargetBytes) pps = 2;
+    const int pps = pages_per_step(hpb);
     const int stage_bytes = pps * hpb;
+    const FastEntry fe = a.d == 128 ? fast_entry(es, a.r_k, a.r_v) : FastEntry{nullptr, 1};
+    const int ctas = fe.launch ? fe.ctas : 1;
+    const int budget = ctas == 2 ? kHalfSmem : kSmemLimit;
     const Layout base = make_layout(0, stage_bytes, a.B, a.r_k, a.r_v, a.d);
-    int stages = (kSmemLimit - base.total) / stage_bytes;
+    int stages = (budget - base.total) / stage_bytes;
     if (stages > kMaxStages) stages = kMaxStages;
     if (stages < 2) return LLA_ERR_UNSUPPORTED;
     const int smem = make_layout(stages, stage_bytes, a.B, a.r_k, a.r_v, a.d).total;
-    const int grid = num_sms();
-    if (grid <= 0) return LLA_ERR_CUDA;
+    const int sms = num_sms();
+    if (sms <= 0) return LLA_ERR_CUDA;
+    const int grid = ctas * sms;
     if (a.workspace_bytes < decode_workspace_bytes(a.r_v, a.B, a.H, grid)) return LLA_ERR_WORKSPACE;
     lla_status st = LLA_OK;
     unsigned *err = device_error_word(&st);
@@ -652,17 +1216,19 @@ lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream) {
     p.pps = pps; p.stages = stages; p.stage_bytes = stage_bytes;
     p.err = err;
 
+    if (fe.launch) return fe.launch(p, grid, smem, stream);
+
     const int gk = granule_bytes(a.r_k, es), vb = granule_bytes(a.r_v, es);
     if (es == 2) {
-        if (gk == 16 && vb == 16) return launch_t<2, 16, 16>(p, grid, smem, stream);
-        if (gk == 16 && vb == 4) return launch_t<2, 16, 4>(p, grid, smem, stream);
-        if (gk == 4 && vb == 16) return launch_t<2, 4, 16>(p, grid, smem, stream);
-        return launch_t<2, 4, 4>(p, grid, smem, stream);
+        if (gk == 16 && vb == 16) return launch_generic<2, 16, 16>(p, grid, smem, stream);
+        if (gk == 16 && vb == 4) return launch_generic<2, 16, 4>(p, grid, smem, stream);
+        if (gk == 4 && vb == 16) return launch_generic<2, 4, 16>(p, grid, smem, stream);
+        return launch_generic<2, 4, 4>(p, grid, smem, stream);
     }
-    if (gk == 16 && vb == 16) return launch_t<4, 16, 16>(p, grid, smem, stream);
-    if (gk == 16 && vb == 4) return launch_t<4, 16, 4>(p, grid, smem, stream);
-    if (gk == 4 && vb == 16) return launch_t<4, 4, 16>(p, grid, smem, stream);
-    return launch_t<4, 4, 4>(p, grid, smem, stream);
+    if (gk == 16 && vb == 16) return launch_generic<4, 16, 16>(p, grid, smem, stream);
+    if (gk == 16 && vb == 4) return launch_generic<4, 16, 4>(p, grid, smem, stream);
+    if (gk == 4 && vb == 16) return launch_generic<4, 4, 16>(p, grid, smem, stream);
+    return launch_generic<4, 4, 4>(p, grid, smem, stream);
 }
 
 }  // namespace lla
