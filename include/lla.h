@@ -90,8 +90,8 @@ typedef struct {
 typedef struct {
     const void *w_down_k; /* [H][T*d][r_k] storage dtype: W_down of the K axis */
     const void *w_down_v; /* [H][T*d][r_v] storage dtype */
-    const void *w_up_k;   /* [H][T][d][r_k] storage dtype: W_up,t of the K axis */
-    const void *w_up_v;   /* [H][T][d][r_v] storage dtype */
+    const void *w_up_k;   /* [H][T][d][r_k] storage dtype: W_up,t of the K axis (16-B aligned) */
+    const void *w_up_v;   /* [H][T][d][r_v] storage dtype (16-B aligned) */
     const float *mu_k;    /* [H][T*d] fp32 calibration mean, or NULL for mu = 0 */
     const float *mu_v;    /* [H][T*d] fp32, or NULL */
 } lla_codec;

@@ -134,7 +134,7 @@ lla_status lla_decode_workspace_size(const lla_geometry *g, int32_t B, size_t *b
     if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
     const int sms = num_sms();
     if (sms <= 0) return LLA_ERR_CUDA;
-    *bytes = decode_workspace_bytes(g->r_v, B, g->H, 2 * sms);  // up to two CTAs per SM
+    *bytes = decode_workspace_bytes(g->r_v, B, g->H, sms);  // one CTA per SM
     return LLA_OK;
 }
 
@@ -159,8 +159,7 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
     const int es = elem_size(g->storage);
     if (absorbed) {
         if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;
-        if (!aligned(codec->w_up_k, 2 * es) || !aligned(codec->w_up_v, 2 * es))
-            return LLA_ERR_INVALID_ARG;
+        if (!aligned(codec->w_up_k, 16) || !aligned(codec->w_up_v, 16)) return LLA_ERR_INVALID_ARG;
         if (loop < 0 || loop >= g->T) return LLA_ERR_INVALID_ARG;
     } else if (g->r_k != g->d || g->r_v != g->d) {
         return LLA_ERR_INVALID_ARG;

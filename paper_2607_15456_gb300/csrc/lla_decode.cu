@@ -41,7 +41,6 @@ constexpr int kComputeThreads = kComputeWarps * 32;
 constexpr int kThreads = kComputeThreads + 32;  // + one producer warp
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
-constexpr int kHalfSmem = 113 * 1024;  // per CTA when two CTAs share an SM
 constexpr int kStepTargetBytes = 32 * 1024;
 constexpr int kBarAll = 1;  // named barrier over the 256 consumer threads
 constexpr int kBarTok = 2;  // named barrier over the score threads
@@ -289,7 +288,8 @@ __device__ void producer(const Params &p, const Smem &s, const Range &rg) {
     const int lane = threadIdx.x & 31;
     const int hpb = p.head_page_bytes;
     const uint64_t pol = policy_evict_first();
-    int it = 0;
+    int it = 0, st = 0;
+    uint32_t sph = 0;
     for (int64_t u = rg.A0; u < rg.A1;) {
         const Run R = locate_run(p, s, u, rg.A1);
         const int32_t *bt = p.block_table + static_cast<int64_t>(R.b) * p.max_blocks + R.pg0;
@@ -297,13 +297,17 @@ __device__ void producer(const Params &p, const Smem &s, const Range &rg) {
             const int32_t blk_lane = (k0 + lane < R.npages) ? bt[k0 + lane] : -1;
             const int kend = min(R.npages, k0 + 32);
             for (int k = k0; k < kend; k += p.pps, ++it) {
+                const int stage = st;
+                const uint32_t ph = sph;
+                if (++st == p.stages) {
+                    st = 0;
+                    sph ^= 1u;
+                }
                 int32_t blk[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
                     blk[i] = __shfl_sync(0xffffffffu, blk_lane, (k - k0 + i) & 31);
                 if (lane == 0) {
-                    const int stage = it % p.stages;
-                    const uint32_t ph = (it / p.stages) & 1;
                     mbar_wait(&s.empty[stage], ph ^ 1u, s.abort_flag, p.err);
                     const int n = min(p.pps, R.npages - k);
                     uint32_t bytes = 0;
@@ -558,7 +562,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
     const int vu = tid % NVU, tg = tid / NVU;
     const bool vthread = tg < NTG;
 
-    int it = 0;
+    int stage = 0;
+    uint32_t ph = 0;
     for (int64_t u = rg.A0; u < rg.A1;) {
         const Run R = locate_run(p, s, u, rg.A1);
         setup_query<ES>(p, s, R.b, R.h);
@@ -569,9 +574,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
 #pragma unroll
         for (int k = 0; k < VE; ++k) accv[k] = 0.f;
 
-        for (int k = 0; k < R.npages; k += p.pps, ++it) {
-            const int stage = it % p.stages;
-            const uint32_t ph = (it / p.stages) & 1;
+        for (int k = 0; k < R.npages; k += p.pps) {
             mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
             const char *sb = s.ring + stage * p.stage_bytes;
             const int n = min(p.pps, R.npages - k);
@@ -632,6 +635,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&s.empty[stage]);
+            if (++stage == p.stages) {
+                stage = 0;
+                ph ^= 1u;
+            }
         }
 
         // reduce the run's softmax state across threads
@@ -683,224 +690,15 @@ struct Fast {
     static constexpr int VB = ((RV * ES) % 16 == 0) ? 16 : 4;  // V unit bytes
     static constexpr int VE = VB / ES;                         // elements per V unit
     static constexpr int VU = RV * ES / VB;                    // V units per row
-    static constexpr int NTG = V_THREADS / VU;                 // token groups of value threads
-    // Two CTAs share an SM when two pipeline stages each fit in half of its shared memory: one
-    // CTA's run set-up and merge then overlap the other's streaming.
-    static constexpr int CTAS = (2 * PPS * HPB + 24 * 1024 <= kHalfSmem) ? 2 : 1;
+    static constexpr int UPT = (VU % 2 == 0 && VU / 2 >= 8) ? 2 : 1;  // units per value thread
+    static constexpr int VC = VU / UPT;                        // value threads per token row
+    static constexpr int NTG = V_THREADS / VC;                 // token groups of value threads
+    static constexpr int ROWB = RV * ES;                       // V-plane row bytes
+    static constexpr int KPLANE = kBlockTokens * RK * ES;      // K-plane bytes
     static_assert(S_THREADS % 32 == 0 && S_WARPS >= 1 && V_WARPS >= 1, "role split");
     static_assert(NTG >= 1 && TT * TPT == TOK, "every token has a score thread");
     static_assert(KE % 4 == 0 || KE <= 2, "q~ vector loads");
     static_assert(TT % 32 == 0, "score-owning threads are whole warps");
-};
-
-// Bytes of the widest aligned load that splits `bytes` evenly (16, 8 or 4).
-__host__ __device__ constexpr int chunk_bytes(int bytes) {
-    return (bytes % 16 == 0) ? 16 : (bytes % 8 == 0) ? 8 : 4;
-}
-
-// Raw (packed) chunk of CB bytes, and its conversion to CB/ES floats.
-template <int CB> struct RawChunk;
-template <> struct RawChunk<16> { using T = uint4; };
-template <> struct RawChunk<8> { using T = uint2; };
-template <> struct RawChunk<4> { using T = uint32_t; };
-
-template <int CB>
-__device__ __forceinline__ typename RawChunk<CB>::T load_raw(const char *p) {
-    return *reinterpret_cast<const typename RawChunk<CB>::T *>(p);
-}
-
-template <int ES>
-__device__ __forceinline__ void unpack_word(uint32_t u, float *v) {
-    if constexpr (ES == 2) {
-        const float2 a = bf2_to_f2(u);
-        v[0] = a.x;
-        v[1] = a.y;
-    } else {
-        v[0] = __uint_as_float(u);
-    }
-}
-
-template <int ES>
-__device__ __forceinline__ void unpack(const uint4 &u, float *v) {
-    constexpr int W = 4 / ES;  // elements per 32-bit word
-    unpack_word<ES>(u.x, v); unpack_word<ES>(u.y, v + W); unpack_word<ES>(u.z, v + 2 * W);
-    unpack_word<ES>(u.w, v + 3 * W);
-}
-template <int ES>
-__device__ __forceinline__ void unpack(const uint2 &u, float *v) {
-    constexpr int W = 4 / ES;
-    unpack_word<ES>(u.x, v); unpack_word<ES>(u.y, v + W);
-}
-template <int ES>
-__device__ __forceinline__ void unpack(const uint32_t &u, float *v) { unpack_word<ES>(u, v); }
-
-constexpr int kMaxChunksInFlight = 10;  // per thread and round trip
-
-// Query set-up with compile-time shapes: every thread issues its W_up,t^K loads (at most
-// kMaxChunksInFlight per round trip) before using any.  q~[j] = sum_e W[e][j] q[e].
-template <int ES, int RK, int D>
-__device__ void fast_setup_query(const Params &p, const Smem &s, int b, int h) {
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int64_t qoff = (static_cast<int64_t>(b) * p.H + h) * D;
-    for (int e = tid; e < D; e += kComputeThreads) s.qfull[e] = load_elem(p.q, qoff + e, p.io_bf16);
-    if (!p.absorbed) {
-        named_bar_sync(kBarAll, kComputeThreads);
-        for (int e = tid; e < D; e += kComputeThreads) s.qlat[e] = s.qfull[e];
-        if (tid == 0) s.misc[kMiscBeta] = 0.f;
-        named_bar_sync(kBarAll, kComputeThreads);
-        return;
-    }
-    constexpr int CB = chunk_bytes(RK * ES);  // load width along a row of W
-    constexpr int CE = CB / ES;
-    constexpr int CPR = RK * ES / CB;          // chunks per row
-    constexpr int RG = kComputeThreads / CPR;  // row groups
-    constexpr int ROWS = (D + RG - 1) / RG;    // rows per thread
-    constexpr int BATCH = ROWS < kMaxChunksInFlight ? ROWS : kMaxChunksInFlight;
-    static_assert(RG * RK <= 8 * kComputeThreads, "partial sums fit the reduction buffer");
-    using Raw = typename RawChunk<CB>::T;
-    const int cg = tid % CPR, rg = tid / CPR;
-    const char *W = static_cast<const char *>(p.w_up_k) +
-                    ((static_cast<int64_t>(h) * p.T + p.loop) * D * RK + cg * CE) * ES;
-    Raw w[BATCH];
-    if (rg < RG) {
-#pragma unroll
-        for (int k = 0; k < BATCH; ++k) {
-            const int e = rg + k * RG;
-            if (e < D) w[k] = load_raw<CB>(W + static_cast<int64_t>(e) * RK * ES);
-        }
-    }
-    named_bar_sync(kBarAll, kComputeThreads);  // qfull ready
-    if (warp == kComputeWarps - 1) {
-        float bsum = 0.f;
-        if (p.mu_k) {
-            const float *mu = p.mu_k + (static_cast<int64_t>(h) * p.T + p.loop) * D;
-            for (int e = lane; e < D; e += 32) bsum = fmaf(s.qfull[e], mu[e], bsum);
-        }
-        bsum = warp_sum(bsum);
-        if (lane == 0) s.misc[kMiscBeta] = bsum;
-    }
-    if (rg < RG) {
-        float acc[CE];
-#pragma unroll
-        for (int i = 0; i < CE; ++i) acc[i] = 0.f;
-#pragma unroll
-        for (int k0 = 0; k0 < ROWS; k0 += BATCH) {
-            if (k0 > 0) {
-#pragma unroll
-                for (int k = 0; k < BATCH; ++k) {
-                    const int e = rg + (k0 + k) * RG;
-                    if (k0 + k < ROWS && e < D) w[k] = load_raw<CB>(W + static_cast<int64_t>(e) * RK * ES);
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < BATCH; ++k) {
-                const int e = rg + (k0 + k) * RG;
-                if (k0 + k < ROWS && e < D) {
-                    float v[CE];
-                    unpack<ES>(w[k], v);
-                    const float qe = s.qfull[e];
-#pragma unroll
-                    for (int i = 0; i < CE; ++i) acc[i] = fmaf(v[i], qe, acc[i]);
-                }
-            }
-        }
-#pragma unroll
-        for (int i = 0; i < CE; ++i) s.red[rg * RK + cg * CE + i] = acc[i];
-    }
-    named_bar_sync(kBarAll, kComputeThreads);
-    for (int j = tid; j < RK; j += kComputeThreads) {
-        float acc = 0.f;
-#pragma unroll 4
-        for (int g = 0; g < RG; ++g) acc += s.red[g * RK + j];
-        s.qlat[j] = acc;
-    }
-    named_bar_sync(kBarAll, kComputeThreads);
-}
-
-// Output with compile-time shapes: TPR threads per output row, each issuing its W_up,t^V
-// loads (at most kMaxChunksInFlight per round trip) before using any.
-// o = (W ovec wl + lc mu^V_t + p_cur v_cur) / (lc + p_cur).
-template <int ES, int RV, int D>
-struct FastFinish {
-    static constexpr int TPR = ((RV / 2) % 2 == 0 && D * 2 <= kComputeThreads) ? 2 : 1;
-    static constexpr int COLS = RV / TPR;      // columns per thread
-    static constexpr int CB = chunk_bytes(COLS * ES);
-    static constexpr int CE = CB / ES;
-    static constexpr int NCH = COLS / CE;      // chunks per thread
-    static constexpr int BATCH = NCH < kMaxChunksInFlight ? NCH : kMaxChunksInFlight;
-    static_assert(D * TPR <= kComputeThreads, "one pass over the rows");
-    using Raw = typename RawChunk<CB>::T;
-
-    __device__ static void run(const Params &p, const Smem &s, int b, int h, float m, float l) {
-        const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-        const bool pass1 = p.cur_k != nullptr;
-        const int64_t row = (static_cast<int64_t>(b) * p.H + h) * D;
-        if (!p.absorbed) {
-            finish_output<ES>(p, s, b, h, m, l);
-            return;
-        }
-        const int e = tid / TPR, half = tid % TPR;
-        const bool active = e < D;
-        const char *W = static_cast<const char *>(p.w_up_v) +
-                        ((static_cast<int64_t>(h) * p.T + p.loop) * D * RV +
-                         static_cast<int64_t>(e) * RV + half * COLS) * ES;
-        Raw w[BATCH];
-        if (active) {
-#pragma unroll
-            for (int k = 0; k < BATCH; ++k) w[k] = load_raw<CB>(W + k * CB);
-        }
-        float vcur = 0.f, muv = 0.f;
-        if (active && half == 0) {
-            if (pass1) vcur = load_elem(p.cur_v, row + e, p.io_bf16);
-            if (p.mu_v) muv = p.mu_v[(static_cast<int64_t>(h) * p.T + p.loop) * D + e];
-        }
-        if (pass1 && warp == 0) {
-            float acc = 0.f;
-            for (int i = lane; i < D; i += 32)
-                acc = fmaf(s.qfull[i], load_elem(p.cur_k, row + i, p.io_bf16), acc);
-            acc = warp_sum(acc);
-            if (lane == 0) s.misc[kMiscScur] = acc * p.scale_log2;
-        }
-        named_bar_sync(kBarAll, kComputeThreads);
-        float M = m, pc = 0.f;
-        if (pass1) {
-            const float sc = s.misc[kMiscScur];
-            M = fmaxf(m, sc);
-            pc = exp2f(sc - M);
-        }
-        const float wl = exp2f(m - M);
-        const float lc = l * wl;
-        const float inv = 1.f / (lc + pc);
-        float acc = 0.f;
-        if (active) {
-            const float *ov = s.ovec + half * COLS;
-#pragma unroll
-            for (int k0 = 0; k0 < NCH; k0 += BATCH) {
-                if (k0 > 0) {
-#pragma unroll
-                    for (int k = 0; k < BATCH; ++k)
-                        if (k0 + k < NCH) w[k] = load_raw<CB>(W + (k0 + k) * CB);
-                }
-#pragma unroll
-                for (int k = 0; k < BATCH; ++k) {
-                    if (k0 + k < NCH) {
-                        float v[CE];
-                        unpack<ES>(w[k], v);
-#pragma unroll
-                        for (int i = 0; i < CE; ++i) acc = fmaf(v[i], ov[(k0 + k) * CE + i], acc);
-                    }
-                }
-            }
-        }
-        if constexpr (TPR == 2) acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-        if (active && half == 0) {
-            float o = acc * wl;
-            if (p.mu_v) o = fmaf(lc, muv, o);
-            if (pass1) o = fmaf(pc, vcur, o);
-            store_elem(p.out, row + e, o * inv, p.io_bf16);
-        }
-        named_bar_sync(kBarAll, kComputeThreads);
-    }
 };
 
 // KE consecutive floats of q~ from shared memory (16-byte aligned at every granule start).
@@ -921,45 +719,520 @@ __device__ __forceinline__ void load_qvec(const float *q, float (&v)[KE]) {
     }
 }
 
+// ------------------------------------------------------------------------------------------
+// Shape-specialised kernel with asynchronous run boundaries.
+//
+// Warp roles (one CTA per SM):
+//   warps 0..S_WARPS-1     score warps: q~ . c_k for the step's tokens, online softmax
+//   warps S_WARPS..7       value warps: sum_i p_i c_v,i
+//   warp 8                 producer: TMA bulk copies of head pages into the ring
+//   warps 9..12            management warps: for run r+1 they load q and W_up,t^K and form
+//                          q~ while the other warps stream run r; for run r-1 they reduce the
+//                          left-behind softmax state, write or merge the split partials and
+//                          apply W_up,t^V.  Their global round trips never stall the stream.
+// Hand-offs are double-buffered by run parity: qready[slot] (management -> score warps, q~ of
+// a run is ready) and stfull[slot] (score + value warps -> management, the run's state is
+// written).  The management warps' order set-up(r), finish(r-1) guarantees that a slot is free
+// before it is written again.  W_up,t rows reach the management warps through a shared staging
+// buffer filled with cp.async, so no register holds them while they are in flight.
+// ------------------------------------------------------------------------------------------
+
+constexpr int kMWarps = 4;
+constexpr int kMThreads = kMWarps * 32;
+constexpr int kMBase = kComputeThreads + 32;       // first management thread
+constexpr int kAsyncThreads = kMBase + kMThreads;  // 416
+constexpr int kBarM = 3;                           // named barrier of the management warps
+constexpr int kBarStart = 4;                       // producer waits for the first set-up's loads
+constexpr int kWstMax = 40 * 1024;                 // staging buffer for W_up,t rows (upper bound)
+
+struct AsyncLayout {
+    int ring, full, empty, pfull, pempty, qready, stfull, prefix, lens, qlat, qfull, spart, psm,
+        lred, red, ovec, mred, mtmp, misc, wst, total;
+};
+
+// Shared-memory sizes of the asynchronous kernel for one rank shape (floats per slot).
 template <int ES, int RK, int RV, int D>
-__global__ void __launch_bounds__(kThreads, Fast<ES, RK, RV>::CTAS) decode_fast_kernel(const Params p) {
+struct AsyncSizes {
+    using F = Fast<ES, RK, RV>;
+    static constexpr int QSLOT = ((RK > D ? RK : D) + 3) & ~3;  // q~ or q, one run
+    static constexpr int REDSLOT = F::NTG * RV;                 // value partials, one run
+    static constexpr int MRED = (kMThreads / (RK / 2)) * RK;    // q~ partial sums
+    // staging buffer: the larger of W_up,t^K and W_up,t^V, at most kWstMax
+    static constexpr int WMAT = D * (RK > RV ? RK : RV) * ES;
+    static constexpr int WST = WMAT < kWstMax ? WMAT : kWstMax;
+};
+
+__host__ __device__ inline AsyncLayout make_async_layout(int stages, int stage_bytes, int B,
+                                                         int qslot, int redslot, int mred, int rv,
+                                                         int wst) {
+    AsyncLayout L;
+    int o = 0;
+    L.ring = o;   o += stages * stage_bytes;
+    L.full = o;   o += stages * 8;
+    L.empty = o;  o += stages * 8;
+    L.pfull = o;  o += 16;
+    L.pempty = o; o += 16;
+    L.qready = o; o += 16;
+    L.stfull = o; o += 16;
+    L.prefix = o; o += up16((B + 1) * 8);
+    L.lens = o;   o += up16(B * 4);
+    L.qlat = o;   o += up16(2 * qslot * 4);
+    L.qfull = o;  o += up16(2 * qslot * 4);
+    L.spart = o;  o += kComputeThreads * 4;
+    L.psm = o;    o += 2 * kComputeThreads * 4;
+    L.lred = o;   o += 2 * kComputeThreads * 4;
+    L.red = o;    o += up16(2 * redslot * 4);
+    L.ovec = o;   o += up16(rv * 4);
+    L.mred = o;   o += up16(mred * 4);
+    L.mtmp = o;   o += 2 * kMThreads * 4;
+    L.misc = o;   o += 64 * 4;
+    L.wst = o;    o += up16(wst);
+    L.total = o;
+    return L;
+}
+
+template <int ES, int RK, int RV, int D>
+__host__ __device__ inline AsyncLayout async_layout(int stages, int stage_bytes, int B) {
+    using Z = AsyncSizes<ES, RK, RV, D>;
+    return make_async_layout(stages, stage_bytes, B, Z::QSLOT, Z::REDSLOT, Z::MRED, RV, Z::WST);
+}
+
+// misc slots of the asynchronous kernel
+constexpr int kAM = 0 /* [2] run maximum by slot */, kABeta = 2 /* [2] */, kAScur = 4,
+              kAPAlpha = 5 /* [2] */, kAWmax = 16 /* [2][8] */, kAAbort = 32, kALast = 33;
+
+struct ASmem {
+    Smem s;  // fields shared with the generic helpers (ring, barriers, prefix, lens, abort flag)
+    uint64_t *qready, *stfull;
+    float *qlat, *qfull, *lred, *red, *mred, *mtmp;
+    char *wst;
+    int qslot, redslot;  // floats per slot
+};
+
+template <int ES, int RK, int RV, int D>
+__device__ __forceinline__ ASmem carve_async(char *smem, const Params &p) {
+    const AsyncLayout L = async_layout<ES, RK, RV, D>(p.stages, p.stage_bytes, p.B);
+    ASmem a;
+    a.s.ring = smem + L.ring;
+    a.s.full = reinterpret_cast<uint64_t *>(smem + L.full);
+    a.s.empty = reinterpret_cast<uint64_t *>(smem + L.empty);
+    a.s.pfull = reinterpret_cast<uint64_t *>(smem + L.pfull);
+    a.s.pempty = reinterpret_cast<uint64_t *>(smem + L.pempty);
+    a.s.prefix = reinterpret_cast<int64_t *>(smem + L.prefix);
+    a.s.lens = reinterpret_cast<int *>(smem + L.lens);
+    a.s.qlat = nullptr;
+    a.s.qfull = nullptr;
+    a.s.spart = reinterpret_cast<float *>(smem + L.spart);
+    a.s.psm = reinterpret_cast<float *>(smem + L.psm);
+    a.s.tmp = nullptr;
+    a.s.red = nullptr;
+    a.s.lred = nullptr;
+    a.s.ovec = reinterpret_cast<float *>(smem + L.ovec);
+    a.s.misc = reinterpret_cast<float *>(smem + L.misc);
+    a.s.abort_flag = reinterpret_cast<volatile int *>(a.s.misc + kAAbort);
+    a.s.last_flag = reinterpret_cast<int *>(a.s.misc + kALast);
+    a.qready = reinterpret_cast<uint64_t *>(smem + L.qready);
+    a.stfull = reinterpret_cast<uint64_t *>(smem + L.stfull);
+    a.qlat = reinterpret_cast<float *>(smem + L.qlat);
+    a.qfull = reinterpret_cast<float *>(smem + L.qfull);
+    a.lred = reinterpret_cast<float *>(smem + L.lred);
+    a.red = reinterpret_cast<float *>(smem + L.red);
+    a.mred = reinterpret_cast<float *>(smem + L.mred);
+    a.mtmp = reinterpret_cast<float *>(smem + L.mtmp);
+    a.wst = smem + L.wst;
+    a.qslot = AsyncSizes<ES, RK, RV, D>::QSLOT;
+    a.redslot = AsyncSizes<ES, RK, RV, D>::REDSLOT;
+    return a;
+}
+
+__device__ __forceinline__ void m_sync() { named_bar_sync(kBarM, kMThreads); }
+
+// Passes through the staging buffer for a D x R matrix of W_up,t: the smallest power of two
+// that makes one pass fit.
+template <int ES, int R, int D, int WST>
+struct WPasses {
+    static constexpr int BYTES = D * R * ES;
+    static constexpr int N = BYTES <= WST ? 1 : BYTES <= 2 * WST ? 2 : BYTES <= 4 * WST ? 4 : 8;
+    static constexpr int ROWS = D / N;                // rows per pass
+    static constexpr int PASS_BYTES = ROWS * R * ES;  // multiple of 16 since D = 128
+    static_assert(D % N == 0 && PASS_BYTES <= WST && PASS_BYTES % 16 == 0, "staging passes");
+};
+
+// Starts the copy of rows [pass*ROWS, (pass+1)*ROWS) of W into the staging buffer.
+template <int ES, int R, int D, int WST>
+__device__ __forceinline__ void m_stage_rows(const ASmem &a, const char *W, int pass, int mt) {
+    using P = WPasses<ES, R, D, WST>;
+    const char *src = W + static_cast<int64_t>(pass) * P::PASS_BYTES;
+    for (int i = mt; i < P::PASS_BYTES / 16; i += kMThreads) cp_async16(a.wst + i * 16, src + i * 16);
+    cp_async_commit();
+}
+
+// Management: q, q~ = W_up,t^K^T q and beta = q . mu^K_t of a run into slot `slot`.
+template <int ES, int RK, int RV, int D>
+__device__ void m_setup(const Params &p, const ASmem &a, int b, int h, int slot, int mt,
+                        bool release_producer) {
+    static_assert(D <= kMThreads, "one management thread per element of q");
+    constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
+    float *qfull = a.qfull + slot * a.qslot;
+    float *qlat = a.qlat + slot * a.qslot;
+    const int mwarp = mt >> 5, lane = mt & 31;
+    const int64_t qoff = (static_cast<int64_t>(b) * p.H + h) * D;
+    cp_async_wait_all();  // nothing of an earlier use of the staging buffer is still in flight
+    m_sync();
+    const float qv = mt < D ? load_elem(p.q, qoff + mt, p.io_bf16) : 0.f;
+    if (!p.absorbed) {
+        if (release_producer) named_bar_arrive(kBarStart, kMThreads + 32);
+        if (mt < D) {
+            qfull[mt] = qv;
+            qlat[mt] = qv;
+        }
+        if (mt == 0) a.s.misc[kABeta + slot] = 0.f;
+        return;
+    }
+    using P = WPasses<ES, RK, D, WST>;
+    constexpr int CPR = RK / 2;          // pairs per row of W
+    constexpr int RG = kMThreads / CPR;  // row groups
+    static_assert(RG >= 1 && RG * RK <= 2048, "partial sums fit the management buffer");
+    const char *W = static_cast<const char *>(p.w_up_k) +
+                    (static_cast<int64_t>(h) * p.T + p.loop) * D * RK * ES;
+    m_stage_rows<ES, RK, D, WST>(a, W, 0, mt);
+    // the first set-up's loads go out before the producer fills the ring, not queued behind it
+    if (release_producer) named_bar_arrive(kBarStart, kMThreads + 32);
+    if (mt < D) qfull[mt] = qv;
+    const int cg = mt % CPR, rg = mt / CPR;
+    float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll 1
+    for (int pass = 0; pass < P::N; ++pass) {
+        cp_async_wait_all();
+        m_sync();  // the pass (and qfull) is in shared memory for every thread
+        if (rg < RG) {
+            for (int el = rg; el < P::ROWS; el += RG) {
+                const float2 w = load_pair<ES>(a.wst, static_cast<int64_t>(el) * RK + cg * 2);
+                const float qe = qfull[pass * P::ROWS + el];
+                acc0 = fmaf(w.x, qe, acc0);
+                acc1 = fmaf(w.y, qe, acc1);
+            }
+        }
+        if (pass + 1 < P::N) {
+            m_sync();  // the buffer is read before the next pass overwrites it
+            m_stage_rows<ES, RK, D, WST>(a, W, pass + 1, mt);
+        }
+    }
+    if (rg < RG) {
+        a.mred[rg * RK + cg * 2] = acc0;
+        a.mred[rg * RK + cg * 2 + 1] = acc1;
+    }
+    if (mwarp == kMWarps - 1) {
+        float bsum = 0.f;
+        if (p.mu_k) {
+            const float *mu = p.mu_k + (static_cast<int64_t>(h) * p.T + p.loop) * D;
+            for (int e = lane; e < D; e += 32) bsum = fmaf(qfull[e], mu[e], bsum);
+        }
+        bsum = warp_sum(bsum);
+        if (lane == 0) a.s.misc[kABeta + slot] = bsum;
+    }
+    m_sync();
+    for (int j = mt; j < RK; j += kMThreads) {
+        float acc = 0.f;
+#pragma unroll 4
+        for (int g = 0; g < RG; ++g) acc += a.mred[g * RK + j];
+        qlat[j] = acc;
+    }
+}
+
+// Management: output of one (sequence, head) from its softmax state (m, l, a.s.ovec).
+// o = (W_up,t^V ovec wl + lc mu^V_t + p_cur v_cur) / (lc + p_cur).  W_up,t^V comes through the
+// staging buffer (its first pass already in flight when `staged`); a warp takes one row at a
+// time, lanes along the row, so the shared-memory reads are conflict-free.
+template <int ES, int RK, int RV, int D>
+__device__ void m_output(const Params &p, const ASmem &a, int b, int h, float m, float l, int slot,
+                         int mt, bool staged) {
+    static_assert(D <= kMThreads, "one management thread per output element");
+    constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
+    using P = WPasses<ES, RV, D, WST>;
+    constexpr int NP = RV / 2;  // pairs per row
+    const float *qfull = a.qfull + slot * a.qslot;
+    const int mwarp = mt >> 5, lane = mt & 31;
+    const bool pass1 = p.cur_k != nullptr;
+    const int64_t orow = (static_cast<int64_t>(b) * p.H + h) * D;
+    const char *W = static_cast<const char *>(p.w_up_v) +
+                    (static_cast<int64_t>(h) * p.T + p.loop) * D * RV * ES;
+    if (p.absorbed && !staged) m_stage_rows<ES, RV, D, WST>(a, W, 0, mt);
+    // per-row extras of this output, one element per thread
+    float *vcur = a.mtmp, *muv = a.mtmp + kMThreads;
+    if (mt < D) {
+        vcur[mt] = pass1 ? load_elem(p.cur_v, orow + mt, p.io_bf16) : 0.f;
+        muv[mt] = (p.absorbed && p.mu_v) ? p.mu_v[(static_cast<int64_t>(h) * p.T + p.loop) * D + mt] : 0.f;
+    }
+    if (pass1 && mwarp == 0) {
+        float acc = 0.f;
+        for (int i = lane; i < D; i += 32) acc = fmaf(qfull[i], load_elem(p.cur_k, orow + i, p.io_bf16), acc);
+        acc = warp_sum(acc);
+        if (lane == 0) a.s.misc[kAScur] = acc * p.scale_log2;
+    }
+    m_sync();
+    float M = m, pc = 0.f;
+    if (pass1) {
+        const float sc = a.s.misc[kAScur];
+        M = fmaxf(m, sc);
+        pc = exp2f(sc - M);
+    }
+    const float wl = exp2f(m - M);
+    const float lc = l * wl;
+    const float inv = 1.f / (lc + pc);
+    if (!p.absorbed) {
+        for (int e = mt; e < D; e += kMThreads) {
+            const float o = fmaf(pc, vcur[e], a.s.ovec[e] * wl);
+            store_elem(p.out, orow + e, o * inv, p.io_bf16);
+        }
+        m_sync();
+        return;
+    }
+#pragma unroll 1
+    for (int pass = 0; pass < P::N; ++pass) {
+        cp_async_wait_all();
+        m_sync();
+#pragma unroll 2
+        for (int er = mwarp; er < P::ROWS; er += kMWarps) {
+            float acc = 0.f;
+            for (int jp = lane; jp < NP; jp += 32) {
+                const float2 w = load_pair<ES>(a.wst, static_cast<int64_t>(er) * RV + 2 * jp);
+                const float2 o2 = *reinterpret_cast<const float2 *>(a.s.ovec + 2 * jp);
+                acc = fmaf(w.x, o2.x, acc);
+                acc = fmaf(w.y, o2.y, acc);
+            }
+            acc = warp_sum(acc);
+            if (lane == 0) {
+                const int e = pass * P::ROWS + er;
+                float o = fmaf(lc, muv[e], acc * wl);
+                o = fmaf(pc, vcur[e], o);
+                store_elem(p.out, orow + e, o * inv, p.io_bf16);
+            }
+        }
+        m_sync();  // the buffer is read before the next pass (or set-up) overwrites it
+        if (pass + 1 < P::N) m_stage_rows<ES, RV, D, WST>(a, W, pass + 1, mt);
+    }
+}
+
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int *addr, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(addr), "r"(v) : "memory");
+    return old;
+}
+
+// Management: the run that left its state in slot `slot` -- reduce it, then finish the
+// (sequence, head) in place, or write a partial and merge all of them if this CTA is the last
+// to arrive.  One acquire-release atomic both publishes this CTA's partial and tells the last
+// CTA that every other partial is visible.
+template <int ES, int RK, int RV, int D, int TT, int NTG>
+__device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t u, const Range &rg,
+                         int slot, uint32_t parity, int mt) {
+    constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
+    mbar_wait(&a.stfull[slot], parity, a.s.abort_flag, p.err);
+    if (p.absorbed) {
+        // the output's first pass of W_up,t^V travels while the partial protocol runs
+        cp_async_wait_all();
+        m_sync();
+        m_stage_rows<ES, RV, D, WST>(a, static_cast<const char *>(p.w_up_v) +
+                                            (static_cast<int64_t>(R.h) * p.T + p.loop) * D * RV * ES,
+                                     0, mt);
+    }
+    const float *red = a.red + slot * a.redslot;
+    const float *lred = a.lred + slot * kComputeThreads;
+    for (int j = mt; j < RV; j += kMThreads) {  // fixed order: bitwise-reproducible sums
+        float acc = 0.f;
+#pragma unroll 4
+        for (int g = 0; g < NTG; ++g) acc += red[g * RV + j];
+        a.s.ovec[j] = acc;
+    }
+    float l = 0.f;
+    for (int i = 0; i < TT; ++i) l += lred[i];
+    const float m = a.s.misc[kAM + slot];
+    m_sync();
+    if (u == R.seg_start && R.run_end == R.seg_end) {
+        m_output<ES, RK, RV, D>(p, a, R.b, R.h, m, l, slot, mt, true);
+        return;
+    }
+    const int c = blockIdx.x;
+    const int pslot = (R.seg_start <= rg.A0) ? 0 : 1;
+    float *rec = p.partials + (static_cast<int64_t>(c) * 2 + pslot) * (RV + 2);
+    if (mt == 0) {
+        rec[0] = m;
+        rec[1] = l;
+    }
+    for (int j = mt; j < RV; j += kMThreads) rec[2 + j] = a.s.ovec[j];
+    m_sync();
+    const int c_first = owner_of(R.seg_start, rg.U, rg.Geff);
+    const int c_last = owner_of(R.seg_end - 1, rg.U, rg.Geff);
+    int *counter = &p.counters[R.b * p.H + R.h];
+    if (mt == 0) {
+        const int prev = atom_add_acq_rel_gpu(counter, 1);
+        *a.s.last_flag = (prev == c_last - c_first);
+    }
+    m_sync();
+    if (!*a.s.last_flag) return;
+    auto record = [&](int cc) {
+        const int sl = (R.seg_start <= range_start(cc, rg.U, rg.Geff)) ? 0 : 1;
+        return p.partials + (static_cast<int64_t>(cc) * 2 + sl) * (RV + 2);
+    };
+    const int nparts = c_last - c_first + 1;
+    constexpr int kQuick = 8;  // parts merged with every load issued in one round trip
+    float M = -INFINITY, lsum = 0.f;
+    if (nparts <= kQuick) {
+        constexpr int JPT = (RV + kMThreads - 1) / kMThreads;  // columns per thread
+        float pm[kQuick], pl[kQuick], po[kQuick][JPT];
+#pragma unroll
+        for (int k = 0; k < kQuick; ++k) {
+            if (k < nparts) {
+                const float *r = record(c_first + k);
+                pm[k] = __ldcg(r);
+                pl[k] = __ldcg(r + 1);
+#pragma unroll
+                for (int q = 0; q < JPT; ++q) {
+                    const int j = mt + q * kMThreads;
+                    po[k][q] = j < RV ? __ldcg(r + 2 + j) : 0.f;
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kQuick; ++k)
+            if (k < nparts) M = fmaxf(M, pm[k]);
+        float acc[JPT];
+#pragma unroll
+        for (int q = 0; q < JPT; ++q) acc[q] = 0.f;
+#pragma unroll
+        for (int k = 0; k < kQuick; ++k) {
+            if (k < nparts) {
+                const float w = exp2f(pm[k] - M);
+                lsum = fmaf(pl[k], w, lsum);
+#pragma unroll
+                for (int q = 0; q < JPT; ++q) acc[q] = fmaf(po[k][q], w, acc[q]);
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < JPT; ++q) {
+            const int j = mt + q * kMThreads;
+            if (j < RV) a.s.ovec[j] = acc[q];
+        }
+    } else {
+        for (int c0 = 0; c0 < nparts; c0 += kMThreads) {
+            const int np = min(kMThreads, nparts - c0);
+            if (mt < np) {
+                const float *r = record(c_first + c0 + mt);
+                a.mtmp[mt] = __ldcg(r);
+                a.mtmp[kMThreads + mt] = __ldcg(r + 1);
+            }
+            m_sync();
+            float Mc = M;
+            for (int i = 0; i < np; ++i) Mc = fmaxf(Mc, a.mtmp[i]);
+            lsum *= exp2f(M - Mc);
+            for (int i = 0; i < np; ++i) lsum = fmaf(a.mtmp[kMThreads + i], exp2f(a.mtmp[i] - Mc), lsum);
+            M = Mc;
+            m_sync();
+        }
+        for (int j = mt; j < RV; j += kMThreads) {
+            float acc = 0.f;
+#pragma unroll 4
+            for (int cc = c_first; cc <= c_last; ++cc) {
+                const float *r = record(cc);
+                acc = fmaf(__ldcg(r + 2 + j), exp2f(__ldcg(r) - M), acc);
+            }
+            a.s.ovec[j] = acc;
+        }
+    }
+    m_sync();
+    m_output<ES, RK, RV, D>(p, a, R.b, R.h, M, lsum, slot, mt, true);
+    if (mt == 0) atomicExch(counter, 0);
+}
+
+template <int ES, int RK, int RV, int D>
+__global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Params p) {
     using F = Fast<ES, RK, RV>;
     extern __shared__ __align__(128) char smem[];
-    const Smem s = carve(smem, p);
+    const ASmem a = carve_async<ES, RK, RV, D>(smem, p);
+    const Smem &s = a.s;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
     pdl_wait();  // inputs may come from the previous kernel in the stream
-    const Range rg = prologue(p, s, F::S_THREADS, F::V_THREADS);
+    if (tid == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&a.qready[i], kMThreads);
+            mbar_init(&a.stfull[i], kComputeThreads);
+        }
+    }
+    const Range rg = prologue(p, s, F::S_THREADS, F::V_THREADS);  // fences the inits above too
     pdl_trigger();
 
     if (warp == kComputeWarps) {
+        if (rg.A0 < rg.A1) named_bar_sync(kBarStart, kMThreads + 32);
         producer(p, s, rg);
         return;
     }
 
+    if (tid >= kMBase) {
+        // ---------------------------------------------------------------- management warps
+        const int mt = tid - kMBase;
+        int r = 0;
+        Run prev{};
+        int64_t prev_u = 0;
+        for (int64_t u = rg.A0; u < rg.A1;) {
+            const Run R = locate_run(p, s, u, rg.A1);
+            const int slot = r & 1;
+            m_setup<ES, RK, RV, D>(p, a, R.b, R.h, slot, mt, r == 0);
+            mbar_arrive(&a.qready[slot]);
+            if (r > 0)
+                m_finish<ES, RK, RV, D, F::TT, F::NTG>(p, a, prev, prev_u, rg, (r - 1) & 1,
+                                                       ((r - 1) >> 1) & 1, mt);
+            prev = R;
+            prev_u = u;
+            ++r;
+            u = R.run_end;
+        }
+        if (r > 0)
+            m_finish<ES, RK, RV, D, F::TT, F::NTG>(p, a, prev, prev_u, rg, (r - 1) & 1,
+                                                   ((r - 1) >> 1) & 1, mt);
+        // sequences with no cached token: pass 1 attends to the current token only
+        const bool pass1 = p.cur_k != nullptr;
+        for (int b = 0; b < p.B; ++b) {
+            if (s.lens[b] != 0) continue;
+            for (int h = 0; h < p.H; ++h) {
+                if ((b * p.H + h) % gridDim.x != blockIdx.x) continue;
+                const int64_t row = (static_cast<int64_t>(b) * p.H + h) * D;
+                if (!pass1 && mt == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
+                for (int e = mt; e < D; e += kMThreads)
+                    store_elem(p.out, row + e, pass1 ? load_elem(p.cur_v, row + e, p.io_bf16) : 0.f,
+                               p.io_bf16);
+            }
+        }
+        cp_async_wait_all();  // no copy into shared memory outlives the CTA
+        return;
+    }
+
+    // ------------------------------------------------------------------ score and value warps
     const bool is_s = warp < F::S_WARPS;
-    // score threads: k-split ks, token thread tt (tokens tt + i*TT)
-    const int ks = tid / F::TT, tt = tid % F::TT;
-    // value threads: column unit vu, token group tg (tokens tg + i*NTG)
-    const int vt = tid - F::S_THREADS;
-    const int vu = vt % F::VU, tg = vt / F::VU;
+    const int ks = tid / F::TT, tt = tid % F::TT;  // score threads
+    const int vt = tid - F::S_THREADS;              // value threads
+    const int vc = vt % F::VC, tg = vt / F::VC;
     const bool vwork = !is_s && tg < F::NTG;
+    constexpr int AV = F::UPT * F::VE;
 
-    int it = 0;
-    for (int64_t u = rg.A0; u < rg.A1;) {
+    int it = 0, stage = 0, r = 0;
+    uint32_t ph = 0;
+    for (int64_t u = rg.A0; u < rg.A1; ++r) {
         const Run R = locate_run(p, s, u, rg.A1);
-        fast_setup_query<ES, RK, D>(p, s, R.b, R.h);
-        const float beta = s.misc[kMiscBeta];
-
+        const int rslot = r & 1;
+        float beta = 0.f;
+        const float *qq = a.qlat + rslot * a.qslot + ks * F::NGT * F::KE;
+        if (is_s) {
+            mbar_wait(&a.qready[rslot], (r >> 1) & 1, s.abort_flag, p.err);
+            beta = s.misc[kABeta + rslot];
+        }
         float m_run = -INFINITY, l_part = 0.f;
-        float accv[F::VE];
+        float accv[AV];
 #pragma unroll
-        for (int e = 0; e < F::VE; ++e) accv[e] = 0.f;
-        const float *qq = s.qlat + ks * F::NGT * F::KE;  // this k-split's part of q~
+        for (int e = 0; e < AV; ++e) accv[e] = 0.f;
 
         for (int k = 0; k < R.npages; k += F::PPS, ++it) {
-            const int stage = it % p.stages;
-            const uint32_t ph = (it / p.stages) & 1;
             const int slot = it & 1;
             const uint32_t pph = (it >> 1) & 1;
             const char *sb = s.ring + stage * p.stage_bytes;
@@ -978,7 +1251,7 @@ __global__ void __launch_bounds__(kThreads, Fast<ES, RK, RV>::CTAS) decode_fast_
                     if (tok < nvalid) {
                         const char *kp = sb + (tok >> 6) * F::HPB + (tok & 63) * F::GK +
                                          ks * F::NGT * (kBlockTokens * F::GK);
-#pragma unroll 4
+#pragma unroll
                         for (int g = 0; g < F::NGT; ++g) {
                             if (F::NGK % F::KSPLIT != 0 && ks * F::NGT + g >= F::NGK) break;
                             float v[F::KE], qv[F::KE];
@@ -1016,7 +1289,7 @@ __global__ void __launch_bounds__(kThreads, Fast<ES, RK, RV>::CTAS) decode_fast_
                     x[i] = valid ? (sc[i] + beta) * p.scale_log2 : -INFINITY;
                     lm = fmaxf(lm, x[i]);
                 }
-                float *wmax = s.misc + kMiscWmax + (it & 1) * 8;
+                float *wmax = s.misc + kAWmax + slot * 8;
                 if (ks == 0) {
                     lm = warp_max(lm);
                     if (lane == 0) wmax[warp] = lm;
@@ -1038,62 +1311,65 @@ __global__ void __launch_bounds__(kThreads, Fast<ES, RK, RV>::CTAS) decode_fast_
                         lsum += pv;
                     }
                     l_part = fmaf(l_part, alpha, lsum);
-                    if (tid == 0) s.misc[kMiscPAlpha + slot] = alpha;
+                    if (tid == 0) s.misc[kAPAlpha + slot] = alpha;
                 }
                 mbar_arrive(&s.pfull[slot]);
             } else {
                 mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
                 mbar_wait(&s.pfull[slot], pph, s.abort_flag, p.err);
                 if (vwork) {
-                    const float alpha = s.misc[kMiscPAlpha + slot];
+                    const float alpha = s.misc[kAPAlpha + slot];
 #pragma unroll
-                    for (int e = 0; e < F::VE; ++e) accv[e] *= alpha;
-                    const char *vp = sb + kBlockTokens * RK * ES + vu * F::VB;
+                    for (int e = 0; e < AV; ++e) accv[e] *= alpha;
+                    const char *vbase = sb + F::KPLANE + vc * (F::UPT * F::VB) + tg * F::ROWB;
+#pragma unroll
+                    for (int pi = 0; pi < F::PPS; ++pi) {
+                        // rows tg, tg + NTG, ... of page pi that hold valid tokens
+                        const int rows = min(kBlockTokens, nvalid - pi * kBlockTokens);
+                        const int cnt = rows > tg ? (rows - tg + F::NTG - 1) / F::NTG : 0;
+                        const char *vp = vbase + pi * F::HPB;
+                        const float *pp = pring + pi * kBlockTokens + tg;
 #pragma unroll 4
-                    for (int tk = tg; tk < nvalid; tk += F::NTG) {
-                        const float pv = pring[tk];
-                        float v[F::VE];
-                        load_gran<ES, F::VB>(vp + (tk >> 6) * F::HPB + (tk & 63) * (RV * ES), v);
+                        for (int i = 0; i < cnt; ++i) {
+                            const float pv = pp[i * F::NTG];
+                            const char *rowp = vp + i * (F::NTG * F::ROWB);
 #pragma unroll
-                        for (int e = 0; e < F::VE; ++e) accv[e] = fmaf(pv, v[e], accv[e]);
+                            for (int uu = 0; uu < F::UPT; ++uu) {
+                                float v[F::VE];
+                                load_gran<ES, F::VB>(rowp + uu * F::VB, v);
+#pragma unroll
+                                for (int e = 0; e < F::VE; ++e)
+                                    accv[uu * F::VE + e] = fmaf(pv, v[e], accv[uu * F::VE + e]);
+                            }
+                        }
                     }
                 }
                 mbar_arrive(&s.pempty[slot]);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&s.empty[stage]);  // V-plane read
             }
+            if (++stage == p.stages) {
+                stage = 0;
+                ph ^= 1u;
+            }
         }
 
-        // reduce the run's softmax state across threads
-        if (is_s && ks == 0) s.lred[tt] = l_part;
+        // leave the run's softmax state in slot rslot for the management warps
+        if (is_s && ks == 0) a.lred[rslot * kComputeThreads + tt] = l_part;
+        if (tid == 0) s.misc[kAM + rslot] = m_run;
         if (vwork) {
 #pragma unroll
-            for (int e = 0; e < F::VE; ++e) s.red[tg * RV + vu * F::VE + e] = accv[e];
+            for (int e = 0; e < AV; ++e) a.red[rslot * a.redslot + tg * RV + vc * AV + e] = accv[e];
         }
-        if (tid == 0) s.misc[kMiscM] = m_run;
-        named_bar_sync(kBarAll, kComputeThreads);
-        for (int j = tid; j < RV; j += kComputeThreads) {
-            float acc = 0.f;
-#pragma unroll 4
-            for (int g = 0; g < F::NTG; ++g) acc += s.red[g * RV + j];
-            s.ovec[j] = acc;
-        }
-        if (warp == 0) {
-            float acc = 0.f;
-            for (int i = lane; i < F::TT; i += 32) acc += s.lred[i];
-            acc = warp_sum(acc);
-            if (lane == 0) s.misc[kMiscL] = acc;
-        }
-        named_bar_sync(kBarAll, kComputeThreads);
-        finish_run<FastFinish<ES, RV, D>>(p, s, R, u, rg);
+        mbar_arrive(&a.stfull[rslot]);
         u = R.run_end;
     }
-    empty_sequences(p, s);
 }
+
 
 template <typename Kern>
 lla_status launch_kernel(Kern kern, bool *configured, const Params &prm, int grid, int smem,
-                         cudaStream_t stream) {
+                         cudaStream_t stream, int threads = kThreads) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     if (dev < 64 && !configured[dev]) {
@@ -1104,7 +1380,7 @@ lla_status launch_kernel(Kern kern, bool *configured, const Params &prm, int gri
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(kThreads);
+    cfg.blockDim = dim3(threads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -1125,7 +1401,13 @@ lla_status launch_generic(const Params &prm, int grid, int smem, cudaStream_t st
 template <int ES, int RK, int RV>
 lla_status launch_fast(const Params &prm, int grid, int smem, cudaStream_t stream) {
     static bool configured[64] = {};
-    return launch_kernel(decode_fast_kernel<ES, RK, RV, 128>, configured, prm, grid, smem, stream);
+    return launch_kernel(decode_async_kernel<ES, RK, RV, 128>, configured, prm, grid, smem, stream,
+                         kAsyncThreads);
+}
+
+template <int ES, int RK, int RV>
+int fast_layout_bytes(int stages, int stage_bytes, int B) {
+    return async_layout<ES, RK, RV, 128>(stages, stage_bytes, B).total;
 }
 
 // Pages per pipeline step: small head pages are grouped so one step moves about 32 KiB.
@@ -1135,16 +1417,17 @@ int pages_per_step(int hpb) {
     return 1;
 }
 
-// Shape-specialised kernel for (es, r_k, r_v): its launcher and CTAs per SM (launcher null when
-// the shape has none).
+// Shape-specialised kernel for (es, r_k, r_v): its launcher and shared-memory layout size
+// (both null when the shape has none).
 using FastLauncher = lla_status (*)(const Params &, int, int, cudaStream_t);
+using FastLayout = int (*)(int, int, int);
 struct FastEntry {
     FastLauncher launch;
-    int ctas;
+    FastLayout layout;
 };
 FastEntry fast_entry(int es, int r_k, int r_v) {
 #define LLA_FAST(E, K, V) \
-    if (es == E && r_k == K && r_v == V) return FastEntry{launch_fast<E, K, V>, Fast<E, K, V>::CTAS};
+    if (es == E && r_k == K && r_v == V) return FastEntry{launch_fast<E, K, V>, fast_layout_bytes<E, K, V>};
     LLA_FAST(2, 96, 160)
     LLA_FAST(2, 192, 320)
     LLA_FAST(2, 72, 120)
@@ -1155,7 +1438,7 @@ FastEntry fast_entry(int es, int r_k, int r_v) {
     LLA_FAST(4, 18, 30)
     LLA_FAST(4, 128, 128)
 #undef LLA_FAST
-    return FastEntry{nullptr, 1};
+    return FastEntry{nullptr, nullptr};
 }
 
 }  // namespace
@@ -1169,8 +1452,10 @@ size_t decode_workspace_bytes(int r_v, int B, int H, int grid) {
 lla_status decode_fits(int r_k, int r_v, int es, int d) {
     const int hpb = static_cast<int>(head_page_bytes(r_k, r_v, es));
     const int pps = pages_per_step(hpb);
-    const Layout base = make_layout(0, pps * hpb, LLA_MAX_BATCH, r_k, r_v, d);
-    if ((kSmemLimit - base.total) / (pps * hpb) < 2) return LLA_ERR_UNSUPPORTED;
+    int fixed = make_layout(0, pps * hpb, LLA_MAX_BATCH, r_k, r_v, d).total;
+    const FastEntry fe = d == 128 ? fast_entry(es, r_k, r_v) : FastEntry{nullptr, nullptr};
+    if (fe.layout) fixed = fe.layout(0, pps * hpb, LLA_MAX_BATCH);
+    if ((kSmemLimit - fixed) / (pps * hpb) < 2) return LLA_ERR_UNSUPPORTED;
     if (r_v * es / granule_bytes(r_v, es) > kComputeThreads) return LLA_ERR_UNSUPPORTED;
     return LLA_OK;
 }
@@ -1180,17 +1465,16 @@ lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream) {
     const int hpb = static_cast<int>(head_page_bytes(a.r_k, a.r_v, es));
     const int pps = pages_per_step(hpb);
     const int stage_bytes = pps * hpb;
-    const FastEntry fe = a.d == 128 ? fast_entry(es, a.r_k, a.r_v) : FastEntry{nullptr, 1};
-    const int ctas = fe.launch ? fe.ctas : 1;
-    const int budget = ctas == 2 ? kHalfSmem : kSmemLimit;
-    const Layout base = make_layout(0, stage_bytes, a.B, a.r_k, a.r_v, a.d);
-    int stages = (budget - base.total) / stage_bytes;
+    const FastEntry fe = a.d == 128 ? fast_entry(es, a.r_k, a.r_v) : FastEntry{nullptr, nullptr};
+    const int fixed = fe.launch ? fe.layout(0, stage_bytes, a.B)
+                                : make_layout(0, stage_bytes, a.B, a.r_k, a.r_v, a.d).total;
+    int stages = (kSmemLimit - fixed) / stage_bytes;
     if (stages > kMaxStages) stages = kMaxStages;
     if (stages < 2) return LLA_ERR_UNSUPPORTED;
-    const int smem = make_layout(stages, stage_bytes, a.B, a.r_k, a.r_v, a.d).total;
-    const int sms = num_sms();
-    if (sms <= 0) return LLA_ERR_CUDA;
-    const int grid = ctas * sms;
+    const int smem = fe.launch ? fe.layout(stages, stage_bytes, a.B)
+                               : make_layout(stages, stage_bytes, a.B, a.r_k, a.r_v, a.d).total;
+    const int grid = num_sms();  // one CTA per SM
+    if (grid <= 0) return LLA_ERR_CUDA;
     if (a.workspace_bytes < decode_workspace_bytes(a.r_v, a.B, a.H, grid)) return LLA_ERR_WORKSPACE;
     lla_status st = LLA_OK;
     unsigned *err = device_error_word(&st);
