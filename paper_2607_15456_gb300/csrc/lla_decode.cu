@@ -747,7 +747,7 @@ constexpr int kWstMax = 40 * 1024;                 // staging buffer for W_up,t 
 
 struct AsyncLayout {
     int ring, full, empty, pfull, pempty, qready, stfull, prefix, lens, qlat, qfull, spart, psm,
-        lred, red, ovec, mred, mtmp, misc, wst, total;
+        lred, red, ovec, mred, mtmp, xtra, misc, wst, total;
 };
 
 // Shared-memory sizes of the asynchronous kernel for one rank shape (floats per slot).
@@ -764,7 +764,7 @@ struct AsyncSizes {
 
 __host__ __device__ inline AsyncLayout make_async_layout(int stages, int stage_bytes, int B,
                                                          int qslot, int redslot, int mred, int rv,
-                                                         int wst) {
+                                                         int xslot, int wst) {
     AsyncLayout L;
     int o = 0;
     L.ring = o;   o += stages * stage_bytes;
@@ -785,6 +785,7 @@ __host__ __device__ inline AsyncLayout make_async_layout(int stages, int stage_b
     L.ovec = o;   o += up16(rv * 4);
     L.mred = o;   o += up16(mred * 4);
     L.mtmp = o;   o += 2 * kMThreads * 4;
+    L.xtra = o;   o += up16(2 * xslot * 4);
     L.misc = o;   o += 64 * 4;
     L.wst = o;    o += up16(wst);
     L.total = o;
@@ -794,17 +795,19 @@ __host__ __device__ inline AsyncLayout make_async_layout(int stages, int stage_b
 template <int ES, int RK, int RV, int D>
 __host__ __device__ inline AsyncLayout async_layout(int stages, int stage_bytes, int B) {
     using Z = AsyncSizes<ES, RK, RV, D>;
-    return make_async_layout(stages, stage_bytes, B, Z::QSLOT, Z::REDSLOT, Z::MRED, RV, Z::WST);
+    return make_async_layout(stages, stage_bytes, B, Z::QSLOT, Z::REDSLOT, Z::MRED, RV, 2 * D, Z::WST);
 }
 
 // misc slots of the asynchronous kernel
-constexpr int kAM = 0 /* [2] run maximum by slot */, kABeta = 2 /* [2] */, kAScur = 4,
-              kAPAlpha = 5 /* [2] */, kAWmax = 16 /* [2][8] */, kAAbort = 32, kALast = 33;
+constexpr int kAM = 0 /* [2] run maximum by slot */, kAPAlpha = 5 /* [2] */,
+              kAWmax = 16 /* [2][8] */, kAAbort = 32, kALast = 33,
+              kAPart = 40 /* [2][4 warps][q.k_cur, q.mu^K] */;
 
 struct ASmem {
     Smem s;  // fields shared with the generic helpers (ring, barriers, prefix, lens, abort flag)
     uint64_t *qready, *stfull;
     float *qlat, *qfull, *lred, *red, *mred, *mtmp;
+    float *xtra;  // [2][v_cur (D), mu^V_t (D)] by run slot
     char *wst;
     int qslot, redslot;  // floats per slot
 };
@@ -839,6 +842,7 @@ __device__ __forceinline__ ASmem carve_async(char *smem, const Params &p) {
     a.red = reinterpret_cast<float *>(smem + L.red);
     a.mred = reinterpret_cast<float *>(smem + L.mred);
     a.mtmp = reinterpret_cast<float *>(smem + L.mtmp);
+    a.xtra = reinterpret_cast<float *>(smem + L.xtra);
     a.wst = smem + L.wst;
     a.qslot = AsyncSizes<ES, RK, RV, D>::QSLOT;
     a.redslot = AsyncSizes<ES, RK, RV, D>::REDSLOT;
@@ -867,7 +871,37 @@ __device__ __forceinline__ void m_stage_rows(const ASmem &a, const char *W, int 
     cp_async_commit();
 }
 
-// Management: q, q~ = W_up,t^K^T q and beta = q . mu^K_t of a run into slot `slot`.
+// Chunk geometry of W_up,t^V in the staging buffer: rows cut into CB-byte chunks, stored chunk
+// by chunk (chunk c of row e of a pass at (c * ROWS + e) * CB), so that threads owning
+// consecutive rows read consecutive chunks.
+template <int ES, int RV, int D, int WST>
+struct VStage {
+    using P = WPasses<ES, RV, D, WST>;
+    static constexpr int CB = (RV * ES) % 16 == 0 ? 16 : 4;  // chunk bytes
+    static constexpr int CPR = RV * ES / CB;                 // chunks per row
+    static constexpr int EPC = CB / ES;                      // elements per chunk
+    static constexpr int TPR = kMThreads / P::ROWS;          // threads per row
+    static_assert(kMThreads % P::ROWS == 0 && (RV * ES) % 4 == 0, "row ownership");
+};
+
+// Starts the copy of pass `pass` of W_up,t^V into the staging buffer, chunk-major.
+template <int ES, int RV, int D, int WST>
+__device__ __forceinline__ void m_stage_v(const ASmem &a, const char *W, int pass, int mt) {
+    using V = VStage<ES, RV, D, WST>;
+    const char *src = W + static_cast<int64_t>(pass) * V::P::PASS_BYTES;
+    for (int i = mt; i < V::P::ROWS * V::CPR; i += kMThreads) {
+        const int e = i / V::CPR, c = i - e * V::CPR;
+        char *dst = a.wst + (c * V::P::ROWS + e) * V::CB;
+        if constexpr (V::CB == 16) cp_async16(dst, src + i * 16);
+        else cp_async4(dst, src + i * 4);
+    }
+    cp_async_commit();
+}
+
+// Management: everything a run needs that does not depend on its results, into slot `slot`:
+// q, q~ = W_up,t^K^T q, and the per-warp partial sums of beta = q . mu^K_t and of q . k_cur;
+// v_cur and mu^V_t for its output.  All of its global loads go out together, so the set-up costs
+// one round trip plus the W_up,t^K passes, and the run's finish needs none of them.
 template <int ES, int RK, int RV, int D>
 __device__ void m_setup(const Params &p, const ASmem &a, int b, int h, int slot, int mt,
                         bool release_producer) {
@@ -875,30 +909,43 @@ __device__ void m_setup(const Params &p, const ASmem &a, int b, int h, int slot,
     constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
     float *qfull = a.qfull + slot * a.qslot;
     float *qlat = a.qlat + slot * a.qslot;
+    float *xtra = a.xtra + slot * 2 * D;
     const int mwarp = mt >> 5, lane = mt & 31;
     const int64_t qoff = (static_cast<int64_t>(b) * p.H + h) * D;
+    const int64_t hl = (static_cast<int64_t>(h) * p.T + p.loop) * D;
+    const bool pass1 = p.cur_k != nullptr;
     cp_async_wait_all();  // nothing of an earlier use of the staging buffer is still in flight
     m_sync();
-    const float qv = mt < D ? load_elem(p.q, qoff + mt, p.io_bf16) : 0.f;
-    if (!p.absorbed) {
-        if (release_producer) named_bar_arrive(kBarStart, kMThreads + 32);
-        if (mt < D) {
-            qfull[mt] = qv;
-            qlat[mt] = qv;
+    using P = WPasses<ES, RK, D, WST>;
+    const char *W = static_cast<const char *>(p.w_up_k) + hl * RK * ES;
+    if (p.absorbed) m_stage_rows<ES, RK, D, WST>(a, W, 0, mt);
+    // the first set-up's loads go out before the producer fills the ring, not queued behind it
+    if (release_producer) named_bar_arrive(kBarStart, kMThreads + 32);
+    float qv = 0.f, ck = 0.f, cv = 0.f, muk = 0.f, muv = 0.f;
+    if (mt < D) {
+        qv = load_elem(p.q, qoff + mt, p.io_bf16);
+        if (pass1) {
+            ck = load_elem(p.cur_k, qoff + mt, p.io_bf16);
+            cv = load_elem(p.cur_v, qoff + mt, p.io_bf16);
         }
-        if (mt == 0) a.s.misc[kABeta + slot] = 0.f;
+        if (p.absorbed && p.mu_k) muk = p.mu_k[hl + mt];
+        if (p.absorbed && p.mu_v) muv = p.mu_v[hl + mt];
+        qfull[mt] = qv;
+        xtra[mt] = cv;
+        xtra[D + mt] = muv;
+    }
+    const float ps = warp_sum(qv * ck), pb = warp_sum(qv * muk);
+    if (lane == 0) {
+        a.s.misc[kAPart + slot * 8 + mwarp * 2] = ps;
+        a.s.misc[kAPart + slot * 8 + mwarp * 2 + 1] = pb;
+    }
+    if (!p.absorbed) {
+        if (mt < D) qlat[mt] = qv;
         return;
     }
-    using P = WPasses<ES, RK, D, WST>;
     constexpr int CPR = RK / 2;          // pairs per row of W
     constexpr int RG = kMThreads / CPR;  // row groups
     static_assert(RG >= 1 && RG * RK <= 2048, "partial sums fit the management buffer");
-    const char *W = static_cast<const char *>(p.w_up_k) +
-                    (static_cast<int64_t>(h) * p.T + p.loop) * D * RK * ES;
-    m_stage_rows<ES, RK, D, WST>(a, W, 0, mt);
-    // the first set-up's loads go out before the producer fills the ring, not queued behind it
-    if (release_producer) named_bar_arrive(kBarStart, kMThreads + 32);
-    if (mt < D) qfull[mt] = qv;
     const int cg = mt % CPR, rg = mt / CPR;
     float acc0 = 0.f, acc1 = 0.f;
 #pragma unroll 1
@@ -922,15 +969,6 @@ __device__ void m_setup(const Params &p, const ASmem &a, int b, int h, int slot,
         a.mred[rg * RK + cg * 2] = acc0;
         a.mred[rg * RK + cg * 2 + 1] = acc1;
     }
-    if (mwarp == kMWarps - 1) {
-        float bsum = 0.f;
-        if (p.mu_k) {
-            const float *mu = p.mu_k + (static_cast<int64_t>(h) * p.T + p.loop) * D;
-            for (int e = lane; e < D; e += 32) bsum = fmaf(qfull[e], mu[e], bsum);
-        }
-        bsum = warp_sum(bsum);
-        if (lane == 0) a.s.misc[kABeta + slot] = bsum;
-    }
     m_sync();
     for (int j = mt; j < RK; j += kMThreads) {
         float acc = 0.f;
@@ -940,40 +978,30 @@ __device__ void m_setup(const Params &p, const ASmem &a, int b, int h, int slot,
     }
 }
 
+// Sum of the management warps' partials k (0: q . k_cur, 1: q . mu^K_t) of a slot.
+__device__ __forceinline__ float m_part(const ASmem &a, int slot, int k) {
+    const float *pp = a.s.misc + kAPart + slot * 8 + k;
+    return (pp[0] + pp[2]) + (pp[4] + pp[6]);
+}
+
 // Management: output of one (sequence, head) from its softmax state (m, l, a.s.ovec).
-// o = (W_up,t^V ovec wl + lc mu^V_t + p_cur v_cur) / (lc + p_cur).  W_up,t^V comes through the
-// staging buffer (its first pass already in flight when `staged`); a warp takes one row at a
-// time, lanes along the row, so the shared-memory reads are conflict-free.
+// o = (W_up,t^V ovec wl + lc mu^V_t + p_cur v_cur) / (lc + p_cur).  The first pass of W_up,t^V
+// is already in flight in the staging buffer.  Each row of the pass has TPR threads (one when
+// the pass holds all D rows); their chunk reads are conflict-free, ovec reads are broadcasts
+// and the output stores coalesce.
 template <int ES, int RK, int RV, int D>
 __device__ void m_output(const Params &p, const ASmem &a, int b, int h, float m, float l, int slot,
-                         int mt, bool staged) {
+                         int mt) {
     static_assert(D <= kMThreads, "one management thread per output element");
     constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
-    using P = WPasses<ES, RV, D, WST>;
-    constexpr int NP = RV / 2;  // pairs per row
-    const float *qfull = a.qfull + slot * a.qslot;
-    const int mwarp = mt >> 5, lane = mt & 31;
+    using V = VStage<ES, RV, D, WST>;
+    using P = typename V::P;
+    const float *vcur = a.xtra + slot * 2 * D, *muv = vcur + D;
     const bool pass1 = p.cur_k != nullptr;
     const int64_t orow = (static_cast<int64_t>(b) * p.H + h) * D;
-    const char *W = static_cast<const char *>(p.w_up_v) +
-                    (static_cast<int64_t>(h) * p.T + p.loop) * D * RV * ES;
-    if (p.absorbed && !staged) m_stage_rows<ES, RV, D, WST>(a, W, 0, mt);
-    // per-row extras of this output, one element per thread
-    float *vcur = a.mtmp, *muv = a.mtmp + kMThreads;
-    if (mt < D) {
-        vcur[mt] = pass1 ? load_elem(p.cur_v, orow + mt, p.io_bf16) : 0.f;
-        muv[mt] = (p.absorbed && p.mu_v) ? p.mu_v[(static_cast<int64_t>(h) * p.T + p.loop) * D + mt] : 0.f;
-    }
-    if (pass1 && mwarp == 0) {
-        float acc = 0.f;
-        for (int i = lane; i < D; i += 32) acc = fmaf(qfull[i], load_elem(p.cur_k, orow + i, p.io_bf16), acc);
-        acc = warp_sum(acc);
-        if (lane == 0) a.s.misc[kAScur] = acc * p.scale_log2;
-    }
-    m_sync();
     float M = m, pc = 0.f;
     if (pass1) {
-        const float sc = a.s.misc[kAScur];
+        const float sc = m_part(a, slot, 0) * p.scale_log2;
         M = fmaxf(m, sc);
         pc = exp2f(sc - M);
     }
@@ -988,29 +1016,42 @@ __device__ void m_output(const Params &p, const ASmem &a, int b, int h, float m,
         m_sync();
         return;
     }
+    const char *W = static_cast<const char *>(p.w_up_v) +
+                    (static_cast<int64_t>(h) * p.T + p.loop) * D * RV * ES;
+    const int er = mt % P::ROWS, sub = mt / P::ROWS;
 #pragma unroll 1
     for (int pass = 0; pass < P::N; ++pass) {
         cp_async_wait_all();
         m_sync();
-#pragma unroll 2
-        for (int er = mwarp; er < P::ROWS; er += kMWarps) {
-            float acc = 0.f;
-            for (int jp = lane; jp < NP; jp += 32) {
-                const float2 w = load_pair<ES>(a.wst, static_cast<int64_t>(er) * RV + 2 * jp);
-                const float2 o2 = *reinterpret_cast<const float2 *>(a.s.ovec + 2 * jp);
-                acc = fmaf(w.x, o2.x, acc);
-                acc = fmaf(w.y, o2.y, acc);
-            }
-            acc = warp_sum(acc);
-            if (lane == 0) {
-                const int e = pass * P::ROWS + er;
-                float o = fmaf(lc, muv[e], acc * wl);
-                o = fmaf(pc, vcur[e], o);
-                store_elem(p.out, orow + e, o * inv, p.io_bf16);
+        float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll 4
+        for (int c = sub; c < V::CPR; c += V::TPR) {
+            float w[V::EPC];
+            load_gran<ES, V::CB>(a.wst + (c * P::ROWS + er) * V::CB, w);
+            const float *ov = a.s.ovec + c * V::EPC;
+#pragma unroll
+            for (int k = 0; k < V::EPC; ++k) {
+                if (k & 1) acc1 = fmaf(w[k], ov[k], acc1);
+                else acc0 = fmaf(w[k], ov[k], acc0);
             }
         }
-        m_sync();  // the buffer is read before the next pass (or set-up) overwrites it
-        if (pass + 1 < P::N) m_stage_rows<ES, RV, D, WST>(a, W, pass + 1, mt);
+        float acc = acc0 + acc1;
+        if constexpr (V::TPR > 1) {
+            a.mtmp[mt] = acc;
+            m_sync();
+            if (sub == 0) {
+#pragma unroll
+                for (int t = 1; t < V::TPR; ++t) acc += a.mtmp[er + t * P::ROWS];
+            }
+        }
+        if (sub == 0) {
+            const int e = pass * P::ROWS + er;
+            float o = fmaf(lc, muv[e], acc * wl);
+            o = fmaf(pc, vcur[e], o);
+            store_elem(p.out, orow + e, o * inv, p.io_bf16);
+        }
+        m_sync();  // the buffer (and mtmp) is read before the next pass or set-up overwrites it
+        if (pass + 1 < P::N) m_stage_v<ES, RV, D, WST>(a, W, pass + 1, mt);
     }
 }
 
@@ -1028,15 +1069,13 @@ template <int ES, int RK, int RV, int D, int TT, int NTG>
 __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t u, const Range &rg,
                          int slot, uint32_t parity, int mt) {
     constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
+    // The output's first pass of W_up,t^V travels while the run still streams: the set-up
+    // before this finish has read the staging buffer to the end and waited for its copies.
+    if (p.absorbed)
+        m_stage_v<ES, RV, D, WST>(a, static_cast<const char *>(p.w_up_v) +
+                                         (static_cast<int64_t>(R.h) * p.T + p.loop) * D * RV * ES,
+                                  0, mt);
     mbar_wait(&a.stfull[slot], parity, a.s.abort_flag, p.err);
-    if (p.absorbed) {
-        // the output's first pass of W_up,t^V travels while the partial protocol runs
-        cp_async_wait_all();
-        m_sync();
-        m_stage_rows<ES, RV, D, WST>(a, static_cast<const char *>(p.w_up_v) +
-                                            (static_cast<int64_t>(R.h) * p.T + p.loop) * D * RV * ES,
-                                     0, mt);
-    }
     const float *red = a.red + slot * a.redslot;
     const float *lred = a.lred + slot * kComputeThreads;
     for (int j = mt; j < RV; j += kMThreads) {  // fixed order: bitwise-reproducible sums
@@ -1050,7 +1089,7 @@ __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t 
     const float m = a.s.misc[kAM + slot];
     m_sync();
     if (u == R.seg_start && R.run_end == R.seg_end) {
-        m_output<ES, RK, RV, D>(p, a, R.b, R.h, m, l, slot, mt, true);
+        m_output<ES, RK, RV, D>(p, a, R.b, R.h, m, l, slot, mt);
         return;
     }
     const int c = blockIdx.x;
@@ -1141,7 +1180,7 @@ __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t 
         }
     }
     m_sync();
-    m_output<ES, RK, RV, D>(p, a, R.b, R.h, M, lsum, slot, mt, true);
+    m_output<ES, RK, RV, D>(p, a, R.b, R.h, M, lsum, slot, mt);
     if (mt == 0) atomicExch(counter, 0);
 }
 
@@ -1225,7 +1264,7 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
         const float *qq = a.qlat + rslot * a.qslot + ks * F::NGT * F::KE;
         if (is_s) {
             mbar_wait(&a.qready[rslot], (r >> 1) & 1, s.abort_flag, p.err);
-            beta = s.misc[kABeta + rslot];
+            beta = m_part(a, rslot, 1);
         }
         float m_run = -INFINITY, l_part = 0.f;
         float accv[AV];
