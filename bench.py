@@ -332,7 +332,7 @@ def run_ours(args, rank, world, local_rank):
         "roofline": {
             "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
             "frac": achieved / peak, "traffic": ncu_traffic(w.name),
-            "kernel": "decode_kernel (lla_decode_attn)",
+            "kernel": "decode_async_kernel (lla_decode_attn)",
             "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
                            if peak_kind == "measured" else "fallback 6.8 TB/s",
             "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,

@@ -5,7 +5,7 @@ ranks, so every decode launch has exactly the shape and bytes of a launch in the
 benchmark), then runs `--calls` pass-1 decode calls (and one encode call per layer), so that a
 profiler can skip the warm-up launches and capture one to three of them:
 
-    ncu --set full --clock-control none -k regex:decode_kernel -s 6 -c 2 \\
+    ncu --set full --clock-control none -k regex:decode_async_kernel -s 6 -c 1 \\
         python -m paper_2607_15456_gb300.profile_case --workload ouro14_rho4 --layers 2 --calls 10
 """
 from __future__ import annotations
