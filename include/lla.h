@@ -88,8 +88,8 @@ typedef struct {
 
 /* Codec of one layer (Eqs. encode and decode), for all H heads; device pointers. */
 typedef struct {
-    const void *w_down_k; /* [H][T*d][r_k] storage dtype: W_down of the K axis */
-    const void *w_down_v; /* [H][T*d][r_v] storage dtype */
+    const void *w_down_k; /* [H][T*d][r_k] storage dtype: W_down of the K axis (16-B aligned) */
+    const void *w_down_v; /* [H][T*d][r_v] storage dtype (16-B aligned) */
     const void *w_up_k;   /* [H][T][d][r_k] storage dtype: W_up,t of the K axis (16-B aligned) */
     const void *w_up_v;   /* [H][T][d][r_v] storage dtype (16-B aligned) */
     const float *mu_k;    /* [H][T*d] fp32 calibration mean, or NULL for mu = 0 */
@@ -115,8 +115,9 @@ lla_status lla_cache_block_bytes(const lla_geometry *g, size_t *bytes);
 
 /*
  * Eq. encode (Sec. 3) for N newly completed tokens of one layer, written into the cache.
- *   x_k, x_v      device [T][N][H][d] in x_dtype: the pre-RoPE loop-t keys / values of each
- *                 token (Sec. 3 "RoPE and reconstruction"; App. A "LLA codec and conversion")
+ *   x_k, x_v      device [T][N][H][d] in x_dtype, 16-byte aligned: the pre-RoPE loop-t keys /
+ *                 values of each token (Sec. 3 "RoPE and reconstruction"; App. A "LLA codec
+ *                 and conversion")
  *   slot_mapping  device [N] int64: destination slot of each token; a negative slot skips
  *                 the token.  A slot beyond the pool sets LLA_DEVERR_SLOT.
  * Latents are computed with fp32 accumulation and rounded to `storage` (round to nearest

@@ -111,9 +111,8 @@ lla_status lla_encode(const lla_geometry *g, const lla_codec *codec, const lla_c
     if ((st = check_cache(cache, false)) != LLA_OK) return st;
     if (!valid_dtype(x_dtype) || N < 0) return LLA_ERR_INVALID_ARG;
     if (N > 0 && (!x_k || !x_v || !slot_mapping)) return LLA_ERR_INVALID_ARG;
-    const int es = elem_size(g->storage);
-    if (!aligned(codec->w_down_k, 2 * es) || !aligned(codec->w_down_v, 2 * es))
-        return LLA_ERR_INVALID_ARG;
+    if (!aligned(codec->w_down_k, 16) || !aligned(codec->w_down_v, 16)) return LLA_ERR_INVALID_ARG;
+    if (N > 0 && (!aligned(x_k, 16) || !aligned(x_v, 16))) return LLA_ERR_INVALID_ARG;
     if (N == 0) return LLA_OK;
     EncodeArgs a = {};
     a.T = g->T; a.H = g->H; a.d = g->d; a.r_k = g->r_k; a.r_v = g->r_v;

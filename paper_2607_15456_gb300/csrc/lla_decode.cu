@@ -114,8 +114,7 @@ __host__ __device__ inline Layout make_layout(int stages, int stage_bytes, int B
 
 // misc slots
 constexpr int kMiscAlpha = 0, kMiscM = 1, kMiscL = 2, kMiscBeta = 3, kMiscScur = 4,
-              kMiscPAlpha = 5 /* 5, 6 */, kMiscWmax = 16 /* [2][8] */, kMiscAbort = 32,
-              kMiscLast = 33;
+              kMiscWmax = 16 /* [2][8] */, kMiscAbort = 32, kMiscLast = 33;
 
 struct Smem {
     char *ring;

@@ -100,6 +100,10 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_all() {
     asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
+// all but the most recent group of copies have landed
+__device__ __forceinline__ void cp_async_wait_but_one() {
+    asm volatile("cp.async.wait_group 1;" ::: "memory");
+}
 
 __device__ __forceinline__ uint64_t policy_evict_first() {
     uint64_t p;

@@ -8,10 +8,12 @@
 // V-plane of its block's head page.
 //
 // One CTA takes (a tile of up to 16 tokens, a tile of 32 latent columns of one axis, one head).
-// The tile's centred stacked vectors are staged in shared memory (fp32); 256 threads are 16
-// column pairs x 16 slices of the T*d reduction axis, each streaming its slice of W_down with
-// several loads in flight, and the 16 partial sums per output meet in shared memory.  At a decode
-// step (N = batch) this spreads the weight-bound work over H x (r_k + r_v)/32 CTAs.
+// Everything the CTA reads is in flight at once: its W_down columns move into shared memory with
+// cp.async in chunks of the T*d reduction axis (double-buffered when T*d is long), and the tile's
+// stacked loop vectors are loaded four 16-byte words per thread before any is used, then centred
+// (x - mu) into shared memory as fp32.  At a decode step (N = batch) a launch therefore costs
+// about one memory round trip.  256 threads are 16 column pairs x 4 groups of 4 tokens x 4
+// slices of the reduction axis; the 4 partial sums per output meet in shared memory.
 #include <cuda_runtime.h>
 
 #include "lla_device.cuh"
@@ -23,9 +25,12 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kColTile = 32;          // latent columns per CTA
 constexpr int kPairs = kColTile / 2;  // column pairs per CTA
-constexpr int kSlices = kThreads / kPairs;  // slices of the reduction axis
 constexpr int kMaxTileTokens = 16;
+constexpr int kTokGroups = kMaxTileTokens / 4;          // groups of 4 tokens
+constexpr int kKSlices = kThreads / (kPairs * kTokGroups);  // slices of the reduction axis
 constexpr int kXsBudget = 96 * 1024;  // shared bytes for the staged token tile
+constexpr int kWBuf = 32 * 1024;      // one chunk of W_down columns (two are in flight)
+constexpr int kXBatch = 4;            // 16-byte words of x in flight per thread
 
 struct EncParams {
     int T, H, d, r_k, r_v, x_bf16;
@@ -52,12 +57,38 @@ __device__ __forceinline__ void store_latent(char *dst, float v) {
     else *reinterpret_cast<float *>(dst) = v;
 }
 
+// Rows of W_down per shared-memory chunk.
+template <int ES>
+__host__ __device__ constexpr int chunk_rows() { return kWBuf / (kColTile * ES); }
+
+// Starts the copy of rows [k0, k0 + rows) x columns [col0, col0 + ncol) of W (row length r)
+// into wb ([rows][kColTile] storage dtype).  16-byte copies when every row segment is 16-byte
+// aligned, 4-byte copies otherwise (r x es not a multiple of 16).
+template <int ES>
+__device__ __forceinline__ void stage_w(char *wb, const char *W, int r, int col0, int ncol, int k0,
+                                        int rows, int tid) {
+    const bool wide = (r * ES) % 16 == 0 && (ncol * ES) % 16 == 0;
+    const int unit = wide ? 16 : 4;
+    const int per_row = ncol * ES / unit;
+    const int total = rows * per_row;
+    for (int i = tid; i < total; i += kThreads) {
+        const int k = i / per_row, c = i - k * per_row;
+        const char *src = W + (static_cast<int64_t>(k0 + k) * r + col0) * ES + c * unit;
+        char *dst = wb + k * (kColTile * ES) + c * unit;
+        if (wide) cp_async16(dst, src);
+        else cp_async4(dst, src);
+    }
+    cp_async_commit();
+}
+
 template <int ES>
 __global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
     extern __shared__ __align__(16) float smem_f[];
+    constexpr int KC = chunk_rows<ES>();
     const int Td = p.T * p.d;
-    float *xs = smem_f;                          // [tile][Td] centred stacked vectors
-    float *red = smem_f + p.tile * Td;           // [kSlices][tile][kColTile] partial sums
+    float *xs = smem_f;                                       // [tile][Td] centred stacked vectors
+    char *wbuf = reinterpret_cast<char *>(xs + p.tile * Td);  // [2][KC][kColTile] W_down chunks
+    float *red = reinterpret_cast<float *>(wbuf + 2 * kWBuf);  // [kKSlices][tile][kColTile]
     const int ct = blockIdx.y;
     const int axis = ct < p.ctiles_k ? 0 : 1;
     const int col0 = (axis ? ct - p.ctiles_k : ct) * kColTile;
@@ -65,67 +96,116 @@ __global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
     const int n0 = blockIdx.x * p.tile;
     const int nt = min(p.tile, p.N - n0);
     const int r = axis ? p.r_v : p.r_k;
-    const void *W = axis ? p.w_down_v : p.w_down_k;
+    const int ncol = min(kColTile, r - col0);
+    const char *W = static_cast<const char *>(axis ? p.w_down_v : p.w_down_k) +
+                    static_cast<int64_t>(h) * Td * r * ES;
     const float *mu = axis ? p.mu_v : p.mu_k;
-    const void *x = axis ? p.x_v : p.x_k;
+    const char *x = static_cast<const char *>(axis ? p.x_v : p.x_k);
     const int tid = threadIdx.x;
+    const int nch = (Td + KC - 1) / KC;
 
     pdl_wait();
-    // stack the loop vectors of the tile's tokens and centre them: x - mu
-    for (int idx = tid; idx < nt * Td; idx += kThreads) {
-        const int n = idx / Td, k = idx - n * Td;
-        const int t = k / p.d, e = k - t * p.d;
-        const int64_t src = ((static_cast<int64_t>(t) * p.N + n0 + n) * p.H + h) * p.d + e;
-        float v = load_elem(x, src, p.x_bf16);
-        if (mu) v -= mu[static_cast<int64_t>(h) * Td + k];
-        xs[n * Td + k] = v;
-    }
-    __syncthreads();
+    stage_w<ES>(wbuf, W, r, col0, ncol, 0, min(KC, Td), tid);
+    if (nch > 1) stage_w<ES>(wbuf + kWBuf, W, r, col0, ncol, KC, min(KC, Td - KC), tid);
 
-    // c = (x - mu) W_down over this thread's slice of the reduction axis
-    const int jp = tid % kPairs, sl = tid / kPairs;
-    const int col = col0 + 2 * jp;
-    const bool active = col < r;
-    float2 acc[kMaxTileTokens];
+    // stack the loop vectors of the tile's tokens and centre them: x - mu.  Rows (n, t) of d
+    // elements are contiguous in x; kXBatch 16-byte words per thread are loaded before use.
+    {
+        const int xes = p.x_bf16 ? 2 : 4;
+        const int wpr = p.d * xes / 16;  // 16-byte words per row (d is a multiple of 8)
+        const int epw = 16 / xes;        // elements per word
+        const int total = nt * p.T * wpr;
+        for (int base = 0; base < total; base += kThreads * kXBatch) {
+            uint4 v[kXBatch];
 #pragma unroll
-    for (int i = 0; i < kMaxTileTokens; ++i) acc[i] = make_float2(0.f, 0.f);
-    if (active) {
-        const int64_t wbase = static_cast<int64_t>(h) * Td * r + col;
-        int k = sl;
-        for (; k + 3 * kSlices < Td; k += 4 * kSlices) {
-            float2 w[4];
+            for (int b = 0; b < kXBatch; ++b) {
+                const int i = base + b * kThreads + tid;
+                if (i < total) {
+                    const int row = i / wpr, c = i - row * wpr;
+                    const int n = row / p.T, t = row - n * p.T;
+                    const int64_t off =
+                        ((static_cast<int64_t>(t) * p.N + n0 + n) * p.H + h) * p.d * xes + c * 16;
+                    v[b] = *reinterpret_cast<const uint4 *>(x + off);
+                }
+            }
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
-                w[u] = load_pair<ES>(W, wbase + static_cast<int64_t>(k + u * kSlices) * r);
+            for (int b = 0; b < kXBatch; ++b) {
+                const int i = base + b * kThreads + tid;
+                if (i < total) {
+                    const int row = i / wpr, c = i - row * wpr;
+                    const int n = row / p.T, t = row - n * p.T;
+                    const int k0 = t * p.d + c * epw;
+                    float f[8];
+                    if (p.x_bf16) {
+                        const float2 a = bf2_to_f2(v[b].x), bb = bf2_to_f2(v[b].y),
+                                     cc = bf2_to_f2(v[b].z), e = bf2_to_f2(v[b].w);
+                        f[0] = a.x; f[1] = a.y; f[2] = bb.x; f[3] = bb.y;
+                        f[4] = cc.x; f[5] = cc.y; f[6] = e.x; f[7] = e.y;
+                    } else {
+                        f[0] = __uint_as_float(v[b].x); f[1] = __uint_as_float(v[b].y);
+                        f[2] = __uint_as_float(v[b].z); f[3] = __uint_as_float(v[b].w);
+                        f[4] = f[5] = f[6] = f[7] = 0.f;
+                    }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-#pragma unroll
-                for (int i = 0; i < kMaxTileTokens; ++i) {
-                    if (i < nt) {
-                        const float xv = xs[i * Td + k + u * kSlices];
-                        acc[i].x = fmaf(xv, w[u].x, acc[i].x);
-                        acc[i].y = fmaf(xv, w[u].y, acc[i].y);
+                    for (int q = 0; q < 8; ++q) {
+                        if (q < epw) {
+                            float val = f[q];
+                            if (mu) val -= mu[static_cast<int64_t>(h) * Td + k0 + q];
+                            xs[n * Td + k0 + q] = val;
+                        }
                     }
                 }
             }
         }
-        for (; k < Td; k += kSlices) {
-            const float2 w = load_pair<ES>(W, wbase + static_cast<int64_t>(k) * r);
+    }
+
+    // c = (x - mu) W_down.  Thread = (column pair jp, group of 4 tokens tg, reduction slice
+    // ks); slice ks takes the row quads q = ks, ks + 4, ... of each chunk, so a thread reads a
+    // float4 of x per token and one W pair per row.
+    const int jp = tid % kPairs, tg = (tid / kPairs) % kTokGroups, ks = tid / (kPairs * kTokGroups);
+    const bool active = 2 * jp < ncol && 4 * tg < nt;
+    float2 acc[4];
 #pragma unroll
-            for (int i = 0; i < kMaxTileTokens; ++i) {
-                if (i < nt) {
-                    const float xv = xs[i * Td + k];
-                    acc[i].x = fmaf(xv, w.x, acc[i].x);
-                    acc[i].y = fmaf(xv, w.y, acc[i].y);
+    for (int i = 0; i < 4; ++i) acc[i] = make_float2(0.f, 0.f);
+    for (int ch = 0; ch < nch; ++ch) {
+        if (ch + 1 < nch) cp_async_wait_but_one();
+        else cp_async_wait_all();
+        __syncthreads();  // chunk ch (and, the first time, the token tile) is visible
+        const char *wb = wbuf + (ch & 1) * kWBuf;
+        const int kc0 = ch * KC;
+        const int quads = min(KC, Td - kc0) / 4;  // T*d and KC are multiples of 8
+        if (active) {
+            const float *x0 = xs + (4 * tg) * Td + kc0;
+#pragma unroll 2
+            for (int q = ks; q < quads; q += kKSlices) {
+                float4 xv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) xv[i] = *reinterpret_cast<const float4 *>(x0 + i * Td + 4 * q);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const float2 w = load_pair<ES>(wb, static_cast<int64_t>(4 * q + u) * kColTile + 2 * jp);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float xe = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
+                        acc[i].x = fmaf(xe, w.x, acc[i].x);
+                        acc[i].y = fmaf(xe, w.y, acc[i].y);
+                    }
                 }
             }
         }
+        if (ch + 2 < nch) {
+            __syncthreads();  // every thread is done with this buffer
+            stage_w<ES>(wbuf + (ch & 1) * kWBuf, W, r, col0, ncol, (ch + 2) * KC,
+                        min(KC, Td - (ch + 2) * KC), tid);
+        }
     }
+    pdl_trigger();  // the next kernel in the stream may start its launch
 #pragma unroll
-    for (int i = 0; i < kMaxTileTokens; ++i) {
-        if (i < nt) {
-            red[(sl * p.tile + i) * kColTile + 2 * jp] = acc[i].x;
-            red[(sl * p.tile + i) * kColTile + 2 * jp + 1] = acc[i].y;
+    for (int i = 0; i < 4; ++i) {
+        const int n = 4 * tg + i;
+        if (n < nt) {
+            red[(ks * p.tile + n) * kColTile + 2 * jp] = acc[i].x;
+            red[(ks * p.tile + n) * kColTile + 2 * jp + 1] = acc[i].y;
         }
     }
     __syncthreads();
@@ -135,9 +215,9 @@ __global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
     for (int o = tid; o < nt * kColTile; o += kThreads) {
         const int i = o / kColTile, c = o % kColTile;
         const int j = col0 + c;
-        if (j >= r) continue;
+        if (c >= ncol) continue;
         float v = 0.f;
-        for (int s2 = 0; s2 < kSlices; ++s2) v += red[(s2 * p.tile + i) * kColTile + c];
+        for (int s2 = 0; s2 < kKSlices; ++s2) v += red[(s2 * p.tile + i) * kColTile + c];
         const int64_t slot = p.slot_mapping[n0 + i];
         if (slot < 0) continue;
         const int64_t blk = slot / kBlockTokens;
@@ -199,7 +279,8 @@ lla_status set_smem(int dev) {
     static bool configured[64] = {};
     if (dev < 64 && configured[dev]) return LLA_OK;
     if (cudaFuncSetAttribute(encode_kernel<ES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kXsBudget + kSlices * kMaxTileTokens * kColTile * 4) != cudaSuccess)
+                             kXsBudget + 2 * kWBuf + kKSlices * kMaxTileTokens * kColTile * 4) !=
+        cudaSuccess)
         return LLA_ERR_CUDA;
     if (dev < 64) configured[dev] = true;
     return LLA_OK;
@@ -237,7 +318,7 @@ lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream) {
     p.tile = tile;
     p.ctiles_k = (a.r_k + kColTile - 1) / kColTile;
     const int ctiles_v = (a.r_v + kColTile - 1) / kColTile;
-    const int smem = (tile * Td + kSlices * tile * kColTile) * 4;
+    const int smem = (tile * Td + kKSlices * tile * kColTile) * 4 + 2 * kWBuf;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     st = es == 2 ? set_smem<2>(dev) : set_smem<4>(dev);
