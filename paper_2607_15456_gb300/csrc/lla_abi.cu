@@ -239,9 +239,8 @@ lla_status lla_prefill_attn(const lla_geometry *g, const lla_codec *codec, const
     if (st != LLA_OK) return st;
     if ((st = check_cache(cache, true)) != LLA_OK) return st;
     if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;
-    const int es = elem_size(g->storage);
-    if (!aligned(codec->w_up_k, 2 * es) || !aligned(codec->w_up_v, 2 * es))
-        return LLA_ERR_INVALID_ARG;
+    if (!aligned(codec->w_up_k, 16) || !aligned(codec->w_up_v, 16)) return LLA_ERR_INVALID_ARG;
+    if ((q && !aligned(q, 16)) || (out && !aligned(out, 16))) return LLA_ERR_INVALID_ARG;
     if (loop < 0 || loop >= g->T || B < 0 || B > LLA_MAX_BATCH || !valid_dtype(io_dtype))
         return LLA_ERR_INVALID_ARG;
     if (max_len < 0 || static_cast<int64_t>(max_len) >

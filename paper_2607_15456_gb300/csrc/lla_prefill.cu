@@ -1,8 +1,673 @@
-// lla_prefill.cu -- causal pass-2 prefill attention over latents.
+// lla_prefill.cu -- causal pass-2 prefill attention over latents (App. A, two-pass prefill;
+// App. J absorbed attention).
+//
+// For a prompt of L tokens whose latents are all in the cache, query i at loop t attends to
+// keys 0..i:
+//   q~_i = W_up,t^K^T q_i                       (the constant q_i . mu^K_t cancels in softmax)
+//   s_ij = scale * q~_i . c_k,j,   p_i = softmax_j<=i(s_i)
+//   o_i  = W_up,t^V (sum_j p_ij c_v,j) + mu^V_t
+//
+// Tensor-core path (bf16 storage, d = 128, r_k and r_v multiples of 16): one CTA per
+// (128-query tile, sequence, head) and four warp roles.
+//   warp 0      producer: W_up,t^K into shared memory (cp.async), then per page of 64 keys the
+//               K-plane (one bulk copy: its granule-interleaved layout is already the
+//               core-matrix layout of a K-major MMA operand) and the V-plane (16-byte cp.async
+//               gathers into an MN-major core-matrix layout; rows past the prompt are zeroed),
+//               and W_up,t^V for the epilogue
+//   warp 1      MMA issuer (one thread) and TMEM owner:
+//                 Q~ = Q W_up,t^K             M=128, N=r_k, K=d
+//                 S_j = Q~ C_k,j^T            M=128, N=64,  K=r_k   (one page ahead of PV)
+//                 O += P_j C_v,j              M=128, N=r_v (split at 256), K=64
+//                 out = (O/l) W_up,t^V^T      M=128, N=d,   K=r_v
+//   warps 2-5   one query row per thread: Q and Q~ into bf16 operands, causal mask and online
+//               softmax in the exp2 domain, P into a bf16 operand, O rescaled in TMEM only when
+//               a row maximum grows by more than 2^8, then the epilogue.
+// Accumulators are fp32 in TMEM; operands are bf16 (q~ carries scale * log2 e).
+//
+// CUDA-core path (fp32 storage, other ranks, d != 128): one CTA per (query, sequence, head),
+// fp32 throughout.
+#include <cuda_runtime.h>
+
+#include "lla_device.cuh"
 #include "lla_internal.h"
+#include "lla_tcgen05.cuh"
 
 namespace lla {
+namespace {
 
-lla_status launch_prefill(const PrefillArgs &, cudaStream_t) { return LLA_ERR_UNSUPPORTED; }
+constexpr int kBM = 128;        // queries per tile
+constexpr int kPT = 64;         // keys per page
+constexpr int kPThreads = 192;  // producer, MMA, 4 softmax warps
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kRescaleLog2 = 8.f;  // rescale O only when a row maximum grows by more
+
+struct PParams {
+    int T, H, loop, io_bf16;
+    float scale_log2;
+    const void *w_up_k, *w_up_v;
+    const float *mu_v;
+    const char *pool;
+    int64_t num_blocks, block_bytes;
+    int head_page_bytes;
+    const int32_t *block_table;
+    int max_blocks;
+    const int32_t *cu_seqlens;
+    int B, max_len;
+    const void *q;
+    void *out;
+    unsigned *err;
+};
+
+// Shared-memory plan of the tensor-core kernel for ranks (RK, RV); d = 128.
+template <int RK, int RV>
+struct PF {
+    static constexpr int D = 128;
+    static constexpr int NKC = RK / 8;               // 16-byte chunks of a K row
+    static constexpr int NVC = RV / 8;               // 16-byte chunks of a V row
+    static constexpr int NSPL = RV > 256 ? 2 : 1;    // PV MMAs per K step (N <= 256)
+    static constexpr int NV = RV / NSPL;
+    static constexpr int KPAGE = kPT * RK * 2;
+    static constexpr int VPAGE = kPT * RV * 2;
+    static constexpr int QT = kBM * RK * 2;          // q~ operand
+    static constexpr int PB = kBM * kPT * 2;         // P operand (one of two)
+    static constexpr int QA = kBM * D * 2;           // q operand (prologue)
+    static constexpr int WK = D * RK * 2;            // W_up,t^K operand (prologue)
+    static constexpr int WV = D * RV * 2;            // W_up,t^V operand (epilogue)
+    static constexpr int OA = kBM * RV * 2;          // O / l operand (epilogue)
+    static constexpr int ST = 2;                     // K and V pipeline stages
+    static constexpr int oQT = 0;
+    static constexpr int oK = oQT + QT;
+    static constexpr int oV = oK + ST * KPAGE;
+    static constexpr int oP = oV + ST * VPAGE;
+    static constexpr int oEnd = oP + 2 * PB;
+    // the prologue operands alias the V ring and P; the epilogue operands alias K, V and P
+    static constexpr int oQA = oV, oWK = oV + QA;
+    static constexpr int oOA = oK, oWV = oK + OA;
+    static constexpr int oBar = oEnd;
+    static constexpr int NBAR = 32;
+    static constexpr int SMEM = oBar + NBAR * 8 + 16;
+    // TMEM columns: S double buffer [0, 128), O [128, 128 + RV); q~ and out reuse [0, ...)
+    static constexpr uint32_t TM_S = 0, TM_O = 128, TM_COLS = 512;
+    static_assert(RK % 16 == 0 && RV % 16 == 0 && RK <= 256 && 128 + RV <= 512, "ranks");
+    static_assert(NV % 16 == 0 && NV <= 256, "PV split");
+    static_assert(oWK + WK <= oEnd && oWV + WV <= oEnd, "aliased operands fit");
+    static_assert(SMEM <= 227 * 1024, "shared memory");
+};
+
+// barrier indices
+enum {
+    kBSetup = 0, kBQt, kBQs, kBOa, kBWv, kBOut, kBOdone, kBOfin,
+    kBOa2 = 24, kBOut1 = 25,
+    kBKfull = 8 /* [2] */, kBKempty = 10, kBVfull = 12, kBVempty = 14,
+    kBSfull = 16, kBSfree = 18, kBPfull = 20, kBPfree = 22,
+    kBAbort = 31  // slot used as the CTA's abort flag
+};
+
+template <int RK, int RV>
+__global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams p) {
+    using F = PF<RK, RV>;
+    constexpr int D = F::D;
+    extern __shared__ __align__(1024) char sm[];
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + F::oBar);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar + kBAbort);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + F::NBAR);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    const int nqt = (p.max_len + kBM - 1) / kBM;
+    const int qt = nqt - 1 - static_cast<int>(blockIdx.x);  // longest causal ranges first
+    const int b = blockIdx.y, h = blockIdx.z;
+    pdl_wait();
+    const int q0 = p.cu_seqlens[b];
+    const int L = p.cu_seqlens[b + 1] - q0;
+    if (L > p.max_len || L < 0) {
+        if (tid == 0 && qt == nqt - 1) atomicOr(p.err, LLA_DEVERR_CONTEXT);
+        return;
+    }
+    const int i0 = qt * kBM;
+    if (i0 >= L) return;  // uniform over the CTA, before any barrier or TMEM use
+    const int iend = min(L, i0 + kBM);
+    const int NP = (iend - 1) / kPT + 1;  // pages 0..NP-1 hold every key of the tile
+    const int64_t wofs = (static_cast<int64_t>(h) * p.T + p.loop) * D;
+    const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks;
+
+    if (tid == 0) {
+        mbar_init(&bar[kBSetup], 32 + 128);
+        mbar_init(&bar[kBQt], 1);
+        mbar_init(&bar[kBQs], 128);
+        mbar_init(&bar[kBOa], 128);
+        mbar_init(&bar[kBWv], 32);
+        mbar_init(&bar[kBOut], 1);
+        mbar_init(&bar[kBOdone], 1);
+        mbar_init(&bar[kBOfin], 1);
+        mbar_init(&bar[kBOa2], 128);
+        mbar_init(&bar[kBOut1], 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&bar[kBKfull + s], 1);
+            mbar_init(&bar[kBKempty + s], 1);
+            mbar_init(&bar[kBVfull + s], 32);
+            mbar_init(&bar[kBVempty + s], 1);
+            mbar_init(&bar[kBSfull + s], 1);
+            mbar_init(&bar[kBSfree + s], 128);
+            mbar_init(&bar[kBPfull + s], 128);
+            mbar_init(&bar[kBPfree + s], 1);
+        }
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) tmem_alloc(tslot, F::TM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------------------- producer
+        const char *wk = static_cast<const char *>(p.w_up_k) + wofs * RK * 2;
+        // W_up,t^K [d][r_k] as an MN-major operand: (row e, column chunk g) at g*(d*16) + e*16
+        for (int i = lane; i < D * F::NKC; i += 32) {
+            const int e = i / F::NKC, g = i - e * F::NKC;
+            cp_async16(sm + F::oWK + g * (D * 16) + e * 16, wk + (static_cast<int64_t>(e) * RK + g * 8) * 2);
+        }
+        cp_async_commit();
+        cp_async_wait_all();
+        fence_proxy_async_smem();
+        mbar_arrive(&bar[kBSetup]);
+        const uint64_t pol = policy_evict_first();
+        for (int j = 0; j < NP; ++j) {
+            const int s = j & 1;
+            const uint32_t ph = (j >> 1) & 1;
+            int32_t blk = bt[j];
+            if (blk < 0 || blk >= p.num_blocks) {
+                if (lane == 0) atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                blk = 0;
+            }
+            const char *page = p.pool + blk * p.block_bytes + static_cast<int64_t>(h) * p.head_page_bytes;
+            if (lane == 0) {
+                mbar_wait(&bar[kBKempty + s], ph ^ 1u, abort_flag, p.err);
+                mbar_arrive_expect_tx(&bar[kBKfull + s], F::KPAGE);
+                bulk_g2s(sm + F::oK + s * F::KPAGE, page, F::KPAGE, &bar[kBKfull + s], pol);
+            }
+            // the V ring aliases the prologue operands: wait until Q~ has been computed
+            if (j == 0) mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
+            mbar_wait(&bar[kBVempty + s], ph ^ 1u, abort_flag, p.err);
+            // V-plane [64][r_v] row-major -> MN-major operand: (token i, chunk g) at g*1024 + i*16
+            const char *vp = page + F::KPAGE;
+            char *vs = sm + F::oV + s * F::VPAGE;
+            const int valid = min(kPT, L - j * kPT);
+            for (int it = lane; it < kPT * F::NVC; it += 32) {
+                const int i = it / F::NVC, g = it - i * F::NVC;
+                char *dst = vs + g * (kPT * 16) + i * 16;
+                if (i < valid) cp_async16(dst, vp + (i * RV + g * 8) * 2);
+                else *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
+            }
+            cp_async_commit();
+            if (j > 0) {
+                cp_async_wait_but_one();
+                fence_proxy_async_smem();
+                mbar_arrive(&bar[kBVfull + ((j - 1) & 1)]);
+            }
+        }
+        cp_async_wait_all();
+        fence_proxy_async_smem();
+        mbar_arrive(&bar[kBVfull + ((NP - 1) & 1)]);
+        // epilogue operand W_up,t^V [d][r_v] (K-major): (row e, chunk c) at c*(d*16) + e*16,
+        // into the K ring once every MMA of the loop has completed
+        mbar_wait(&bar[kBOfin], 0, abort_flag, p.err);
+        const char *wv = static_cast<const char *>(p.w_up_v) + wofs * RV * 2;
+        for (int i = lane; i < D * F::NVC; i += 32) {
+            const int e = i / F::NVC, c = i - e * F::NVC;
+            cp_async16(sm + F::oWV + c * (D * 16) + e * 16, wv + (static_cast<int64_t>(e) * RV + c * 8) * 2);
+        }
+        cp_async_commit();
+        cp_async_wait_all();
+        fence_proxy_async_smem();
+        mbar_arrive(&bar[kBWv]);
+    } else if (warp == 1) {
+        // ------------------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t base = smem_addr(sm);
+            mbar_wait(&bar[kBSetup], 0, abort_flag, p.err);
+            tc_fence_after();
+            constexpr uint32_t idq = umma_idesc_bf16(128, RK, 0, 1);
+#pragma unroll 1
+            for (int ks = 0; ks < D / 16; ++ks)
+                umma_bf16(tmem + 0, umma_desc(base + F::oQA + ks * 4096, 2048, 128),
+                          umma_desc(base + F::oWK + ks * 256, 128, 2048), idq, ks > 0);
+            umma_commit(&bar[kBQt]);
+            mbar_wait(&bar[kBQs], 0, abort_flag, p.err);
+            tc_fence_after();
+            constexpr uint32_t ids = umma_idesc_bf16(128, kPT, 0, 0);
+            constexpr uint32_t idv = umma_idesc_bf16(128, F::NV, 0, 1);
+#pragma unroll 1
+            for (int j = 0; j <= NP; ++j) {
+                if (j < NP) {
+                    const int s = j & 1;
+                    mbar_wait(&bar[kBKfull + s], (j >> 1) & 1, abort_flag, p.err);
+                    if (j >= 2) mbar_wait(&bar[kBSfree + s], ((j - 2) >> 1) & 1, abort_flag, p.err);
+                    tc_fence_after();
+#pragma unroll 1
+                    for (int ks = 0; ks < RK / 16; ++ks)
+                        umma_bf16(tmem + F::TM_S + s * kPT,
+                                  umma_desc(base + F::oQT + ks * 4096, 2048, 128),
+                                  umma_desc(base + F::oK + s * F::KPAGE + ks * 2048, 1024, 128), ids,
+                                  ks > 0);
+                    umma_commit(&bar[kBSfull + s]);
+                    umma_commit(&bar[kBKempty + s]);
+                }
+                if (j >= 1) {
+                    const int jj = j - 1, s = jj & 1;
+                    mbar_wait(&bar[kBPfull + s], (jj >> 1) & 1, abort_flag, p.err);
+                    mbar_wait(&bar[kBVfull + s], (jj >> 1) & 1, abort_flag, p.err);
+                    tc_fence_after();
+#pragma unroll 1
+                    for (int sp = 0; sp < F::NSPL; ++sp)
+#pragma unroll 1
+                        for (int ks = 0; ks < kPT / 16; ++ks)
+                            umma_bf16(tmem + F::TM_O + sp * F::NV,
+                                      umma_desc(base + F::oP + s * F::PB + ks * 4096, 2048, 128),
+                                      umma_desc(base + F::oV + s * F::VPAGE + sp * (F::NV / 8) * 1024 +
+                                                    ks * 256,
+                                                128, 1024),
+                                      idv, jj > 0 || ks > 0);
+                    umma_commit(&bar[kBVempty + s]);
+                    umma_commit(&bar[kBPfree + s]);
+                    umma_commit(&bar[kBOdone]);
+                }
+            }
+            umma_commit(&bar[kBOfin]);  // every MMA of the loop has completed
+            // out = (O / l) W_up,t^V^T, with O / l = hi + lo as two bf16 operands in turn, so
+            // that the projection sees O / l to about 16 significant bits
+            mbar_wait(&bar[kBWv], 0, abort_flag, p.err);
+            constexpr uint32_t ido = umma_idesc_bf16(128, D, 0, 0);
+#pragma unroll 1
+            for (int part = 0; part < 2; ++part) {
+                mbar_wait(&bar[part ? kBOa2 : kBOa], 0, abort_flag, p.err);
+                tc_fence_after();
+#pragma unroll 1
+                for (int ks = 0; ks < RV / 16; ++ks)
+                    umma_bf16(tmem + 0, umma_desc(base + F::oOA + ks * 4096, 2048, 128),
+                              umma_desc(base + F::oWV + ks * 4096, 2048, 128), ido, part > 0 || ks > 0);
+                umma_commit(&bar[part ? kBOut : kBOut1]);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ softmax and epilogue
+        const int quarter = warp & 3;
+        const int row = quarter * 32 + lane;
+        const uint32_t tl = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        const int qi = i0 + row;
+        const bool valid_row = qi < L;
+        const int64_t qrow = (static_cast<int64_t>(q0) + qi) * p.H + h;
+        // q row -> bf16 K-major operand: chunk c at c*2048 + row*16
+        {
+            char *qa = sm + F::oQA + row * 16;
+            if (p.io_bf16) {
+                const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const char *>(p.q) + qrow * D * 2);
+#pragma unroll 4
+                for (int c = 0; c < D / 8; ++c)
+                    *reinterpret_cast<uint4 *>(qa + c * 2048) = valid_row ? src[c] : make_uint4(0, 0, 0, 0);
+            } else {
+                const float4 *src = reinterpret_cast<const float4 *>(static_cast<const char *>(p.q) + qrow * D * 4);
+#pragma unroll 4
+                for (int c = 0; c < D / 8; ++c) {
+                    float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b2 = a;
+                    if (valid_row) {
+                        a = src[2 * c];
+                        b2 = src[2 * c + 1];
+                    }
+                    *reinterpret_cast<uint4 *>(qa + c * 2048) =
+                        make_uint4(pack_bf16(a.x, a.y), pack_bf16(a.z, a.w), pack_bf16(b2.x, b2.y),
+                                   pack_bf16(b2.z, b2.w));
+                }
+            }
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(&bar[kBSetup]);
+        // q~ (scaled into the exp2 domain) -> bf16 K-major operand
+        mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
+        tc_fence_after();
+#pragma unroll 1
+        for (int c0 = 0; c0 < RK; c0 += 32) {
+            float v[32];
+            tmem_ld32(tl + c0, v);
+            char *qt_ = sm + F::oQT + row * 16;
+#pragma unroll
+            for (int k = 0; k < 32; k += 8) {
+                if (c0 + k < RK) {
+                    const float s = p.scale_log2;
+                    *reinterpret_cast<uint4 *>(qt_ + ((c0 + k) / 8) * 2048) =
+                        make_uint4(pack_bf16(v[k] * s, v[k + 1] * s), pack_bf16(v[k + 2] * s, v[k + 3] * s),
+                                   pack_bf16(v[k + 4] * s, v[k + 5] * s), pack_bf16(v[k + 6] * s, v[k + 7] * s));
+                }
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(&bar[kBQs]);
+
+        const int lim = min(qi, L - 1);  // keys 0..lim are visible to this row
+        float m = -INFINITY, l = 0.f;
+#pragma unroll 1
+        for (int j = 0; j < NP; ++j) {
+            const int s = j & 1;
+            mbar_wait(&bar[kBSfull + s], (j >> 1) & 1, abort_flag, p.err);
+            tc_fence_after();
+            float x[64];
+            {
+                float v[32];
+                tmem_ld32(tl + F::TM_S + s * kPT, v);
+#pragma unroll
+                for (int c = 0; c < 32; ++c) x[c] = v[c];
+                tmem_ld32(tl + F::TM_S + s * kPT + 32, v);
+#pragma unroll
+                for (int c = 0; c < 32; ++c) x[32 + c] = v[c];
+            }
+            tc_fence_before();
+            mbar_arrive(&bar[kBSfree + s]);
+            const int kb = j * kPT;
+            float mx = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+                x[c] = (kb + c <= lim) ? x[c] : -INFINITY;
+                mx = fmaxf(mx, x[c]);
+            }
+            const float m_new = fmaxf(m, mx);
+            const bool need = m_new > m + kRescaleLog2;  // also the first finite maximum
+            const float factor = need ? exp2f(m - m_new) : 1.f;
+            if (need) {
+                l *= factor;
+                m = m_new;
+            }
+            if (__any_sync(0xffffffffu, need && j > 0)) {
+                // O holds pages 0..j-1: wait for the last of them, then rescale this row
+                mbar_wait(&bar[kBOdone], (j - 1) & 1, abort_flag, p.err);
+                tc_fence_after();
+#pragma unroll 1
+                for (int c0 = 0; c0 < RV; c0 += 32) {
+                    float v[32];
+                    tmem_ld32(tl + F::TM_O + c0, v);
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) v[c] *= factor;
+                    tmem_st32(tl + F::TM_O + c0, v);
+                }
+            }
+            if (j >= 2) mbar_wait(&bar[kBPfree + s], ((j - 2) >> 1) & 1, abort_flag, p.err);
+            char *pr = sm + F::oP + s * F::PB + row * 16;
+#pragma unroll
+            for (int c = 0; c < 64; c += 8) {
+                uint32_t w[4];
+#pragma unroll
+                for (int k = 0; k < 8; k += 2) {
+                    const float a = m == -INFINITY ? 0.f : exp2f(x[c + k] - m);
+                    const float bb = m == -INFINITY ? 0.f : exp2f(x[c + k + 1] - m);
+                    w[k / 2] = pack_bf16(a, bb);
+                    l += __uint_as_float(w[k / 2] << 16) + __uint_as_float(w[k / 2] & 0xffff0000u);
+                }
+                *reinterpret_cast<uint4 *>(pr + (c / 8) * 2048) = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(&bar[kBPfull + s]);
+        }
+        // epilogue: O / l -> two bf16 K-major operands in turn (hi, then lo = O/l - hi) in one
+        // buffer that aliases the K ring; O stays in TMEM between the two
+        mbar_wait(&bar[kBOfin], 0, abort_flag, p.err);
+        tc_fence_after();
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll 1
+        for (int part = 0; part < 2; ++part) {
+            if (part) {
+                mbar_wait(&bar[kBOut1], 0, abort_flag, p.err);  // the hi product has read the buffer
+                tc_fence_after();
+            }
+#pragma unroll 1
+            for (int c0 = 0; c0 < RV; c0 += 32) {
+                float v[32];
+                tmem_ld32(tl + F::TM_O + c0, v);
+#pragma unroll
+                for (int k = 0; k < 32; ++k) {
+                    const float x = v[k] * inv;
+                    const float hi = __bfloat162float(__float2bfloat16_rn(x));
+                    v[k] = part ? x - hi : hi;
+                }
+                char *oa = sm + F::oOA + row * 16;
+#pragma unroll
+                for (int k = 0; k < 32; k += 8)
+                    *reinterpret_cast<uint4 *>(oa + ((c0 + k) / 8) * 2048) =
+                        make_uint4(pack_bf16(v[k], v[k + 1]), pack_bf16(v[k + 2], v[k + 3]),
+                                   pack_bf16(v[k + 4], v[k + 5]), pack_bf16(v[k + 6], v[k + 7]));
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(&bar[part ? kBOa2 : kBOa]);
+        }
+        mbar_wait(&bar[kBOut], 0, abort_flag, p.err);
+        tc_fence_after();
+        const float *muv = p.mu_v ? p.mu_v + wofs : nullptr;
+#pragma unroll 1
+        for (int c0 = 0; c0 < D; c0 += 32) {
+            float v[32];
+            tmem_ld32(tl + c0, v);
+            if (muv) {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) v[c] += muv[c0 + c];
+            }
+            if (valid_row) {
+                char *dst = static_cast<char *>(p.out) + (qrow * D + c0) * (p.io_bf16 ? 2 : 4);
+                if (p.io_bf16) {
+#pragma unroll
+                    for (int k = 0; k < 32; k += 8)
+                        *reinterpret_cast<uint4 *>(dst + k * 2) =
+                            make_uint4(pack_bf16(v[k], v[k + 1]), pack_bf16(v[k + 2], v[k + 3]),
+                                       pack_bf16(v[k + 4], v[k + 5]), pack_bf16(v[k + 6], v[k + 7]));
+                } else {
+#pragma unroll
+                    for (int k = 0; k < 32; k += 4)
+                        *reinterpret_cast<float4 *>(dst + k * 4) = make_float4(v[k], v[k + 1], v[k + 2], v[k + 3]);
+                }
+            }
+        }
+    }
+    pdl_trigger();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, F::TM_COLS);
+    }
+}
+
+// ------------------------------------------------------------------------- CUDA-core path
+
+struct GParams {
+    int T, H, d, r_k, r_v, loop, storage_bf16, io_bf16;
+    float scale_log2;
+    const void *w_up_k, *w_up_v;
+    const float *mu_v;
+    const char *pool;
+    int64_t num_blocks, block_bytes;
+    int head_page_bytes, kplane_bytes;
+    const int32_t *block_table;
+    int max_blocks;
+    const int32_t *cu_seqlens;
+    int max_len;
+    const void *q;
+    void *out;
+    unsigned *err;
+};
+
+constexpr int kGThreads = 128;
+constexpr int kGKeys = 128;  // keys per step
+
+// One CTA per (query, sequence, head), fp32 accumulation.  Shared memory: q [d], q~ [r_k],
+// o~ [r_v], p [kGKeys], reduction scratch.
+__global__ void __launch_bounds__(kGThreads) prefill_generic_kernel(const GParams p) {
+    extern __shared__ __align__(16) float gs[];
+    const int qi = blockIdx.x, b = blockIdx.y, h = blockIdx.z, tid = threadIdx.x;
+    pdl_wait();
+    const int q0 = p.cu_seqlens[b];
+    const int L = p.cu_seqlens[b + 1] - q0;
+    if (L > p.max_len || L < 0) {
+        if (tid == 0 && qi == 0) atomicOr(p.err, LLA_DEVERR_CONTEXT);
+        return;
+    }
+    if (qi >= L) return;
+    const int es = p.storage_bf16 ? 2 : 4;
+    float *qv = gs, *qt = qv + p.d, *ov = qt + p.r_k, *pv = ov + p.r_v, *red = pv + kGKeys;
+    const int64_t qrow = (static_cast<int64_t>(q0) + qi) * p.H + h;
+    const int64_t wofs = (static_cast<int64_t>(h) * p.T + p.loop) * p.d;
+    for (int e = tid; e < p.d; e += kGThreads) qv[e] = load_elem(p.q, qrow * p.d + e, p.io_bf16);
+    for (int j = tid; j < p.r_v; j += kGThreads) ov[j] = 0.f;
+    __syncthreads();
+    for (int j = tid; j < p.r_k; j += kGThreads) {  // q~ = W_up,t^K^T q
+        float acc = 0.f;
+        for (int e = 0; e < p.d; ++e)
+            acc = fmaf(load_elem(p.w_up_k, (wofs + e) * p.r_k + j, p.storage_bf16), qv[e], acc);
+        qt[j] = acc * p.scale_log2;
+    }
+    __syncthreads();
+    const int gk = granule_bytes(p.r_k, es);
+    const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks;
+    float m = -INFINITY, l = 0.f;
+    for (int k0 = 0; k0 <= qi; k0 += kGKeys) {
+        const int kj = k0 + tid;
+        float s = -INFINITY;
+        if (kj <= qi) {
+            int32_t blk = bt[kj / kPT];
+            if (blk < 0 || blk >= p.num_blocks) {
+                atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                blk = 0;
+            }
+            const char *page = p.pool + blk * p.block_bytes + static_cast<int64_t>(h) * p.head_page_bytes;
+            float acc = 0.f;
+            for (int j = 0; j < p.r_k; ++j) {
+                const char *e = page + kplane_offset(kj % kPT, j, es, gk);
+                acc = fmaf(qt[j], es == 2 ? bf_to_f(*reinterpret_cast<const uint16_t *>(e))
+                                          : *reinterpret_cast<const float *>(e), acc);
+            }
+            s = acc;
+        }
+        // block maximum
+        float mx = warp_max(s);
+        if ((tid & 31) == 0) red[tid >> 5] = mx;
+        __syncthreads();
+        mx = red[0];
+        for (int w = 1; w < kGThreads / 32; ++w) mx = fmaxf(mx, red[w]);
+        const float m_new = fmaxf(m, mx);
+        const float alpha = exp2f(m - m_new);
+        const float pj = kj <= qi ? exp2f(s - m_new) : 0.f;
+        pv[tid] = pj;
+        float ps = warp_sum(pj);
+        __syncthreads();  // every thread has read red[] for the maximum
+        if ((tid & 31) == 0) red[tid >> 5] = ps;
+        __syncthreads();
+        float psum = 0.f;
+        for (int w = 0; w < kGThreads / 32; ++w) psum += red[w];
+        l = l * alpha + psum;
+        m = m_new;
+        const int nk = min(kGKeys, qi + 1 - k0);
+        for (int j = tid; j < p.r_v; j += kGThreads) {
+            float acc = ov[j] * alpha;
+            for (int t = 0; t < nk; ++t) {
+                const int kk = k0 + t;
+                int32_t blk = bt[kk / kPT];
+                if (blk < 0 || blk >= p.num_blocks) blk = 0;
+                const char *e = p.pool + blk * p.block_bytes + static_cast<int64_t>(h) * p.head_page_bytes +
+                                p.kplane_bytes + (static_cast<int64_t>(kk % kPT) * p.r_v + j) * es;
+                acc = fmaf(pv[t], es == 2 ? bf_to_f(*reinterpret_cast<const uint16_t *>(e))
+                                          : *reinterpret_cast<const float *>(e), acc);
+            }
+            ov[j] = acc;
+        }
+        __syncthreads();
+    }
+    const float inv = 1.f / l;
+    for (int e = tid; e < p.d; e += kGThreads) {
+        float acc = 0.f;
+        for (int j = 0; j < p.r_v; ++j)
+            acc = fmaf(load_elem(p.w_up_v, (wofs + e) * p.r_v + j, p.storage_bf16), ov[j], acc);
+        float o = acc * inv;
+        if (p.mu_v) o += p.mu_v[wofs + e];
+        store_elem(p.out, qrow * p.d + e, o, p.io_bf16);
+    }
+    pdl_trigger();
+}
+
+template <typename K, typename P>
+lla_status launch_pf(K kern, dim3 grid, int threads, int smem, cudaStream_t stream, const P &prm) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, kern, prm) != cudaSuccess) return LLA_ERR_CUDA;
+    return LLA_OK;
+}
+
+template <int RK, int RV>
+lla_status launch_tc(const PParams &prm, int nqt, int B, int H, cudaStream_t stream) {
+    static bool configured[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
+    if (dev < 64 && !configured[dev]) {
+        if (cudaFuncSetAttribute(prefill_tc_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 PF<RK, RV>::SMEM) != cudaSuccess)
+            return LLA_ERR_CUDA;
+        configured[dev] = true;
+    }
+    return launch_pf(prefill_tc_kernel<RK, RV>, dim3(nqt, B, H), kPThreads, PF<RK, RV>::SMEM, stream, prm);
+}
+
+}  // namespace
+
+lla_status launch_prefill(const PrefillArgs &a, cudaStream_t stream) {
+    lla_status st = LLA_OK;
+    unsigned *err = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    const int es = a.storage_bf16 ? 2 : 4;
+    const int hpb = static_cast<int>(head_page_bytes(a.r_k, a.r_v, es));
+    if (a.B > 65535 || a.H > 65535) return LLA_ERR_UNSUPPORTED;
+    if (a.storage_bf16 && a.d == 128) {
+        PParams p = {};
+        p.T = a.T; p.H = a.H; p.loop = a.loop; p.io_bf16 = a.io_bf16;
+        p.scale_log2 = a.scale * kLog2e;
+        p.w_up_k = a.w_up_k; p.w_up_v = a.w_up_v; p.mu_v = a.mu_v;
+        p.pool = static_cast<const char *>(a.pool);
+        p.num_blocks = a.num_blocks;
+        p.head_page_bytes = hpb;
+        p.block_bytes = static_cast<int64_t>(hpb) * a.H;
+        p.block_table = a.block_table; p.max_blocks = a.max_blocks;
+        p.cu_seqlens = a.cu_seqlens; p.B = a.B; p.max_len = a.max_len;
+        p.q = a.q; p.out = a.out; p.err = err;
+        const int nqt = (a.max_len + kBM - 1) / kBM;
+#define LLA_PF(K, V) \
+        if (a.r_k == K && a.r_v == V) return launch_tc<K, V>(p, nqt, a.B, a.H, stream);
+        LLA_PF(96, 160)
+        LLA_PF(192, 320)
+        LLA_PF(128, 128)
+#undef LLA_PF
+    }
+    GParams g = {};
+    g.T = a.T; g.H = a.H; g.d = a.d; g.r_k = a.r_k; g.r_v = a.r_v; g.loop = a.loop;
+    g.storage_bf16 = a.storage_bf16; g.io_bf16 = a.io_bf16;
+    g.scale_log2 = a.scale * kLog2e;
+    g.w_up_k = a.w_up_k; g.w_up_v = a.w_up_v; g.mu_v = a.mu_v;
+    g.pool = static_cast<const char *>(a.pool);
+    g.num_blocks = a.num_blocks;
+    g.head_page_bytes = hpb;
+    g.block_bytes = static_cast<int64_t>(hpb) * a.H;
+    g.kplane_bytes = kPT * a.r_k * es;
+    g.block_table = a.block_table; g.max_blocks = a.max_blocks;
+    g.cu_seqlens = a.cu_seqlens; g.max_len = a.max_len;
+    g.q = a.q; g.out = a.out; g.err = err;
+    const int smem = (a.d + a.r_k + a.r_v + kGKeys + 32) * 4;
+    return launch_pf(prefill_generic_kernel, dim3(a.max_len, a.B, a.H), kGThreads, smem, stream, g);
+}
 
 }  // namespace lla
