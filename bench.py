@@ -46,6 +46,8 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0,
                    help="target CPU time of the oracle sample")
+    p.add_argument("--no-extras", action="store_true",
+                   help="skip the prefill, prefill-size encode and comparator measurements")
     return p.parse_args()
 
 
@@ -348,7 +350,134 @@ def run_ours(args, rank, world, local_rank):
         result["e2e"] = run_e2e(bench, args, world)
     if not args.no_cpu_baseline and rank == 0 and world == 1:
         result["cpu_baseline"] = cpu_baseline(bench.w, bench.lens, args.cpu_seconds)
+    if not args.no_extras and rank == 0:
+        del bench
+        torch.cuda.empty_cache()
+        result.update(run_extras(device))
     return result
+
+
+def _time_ms(fn, reps=5, warm=2):
+    """Best of `reps` CUDA-event timings of fn() on the current stream, after `warm` calls."""
+    import torch
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    best = float("inf")
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        fn()
+        b.record()
+        torch.cuda.synchronize()
+        best = min(best, a.elapsed_time(b))
+    return best
+
+
+def run_extras(device):
+    """The other rows of the hot path on their own workloads, each against its roofline:
+    causal prefill attention and the encode of a prefilled prompt (Ouro-1.4B at rho = 2,
+    4 prompts of 8192 tokens, one layer and loop per call), and the uncompressed loop-t decode
+    comparator on the headline batch (D x T calls over plain K/V pages of d = 128)."""
+    import torch
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except Exception:
+        pass
+    tc_peak = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    out = {}
+
+    # prefill: ouro14_rho2, 4 x 8192 tokens
+    w = W.WORKLOADS["ouro14_rho2"]
+    nseq, L = w.prefill
+    T, H, d = w.T, w.H, w.d
+    geom = lla.Geometry(T, H, d, w.r_k, w.r_v, "bf16")
+    codec = lla.Codec(**W.codec_tensors(T, H, d, w.r_k, w.r_v, w.seed, 0, device=device))
+    lens = [L] * nseq
+    pt = W.page_table(lens, w.seed, extra_tokens=0)
+    pool = torch.zeros(pt.num_blocks * lla.lla_cache_block_bytes(geom), dtype=torch.uint8, device=device)
+    cache = lla.Cache(pool, pt.num_blocks, pt.block_table.to(device), pt.max_blocks)
+    N = nseq * L
+    slots = torch.cat([pt.slots(b, range(L)) for b in range(nseq)]).to(device)
+    xk = W.normal((T, N, H, d), w.seed, 300, device=device)
+    xv = W.normal((T, N, H, d), w.seed, 301, device=device)
+    enc_ms = _time_ms(lambda: lla.lla_encode(geom, codec, cache, xk, xv, slots), reps=3, warm=1)
+    enc_bytes = 2 * xk.numel() * 2 + H * T * d * (w.r_k + w.r_v) * 2 + N * H * (w.r_k + w.r_v) * 2
+    enc_flops = 2.0 * N * H * T * d * (w.r_k + w.r_v)
+    out["encode_prefill"] = {
+        "workload": f"{w.name} prompt encode, {nseq}x{L} tokens, H={H}, (r_k, r_v)=({w.r_k}, {w.r_v})",
+        "kernel": "encode_kernel (lla_encode)", "ms_per_call": enc_ms,
+        "GB_s": enc_bytes / (enc_ms / 1e3) / 1e9, "hbm_frac": enc_bytes / (enc_ms / 1e3) / 1e9 / hbm,
+        "TFLOP_s": enc_flops / (enc_ms / 1e3) / 1e12,
+        "tensor_frac": enc_flops / (enc_ms / 1e3) / 1e12 / tc_peak,
+        "bytes_per_call": enc_bytes, "flops_per_call": enc_flops}
+    del xk, xv
+    q = W.normal((N, H, d), w.seed, 302, device=device)
+    o = torch.empty_like(q)
+    cu = torch.tensor([i * L for i in range(nseq + 1)], dtype=torch.int32, device=device)
+    pf_ms = _time_ms(lambda: lla.lla_prefill_attn(geom, codec, cache, cu, L, 1, q, o))
+    pairs = nseq * H * L * (L + 1) / 2
+    pf_flops = pairs * 2 * (w.r_k + w.r_v) + N * H * 2 * d * (w.r_k + w.r_v)
+    out["prefill"] = {
+        "workload": f"{w.name} causal prefill, {nseq}x{L} tokens, H={H}, one layer and loop",
+        "kernel": "prefill_tc_kernel (lla_prefill_attn)", "bound": "tensor",
+        "ms_per_call": pf_ms, "tokens_per_s": N / (pf_ms / 1e3),
+        "TFLOP_s": pf_flops / (pf_ms / 1e3) / 1e12, "peak_TFLOP_s": tc_peak,
+        "frac": pf_flops / (pf_ms / 1e3) / 1e12 / tc_peak,
+        "peak_source": "measured sustained cuBLAS bf16 (MEASURED_PEAKS.json bf16_tflops_sustained)",
+        "flops_per_call": pf_flops}
+    del q, o, pool, cache
+
+    # comparator: plain loop-t K/V of the headline batch, d = 128
+    w = W.WORKLOADS["ouro14_rho4"]
+    lens = W.context_lengths(w)
+    B = len(lens)
+    dgeom = lla.Geometry(1, w.H, w.d, w.d, w.d, "bf16")
+    pt = W.page_table(lens, w.seed, extra_tokens=1)
+    table = pt.block_table.to(device)
+    Nt = sum(lens)
+    slots = torch.cat([pt.slots(b, range(Lb)) for b, Lb in enumerate(lens)]).to(device)
+    caches = []
+    for t in range(w.T):  # the teacher cache holds every loop's keys and values
+        pool = torch.empty(pt.num_blocks * lla.lla_cache_block_bytes(dgeom), dtype=torch.uint8, device=device)
+        cache = lla.Cache(pool, pt.num_blocks, table, pt.max_blocks)
+        k = W.normal((Nt, w.H, w.d), w.seed, 310, t, device=device)
+        v = W.normal((Nt, w.H, w.d), w.seed, 311, t, device=device)
+        lla.lla_dense_store(dgeom, cache, k, v, slots)
+        caches.append((pool, cache))
+        del k, v
+    ctx = torch.tensor(lens, dtype=torch.int32, device=device)
+    qs = W.normal((w.T, B, w.H, w.d), w.seed, 312, device=device)
+    cks = W.normal((w.T, B, w.H, w.d), w.seed, 313, device=device)
+    cvs = W.normal((w.T, B, w.H, w.d), w.seed, 314, device=device)
+    os_ = torch.empty_like(qs)
+    ws = torch.zeros(lla.lla_decode_workspace_size(dgeom, B), dtype=torch.uint8, device=device)
+
+    def sweep():
+        for _ in range(w.D):
+            for t in range(w.T):
+                lla.lla_dense_decode_attn(dgeom, caches[t][1], ctx, max(lens), qs[t], cks[t], cvs[t],
+                                          os_[t], ws)
+    cmp_ms = _time_ms(sweep, reps=3, warm=1)
+    per_launch = cmp_ms / (w.D * w.T)
+    cbytes = Nt * w.H * 2 * w.d * 2 + 4 * B * w.H * w.d * 2
+    out["comparator"] = {
+        "workload": f"{w.name} batch, uncompressed loop-t K/V (d={w.d}), {w.D}x{w.T} calls per step",
+        "kernel": "decode_async_kernel<2,128,128> (lla_dense_decode_attn)",
+        "tokens_per_s": B / (cmp_ms / 1e3), "ms_per_step_decode_only": cmp_ms,
+        "avg_launch_us": per_launch * 1e3, "GB_s": cbytes / (per_launch / 1e3) / 1e9,
+        "hbm_frac": cbytes / (per_launch / 1e3) / 1e9 / hbm, "bytes_per_launch": cbytes,
+        "note": "same bytes per call as the latent cache at rho = 4 (2d = r_k + r_v); the "
+                "teacher cache of the whole model is rho times the latent cache"}
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the extra measurements")
+    return out
 
 
 def run_e2e(bench, args, world):

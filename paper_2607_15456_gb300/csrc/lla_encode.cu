@@ -290,6 +290,7 @@ lla_status set_smem(int dev) {
 
 lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream) {
     if (a.N == 0) return LLA_OK;
+    if (encode_tc_supported(a)) return launch_encode_tc(a, stream);
     const int es = a.storage_bf16 ? 2 : 4;
     lla_status st = LLA_OK;
     unsigned *err = device_error_word(&st);

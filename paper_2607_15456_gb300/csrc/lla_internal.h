@@ -72,6 +72,9 @@ lla_status decode_fits(int r_k, int r_v, int es, int d);  // UNSUPPORTED if no k
 lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream);
 
 lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream);
+// Tensor-core encode for prompts (bf16 x and storage, N >= 128, instantiated ranks).
+bool encode_tc_supported(const EncodeArgs &a);
+lla_status launch_encode_tc(const EncodeArgs &a, cudaStream_t stream);
 lla_status launch_prefill(const PrefillArgs &a, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached), 0 on failure

@@ -25,6 +25,32 @@ __device__ __forceinline__ uint64_t umma_desc(uint32_t smem_byte_addr, uint32_t 
     return d;
 }
 
+// Shared-memory matrix descriptor for 128-byte swizzled operands, as a TMA load with 128-byte
+// swizzle writes them: rows of 128 bytes whose 16-byte chunks are permuted by (row % 8), in
+// 1024-byte atoms of 8 rows (1024-byte aligned).
+//   K-major:  rows along M/N hold 64 K elements; next 8 rows at +1024; a K step of 16 elements
+//             moves the start address by 32 bytes.
+//   MN-major: rows along K hold 64 M/N elements; next 8 K rows at +1024; the next 64 M/N
+//             elements at +mn_atom_stride; a K step of 16 rows moves the start by 2048.
+__device__ __forceinline__ uint64_t umma_desc_sw128_k(uint32_t smem_byte_addr) {
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((smem_byte_addr >> 4) & 0x3FFFu);
+    d |= static_cast<uint64_t>(1) << 16;                  // leading offset unused (16 bytes)
+    d |= static_cast<uint64_t>(1024 >> 4) << 32;          // 8-row atoms
+    d |= static_cast<uint64_t>(1) << 46;
+    d |= static_cast<uint64_t>(2) << 61;                  // 128-byte swizzle
+    return d;
+}
+__device__ __forceinline__ uint64_t umma_desc_sw128_mn(uint32_t smem_byte_addr, uint32_t mn_atom_stride) {
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((smem_byte_addr >> 4) & 0x3FFFu);
+    d |= static_cast<uint64_t>((mn_atom_stride >> 4) & 0x3FFFu) << 16;
+    d |= static_cast<uint64_t>(1024 >> 4) << 32;
+    d |= static_cast<uint64_t>(1) << 46;
+    d |= static_cast<uint64_t>(2) << 61;
+    return d;
+}
+
 // Instruction descriptor of kind::f16 with bf16 A and B and an fp32 accumulator.
 // a_mn / b_mn: 0 = K-major, 1 = MN-major.
 __host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N, int a_mn, int b_mn) {
@@ -116,6 +142,29 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     const uint32_t a = __bfloat16_as_ushort(__float2bfloat16_rn(lo));
     const uint32_t b = __bfloat16_as_ushort(__float2bfloat16_rn(hi));
     return a | (b << 16);
+}
+
+}  // namespace lla
+
+namespace lla {
+
+// Tiled TMA loads (tensor map in a __grid_constant__ kernel parameter) completing on `bar`.
+__device__ __forceinline__ void tma_load_3d(void *dst, const void *tmap, int c0, int c1, int c2,
+                                            uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(
+            smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_addr(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d(void *dst, const void *tmap, int c0, int c1, int c2,
+                                            int c3, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(
+            smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_addr(bar))
+        : "memory");
 }
 
 }  // namespace lla

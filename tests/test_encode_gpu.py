@@ -5,7 +5,8 @@ compared with oracle.encode on the same inputs (bf16 storage: max abs <= 2e-2 an
 L2 <= 5e-3; fp32 storage and fp32 x: relative L2 <= 1e-5).  The cases reach the kernel's
 separate code paths: a reduction axis T*d longer than one shared-memory chunk of W_down (fp32
 and bf16), ranks whose rows are not a multiple of 16 bytes (4-byte copies), token counts that
-leave a ragged last tile, x in bf16 and fp32, with and without mu, and a decode-step batch.
+leave a ragged last tile, x in bf16 and fp32, with and without mu, a decode-step batch, and
+prompts of 128 tokens or more in bf16, which take the tensor-core kernel.
 """
 import pytest
 import torch
@@ -83,3 +84,14 @@ def test_encode_fp32_small_ranks(lla):
 def test_encode_decode_step_batch(lla):
     # the decode-step shape: one completed token for each of 16 sequences, all 16 heads
     _encode_and_compare(lla, 4, 16, 128, 96, 160, "bf16", "bf16", [1] * 16, False, 6)
+
+
+@pytest.mark.parametrize("r_k,r_v,with_mu", [(96, 160, True), (192, 320, False), (128, 128, True)])
+def test_encode_prompt_on_tensor_cores(lla, r_k, r_v, with_mu):
+    # 300 tokens in three sequences: three tiles of 128 tokens, the last one ragged (44 tokens)
+    _encode_and_compare(lla, 4, 3, 128, r_k, r_v, "bf16", "bf16", [130, 101, 69], with_mu, 7)
+
+
+def test_encode_prompt_long_reduction_on_tensor_cores(lla):
+    # T*d = 16 * 256 = 4096: 64 slabs of the reduction axis through the stage ring
+    _encode_and_compare(lla, 16, 2, 256, 96, 160, "bf16", "bf16", [150], True, 8)
