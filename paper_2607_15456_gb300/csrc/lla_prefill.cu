@@ -7,21 +7,24 @@
 //   s_ij = scale * q~_i . c_k,j,   p_i = softmax_j<=i(s_i)
 //   o_i  = W_up,t^V (sum_j p_ij c_v,j) + mu^V_t
 //
-// Tensor-core path (bf16 storage, d = 128, r_k and r_v multiples of 16): one CTA per
+// Tensor-core path (bf16 storage, d = 128, r_k and r_v multiples of 32): one CTA per
 // (128-query tile, sequence, head) and four warp roles.
 //   warp 0      producer: W_up,t^K into shared memory (cp.async), then per page of 64 keys the
 //               K-plane (one bulk copy: its granule-interleaved layout is already the
-//               core-matrix layout of a K-major MMA operand) and the V-plane (16-byte cp.async
-//               gathers into an MN-major core-matrix layout; rows past the prompt are zeroed),
-//               and W_up,t^V for the epilogue
+//               core-matrix layout of a K-major MMA operand) and the V-plane (one TMA tensor
+//               load with 128-byte swizzle per 64 latent columns: an MN-major operand), and
+//               W_up,t^V for the epilogue
 //   warp 1      MMA issuer (one thread) and TMEM owner:
 //                 Q~ = Q W_up,t^K             M=128, N=r_k, K=d
 //                 S_j = Q~ C_k,j^T            M=128, N=64,  K=r_k   (one page ahead of PV)
 //                 O += P_j C_v,j              M=128, N=r_v (split at 256), K=64
 //                 out = (O/l) W_up,t^V^T      M=128, N=d,   K=r_v
-//   warps 2-5   one query row per thread: Q and Q~ into bf16 operands, causal mask and online
-//               softmax in the exp2 domain, P into a bf16 operand, O rescaled in TMEM only when
-//               a row maximum grows by more than 2^8, then the epilogue.
+//   warps 2-9   two threads per query row, each with 32 keys of every page (warps w and w + 4
+//               share TMEM lanes): Q and Q~ into bf16 operands, causal mask on diagonal pages,
+//               online softmax in the exp2 domain with the row maximum exchanged through shared
+//               memory, P into a bf16 operand, O rescaled in TMEM only when a row maximum grows
+//               by more than 2^8, V rows past the prompt zeroed on its last page, then the
+//               epilogue.
 // Accumulators are fp32 in TMEM; operands are bf16 (q~ carries scale * log2 e).
 //
 // CUDA-core path (fp32 storage, other ranks, d != 128): one CTA per (query, sequence, head),
@@ -31,13 +34,16 @@
 #include "lla_device.cuh"
 #include "lla_internal.h"
 #include "lla_tcgen05.cuh"
+#include "lla_tmap.h"
 
 namespace lla {
 namespace {
 
-constexpr int kBM = 128;        // queries per tile
-constexpr int kPT = 64;         // keys per page
-constexpr int kPThreads = 192;  // producer, MMA, 4 softmax warps
+constexpr int kBM = 128;         // queries per tile
+constexpr int kPT = 64;          // keys per page
+constexpr int kSWarps = 8;       // softmax warps: two threads per query row
+constexpr int kPThreads = 64 + kSWarps * 32;
+constexpr int kSThreads = kSWarps * 32;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when a row maximum grows by more
 
@@ -58,16 +64,18 @@ struct PParams {
     unsigned *err;
 };
 
-// Shared-memory plan of the tensor-core kernel for ranks (RK, RV); d = 128.
+// Shared-memory plan of the tensor-core kernel for ranks (RK, RV); d = 128.  Offsets are
+// multiples of 1024 bytes from a 1024-byte aligned base (128-byte swizzle atoms).
 template <int RK, int RV>
 struct PF {
     static constexpr int D = 128;
     static constexpr int NKC = RK / 8;               // 16-byte chunks of a K row
     static constexpr int NVC = RV / 8;               // 16-byte chunks of a V row
-    static constexpr int NSPL = RV > 256 ? 2 : 1;    // PV MMAs per K step (N <= 256)
-    static constexpr int NV = RV / NSPL;
+    static constexpr int VATOMS = (RV + 63) / 64;    // 64-column atoms of a V page (TMA boxes)
+    static constexpr int N0 = RV > 256 ? 256 : RV;   // PV MMA split on atom boundaries
+    static constexpr int N1 = RV - N0;
     static constexpr int KPAGE = kPT * RK * 2;
-    static constexpr int VPAGE = kPT * RV * 2;
+    static constexpr int VPAGE = VATOMS * kPT * 128;
     static constexpr int QT = kBM * RK * 2;          // q~ operand
     static constexpr int PB = kBM * kPT * 2;         // P operand (one of two)
     static constexpr int QA = kBM * D * 2;           // q operand (prologue)
@@ -83,13 +91,16 @@ struct PF {
     // the prologue operands alias the V ring and P; the epilogue operands alias K, V and P
     static constexpr int oQA = oV, oWK = oV + QA;
     static constexpr int oOA = oK, oWV = oK + OA;
-    static constexpr int oBar = oEnd;
+    static constexpr int oX = oEnd;                   // [2 pages][2 halves][128 rows] maxima
+    static constexpr int oL = oX + 2 * 2 * kBM * 4;   // [2 halves][128 rows] row sums
+    static constexpr int oBar = oL + 2 * kBM * 4;
     static constexpr int NBAR = 32;
-    static constexpr int SMEM = oBar + NBAR * 8 + 16;
+    static constexpr int SMEM = 1024 + oBar + NBAR * 8 + 16;
     // TMEM columns: S double buffer [0, 128), O [128, 128 + RV); q~ and out reuse [0, ...)
     static constexpr uint32_t TM_S = 0, TM_O = 128, TM_COLS = 512;
-    static_assert(RK % 16 == 0 && RV % 16 == 0 && RK <= 256 && 128 + RV <= 512, "ranks");
-    static_assert(NV % 16 == 0 && NV <= 256, "PV split");
+    static_assert(RK % 32 == 0 && RV % 32 == 0 && RK <= 256 && 128 + RV <= 512, "ranks");
+    static_assert(N0 % 16 == 0 && N1 % 16 == 0 && N1 <= 256, "PV split");
+    static_assert(oK % 1024 == 0 && oV % 1024 == 0 && oP % 1024 == 0 && VPAGE % 1024 == 0, "align");
     static_assert(oWK + WK <= oEnd && oWV + WV <= oEnd, "aliased operands fit");
     static_assert(SMEM <= 227 * 1024, "shared memory");
 };
@@ -97,20 +108,24 @@ struct PF {
 // barrier indices
 enum {
     kBSetup = 0, kBQt, kBQs, kBOa, kBWv, kBOut, kBOdone, kBOfin,
-    kBOa2 = 24, kBOut1 = 25,
     kBKfull = 8 /* [2] */, kBKempty = 10, kBVfull = 12, kBVempty = 14,
     kBSfull = 16, kBSfree = 18, kBPfull = 20, kBPfree = 22,
+    kBOa2 = 24, kBOut1 = 25,
     kBAbort = 31  // slot used as the CTA's abort flag
 };
 
 template <int RK, int RV>
-__global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams p) {
+__global__ void __launch_bounds__(kPThreads, 1)
+    prefill_tc_kernel(const __grid_constant__ CUtensorMap tv, const PParams p) {
     using F = PF<RK, RV>;
     constexpr int D = F::D;
-    extern __shared__ __align__(1024) char sm[];
+    extern __shared__ __align__(1024) char sm_raw[];
+    char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + F::oBar);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(bar + kBAbort);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + F::NBAR);
+    float *xmax = reinterpret_cast<float *>(sm + F::oX);
+    float *xsum = reinterpret_cast<float *>(sm + F::oL);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
     const int nqt = (p.max_len + kBM - 1) / kBM;
@@ -131,24 +146,24 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
     const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks;
 
     if (tid == 0) {
-        mbar_init(&bar[kBSetup], 32 + 128);
+        mbar_init(&bar[kBSetup], 32 + kSThreads);
         mbar_init(&bar[kBQt], 1);
-        mbar_init(&bar[kBQs], 128);
-        mbar_init(&bar[kBOa], 128);
+        mbar_init(&bar[kBQs], kSThreads);
+        mbar_init(&bar[kBOa], kSThreads);
+        mbar_init(&bar[kBOa2], kSThreads);
         mbar_init(&bar[kBWv], 32);
+        mbar_init(&bar[kBOut1], 1);
         mbar_init(&bar[kBOut], 1);
         mbar_init(&bar[kBOdone], 1);
         mbar_init(&bar[kBOfin], 1);
-        mbar_init(&bar[kBOa2], 128);
-        mbar_init(&bar[kBOut1], 1);
         for (int s = 0; s < 2; ++s) {
             mbar_init(&bar[kBKfull + s], 1);
             mbar_init(&bar[kBKempty + s], 1);
-            mbar_init(&bar[kBVfull + s], 32);
+            mbar_init(&bar[kBVfull + s], 1);
             mbar_init(&bar[kBVempty + s], 1);
             mbar_init(&bar[kBSfull + s], 1);
-            mbar_init(&bar[kBSfree + s], 128);
-            mbar_init(&bar[kBPfull + s], 128);
+            mbar_init(&bar[kBSfree + s], kSThreads);
+            mbar_init(&bar[kBPfull + s], kSThreads);
             mbar_init(&bar[kBPfree + s], 1);
         }
         *abort_flag = 0;
@@ -172,44 +187,32 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
         cp_async_wait_all();
         fence_proxy_async_smem();
         mbar_arrive(&bar[kBSetup]);
-        const uint64_t pol = policy_evict_first();
-        for (int j = 0; j < NP; ++j) {
-            const int s = j & 1;
-            const uint32_t ph = (j >> 1) & 1;
-            int32_t blk = bt[j];
-            if (blk < 0 || blk >= p.num_blocks) {
-                if (lane == 0) atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
-                blk = 0;
-            }
-            const char *page = p.pool + blk * p.block_bytes + static_cast<int64_t>(h) * p.head_page_bytes;
-            if (lane == 0) {
+        if (lane == 0) {
+            const uint64_t pol = policy_evict_first();
+            for (int j = 0; j < NP; ++j) {
+                const int s = j & 1;
+                const uint32_t ph = (j >> 1) & 1;
+                int32_t blk = bt[j];
+                if (blk < 0 || blk >= p.num_blocks) {
+                    atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                    blk = 0;
+                }
+                const int64_t hp = static_cast<int64_t>(blk) * p.H + h;  // head page index
                 mbar_wait(&bar[kBKempty + s], ph ^ 1u, abort_flag, p.err);
                 mbar_arrive_expect_tx(&bar[kBKfull + s], F::KPAGE);
-                bulk_g2s(sm + F::oK + s * F::KPAGE, page, F::KPAGE, &bar[kBKfull + s], pol);
-            }
-            // the V ring aliases the prologue operands: wait until Q~ has been computed
-            if (j == 0) mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
-            mbar_wait(&bar[kBVempty + s], ph ^ 1u, abort_flag, p.err);
-            // V-plane [64][r_v] row-major -> MN-major operand: (token i, chunk g) at g*1024 + i*16
-            const char *vp = page + F::KPAGE;
-            char *vs = sm + F::oV + s * F::VPAGE;
-            const int valid = min(kPT, L - j * kPT);
-            for (int it = lane; it < kPT * F::NVC; it += 32) {
-                const int i = it / F::NVC, g = it - i * F::NVC;
-                char *dst = vs + g * (kPT * 16) + i * 16;
-                if (i < valid) cp_async16(dst, vp + (i * RV + g * 8) * 2);
-                else *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
-            }
-            cp_async_commit();
-            if (j > 0) {
-                cp_async_wait_but_one();
-                fence_proxy_async_smem();
-                mbar_arrive(&bar[kBVfull + ((j - 1) & 1)]);
+                bulk_g2s(sm + F::oK + s * F::KPAGE, p.pool + hp * p.head_page_bytes, F::KPAGE,
+                         &bar[kBKfull + s], pol);
+                // the V ring aliases the prologue operands: wait until Q~ has been computed
+                if (j == 0) mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
+                mbar_wait(&bar[kBVempty + s], ph ^ 1u, abort_flag, p.err);
+                mbar_arrive_expect_tx(&bar[kBVfull + s], F::VPAGE);
+                char *vs = sm + F::oV + s * F::VPAGE;
+#pragma unroll
+                for (int a = 0; a < F::VATOMS; ++a)
+                    tma_load_3d(vs + a * (kPT * 128), &tv, a * 64, 0, static_cast<int>(hp), &bar[kBVfull + s]);
             }
         }
-        cp_async_wait_all();
-        fence_proxy_async_smem();
-        mbar_arrive(&bar[kBVfull + ((NP - 1) & 1)]);
+        __syncwarp();
         // epilogue operand W_up,t^V [d][r_v] (K-major): (row e, chunk c) at c*(d*16) + e*16,
         // into the K ring once every MMA of the loop has completed
         mbar_wait(&bar[kBOfin], 0, abort_flag, p.err);
@@ -237,7 +240,8 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
             mbar_wait(&bar[kBQs], 0, abort_flag, p.err);
             tc_fence_after();
             constexpr uint32_t ids = umma_idesc_bf16(128, kPT, 0, 0);
-            constexpr uint32_t idv = umma_idesc_bf16(128, F::NV, 0, 1);
+            constexpr uint32_t idv0 = umma_idesc_bf16(128, F::N0, 0, 1);
+            constexpr uint32_t idv1 = umma_idesc_bf16(128, F::N1 > 0 ? F::N1 : 16, 0, 1);
 #pragma unroll 1
             for (int j = 0; j <= NP; ++j) {
                 if (j < NP) {
@@ -259,16 +263,17 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
                     mbar_wait(&bar[kBPfull + s], (jj >> 1) & 1, abort_flag, p.err);
                     mbar_wait(&bar[kBVfull + s], (jj >> 1) & 1, abort_flag, p.err);
                     tc_fence_after();
+                    const uint32_t vb = base + F::oV + s * F::VPAGE;
 #pragma unroll 1
-                    for (int sp = 0; sp < F::NSPL; ++sp)
-#pragma unroll 1
-                        for (int ks = 0; ks < kPT / 16; ++ks)
-                            umma_bf16(tmem + F::TM_O + sp * F::NV,
-                                      umma_desc(base + F::oP + s * F::PB + ks * 4096, 2048, 128),
-                                      umma_desc(base + F::oV + s * F::VPAGE + sp * (F::NV / 8) * 1024 +
-                                                    ks * 256,
-                                                128, 1024),
-                                      idv, jj > 0 || ks > 0);
+                    for (int ks = 0; ks < kPT / 16; ++ks) {
+                        const uint64_t da = umma_desc(base + F::oP + s * F::PB + ks * 4096, 2048, 128);
+                        umma_bf16(tmem + F::TM_O, da, umma_desc_sw128_mn(vb + ks * 2048, kPT * 128), idv0,
+                                  jj > 0 || ks > 0);
+                        if constexpr (F::N1 > 0)
+                            umma_bf16(tmem + F::TM_O + F::N0, da,
+                                      umma_desc_sw128_mn(vb + (F::N0 / 64) * (kPT * 128) + ks * 2048, kPT * 128),
+                                      idv1, jj > 0 || ks > 0);
+                    }
                     umma_commit(&bar[kBVempty + s]);
                     umma_commit(&bar[kBPfree + s]);
                     umma_commit(&bar[kBOdone]);
@@ -293,123 +298,154 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
         __syncwarp();
     } else {
         // ------------------------------------------------------------ softmax and epilogue
+        // warps 2..9: quarter (TMEM lanes) = warp % 4, half = which 32 keys of a page (and which
+        // half of every other row-wise job) this thread owns; warps w and w + 4 share rows
         const int quarter = warp & 3;
+        const int half = (warp - 2) >> 2;
         const int row = quarter * 32 + lane;
+        const int pair_bar = 2 + quarter;  // named barrier of the two warps of this quarter
         const uint32_t tl = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
         const int qi = i0 + row;
         const bool valid_row = qi < L;
         const int64_t qrow = (static_cast<int64_t>(q0) + qi) * p.H + h;
-        // q row -> bf16 K-major operand: chunk c at c*2048 + row*16
+        // q row (this half's 64 elements) -> bf16 K-major operand: chunk c at c*2048 + row*16
         {
             char *qa = sm + F::oQA + row * 16;
+            const int c0 = half * (D / 16);
             if (p.io_bf16) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const char *>(p.q) + qrow * D * 2);
-#pragma unroll 4
-                for (int c = 0; c < D / 8; ++c)
+#pragma unroll
+                for (int c = c0; c < c0 + D / 16; ++c)
                     *reinterpret_cast<uint4 *>(qa + c * 2048) = valid_row ? src[c] : make_uint4(0, 0, 0, 0);
             } else {
                 const float4 *src = reinterpret_cast<const float4 *>(static_cast<const char *>(p.q) + qrow * D * 4);
-#pragma unroll 4
-                for (int c = 0; c < D / 8; ++c) {
+#pragma unroll
+                for (int c = c0; c < c0 + D / 16; ++c) {
                     float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b2 = a;
                     if (valid_row) {
                         a = src[2 * c];
                         b2 = src[2 * c + 1];
                     }
                     *reinterpret_cast<uint4 *>(qa + c * 2048) =
-                        make_uint4(pack_bf16(a.x, a.y), pack_bf16(a.z, a.w), pack_bf16(b2.x, b2.y),
-                                   pack_bf16(b2.z, b2.w));
+                        make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w), pack_bf16x2(b2.x, b2.y),
+                                   pack_bf16x2(b2.z, b2.w));
                 }
             }
         }
         fence_proxy_async_smem();
         mbar_arrive(&bar[kBSetup]);
-        // q~ (scaled into the exp2 domain) -> bf16 K-major operand
+        // q~ (scaled into the exp2 domain) -> bf16 K-major operand; this half's RK/2 columns
         mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
         tc_fence_after();
 #pragma unroll 1
-        for (int c0 = 0; c0 < RK; c0 += 32) {
-            float v[32];
-            tmem_ld32(tl + c0, v);
+        for (int c0 = half * (RK / 2); c0 < (half + 1) * (RK / 2); c0 += 16) {
+            float v[16];
+            tmem_ld16(tl + c0, v);
             char *qt_ = sm + F::oQT + row * 16;
+            const float sc = p.scale_log2;
 #pragma unroll
-            for (int k = 0; k < 32; k += 8) {
-                if (c0 + k < RK) {
-                    const float s = p.scale_log2;
-                    *reinterpret_cast<uint4 *>(qt_ + ((c0 + k) / 8) * 2048) =
-                        make_uint4(pack_bf16(v[k] * s, v[k + 1] * s), pack_bf16(v[k + 2] * s, v[k + 3] * s),
-                                   pack_bf16(v[k + 4] * s, v[k + 5] * s), pack_bf16(v[k + 6] * s, v[k + 7] * s));
-                }
-            }
+            for (int k = 0; k < 16; k += 8)
+                *reinterpret_cast<uint4 *>(qt_ + ((c0 + k) / 8) * 2048) =
+                    make_uint4(pack_bf16x2(v[k] * sc, v[k + 1] * sc), pack_bf16x2(v[k + 2] * sc, v[k + 3] * sc),
+                               pack_bf16x2(v[k + 4] * sc, v[k + 5] * sc), pack_bf16x2(v[k + 6] * sc, v[k + 7] * sc));
         }
         fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(&bar[kBQs]);
 
         const int lim = min(qi, L - 1);  // keys 0..lim are visible to this row
+        const int kofs = half * 32;      // this thread's keys within a page
         float m = -INFINITY, l = 0.f;
 #pragma unroll 1
         for (int j = 0; j < NP; ++j) {
             const int s = j & 1;
+            const int kb = j * kPT;
             mbar_wait(&bar[kBSfull + s], (j >> 1) & 1, abort_flag, p.err);
             tc_fence_after();
-            float x[64];
-            {
-                float v[32];
-                tmem_ld32(tl + F::TM_S + s * kPT, v);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) x[c] = v[c];
-                tmem_ld32(tl + F::TM_S + s * kPT + 32, v);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) x[32 + c] = v[c];
-            }
+            float x[32];
+            tmem_ld32(tl + F::TM_S + s * kPT + kofs, x);
             tc_fence_before();
             mbar_arrive(&bar[kBSfree + s]);
-            const int kb = j * kPT;
-            float mx = -INFINITY;
+            if (kb + kPT - 1 > i0) {  // a page on the diagonal (or past the prompt): mask
+                const int nv = lim - (kb + kofs);  // keys c <= nv are visible
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                x[c] = (kb + c <= lim) ? x[c] : -INFINITY;
-                mx = fmaxf(mx, x[c]);
+                for (int c = 0; c < 32; ++c) x[c] = c <= nv ? x[c] : -INFINITY;
             }
+            float mx;
+            {  // tree maximum: 5 dependent steps instead of 32
+                float t[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c) t[c] = fmaxf(x[c], x[c + 16]);
+#pragma unroll
+                for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+                    for (int c = 0; c < w; ++c) t[c] = fmaxf(t[c], t[c + w]);
+                mx = t[0];
+            }
+            // the row maximum over both halves
+            xmax[(s * 2 + half) * kBM + row] = mx;
+            named_bar_sync(pair_bar, 64);
+            mx = fmaxf(mx, xmax[(s * 2 + (half ^ 1)) * kBM + row]);
             const float m_new = fmaxf(m, mx);
             const bool need = m_new > m + kRescaleLog2;  // also the first finite maximum
-            const float factor = need ? exp2f(m - m_new) : 1.f;
+            const float factor = need ? ex2_approx(m - m_new) : 1.f;
             if (need) {
                 l *= factor;
                 m = m_new;
             }
             if (__any_sync(0xffffffffu, need && j > 0)) {
-                // O holds pages 0..j-1: wait for the last of them, then rescale this row
+                // O holds pages 0..j-1: wait for the last of them, then rescale this half
                 mbar_wait(&bar[kBOdone], (j - 1) & 1, abort_flag, p.err);
                 tc_fence_after();
 #pragma unroll 1
-                for (int c0 = 0; c0 < RV; c0 += 32) {
-                    float v[32];
-                    tmem_ld32(tl + F::TM_O + c0, v);
+                for (int c0 = half * (RV / 2); c0 < (half + 1) * (RV / 2); c0 += 16) {
+                    float v[16];
+                    tmem_ld16(tl + F::TM_O + c0, v);
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) v[c] *= factor;
-                    tmem_st32(tl + F::TM_O + c0, v);
+                    for (int c = 0; c < 16; ++c) v[c] *= factor;
+                    tmem_st16(tl + F::TM_O + c0, v);
                 }
             }
             if (j >= 2) mbar_wait(&bar[kBPfree + s], ((j - 2) >> 1) & 1, abort_flag, p.err);
-            char *pr = sm + F::oP + s * F::PB + row * 16;
+            char *pr = sm + F::oP + s * F::PB + row * 16 + (kofs / 8) * 2048;
 #pragma unroll
-            for (int c = 0; c < 64; c += 8) {
-                uint32_t w[4];
+            for (int c = 0; c < 32; ++c) x[c] = ex2_approx(x[c] - m);
 #pragma unroll
-                for (int k = 0; k < 8; k += 2) {
-                    const float a = m == -INFINITY ? 0.f : exp2f(x[c + k] - m);
-                    const float bb = m == -INFINITY ? 0.f : exp2f(x[c + k + 1] - m);
-                    w[k / 2] = pack_bf16(a, bb);
-                    l += __uint_as_float(w[k / 2] << 16) + __uint_as_float(w[k / 2] & 0xffff0000u);
+            for (int c = 0; c < 32; c += 8)
+                *reinterpret_cast<uint4 *>(pr + (c / 8) * 2048) =
+                    make_uint4(pack_bf16x2(x[c], x[c + 1]), pack_bf16x2(x[c + 2], x[c + 3]),
+                               pack_bf16x2(x[c + 4], x[c + 5]), pack_bf16x2(x[c + 6], x[c + 7]));
+            {  // tree sum of this half's probabilities
+                float t[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c) t[c] = x[c] + x[c + 16];
+#pragma unroll
+                for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+                    for (int c = 0; c < w; ++c) t[c] += t[c + w];
+                l += t[0];
+            }
+            if (j == NP - 1 && kb + kPT > L) {
+                // last page of the prompt: V rows past it hold no latents; zero them before the
+                // PV product reads them (0 * NaN would poison the sum)
+                mbar_wait(&bar[kBVfull + s], (j >> 1) & 1, abort_flag, p.err);
+                char *vs = sm + F::oV + s * F::VPAGE;
+                const int valid = L - kb;
+                const int nz = (kPT - valid) * F::VATOMS * 8;  // 16-byte words to clear
+                for (int w = tid - 64; w < nz; w += kSThreads) {
+                    const int c = w & 7, r2 = w >> 3;
+                    const int a = r2 % F::VATOMS, i = valid + r2 / F::VATOMS;
+                    *reinterpret_cast<uint4 *>(vs + a * (kPT * 128) + i * 128 + c * 16) = make_uint4(0, 0, 0, 0);
                 }
-                *reinterpret_cast<uint4 *>(pr + (c / 8) * 2048) = make_uint4(w[0], w[1], w[2], w[3]);
             }
             fence_proxy_async_smem();
             tc_fence_before();
             mbar_arrive(&bar[kBPfull + s]);
         }
+        // the row sum over both halves
+        xsum[half * kBM + row] = l;
+        named_bar_sync(pair_bar, 64);
+        l += xsum[(half ^ 1) * kBM + row];
         // epilogue: O / l -> two bf16 K-major operands in turn (hi, then lo = O/l - hi) in one
         // buffer that aliases the K ring; O stays in TMEM between the two
         mbar_wait(&bar[kBOfin], 0, abort_flag, p.err);
@@ -422,21 +458,21 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
                 tc_fence_after();
             }
 #pragma unroll 1
-            for (int c0 = 0; c0 < RV; c0 += 32) {
-                float v[32];
-                tmem_ld32(tl + F::TM_O + c0, v);
+            for (int c0 = half * (RV / 2); c0 < (half + 1) * (RV / 2); c0 += 16) {
+                float v[16];
+                tmem_ld16(tl + F::TM_O + c0, v);
 #pragma unroll
-                for (int k = 0; k < 32; ++k) {
-                    const float x = v[k] * inv;
-                    const float hi = __bfloat162float(__float2bfloat16_rn(x));
-                    v[k] = part ? x - hi : hi;
+                for (int k = 0; k < 16; ++k) {
+                    const float xv = v[k] * inv;
+                    const float hi = __bfloat162float(__float2bfloat16_rn(xv));
+                    v[k] = part ? xv - hi : hi;
                 }
                 char *oa = sm + F::oOA + row * 16;
 #pragma unroll
-                for (int k = 0; k < 32; k += 8)
+                for (int k = 0; k < 16; k += 8)
                     *reinterpret_cast<uint4 *>(oa + ((c0 + k) / 8) * 2048) =
-                        make_uint4(pack_bf16(v[k], v[k + 1]), pack_bf16(v[k + 2], v[k + 3]),
-                                   pack_bf16(v[k + 4], v[k + 5]), pack_bf16(v[k + 6], v[k + 7]));
+                        make_uint4(pack_bf16x2(v[k], v[k + 1]), pack_bf16x2(v[k + 2], v[k + 3]),
+                                   pack_bf16x2(v[k + 4], v[k + 5]), pack_bf16x2(v[k + 6], v[k + 7]));
             }
             fence_proxy_async_smem();
             tc_fence_before();
@@ -446,7 +482,7 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
         tc_fence_after();
         const float *muv = p.mu_v ? p.mu_v + wofs : nullptr;
 #pragma unroll 1
-        for (int c0 = 0; c0 < D; c0 += 32) {
+        for (int c0 = half * (D / 2); c0 < (half + 1) * (D / 2); c0 += 32) {
             float v[32];
             tmem_ld32(tl + c0, v);
             if (muv) {
@@ -459,8 +495,8 @@ __global__ void __launch_bounds__(kPThreads, 1) prefill_tc_kernel(const PParams 
 #pragma unroll
                     for (int k = 0; k < 32; k += 8)
                         *reinterpret_cast<uint4 *>(dst + k * 2) =
-                            make_uint4(pack_bf16(v[k], v[k + 1]), pack_bf16(v[k + 2], v[k + 3]),
-                                       pack_bf16(v[k + 4], v[k + 5]), pack_bf16(v[k + 6], v[k + 7]));
+                            make_uint4(pack_bf16x2(v[k], v[k + 1]), pack_bf16x2(v[k + 2], v[k + 3]),
+                                       pack_bf16x2(v[k + 4], v[k + 5]), pack_bf16x2(v[k + 6], v[k + 7]));
                 } else {
 #pragma unroll
                     for (int k = 0; k < 32; k += 4)
@@ -621,7 +657,25 @@ lla_status launch_tc(const PParams &prm, int nqt, int B, int H, cudaStream_t str
             return LLA_ERR_CUDA;
         configured[dev] = true;
     }
-    return launch_pf(prefill_tc_kernel<RK, RV>, dim3(nqt, B, H), kPThreads, PF<RK, RV>::SMEM, stream, prm);
+    // the V-planes of every head page: [pages][64 tokens][r_v] bf16, one page = one head page
+    CUtensorMap tv;
+    const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT),
+                              static_cast<uint64_t>(prm.num_blocks) * prm.H};
+    const uint64_t strides[2] = {static_cast<uint64_t>(RV) * 2, static_cast<uint64_t>(prm.head_page_bytes)};
+    const uint32_t box[3] = {64, kPT, 1};
+    if (!encode_tmap_bf16(&tv, prm.pool + kPT * RK * 2, 3, dims, strides, box, true)) return LLA_ERR_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(nqt, B, H);
+    cfg.blockDim = dim3(kPThreads);
+    cfg.dynamicSmemBytes = PF<RK, RV>::SMEM;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, prefill_tc_kernel<RK, RV>, tv, prm) != cudaSuccess) return LLA_ERR_CUDA;
+    return LLA_OK;
 }
 
 }  // namespace
@@ -633,7 +687,8 @@ lla_status launch_prefill(const PrefillArgs &a, cudaStream_t stream) {
     const int es = a.storage_bf16 ? 2 : 4;
     const int hpb = static_cast<int>(head_page_bytes(a.r_k, a.r_v, es));
     if (a.B > 65535 || a.H > 65535) return LLA_ERR_UNSUPPORTED;
-    if (a.storage_bf16 && a.d == 128) {
+    // the tensor-core kernel addresses head pages with a 32-bit TMA coordinate
+    if (a.storage_bf16 && a.d == 128 && a.num_blocks * a.H < (int64_t(1) << 31)) {
         PParams p = {};
         p.T = a.T; p.H = a.H; p.loop = a.loop; p.io_bf16 = a.io_bf16;
         p.scale_log2 = a.scale * kLog2e;

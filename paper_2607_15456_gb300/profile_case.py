@@ -1,12 +1,19 @@
-"""A small, fixed case of one kernel for ncu captures.
+"""Small, fixed cases of one kernel each, for ncu captures.
 
-Builds a workload's latent cache for a few layers only (same batch, context lengths, heads and
-ranks, so every decode launch has exactly the shape and bytes of a launch in the full
-benchmark), then runs `--calls` pass-1 decode calls (and one encode call per layer), so that a
-profiler can skip the warm-up launches and capture one to three of them:
+decode (default): builds a workload's latent cache for a few layers only (same batch, context
+lengths, heads and ranks, so every decode launch has exactly the shape and bytes of a launch in
+the full benchmark), then runs `--calls` pass-1 decode calls (and one encode call per layer), so
+that a profiler can skip the warm-up launches and capture one to three of them:
 
     ncu --set full --clock-control none -k regex:decode_async_kernel -s 6 -c 1 \\
         python -m paper_2607_15456_gb300.profile_case --workload ouro14_rho4 --layers 2 --calls 10
+
+prefill: encodes `--prompts` prompts of `--len` tokens of a workload's ranks (tensor-core encode,
+one launch per axis), then runs `--calls` causal prefill calls over them:
+
+    ncu --set full --clock-control none -k regex:"encode_tc_kernel|prefill_tc_kernel" -c 3 \\
+        python -m paper_2607_15456_gb300.profile_case --case prefill --workload ouro14_rho2 \\
+        --prompts 4 --len 8192 --calls 1
 """
 from __future__ import annotations
 
@@ -19,12 +26,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--workload", default="ouro14_rho4")
-    ap.add_argument("--layers", type=int, default=2)
-    ap.add_argument("--calls", type=int, default=10)
-    args = ap.parse_args()
+def decode_case(args):
     import torch
 
     from bench import DecodeBench
@@ -46,6 +48,57 @@ def main():
         raise SystemExit(f"device error word {err:#x}")
     print(f"profile case done: {args.workload}, {w.D} layers, {args.calls} decode calls, "
           f"{bench.decode_bytes_per_launch()} algorithmic bytes per decode launch")
+
+
+def prefill_case(args):
+    import torch
+
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = W.WORKLOADS[args.workload]
+    T, H, d = w.T, w.H, w.d
+    geom = lla.Geometry(T, H, d, w.r_k, w.r_v, "bf16")
+    codec = lla.Codec(**W.codec_tensors(T, H, d, w.r_k, w.r_v, w.seed, 0, device=dev))
+    lens = [args.len] * args.prompts
+    pt = W.page_table(lens, w.seed, extra_tokens=0)
+    pool = torch.zeros(pt.num_blocks * lla.lla_cache_block_bytes(geom), dtype=torch.uint8, device=dev)
+    cache = lla.Cache(pool, pt.num_blocks, pt.block_table.to(dev), pt.max_blocks)
+    N = sum(lens)
+    slots = torch.cat([pt.slots(b, range(L)) for b, L in enumerate(lens)]).to(dev)
+    xk = W.normal((T, N, H, d), w.seed, 300, device=dev)
+    xv = W.normal((T, N, H, d), w.seed, 301, device=dev)
+    lla.lla_encode(geom, codec, cache, xk, xv, slots)
+    del xk, xv
+    q = W.normal((N, H, d), w.seed, 302, device=dev)
+    out = torch.empty_like(q)
+    cu = torch.tensor([i * args.len for i in range(args.prompts + 1)], dtype=torch.int32, device=dev)
+    for _ in range(args.calls):
+        lla.lla_prefill_attn(geom, codec, cache, cu, args.len, 1, q, out)
+    torch.cuda.synchronize()
+    err = lla.lla_get_device_error()
+    if err:
+        raise SystemExit(f"device error word {err:#x}")
+    pairs = args.prompts * H * args.len * (args.len + 1) // 2
+    print(f"profile case done: {args.workload} prefill, {args.prompts} x {args.len} tokens, "
+          f"{pairs} (query, key) pairs per call, {args.calls} calls")
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--case", choices=["decode", "prefill"], default="decode")
+    ap.add_argument("--workload", default="ouro14_rho4")
+    ap.add_argument("--layers", type=int, default=2)
+    ap.add_argument("--calls", type=int, default=10)
+    ap.add_argument("--prompts", type=int, default=4)
+    ap.add_argument("--len", type=int, default=8192)
+    args = ap.parse_args()
+    if args.case == "decode":
+        decode_case(args)
+    else:
+        prefill_case(args)
 
 
 if __name__ == "__main__":
