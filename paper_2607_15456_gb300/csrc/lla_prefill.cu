@@ -9,17 +9,21 @@
 //
 // Tensor-core path (bf16 storage, d = 128, r_k and r_v multiples of 32): one CTA per
 // (128-query tile, sequence, head) and four warp roles.
-//   warp 0      producer: W_up,t^K into shared memory (cp.async), then per page of 64 keys the
-//               K-plane (one bulk copy: its granule-interleaved layout is already the
-//               core-matrix layout of a K-major MMA operand) and the V-plane (one TMA tensor
-//               load with 128-byte swizzle per 64 latent columns: an MN-major operand), and
-//               W_up,t^V for the epilogue
-//   warp 1      MMA issuer (one thread) and TMEM owner:
+//   warp 0      K producer: W_up,t^K into shared memory (cp.async), then per page of 64 keys
+//               the K-plane (one bulk copy: its granule-interleaved layout is already the
+//               core-matrix layout of a K-major MMA operand), and W_up,t^V for the epilogue;
+//               the V-plane of each page comes as one TMA tensor load with 128-byte swizzle per
+//               64 latent columns (an MN-major operand)
+//   warp 2      V producer (one thread), decoupled from the K-planes so that neither ring
+//               waits on the other
+//   warp 1      Q~ and S issuer (one thread) and TMEM owner:
 //                 Q~ = Q W_up,t^K             M=128, N=r_k, K=d
-//                 S_j = Q~ C_k,j^T            M=128, N=64,  K=r_k   (one page ahead of PV)
+//                 S_j = Q~ C_k,j^T            M=128, N=64,  K=r_k   (double-buffered in TMEM)
+//   warp 3      PV and output issuer (one thread), so that neither MMA stream waits behind the
+//               other's barriers:
 //                 O += P_j C_v,j              M=128, N=r_v (split at 256), K=64
 //                 out = (O/l) W_up,t^V^T      M=128, N=d,   K=r_v
-//   warps 2-9   two threads per query row, each with 32 keys of every page (warps w and w + 4
+//   warps 4-11  two threads per query row, each with 32 keys of every page (warps w and w + 4
 //               share TMEM lanes): Q and Q~ into bf16 operands, causal mask on diagonal pages,
 //               online softmax in the exp2 domain with the row maximum exchanged through shared
 //               memory, P into a bf16 operand, O rescaled in TMEM only when a row maximum grows
@@ -42,7 +46,8 @@ namespace {
 constexpr int kBM = 128;         // queries per tile
 constexpr int kPT = 64;          // keys per page
 constexpr int kSWarps = 8;       // softmax warps: two threads per query row
-constexpr int kPThreads = 64 + kSWarps * 32;
+constexpr int kSWarp0 = 4;       // K producer, S issuer, V producer, PV issuer, then softmax
+constexpr int kPThreads = (kSWarp0 + kSWarps) * 32;
 constexpr int kSThreads = kSWarps * 32;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when a row maximum grows by more
@@ -82,11 +87,15 @@ struct PF {
     static constexpr int WK = D * RK * 2;            // W_up,t^K operand (prologue)
     static constexpr int WV = D * RV * 2;            // W_up,t^V operand (epilogue)
     static constexpr int OA = kBM * RV * 2;          // O / l operand (epilogue)
-    static constexpr int ST = 2;                     // K and V pipeline stages
+    // K and V pipeline stages: as deep as shared memory allows (up to 4), V at least 2 deep
+    static constexpr int BUDGET = 220 * 1024 - QT - 2 * PB;
+    static constexpr int STV = (BUDGET - 2 * KPAGE) / VPAGE >= 4 ? 4 : (BUDGET - 2 * KPAGE) / VPAGE >= 3 ? 3 : 2;
+    static constexpr int STK0 = (BUDGET - STV * VPAGE) / KPAGE;
+    static constexpr int STK = STK0 > 4 ? 4 : STK0;
     static constexpr int oQT = 0;
     static constexpr int oK = oQT + QT;
-    static constexpr int oV = oK + ST * KPAGE;
-    static constexpr int oP = oV + ST * VPAGE;
+    static constexpr int oV = oK + STK * KPAGE;
+    static constexpr int oP = oV + STV * VPAGE;
     static constexpr int oEnd = oP + 2 * PB;
     // the prologue operands alias the V ring and P; the epilogue operands alias K, V and P
     static constexpr int oQA = oV, oWK = oV + QA;
@@ -94,12 +103,13 @@ struct PF {
     static constexpr int oX = oEnd;                   // [2 pages][2 halves][128 rows] maxima
     static constexpr int oL = oX + 2 * 2 * kBM * 4;   // [2 halves][128 rows] row sums
     static constexpr int oBar = oL + 2 * kBM * 4;
-    static constexpr int NBAR = 32;
+    static constexpr int NBAR = 40;
     static constexpr int SMEM = 1024 + oBar + NBAR * 8 + 16;
     // TMEM columns: S double buffer [0, 128), O [128, 128 + RV); q~ and out reuse [0, ...)
     static constexpr uint32_t TM_S = 0, TM_O = 128, TM_COLS = 512;
     static_assert(RK % 32 == 0 && RV % 32 == 0 && RK <= 256 && 128 + RV <= 512, "ranks");
     static_assert(N0 % 16 == 0 && N1 % 16 == 0 && N1 <= 256, "PV split");
+    static_assert(STK >= 2 && STV >= 2, "pipeline depth");
     static_assert(oK % 1024 == 0 && oV % 1024 == 0 && oP % 1024 == 0 && VPAGE % 1024 == 0, "align");
     static_assert(oWK + WK <= oEnd && oWV + WV <= oEnd, "aliased operands fit");
     static_assert(SMEM <= 227 * 1024, "shared memory");
@@ -108,10 +118,10 @@ struct PF {
 // barrier indices
 enum {
     kBSetup = 0, kBQt, kBQs, kBOa, kBWv, kBOut, kBOdone, kBOfin,
-    kBKfull = 8 /* [2] */, kBKempty = 10, kBVfull = 12, kBVempty = 14,
-    kBSfull = 16, kBSfree = 18, kBPfull = 20, kBPfree = 22,
-    kBOa2 = 24, kBOut1 = 25,
-    kBAbort = 31  // slot used as the CTA's abort flag
+    kBSfull = 8 /* [2] */, kBSfree = 10, kBPfull = 12, kBPfree = 14,
+    kBOa2 = 16, kBOut1 = 17,
+    kBKfull = 18 /* [4] */, kBKempty = 22, kBVfull = 26, kBVempty = 30,
+    kBAbort = 34  // slot used as the CTA's abort flag
 };
 
 template <int RK, int RV>
@@ -156,11 +166,15 @@ __global__ void __launch_bounds__(kPThreads, 1)
         mbar_init(&bar[kBOut], 1);
         mbar_init(&bar[kBOdone], 1);
         mbar_init(&bar[kBOfin], 1);
-        for (int s = 0; s < 2; ++s) {
+        for (int s = 0; s < F::STK; ++s) {
             mbar_init(&bar[kBKfull + s], 1);
             mbar_init(&bar[kBKempty + s], 1);
+        }
+        for (int s = 0; s < F::STV; ++s) {
             mbar_init(&bar[kBVfull + s], 1);
             mbar_init(&bar[kBVempty + s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
             mbar_init(&bar[kBSfull + s], 1);
             mbar_init(&bar[kBSfree + s], kSThreads);
             mbar_init(&bar[kBPfull + s], kSThreads);
@@ -187,11 +201,11 @@ __global__ void __launch_bounds__(kPThreads, 1)
         cp_async_wait_all();
         fence_proxy_async_smem();
         mbar_arrive(&bar[kBSetup]);
-        if (lane == 0) {
+        if (lane == 0) {  // K-planes: one bulk copy per page
             const uint64_t pol = policy_evict_first();
             for (int j = 0; j < NP; ++j) {
-                const int s = j & 1;
-                const uint32_t ph = (j >> 1) & 1;
+                const int s = j % F::STK;
+                const uint32_t ph = (j / F::STK) & 1;
                 int32_t blk = bt[j];
                 if (blk < 0 || blk >= p.num_blocks) {
                     atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
@@ -202,14 +216,6 @@ __global__ void __launch_bounds__(kPThreads, 1)
                 mbar_arrive_expect_tx(&bar[kBKfull + s], F::KPAGE);
                 bulk_g2s(sm + F::oK + s * F::KPAGE, p.pool + hp * p.head_page_bytes, F::KPAGE,
                          &bar[kBKfull + s], pol);
-                // the V ring aliases the prologue operands: wait until Q~ has been computed
-                if (j == 0) mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
-                mbar_wait(&bar[kBVempty + s], ph ^ 1u, abort_flag, p.err);
-                mbar_arrive_expect_tx(&bar[kBVfull + s], F::VPAGE);
-                char *vs = sm + F::oV + s * F::VPAGE;
-#pragma unroll
-                for (int a = 0; a < F::VATOMS; ++a)
-                    tma_load_3d(vs + a * (kPT * 128), &tv, a * 64, 0, static_cast<int>(hp), &bar[kBVfull + s]);
             }
         }
         __syncwarp();
@@ -225,83 +231,114 @@ __global__ void __launch_bounds__(kPThreads, 1)
         cp_async_wait_all();
         fence_proxy_async_smem();
         mbar_arrive(&bar[kBWv]);
+    } else if (warp == 2) {
+        // ---------------------------------------------------------------------- V producer
+        if (lane == 0) {  // V-planes: one TMA tensor load with 128-byte swizzle per 64 columns
+            // the V ring aliases the prologue operands: wait until Q~ has been computed
+            mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
+            for (int j = 0; j < NP; ++j) {
+                const int s = j % F::STV;
+                const uint32_t ph = (j / F::STV) & 1;
+                int32_t blk = bt[j];
+                if (blk < 0 || blk >= p.num_blocks) blk = 0;  // flagged by the K producer
+                const int64_t hp = static_cast<int64_t>(blk) * p.H + h;
+                mbar_wait(&bar[kBVempty + s], ph ^ 1u, abort_flag, p.err);
+                mbar_arrive_expect_tx(&bar[kBVfull + s], F::VPAGE);
+                char *vs = sm + F::oV + s * F::VPAGE;
+#pragma unroll
+                for (int a = 0; a < F::VATOMS; ++a)
+                    tma_load_3d(vs + a * (kPT * 128), &tv, a * 64, 0, static_cast<int>(hp), &bar[kBVfull + s]);
+            }
+        }
+        __syncwarp();
     } else if (warp == 1) {
-        // ------------------------------------------------------------------------ MMA issuer
+        // -------------------------------------------------------------- Q~ and S MMA issuer
         if (lane == 0) {
             const uint32_t base = smem_addr(sm);
             mbar_wait(&bar[kBSetup], 0, abort_flag, p.err);
             tc_fence_after();
             constexpr uint32_t idq = umma_idesc_bf16(128, RK, 0, 1);
-#pragma unroll 1
+            const uint64_t dqa = umma_desc(base + F::oQA, 2048, 128);
+            const uint64_t dwk = umma_desc(base + F::oWK, 128, 2048);
+#pragma unroll
             for (int ks = 0; ks < D / 16; ++ks)
-                umma_bf16(tmem + 0, umma_desc(base + F::oQA + ks * 4096, 2048, 128),
-                          umma_desc(base + F::oWK + ks * 256, 128, 2048), idq, ks > 0);
+                umma_bf16(tmem + 0, dqa + ks * (4096 >> 4), dwk + ks * (256 >> 4), idq, ks > 0);
             umma_commit(&bar[kBQt]);
             mbar_wait(&bar[kBQs], 0, abort_flag, p.err);
             tc_fence_after();
             constexpr uint32_t ids = umma_idesc_bf16(128, kPT, 0, 0);
+            // descriptors are built once; a byte offset moves the start-address field by offset/16
+            const uint64_t dq = umma_desc(base + F::oQT, 2048, 128);
+            const uint64_t dk0 = umma_desc(base + F::oK, 1024, 128);
+#pragma unroll 1
+            for (int j = 0; j < NP; ++j) {
+                const int s = j & 1, sk = j % F::STK;
+                mbar_wait(&bar[kBKfull + sk], (j / F::STK) & 1, abort_flag, p.err);
+                if (j >= 2) mbar_wait(&bar[kBSfree + s], ((j - 2) >> 1) & 1, abort_flag, p.err);
+                tc_fence_after();
+                const uint64_t dk = dk0 + static_cast<uint64_t>(sk * (F::KPAGE >> 4));
+                const uint32_t ds = tmem + F::TM_S + s * kPT;
+#pragma unroll
+                for (int ks = 0; ks < RK / 16; ++ks)
+                    umma_bf16(ds, dq + ks * (4096 >> 4), dk + ks * (2048 >> 4), ids, ks > 0);
+                umma_commit(&bar[kBSfull + s]);
+                umma_commit(&bar[kBKempty + sk]);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 3) {
+        // ----------------------------------------------------------- PV and output MMA issuer
+        if (lane == 0) {
+            const uint32_t base = smem_addr(sm);
             constexpr uint32_t idv0 = umma_idesc_bf16(128, F::N0, 0, 1);
             constexpr uint32_t idv1 = umma_idesc_bf16(128, F::N1 > 0 ? F::N1 : 16, 0, 1);
+            const uint64_t dp0 = umma_desc(base + F::oP, 2048, 128);
+            const uint64_t dv0 = umma_desc_sw128_mn(base + F::oV, kPT * 128);
 #pragma unroll 1
-            for (int j = 0; j <= NP; ++j) {
-                if (j < NP) {
-                    const int s = j & 1;
-                    mbar_wait(&bar[kBKfull + s], (j >> 1) & 1, abort_flag, p.err);
-                    if (j >= 2) mbar_wait(&bar[kBSfree + s], ((j - 2) >> 1) & 1, abort_flag, p.err);
-                    tc_fence_after();
-#pragma unroll 1
-                    for (int ks = 0; ks < RK / 16; ++ks)
-                        umma_bf16(tmem + F::TM_S + s * kPT,
-                                  umma_desc(base + F::oQT + ks * 4096, 2048, 128),
-                                  umma_desc(base + F::oK + s * F::KPAGE + ks * 2048, 1024, 128), ids,
-                                  ks > 0);
-                    umma_commit(&bar[kBSfull + s]);
-                    umma_commit(&bar[kBKempty + s]);
+            for (int jj = 0; jj < NP; ++jj) {
+                const int s = jj & 1, sv = jj % F::STV;
+                mbar_wait(&bar[kBPfull + s], (jj >> 1) & 1, abort_flag, p.err);
+                mbar_wait(&bar[kBVfull + sv], (jj / F::STV) & 1, abort_flag, p.err);
+                tc_fence_after();
+                const uint64_t dp = dp0 + static_cast<uint64_t>(s * (F::PB >> 4));
+                const uint64_t dv = dv0 + static_cast<uint64_t>(sv * (F::VPAGE >> 4));
+                const bool acc = jj > 0;
+#pragma unroll
+                for (int ks = 0; ks < kPT / 16; ++ks) {
+                    umma_bf16(tmem + F::TM_O, dp + ks * (4096 >> 4), dv + ks * (2048 >> 4), idv0, acc || ks > 0);
+                    if constexpr (F::N1 > 0)
+                        umma_bf16(tmem + F::TM_O + F::N0, dp + ks * (4096 >> 4),
+                                  dv + ((F::N0 / 64) * (kPT * 128) >> 4) + ks * (2048 >> 4), idv1,
+                                  acc || ks > 0);
                 }
-                if (j >= 1) {
-                    const int jj = j - 1, s = jj & 1;
-                    mbar_wait(&bar[kBPfull + s], (jj >> 1) & 1, abort_flag, p.err);
-                    mbar_wait(&bar[kBVfull + s], (jj >> 1) & 1, abort_flag, p.err);
-                    tc_fence_after();
-                    const uint32_t vb = base + F::oV + s * F::VPAGE;
-#pragma unroll 1
-                    for (int ks = 0; ks < kPT / 16; ++ks) {
-                        const uint64_t da = umma_desc(base + F::oP + s * F::PB + ks * 4096, 2048, 128);
-                        umma_bf16(tmem + F::TM_O, da, umma_desc_sw128_mn(vb + ks * 2048, kPT * 128), idv0,
-                                  jj > 0 || ks > 0);
-                        if constexpr (F::N1 > 0)
-                            umma_bf16(tmem + F::TM_O + F::N0, da,
-                                      umma_desc_sw128_mn(vb + (F::N0 / 64) * (kPT * 128) + ks * 2048, kPT * 128),
-                                      idv1, jj > 0 || ks > 0);
-                    }
-                    umma_commit(&bar[kBVempty + s]);
-                    umma_commit(&bar[kBPfree + s]);
-                    umma_commit(&bar[kBOdone]);
-                }
+                umma_commit(&bar[kBVempty + sv]);
+                umma_commit(&bar[kBPfree + s]);
+                umma_commit(&bar[kBOdone]);
             }
-            umma_commit(&bar[kBOfin]);  // every MMA of the loop has completed
+            umma_commit(&bar[kBOfin]);  // every PV MMA (and, before them, every S MMA) has completed
             // out = (O / l) W_up,t^V^T, with O / l = hi + lo as two bf16 operands in turn, so
             // that the projection sees O / l to about 16 significant bits
             mbar_wait(&bar[kBWv], 0, abort_flag, p.err);
             constexpr uint32_t ido = umma_idesc_bf16(128, D, 0, 0);
+            const uint64_t doa = umma_desc(base + F::oOA, 2048, 128);
+            const uint64_t dwv = umma_desc(base + F::oWV, 2048, 128);
 #pragma unroll 1
             for (int part = 0; part < 2; ++part) {
                 mbar_wait(&bar[part ? kBOa2 : kBOa], 0, abort_flag, p.err);
                 tc_fence_after();
 #pragma unroll 1
                 for (int ks = 0; ks < RV / 16; ++ks)
-                    umma_bf16(tmem + 0, umma_desc(base + F::oOA + ks * 4096, 2048, 128),
-                              umma_desc(base + F::oWV + ks * 4096, 2048, 128), ido, part > 0 || ks > 0);
+                    umma_bf16(tmem + 0, doa + ks * (4096 >> 4), dwv + ks * (4096 >> 4), ido, part > 0 || ks > 0);
                 umma_commit(&bar[part ? kBOut : kBOut1]);
             }
         }
         __syncwarp();
     } else {
         // ------------------------------------------------------------ softmax and epilogue
-        // warps 2..9: quarter (TMEM lanes) = warp % 4, half = which 32 keys of a page (and which
+        // warps 4..11: quarter (TMEM lanes) = warp % 4, half = which 32 keys of a page (and which
         // half of every other row-wise job) this thread owns; warps w and w + 4 share rows
         const int quarter = warp & 3;
-        const int half = (warp - 2) >> 2;
+        const int half = (warp - kSWarp0) >> 2;
         const int row = quarter * 32 + lane;
         const int pair_bar = 2 + quarter;  // named barrier of the two warps of this quarter
         const uint32_t tl = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
@@ -428,11 +465,12 @@ __global__ void __launch_bounds__(kPThreads, 1)
             if (j == NP - 1 && kb + kPT > L) {
                 // last page of the prompt: V rows past it hold no latents; zero them before the
                 // PV product reads them (0 * NaN would poison the sum)
-                mbar_wait(&bar[kBVfull + s], (j >> 1) & 1, abort_flag, p.err);
-                char *vs = sm + F::oV + s * F::VPAGE;
+                const int sv = j % F::STV;
+                mbar_wait(&bar[kBVfull + sv], (j / F::STV) & 1, abort_flag, p.err);
+                char *vs = sm + F::oV + sv * F::VPAGE;
                 const int valid = L - kb;
                 const int nz = (kPT - valid) * F::VATOMS * 8;  // 16-byte words to clear
-                for (int w = tid - 64; w < nz; w += kSThreads) {
+                for (int w = tid - kSWarp0 * 32; w < nz; w += kSThreads) {
                     const int c = w & 7, r2 = w >> 3;
                     const int a = r2 % F::VATOMS, i = valid + r2 / F::VATOMS;
                     *reinterpret_cast<uint4 *>(vs + a * (kPT * 128) + i * 128 + c * 16) = make_uint4(0, 0, 0, 0);
