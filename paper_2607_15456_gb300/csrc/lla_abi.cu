@@ -167,6 +167,10 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
     if (max_ctx < 0 || static_cast<int64_t>(max_ctx) >
                            static_cast<int64_t>(cache->max_blocks_per_seq) * LLA_BLOCK_TOKENS)
         return LLA_ERR_INVALID_ARG;
+    // a sequence's pages of all heads are counted in 32 bits inside the kernel
+    if (static_cast<int64_t>(g->H) * ((static_cast<int64_t>(max_ctx) + LLA_BLOCK_TOKENS - 1) / LLA_BLOCK_TOKENS) >=
+        (int64_t(1) << 31))
+        return LLA_ERR_UNSUPPORTED;
     if ((cur_k == nullptr) != (cur_v == nullptr)) return LLA_ERR_INVALID_ARG;
     if (B > 0 && (!context_lens || !q || !out)) return LLA_ERR_INVALID_ARG;
     if ((st = decode_fits(g->r_k, g->r_v, es, g->d)) != LLA_OK) return st;

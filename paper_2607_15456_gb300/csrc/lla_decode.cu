@@ -202,6 +202,8 @@ __device__ __forceinline__ int64_t range_start(int c, int64_t U, int Geff) {
 struct Range {
     int64_t U, A0, A1;
     int Geff;
+    // the order in which the CTA walks its runs: [lo[0], hi[0]), [lo[1], hi[1]), [lo[2], hi[2])
+    int64_t lo[3], hi[3];
 };
 
 // Barrier set-up and the per-sequence unit prefix (H heads x pages), with device-side length
@@ -256,6 +258,9 @@ __device__ Range prologue(const Params &p, const Smem &s, uint32_t pfull_count,
         r.A0 = range_start(blockIdx.x, r.U, r.Geff);
         r.A1 = range_start(blockIdx.x + 1, r.U, r.Geff);
     }
+    r.lo[0] = r.A0;
+    r.hi[0] = r.A1;
+    r.lo[1] = r.hi[1] = r.lo[2] = r.hi[2] = 0;
     return r;
 }
 
@@ -269,15 +274,38 @@ __device__ __forceinline__ Run locate_run(const Params &p, const Smem &s, int64_
     Run R;
     R.b = seq_of_unit(s.prefix, p.B, u);
     R.Lb = s.lens[R.b];
-    const int np = static_cast<int>((s.prefix[R.b + 1] - s.prefix[R.b]) / p.H);
-    const int64_t off = u - s.prefix[R.b];
-    R.h = static_cast<int>(off / np);
-    R.pg0 = static_cast<int>(off % np);
+    // 32-bit arithmetic only: a 64-bit division is a called subroutine, cold in the instruction
+    // cache at run boundaries while the streaming loops run
+    const int np = (R.Lb + kBlockTokens - 1) / kBlockTokens;  // pages of the sequence
+    const int off = static_cast<int>(u - s.prefix[R.b]);      // < H * np
+    R.h = off / np;
+    R.pg0 = off - R.h * np;
     R.seg_start = s.prefix[R.b] + static_cast<int64_t>(R.h) * np;
     R.seg_end = R.seg_start + np;
     R.run_end = R.seg_end < A1 ? R.seg_end : A1;
     R.npages = static_cast<int>(R.run_end - u);
     return R;
+}
+
+// Split runs first: a CTA streams its first run, then its last run when that is the start of a
+// (sequence, head) the next CTA finishes, then the runs between them.  Both split runs are
+// then merged while the CTA still streams, and it ends on a whole (sequence, head) that it
+// finishes in place, so the launch does not end on a merge; a short first run is followed by
+// a run whose query set-up is already done.
+__device__ __forceinline__ void order_runs(const Params &p, const Smem &s, Range &r) {
+    if (r.A1 <= r.A0) return;
+    const Run T = locate_run(p, s, r.A1 - 1, r.A1);
+    const int64_t ts = T.seg_start > r.A0 ? T.seg_start : r.A0;  // start of the last run
+    if (ts == r.A0 || r.A1 == T.seg_end) return;                  // one run, or the last is whole
+    const Run Hd = locate_run(p, s, r.A0, r.A1);
+    const int64_t he = Hd.run_end;                                // end of the first run
+    if (he >= ts) return;                                         // two runs: already in order
+    r.lo[0] = r.A0;
+    r.hi[0] = he;
+    r.lo[1] = ts;
+    r.hi[1] = r.A1;
+    r.lo[2] = he;
+    r.hi[2] = ts;
 }
 
 // Producer: the whole warp walks the CTA's range.  Block ids are fetched 32 pages at a time
@@ -289,8 +317,9 @@ __device__ void producer(const Params &p, const Smem &s, const Range &rg) {
     const uint64_t pol = policy_evict_first();
     int it = 0, st = 0;
     uint32_t sph = 0;
-    for (int64_t u = rg.A0; u < rg.A1;) {
-        const Run R = locate_run(p, s, u, rg.A1);
+    for (int pass = 0; pass < 3; ++pass)
+    for (int64_t u = rg.lo[pass]; u < rg.hi[pass];) {
+        const Run R = locate_run(p, s, u, rg.hi[pass]);
         const int32_t *bt = p.block_table + static_cast<int64_t>(R.b) * p.max_blocks + R.pg0;
         for (int k0 = 0; k0 < R.npages; k0 += 32) {
             const int32_t blk_lane = (k0 + lane < R.npages) ? bt[k0 + lane] : -1;
@@ -543,7 +572,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
     const int hpb = p.head_page_bytes;
 
     pdl_wait();  // inputs may come from the previous kernel in the stream
-    const Range rg = prologue(p, s, 1, 1);
+    Range rg = prologue(p, s, 1, 1);
+    order_runs(p, s, rg);
     pdl_trigger();
 
     if (warp == kComputeWarps) {
@@ -563,8 +593,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
 
     int stage = 0;
     uint32_t ph = 0;
-    for (int64_t u = rg.A0; u < rg.A1;) {
-        const Run R = locate_run(p, s, u, rg.A1);
+    for (int pass = 0; pass < 3; ++pass)
+    for (int64_t u = rg.lo[pass]; u < rg.hi[pass];) {
+        const Run R = locate_run(p, s, u, rg.hi[pass]);
         setup_query<ES>(p, s, R.b, R.h);
         const float beta = s.misc[kMiscBeta];
 
@@ -729,14 +760,18 @@ __device__ __forceinline__ void load_qvec(const float *q, float (&v)[KE]) {
 //                          q~ while the other warps stream run r; for run r-1 they reduce the
 //                          left-behind softmax state, write or merge the split partials and
 //                          apply W_up,t^V.  Their global round trips never stall the stream.
-// Hand-offs are double-buffered by run parity: qready[slot] (management -> score warps, q~ of
-// a run is ready) and stfull[slot] (score + value warps -> management, the run's state is
-// written).  The management warps' order set-up(r), finish(r-1) guarantees that a slot is free
-// before it is written again.  W_up,t rows reach the management warps through a shared staging
-// buffer filled with cp.async, so no register holds them while they are in flight.
+// Hand-offs: qready[r % 3] (management -> score warps: q~ of run r is ready), stfull[r % 2]
+// (score + value warps -> management: the run's softmax state is written) and stfree[r % 2]
+// (management -> score and value warps: that state has been read).  The management warps set
+// up run r, then finish run r - 2; three query slots keep a set-up from overwriting what a
+// pending finish still reads, and the stfree wait keeps run r from overwriting the state of run
+// r - 2 before its finish has read it.  W_up,t rows reach the management warps through a shared
+// staging buffer filled with cp.async, so no register holds them while they are in flight.
 // ------------------------------------------------------------------------------------------
 
 constexpr int kMWarps = 4;
+constexpr int kQSlots = 3;  // query slots: set-ups run two runs ahead of finishes
+constexpr int kLredSlot = 128;  // row sums of one run (one per score thread of a k-split)
 constexpr int kMThreads = kMWarps * 32;
 constexpr int kMBase = kComputeThreads + 32;       // first management thread
 constexpr int kAsyncThreads = kMBase + kMThreads;  // 416
@@ -745,8 +780,8 @@ constexpr int kBarStart = 4;                       // producer waits for the fir
 constexpr int kWstMax = 40 * 1024;                 // staging buffer for W_up,t rows (upper bound)
 
 struct AsyncLayout {
-    int ring, full, empty, pfull, pempty, qready, stfull, prefix, lens, qlat, qfull, spart, psm,
-        lred, red, ovec, mred, mtmp, xtra, misc, wst, total;
+    int ring, full, empty, pfull, pempty, qready, stfull, stfree, prefix, lens, qlat, qfull, spart,
+        psm, lred, red, ovec, mred, mtmp, xtra, misc, wst, total;
 };
 
 // Shared-memory sizes of the asynchronous kernel for one rank shape (floats per slot).
@@ -771,20 +806,21 @@ __host__ __device__ inline AsyncLayout make_async_layout(int stages, int stage_b
     L.empty = o;  o += stages * 8;
     L.pfull = o;  o += 16;
     L.pempty = o; o += 16;
-    L.qready = o; o += 16;
+    L.qready = o; o += 32;  // [kQSlots]
     L.stfull = o; o += 16;
+    L.stfree = o; o += 16;
     L.prefix = o; o += up16((B + 1) * 8);
     L.lens = o;   o += up16(B * 4);
-    L.qlat = o;   o += up16(2 * qslot * 4);
-    L.qfull = o;  o += up16(2 * qslot * 4);
+    L.qlat = o;   o += up16(kQSlots * qslot * 4);
+    L.qfull = o;  o += up16(qslot * 4);  // q of the set-up in progress
     L.spart = o;  o += kComputeThreads * 4;
     L.psm = o;    o += 2 * kComputeThreads * 4;
-    L.lred = o;   o += 2 * kComputeThreads * 4;
+    L.lred = o;   o += 2 * kLredSlot * 4;
     L.red = o;    o += up16(2 * redslot * 4);
     L.ovec = o;   o += up16(rv * 4);
     L.mred = o;   o += up16(mred * 4);
     L.mtmp = o;   o += 2 * kMThreads * 4;
-    L.xtra = o;   o += up16(2 * xslot * 4);
+    L.xtra = o;   o += up16(kQSlots * xslot * 4);
     L.misc = o;   o += 64 * 4;
     L.wst = o;    o += up16(wst);
     L.total = o;
@@ -798,15 +834,15 @@ __host__ __device__ inline AsyncLayout async_layout(int stages, int stage_bytes,
 }
 
 // misc slots of the asynchronous kernel
-constexpr int kAM = 0 /* [2] run maximum by slot */, kAPAlpha = 5 /* [2] */,
+constexpr int kAM = 0 /* [2] run maximum by state slot */, kAPAlpha = 5 /* [2] */,
               kAWmax = 16 /* [2][8] */, kAAbort = 32, kALast = 33,
-              kAPart = 40 /* [2][4 warps][q.k_cur, q.mu^K] */;
+              kAPart = 40 /* [3 query slots][4 warps][q.k_cur, q.mu^K] */;
 
 struct ASmem {
     Smem s;  // fields shared with the generic helpers (ring, barriers, prefix, lens, abort flag)
-    uint64_t *qready, *stfull;
+    uint64_t *qready, *stfull, *stfree;
     float *qlat, *qfull, *lred, *red, *mred, *mtmp;
-    float *xtra;  // [2][v_cur (D), mu^V_t (D)] by run slot
+    float *xtra;  // [kQSlots][v_cur (D), mu^V_t (D)] by query slot
     char *wst;
     int qslot, redslot;  // floats per slot
 };
@@ -835,6 +871,7 @@ __device__ __forceinline__ ASmem carve_async(char *smem, const Params &p) {
     a.s.last_flag = reinterpret_cast<int *>(a.s.misc + kALast);
     a.qready = reinterpret_cast<uint64_t *>(smem + L.qready);
     a.stfull = reinterpret_cast<uint64_t *>(smem + L.stfull);
+    a.stfree = reinterpret_cast<uint64_t *>(smem + L.stfree);
     a.qlat = reinterpret_cast<float *>(smem + L.qlat);
     a.qfull = reinterpret_cast<float *>(smem + L.qfull);
     a.lred = reinterpret_cast<float *>(smem + L.lred);
@@ -906,7 +943,7 @@ __device__ void m_setup(const Params &p, const ASmem &a, int b, int h, int slot,
                         bool release_producer) {
     static_assert(D <= kMThreads, "one management thread per element of q");
     constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
-    float *qfull = a.qfull + slot * a.qslot;
+    float *qfull = a.qfull;
     float *qlat = a.qlat + slot * a.qslot;
     float *xtra = a.xtra + slot * 2 * D;
     const int mwarp = mt >> 5, lane = mt & 31;
@@ -1066,17 +1103,21 @@ __device__ __forceinline__ int atom_add_acq_rel_gpu(int *addr, int v) {
 // CTA that every other partial is visible.
 template <int ES, int RK, int RV, int D, int TT, int NTG>
 __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t u, const Range &rg,
-                         int slot, uint32_t parity, int mt) {
+                         int slot, uint32_t parity, int qs, int mt) {
     constexpr int WST = AsyncSizes<ES, RK, RV, D>::WST;
-    // The output's first pass of W_up,t^V travels while the run still streams: the set-up
-    // before this finish has read the staging buffer to the end and waited for its copies.
-    if (p.absorbed)
+    // The output's first pass of W_up,t^V travels while the run still streams.  Earlier uses of
+    // the staging buffer (a set-up's reads, a finish that returned with its copies in flight)
+    // are over before it is written again.
+    if (p.absorbed) {
+        cp_async_wait_all();
+        m_sync();
         m_stage_v<ES, RV, D, WST>(a, static_cast<const char *>(p.w_up_v) +
                                          (static_cast<int64_t>(R.h) * p.T + p.loop) * D * RV * ES,
                                   0, mt);
+    }
     mbar_wait(&a.stfull[slot], parity, a.s.abort_flag, p.err);
     const float *red = a.red + slot * a.redslot;
-    const float *lred = a.lred + slot * kComputeThreads;
+    const float *lred = a.lred + slot * kLredSlot;
     for (int j = mt; j < RV; j += kMThreads) {  // fixed order: bitwise-reproducible sums
         float acc = 0.f;
 #pragma unroll 4
@@ -1087,8 +1128,9 @@ __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t 
     for (int i = 0; i < TT; ++i) l += lred[i];
     const float m = a.s.misc[kAM + slot];
     m_sync();
+    mbar_arrive(&a.stfree[slot]);  // the run's state slot may take a later run's state
     if (u == R.seg_start && R.run_end == R.seg_end) {
-        m_output<ES, RK, RV, D>(p, a, R.b, R.h, m, l, slot, mt);
+        m_output<ES, RK, RV, D>(p, a, R.b, R.h, m, l, qs, mt);
         return;
     }
     const int c = blockIdx.x;
@@ -1179,7 +1221,7 @@ __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t 
         }
     }
     m_sync();
-    m_output<ES, RK, RV, D>(p, a, R.b, R.h, M, lsum, slot, mt);
+    m_output<ES, RK, RV, D>(p, a, R.b, R.h, M, lsum, qs, mt);
     if (mt == 0) atomicExch(counter, 0);
 }
 
@@ -1193,12 +1235,14 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
 
     pdl_wait();  // inputs may come from the previous kernel in the stream
     if (tid == 0) {
+        for (int i = 0; i < kQSlots; ++i) mbar_init(&a.qready[i], kMThreads);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&a.qready[i], kMThreads);
             mbar_init(&a.stfull[i], kComputeThreads);
+            mbar_init(&a.stfree[i], kMThreads);
         }
     }
-    const Range rg = prologue(p, s, F::S_THREADS, F::V_THREADS);  // fences the inits above too
+    Range rg = prologue(p, s, F::S_THREADS, F::V_THREADS);  // fences the inits above too
+    order_runs(p, s, rg);
     pdl_trigger();
 
     if (warp == kComputeWarps) {
@@ -1210,25 +1254,30 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
     if (tid >= kMBase) {
         // ---------------------------------------------------------------- management warps
         const int mt = tid - kMBase;
+        // set-ups run two runs ahead of finishes: set-up(r), then finish(r - 2), so that a short
+        // run is never followed by a wait for the next run's q~ behind a merge
+        auto finish = [&](const Run &R, int64_t u, int k) {
+            m_finish<ES, RK, RV, D, F::TT, F::NTG>(p, a, R, u, rg, k & 1, (k >> 1) & 1, k % kQSlots, mt);
+        };
         int r = 0;
-        Run prev{};
-        int64_t prev_u = 0;
-        for (int64_t u = rg.A0; u < rg.A1;) {
-            const Run R = locate_run(p, s, u, rg.A1);
-            const int slot = r & 1;
+        Run q0{}, q1{};  // runs r - 2 and r - 1, awaiting their finish
+        int64_t u0 = 0, u1 = 0;
+        for (int pass = 0; pass < 3; ++pass)
+        for (int64_t u = rg.lo[pass]; u < rg.hi[pass];) {
+            const Run R = locate_run(p, s, u, rg.hi[pass]);
+            const int slot = r % kQSlots;
             m_setup<ES, RK, RV, D>(p, a, R.b, R.h, slot, mt, r == 0);
             mbar_arrive(&a.qready[slot]);
-            if (r > 0)
-                m_finish<ES, RK, RV, D, F::TT, F::NTG>(p, a, prev, prev_u, rg, (r - 1) & 1,
-                                                       ((r - 1) >> 1) & 1, mt);
-            prev = R;
-            prev_u = u;
+            if (r >= 2) finish(q0, u0, r - 2);
+            q0 = q1;
+            u0 = u1;
+            q1 = R;
+            u1 = u;
             ++r;
             u = R.run_end;
         }
-        if (r > 0)
-            m_finish<ES, RK, RV, D, F::TT, F::NTG>(p, a, prev, prev_u, rg, (r - 1) & 1,
-                                                   ((r - 1) >> 1) & 1, mt);
+        if (r >= 2) finish(q0, u0, r - 2);
+        if (r >= 1) finish(q1, u1, r - 1);
         // sequences with no cached token: pass 1 attends to the current token only
         const bool pass1 = p.cur_k != nullptr;
         for (int b = 0; b < p.B; ++b) {
@@ -1256,14 +1305,16 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
 
     int it = 0, stage = 0, r = 0;
     uint32_t ph = 0;
-    for (int64_t u = rg.A0; u < rg.A1; ++r) {
-        const Run R = locate_run(p, s, u, rg.A1);
-        const int rslot = r & 1;
+    for (int pass = 0; pass < 3; ++pass)
+    for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
+        const Run R = locate_run(p, s, u, rg.hi[pass]);
+        const int rslot = r & 1;         // state slot
+        const int qslot = r % kQSlots;   // query slot
         float beta = 0.f;
-        const float *qq = a.qlat + rslot * a.qslot + ks * F::NGT * F::KE;
+        const float *qq = a.qlat + qslot * a.qslot + ks * F::NGT * F::KE;
         if (is_s) {
-            mbar_wait(&a.qready[rslot], (r >> 1) & 1, s.abort_flag, p.err);
-            beta = m_part(a, rslot, 1);
+            mbar_wait(&a.qready[qslot], (r / kQSlots) & 1, s.abort_flag, p.err);
+            beta = m_part(a, qslot, 1);
         }
         float m_run = -INFINITY, l_part = 0.f;
         float accv[AV];
@@ -1392,8 +1443,10 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
             }
         }
 
-        // leave the run's softmax state in slot rslot for the management warps
-        if (is_s && ks == 0) a.lred[rslot * kComputeThreads + tt] = l_part;
+        // leave the run's softmax state in slot rslot for the management warps, once the run
+        // that used the slot before (r - 2) has been read
+        if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
+        if (is_s && ks == 0) a.lred[rslot * kLredSlot + tt] = l_part;
         if (tid == 0) s.misc[kAM + rslot] = m_run;
         if (vwork) {
 #pragma unroll
@@ -1493,7 +1546,7 @@ lla_status decode_fits(int r_k, int r_v, int es, int d) {
     int fixed = make_layout(0, pps * hpb, LLA_MAX_BATCH, r_k, r_v, d).total;
     const FastEntry fe = d == 128 ? fast_entry(es, r_k, r_v) : FastEntry{nullptr, nullptr};
     if (fe.layout) fixed = fe.layout(0, pps * hpb, LLA_MAX_BATCH);
-    if ((kSmemLimit - fixed) / (pps * hpb) < 2) return LLA_ERR_UNSUPPORTED;
+    if ((kSmemLimit - fixed) / (pps * hpb + 16) < 2) return LLA_ERR_UNSUPPORTED;
     if (r_v * es / granule_bytes(r_v, es) > kComputeThreads) return LLA_ERR_UNSUPPORTED;
     return LLA_OK;
 }
@@ -1506,7 +1559,7 @@ lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream) {
     const FastEntry fe = a.d == 128 ? fast_entry(es, a.r_k, a.r_v) : FastEntry{nullptr, nullptr};
     const int fixed = fe.launch ? fe.layout(0, stage_bytes, a.B)
                                 : make_layout(0, stage_bytes, a.B, a.r_k, a.r_v, a.d).total;
-    int stages = (kSmemLimit - fixed) / stage_bytes;
+    int stages = (kSmemLimit - fixed) / (stage_bytes + 16);  // + its full and empty barriers
     if (stages > kMaxStages) stages = kMaxStages;
     if (stages < 2) return LLA_ERR_UNSUPPORTED;
     const int smem = fe.launch ? fe.layout(stages, stage_bytes, a.B)
