@@ -11,6 +11,8 @@ longest sequence and four more, each at three heads.
     sampled rows, max abs <= 2e-2 (bf16 output).
   * encode: for the sampled (sequence, head) pairs, 64 positions spread over the context are
     re-encoded by the oracle from the same inputs and compared with the stored latents.
+  * prefill: the rho = 2 workload's prompts (4 x 8192 tokens), sampled rows checked as pass-2
+    decodes of their causal prefixes.
 """
 import numpy as np
 import pytest
@@ -98,3 +100,56 @@ def test_full_size_decode_and_encode_sampled(wname, loop):
             assert_parity(c_k[positions], ek, "bf16", f"{wname} c_k b{b} h{h}")
             assert_parity(c_v[positions], ev, "bf16", f"{wname} c_v b{b} h{h}")
     assert_parity(np.stack(got_rows), np.stack(ref_rows), "bf16", f"{wname} decode loop {loop}")
+
+
+def test_full_size_prefill_sampled_rows():
+    """Causal prefill at the benchmark's prompt size (Ouro-1.4B at rho = 2: 4 prompts of 8192
+    tokens, 16 heads), in the launch configuration bench.py times.  Row i of a prompt is the
+    pass-2 decode of query i over keys 0..i, so sampled rows are checked with the oracle's decode
+    on the latents the GPU stored (first and last rows, rows on tile and page boundaries, and
+    random rows), against the bf16 bound taken before the output's own rounding."""
+    ensure_library()
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+
+    dev = torch.device(DEV, 0)
+    w = W.WORKLOADS["ouro14_rho2"]
+    nseq, L = w.prefill
+    T, H, d = w.T, w.H, w.d
+    geom = lla.Geometry(T, H, d, w.r_k, w.r_v, "bf16")
+    cod = W.codec_tensors(T, H, d, w.r_k, w.r_v, w.seed, 0, device=dev)
+    codec = lla.Codec(**cod)
+    lens = [L] * nseq
+    pt = W.page_table(lens, w.seed, extra_tokens=0)
+    bb = lla.lla_cache_block_bytes(geom)
+    pool = torch.zeros(pt.num_blocks * bb, dtype=torch.uint8, device=dev)
+    cache = lla.Cache(pool, pt.num_blocks, pt.block_table.to(dev), pt.max_blocks)
+    N = nseq * L
+    slots = torch.cat([pt.slots(b, range(L)) for b in range(nseq)]).to(dev)
+    lla.lla_encode(geom, codec, cache, W.normal((T, N, H, d), w.seed, 300, device=dev),
+                   W.normal((T, N, H, d), w.seed, 301, device=dev), slots)
+    q = W.normal((N, H, d), w.seed, 302, device=dev)
+    out = torch.empty_like(q)
+    cu = torch.tensor([i * L for i in range(nseq + 1)], dtype=torch.int32, device=dev)
+    lla.lla_clear_device_error()
+    loop = 1
+    lla.lla_prefill_attn(geom, codec, cache, cu, L, loop, q, out)
+    torch.cuda.synchronize()
+    assert lla.lla_get_device_error() == 0
+    w64 = {k: (None if v is None else f64(v)) for k, v in cod.items()}
+    scale = 1.0 / np.sqrt(d)
+    rng = np.random.default_rng(11)
+    rows = sorted({0, 1, 63, 64, 127, 128, 129, 4095, 4096, L - 2, L - 1} |
+                  set(int(x) for x in rng.integers(0, L, 6)))
+    got, ref = [], []
+    for b, h in ((0, 0), (3, 15), (1, 7)):
+        pages, table = _compact_pages(pool, pt.block_table[b], L, bb)
+        c_k, c_v = unpack_head(pages, H, w.r_k, w.r_v, "bf16", table, L, h)
+        qb = f64(q[b * L:(b + 1) * L, h])
+        ob = f64(out[b * L:(b + 1) * L, h])
+        for i in rows:
+            ref.append(oracle.decode(loop, c_k[:i + 1], c_v[:i + 1], w64["w_up_k"][h], w64["w_up_v"][h],
+                                     None, None, qb[i], None, None, scale))
+            got.append(ob[i])
+    assert_parity(np.stack(got), np.stack(ref), "bf16", "full-size prefill rows", io="bf16",
+                  output_rounding=True)
