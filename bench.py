@@ -482,35 +482,66 @@ def run_extras(device):
 
 def run_e2e(bench, args, world):
     """Same step with the step's inputs (q, k_cur, v_cur of every call) copied from pinned
-    host memory and the outputs copied back, inside the timed region."""
+    host memory and the outputs copied back, inside the timed region.  Inputs and outputs are
+    double-buffered on the device: one stream copies step k+1's inputs in and another copies
+    step k-1's outputs out while step k computes."""
     import torch
     import torch.distributed as dist
 
     q_h = bench.q.cpu().pin_memory()
     k_h = bench.cur_k.cpu().pin_memory()
     v_h = bench.cur_v.cpu().pin_memory()
-    o_h = torch.empty(bench.out.shape, dtype=bench.out.dtype).pin_memory()
-    stream = torch.cuda.current_stream()
+    o_h = [torch.empty(bench.out.shape, dtype=bench.out.dtype).pin_memory() for _ in range(2)]
+    bufs = [(bench.q, bench.cur_k, bench.cur_v, bench.out),
+            tuple(torch.empty_like(t) for t in (bench.q, bench.cur_k, bench.cur_v, bench.out))]
+    main = torch.cuda.current_stream()
+    copy = torch.cuda.Stream(device=bench.device)    # inputs in
+    copy_out = torch.cuda.Stream(device=bench.device)  # outputs out
     K = max(1, args.steps)
+    ev = lambda: torch.cuda.Event()
 
-    def one():
-        bench.q.copy_(q_h, non_blocking=True)
-        bench.cur_k.copy_(k_h, non_blocking=True)
-        bench.cur_v.copy_(v_h, non_blocking=True)
-        bench.step()
-        o_h.copy_(bench.out, non_blocking=True)
+    def run(nsteps):
+        copy.wait_stream(main)  # nothing on the copy streams starts before the timed region
+        copy_out.wait_stream(main)
+        copied = [None, None]   # inputs of the step using buffer i are on the device
+        done = [None, None]     # the step using buffer i has finished computing
+        drained = [None, None]  # the outputs of buffer i have been copied out
+        for k in range(nsteps):
+            i = k & 1
+            q, ck, cv, out = bufs[i]
+            with torch.cuda.stream(copy):
+                if done[i] is not None:
+                    copy.wait_event(done[i])       # step k-2 no longer reads these inputs
+                q.copy_(q_h, non_blocking=True)
+                ck.copy_(k_h, non_blocking=True)
+                cv.copy_(v_h, non_blocking=True)
+                copied[i] = ev()
+                copied[i].record(copy)
+            main.wait_event(copied[i])
+            if drained[i] is not None:
+                main.wait_event(drained[i])        # step k-2's outputs have left the buffer
+            bench.q, bench.cur_k, bench.cur_v, bench.out = q, ck, cv, out
+            bench.step()
+            done[i] = ev()
+            done[i].record(main)
+            with torch.cuda.stream(copy_out):
+                copy_out.wait_event(done[i])
+                o_h[i].copy_(out, non_blocking=True)
+                drained[i] = ev()
+                drained[i].record(copy_out)
+        main.wait_stream(copy)
+        main.wait_stream(copy_out)
 
-    for _ in range(max(1, args.warmup)):
-        one()
+    run(max(1, args.warmup))
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    for _ in range(K):
-        one()
-    b.record(stream)
+    a.record(main)
+    run(K)
+    b.record(main)
     torch.cuda.synchronize()
+    bench.q, bench.cur_k, bench.cur_v, bench.out = bufs[0]
     ms = a.elapsed_time(b)
     if world > 1:
         t = torch.tensor([ms], dtype=torch.float64, device=bench.device)
@@ -519,7 +550,9 @@ def run_e2e(bench, args, world):
     nbytes = lambda t: t.numel() * t.element_size()
     return {"value": world * bench.B / (ms / K / 1e3), "unit": "tokens/s",
             "h2d_bytes_per_step": nbytes(q_h) + nbytes(k_h) + nbytes(v_h),
-            "d2h_bytes_per_step": nbytes(o_h), "ms_per_step": ms / K}
+            "d2h_bytes_per_step": nbytes(o_h[0]), "ms_per_step": ms / K,
+            "copies": "double-buffered; inputs and outputs on their own streams, overlapping the "
+                      "neighbouring steps"}
 
 
 # ----------------------------------------------------------------- oracle (CPU) timing
