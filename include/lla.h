@@ -127,6 +127,22 @@ lla_status lla_encode(const lla_geometry *g, const lla_codec *codec, const lla_c
                       const void *x_k, const void *x_v, lla_dtype x_dtype,
                       const int64_t *slot_mapping, int32_t N, void *stream);
 
+/*
+ * lla_encode for L layers in one call (one launch for a decode batch): the completed tokens of
+ * a step are encoded in every layer at once, instead of one launch per layer.  The paper has no
+ * counterpart; this is a scheduling convenience over Eq. encode (Sec. 3).
+ *   codecs, caches  host arrays of L structs: layer l's codec and cache (same geometry)
+ *   x_k, x_v        host arrays of L device pointers: layer l's [T][N][H][d] inputs in x_dtype,
+ *                   16-byte aligned
+ *   slot_mapping    device [N] int64, the same slots in every layer (one page table)
+ * L <= 64 (LLA_ERR_UNSUPPORTED beyond); L = 0 or N = 0 is a valid no-op.  Results are those of
+ * L lla_encode calls.
+ */
+lla_status lla_encode_layers(const lla_geometry *g, int32_t L, const lla_codec *codecs,
+                             const lla_cache *caches, const void *const *x_k,
+                             const void *const *x_v, lla_dtype x_dtype,
+                             const int64_t *slot_mapping, int32_t N, void *stream);
+
 /* Workspace bytes lla_decode_attn needs for a batch of B sequences on the current device. */
 lla_status lla_decode_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes);
 

@@ -127,6 +127,38 @@ lla_status lla_encode(const lla_geometry *g, const lla_codec *codec, const lla_c
     return launch_encode(a, static_cast<cudaStream_t>(stream));
 }
 
+lla_status lla_encode_layers(const lla_geometry *g, int32_t L, const lla_codec *codecs,
+                             const lla_cache *caches, const void *const *x_k,
+                             const void *const *x_v, lla_dtype x_dtype,
+                             const int64_t *slot_mapping, int32_t N, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (L < 0 || !valid_dtype(x_dtype) || N < 0) return LLA_ERR_INVALID_ARG;
+    if (L == 0 || N == 0) return LLA_OK;
+    if (L > kMaxEncodeLayers) return LLA_ERR_UNSUPPORTED;
+    if (!codecs || !caches || !x_k || !x_v || !slot_mapping) return LLA_ERR_INVALID_ARG;
+    EncodeArgs a[kMaxEncodeLayers];
+    for (int l = 0; l < L; ++l) {
+        const lla_codec *codec = &codecs[l];
+        if (!codec->w_down_k || !codec->w_down_v) return LLA_ERR_INVALID_ARG;
+        if ((st = check_cache(&caches[l], false)) != LLA_OK) return st;
+        if (!x_k[l] || !x_v[l]) return LLA_ERR_INVALID_ARG;
+        if (!aligned(codec->w_down_k, 16) || !aligned(codec->w_down_v, 16)) return LLA_ERR_INVALID_ARG;
+        if (!aligned(x_k[l], 16) || !aligned(x_v[l], 16)) return LLA_ERR_INVALID_ARG;
+        a[l] = EncodeArgs{};
+        a[l].T = g->T; a[l].H = g->H; a[l].d = g->d; a[l].r_k = g->r_k; a[l].r_v = g->r_v;
+        a[l].storage_bf16 = g->storage == LLA_BF16;
+        a[l].x_bf16 = x_dtype == LLA_BF16;
+        a[l].w_down_k = codec->w_down_k; a[l].w_down_v = codec->w_down_v;
+        a[l].mu_k = codec->mu_k; a[l].mu_v = codec->mu_v;
+        a[l].x_k = x_k[l]; a[l].x_v = x_v[l];
+        a[l].pool = caches[l].pool; a[l].num_blocks = caches[l].num_blocks;
+        a[l].slot_mapping = slot_mapping; a[l].N = N;
+        a[l].dense = 0;
+    }
+    return launch_encode_layers(a, L, static_cast<cudaStream_t>(stream));
+}
+
 lla_status lla_decode_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes) {
     lla_status st = check_geometry(g);
     if (st != LLA_OK) return st;

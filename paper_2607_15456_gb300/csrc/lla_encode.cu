@@ -42,6 +42,7 @@ struct EncParams {
     int head_page_bytes, kplane_bytes;
     const int64_t *slot_mapping;
     int N, tile, ctiles_k;
+    int nbuf;  // W_down chunk buffers: 1 when T*d fits one chunk, else 2
     unsigned *err;
 };
 
@@ -82,17 +83,16 @@ __device__ __forceinline__ void stage_w(char *wb, const char *W, int r, int col0
 }
 
 template <int ES>
-__global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
+__device__ __forceinline__ void encode_body(const EncParams &p, const int h) {
     extern __shared__ __align__(16) float smem_f[];
     constexpr int KC = chunk_rows<ES>();
     const int Td = p.T * p.d;
     float *xs = smem_f;                                       // [tile][Td] centred stacked vectors
     char *wbuf = reinterpret_cast<char *>(xs + p.tile * Td);  // [2][KC][kColTile] W_down chunks
-    float *red = reinterpret_cast<float *>(wbuf + 2 * kWBuf);  // [kKSlices][tile][kColTile]
+    float *red = reinterpret_cast<float *>(wbuf + p.nbuf * kWBuf);  // [kKSlices][tile][kColTile]
     const int ct = blockIdx.y;
     const int axis = ct < p.ctiles_k ? 0 : 1;
     const int col0 = (axis ? ct - p.ctiles_k : ct) * kColTile;
-    const int h = blockIdx.z;
     const int n0 = blockIdx.x * p.tile;
     const int nt = min(p.tile, p.N - n0);
     const int r = axis ? p.r_v : p.r_k;
@@ -234,6 +234,41 @@ __global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
     }
 }
 
+template <int ES>
+__global__ void __launch_bounds__(kThreads) encode_kernel(const EncParams p) {
+    encode_body<ES>(p, blockIdx.z);
+}
+
+// Several layers in one launch: blockIdx.z = layer * H + head; each layer's pointers come from
+// a table in the kernel parameters.
+struct EncLayer {
+    const void *w_down_k, *w_down_v;
+    const float *mu_k, *mu_v;
+    const void *x_k, *x_v;
+    char *pool;
+    int64_t num_blocks;
+};
+struct EncLayers {
+    EncLayer l[kMaxEncodeLayers];
+};
+
+template <int ES>
+__global__ void __launch_bounds__(kThreads) encode_layers_kernel(const EncParams p0,
+                                                                  const __grid_constant__ EncLayers t) {
+    const int layer = blockIdx.z / p0.H;
+    EncParams p = p0;
+    const EncLayer &e = t.l[layer];
+    p.w_down_k = e.w_down_k;
+    p.w_down_v = e.w_down_v;
+    p.mu_k = e.mu_k;
+    p.mu_v = e.mu_v;
+    p.x_k = e.x_k;
+    p.x_v = e.x_v;
+    p.pool = e.pool;
+    p.num_blocks = e.num_blocks;
+    encode_body<ES>(p, blockIdx.z - layer * p0.H);
+}
+
 // Plain K/V store for the uncompressed comparator: k, v [N][H][d] -> K-plane / V-plane of the
 // token's slot (r_k = r_v = d).
 template <int ES>
@@ -275,6 +310,18 @@ lla_status launch(K kern, dim3 grid, dim3 block, int smem, cudaStream_t stream, 
 }
 
 template <int ES>
+lla_status set_smem_layers(int dev) {
+    static bool configured[64] = {};
+    if (dev < 64 && configured[dev]) return LLA_OK;
+    if (cudaFuncSetAttribute(encode_layers_kernel<ES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kXsBudget + 2 * kWBuf + kKSlices * kMaxTileTokens * kColTile * 4) !=
+        cudaSuccess)
+        return LLA_ERR_CUDA;
+    if (dev < 64) configured[dev] = true;
+    return LLA_OK;
+}
+
+template <int ES>
 lla_status set_smem(int dev) {
     static bool configured[64] = {};
     if (dev < 64 && configured[dev]) return LLA_OK;
@@ -287,6 +334,63 @@ lla_status set_smem(int dev) {
 }
 
 }  // namespace
+
+lla_status launch_encode_layers(const EncodeArgs *a, int L, cudaStream_t stream) {
+    if (L <= 0 || a[0].N == 0) return LLA_OK;
+    const EncodeArgs &a0 = a[0];
+    // prompts take the tensor-core kernel layer by layer; decode batches share one launch
+    if (encode_tc_supported(a0) || a0.dense || L > kMaxEncodeLayers) {
+        for (int l = 0; l < L; ++l) {
+            const lla_status st = launch_encode(a[l], stream);
+            if (st != LLA_OK) return st;
+        }
+        return LLA_OK;
+    }
+    const int es = a0.storage_bf16 ? 2 : 4;
+    lla_status st = LLA_OK;
+    unsigned *err = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    EncParams p = {};
+    p.T = a0.T; p.H = a0.H; p.d = a0.d; p.r_k = a0.r_k; p.r_v = a0.r_v; p.x_bf16 = a0.x_bf16;
+    p.head_page_bytes = static_cast<int>(head_page_bytes(a0.r_k, a0.r_v, es));
+    p.block_bytes = static_cast<int64_t>(p.head_page_bytes) * a0.H;
+    p.kplane_bytes = LLA_BLOCK_TOKENS * a0.r_k * es;
+    p.slot_mapping = a0.slot_mapping;
+    p.N = a0.N;
+    p.err = err;
+    EncLayers t = {};
+    for (int l = 0; l < L; ++l)
+        t.l[l] = EncLayer{a[l].w_down_k, a[l].w_down_v, a[l].mu_k, a[l].mu_v, a[l].x_k, a[l].x_v,
+                          static_cast<char *>(a[l].pool), a[l].num_blocks};
+    const int Td = a0.T * a0.d;
+    int tile = kXsBudget / (Td * 4);
+    if (tile > kMaxTileTokens) tile = kMaxTileTokens;
+    if (tile < 1) return LLA_ERR_UNSUPPORTED;
+    p.tile = tile;
+    p.ctiles_k = (a0.r_k + kColTile - 1) / kColTile;
+    p.nbuf = Td > (es == 2 ? chunk_rows<2>() : chunk_rows<4>()) ? 2 : 1;
+    const int ctiles_v = (a0.r_v + kColTile - 1) / kColTile;
+    const int smem = (tile * Td + kKSlices * tile * kColTile) * 4 + p.nbuf * kWBuf;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
+    st = es == 2 ? set_smem_layers<2>(dev) : set_smem_layers<4>(dev);
+    if (st != LLA_OK) return st;
+    if (static_cast<int64_t>(a0.H) * L > 65535) return LLA_ERR_UNSUPPORTED;
+    const dim3 grid((a0.N + tile - 1) / tile, p.ctiles_k + ctiles_v, a0.H * L), block(kThreads);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = es == 2 ? cudaLaunchKernelEx(&cfg, encode_layers_kernel<2>, p, t)
+                                  : cudaLaunchKernelEx(&cfg, encode_layers_kernel<4>, p, t);
+    return e == cudaSuccess ? LLA_OK : LLA_ERR_CUDA;
+}
 
 lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream) {
     if (a.N == 0) return LLA_OK;
@@ -318,8 +422,9 @@ lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream) {
     if (tile < 1) return LLA_ERR_UNSUPPORTED;
     p.tile = tile;
     p.ctiles_k = (a.r_k + kColTile - 1) / kColTile;
+    p.nbuf = Td > (es == 2 ? chunk_rows<2>() : chunk_rows<4>()) ? 2 : 1;
     const int ctiles_v = (a.r_v + kColTile - 1) / kColTile;
-    const int smem = (tile * Td + kKSlices * tile * kColTile) * 4 + 2 * kWBuf;
+    const int smem = (tile * Td + kKSlices * tile * kColTile) * 4 + p.nbuf * kWBuf;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     st = es == 2 ? set_smem<2>(dev) : set_smem<4>(dev);

@@ -72,6 +72,9 @@ lla_status decode_fits(int r_k, int r_v, int es, int d);  // UNSUPPORTED if no k
 lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream);
 
 lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream);
+// The same encode for L layers (one launch for decode batches).
+constexpr int kMaxEncodeLayers = 64;
+lla_status launch_encode_layers(const EncodeArgs *a, int L, cudaStream_t stream);
 // Tensor-core encode for prompts (bf16 x and storage, N >= 128, instantiated ranks).
 bool encode_tc_supported(const EncodeArgs &a);
 lla_status launch_encode_tc(const EncodeArgs &a, cudaStream_t stream);

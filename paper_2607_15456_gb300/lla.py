@@ -69,6 +69,7 @@ def library() -> ctypes.CDLL:
             "lla_version": (I32, []),
             "lla_cache_block_bytes": (I32, [P, P]),
             "lla_encode": (I32, [P, P, P, P, P, I32, P, I32, P]),
+            "lla_encode_layers": (I32, [P, I32, P, P, P, P, I32, P, I32, P]),
             "lla_decode_workspace_size": (I32, [P, I32, P]),
             "lla_decode_workspace_init": (I32, [P, SZ, P]),
             "lla_decode_attn": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ, P]),
@@ -190,6 +191,24 @@ def lla_encode(geom: Geometry, codec: Codec, cache: Cache, x_k: torch.Tensor, x_
     _check("lla_encode", library().lla_encode(
         ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(x_k), _ptr(x_v),
         _dtype_code(x_k), _ptr(slot_mapping), N, _stream(stream)))
+
+
+def lla_encode_layers(geom: Geometry, codecs, caches, x_k, x_v, slot_mapping: torch.Tensor,
+                      stream=None) -> None:
+    """The same encode in several layers at once: codecs, caches, x_k, x_v are per-layer lists
+    (x_k[l], x_v[l] [T][N][H][d]); slot_mapping [N] int64 is shared."""
+    L = len(codecs)
+    if not (len(caches) == len(x_k) == len(x_v) == L):
+        raise ValueError("one codec, cache and input pair per layer")
+    g = geom.c()
+    cds = (lla_codec * max(L, 1))(*[c.c() for c in codecs])
+    chs = (lla_cache * max(L, 1))(*[c.c() for c in caches])
+    xk = (ctypes.c_void_p * max(L, 1))(*[_ptr(t) for t in x_k])
+    xv = (ctypes.c_void_p * max(L, 1))(*[_ptr(t) for t in x_v])
+    N = x_k[0].shape[1] if L and x_k[0].dim() == 4 else 0
+    _check("lla_encode_layers", library().lla_encode_layers(
+        ctypes.byref(g), L, cds, chs, xk, xv, _dtype_code(x_k[0]) if L else 0, _ptr(slot_mapping), N,
+        _stream(stream)))
 
 
 def lla_decode_workspace_size(geom: Geometry, B: int) -> int:

@@ -170,3 +170,28 @@ def test_prefill_argument_checks(lib):
 
 def test_workspace_init_rejects_null(lib):
     assert lib.library().lla_decode_workspace_init(None, 16, None) == INVALID
+
+
+def test_encode_layers_argument_checks(lib):
+    so = lib.library()
+    g = _g(lib)
+    L = 2
+    codecs = (lib.lla_codec * L)(*[_codec(lib) for _ in range(L)])
+    caches = (lib.lla_cache * L)(*[_cache(lib) for _ in range(L)])
+    ptrs = (ctypes.c_void_p * L)(FAKE, FAKE)
+
+    def enc(L=2, codecs=codecs, caches=caches, xk=ptrs, xv=ptrs, slots=FAKE, N=8, xd=0):
+        return so.lla_encode_layers(ctypes.byref(g), L, codecs, caches, xk, xv, xd, slots, N, None)
+
+    assert enc(L=0, codecs=None, caches=None, xk=None, xv=None, slots=None) == OK  # no layers
+    assert enc(N=0) == OK
+    assert enc(L=65) == UNSUPPORTED
+    assert enc(L=-1) == INVALID
+    assert enc(codecs=None) == INVALID
+    assert enc(xk=None) == INVALID
+    assert enc(slots=None) == INVALID
+    assert enc(xd=5) == INVALID
+    bad = (ctypes.c_void_p * L)(FAKE, FAKE + 8)  # layer 1's input not 16-byte aligned
+    assert enc(xv=bad) == INVALID
+    nocodec = (lib.lla_codec * L)(_codec(lib), _codec(lib, w_down_v=None))
+    assert enc(codecs=nocodec) == INVALID

@@ -95,3 +95,34 @@ def test_encode_prompt_on_tensor_cores(lla, r_k, r_v, with_mu):
 def test_encode_prompt_long_reduction_on_tensor_cores(lla):
     # T*d = 16 * 256 = 4096: 64 slabs of the reduction axis through the stage ring
     _encode_and_compare(lla, 16, 2, 256, 96, 160, "bf16", "bf16", [150], True, 8)
+
+
+@pytest.mark.parametrize("N,storage", [(16, "bf16"), (16, "fp32"), (200, "bf16")])
+def test_encode_layers_equals_per_layer_calls(lla, N, storage):
+    """lla_encode_layers writes exactly what one lla_encode call per layer writes (one launch
+    for a decode batch; prompts go layer by layer through the tensor-core kernel)."""
+    from paper_2607_15456_gb300 import workloads as W
+    T, H, d, r_k, r_v, L = 4, 16, 128, 96, 160, 3
+    geom = lla.Geometry(T, H, d, r_k, r_v, storage)
+    pt = W.page_table([N], 9, extra_tokens=0)
+    bb = lla.lla_cache_block_bytes(geom)
+    slots = pt.slots(0, range(N)).to(DEV)
+    table = pt.block_table.to(DEV)
+    codecs, caches_a, caches_b, xs_k, xs_v, pools = [], [], [], [], [], []
+    for l in range(L):
+        cod = W.codec_tensors(T, H, d, r_k, r_v, 9, l, dtype=_dt(storage), device=DEV, with_mu=(l == 1))
+        codecs.append(lla.Codec(**cod))
+        for lst in (caches_a, caches_b):
+            pool = torch.full((pt.num_blocks * bb,), 0xFF, dtype=torch.uint8, device=DEV)
+            pools.append(pool)
+            lst.append(lla.Cache(pool, pt.num_blocks, table, pt.max_blocks))
+        xs_k.append(W.normal((T, N, H, d), 9, 50, l, device=DEV))
+        xs_v.append(W.normal((T, N, H, d), 9, 51, l, device=DEV))
+    lla.lla_clear_device_error()
+    lla.lla_encode_layers(geom, codecs, caches_a, xs_k, xs_v, slots)
+    for l in range(L):
+        lla.lla_encode(geom, codecs[l], caches_b[l], xs_k[l], xs_v[l], slots)
+    torch.cuda.synchronize()
+    assert lla.lla_get_device_error() == 0
+    for l in range(L):
+        assert torch.equal(caches_a[l].pool, caches_b[l].pool), l
