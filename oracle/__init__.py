@@ -20,6 +20,10 @@ calls it through ctypes.  Citations (paper sections and equations):
                                        decoder (App. A, "Decoding and caching")
 * ``prefill``                       -- causal pass-2 prefill over latents (App. A; App. J,
                                        "Eviction and long-context prefill")
+* ``rope``                          -- rotary position embedding (RoFormer), applied after
+                                       reconstruction (Sec. 3, "RoPE and reconstruction")
+* ``decode_rope``, ``prefill_rope`` -- ``decode`` / ``prefill`` with every reconstructed key
+                                       and the query rotated at their token positions
 
 Parity status of every function: pinned (see ``tests/test_oracle_pins.py``).
 """
@@ -59,6 +63,14 @@ def _load():
         lib.lla_oracle_decode.argtypes = [i32, i32, i32, i32, i32, i64] + [p] * 9 + [d, p]
         lib.lla_oracle_prefill.restype = i32
         lib.lla_oracle_prefill.argtypes = [i32, i32, i32, i32, i32, i64] + [p] * 7 + [d, p]
+        lib.lla_oracle_rope.restype = None
+        lib.lla_oracle_rope.argtypes = [i32, i32, d, i64, p, p]
+        lib.lla_oracle_decode_rope.restype = i32
+        lib.lla_oracle_decode_rope.argtypes = ([i32, i32, i32, i32, i32, i64] + [p] * 9 +
+                                               [d, i32, d, i64, p])
+        lib.lla_oracle_prefill_rope.restype = i32
+        lib.lla_oracle_prefill_rope.argtypes = ([i32, i32, i32, i32, i32, i64] + [p] * 7 +
+                                                [d, i32, d, i64, p])
         lib.lla_oracle_decode_batch.restype = i32
         lib.lla_oracle_decode_batch.argtypes = [i32, i32, i32, i32, d, i64, p, i32]
         lib.lla_oracle_encode_batch.restype = i32
@@ -175,10 +187,72 @@ def prefill(t: int, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, scale: float) -> np
     return out
 
 
+# ---------------------------------------------------------------- rotary positions (Sec. 3)
+
+ROPE_HALF, ROPE_ADJACENT = 0, 1  # pair j = (x[j], x[j + d/2])  or  (x[2j], x[2j + 1])
+
+
+def rope(x, pos: int, base: float = 10000.0, pairing: int = ROPE_HALF) -> np.ndarray:
+    """RoFormer rotation of x [d] at integer position pos: pair j turned by pos * base^(-2j/d)."""
+    x = _f64(x)
+    d = x.shape[-1]
+    assert x.ndim == 1 and d % 2 == 0
+    y = np.zeros(d, dtype=np.float64)
+    _load().lla_oracle_rope(d, pairing, base, pos, _ptr(x), _ptr(y))
+    return y
+
+
+def decode_rope(t: int, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, cur_k, cur_v, scale: float,
+                base: float = 10000.0, pairing: int = ROPE_HALF, pos0: int = 0) -> np.ndarray:
+    """``decode`` with RoPE after reconstruction: cached token i at position pos0 + i, the
+    current token (and the query) at pos0 + L in pass 1 and pos0 + L - 1 in pass 2."""
+    w_up_k, w_up_v = _f64(w_up_k), _f64(w_up_v)
+    T, d, r_k = w_up_k.shape
+    r_v = w_up_v.shape[2]
+    c_k = _f64(c_k).reshape(-1, r_k)
+    c_v = _f64(c_v).reshape(-1, r_v)
+    L = c_k.shape[0]
+    mu_k = None if mu_k is None else _f64(mu_k).reshape(T * d)
+    mu_v = None if mu_v is None else _f64(mu_v).reshape(T * d)
+    q = _f64(q).reshape(d)
+    cur_k = None if cur_k is None else _f64(cur_k).reshape(d)
+    cur_v = None if cur_v is None else _f64(cur_v).reshape(d)
+    out = np.zeros(d, dtype=np.float64)
+    rc = _load().lla_oracle_decode_rope(T, d, r_k, r_v, t, L, _ptr(c_k), _ptr(c_v),
+                                        _ptr(w_up_k), _ptr(w_up_v), _ptr(mu_k), _ptr(mu_v),
+                                        _ptr(q), _ptr(cur_k), _ptr(cur_v), scale, pairing, base,
+                                        pos0, _ptr(out))
+    if rc:
+        raise ValueError("bad decode arguments")
+    return out
+
+
+def prefill_rope(t: int, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, scale: float,
+                 base: float = 10000.0, pairing: int = ROPE_HALF, pos0: int = 0) -> np.ndarray:
+    """``prefill`` with RoPE after reconstruction: prompt token i at position pos0 + i."""
+    w_up_k, w_up_v = _f64(w_up_k), _f64(w_up_v)
+    T, d, r_k = w_up_k.shape
+    r_v = w_up_v.shape[2]
+    c_k = _f64(c_k).reshape(-1, r_k)
+    c_v = _f64(c_v).reshape(-1, r_v)
+    N = c_k.shape[0]
+    mu_k = None if mu_k is None else _f64(mu_k).reshape(T * d)
+    mu_v = None if mu_v is None else _f64(mu_v).reshape(T * d)
+    q = _f64(q).reshape(N, d)
+    out = np.zeros((N, d), dtype=np.float64)
+    rc = _load().lla_oracle_prefill_rope(T, d, r_k, r_v, t, N, _ptr(c_k), _ptr(c_v),
+                                         _ptr(w_up_k), _ptr(w_up_v), _ptr(mu_k), _ptr(mu_v),
+                                         _ptr(q), scale, pairing, base, pos0, _ptr(out))
+    if rc:
+        raise ValueError("bad prefill arguments")
+    return out
+
+
 # ---------------------------------------------------------------- batched drivers (OpenMP)
 
 class _DecodeItem(ctypes.Structure):
-    _fields_ = [("t", ctypes.c_int32), ("pad_", ctypes.c_int32), ("L", ctypes.c_int64)] + [
+    _fields_ = [("t", ctypes.c_int32), ("rope", ctypes.c_int32), ("L", ctypes.c_int64),
+                ("rope_base", ctypes.c_double)] + [
         (n, ctypes.c_void_p) for n in
         ("c_k", "c_v", "w_up_k", "w_up_v", "mu_k", "mu_v", "q", "cur_k", "cur_v", "out")]
 
@@ -195,8 +269,9 @@ def max_threads() -> int:
 def decode_batch(T: int, d: int, r_k: int, r_v: int, scale: float, items: Sequence[dict],
                  n_threads: int = 0) -> list:
     """Runs independent decode problems side by side.  Each item is a dict with keys
-    t, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, cur_k, cur_v (arrays as in ``decode``).
-    Returns the list of outputs [d]."""
+    t, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, cur_k, cur_v (arrays as in ``decode``) and an
+    optional ``rope`` = (pairing, base), which makes the item a ``decode_rope`` problem with
+    pos0 = 0.  Returns the list of outputs [d]."""
     keep, outs = [], []
     arr = (_DecodeItem * len(items))()
     for k, it in enumerate(items):
@@ -210,6 +285,9 @@ def decode_batch(T: int, d: int, r_k: int, r_v: int, scale: float, items: Sequen
         out = np.zeros(d, dtype=np.float64)
         outs.append(out)
         arr[k].t = it["t"]
+        if it.get("rope") is not None:
+            arr[k].rope = int(it["rope"][0]) + 1
+            arr[k].rope_base = float(it["rope"][1])
         arr[k].L = _f64(it["c_k"]).size // r_k
         for name, v in fields.items():
             setattr(arr[k], name, v)
@@ -242,5 +320,6 @@ def encode_batch(T: int, d: int, items: Sequence[dict], n_threads: int = 0) -> l
 
 
 __all__ = ["ratio", "teacher_cache_bytes_per_token", "latent_cache_bytes_per_token", "encode",
-           "reconstruct", "attention", "decode", "prefill", "decode_batch", "encode_batch",
+           "reconstruct", "attention", "decode", "prefill", "rope", "decode_rope",
+           "prefill_rope", "ROPE_HALF", "ROPE_ADJACENT", "decode_batch", "encode_batch",
            "max_threads", "build_oracle", "library_path"]

@@ -14,6 +14,10 @@
  * and softmax attention over the explicitly reconstructed keys and values:
  *   s_i = scale * q . Khat_t[i],  a = softmax(s),  o = sum_i a_i Vhat_t[i].
  *
+ * Rotary positions (RoFormer) are applied after reconstruction when asked for (Sec. 3 "RoPE
+ * and reconstruction"): the codec works on pre-RoPE keys, and each reconstructed key is rotated
+ * at its token's position before the dot product with the rotated query.
+ *
  * Decode follows the two-pass cached reconstruction decoder (App. A, "Decoding and
  * caching"): in pass 1 the current token's stacked vector is not complete yet, so at loop t
  * it attends with its own exact loop-t key and value; in pass 2 the current token has been
@@ -140,6 +144,26 @@ int lla_oracle_attention(int d, int64_t L, const double *q, const double *K, con
 }
 
 /*
+ * The keys and values one loop-t query attends to: Khat_t and Vhat_t of the L cached tokens
+ * by Eq. decode, in rows 0 .. L-1 of K and V [L + 1][d]; in pass 1 (cur_k, cur_v not NULL) the
+ * current token's exact loop-t key and value as row L.
+ */
+static void loop_keys_values(int d, int r_k, int r_v, int t, int64_t L, const double *c_k,
+                             const double *c_v, const double *w_up_k, const double *w_up_v,
+                             const double *mu_k, const double *mu_v, const double *cur_k,
+                             const double *cur_v, double *K, double *V)
+{
+    lla_oracle_reconstruct(d, r_k, L, c_k, w_up_k + (int64_t)t * d * r_k,
+                           mu_k ? mu_k + (int64_t)t * d : NULL, K);
+    lla_oracle_reconstruct(d, r_v, L, c_v, w_up_v + (int64_t)t * d * r_v,
+                           mu_v ? mu_v + (int64_t)t * d : NULL, V);
+    if (cur_k) {
+        memcpy(K + L * d, cur_k, sizeof(double) * (size_t)d);
+        memcpy(V + L * d, cur_v, sizeof(double) * (size_t)d);
+    }
+}
+
+/*
  * One decode call for one (sequence, head) at loop t (0-based) of one layer.
  *   c_k [L][r_k], c_v [L][r_v]       latents of the L cached tokens
  *   w_up_k [T][d][r_k], w_up_v [T][d][r_v]
@@ -165,16 +189,9 @@ int lla_oracle_decode(int T, int d, int r_k, int r_v, int t, int64_t L, const do
     const int64_t n = L + (pass1 ? 1 : 0);
     double *K = (double *)malloc(sizeof(double) * (size_t)(n * d));
     double *V = (double *)malloc(sizeof(double) * (size_t)(n * d));
-    /* Eq. decode, loop t, for every cached token */
-    lla_oracle_reconstruct(d, r_k, L, c_k, w_up_k + (int64_t)t * d * r_k,
-                           mu_k ? mu_k + (int64_t)t * d : NULL, K);
-    lla_oracle_reconstruct(d, r_v, L, c_v, w_up_v + (int64_t)t * d * r_v,
-                           mu_v ? mu_v + (int64_t)t * d : NULL, V);
-    /* pass 1: the current token joins with its exact loop-t key and value */
-    if (pass1) {
-        memcpy(K + L * d, cur_k, sizeof(double) * (size_t)d);
-        memcpy(V + L * d, cur_v, sizeof(double) * (size_t)d);
-    }
+    /* Eq. decode, loop t, for every cached token; pass 1: the current token joins with its
+       exact loop-t key and value */
+    loop_keys_values(d, r_k, r_v, t, L, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, cur_k, cur_v, K, V);
     int rc = lla_oracle_attention(d, n, q, K, V, scale, out);
     free(K);
     free(V);
@@ -196,10 +213,7 @@ int lla_oracle_prefill(int T, int d, int r_k, int r_v, int t, int64_t N, const d
         return -1;
     double *K = (double *)malloc(sizeof(double) * (size_t)(N * d + 1));
     double *V = (double *)malloc(sizeof(double) * (size_t)(N * d + 1));
-    lla_oracle_reconstruct(d, r_k, N, c_k, w_up_k + (int64_t)t * d * r_k,
-                           mu_k ? mu_k + (int64_t)t * d : NULL, K);
-    lla_oracle_reconstruct(d, r_v, N, c_v, w_up_v + (int64_t)t * d * r_v,
-                           mu_v ? mu_v + (int64_t)t * d : NULL, V);
+    loop_keys_values(d, r_k, r_v, t, N, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, NULL, NULL, K, V);
     int rc = 0;
     for (int64_t i = 0; i < N && rc == 0; ++i)
         rc = lla_oracle_attention(d, i + 1, q + i * d, K, V, scale, out + i * d);
@@ -208,11 +222,104 @@ int lla_oracle_prefill(int T, int d, int r_k, int r_v, int t, int64_t N, const d
     return rc;
 }
 
+/*
+ * Rotary position embedding (RoFormer; Sec. 3 "RoPE and reconstruction") of one d-vector at
+ * integer position pos.  Pair j (j = 0 .. d/2 - 1) of x is turned by the angle
+ * pos * theta_j with theta_j = base^(-2j/d):
+ *   pairing 0 ("rotate half"):     pair j = (x[j], x[j + d/2])
+ *   pairing 1 (adjacent elements): pair j = (x[2j], x[2j + 1])
+ *   y[a] = x[a] cos(pos theta_j) - x[b] sin(pos theta_j)
+ *   y[b] = x[a] sin(pos theta_j) + x[b] cos(pos theta_j)
+ * y must not alias x.
+ */
+void lla_oracle_rope(int d, int pairing, double base, int64_t pos, const double *x, double *y)
+{
+    const int h = d / 2;
+    for (int j = 0; j < h; ++j) {
+        const int a = pairing ? 2 * j : j;
+        const int b = pairing ? 2 * j + 1 : j + h;
+        const double theta = pow(base, -2.0 * j / d);
+        const double ang = (double)pos * theta;
+        const double c = cos(ang), s = sin(ang);
+        y[a] = x[a] * c - x[b] * s;
+        y[b] = x[a] * s + x[b] * c;
+    }
+}
+
+/*
+ * lla_oracle_decode with rotary positions applied after reconstruction (Sec. 3 "RoPE and
+ * reconstruction": the latent holds the pre-RoPE key; a token keeps its position at every
+ * loop).  Cached token i sits at position pos0 + i; in pass 1 the current token's exact key
+ * sits at pos0 + L.  The query belongs to the current token, the last key of the attended set:
+ * position pos0 + L in pass 1 and pos0 + L - 1 in pass 2.  Values carry no rotation.
+ */
+int lla_oracle_decode_rope(int T, int d, int r_k, int r_v, int t, int64_t L, const double *c_k,
+                           const double *c_v, const double *w_up_k, const double *w_up_v,
+                           const double *mu_k, const double *mu_v, const double *q,
+                           const double *cur_k, const double *cur_v, double scale, int pairing,
+                           double base, int64_t pos0, double *out)
+{
+    if (t < 0 || t >= T || L < 0 || d < 2 || d % 2 != 0 || base <= 0.0)
+        return -1;
+    if ((cur_k == NULL) != (cur_v == NULL))
+        return -1;
+    const int pass1 = cur_k != NULL;
+    if (!pass1 && L < 1)
+        return -1;
+    const int64_t n = L + (pass1 ? 1 : 0);
+    double *K = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    double *Kr = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    double *V = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    loop_keys_values(d, r_k, r_v, t, L, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, cur_k, cur_v, K, V);
+    /* RoPE after reconstruction: every key at its own position, the query at the last one */
+    for (int64_t i = 0; i < n; ++i)
+        lla_oracle_rope(d, pairing, base, pos0 + i, K + i * d, Kr + i * d);
+    lla_oracle_rope(d, pairing, base, pos0 + n - 1, q, qr);
+    int rc = lla_oracle_attention(d, n, qr, Kr, V, scale, out);
+    free(K);
+    free(Kr);
+    free(V);
+    free(qr);
+    return rc;
+}
+
+/*
+ * lla_oracle_prefill with rotary positions after reconstruction: prompt token i (query and
+ * key) at position pos0 + i.
+ */
+int lla_oracle_prefill_rope(int T, int d, int r_k, int r_v, int t, int64_t N, const double *c_k,
+                            const double *c_v, const double *w_up_k, const double *w_up_v,
+                            const double *mu_k, const double *mu_v, const double *q,
+                            double scale, int pairing, double base, int64_t pos0, double *out)
+{
+    if (t < 0 || t >= T || N < 0 || d < 2 || d % 2 != 0 || base <= 0.0)
+        return -1;
+    double *K = (double *)malloc(sizeof(double) * (size_t)(N * d + 1));
+    double *Kr = (double *)malloc(sizeof(double) * (size_t)(N * d + 1));
+    double *V = (double *)malloc(sizeof(double) * (size_t)(N * d + 1));
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    loop_keys_values(d, r_k, r_v, t, N, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, NULL, NULL, K, V);
+    for (int64_t i = 0; i < N; ++i)
+        lla_oracle_rope(d, pairing, base, pos0 + i, K + i * d, Kr + i * d);
+    int rc = 0;
+    for (int64_t i = 0; i < N && rc == 0; ++i) {
+        lla_oracle_rope(d, pairing, base, pos0 + i, q + i * d, qr);
+        rc = lla_oracle_attention(d, i + 1, qr, Kr, V, scale, out + i * d);
+    }
+    free(K);
+    free(Kr);
+    free(V);
+    free(qr);
+    return rc;
+}
+
 /* One independent decode problem for lla_oracle_decode_batch. */
 typedef struct {
     int32_t t;
-    int32_t pad_;
+    int32_t rope; /* 0: no rotary positions; 1: RoPE, rotate-half pairs; 2: RoPE, adjacent pairs */
     int64_t L;
+    double rope_base;
     const double *c_k, *c_v, *w_up_k, *w_up_v, *mu_k, *mu_v;
     const double *q, *cur_k, *cur_v;
     double *out;
@@ -231,9 +338,14 @@ int lla_oracle_decode_batch(int T, int d, int r_k, int r_v, double scale, int64_
 #endif
     for (int64_t i = 0; i < n_items; ++i) {
         const lla_oracle_decode_item *it = &items[i];
-        int rc = lla_oracle_decode(T, d, r_k, r_v, it->t, it->L, it->c_k, it->c_v, it->w_up_k,
-                                   it->w_up_v, it->mu_k, it->mu_v, it->q, it->cur_k, it->cur_v,
-                                   scale, it->out);
+        int rc = it->rope
+                     ? lla_oracle_decode_rope(T, d, r_k, r_v, it->t, it->L, it->c_k, it->c_v,
+                                              it->w_up_k, it->w_up_v, it->mu_k, it->mu_v, it->q,
+                                              it->cur_k, it->cur_v, scale, it->rope - 1,
+                                              it->rope_base, 0, it->out)
+                     : lla_oracle_decode(T, d, r_k, r_v, it->t, it->L, it->c_k, it->c_v,
+                                         it->w_up_k, it->w_up_v, it->mu_k, it->mu_v, it->q,
+                                         it->cur_k, it->cur_v, scale, it->out);
         if (rc != 0) {
 #ifdef _OPENMP
 #pragma omp critical

@@ -34,6 +34,18 @@ MUTANTS = [
     ("pass1_value_is_key", "memcpy(V + L * d, cur_v,", "memcpy(V + L * d, cur_k,"),
     ("prefill_not_causal", "rc = lla_oracle_attention(d, i + 1, q + i * d, K, V, scale, out + i * d);",
      "rc = lla_oracle_attention(d, N, q + i * d, K, V, scale, out + i * d);"),
+    ("rope_sin_sign", "y[a] = x[a] * c - x[b] * s;", "y[a] = x[a] * c + x[b] * s;"),
+    ("rope_theta_exponent", "const double theta = pow(base, -2.0 * j / d);",
+     "const double theta = pow(base, -1.0 * j / d);"),
+    ("rope_pairing_mixed", "const int b = pairing ? 2 * j + 1 : j + h;",
+     "const int b = pairing ? j + h : 2 * j + 1;"),
+    ("rope_query_position", "lla_oracle_rope(d, pairing, base, pos0 + n - 1, q, qr);",
+     "lla_oracle_rope(d, pairing, base, pos0 + L, q, qr);"),
+    ("rope_keys_not_rotated",
+     "for (int64_t i = 0; i < n; ++i)\n        lla_oracle_rope(d, pairing, base, pos0 + i, K + i * d, Kr + i * d);",
+     "for (int64_t i = 0; i < n; ++i)\n        memcpy(Kr + i * d, K + i * d, sizeof(double) * (size_t)d);"),
+    ("prefill_rope_query_position", "lla_oracle_rope(d, pairing, base, pos0 + i, q + i * d, qr);",
+     "lla_oracle_rope(d, pairing, base, pos0, q + i * d, qr);"),
 ]
 
 

@@ -346,3 +346,211 @@ def test_batched_drivers_equal_single_calls():
                       w_down=g.standard_normal((T * d, r))) for r in (3, 8)]
     for it, c in zip(enc_items, oracle.encode_batch(T, d, enc_items, n_threads=2)):
         np.testing.assert_array_equal(c, oracle.encode(it["x"], it["mu"], it["w_down"]))
+
+
+# ------------------------------------------------------------------ RoPE after reconstruction
+# Sec. 3 "RoPE and reconstruction": the codec holds pre-RoPE keys and the rotation (RoFormer)
+# is applied to each reconstructed key at its token's position.
+
+def _rot_complex(x, pos, base, pairing):
+    """RoFormer's complex form: pair j as a complex number, multiplied by exp(i pos theta_j),
+    theta_j = base^(-2j/d)."""
+    d = x.shape[-1]
+    h = d // 2
+    theta = base ** (-2.0 * np.arange(h) / d)
+    z = (x[:h] + 1j * x[h:]) if pairing == 0 else (x[0::2] + 1j * x[1::2])
+    z = z * np.exp(1j * pos * theta)
+    y = np.empty(d)
+    if pairing == 0:
+        y[:h], y[h:] = z.real, z.imag
+    else:
+        y[0::2], y[1::2] = z.real, z.imag
+    return y
+
+
+@pytest.mark.parametrize("pairing", [oracle.ROPE_HALF, oracle.ROPE_ADJACENT])
+def test_rope_closed_form_pair_scores(pairing):
+    """Unit vectors of one pair: rot(e_a, P) . rot(e_a, p) = cos((P - p) theta_j) and
+    rot(e_a, P) . rot(e_b, p) = sin((P - p) theta_j); at d = 128 and base 10^4 the pair j = 32
+    turns at theta = 0.01 and j = 0 at theta = 1."""
+    d = 128
+    for j, theta in ((0, 1.0), (32, 0.01), (63, 10000.0 ** (-126 / 128))):
+        a, b = (j, j + 64) if pairing == oracle.ROPE_HALF else (2 * j, 2 * j + 1)
+        ea, eb = np.zeros(d), np.zeros(d)
+        ea[a], eb[b] = 1.0, 1.0
+        for P, p in ((5, 2), (4097, 0), (30000, 29999), (7, 7)):
+            qa = oracle.rope(ea, P, 10000.0, pairing)
+            assert qa @ oracle.rope(ea, p, 10000.0, pairing) == pytest.approx(
+                math.cos((P - p) * theta), abs=1e-12)
+            assert qa @ oracle.rope(eb, p, 10000.0, pairing) == pytest.approx(
+                math.sin((P - p) * theta), abs=1e-12)
+
+
+@pytest.mark.parametrize("pairing", [oracle.ROPE_HALF, oracle.ROPE_ADJACENT])
+def test_rope_is_a_rotation(pairing):
+    """Complex multiplication form, norm preservation, rot(x, 0) = x, and
+    rot(rot(x, a), b) = rot(x, a + b)."""
+    g = _rng(40)
+    for d, base in ((128, 10000.0), (64, 500000.0), (8, 10.0)):
+        x = g.standard_normal(d)
+        for pos in (0, 1, 17, 4095, 32767):
+            y = oracle.rope(x, pos, base, pairing)
+            # the angle pos * theta_j carries one rounding of theta_j, scaled by pos
+            np.testing.assert_allclose(y, _rot_complex(x, pos, base, pairing), rtol=0,
+                                       atol=1e-13 * (1 + pos))
+            assert np.linalg.norm(y) == pytest.approx(np.linalg.norm(x), rel=1e-14)
+        np.testing.assert_array_equal(oracle.rope(x, 0, base, pairing), x)
+        np.testing.assert_allclose(
+            oracle.rope(oracle.rope(x, 300, base, pairing), 1234, base, pairing),
+            oracle.rope(x, 1534, base, pairing), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("pairing", [oracle.ROPE_HALF, oracle.ROPE_ADJACENT])
+def test_rope_decode_tiny_case_expanded_by_hand(pairing):
+    """T = 1, d = 4, identity codec (Khat = c_k, Vhat = c_v), base 10^4: the two pairs turn at
+    theta = 1 and theta = 0.01.  Two keys at positions 0 and 1, the query at position 1 (pass 2
+    with L = 2, or pass 1 with one cached token and the current one)."""
+    e = np.eye(4)
+    if pairing == oracle.ROPE_HALF:  # pairs (0, 2) and (1, 3)
+        a0, b0, a1 = 0, 2, 1
+    else:                            # pairs (0, 1) and (2, 3)
+        a0, b0, a1 = 0, 1, 2
+    q = e[a0] + e[a1]
+    k0 = e[b0] + e[a1]   # position 0: distance 1 from the query
+    k1 = e[a0]           # position 1: same position as the query, plain dot product 1
+    v0, v1 = np.array([1.0, 2.0, 3.0, 4.0]), np.array([-1.0, 0.0, 5.0, 2.0])
+    scale = 0.7
+    s0 = scale * (math.sin(1.0) + math.cos(0.01))
+    s1 = scale * 1.0
+    expect = (math.exp(s0) * v0 + math.exp(s1) * v1) / (math.exp(s0) + math.exp(s1))
+    w = np.eye(4)[None]
+    out2 = oracle.decode_rope(0, np.stack([k0, k1]), np.stack([v0, v1]), w, w, None, None, q,
+                              None, None, scale, 10000.0, pairing)
+    np.testing.assert_allclose(out2, expect, rtol=0, atol=1e-14)
+    out1 = oracle.decode_rope(0, k0[None], v0[None], w, w, None, None, q, k1, v1, scale,
+                              10000.0, pairing)
+    np.testing.assert_allclose(out1, expect, rtol=0, atol=1e-14)
+
+
+def _relative_form(t, c_k, c_v, cod, q, cur_k, cur_v, scale, base, pairing):
+    """The same attention written through relative positions, independently of the oracle:
+    rot(q, P) . rot(k_i, p_i) = rot(q, P - p_i) . k_i, with Khat and Vhat by Eq. decode in numpy."""
+    d = q.shape[0]
+    L = c_k.shape[0]
+    mk = np.zeros(d) if cod["mu_k"] is None else cod["mu_k"][t * d:(t + 1) * d]
+    mv = np.zeros(d) if cod["mu_v"] is None else cod["mu_v"][t * d:(t + 1) * d]
+    K = c_k @ cod["w_up_k"][t].T + mk
+    V = c_v @ cod["w_up_v"][t].T + mv
+    if cur_k is not None:
+        K, V = np.vstack([K, cur_k]), np.vstack([V, cur_v])
+    P = K.shape[0] - 1
+    s = np.array([scale * (_rot_complex(q, P - i, base, pairing) @ K[i]) for i in range(P + 1)])
+    p = np.exp(s - s.max())
+    return (p @ V) / p.sum()
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+@pytest.mark.parametrize("pairing", [oracle.ROPE_HALF, oracle.ROPE_ADJACENT])
+def test_rope_decode_equals_relative_position_form(pass1, pairing):
+    T, d, r_k, r_v, L = 4, 128, 96, 160, 150
+    g = _rng(41)
+    cod = _random_codec(T, d, r_k, r_v, 42)
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    q = g.standard_normal(d)
+    cur_k = g.standard_normal(d) if pass1 else None
+    cur_v = g.standard_normal(d) if pass1 else None
+    scale = 1 / math.sqrt(d)
+    for t in (0, 3):
+        out = oracle.decode_rope(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], cod["mu_k"],
+                                 cod["mu_v"], q, cur_k, cur_v, scale, 10000.0, pairing)
+        ref = _relative_form(t, c_k, c_v, cod, q, cur_k, cur_v, scale, 10000.0, pairing)
+        np.testing.assert_allclose(out, ref, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+def test_rope_decode_depends_on_relative_positions_only(pass1):
+    """Moving every position by the same offset leaves the output unchanged; a different
+    rotation base changes it."""
+    T, d, r_k, r_v, L = 2, 128, 96, 160, 60
+    g = _rng(43)
+    cod = _random_codec(T, d, r_k, r_v, 44)
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    q = 3 * g.standard_normal(d)
+    cur_k = g.standard_normal(d) if pass1 else None
+    cur_v = g.standard_normal(d) if pass1 else None
+    dec = lambda pos0, base: oracle.decode_rope(1, c_k, c_v, cod["w_up_k"], cod["w_up_v"],
+                                                cod["mu_k"], cod["mu_v"], q, cur_k, cur_v,
+                                                0.125, base, oracle.ROPE_HALF, pos0)
+    base_out = dec(0, 10000.0)
+    for pos0 in (1, 1000, 123457):
+        np.testing.assert_allclose(dec(pos0, 10000.0), base_out, rtol=0, atol=1e-11)
+    assert np.abs(dec(0, 500000.0) - base_out).max() > 1e-3
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+def test_rope_full_rank_decode_equals_uncompressed_attention(pass1):
+    """Lossless full-rank codec: LLA decode with RoPE is exactly RoPE attention over the raw
+    loop-t keys and values (torch SDPA over keys and query rotated in complex form)."""
+    T, d, L = 2, 128, 25
+    g = _rng(45)
+    Qk, Qv = _orthogonal(T * d, 46), _orthogonal(T * d, 47)
+    xk, xv = g.standard_normal((T, L + 1, d)), g.standard_normal((T, L + 1, d))
+    mu_k, mu_v = g.standard_normal(T * d), g.standard_normal(T * d)
+    n_cached = L if pass1 else L + 1
+    c_k = oracle.encode(xk[:, :n_cached], mu_k, Qk)
+    c_v = oracle.encode(xv[:, :n_cached], mu_v, Qv)
+    w_up_k = np.stack([Qk[t * d:(t + 1) * d] for t in range(T)])
+    w_up_v = np.stack([Qv[t * d:(t + 1) * d] for t in range(T)])
+    scale = 1 / math.sqrt(d)
+    for t in range(T):
+        q = g.standard_normal(d)
+        out = oracle.decode_rope(t, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q,
+                                 xk[t, L] if pass1 else None, xv[t, L] if pass1 else None,
+                                 scale, 10000.0, oracle.ROPE_HALF)
+        Kr = np.stack([_rot_complex(xk[t, i], i, 10000.0, 0) for i in range(L + 1)])
+        ref = _sdpa(_rot_complex(q, L, 10000.0, 0), Kr, xv[t], scale)[0]
+        np.testing.assert_allclose(out, ref, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("pairing", [oracle.ROPE_HALF, oracle.ROPE_ADJACENT])
+def test_rope_prefill_matches_causal_sdpa_and_decode(pairing):
+    T, d, r_k, r_v, N = 4, 128, 96, 160, 40
+    g = _rng(48)
+    cod = _random_codec(T, d, r_k, r_v, 49)
+    c_k, c_v = g.standard_normal((N, r_k)), g.standard_normal((N, r_v))
+    q = g.standard_normal((N, d))
+    scale = 1 / math.sqrt(d)
+    t = 2
+    out = oracle.prefill_rope(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], cod["mu_k"],
+                              cod["mu_v"], q, scale, 10000.0, pairing)
+    K = c_k @ cod["w_up_k"][t].T + cod["mu_k"][t * d:(t + 1) * d]
+    V = c_v @ cod["w_up_v"][t].T + cod["mu_v"][t * d:(t + 1) * d]
+    Kr = np.stack([_rot_complex(K[i], i, 10000.0, pairing) for i in range(N)])
+    Qr = np.stack([_rot_complex(q[i], i, 10000.0, pairing) for i in range(N)])
+    np.testing.assert_allclose(out, _sdpa(Qr, Kr, V, scale, causal=True), rtol=0, atol=1e-12)
+    for i in (0, 1, 23, N - 1):
+        row = oracle.decode_rope(t, c_k[:i + 1], c_v[:i + 1], cod["w_up_k"], cod["w_up_v"],
+                                 cod["mu_k"], cod["mu_v"], q[i], None, None, scale, 10000.0,
+                                 pairing)
+        np.testing.assert_allclose(out[i], row, rtol=0, atol=1e-12)
+
+
+def test_rope_batched_driver_equals_single_calls():
+    T, d, r_k, r_v = 2, 32, 16, 24
+    g = _rng(50)
+    cod = _random_codec(T, d, r_k, r_v, 51)
+    items = []
+    for k in range(6):
+        L = int(g.integers(1, 30))
+        pass1 = k % 2 == 0
+        items.append(dict(t=k % T, c_k=g.standard_normal((L, r_k)),
+                          c_v=g.standard_normal((L, r_v)), q=g.standard_normal(d),
+                          cur_k=g.standard_normal(d) if pass1 else None,
+                          cur_v=g.standard_normal(d) if pass1 else None,
+                          rope=(k % 2, 10000.0 if k < 3 else 1e6), **cod))
+    outs = oracle.decode_batch(T, d, r_k, r_v, 0.2, items, n_threads=2)
+    for it, o in zip(items, outs):
+        ref = oracle.decode_rope(it["t"], it["c_k"], it["c_v"], cod["w_up_k"], cod["w_up_v"],
+                                 cod["mu_k"], cod["mu_v"], it["q"], it["cur_k"], it["cur_v"],
+                                 0.2, it["rope"][1], it["rope"][0])
+        np.testing.assert_array_equal(o, ref)
