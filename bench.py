@@ -30,6 +30,7 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+ROPE_BASE = 10000.0
 METRIC = "LLA decode-attn tokens/s, Ouro-1.4B shape, rho=4; HBM GB/s as % of peak"
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
@@ -65,7 +66,9 @@ def measured_peaks():
 
 def decode_source_hash() -> str:
     h = hashlib.sha256()
-    for rel in ("paper_2607_15456_gb300/csrc/lla_decode.cu", "paper_2607_15456_gb300/csrc/lla_device.cuh"):
+    for rel in ("paper_2607_15456_gb300/csrc/lla_decode.cu",
+                "paper_2607_15456_gb300/csrc/lla_decode_common.cuh",
+                "paper_2607_15456_gb300/csrc/lla_device.cuh"):
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -217,6 +220,17 @@ class DecodeBench:
                                     self.max_ctx, t, self.q[l, t], self.cur_k[l, t],
                                     self.cur_v[l, t], self.out[l, t], self.ws)
 
+    def decode_calls_rope(self, base=ROPE_BASE):
+        """The same pass-1 sweep with rotary positions applied after reconstruction (keys
+        rebuilt on the tensor cores, lla_decode_attn_rope)."""
+        w, lla = self.w, self.lla
+        for t in range(w.T):
+            for l in range(w.D):
+                lla.lla_decode_attn_rope(self.geom, self.codecs[l], self.caches[l], base,
+                                         lla.LLA_ROPE_HALF, self.ctx, self.max_ctx, t,
+                                         self.q[l, t], self.cur_k[l, t], self.cur_v[l, t],
+                                         self.out[l, t], self.ws)
+
     def encode_calls(self):
         # the completed token of every sequence, in every layer: its stacked loop-t keys and
         # values (one lla_encode_layers launch for all layers)
@@ -353,6 +367,7 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_cpu_baseline and rank == 0 and world == 1:
         result["cpu_baseline"] = cpu_baseline(bench.w, bench.lens, args.cpu_seconds)
     if not args.no_extras and rank == 0:
+        result.update(run_rope_extra(bench))
         del bench
         torch.cuda.empty_cache()
         result.update(run_extras(device))
@@ -374,6 +389,30 @@ def _time_ms(fn, reps=5, warm=2):
         torch.cuda.synchronize()
         best = min(best, a.elapsed_time(b))
     return best
+
+
+def run_rope_extra(bench):
+    """The full-RoPE decode (f1: keys rebuilt on the tensor cores and rotated at their
+    positions, Sec. 3 "RoPE and reconstruction") on the headline batch: the same D x T pass-1
+    sweep through lla_decode_attn_rope, against the HBM roofline of the same algorithmic bytes
+    as the absorbed decode, with the key rebuild's tensor work beside it."""
+    w, lla = bench.w, bench.lla
+    peak, _ = measured_peaks()
+    ms = _time_ms(bench.decode_calls_rope, reps=3, warm=1)
+    launches = w.D * w.T
+    per_launch_s = ms / 1e3 / launches
+    nbytes = bench.decode_bytes_per_launch()
+    rebuild_flops = 2.0 * sum(bench.lens) * w.H * w.d * w.r_k
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the RoPE decode measurement")
+    return {"rope_decode": {
+        "workload": f"{w.name} batch, RoPE after reconstruction (base {ROPE_BASE:g}, rotate-half "
+                    f"pairs), {w.D}x{w.T} pass-1 calls",
+        "kernel": "decode_rope_kernel (lla_decode_attn_rope)", "bound": "hbm",
+        "ms_per_sweep": ms, "avg_launch_us": per_launch_s * 1e6,
+        "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
+        "bytes_per_launch": nbytes, "key_rebuild_TFLOP_s": rebuild_flops / per_launch_s / 1e12,
+        "tokens_per_s_decode_only": bench.B / (ms / 1e3)}}
 
 
 def run_extras(device):

@@ -11,6 +11,8 @@
  *   lla_decode_attn      one decode call (one layer, one loop) over the paged latent cache,
  *                        for a batch of sequences of different lengths (App. A, "Decoding and
  *                        caching": pass 1 and pass 2 of the cached reconstruction decoder)
+ *   lla_decode_attn_rope the same with rotary positions applied after reconstruction (Sec. 3,
+ *                        "RoPE and reconstruction"), keys rebuilt on the tensor cores
  *   lla_prefill_attn     causal pass-2 prefill attention over the latents of a prompt
  *   lla_dense_*          the uncompressed loop-t KV decode in the same kernel style (the
  *                        "teacher" column of Table absorbed_latency, App. J), for comparison
@@ -172,6 +174,39 @@ lla_status lla_decode_attn(const lla_geometry *g, const lla_codec *codec, const 
                            const void *q, const void *cur_k, const void *cur_v,
                            lla_dtype io_dtype, void *out, void *workspace,
                            size_t workspace_bytes, void *stream);
+
+/* Rotary position embedding (RoFormer) applied after reconstruction (Sec. 3 "RoPE and
+ * reconstruction"): pair j of a d-vector at position p is turned by the angle p * base^(-2j/d). */
+typedef enum {
+    LLA_ROPE_HALF = 0,     /* pair j = (x[j], x[j + d/2])  ("rotate half") */
+    LLA_ROPE_ADJACENT = 1  /* pair j = (x[2j], x[2j + 1]) */
+} lla_rope_pairing;
+
+typedef struct {
+    double base;              /* rotation base, > 1 (10000 in RoFormer) */
+    lla_rope_pairing pairing;
+} lla_rope;
+
+/*
+ * lla_decode_attn with rotary positions applied after reconstruction: the full-RoPE decoder
+ * (Sec. 3 "RoPE and reconstruction"; App. A "Decoding and caching").  The latents hold pre-RoPE
+ * keys.  Cached key i of sequence b (its index in the sequence) is rebuilt by Eq. decode and
+ * rotated at position i; the query, and in pass 1 the current token's exact key, at the current
+ * token's position: context_lens[b] in pass 1, context_lens[b] - 1 in pass 2.  Values are not
+ * rotated.
+ *   rope          host pointer to the rotation (read during the call)
+ *   q, cur_k      pre-RoPE: the call rotates them
+ * Every other argument, the workspace (lla_decode_workspace_size) and the error behaviour are
+ * those of lla_decode_attn.  Keys are rebuilt on the tensor cores: storage must be LLA_BF16,
+ * d = 128 and (r_k, r_v) one of (96, 160), (128, 128), else LLA_ERR_UNSUPPORTED.  q, cur_k,
+ * cur_v and out must be 16-byte aligned.
+ */
+lla_status lla_decode_attn_rope(const lla_geometry *g, const lla_codec *codec,
+                                const lla_cache *cache, const lla_rope *rope,
+                                const int32_t *context_lens, int32_t B, int32_t max_ctx,
+                                int32_t loop, const void *q, const void *cur_k, const void *cur_v,
+                                lla_dtype io_dtype, void *out, void *workspace,
+                                size_t workspace_bytes, void *stream);
 
 /*
  * lla_decode_attn for callers that cannot allocate device memory (for example a plug-in inside a

@@ -183,7 +183,7 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
                          const int32_t *context_lens, int32_t B, int32_t max_ctx, int32_t loop,
                          const void *q, const void *cur_k, const void *cur_v, lla_dtype io_dtype,
                          void *out, void *workspace, size_t workspace_bytes, void *stream,
-                         bool absorbed) {
+                         bool absorbed, const lla_rope *rope = nullptr) {
     lla_status st = check_geometry(g);
     if (st != LLA_OK) return st;
     if ((st = check_cache(cache, true)) != LLA_OK) return st;
@@ -205,7 +205,17 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
         return LLA_ERR_UNSUPPORTED;
     if ((cur_k == nullptr) != (cur_v == nullptr)) return LLA_ERR_INVALID_ARG;
     if (B > 0 && (!context_lens || !q || !out)) return LLA_ERR_INVALID_ARG;
-    if ((st = decode_fits(g->r_k, g->r_v, es, g->d)) != LLA_OK) return st;
+    if (rope) {
+        if (!(rope->base > 1.0) || !(rope->base < 1e300)) return LLA_ERR_INVALID_ARG;
+        if (rope->pairing != LLA_ROPE_HALF && rope->pairing != LLA_ROPE_ADJACENT)
+            return LLA_ERR_INVALID_ARG;
+        if ((q && !aligned(q, 16)) || (cur_k && !aligned(cur_k, 16)) ||
+            (cur_v && !aligned(cur_v, 16)) || (out && !aligned(out, 16)))
+            return LLA_ERR_INVALID_ARG;
+        if ((st = decode_rope_fits(g->r_k, g->r_v, es, g->d, B)) != LLA_OK) return st;
+    } else if ((st = decode_fits(g->r_k, g->r_v, es, g->d)) != LLA_OK) {
+        return st;
+    }
     if (B == 0) return LLA_OK;
     if (!workspace) return LLA_ERR_INVALID_ARG;
     DecodeArgs a = {};
@@ -224,6 +234,9 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
     a.context_lens = context_lens; a.B = B; a.max_ctx = max_ctx;
     a.q = q; a.cur_k = cur_k; a.cur_v = cur_v; a.out = out;
     a.workspace = workspace; a.workspace_bytes = workspace_bytes;
+    if (rope)
+        return launch_decode_rope(a, rope->base, rope->pairing == LLA_ROPE_ADJACENT ? 1 : 0,
+                                  static_cast<cudaStream_t>(stream));
     return launch_decode(a, static_cast<cudaStream_t>(stream));
 }
 
@@ -236,6 +249,17 @@ lla_status lla_decode_attn(const lla_geometry *g, const lla_codec *codec, const 
                            size_t workspace_bytes, void *stream) {
     return decode_common(g, codec, cache, context_lens, B, max_ctx, loop, q, cur_k, cur_v,
                          io_dtype, out, workspace, workspace_bytes, stream, true);
+}
+
+lla_status lla_decode_attn_rope(const lla_geometry *g, const lla_codec *codec,
+                                const lla_cache *cache, const lla_rope *rope,
+                                const int32_t *context_lens, int32_t B, int32_t max_ctx,
+                                int32_t loop, const void *q, const void *cur_k, const void *cur_v,
+                                lla_dtype io_dtype, void *out, void *workspace,
+                                size_t workspace_bytes, void *stream) {
+    if (!rope) return LLA_ERR_INVALID_ARG;
+    return decode_common(g, codec, cache, context_lens, B, max_ctx, loop, q, cur_k, cur_v,
+                         io_dtype, out, workspace, workspace_bytes, stream, true, rope);
 }
 
 lla_status lla_dense_decode_attn(const lla_geometry *g, const lla_cache *cache,

@@ -1,0 +1,532 @@
+// lla_decode_rope.cu -- decode with rotary positions applied after reconstruction: the full-RoPE
+// decoder of Looped Latent Attention (Sec. 3 "RoPE and reconstruction"; App. A "Decoding and
+// caching").
+//
+// The codec holds pre-RoPE keys.  Cached key i of a sequence sits at position p_i = i; the query
+// (and, in pass 1, the current token's exact key) at P = L in pass 1 and P = L - 1 in pass 2.
+// RoPE (RoFormer) turns pair j of a vector at position p by p theta_j, theta_j = base^(-2j/d):
+//   s_i = scale rot(q, P) . rot(khat_i, p_i) = scale rot(q, P - p_i) . khat_i,
+//   khat_i = W_up,t^K c_k,i + mu^K_t                                           (Eq. decode)
+// The rotation depends on i, so the key up-projection cannot move onto the query as in the
+// absorbed kernel; each page's keys are rebuilt on the tensor cores instead.  Values carry no
+// rotation, so the value side stays in latent space as in lla_decode.cu:
+//   o = (W_up,t^V sum_i p_i c_v,i + (sum_i p_i) mu^V_t + p_cur v_cur) / (sum_i p_i + p_cur).
+//
+// GB300 mapping (one CTA per SM; the persistent split of (sequence, head, page) units over the
+// CTAs, the TMA ring, the split-KV merge and the output projection are shared with lla_decode.cu
+// through lla_decode_common.cuh):
+//   * producer warp: TMA bulk copies of whole head pages (K-plane + V-plane) into the ring.
+//   * MMA warp: per page, Khat^T (d x 64) = W_up,t^K (d x r_k) . C_k^T with tcgen05.mma.  A is
+//     W_up,t^K, staged once per run as no-swizzle K-major core matrices; B is the page's K-plane
+//     exactly as it sits in the ring (its granule-interleaved layout is a no-swizzle K-major
+//     operand with the 64 tokens along N); one more K step adds mu^K_t as a (mu_hi, mu_lo) pair
+//     of bf16 columns against a pair of ones.  D lands in TMEM (lane = key dimension, column =
+//     token), in two buffers so that a page's MMA overlaps the previous page's epilogue.
+//   * four epilogue warps (one per TMEM lane quarter): lane m multiplies its 64 columns by
+//     element m of rot(q, P - p_i).  Along a page that element is a sinusoid in i; it starts from
+//     a phase computed exactly per page (64-bit fixed-point turns) and steps through the tokens
+//     with a second-order recurrence (two flops per token).  The 128 products of a token are
+//     summed through a shared-memory transpose, then the online softmax runs as in the absorbed
+//     kernel.
+//   * four value warps: sum_i p_i c_v,i from the V-plane (shared with lla_decode.cu).
+//   * four management warps: per run, W_up,t^K and mu^K_t into an A slot and q into a query
+//     slot; the merge of split runs and W_up,t^V, mu^V_t, 1/l (shared with lla_decode.cu).
+#include "lla_decode_common.cuh"
+#include "lla_tcgen05.cuh"
+
+namespace lla {
+namespace {
+
+constexpr int kRopeD = 128;                        // head width of the tensor-core path
+constexpr int kRopePairs = kRopeD / 2;
+constexpr int kMmaWarp = kAsyncThreads / 32;       // warp 13, after the management warps
+constexpr int kRopeThreads = kAsyncThreads + 32;   // 448
+constexpr int kRopeWst = 20 * 1024;                // staging buffer of W_up,t^V rows
+constexpr int kBarTmem = 5;                        // epilogue warps + MMA warp, before dealloc
+constexpr int kXposeStride = 20;                   // floats per row of a transpose buffer
+constexpr int kXposeFloats = 32 * kXposeStride + 16;
+
+// Launch parameters: the decode parameters plus, per rotation pair j, the phase step theta_j as
+// 64-bit fixed-point turns (theta_j / 2 pi * 2^64), sin theta_j, 1 - cos theta_j, and
+// cos / sin of 16 theta_j, all computed on the host in double precision.
+struct RopeParams {
+    Params p;
+    unsigned long long phi[kRopePairs];
+    float sn[kRopePairs], hc[kRopePairs], c16[kRopePairs], s16[kRopePairs];
+    int pairing;  // 0: pair j = (j, j + d/2); 1: pair j = (2j, 2j + 1)
+};
+
+template <int RK, int RV>
+struct RopeShape {
+    using F = Fast<2, RK, RV>;
+    static constexpr int NG = RK / 8;               // 16-byte granules per row of W_up,t^K
+    static constexpr int KSTEPS = RK / 16;          // MMAs of K = 16 per page
+    static constexpr int A_BYTES = NG * kRopeD * 16;
+    // A slot: the NG granules of W_up,t^K, then (mu_hi, mu_lo, 0, ...) and a zero granule
+    static constexpr int A_SLOT = A_BYTES + 2 * kRopeD * 16;
+    static constexpr uint32_t IDESC = umma_idesc_bf16(kRopeD, 64, 0, 0);
+    static_assert(RK % 16 == 0, "whole K steps of 16 latent columns");
+    static_assert(F::PPS == 1 && F::TT == 64, "one page per pipeline step");
+    static_assert(F::S_WARPS == 4 && F::V_WARPS == 4, "four epilogue and four value warps");
+};
+
+struct RopeLayout {
+    int aslot, ones, xpose, red, bars, tmem, total;
+};
+
+template <int RK, int RV>
+__host__ __device__ inline RopeLayout rope_layout(int stages, int stage_bytes, int B) {
+    using Z = RopeShape<RK, RV>;
+    RopeLayout L;
+    int o = (async_layout<2, RK, RV, kRopeD, kRopeWst>(stages, stage_bytes, B).total + 127) & ~127;
+    L.aslot = o; o += 2 * Z::A_SLOT;
+    L.ones = o;  o += 2 * 64 * 16;                // B operand of the mu step: (1, 1, 0...) and zeros
+    L.xpose = o; o += 4 * kXposeFloats * 4;
+    L.red = o;   o += 4 * 64 * 4;
+    L.bars = o;  o += 8 * 8;                      // aful[2], afree[2], tfull[2], tfree[2]
+    L.tmem = o;  o += 16;
+    L.total = o;
+    return L;
+}
+
+template <int RK, int RV>
+__global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __grid_constant__ RopeParams rp) {
+    using Z = RopeShape<RK, RV>;
+    using F = typename Z::F;
+    constexpr int ES = 2, D = kRopeD;
+    const Params &p = rp.p;
+    extern __shared__ __align__(128) char smem[];
+    const ASmem a = carve_async<ES, RK, RV, D, kRopeWst>(smem, p);
+    const Smem &s = a.s;
+    const RopeLayout RL = rope_layout<RK, RV>(p.stages, p.stage_bytes, p.B);
+    char *aslot = smem + RL.aslot;
+    char *ones = smem + RL.ones;
+    float *xpose = reinterpret_cast<float *>(smem + RL.xpose);
+    float *red4 = reinterpret_cast<float *>(smem + RL.red);
+    uint64_t *aful = reinterpret_cast<uint64_t *>(smem + RL.bars);
+    uint64_t *afree = aful + 2, *tfull = aful + 4, *tfree = aful + 6;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + RL.tmem);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bool pass1 = p.cur_k != nullptr;
+
+    pdl_wait();  // inputs may come from the previous kernel in the stream
+    if (tid == 0) {
+        for (int i = 0; i < kQSlots; ++i) mbar_init(&a.qready[i], kMThreads);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&a.stfull[i], kComputeThreads);
+            mbar_init(&a.stfree[i], kMThreads);
+            mbar_init(&aful[i], 1);
+            mbar_init(&afree[i], 1);
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tfree[i], 4);
+        }
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(tmem_slot, 128);  // two 64-column accumulators
+        // constant operand parts: the ones column pair of the mu step and the zero granules
+        uint4 *o4 = reinterpret_cast<uint4 *>(ones);
+        for (int i = lane; i < 128; i += 32)
+            o4[i] = i < 64 ? make_uint4(0x3f803f80u, 0u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
+        for (int sl = 0; sl < 2; ++sl) {
+            uint4 *z4 = reinterpret_cast<uint4 *>(aslot + sl * Z::A_SLOT + Z::A_BYTES + D * 16);
+            for (int i = lane; i < D; i += 32) z4[i] = make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+    }
+    // one arrival per pipeline step on empty: the MMA warp's commit and the four value warps
+    Range rg = prologue(p, s, kComputeThreads / 2, F::V_THREADS, 1 + F::V_WARPS);
+    order_runs(p, s, rg);
+    pdl_trigger();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == kComputeWarps) {
+        if (rg.A0 < rg.A1) named_bar_sync(kBarStart, kMThreads + 32);
+        producer(p, s, rg);
+        return;
+    }
+
+    if (warp == kMmaWarp) {
+        // ------------------------------------------------------------------------- MMA warp
+        int it = 0, stage = 0, r = 0;
+        uint32_t ph = 0;
+        const bool has_mu = p.mu_k != nullptr;
+        const uint32_t ones_desc_lo = smem_addr(ones);
+        for (int pass = 0; pass < 3; ++pass)
+        for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
+            const Run R = locate_run(p, s, u, rg.hi[pass]);
+            const int as = r & 1;
+            const uint32_t abase = smem_addr(aslot + as * Z::A_SLOT);
+            if (lane == 0) mbar_wait(&aful[as], (r >> 1) & 1, s.abort_flag, p.err);
+            for (int k = 0; k < R.npages; ++k, ++it) {
+                const int b = it & 1;
+                if (lane == 0) {
+                    mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+                    if (it >= 2) mbar_wait(&tfree[b], ((it - 2) >> 1) & 1, s.abort_flag, p.err);
+                    tc_fence_after();
+                    const uint32_t d = tmem_base + b * 64;
+                    const uint32_t bbase = smem_addr(s.ring + stage * p.stage_bytes);
+#pragma unroll
+                    for (int st = 0; st < Z::KSTEPS; ++st)
+                        umma_bf16(d, umma_desc(abase + st * 4096, 2048, 128),
+                                  umma_desc(bbase + st * 2048, 1024, 128), Z::IDESC, st > 0);
+                    if (has_mu)
+                        umma_bf16(d, umma_desc(abase + Z::A_BYTES, 2048, 128),
+                                  umma_desc(ones_desc_lo, 1024, 128), Z::IDESC, true);
+                    umma_commit(&tfull[b]);
+                    umma_commit(&s.empty[stage]);  // the K-plane has been read
+                    if (k == R.npages - 1) umma_commit(&afree[as]);
+                }
+                __syncwarp();
+                if (++stage == p.stages) {
+                    stage = 0;
+                    ph ^= 1u;
+                }
+            }
+            u = R.run_end;
+        }
+        // every MMA has completed before TMEM is released, even after an abort
+        if (lane == 0 && it > 0) {
+            volatile int never = 0;
+            mbar_wait(&tfull[(it - 1) & 1], ((it - 1) >> 1) & 1, &never, p.err);
+        }
+        named_bar_sync(kBarTmem, 128 + 32);  // the epilogue warps have read every buffer
+        tc_fence_after();
+        tmem_dealloc(tmem_base, 128);
+        return;
+    }
+
+    if (tid >= kMBase) {
+        // ------------------------------------------------------------------ management warps
+        const int mt = tid - kMBase;
+        auto finish = [&](const Run &R, int64_t u, int k) {
+            m_finish<ES, RK, RV, D, F::TT, F::NTG, kRopeWst>(p, a, R, u, rg, k & 1, (k >> 1) & 1,
+                                                            k % kQSlots, mt);
+        };
+        int r = 0;
+        Run q0{}, q1{};
+        int64_t u0 = 0, u1 = 0;
+        for (int pass = 0; pass < 3; ++pass)
+        for (int64_t u = rg.lo[pass]; u < rg.hi[pass];) {
+            const Run R = locate_run(p, s, u, rg.hi[pass]);
+            const int slot = r % kQSlots, as = r & 1;
+            // W_up,t^K of head R.h into A slot `as` once run r - 2's MMAs have read it
+            if (r >= 2) mbar_wait(&afree[as], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
+            char *A = aslot + as * Z::A_SLOT;
+            const int64_t hl = (static_cast<int64_t>(R.h) * p.T + p.loop) * D;
+            const char *W = static_cast<const char *>(p.w_up_k) + hl * RK * ES;
+            cp_async_wait_all();  // no earlier copy of this thread is still in flight
+            for (int i = mt; i < D * Z::NG; i += kMThreads) {
+                const int row = i / Z::NG, g = i - row * Z::NG;
+                cp_async16(A + g * (D * 16) + row * 16, W + row * (RK * ES) + g * 16);
+            }
+            cp_async_commit();
+            if (r == 0) named_bar_arrive(kBarStart, kMThreads + 32);  // the ring may start
+            if (mt < D) {
+                const float mu = p.mu_k ? p.mu_k[hl + mt] : 0.f;
+                const __nv_bfloat16 hi = __float2bfloat16_rn(mu);
+                const __nv_bfloat16 lo = __float2bfloat16_rn(mu - __bfloat162float(hi));
+                const uint32_t w0 = static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
+                                    (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16);
+                *reinterpret_cast<uint4 *>(A + Z::A_BYTES + mt * 16) = make_uint4(w0, 0u, 0u, 0u);
+            }
+            cp_async_wait_all();
+            fence_proxy_async_smem();  // the slot's writes become visible to the tensor core
+            m_sync();
+            if (mt == 0) mbar_arrive(&aful[as]);
+            m_setup<ES, RK, RV, D, false, kRopeWst>(p, a, R.b, R.h, slot, mt, false);
+            mbar_arrive(&a.qready[slot]);
+            if (r >= 2) finish(q0, u0, r - 2);
+            q0 = q1;
+            u0 = u1;
+            q1 = R;
+            u1 = u;
+            ++r;
+            u = R.run_end;
+        }
+        if (r >= 2) finish(q0, u0, r - 2);
+        if (r >= 1) finish(q1, u1, r - 1);
+        for (int b = 0; b < p.B; ++b) {  // no cached token: pass 1 attends to the current token
+            if (s.lens[b] != 0) continue;
+            for (int h = 0; h < p.H; ++h) {
+                if ((b * p.H + h) % gridDim.x != blockIdx.x) continue;
+                const int64_t row = (static_cast<int64_t>(b) * p.H + h) * D;
+                if (!pass1 && mt == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
+                for (int e = mt; e < D; e += kMThreads)
+                    store_elem(p.out, row + e, pass1 ? load_elem(p.cur_v, row + e, p.io_bf16) : 0.f,
+                               p.io_bf16);
+            }
+        }
+        cp_async_wait_all();
+        return;
+    }
+
+    if (warp < F::S_WARPS) {
+        // ------------------------------------------------------------------- epilogue warps
+        // lane m = key dimension m; its rotation pair j and its role in the pair
+        const int m = tid;
+        const int j = rp.pairing ? (m >> 1) : (m & (kRopePairs - 1));
+        const bool upper = rp.pairing ? (m & 1) : (m >= kRopePairs);
+        const int ia = rp.pairing ? 2 * j : j, ib = rp.pairing ? 2 * j + 1 : j + kRopePairs;
+        const unsigned long long phi = rp.phi[j];
+        const float sn = rp.sn[j], hc = rp.hc[j], lam = 2.f * rp.hc[j];
+        const float c16 = rp.c16[j], s16 = rp.s16[j];
+        float *xb = xpose + warp * kXposeFloats;
+        float *xrow = xb + lane * kXposeStride + (lane >= 16 ? 16 : 0);
+        const int hf = lane >> 4, col = lane & 15;
+        const float *xcol = xb + hf * 16 * kXposeStride + hf * 16 + col;
+        const uint32_t tlane = tmem_base + (static_cast<uint32_t>(32 * warp) << 16);
+        int it = 0, r = 0;
+        for (int pass = 0; pass < 3; ++pass)
+        for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
+            const Run R = locate_run(p, s, u, rg.hi[pass]);
+            const int rslot = r & 1, qslot = r % kQSlots;
+            mbar_wait(&a.qready[qslot], (r / kQSlots) & 1, s.abort_flag, p.err);
+            // element m of rot(q, Delta) = Re(G e^{i Delta theta_j}), scaled to log2 units
+            float Gr, Gi;
+            {
+                const float *qv = a.qlat + qslot * a.qslot;
+                const float qa = qv[ia], qb = qv[ib];
+                Gr = (upper ? qb : qa) * p.scale_log2;
+                Gi = (upper ? -qa : qb) * p.scale_log2;
+            }
+            const int P = pass1 ? R.Lb : R.Lb - 1;  // the query's position
+            float m_run = -INFINITY, l_part = 0.f;
+            for (int k = 0; k < R.npages; ++k, ++it) {
+                const int b = it & 1, slot = it & 1;
+                const uint32_t pph = (it >> 1) & 1;
+                const int pg = R.pg0 + k;
+                const int nvalid = min(kBlockTokens, R.Lb - pg * kBlockTokens);
+                mbar_wait(&tfull[b], (it >> 1) & 1, s.abort_flag, p.err);
+                tc_fence_after();
+                // exact phase of the page's first token: Delta0 theta_j in turns, mod 1
+                const int delta0 = P - pg * kBlockTokens;  // >= 0: the page holds a cached token
+                const unsigned long long turns = static_cast<unsigned long long>(delta0) * phi;
+                const float tf = __uint2float_rn(static_cast<uint32_t>(turns >> 32)) * 2.3283064365386963e-10f;
+                float sa, ca;
+                sincospif(2.f * tf, &sa, &ca);
+                float zr = Gr * ca - Gi * sa, zi = Gr * sa + Gi * ca;
+#pragma unroll
+                for (int hv = 0; hv < 2; ++hv) {  // tokens 32 hv .. 32 hv + 31
+                    float v[32];
+                    tmem_ld32(tlane + b * 64 + 32 * hv, v);
+                    if (hv == 1) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&tfree[b]);  // the buffer may take page it + 2
+                    }
+                    // two chains of 16 tokens: x = Re(z e^{-i r theta}), dd = x_r - x_{r-1}
+                    float x[2], dd[2];
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        x[c] = zr;
+                        dd[c] = fmaf(zr, hc, zi * sn);
+                        const float nr = fmaf(zr, c16, zi * s16), ni = fmaf(zi, c16, -zr * s16);
+                        zr = nr;
+                        zi = ni;
+                    }
+#pragma unroll
+                    for (int t = 0; t < 16; ++t) {
+#pragma unroll
+                        for (int c = 0; c < 2; ++c) {
+                            v[c * 16 + t] *= x[c];
+                            dd[c] = fmaf(-lam, x[c], dd[c]);
+                            x[c] += dd[c];
+                        }
+                    }
+                    // sum over the 128 dimensions of each token: per warp through a transpose
+                    // of 16-token chunks, then across the four warps
+#pragma unroll
+                    for (int ch = 0; ch < 2; ++ch) {
+#pragma unroll
+                        for (int q4 = 0; q4 < 4; ++q4)
+                            *reinterpret_cast<float4 *>(xrow + 4 * q4) =
+                                make_float4(v[ch * 16 + 4 * q4], v[ch * 16 + 4 * q4 + 1],
+                                            v[ch * 16 + 4 * q4 + 2], v[ch * 16 + 4 * q4 + 3]);
+                        __syncwarp();
+                        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+                        for (int kk = 0; kk < 16; kk += 4) {
+                            s0 += xcol[(kk + 0) * kXposeStride];
+                            s1 += xcol[(kk + 1) * kXposeStride];
+                            s2 += xcol[(kk + 2) * kXposeStride];
+                            s3 += xcol[(kk + 3) * kXposeStride];
+                        }
+                        float acc = (s0 + s1) + (s2 + s3);
+                        acc += __shfl_xor_sync(0xffffffffu, acc, 16);
+                        if (lane < 16) red4[warp * 64 + hv * 32 + ch * 16 + col] = acc;
+                        __syncwarp();
+                    }
+                }
+                named_bar_sync(kBarTok, F::S_THREADS);
+                // online softmax over the page's tokens (threads 0..63, one token each)
+                float *wmax = s.misc + kAWmax + slot * 8;
+                float xs = -INFINITY;
+                if (tid < kBlockTokens) {
+                    const float sc = (red4[tid] + red4[64 + tid]) + (red4[128 + tid] + red4[192 + tid]);
+                    xs = tid < nvalid ? sc : -INFINITY;
+                    const float lm = warp_max(xs);
+                    if (lane == 0) wmax[warp] = lm;
+                }
+                named_bar_sync(kBarTok, F::S_THREADS);
+                float *pring = s.psm + slot * kComputeThreads;
+                if (tid < kBlockTokens) {
+                    const float m_new = fmaxf(m_run, fmaxf(wmax[0], wmax[1]));
+                    const float alpha = exp2f(m_run - m_new);
+                    m_run = m_new;
+                    mbar_wait(&s.pempty[slot], pph ^ 1u, s.abort_flag, p.err);
+                    const float pv = tid < nvalid ? exp2f(xs - m_new) : 0.f;
+                    pring[tid] = pv;
+                    l_part = fmaf(l_part, alpha, pv);
+                    if (tid == 0) s.misc[kAPAlpha + slot] = alpha;
+                }
+                mbar_arrive(&s.pfull[slot]);
+            }
+            if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
+            if (tid < kBlockTokens) a.lred[rslot * kLredSlot + tid] = l_part;
+            if (tid == 0) s.misc[kAM + rslot] = m_run;
+            mbar_arrive(&a.stfull[rslot]);
+            u = R.run_end;
+        }
+        tc_fence_before();
+        named_bar_arrive(kBarTmem, 128 + 32);
+        return;
+    }
+
+    // --------------------------------------------------------------------------- value warps
+    const int vt = tid - F::S_THREADS;
+    const int vc = vt % F::VC, tg = vt / F::VC;
+    const bool vwork = tg < F::NTG;
+    constexpr int AV = F::UPT * F::VE;
+    int it = 0, stage = 0, r = 0;
+    uint32_t ph = 0;
+    for (int pass = 0; pass < 3; ++pass)
+    for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
+        const Run R = locate_run(p, s, u, rg.hi[pass]);
+        const int rslot = r & 1;
+        float accv[AV];
+#pragma unroll
+        for (int e = 0; e < AV; ++e) accv[e] = 0.f;
+        for (int k = 0; k < R.npages; ++k, ++it) {
+            const int slot = it & 1;
+            const uint32_t pph = (it >> 1) & 1;
+            const char *sb = s.ring + stage * p.stage_bytes;
+            const int nvalid = min(kBlockTokens, R.Lb - (R.pg0 + k) * kBlockTokens);
+            mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+            mbar_wait(&s.pfull[slot], pph, s.abort_flag, p.err);
+            if (vwork)
+                value_step<ES, RK, RV>(accv, sb, s.psm + slot * kComputeThreads,
+                                       s.misc[kAPAlpha + slot], nvalid, vc, tg);
+            mbar_arrive(&s.pempty[slot]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.empty[stage]);  // V-plane read
+            if (++stage == p.stages) {
+                stage = 0;
+                ph ^= 1u;
+            }
+        }
+        if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
+        if (vwork) {
+#pragma unroll
+            for (int e = 0; e < AV; ++e) a.red[rslot * a.redslot + tg * RV + vc * AV + e] = accv[e];
+        }
+        mbar_arrive(&a.stfull[rslot]);
+        u = R.run_end;
+    }
+}
+
+template <int RK, int RV>
+lla_status launch_rope(const RopeParams &prm, int grid, int smem, cudaStream_t stream) {
+    static bool configured[64] = {};
+    return launch_kernel(decode_rope_kernel<RK, RV>, configured, prm, grid, smem, stream,
+                         kRopeThreads);
+}
+
+template <int RK, int RV>
+int rope_layout_bytes(int stages, int stage_bytes, int B) {
+    return rope_layout<RK, RV>(stages, stage_bytes, B).total;
+}
+
+using RopeLauncher = lla_status (*)(const RopeParams &, int, int, cudaStream_t);
+using RopeLayoutFn = int (*)(int, int, int);
+struct RopeEntry {
+    RopeLauncher launch;
+    RopeLayoutFn layout;
+};
+RopeEntry rope_entry(int es, int d, int r_k, int r_v) {
+    if (es != 2 || d != kRopeD) return RopeEntry{nullptr, nullptr};
+    if (r_k == 96 && r_v == 160) return RopeEntry{launch_rope<96, 160>, rope_layout_bytes<96, 160>};
+    if (r_k == 128 && r_v == 128) return RopeEntry{launch_rope<128, 128>, rope_layout_bytes<128, 128>};
+    return RopeEntry{nullptr, nullptr};
+}
+
+// Ring stages that fit beside the fixed layout (head pages of stage_bytes each).
+int rope_stages(const RopeEntry &e, int stage_bytes, int B) {
+    const int fixed = e.layout(0, stage_bytes, B);
+    int stages = (kSmemLimit - fixed) / (stage_bytes + 16);
+    return stages > kMaxStages ? kMaxStages : stages;
+}
+
+}  // namespace
+
+lla_status decode_rope_fits(int r_k, int r_v, int es, int d, int B) {
+    const RopeEntry e = rope_entry(es, d, r_k, r_v);
+    if (!e.launch) return LLA_ERR_UNSUPPORTED;
+    const int hpb = static_cast<int>(head_page_bytes(r_k, r_v, es));
+    return rope_stages(e, hpb, B) >= 2 ? LLA_OK : LLA_ERR_UNSUPPORTED;
+}
+
+lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cudaStream_t stream) {
+    const int es = a.storage_bf16 ? 2 : 4;
+    const RopeEntry e = rope_entry(es, a.d, a.r_k, a.r_v);
+    if (!e.launch) return LLA_ERR_UNSUPPORTED;
+    const int hpb = static_cast<int>(head_page_bytes(a.r_k, a.r_v, es));
+    const int stages = rope_stages(e, hpb, a.B);
+    if (stages < 2) return LLA_ERR_UNSUPPORTED;
+    const int smem = e.layout(stages, hpb, a.B);
+    const int grid = num_sms();
+    if (grid <= 0) return LLA_ERR_CUDA;
+    if (a.workspace_bytes < decode_workspace_bytes(a.r_v, a.B, a.H, grid)) return LLA_ERR_WORKSPACE;
+    lla_status st = LLA_OK;
+    unsigned *err = device_error_word(&st);
+    if (st != LLA_OK) return st;
+
+    RopeParams rp = {};
+    Params &p = rp.p;
+    p.T = a.T; p.H = a.H; p.d = a.d; p.r_k = a.r_k; p.r_v = a.r_v; p.loop = a.loop;
+    p.absorbed = 1; p.io_bf16 = a.io_bf16;
+    p.scale_log2 = a.scale * 1.4426950408889634f;
+    p.w_up_k = a.w_up_k; p.w_up_v = a.w_up_v; p.mu_k = a.mu_k; p.mu_v = a.mu_v;
+    p.pool = static_cast<const char *>(a.pool);
+    p.num_blocks = a.num_blocks;
+    p.block_bytes = static_cast<int64_t>(hpb) * a.H;
+    p.head_page_bytes = hpb;
+    p.kplane_bytes = kBlockTokens * a.r_k * es;
+    p.block_table = a.block_table; p.max_blocks = a.max_blocks;
+    p.context_lens = a.context_lens; p.B = a.B; p.max_ctx = a.max_ctx;
+    p.q = a.q; p.cur_k = a.cur_k; p.cur_v = a.cur_v; p.out = a.out;
+    const size_t part = static_cast<size_t>(grid) * 2 * (a.r_v + 2) * sizeof(float);
+    const size_t part_al = (part + 255) & ~static_cast<size_t>(255);
+    p.partials = static_cast<float *>(a.workspace);
+    p.counters = reinterpret_cast<int *>(static_cast<char *>(a.workspace) + part_al);
+    p.pps = 1; p.stages = stages; p.stage_bytes = hpb;
+    p.err = err;
+    // theta_j = base^(-2j/d): its phase step in 64-bit fixed-point turns and the per-pair
+    // constants of the recurrence, in double precision
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int j = 0; j < kRopePairs; ++j) {
+        const double theta = pow(base, -2.0 * j / a.d);
+        const double turns = theta / two_pi;  // < 1: theta_j <= 1
+        rp.phi[j] = static_cast<unsigned long long>(ldexp(turns, 64));
+        rp.sn[j] = static_cast<float>(sin(theta));
+        const double sh = sin(0.5 * theta);
+        rp.hc[j] = static_cast<float>(2.0 * sh * sh);  // 1 - cos theta, without cancellation
+        rp.c16[j] = static_cast<float>(cos(16.0 * theta));
+        rp.s16[j] = static_cast<float>(sin(16.0 * theta));
+    }
+    rp.pairing = pairing;
+    return e.launch(rp, grid, smem, stream);
+}
+
+}  // namespace lla

@@ -70,6 +70,11 @@ inline size_t head_page_bytes(int r_k, int r_v, int es) {
 size_t decode_workspace_bytes(int r_v, int B, int H, int grid);
 lla_status decode_fits(int r_k, int r_v, int es, int d);  // UNSUPPORTED if no kernel shape fits
 lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream);
+// Decode with rotary positions after reconstruction (tensor-core key rebuild): UNSUPPORTED
+// unless a kernel shape exists and fits for B sequences; the launch takes the rotation base and
+// pairing (0: (j, j + d/2), 1: (2j, 2j + 1)).
+lla_status decode_rope_fits(int r_k, int r_v, int es, int d, int B);
+lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cudaStream_t stream);
 
 lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream);
 // The same encode for L layers (one launch for decode batches).

@@ -20,6 +20,7 @@ from .build import LIB
 LLA_BLOCK_TOKENS = 64
 LLA_MAX_BATCH = 1024
 LLA_BF16, LLA_F32 = 0, 1
+LLA_ROPE_HALF, LLA_ROPE_ADJACENT = 0, 1
 LLA_DEVERR_BLOCK_ID = 0x1
 LLA_DEVERR_CONTEXT = 0x2
 LLA_DEVERR_EMPTY_PASS2 = 0x4
@@ -45,6 +46,10 @@ class lla_geometry(ctypes.Structure):
 class lla_codec(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
                 ("w_down_k", "w_down_v", "w_up_k", "w_up_v", "mu_k", "mu_v")]
+
+
+class lla_rope(ctypes.Structure):
+    _fields_ = [("base", ctypes.c_double), ("pairing", ctypes.c_int32)]
 
 
 class lla_cache(ctypes.Structure):
@@ -74,6 +79,8 @@ def library() -> ctypes.CDLL:
             "lla_decode_workspace_init": (I32, [P, SZ, P]),
             "lla_decode_attn": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ, P]),
             "lla_decode_attn_noalloc": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P]),
+            "lla_decode_attn_rope": (I32, [P, P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ,
+                                           P]),
             "lla_prefill_attn": (I32, [P, P, P, P, I32, I32, I32, P, I32, P, P]),
             "lla_dense_store": (I32, [P, P, P, P, I32, P, I32, P]),
             "lla_dense_decode_attn": (I32, [P, P, P, I32, I32, P, P, P, I32, P, P, SZ, P]),
@@ -236,6 +243,22 @@ def lla_decode_attn(geom: Geometry, codec: Codec, cache: Cache, context_lens: to
         ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(context_lens), B, max_ctx,
         loop, _ptr(q), _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def lla_decode_attn_rope(geom: Geometry, codec: Codec, cache: Cache, rope_base: float,
+                         rope_pairing: int, context_lens: torch.Tensor, max_ctx: int, loop: int,
+                         q: torch.Tensor, cur_k: Optional[torch.Tensor],
+                         cur_v: Optional[torch.Tensor], out: torch.Tensor,
+                         workspace: torch.Tensor, stream=None) -> None:
+    """lla_decode_attn with RoPE after reconstruction; q and cur_k pre-RoPE.  rope_pairing:
+    LLA_ROPE_HALF (pairs (j, j + d/2)) or LLA_ROPE_ADJACENT (pairs (2j, 2j + 1))."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    rp = lla_rope(float(rope_base), int(rope_pairing))
+    _check("lla_decode_attn_rope", library().lla_decode_attn_rope(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), ctypes.byref(rp),
+        _ptr(context_lens), q.shape[0], max_ctx, loop, _ptr(q), _ptr(cur_k), _ptr(cur_v),
+        _dtype_code(q), _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
 
 
 def lla_decode_attn_noalloc(geom: Geometry, codec: Codec, cache: Cache,

@@ -8,6 +8,11 @@ that a profiler can skip the warm-up launches and capture one to three of them:
     ncu --set full --clock-control none -k regex:decode_async_kernel -s 6 -c 1 \\
         python -m paper_2607_15456_gb300.profile_case --workload ouro14_rho4 --layers 2 --calls 10
 
+rope: the same decode calls through lla_decode_attn_rope (RoPE after reconstruction, base 10^4):
+
+    ncu --set full --clock-control none -k regex:decode_rope_kernel -s 6 -c 1 \\
+        python -m paper_2607_15456_gb300.profile_case --case rope --workload ouro14_rho4 --layers 2 --calls 10
+
 prefill: encodes `--prompts` prompts of `--len` tokens of a workload's ranks (tensor-core encode,
 one launch per axis), then runs `--calls` causal prefill calls over them:
 
@@ -38,9 +43,15 @@ def decode_case(args):
     w = bench.w
     for i in range(args.calls):
         l, t = i % w.D, (i // w.D) % w.T
-        lla.lla_decode_attn(bench.geom, bench.codecs[l], bench.caches[l], bench.ctx, bench.max_ctx,
-                            t, bench.q[l, t], bench.cur_k[l, t], bench.cur_v[l, t], bench.out[l, t],
-                            bench.ws)
+        if args.case == "rope":
+            lla.lla_decode_attn_rope(bench.geom, bench.codecs[l], bench.caches[l], 10000.0,
+                                     lla.LLA_ROPE_HALF, bench.ctx, bench.max_ctx, t, bench.q[l, t],
+                                     bench.cur_k[l, t], bench.cur_v[l, t], bench.out[l, t],
+                                     bench.ws)
+        else:
+            lla.lla_decode_attn(bench.geom, bench.codecs[l], bench.caches[l], bench.ctx,
+                                bench.max_ctx, t, bench.q[l, t], bench.cur_k[l, t],
+                                bench.cur_v[l, t], bench.out[l, t], bench.ws)
     bench.encode_calls()
     torch.cuda.synchronize()
     err = lla.lla_get_device_error()
@@ -88,14 +99,14 @@ def prefill_case(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--case", choices=["decode", "prefill"], default="decode")
+    ap.add_argument("--case", choices=["decode", "rope", "prefill"], default="decode")
     ap.add_argument("--workload", default="ouro14_rho4")
     ap.add_argument("--layers", type=int, default=2)
     ap.add_argument("--calls", type=int, default=10)
     ap.add_argument("--prompts", type=int, default=4)
     ap.add_argument("--len", type=int, default=8192)
     args = ap.parse_args()
-    if args.case == "decode":
+    if args.case in ("decode", "rope"):
         decode_case(args)
     else:
         prefill_case(args)

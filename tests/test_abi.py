@@ -195,3 +195,35 @@ def test_encode_layers_argument_checks(lib):
     assert enc(xv=bad) == INVALID
     nocodec = (lib.lla_codec * L)(_codec(lib), _codec(lib, w_down_v=None))
     assert enc(codecs=nocodec) == INVALID
+
+
+def _decode_rope(lib, rope=None, g=None, codec=None, cache=None, lens=FAKE, B=4, max_ctx=128,
+                 loop=0, q=FAKE, ck=FAKE, cv=FAKE, io=0, out=FAKE, ws=FAKE, ws_bytes=1 << 20,
+                 no_rope=False):
+    so = lib.library()
+    g = g or _g(lib)
+    codec = codec or _codec(lib)
+    cache = cache or _cache(lib)
+    rope = rope or lib.lla_rope(10000.0, lib.LLA_ROPE_HALF)
+    return so.lla_decode_attn_rope(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache),
+                                   None if no_rope else ctypes.byref(rope), lens, B, max_ctx,
+                                   loop, q, ck, cv, io, out, ws, ws_bytes, None)
+
+
+def test_decode_rope_argument_checks(lib):
+    assert _decode_rope(lib, no_rope=True) == INVALID
+    assert _decode_rope(lib, rope=lib.lla_rope(1.0, 0)) == INVALID        # base must exceed 1
+    assert _decode_rope(lib, rope=lib.lla_rope(float("nan"), 0)) == INVALID
+    assert _decode_rope(lib, rope=lib.lla_rope(10000.0, 2)) == INVALID    # unknown pairing
+    assert _decode_rope(lib, q=FAKE + 8) == INVALID                       # q not 16-B aligned
+    assert _decode_rope(lib, out=FAKE + 4) == INVALID
+    assert _decode_rope(lib, ck=None) == INVALID                          # cur_k without cur_v
+    assert _decode_rope(lib, loop=4) == INVALID
+    assert _decode_rope(lib, ws=None) == INVALID
+    # shapes without a tensor-core key rebuild
+    assert _decode_rope(lib, g=_g(lib, r_k=72, r_v=120)) == UNSUPPORTED   # r_k not a multiple of 16
+    assert _decode_rope(lib, g=_g(lib, storage="fp32")) == UNSUPPORTED
+    assert _decode_rope(lib, g=_g(lib, d=64)) == UNSUPPORTED
+    assert _decode_rope(lib, B=0, lens=None, q=None, out=None, ws=None) == OK
+    assert _decode_rope(lib, rope=lib.lla_rope(500000.0, lib.LLA_ROPE_ADJACENT), B=0, lens=None,
+                        q=None, out=None, ws=None) == OK
