@@ -364,10 +364,7 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
         if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
         if (is_s && ks == 0) a.lred[rslot * kLredSlot + tt] = l_part;
         if (tid == 0) s.misc[kAM + rslot] = m_run;
-        if (vwork) {
-#pragma unroll
-            for (int e = 0; e < AV; ++e) a.red[rslot * a.redslot + tg * RV + vc * AV + e] = accv[e];
-        }
+        if (vwork) value_store<ES, RK, RV>(a.red + rslot * a.redslot, accv, vc, tg);
         mbar_arrive(&a.stfull[rslot]);
         u = R.run_end;
     }

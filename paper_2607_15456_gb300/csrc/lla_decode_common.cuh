@@ -596,7 +596,9 @@ __device__ __forceinline__ void load_qvec(const float *q, float (&v)[KE]) {
 
 // Value warps, one pipeline step: rescale this thread's latent value sums by the step's alpha,
 // then add p_i c_v,i for the step's valid tokens from the V-planes of the stage at `sb`.  The
-// thread owns UPT units of VE columns (vc) and the token rows tg, tg + NTG, ... of each page.
+// thread owns the units vc, vc + VC, ... (UPT units of VE columns, spread over the row so that
+// the eight threads of a shared-memory phase read neighbouring units) and the token rows
+// tg, tg + NTG, ... of each page.
 template <int ES, int RK, int RV>
 __device__ __forceinline__ void value_step(float (&accv)[Fast<ES, RK, RV>::UPT * Fast<ES, RK, RV>::VE],
                                            const char *sb, const float *pring, float alpha,
@@ -605,7 +607,7 @@ __device__ __forceinline__ void value_step(float (&accv)[Fast<ES, RK, RV>::UPT *
     constexpr int AV = F::UPT * F::VE;
 #pragma unroll
     for (int e = 0; e < AV; ++e) accv[e] *= alpha;
-    const char *vbase = sb + F::KPLANE + vc * (F::UPT * F::VB) + tg * F::ROWB;
+    const char *vbase = sb + F::KPLANE + vc * F::VB + tg * F::ROWB;
 #pragma unroll
     for (int pi = 0; pi < F::PPS; ++pi) {
         // rows tg, tg + NTG, ... of page pi that hold valid tokens
@@ -620,13 +622,38 @@ __device__ __forceinline__ void value_step(float (&accv)[Fast<ES, RK, RV>::UPT *
 #pragma unroll
             for (int uu = 0; uu < F::UPT; ++uu) {
                 float v[F::VE];
-                load_gran<ES, F::VB>(rowp + uu * F::VB, v);
+                load_gran<ES, F::VB>(rowp + uu * (F::VC * F::VB), v);
+                if constexpr (F::VE % 2 == 0) {
+                    const float2 p2 = make_float2(pv, pv);
 #pragma unroll
-                for (int e = 0; e < F::VE; ++e)
-                    accv[uu * F::VE + e] = fmaf(pv, v[e], accv[uu * F::VE + e]);
+                    for (int e = 0; e < F::VE; e += 2) {
+                        const float2 r = __ffma2_rn(p2, make_float2(v[e], v[e + 1]),
+                                                    make_float2(accv[uu * F::VE + e],
+                                                                accv[uu * F::VE + e + 1]));
+                        accv[uu * F::VE + e] = r.x;
+                        accv[uu * F::VE + e + 1] = r.y;
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < F::VE; ++e)
+                        accv[uu * F::VE + e] = fmaf(pv, v[e], accv[uu * F::VE + e]);
+                }
             }
         }
     }
+}
+
+// Value warps at a run's end: this thread's latent value sums into its token group's row of the
+// run's state (red [NTG][RV]), at the columns of the units it owns.
+template <int ES, int RK, int RV>
+__device__ __forceinline__ void value_store(float *red, const float (&accv)[Fast<ES, RK, RV>::UPT * Fast<ES, RK, RV>::VE],
+                                            int vc, int tg) {
+    using F = Fast<ES, RK, RV>;
+#pragma unroll
+    for (int uu = 0; uu < F::UPT; ++uu)
+#pragma unroll
+        for (int e = 0; e < F::VE; ++e)
+            red[tg * RV + (vc + uu * F::VC) * F::VE + e] = accv[uu * F::VE + e];
 }
 
 // ------------------------------------------------------------------------------------------

@@ -43,46 +43,44 @@ constexpr int kMmaWarp = kAsyncThreads / 32;       // warp 13, after the managem
 constexpr int kRopeThreads = kAsyncThreads + 32;   // 448
 constexpr int kRopeWst = 20 * 1024;                // staging buffer of W_up,t^V rows
 constexpr int kBarTmem = 5;                        // epilogue warps + MMA warp, before dealloc
-constexpr int kXposeStride = 20;                   // floats per row of a transpose buffer
-constexpr int kXposeFloats = 32 * kXposeStride + 16;
 
 // Launch parameters: the decode parameters plus, per rotation pair j, the phase step theta_j as
-// 64-bit fixed-point turns (theta_j / 2 pi * 2^64), sin theta_j, 1 - cos theta_j, and
-// cos / sin of 16 theta_j, all computed on the host in double precision.
+// 64-bit fixed-point turns (theta_j / 2 pi * 2^64), cos / sin of theta_j and of 32 theta_j, and
+// sin 2 theta_j and 1 - cos 2 theta_j, all computed on the host in double precision.
 struct RopeParams {
     Params p;
     unsigned long long phi[kRopePairs];
-    float sn[kRopePairs], hc[kRopePairs], c16[kRopePairs], s16[kRopePairs];
+    float c1[kRopePairs], s1[kRopePairs], c32[kRopePairs], s32[kRopePairs];
+    float s2[kRopePairs], h2[kRopePairs];
     int pairing;  // 0: pair j = (j, j + d/2); 1: pair j = (2j, 2j + 1)
 };
 
 template <int RK, int RV>
 struct RopeShape {
     using F = Fast<2, RK, RV>;
-    static constexpr int NG = RK / 8;               // 16-byte granules per row of W_up,t^K
     static constexpr int KSTEPS = RK / 16;          // MMAs of K = 16 per page
-    static constexpr int A_BYTES = NG * kRopeD * 16;
-    // A slot: the NG granules of W_up,t^K, then (mu_hi, mu_lo, 0, ...) and a zero granule
-    static constexpr int A_SLOT = A_BYTES + 2 * kRopeD * 16;
+    // TMEM columns: two 64-column accumulators, then two A slots of W_up,t^K (two bf16 per
+    // column) followed by the mu step's (mu_hi, mu_lo, 0, ...) in 8 more columns
+    static constexpr int A_COLS = RK / 2 + 8;
+    static constexpr int A_STRIDE = A_COLS <= 64 ? 64 : 96;
+    static constexpr int TMEM_COLS = 128 + 2 * A_STRIDE <= 256 ? 256 : 512;
     static constexpr uint32_t IDESC = umma_idesc_bf16(kRopeD, 64, 0, 0);
-    static_assert(RK % 16 == 0, "whole K steps of 16 latent columns");
+    static_assert(RK % 32 == 0, "whole K steps, W_up,t^K rows in 16-column TMEM stores");
+    static_assert(A_COLS <= A_STRIDE, "A slot");
     static_assert(F::PPS == 1 && F::TT == 64, "one page per pipeline step");
     static_assert(F::S_WARPS == 4 && F::V_WARPS == 4, "four epilogue and four value warps");
 };
 
 struct RopeLayout {
-    int aslot, ones, xpose, red, bars, tmem, total;
+    int ones, red, bars, tmem, total;
 };
 
 template <int RK, int RV>
 __host__ __device__ inline RopeLayout rope_layout(int stages, int stage_bytes, int B) {
-    using Z = RopeShape<RK, RV>;
     RopeLayout L;
     int o = (async_layout<2, RK, RV, kRopeD, kRopeWst>(stages, stage_bytes, B).total + 127) & ~127;
-    L.aslot = o; o += 2 * Z::A_SLOT;
     L.ones = o;  o += 2 * 64 * 16;                // B operand of the mu step: (1, 1, 0...) and zeros
-    L.xpose = o; o += 4 * kXposeFloats * 4;
-    L.red = o;   o += 4 * 64 * 4;
+    L.red = o;   o += 2 * 4 * 64 * 4;             // per-warp partial scores, two page slots
     L.bars = o;  o += 8 * 8;                      // aful[2], afree[2], tfull[2], tfree[2]
     L.tmem = o;  o += 16;
     L.total = o;
@@ -99,9 +97,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
     const ASmem a = carve_async<ES, RK, RV, D, kRopeWst>(smem, p);
     const Smem &s = a.s;
     const RopeLayout RL = rope_layout<RK, RV>(p.stages, p.stage_bytes, p.B);
-    char *aslot = smem + RL.aslot;
     char *ones = smem + RL.ones;
-    float *xpose = reinterpret_cast<float *>(smem + RL.xpose);
     float *red4 = reinterpret_cast<float *>(smem + RL.red);
     uint64_t *aful = reinterpret_cast<uint64_t *>(smem + RL.bars);
     uint64_t *afree = aful + 2, *tfull = aful + 4, *tfree = aful + 6;
@@ -113,7 +109,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
     if (tid == 0) {
         for (int i = 0; i < kQSlots; ++i) mbar_init(&a.qready[i], kMThreads);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&a.stfull[i], kComputeThreads);
+            mbar_init(&a.stfull[i], F::V_THREADS);  // the value warps hold a run's state
             mbar_init(&a.stfree[i], kMThreads);
             mbar_init(&aful[i], 1);
             mbar_init(&afree[i], 1);
@@ -122,19 +118,16 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         }
     }
     if (warp == kMmaWarp) {
-        tmem_alloc(tmem_slot, 128);  // two 64-column accumulators
-        // constant operand parts: the ones column pair of the mu step and the zero granules
+        tmem_alloc(tmem_slot, Z::TMEM_COLS);
+        // the B operand of the mu step: a (1, 1) pair per token, then a zero granule
         uint4 *o4 = reinterpret_cast<uint4 *>(ones);
         for (int i = lane; i < 128; i += 32)
             o4[i] = i < 64 ? make_uint4(0x3f803f80u, 0u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
-        for (int sl = 0; sl < 2; ++sl) {
-            uint4 *z4 = reinterpret_cast<uint4 *>(aslot + sl * Z::A_SLOT + Z::A_BYTES + D * 16);
-            for (int i = lane; i < D; i += 32) z4[i] = make_uint4(0u, 0u, 0u, 0u);
-        }
         fence_proxy_async_smem();
         tc_fence_before();
     }
-    // one arrival per pipeline step on empty: the MMA warp's commit and the four value warps
+    // empty: one arrival per page from the MMA warp's commit and one from each value warp;
+    // pfull: the epilogue threads (a page's partial scores); pempty: the value threads
     Range rg = prologue(p, s, kComputeThreads / 2, F::V_THREADS, 1 + F::V_WARPS);
     order_runs(p, s, rg);
     pdl_trigger();
@@ -152,12 +145,12 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         int it = 0, stage = 0, r = 0;
         uint32_t ph = 0;
         const bool has_mu = p.mu_k != nullptr;
-        const uint32_t ones_desc_lo = smem_addr(ones);
+        const uint64_t ones_desc = umma_desc(smem_addr(ones), 1024, 128);
         for (int pass = 0; pass < 3; ++pass)
         for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
             const Run R = locate_run(p, s, u, rg.hi[pass]);
             const int as = r & 1;
-            const uint32_t abase = smem_addr(aslot + as * Z::A_SLOT);
+            const uint32_t acol = tmem_base + 128 + as * Z::A_STRIDE;
             if (lane == 0) mbar_wait(&aful[as], (r >> 1) & 1, s.abort_flag, p.err);
             for (int k = 0; k < R.npages; ++k, ++it) {
                 const int b = it & 1;
@@ -169,11 +162,9 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
                     const uint32_t bbase = smem_addr(s.ring + stage * p.stage_bytes);
 #pragma unroll
                     for (int st = 0; st < Z::KSTEPS; ++st)
-                        umma_bf16(d, umma_desc(abase + st * 4096, 2048, 128),
-                                  umma_desc(bbase + st * 2048, 1024, 128), Z::IDESC, st > 0);
-                    if (has_mu)
-                        umma_bf16(d, umma_desc(abase + Z::A_BYTES, 2048, 128),
-                                  umma_desc(ones_desc_lo, 1024, 128), Z::IDESC, true);
+                        umma_bf16_ts(d, acol + st * 8, umma_desc(bbase + st * 2048, 1024, 128),
+                                     Z::IDESC, st > 0);
+                    if (has_mu) umma_bf16_ts(d, acol + RK / 2, ones_desc, Z::IDESC, true);
                     umma_commit(&tfull[b]);
                     umma_commit(&s.empty[stage]);  // the K-plane has been read
                     if (k == R.npages - 1) umma_commit(&afree[as]);
@@ -193,7 +184,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         }
         named_bar_sync(kBarTmem, 128 + 32);  // the epilogue warps have read every buffer
         tc_fence_after();
-        tmem_dealloc(tmem_base, 128);
+        tmem_dealloc(tmem_base, Z::TMEM_COLS);
         return;
     }
 
@@ -204,6 +195,9 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
             m_finish<ES, RK, RV, D, F::TT, F::NTG, kRopeWst>(p, a, R, u, rg, k & 1, (k >> 1) & 1,
                                                             k % kQSlots, mt);
         };
+        // this thread's row of W_up,t^K is TMEM lane `row` (the warp's lane quarter)
+        const int row = 32 * (warp & 3) + lane;
+        const uint32_t tlane = tmem_base + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         int r = 0;
         Run q0{}, q1{};
         int64_t u0 = 0, u1 = 0;
@@ -211,28 +205,39 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         for (int64_t u = rg.lo[pass]; u < rg.hi[pass];) {
             const Run R = locate_run(p, s, u, rg.hi[pass]);
             const int slot = r % kQSlots, as = r & 1;
-            // W_up,t^K of head R.h into A slot `as` once run r - 2's MMAs have read it
-            if (r >= 2) mbar_wait(&afree[as], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
-            char *A = aslot + as * Z::A_SLOT;
-            const int64_t hl = (static_cast<int64_t>(R.h) * p.T + p.loop) * D;
-            const char *W = static_cast<const char *>(p.w_up_k) + hl * RK * ES;
-            cp_async_wait_all();  // no earlier copy of this thread is still in flight
-            for (int i = mt; i < D * Z::NG; i += kMThreads) {
-                const int row = i / Z::NG, g = i - row * Z::NG;
-                cp_async16(A + g * (D * 16) + row * 16, W + row * (RK * ES) + g * 16);
-            }
-            cp_async_commit();
             if (r == 0) named_bar_arrive(kBarStart, kMThreads + 32);  // the ring may start
-            if (mt < D) {
-                const float mu = p.mu_k ? p.mu_k[hl + mt] : 0.f;
-                const __nv_bfloat16 hi = __float2bfloat16_rn(mu);
-                const __nv_bfloat16 lo = __float2bfloat16_rn(mu - __bfloat162float(hi));
-                const uint32_t w0 = static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
-                                    (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16);
-                *reinterpret_cast<uint4 *>(A + Z::A_BYTES + mt * 16) = make_uint4(w0, 0u, 0u, 0u);
+            // W_up,t^K of head R.h and mu^K_t into A slot `as` once run r - 2's MMAs have read it
+            const int64_t hl = (static_cast<int64_t>(R.h) * p.T + p.loop) * D;
+            const uint4 *W4 = reinterpret_cast<const uint4 *>(
+                static_cast<const char *>(p.w_up_k) + (hl + row) * (RK * ES));
+            uint32_t wv[RK / 2];
+#pragma unroll
+            for (int g = 0; g < RK / 8; ++g) {
+                const uint4 w = W4[g];
+                wv[4 * g] = w.x;
+                wv[4 * g + 1] = w.y;
+                wv[4 * g + 2] = w.z;
+                wv[4 * g + 3] = w.w;
             }
-            cp_async_wait_all();
-            fence_proxy_async_smem();  // the slot's writes become visible to the tensor core
+            const float mu = p.mu_k ? p.mu_k[hl + row] : 0.f;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(mu);
+            const __nv_bfloat16 lo = __float2bfloat16_rn(mu - __bfloat162float(hi));
+            uint32_t mv[8] = {static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
+                                  (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16),
+                              0u, 0u, 0u, 0u, 0u, 0u, 0u};
+            if (r >= 2) mbar_wait(&afree[as], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
+            tc_fence_after();
+            const uint32_t acol = tlane + 128 + as * Z::A_STRIDE;
+#pragma unroll
+            for (int c = 0; c < RK / 32; ++c) {
+                uint32_t part[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) part[i] = wv[16 * c + i];
+                tmem_st16u(acol + 16 * c, part);
+            }
+            tmem_st8u(acol + RK / 2, mv);
+            tmem_wait_st();
+            tc_fence_before();
             m_sync();
             if (mt == 0) mbar_arrive(&aful[as]);
             m_setup<ES, RK, RV, D, false, kRopeWst>(p, a, R.b, R.h, slot, mt, false);
@@ -251,10 +256,10 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
             if (s.lens[b] != 0) continue;
             for (int h = 0; h < p.H; ++h) {
                 if ((b * p.H + h) % gridDim.x != blockIdx.x) continue;
-                const int64_t row = (static_cast<int64_t>(b) * p.H + h) * D;
+                const int64_t orow = (static_cast<int64_t>(b) * p.H + h) * D;
                 if (!pass1 && mt == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
                 for (int e = mt; e < D; e += kMThreads)
-                    store_elem(p.out, row + e, pass1 ? load_elem(p.cur_v, row + e, p.io_bf16) : 0.f,
+                    store_elem(p.out, orow + e, pass1 ? load_elem(p.cur_v, orow + e, p.io_bf16) : 0.f,
                                p.io_bf16);
             }
         }
@@ -270,18 +275,15 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         const bool upper = rp.pairing ? (m & 1) : (m >= kRopePairs);
         const int ia = rp.pairing ? 2 * j : j, ib = rp.pairing ? 2 * j + 1 : j + kRopePairs;
         const unsigned long long phi = rp.phi[j];
-        const float sn = rp.sn[j], hc = rp.hc[j], lam = 2.f * rp.hc[j];
-        const float c16 = rp.c16[j], s16 = rp.s16[j];
-        float *xb = xpose + warp * kXposeFloats;
-        float *xrow = xb + lane * kXposeStride + (lane >= 16 ? 16 : 0);
-        const int hf = lane >> 4, col = lane & 15;
-        const float *xcol = xb + hf * 16 * kXposeStride + hf * 16 + col;
+        const float c1 = rp.c1[j], s1 = rp.s1[j], c32 = rp.c32[j], s32 = rp.s32[j];
+        const float s2 = rp.s2[j], h2 = rp.h2[j];
+        const float2 nlam = make_float2(-2.f * h2, -2.f * h2);  // -(2 - 2 cos 2 theta_j)
         const uint32_t tlane = tmem_base + (static_cast<uint32_t>(32 * warp) << 16);
         int it = 0, r = 0;
         for (int pass = 0; pass < 3; ++pass)
         for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
             const Run R = locate_run(p, s, u, rg.hi[pass]);
-            const int rslot = r & 1, qslot = r % kQSlots;
+            const int qslot = r % kQSlots;
             mbar_wait(&a.qready[qslot], (r / kQSlots) & 1, s.abort_flag, p.err);
             // element m of rot(q, Delta) = Re(G e^{i Delta theta_j}), scaled to log2 units
             float Gr, Gi;
@@ -292,101 +294,98 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
                 Gi = (upper ? -qa : qb) * p.scale_log2;
             }
             const int P = pass1 ? R.Lb : R.Lb - 1;  // the query's position
-            float m_run = -INFINITY, l_part = 0.f;
             for (int k = 0; k < R.npages; ++k, ++it) {
                 const int b = it & 1, slot = it & 1;
-                const uint32_t pph = (it >> 1) & 1;
                 const int pg = R.pg0 + k;
-                const int nvalid = min(kBlockTokens, R.Lb - pg * kBlockTokens);
-                mbar_wait(&tfull[b], (it >> 1) & 1, s.abort_flag, p.err);
-                tc_fence_after();
                 // exact phase of the page's first token: Delta0 theta_j in turns, mod 1
                 const int delta0 = P - pg * kBlockTokens;  // >= 0: the page holds a cached token
                 const unsigned long long turns = static_cast<unsigned long long>(delta0) * phi;
                 const float tf = __uint2float_rn(static_cast<uint32_t>(turns >> 32)) * 2.3283064365386963e-10f;
                 float sa, ca;
                 sincospif(2.f * tf, &sa, &ca);
-                float zr = Gr * ca - Gi * sa, zi = Gr * sa + Gi * ca;
+                const float zr = Gr * ca - Gi * sa, zi = Gr * sa + Gi * ca;
+                // x_i = Re(z e^{-i i theta}) for the page's tokens i, in four chains that step two
+                // tokens at a time (even and odd tokens of each half, packed in pairs):
+                // dd = x_i - x_{i-2};  dd' = dd - (2 - 2 cos 2 theta) x;  x' = x + dd'
+                float2 X[2], DD[2];
 #pragma unroll
-                for (int hv = 0; hv < 2; ++hv) {  // tokens 32 hv .. 32 hv + 31
-                    float v[32];
-                    tmem_ld32(tlane + b * 64 + 32 * hv, v);
-                    if (hv == 1) {
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&tfree[b]);  // the buffer may take page it + 2
-                    }
-                    // two chains of 16 tokens: x = Re(z e^{-i r theta}), dd = x_r - x_{r-1}
-                    float x[2], dd[2];
+                for (int hv = 0; hv < 2; ++hv) {
+                    // the half's first token: z e^{-i 32 hv theta}; the odd chain one token later
+                    const float er = hv ? fmaf(zr, c32, zi * s32) : zr;
+                    const float ei = hv ? fmaf(zi, c32, -zr * s32) : zi;
+                    const float orr = fmaf(er, c1, ei * s1), oi = fmaf(ei, c1, -er * s1);
+                    X[hv] = make_float2(er, orr);
+                    DD[hv] = make_float2(fmaf(er, h2, ei * s2), fmaf(orr, h2, oi * s2));
+                }
+                uint32_t v0[32], v1[32];  // this dimension of tokens 0..31 and 32..63
+                mbar_wait(&tfull[b], (it >> 1) & 1, s.abort_flag, p.err);
+                tc_fence_after();
+                const uint32_t tcol = tlane + b * 64;
+                tmem_ld32_nowait(tcol, v0);
+                tmem_ld32_nowait(tcol + 32, v1);
+                tmem_wait_ld(v0);
+                tmem_wait_ld(v1);
+                // this dimension's score terms in place
 #pragma unroll
-                    for (int c = 0; c < 2; ++c) {
-                        x[c] = zr;
-                        dd[c] = fmaf(zr, hc, zi * sn);
-                        const float nr = fmaf(zr, c16, zi * s16), ni = fmaf(zi, c16, -zr * s16);
-                        zr = nr;
-                        zi = ni;
-                    }
+                for (int t = 0; t < 16; ++t) {
+                    float2 a0 = make_float2(__uint_as_float(v0[2 * t]), __uint_as_float(v0[2 * t + 1]));
+                    float2 a1 = make_float2(__uint_as_float(v1[2 * t]), __uint_as_float(v1[2 * t + 1]));
+                    a0 = __fmul2_rn(a0, X[0]);
+                    a1 = __fmul2_rn(a1, X[1]);
+                    v0[2 * t] = __float_as_uint(a0.x);
+                    v0[2 * t + 1] = __float_as_uint(a0.y);
+                    v1[2 * t] = __float_as_uint(a1.x);
+                    v1[2 * t + 1] = __float_as_uint(a1.y);
+                    DD[0] = __ffma2_rn(nlam, X[0], DD[0]);
+                    DD[1] = __ffma2_rn(nlam, X[1], DD[1]);
+                    X[0] = __fadd2_rn(X[0], DD[0]);
+                    X[1] = __fadd2_rn(X[1], DD[1]);
+                }
+                // sum over the 128 dimensions of each token: the terms go back to TMEM and return
+                // in the 16x256b layout (4 dimensions x 16 tokens per thread), are summed over
+                // the 4 dimensions, then over the 8 threads of each token group by shuffles
+                tmem_st32u_nowait(tcol, v0);
+                tmem_st32u_nowait(tcol + 32, v1);
+                tmem_wait_st();
+                tmem_ld16x256_x8_nowait(tcol, v0);                                  // dims +0, +8
+                tmem_ld16x256_x8_nowait(tcol + (static_cast<uint32_t>(16) << 16), v1);  // +16, +24
+                tmem_wait_ld(v0);
+                tmem_wait_ld(v1);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tfree[b]);  // the buffer may take page it + 2
+                float S[16];  // S[2k + e]: token 8k + 2(lane % 4) + e, summed over 4 dimensions
 #pragma unroll
-                    for (int t = 0; t < 16; ++t) {
+                for (int k8 = 0; k8 < 8; ++k8) {
+                    const float2 a = __fadd2_rn(
+                        make_float2(__uint_as_float(v0[4 * k8]), __uint_as_float(v0[4 * k8 + 1])),
+                        make_float2(__uint_as_float(v0[4 * k8 + 2]), __uint_as_float(v0[4 * k8 + 3])));
+                    const float2 c = __fadd2_rn(
+                        make_float2(__uint_as_float(v1[4 * k8]), __uint_as_float(v1[4 * k8 + 1])),
+                        make_float2(__uint_as_float(v1[4 * k8 + 2]), __uint_as_float(v1[4 * k8 + 3])));
+                    const float2 sum = __fadd2_rn(a, c);
+                    S[2 * k8] = sum.x;
+                    S[2 * k8 + 1] = sum.y;
+                }
+                // lanes differing in bits 4, 3, 2 hold the same tokens: halve the token set per
+                // level, keeping the half that the lane's bit selects
 #pragma unroll
-                        for (int c = 0; c < 2; ++c) {
-                            v[c * 16 + t] *= x[c];
-                            dd[c] = fmaf(-lam, x[c], dd[c]);
-                            x[c] += dd[c];
-                        }
-                    }
-                    // sum over the 128 dimensions of each token: per warp through a transpose
-                    // of 16-token chunks, then across the four warps
+                for (int lv = 0; lv < 3; ++lv) {
+                    const int half = 8 >> lv, bit = 16 >> lv;
+                    const bool up = lane & bit;
 #pragma unroll
-                    for (int ch = 0; ch < 2; ++ch) {
-#pragma unroll
-                        for (int q4 = 0; q4 < 4; ++q4)
-                            *reinterpret_cast<float4 *>(xrow + 4 * q4) =
-                                make_float4(v[ch * 16 + 4 * q4], v[ch * 16 + 4 * q4 + 1],
-                                            v[ch * 16 + 4 * q4 + 2], v[ch * 16 + 4 * q4 + 3]);
-                        __syncwarp();
-                        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-                        for (int kk = 0; kk < 16; kk += 4) {
-                            s0 += xcol[(kk + 0) * kXposeStride];
-                            s1 += xcol[(kk + 1) * kXposeStride];
-                            s2 += xcol[(kk + 2) * kXposeStride];
-                            s3 += xcol[(kk + 3) * kXposeStride];
-                        }
-                        float acc = (s0 + s1) + (s2 + s3);
-                        acc += __shfl_xor_sync(0xffffffffu, acc, 16);
-                        if (lane < 16) red4[warp * 64 + hv * 32 + ch * 16 + col] = acc;
-                        __syncwarp();
+                    for (int i = 0; i < half; ++i) {
+                        const float lo = S[i], hi = S[i + half];
+                        const float keep = up ? hi : lo, send = up ? lo : hi;
+                        S[i] = keep + __shfl_xor_sync(0xffffffffu, send, bit);
                     }
                 }
-                named_bar_sync(kBarTok, F::S_THREADS);
-                // online softmax over the page's tokens (threads 0..63, one token each)
-                float *wmax = s.misc + kAWmax + slot * 8;
-                float xs = -INFINITY;
-                if (tid < kBlockTokens) {
-                    const float sc = (red4[tid] + red4[64 + tid]) + (red4[128 + tid] + red4[192 + tid]);
-                    xs = tid < nvalid ? sc : -INFINITY;
-                    const float lm = warp_max(xs);
-                    if (lane == 0) wmax[warp] = lm;
-                }
-                named_bar_sync(kBarTok, F::S_THREADS);
-                float *pring = s.psm + slot * kComputeThreads;
-                if (tid < kBlockTokens) {
-                    const float m_new = fmaxf(m_run, fmaxf(wmax[0], wmax[1]));
-                    const float alpha = exp2f(m_run - m_new);
-                    m_run = m_new;
-                    mbar_wait(&s.pempty[slot], pph ^ 1u, s.abort_flag, p.err);
-                    const float pv = tid < nvalid ? exp2f(xs - m_new) : 0.f;
-                    pring[tid] = pv;
-                    l_part = fmaf(l_part, alpha, pv);
-                    if (tid == 0) s.misc[kAPAlpha + slot] = alpha;
-                }
+                // this lane holds the warp's sums for tokens 2 lane and 2 lane + 1
+                mbar_wait(&s.pempty[slot], ((it >> 1) & 1) ^ 1u, s.abort_flag, p.err);
+                *reinterpret_cast<float2 *>(red4 + slot * 256 + warp * 64 + 2 * lane) =
+                    make_float2(S[0], S[1]);
                 mbar_arrive(&s.pfull[slot]);
             }
-            if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
-            if (tid < kBlockTokens) a.lred[rslot * kLredSlot + tid] = l_part;
-            if (tid == 0) s.misc[kAM + rslot] = m_run;
-            mbar_arrive(&a.stfull[rslot]);
             u = R.run_end;
         }
         tc_fence_before();
@@ -395,7 +394,9 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
     }
 
     // --------------------------------------------------------------------------- value warps
-    const int vt = tid - F::S_THREADS;
+    // Per page: the online softmax over the page's scores (threads vt < 64, one token each),
+    // then sum_i p_i c_v,i from the V-plane.
+    const int vt = tid - F::S_THREADS, vwarp = warp - F::S_WARPS;
     const int vc = vt % F::VC, tg = vt / F::VC;
     const bool vwork = tg < F::NTG;
     constexpr int AV = F::UPT * F::VE;
@@ -405,6 +406,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
     for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
         const Run R = locate_run(p, s, u, rg.hi[pass]);
         const int rslot = r & 1;
+        float m_run = -INFINITY, l_part = 0.f;
         float accv[AV];
 #pragma unroll
         for (int e = 0; e < AV; ++e) accv[e] = 0.f;
@@ -413,12 +415,31 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
             const uint32_t pph = (it >> 1) & 1;
             const char *sb = s.ring + stage * p.stage_bytes;
             const int nvalid = min(kBlockTokens, R.Lb - (R.pg0 + k) * kBlockTokens);
-            mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+            float *wmax = s.misc + kAWmax + slot * 8;
+            float *pring = s.psm + slot * kComputeThreads;
             mbar_wait(&s.pfull[slot], pph, s.abort_flag, p.err);
-            if (vwork)
-                value_step<ES, RK, RV>(accv, sb, s.psm + slot * kComputeThreads,
-                                       s.misc[kAPAlpha + slot], nvalid, vc, tg);
-            mbar_arrive(&s.pempty[slot]);
+            float xs = -INFINITY;
+            if (vt < kBlockTokens) {
+                const float *rs = red4 + slot * 256;
+                const float sc = (rs[vt] + rs[64 + vt]) + (rs[128 + vt] + rs[192 + vt]);
+                xs = vt < nvalid ? sc : -INFINITY;
+                const float lm = warp_max(xs);
+                if (lane == 0) wmax[vwarp] = lm;
+            }
+            mbar_arrive(&s.pempty[slot]);  // the partial scores are read
+            named_bar_sync(kBarTok, F::V_THREADS);
+            if (vt < kBlockTokens) {
+                const float m_new = fmaxf(m_run, fmaxf(wmax[0], wmax[1]));
+                const float alpha = exp2f(m_run - m_new);
+                m_run = m_new;
+                const float pv = vt < nvalid ? exp2f(xs - m_new) : 0.f;
+                pring[vt] = pv;
+                l_part = fmaf(l_part, alpha, pv);
+                if (vt == 0) s.misc[kAPAlpha + slot] = alpha;
+            }
+            named_bar_sync(kBarTok, F::V_THREADS);
+            mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+            if (vwork) value_step<ES, RK, RV>(accv, sb, pring, s.misc[kAPAlpha + slot], nvalid, vc, tg);
             __syncwarp();
             if (lane == 0) mbar_arrive(&s.empty[stage]);  // V-plane read
             if (++stage == p.stages) {
@@ -427,10 +448,9 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
             }
         }
         if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
-        if (vwork) {
-#pragma unroll
-            for (int e = 0; e < AV; ++e) a.red[rslot * a.redslot + tg * RV + vc * AV + e] = accv[e];
-        }
+        if (vt < kBlockTokens) a.lred[rslot * kLredSlot + vt] = l_part;
+        if (vt == 0) s.misc[kAM + rslot] = m_run;
+        if (vwork) value_store<ES, RK, RV>(a.red + rslot * a.redslot, accv, vc, tg);
         mbar_arrive(&a.stfull[rslot]);
         u = R.run_end;
     }
@@ -519,11 +539,13 @@ lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cud
         const double theta = pow(base, -2.0 * j / a.d);
         const double turns = theta / two_pi;  // < 1: theta_j <= 1
         rp.phi[j] = static_cast<unsigned long long>(ldexp(turns, 64));
-        rp.sn[j] = static_cast<float>(sin(theta));
-        const double sh = sin(0.5 * theta);
-        rp.hc[j] = static_cast<float>(2.0 * sh * sh);  // 1 - cos theta, without cancellation
-        rp.c16[j] = static_cast<float>(cos(16.0 * theta));
-        rp.s16[j] = static_cast<float>(sin(16.0 * theta));
+        rp.c1[j] = static_cast<float>(cos(theta));
+        rp.s1[j] = static_cast<float>(sin(theta));
+        rp.c32[j] = static_cast<float>(cos(32.0 * theta));
+        rp.s32[j] = static_cast<float>(sin(32.0 * theta));
+        rp.s2[j] = static_cast<float>(sin(2.0 * theta));
+        const double sh = sin(theta);
+        rp.h2[j] = static_cast<float>(2.0 * sh * sh);  // 1 - cos 2 theta, without cancellation
     }
     rp.pairing = pairing;
     return e.launch(rp, grid, smem, stream);
