@@ -31,6 +31,8 @@
 //   * four value warps: sum_i p_i c_v,i from the V-plane (shared with lla_decode.cu).
 //   * four management warps: per run, W_up,t^K and mu^K_t into an A slot and q into a query
 //     slot; the merge of split runs and W_up,t^V, mu^V_t, 1/l (shared with lla_decode.cu).
+#include <string.h>
+
 #include "lla_decode_common.cuh"
 #include "lla_tcgen05.cuh"
 
@@ -105,7 +107,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool pass1 = p.cur_k != nullptr;
 
-    pdl_wait();  // inputs may come from the previous kernel in the stream
+    // set-up that reads no input runs before the previous kernel in the stream has finished
     if (tid == 0) {
         for (int i = 0; i < kQSlots; ++i) mbar_init(&a.qready[i], kMThreads);
         for (int i = 0; i < 2; ++i) {
@@ -126,6 +128,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         fence_proxy_async_smem();
         tc_fence_before();
     }
+    pdl_wait();  // inputs may come from the previous kernel in the stream
     // empty: one arrival per page from the MMA warp's commit and one from each value warp;
     // pfull: the epilogue threads (a page's partial scores); pempty: the value threads
     Range rg = prologue(p, s, kComputeThreads / 2, F::V_THREADS, 1 + F::V_WARPS);
@@ -533,7 +536,25 @@ lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cud
     p.pps = 1; p.stages = stages; p.stage_bytes = hpb;
     p.err = err;
     // theta_j = base^(-2j/d): its phase step in 64-bit fixed-point turns and the per-pair
-    // constants of the recurrence, in double precision
+    // constants of the recurrence, in double precision (kept for the next call with the same
+    // base and head width)
+    struct TableCache {
+        double base = 0.0;
+        int d = 0;
+        RopeParams rp;
+    };
+    static thread_local TableCache cache;
+    if (cache.base == base && cache.d == a.d) {
+        memcpy(rp.phi, cache.rp.phi, sizeof(rp.phi));
+        memcpy(rp.c1, cache.rp.c1, sizeof(rp.c1));
+        memcpy(rp.s1, cache.rp.s1, sizeof(rp.s1));
+        memcpy(rp.c32, cache.rp.c32, sizeof(rp.c32));
+        memcpy(rp.s32, cache.rp.s32, sizeof(rp.s32));
+        memcpy(rp.s2, cache.rp.s2, sizeof(rp.s2));
+        memcpy(rp.h2, cache.rp.h2, sizeof(rp.h2));
+        rp.pairing = pairing;
+        return e.launch(rp, grid, smem, stream);
+    }
     const double two_pi = 6.283185307179586476925286766559;
     for (int j = 0; j < kRopePairs; ++j) {
         const double theta = pow(base, -2.0 * j / a.d);
@@ -548,6 +569,9 @@ lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cud
         rp.h2[j] = static_cast<float>(2.0 * sh * sh);  // 1 - cos 2 theta, without cancellation
     }
     rp.pairing = pairing;
+    cache.base = base;
+    cache.d = a.d;
+    cache.rp = rp;
     return e.launch(rp, grid, smem, stream);
 }
 
