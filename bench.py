@@ -473,7 +473,22 @@ def run_extras(device):
         "frac": pf_flops / (pf_ms / 1e3) / 1e12 / tc_peak,
         "peak_source": "measured sustained cuBLAS bf16 (MEASURED_PEAKS.json bf16_tflops_sustained)",
         "flops_per_call": pf_flops}
-    del q, o, pool, cache
+    # the same prompts with rotary positions after reconstruction: keys rebuilt and rotated
+    # (tcgen05), then the causal attention over them (Sec. 3 "RoPE and reconstruction")
+    ws = torch.empty(lla.lla_prefill_rope_workspace_size(geom, nseq, L), dtype=torch.uint8, device=device)
+    rp_ms = _time_ms(lambda: lla.lla_prefill_attn_rope(geom, codec, cache, ROPE_BASE, lla.LLA_ROPE_HALF,
+                                                       cu, L, 1, q, o, ws))
+    rp_flops = (pairs * 2 * (d + w.r_v) + N * H * 2 * d * w.r_k + N * H * 2 * d * w.r_v)
+    out["rope_prefill"] = {
+        "workload": f"{w.name} causal prefill with RoPE after reconstruction (base {ROPE_BASE:g}), "
+                    f"{nseq}x{L} tokens, H={H}, one layer and loop",
+        "kernel": "rope_rebuild_kernel + prefill_tc_kernel<ROPE> (lla_prefill_attn_rope)",
+        "bound": "tensor", "ms_per_call": rp_ms, "tokens_per_s": N / (rp_ms / 1e3),
+        "TFLOP_s": rp_flops / (rp_ms / 1e3) / 1e12, "peak_TFLOP_s": tc_peak,
+        "frac": rp_flops / (rp_ms / 1e3) / 1e12 / tc_peak, "flops_per_call": rp_flops,
+        "note": "flops: 2 (d + r_v) per causal (query, key) pair, the key rebuild 2 d r_k and the "
+                "output projection 2 d r_v per (token, head)"}
+    del q, o, pool, cache, ws
 
     # comparator: plain loop-t K/V of the headline batch, d = 128
     w = W.WORKLOADS["ouro14_rho4"]

@@ -13,6 +13,7 @@
  *                        caching": pass 1 and pass 2 of the cached reconstruction decoder)
  *   lla_decode_attn_rope the same with rotary positions applied after reconstruction (Sec. 3,
  *                        "RoPE and reconstruction"), keys rebuilt on the tensor cores
+ *   lla_prefill_attn_rope  causal prefill with rotary positions after reconstruction
  *   lla_prefill_attn     causal pass-2 prefill attention over the latents of a prompt
  *   lla_dense_*          the uncompressed loop-t KV decode in the same kernel style (the
  *                        "teacher" column of Table absorbed_latency, App. J), for comparison
@@ -207,6 +208,31 @@ lla_status lla_decode_attn_rope(const lla_geometry *g, const lla_codec *codec,
                                 int32_t loop, const void *q, const void *cur_k, const void *cur_v,
                                 lla_dtype io_dtype, void *out, void *workspace,
                                 size_t workspace_bytes, void *stream);
+
+/* Workspace bytes lla_prefill_attn_rope needs for B prompts of at most max_len tokens. */
+lla_status lla_prefill_rope_workspace_size(const lla_geometry *g, int32_t B, int32_t max_len,
+                                           size_t *bytes);
+
+/*
+ * lla_prefill_attn with rotary positions applied after reconstruction (Sec. 3 "RoPE and
+ * reconstruction"; App. A two-pass prefill, whose pass 2 attends over the rebuilt, rotated
+ * keys).  Prompt token i (query and key) sits at position i of its prompt.  Two launches on
+ * `stream`: every key of the prompts is rebuilt by Eq. decode and rotated, and every query
+ * rotated and scaled, into the workspace (bf16); then the causal tensor-core attention over them,
+ * with values in latent space as in lla_prefill_attn.
+ *   rope        host pointer to the rotation (read during the call)
+ *   q           pre-RoPE, 16-byte aligned
+ *   workspace   device, >= lla_prefill_rope_workspace_size bytes; overwritten (no zero fill
+ *               needed); calls that share it must be ordered
+ * Other arguments and the error behaviour are those of lla_prefill_attn; a prompt whose tokens
+ * reach past row B * max_len of q sets LLA_DEVERR_CONTEXT.  Storage LLA_BF16, d = 128 and
+ * (r_k, r_v) one of (96, 160), (192, 320), (128, 128); LLA_ERR_UNSUPPORTED otherwise.
+ */
+lla_status lla_prefill_attn_rope(const lla_geometry *g, const lla_codec *codec,
+                                 const lla_cache *cache, const lla_rope *rope,
+                                 const int32_t *cu_seqlens, int32_t B, int32_t max_len,
+                                 int32_t loop, const void *q, lla_dtype io_dtype, void *out,
+                                 void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * lla_decode_attn for callers that cannot allocate device memory (for example a plug-in inside a

@@ -322,6 +322,53 @@ lla_status lla_prefill_attn(const lla_geometry *g, const lla_codec *codec, const
     return launch_prefill(a, static_cast<cudaStream_t>(stream));
 }
 
+lla_status lla_prefill_rope_workspace_size(const lla_geometry *g, int32_t B, int32_t max_len,
+                                           size_t *bytes) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!bytes || B < 0 || B > LLA_MAX_BATCH || max_len < 0) return LLA_ERR_INVALID_ARG;
+    if (!prefill_rope_supported(elem_size(g->storage), g->d, g->r_k, g->r_v)) return LLA_ERR_UNSUPPORTED;
+    *bytes = prefill_rope_workspace_bytes(B, max_len, g->H);
+    return LLA_OK;
+}
+
+lla_status lla_prefill_attn_rope(const lla_geometry *g, const lla_codec *codec,
+                                 const lla_cache *cache, const lla_rope *rope,
+                                 const int32_t *cu_seqlens, int32_t B, int32_t max_len,
+                                 int32_t loop, const void *q, lla_dtype io_dtype, void *out,
+                                 void *workspace, size_t workspace_bytes, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if ((st = check_cache(cache, true)) != LLA_OK) return st;
+    if (!rope || !(rope->base > 1.0) || !(rope->base < 1e300)) return LLA_ERR_INVALID_ARG;
+    if (rope->pairing != LLA_ROPE_HALF && rope->pairing != LLA_ROPE_ADJACENT) return LLA_ERR_INVALID_ARG;
+    if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;
+    if (!aligned(codec->w_up_k, 16) || !aligned(codec->w_up_v, 16)) return LLA_ERR_INVALID_ARG;
+    if ((q && !aligned(q, 16)) || (out && !aligned(out, 16))) return LLA_ERR_INVALID_ARG;
+    if (loop < 0 || loop >= g->T || B < 0 || B > LLA_MAX_BATCH || !valid_dtype(io_dtype))
+        return LLA_ERR_INVALID_ARG;
+    if (max_len < 0 || static_cast<int64_t>(max_len) >
+                           static_cast<int64_t>(cache->max_blocks_per_seq) * LLA_BLOCK_TOKENS)
+        return LLA_ERR_INVALID_ARG;
+    if (B > 0 && (!cu_seqlens || !q || !out)) return LLA_ERR_INVALID_ARG;
+    if (!prefill_rope_supported(elem_size(g->storage), g->d, g->r_k, g->r_v)) return LLA_ERR_UNSUPPORTED;
+    if (B == 0 || max_len == 0) return LLA_OK;
+    if (!workspace || !aligned(workspace, 16)) return LLA_ERR_INVALID_ARG;
+    PrefillArgs a = {};
+    a.T = g->T; a.H = g->H; a.d = g->d; a.r_k = g->r_k; a.r_v = g->r_v; a.loop = loop;
+    a.storage_bf16 = g->storage == LLA_BF16;
+    a.io_bf16 = io_dtype == LLA_BF16;
+    a.scale = g->scale;
+    a.w_up_k = codec->w_up_k; a.w_up_v = codec->w_up_v;
+    a.mu_k = codec->mu_k; a.mu_v = codec->mu_v;
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.block_table = cache->block_table; a.max_blocks = cache->max_blocks_per_seq;
+    a.cu_seqlens = cu_seqlens; a.B = B; a.max_len = max_len;
+    a.q = q; a.out = out;
+    return launch_prefill_rope(a, rope->base, rope->pairing == LLA_ROPE_ADJACENT ? 1 : 0, workspace,
+                               workspace_bytes, static_cast<cudaStream_t>(stream));
+}
+
 lla_status lla_get_device_error(void *stream, uint32_t *word) {
     if (!word) return LLA_ERR_INVALID_ARG;
     lla_status st = LLA_OK;

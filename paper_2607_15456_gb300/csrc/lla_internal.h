@@ -84,6 +84,12 @@ lla_status launch_encode_layers(const EncodeArgs *a, int L, cudaStream_t stream)
 bool encode_tc_supported(const EncodeArgs &a);
 lla_status launch_encode_tc(const EncodeArgs &a, cudaStream_t stream);
 lla_status launch_prefill(const PrefillArgs &a, cudaStream_t stream);
+// Prefill with rotary positions after reconstruction: keys rebuilt and rotated into the
+// workspace, then the tensor-core attention over them (bf16 storage, d = 128, the prefill ranks).
+size_t prefill_rope_workspace_bytes(int B, int max_len, int H);
+bool prefill_rope_supported(int es, int d, int r_k, int r_v);
+lla_status launch_prefill_rope(const PrefillArgs &a, double base, int pairing, void *workspace,
+                               size_t workspace_bytes, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached), 0 on failure
 

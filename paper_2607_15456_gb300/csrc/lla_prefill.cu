@@ -67,21 +67,29 @@ struct PParams {
     const void *q;
     void *out;
     unsigned *err;
+    // rotary positions after reconstruction: keys rebuilt and rotated, [B][kpps][H] pages of
+    // 64 keys x d in the K-plane layout, and queries rotated and scaled, [Ntok][H][d], bf16
+    const char *krot;
+    const void *qrot;
+    int kpps;
+    int64_t qrows;  // rows of the rotated-query buffer (B * max_len)
 };
 
 // Shared-memory plan of the tensor-core kernel for ranks (RK, RV); d = 128.  Offsets are
-// multiples of 1024 bytes from a 1024-byte aligned base (128-byte swizzle atoms).
-template <int RK, int RV>
+// multiples of 1024 bytes from a 1024-byte aligned base (128-byte swizzle atoms).  With ROPE
+// the scores are formed from rebuilt, rotated keys of width d instead of latents of width RK.
+template <int RK, int RV, bool ROPE = false>
 struct PF {
     static constexpr int D = 128;
+    static constexpr int RS = ROPE ? D : RK;         // contraction width of the scores
     static constexpr int NKC = RK / 8;               // 16-byte chunks of a K row
     static constexpr int NVC = RV / 8;               // 16-byte chunks of a V row
     static constexpr int VATOMS = (RV + 63) / 64;    // 64-column atoms of a V page (TMA boxes)
     static constexpr int N0 = RV > 256 ? 256 : RV;   // PV MMA split on atom boundaries
     static constexpr int N1 = RV - N0;
-    static constexpr int KPAGE = kPT * RK * 2;
+    static constexpr int KPAGE = kPT * RS * 2;
     static constexpr int VPAGE = VATOMS * kPT * 128;
-    static constexpr int QT = kBM * RK * 2;          // q~ operand
+    static constexpr int QT = kBM * RS * 2;          // q~ (or rotated q) operand
     static constexpr int PB = kBM * kPT * 2;         // P operand (one of two)
     static constexpr int QA = kBM * D * 2;           // q operand (prologue)
     static constexpr int WK = D * RK * 2;            // W_up,t^K operand (prologue)
@@ -124,10 +132,10 @@ enum {
     kBAbort = 34  // slot used as the CTA's abort flag
 };
 
-template <int RK, int RV>
+template <int RK, int RV, bool ROPE>
 __global__ void __launch_bounds__(kPThreads, 1)
     prefill_tc_kernel(const __grid_constant__ CUtensorMap tv, const PParams p) {
-    using F = PF<RK, RV>;
+    using F = PF<RK, RV, ROPE>;
     constexpr int D = F::D;
     extern __shared__ __align__(1024) char sm_raw[];
     char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -144,7 +152,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     pdl_wait();
     const int q0 = p.cu_seqlens[b];
     const int L = p.cu_seqlens[b + 1] - q0;
-    if (L > p.max_len || L < 0) {
+    if (L > p.max_len || L < 0 || (ROPE && static_cast<int64_t>(q0) + L > p.qrows)) {
         if (tid == 0 && qt == nqt - 1) atomicOr(p.err, LLA_DEVERR_CONTEXT);
         return;
     }
@@ -191,15 +199,17 @@ __global__ void __launch_bounds__(kPThreads, 1)
 
     if (warp == 0) {
         // ------------------------------------------------------------------------- producer
-        const char *wk = static_cast<const char *>(p.w_up_k) + wofs * RK * 2;
-        // W_up,t^K [d][r_k] as an MN-major operand: (row e, column chunk g) at g*(d*16) + e*16
-        for (int i = lane; i < D * F::NKC; i += 32) {
-            const int e = i / F::NKC, g = i - e * F::NKC;
-            cp_async16(sm + F::oWK + g * (D * 16) + e * 16, wk + (static_cast<int64_t>(e) * RK + g * 8) * 2);
+        if constexpr (!ROPE) {
+            const char *wk = static_cast<const char *>(p.w_up_k) + wofs * RK * 2;
+            // W_up,t^K [d][r_k] as an MN-major operand: (row e, column chunk g) at g*(d*16) + e*16
+            for (int i = lane; i < D * F::NKC; i += 32) {
+                const int e = i / F::NKC, g = i - e * F::NKC;
+                cp_async16(sm + F::oWK + g * (D * 16) + e * 16, wk + (static_cast<int64_t>(e) * RK + g * 8) * 2);
+            }
+            cp_async_commit();
+            cp_async_wait_all();
+            fence_proxy_async_smem();
         }
-        cp_async_commit();
-        cp_async_wait_all();
-        fence_proxy_async_smem();
         mbar_arrive(&bar[kBSetup]);
         if (lane == 0) {  // K-planes: one bulk copy per page
             const uint64_t pol = policy_evict_first();
@@ -212,10 +222,12 @@ __global__ void __launch_bounds__(kPThreads, 1)
                     blk = 0;
                 }
                 const int64_t hp = static_cast<int64_t>(blk) * p.H + h;  // head page index
+                // the latent K-plane of the page, or its rebuilt and rotated keys
+                const char *src = ROPE ? p.krot + ((static_cast<int64_t>(b) * p.kpps + j) * p.H + h) * F::KPAGE
+                                       : p.pool + hp * p.head_page_bytes;
                 mbar_wait(&bar[kBKempty + s], ph ^ 1u, abort_flag, p.err);
                 mbar_arrive_expect_tx(&bar[kBKfull + s], F::KPAGE);
-                bulk_g2s(sm + F::oK + s * F::KPAGE, p.pool + hp * p.head_page_bytes, F::KPAGE,
-                         &bar[kBKfull + s], pol);
+                bulk_g2s(sm + F::oK + s * F::KPAGE, src, F::KPAGE, &bar[kBKfull + s], pol);
             }
         }
         __syncwarp();
@@ -257,13 +269,17 @@ __global__ void __launch_bounds__(kPThreads, 1)
             const uint32_t base = smem_addr(sm);
             mbar_wait(&bar[kBSetup], 0, abort_flag, p.err);
             tc_fence_after();
-            constexpr uint32_t idq = umma_idesc_bf16(128, RK, 0, 1);
-            const uint64_t dqa = umma_desc(base + F::oQA, 2048, 128);
-            const uint64_t dwk = umma_desc(base + F::oWK, 128, 2048);
+            if constexpr (ROPE) {
+                mbar_arrive(&bar[kBQt]);  // the rotated queries come ready from global memory
+            } else {
+                constexpr uint32_t idq = umma_idesc_bf16(128, RK, 0, 1);
+                const uint64_t dqa = umma_desc(base + F::oQA, 2048, 128);
+                const uint64_t dwk = umma_desc(base + F::oWK, 128, 2048);
 #pragma unroll
-            for (int ks = 0; ks < D / 16; ++ks)
-                umma_bf16(tmem + 0, dqa + ks * (4096 >> 4), dwk + ks * (256 >> 4), idq, ks > 0);
-            umma_commit(&bar[kBQt]);
+                for (int ks = 0; ks < D / 16; ++ks)
+                    umma_bf16(tmem + 0, dqa + ks * (4096 >> 4), dwk + ks * (256 >> 4), idq, ks > 0);
+                umma_commit(&bar[kBQt]);
+            }
             mbar_wait(&bar[kBQs], 0, abort_flag, p.err);
             tc_fence_after();
             constexpr uint32_t ids = umma_idesc_bf16(128, kPT, 0, 0);
@@ -279,7 +295,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
                 const uint64_t dk = dk0 + static_cast<uint64_t>(sk * (F::KPAGE >> 4));
                 const uint32_t ds = tmem + F::TM_S + s * kPT;
 #pragma unroll
-                for (int ks = 0; ks < RK / 16; ++ks)
+                for (int ks = 0; ks < F::RS / 16; ++ks)
                     umma_bf16(ds, dq + ks * (4096 >> 4), dk + ks * (2048 >> 4), ids, ks > 0);
                 umma_commit(&bar[kBSfull + s]);
                 umma_commit(&bar[kBKempty + sk]);
@@ -345,6 +361,19 @@ __global__ void __launch_bounds__(kPThreads, 1)
         const int qi = i0 + row;
         const bool valid_row = qi < L;
         const int64_t qrow = (static_cast<int64_t>(q0) + qi) * p.H + h;
+        if constexpr (ROPE) {
+            // the rotated, scaled q row (this half's 64 elements) -> the score operand directly
+            char *qt_ = sm + F::oQT + row * 16;
+            const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const char *>(p.qrot) + qrow * D * 2);
+            const int c0 = half * (D / 16);
+#pragma unroll
+            for (int c = c0; c < c0 + D / 16; ++c)
+                *reinterpret_cast<uint4 *>(qt_ + c * 2048) = valid_row ? src[c] : make_uint4(0, 0, 0, 0);
+            fence_proxy_async_smem();
+            mbar_arrive(&bar[kBSetup]);
+            mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
+            mbar_arrive(&bar[kBQs]);
+        } else {
         // q row (this half's 64 elements) -> bf16 K-major operand: chunk c at c*2048 + row*16
         {
             char *qa = sm + F::oQA + row * 16;
@@ -389,6 +418,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
         fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(&bar[kBQs]);
+        }
 
         const int lim = min(qi, L - 1);  // keys 0..lim are visible to this row
         const int kofs = half * 32;      // this thread's keys within a page
@@ -668,6 +698,212 @@ __global__ void __launch_bounds__(kGThreads) prefill_generic_kernel(const GParam
     pdl_trigger();
 }
 
+// ------------------------------------------------- rotary positions: rebuild and rotate keys
+//
+// Sec. 3 "RoPE and reconstruction": keys are rebuilt by Eq. decode and rotated at their
+// positions before attention.  One CTA per (sequence, page of 64 prompt tokens) loops over the
+// heads: Khat (64 tokens x d) = C_k W_up,t^K^T + mu^K_t on tcgen05 (M = 64 tokens, N = d,
+// K = r_k, plus one K step for mu^K_t), then each token's pairs are rotated in registers and
+// written as a bf16 page in the K-plane layout (granule g of 8 dimensions at g*1024 + token*16),
+// and the page's queries are rotated and scaled by scale * log2 e into a bf16 copy of q.
+
+struct RParams {
+    int T, H, loop, io_bf16, kpps, pairing;
+    float scale_log2;
+    const void *w_up_k;
+    const float *mu_k;
+    const char *pool;
+    int64_t num_blocks;
+    int head_page_bytes;
+    const int32_t *block_table;
+    int max_blocks;
+    const int32_t *cu_seqlens;
+    int max_len;
+    const void *q;
+    char *krot;
+    void *qrot;
+    int64_t qrows;  // rows of the rotated-query buffer: B * max_len
+    unsigned *err;
+    unsigned long long phi[64];  // theta_j / (2 pi) * 2^64
+};
+
+template <int RK>
+struct RB {
+    static constexpr int D = 128;
+    static constexpr int NG = RK / 8;                 // 16-byte granules of a latent row
+    static constexpr int oTab = 0;                    // [64 tokens][65] (cos, sin) per pair
+    static constexpr int TAB = 64 * 65 * 8;
+    static constexpr int oB = (TAB + 1023) & ~1023;   // (mu_hi, mu_lo) granule, then W_up,t^K
+    static constexpr int oW = oB + D * 16;
+    static constexpr int oA = oW + NG * D * 16;       // the page's K-plane, then ones and zeros
+    static constexpr int oOnes = oA + NG * 64 * 16;
+    static constexpr int oBar = oOnes + 2 * 64 * 16;
+    static constexpr int SMEM = oBar + 16 + 1024;     // + alignment slack
+    static constexpr uint32_t IDESC = umma_idesc_bf16(64, D, 0, 0);
+    static_assert(RK % 16 == 0, "K steps");
+};
+
+template <int RK>
+__global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant__ RParams p) {
+    using Z = RB<RK>;
+    constexpr int D = Z::D;
+    extern __shared__ __align__(1024) char rb_raw[];
+    char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(rb_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    float2 *tab = reinterpret_cast<float2 *>(sm + Z::oTab);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + Z::oBar);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + 1);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int pg = blockIdx.x, b = blockIdx.y;
+    pdl_wait();
+    const int q0 = p.cu_seqlens[b];
+    const int L = p.cu_seqlens[b + 1] - q0;
+    if (L > p.max_len || L < 0 || static_cast<int64_t>(q0) + L > p.qrows) {
+        if (tid == 0 && pg == 0) atomicOr(p.err, LLA_DEVERR_CONTEXT);
+        return;
+    }
+    if (pg * kPT >= L) return;  // uniform, before any barrier
+    const int nvalid = min(kPT, L - pg * kPT);
+    int32_t blk = p.block_table[static_cast<int64_t>(b) * p.max_blocks + pg];
+    if (blk < 0 || blk >= p.num_blocks) {
+        if (tid == 0) atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+        blk = 0;
+    }
+    if (tid == 0) {
+        mbar_init(bar, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) tmem_alloc(tslot, 128);
+    // rotation of each token of the page at each pair's frequency, from exact turns
+    for (int i = tid; i < 64 * 64; i += 128) {
+        const int r = i >> 6, j = i & 63;
+        const unsigned long long turns = static_cast<unsigned long long>(pg * kPT + r) * p.phi[j];
+        const float tf = __uint2float_rn(static_cast<uint32_t>(turns >> 32)) * 2.3283064365386963e-10f;
+        float sa, ca;
+        sincospif(2.f * tf, &sa, &ca);
+        tab[r * 65 + j] = make_float2(ca, sa);
+    }
+    // A of the mu step: a (1, 1) pair per token, then a zero granule
+    for (int i = tid; i < 128; i += 128)
+        reinterpret_cast<uint4 *>(sm + Z::oOnes)[i] = i < 64 ? make_uint4(0x3f803f80u, 0u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+    const uint32_t base = smem_addr(sm);
+    // epilogue geometry (16x256b fragments of the M = 64 accumulator): warp w holds tokens
+    // 16w + lane/4 and 16w + lane/4 + 8; columns 8k + 2c and 8k + 2c + 1, c = lane % 4
+    const int c = lane & 3;
+    const int tok0 = 16 * warp + (lane >> 2);
+    const uint32_t tq = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+    for (int h = 0; h < p.H; ++h) {
+        const int64_t hl = (static_cast<int64_t>(h) * p.T + p.loop) * D;
+        // B: W_up,t^K of head h (row e = dimension, K-major), the (mu_hi, mu_lo) granule before it
+        const char *W = static_cast<const char *>(p.w_up_k) + hl * RK * 2;
+        for (int i = tid; i < D * Z::NG; i += 128) {
+            const int e = i / Z::NG, g = i - e * Z::NG;
+            cp_async16(sm + Z::oW + g * (D * 16) + e * 16, W + (static_cast<int64_t>(e) * RK + g * 8) * 2);
+        }
+        // A: the page's K-plane of head h, as stored
+        const char *K = p.pool + (static_cast<int64_t>(blk) * p.H + h) * p.head_page_bytes;
+        for (int i = tid; i < Z::NG * 64; i += 128) cp_async16(sm + Z::oA + i * 16, K + i * 16);
+        cp_async_commit();
+        {
+            const float mu = p.mu_k ? p.mu_k[hl + tid] : 0.f;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(mu);
+            const __nv_bfloat16 lo = __float2bfloat16_rn(mu - __bfloat162float(hi));
+            *reinterpret_cast<uint4 *>(sm + Z::oB + tid * 16) =
+                make_uint4(static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
+                               (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16),
+                           0u, 0u, 0u);
+        }
+        cp_async_wait_all();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            tc_fence_after();
+#pragma unroll
+            for (int st = 0; st < RK / 16; ++st)
+                umma_bf16(tmem, umma_desc(base + Z::oA + st * 2048, 1024, 128),
+                          umma_desc(base + Z::oW + st * 4096, 2048, 128), Z::IDESC, st > 0);
+            // mu: the ones pair of every token against (mu_hi, mu_lo) of every dimension; the
+            // second granules are zeros (A) and W_up,t^K (B, finite)
+            umma_bf16(tmem, umma_desc(base + Z::oOnes, 1024, 128), umma_desc(base + Z::oB, 2048, 128),
+                      Z::IDESC, true);
+            umma_commit(bar);
+        }
+        {
+            volatile int never = 0;
+            mbar_wait(bar, h & 1, &never, p.err);
+        }
+        tc_fence_after();
+        uint32_t r0[32], r1[32];  // dimensions 0..63 (k = 0..7) and 64..127 (k = 8..15)
+        tmem_ld16x256_x8_nowait(tq, r0);
+        tmem_ld16x256_x8_nowait(tq + 64, r1);
+        tmem_wait_ld(r0);
+        tmem_wait_ld(r1);
+        // rotate each token's pairs and write the page: dims (8k + 2c, +1) of token t at
+        // granule k, byte 4c
+        char *kout = p.krot + ((static_cast<int64_t>(b) * p.kpps + pg) * p.H + h) * (kPT * D * 2);
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int t = tok0 + 8 * u;
+            const float2 *tr = tab + t * 65;
+            const bool ok = t < nvalid;
+            float y[32];  // y[2k + e]: dimension 8k + 2c + e
+            if (p.pairing == 0) {  // pairs (j, j + 64): k and k + 8
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const float xa = __uint_as_float(r0[4 * k + 2 * u + e]);
+                        const float xb = __uint_as_float(r1[4 * k + 2 * u + e]);
+                        const float2 cs = tr[8 * k + 2 * c + e];
+                        y[2 * k + e] = xa * cs.x - xb * cs.y;
+                        y[2 * (k + 8) + e] = xa * cs.y + xb * cs.x;
+                    }
+            } else {  // pairs (2j, 2j + 1), j = 4k + c
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    const uint32_t *rr = k < 8 ? r0 : r1;
+                    const int kk = k & 7;
+                    const float xa = __uint_as_float(rr[4 * kk + 2 * u]);
+                    const float xb = __uint_as_float(rr[4 * kk + 2 * u + 1]);
+                    const float2 cs = tr[4 * k + c];
+                    y[2 * k] = xa * cs.x - xb * cs.y;
+                    y[2 * k + 1] = xa * cs.y + xb * cs.x;
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < 16; ++k)
+                *reinterpret_cast<uint32_t *>(kout + k * 1024 + t * 16 + c * 4) =
+                    ok ? pack_bf16x2(y[2 * k], y[2 * k + 1]) : 0u;
+        }
+        // the page's queries of head h: rotated at their positions, scaled into the exp2 domain
+        {
+            const int r = tid >> 1, hf = tid & 1;
+            if (r < nvalid) {
+                const int64_t qrow = (static_cast<int64_t>(q0) + pg * kPT + r) * p.H + h;
+                const float2 *tr = tab + r * 65;
+                __nv_bfloat16 *qo = static_cast<__nv_bfloat16 *>(p.qrot) + qrow * D;
+                for (int jj = 32 * hf; jj < 32 * hf + 32; ++jj) {
+                    const int ia = p.pairing ? 2 * jj : jj, ib = p.pairing ? 2 * jj + 1 : jj + 64;
+                    const float xa = load_elem(p.q, qrow * D + ia, p.io_bf16);
+                    const float xb = load_elem(p.q, qrow * D + ib, p.io_bf16);
+                    const float2 cs = tr[jj];
+                    qo[ia] = __float2bfloat16_rn((xa * cs.x - xb * cs.y) * p.scale_log2);
+                    qo[ib] = __float2bfloat16_rn((xa * cs.y + xb * cs.x) * p.scale_log2);
+                }
+            }
+        }
+        tc_fence_before();
+        __syncthreads();  // the operands and the accumulator may take the next head
+        tc_fence_after();
+    }
+    pdl_trigger();
+    if (warp == 0) tmem_dealloc(tmem, 128);
+}
+
 template <typename K, typename P>
 lla_status launch_pf(K kern, dim3 grid, int threads, int smem, cudaStream_t stream, const P &prm) {
     cudaLaunchConfig_t cfg = {};
@@ -684,14 +920,14 @@ lla_status launch_pf(K kern, dim3 grid, int threads, int smem, cudaStream_t stre
     return LLA_OK;
 }
 
-template <int RK, int RV>
+template <int RK, int RV, bool ROPE = false>
 lla_status launch_tc(const PParams &prm, int nqt, int B, int H, cudaStream_t stream) {
     static bool configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(prefill_tc_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 PF<RK, RV>::SMEM) != cudaSuccess)
+        if (cudaFuncSetAttribute(prefill_tc_kernel<RK, RV, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 PF<RK, RV, ROPE>::SMEM) != cudaSuccess)
             return LLA_ERR_CUDA;
         configured[dev] = true;
     }
@@ -705,14 +941,14 @@ lla_status launch_tc(const PParams &prm, int nqt, int B, int H, cudaStream_t str
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(nqt, B, H);
     cfg.blockDim = dim3(kPThreads);
-    cfg.dynamicSmemBytes = PF<RK, RV>::SMEM;
+    cfg.dynamicSmemBytes = PF<RK, RV, ROPE>::SMEM;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, prefill_tc_kernel<RK, RV>, tv, prm) != cudaSuccess) return LLA_ERR_CUDA;
+    if (cudaLaunchKernelEx(&cfg, prefill_tc_kernel<RK, RV, ROPE>, tv, prm) != cudaSuccess) return LLA_ERR_CUDA;
     return LLA_OK;
 }
 
@@ -761,6 +997,87 @@ lla_status launch_prefill(const PrefillArgs &a, cudaStream_t stream) {
     g.q = a.q; g.out = a.out; g.err = err;
     const int smem = (a.d + a.r_k + a.r_v + kGKeys + 32) * 4;
     return launch_pf(prefill_generic_kernel, dim3(a.max_len, a.B, a.H), kGThreads, smem, stream, g);
+}
+
+
+size_t prefill_rope_workspace_bytes(int B, int max_len, int H) {
+    const size_t kpps = (static_cast<size_t>(max_len) + kPT - 1) / kPT;
+    const size_t krot = static_cast<size_t>(B) * kpps * H * kPT * 128 * 2;
+    const size_t qrot = static_cast<size_t>(B) * max_len * H * 128 * 2;
+    return krot + qrot;
+}
+
+bool prefill_rope_supported(int es, int d, int r_k, int r_v) {
+    return es == 2 && d == 128 &&
+           ((r_k == 96 && r_v == 160) || (r_k == 192 && r_v == 320) || (r_k == 128 && r_v == 128));
+}
+
+namespace {
+template <int RK>
+lla_status launch_rebuild(const RParams &rp, int kpps, int B, cudaStream_t stream) {
+    static bool configured[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
+    if (dev < 64 && !configured[dev]) {
+        if (cudaFuncSetAttribute(rope_rebuild_kernel<RK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 RB<RK>::SMEM) != cudaSuccess)
+            return LLA_ERR_CUDA;
+        configured[dev] = true;
+    }
+    return launch_pf(rope_rebuild_kernel<RK>, dim3(kpps, B), 128, RB<RK>::SMEM, stream, rp);
+}
+}  // namespace
+
+lla_status launch_prefill_rope(const PrefillArgs &a, double base, int pairing, void *workspace,
+                               size_t workspace_bytes, cudaStream_t stream) {
+    const int es = a.storage_bf16 ? 2 : 4;
+    if (!prefill_rope_supported(es, a.d, a.r_k, a.r_v)) return LLA_ERR_UNSUPPORTED;
+    if (a.B > 65535 || a.H > 65535 || a.num_blocks * a.H >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;
+    if (workspace_bytes < prefill_rope_workspace_bytes(a.B, a.max_len, a.H)) return LLA_ERR_WORKSPACE;
+    lla_status st = LLA_OK;
+    unsigned *err = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    const int hpb = static_cast<int>(head_page_bytes(a.r_k, a.r_v, es));
+    const int kpps = (a.max_len + kPT - 1) / kPT;
+    char *krot = static_cast<char *>(workspace);
+    void *qrot = krot + static_cast<size_t>(a.B) * kpps * a.H * kPT * 128 * 2;
+
+    RParams r = {};
+    r.T = a.T; r.H = a.H; r.loop = a.loop; r.io_bf16 = a.io_bf16; r.kpps = kpps; r.pairing = pairing;
+    r.scale_log2 = a.scale * kLog2e;
+    r.w_up_k = a.w_up_k; r.mu_k = a.mu_k;
+    r.pool = static_cast<const char *>(a.pool); r.num_blocks = a.num_blocks;
+    r.head_page_bytes = hpb;
+    r.block_table = a.block_table; r.max_blocks = a.max_blocks;
+    r.cu_seqlens = a.cu_seqlens; r.max_len = a.max_len;
+    r.q = a.q; r.krot = krot; r.qrot = qrot; r.err = err;
+    r.qrows = static_cast<int64_t>(a.B) * a.max_len;
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int j = 0; j < 64; ++j)
+        r.phi[j] = static_cast<unsigned long long>(ldexp(pow(base, -2.0 * j / a.d) / two_pi, 64));
+    lla_status rs = LLA_ERR_UNSUPPORTED;
+    if (a.r_k == 96) rs = launch_rebuild<96>(r, kpps, a.B, stream);
+    else if (a.r_k == 192) rs = launch_rebuild<192>(r, kpps, a.B, stream);
+    else if (a.r_k == 128) rs = launch_rebuild<128>(r, kpps, a.B, stream);
+    if (rs != LLA_OK) return rs;
+
+    PParams p = {};
+    p.T = a.T; p.H = a.H; p.loop = a.loop; p.io_bf16 = a.io_bf16;
+    p.scale_log2 = a.scale * kLog2e;
+    p.w_up_k = a.w_up_k; p.w_up_v = a.w_up_v; p.mu_v = a.mu_v;
+    p.pool = static_cast<const char *>(a.pool);
+    p.num_blocks = a.num_blocks;
+    p.head_page_bytes = hpb;
+    p.block_bytes = static_cast<int64_t>(hpb) * a.H;
+    p.block_table = a.block_table; p.max_blocks = a.max_blocks;
+    p.cu_seqlens = a.cu_seqlens; p.B = a.B; p.max_len = a.max_len;
+    p.q = a.q; p.out = a.out; p.err = err;
+    p.krot = krot; p.qrot = qrot; p.kpps = kpps;
+    p.qrows = static_cast<int64_t>(a.B) * a.max_len;
+    const int nqt = (a.max_len + kBM - 1) / kBM;
+    if (a.r_k == 96) return launch_tc<96, 160, true>(p, nqt, a.B, a.H, stream);
+    if (a.r_k == 192) return launch_tc<192, 320, true>(p, nqt, a.B, a.H, stream);
+    return launch_tc<128, 128, true>(p, nqt, a.B, a.H, stream);
 }
 
 }  // namespace lla

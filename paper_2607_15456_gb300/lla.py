@@ -82,6 +82,8 @@ def library() -> ctypes.CDLL:
             "lla_decode_attn_rope": (I32, [P, P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ,
                                            P]),
             "lla_prefill_attn": (I32, [P, P, P, P, I32, I32, I32, P, I32, P, P]),
+            "lla_prefill_rope_workspace_size": (I32, [P, I32, I32, P]),
+            "lla_prefill_attn_rope": (I32, [P, P, P, P, P, I32, I32, I32, P, I32, P, P, SZ, P]),
             "lla_dense_store": (I32, [P, P, P, P, I32, P, I32, P]),
             "lla_dense_decode_attn": (I32, [P, P, P, I32, I32, P, P, P, I32, P, P, SZ, P]),
             "lla_get_device_error": (I32, [P, P]),
@@ -284,6 +286,28 @@ def lla_prefill_attn(geom: Geometry, codec: Codec, cache: Cache, cu_seqlens: tor
     _check("lla_prefill_attn", library().lla_prefill_attn(
         ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(cu_seqlens), B, max_len, loop,
         _ptr(q), _dtype_code(q), _ptr(out), _stream(stream)))
+
+
+def lla_prefill_rope_workspace_size(geom: Geometry, B: int, max_len: int) -> int:
+    g = geom.c()
+    out = ctypes.c_size_t()
+    _check("lla_prefill_rope_workspace_size",
+           library().lla_prefill_rope_workspace_size(ctypes.byref(g), B, max_len, ctypes.byref(out)))
+    return out.value
+
+
+def lla_prefill_attn_rope(geom: Geometry, codec: Codec, cache: Cache, rope_base: float,
+                          rope_pairing: int, cu_seqlens: torch.Tensor, max_len: int, loop: int,
+                          q: torch.Tensor, out: torch.Tensor, workspace: torch.Tensor,
+                          stream=None) -> None:
+    """lla_prefill_attn with RoPE after reconstruction; q pre-RoPE [Ntok][H][d]."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    rp = lla_rope(float(rope_base), int(rope_pairing))
+    B = cu_seqlens.shape[0] - 1
+    _check("lla_prefill_attn_rope", library().lla_prefill_attn_rope(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), ctypes.byref(rp), _ptr(cu_seqlens), B,
+        max_len, loop, _ptr(q), _dtype_code(q), _ptr(out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def lla_dense_store(geom: Geometry, cache: Cache, k: torch.Tensor, v: torch.Tensor,

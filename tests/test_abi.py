@@ -227,3 +227,30 @@ def test_decode_rope_argument_checks(lib):
     assert _decode_rope(lib, B=0, lens=None, q=None, out=None, ws=None) == OK
     assert _decode_rope(lib, rope=lib.lla_rope(500000.0, lib.LLA_ROPE_ADJACENT), B=0, lens=None,
                         q=None, out=None, ws=None) == OK
+
+
+def test_prefill_rope_argument_checks(lib):
+    so = lib.library()
+    g, codec, cache = _g(lib), _codec(lib), _cache(lib)
+    rope = lib.lla_rope(10000.0, lib.LLA_ROPE_HALF)
+    size = ctypes.c_size_t()
+    assert so.lla_prefill_rope_workspace_size(ctypes.byref(g), 4, 128, ctypes.byref(size)) == OK
+    assert size.value == 4 * 2 * 16 * 64 * 128 * 2 + 4 * 128 * 16 * 128 * 2
+    g72 = _g(lib, r_k=72, r_v=120)
+    assert so.lla_prefill_rope_workspace_size(ctypes.byref(g72), 4, 128, ctypes.byref(size)) == UNSUPPORTED
+
+    def call(rope_=rope, g_=g, B=4, max_len=128, loop=0, q=FAKE, io=0, out=FAKE, ws=FAKE,
+             cu=FAKE):
+        return so.lla_prefill_attn_rope(ctypes.byref(g_), ctypes.byref(codec), ctypes.byref(cache),
+                                        None if rope_ is None else ctypes.byref(rope_), cu, B,
+                                        max_len, loop, q, io, out, ws, 1 << 30, None)
+    assert call(rope_=None) == INVALID
+    assert call(rope_=lib.lla_rope(0.5, 0)) == INVALID
+    assert call(rope_=lib.lla_rope(10000.0, 7)) == INVALID
+    assert call(loop=4) == INVALID
+    assert call(q=FAKE + 4) == INVALID
+    assert call(ws=None) == INVALID
+    assert call(max_len=4 * 64 + 1) == INVALID
+    assert call(g_=g72) == UNSUPPORTED
+    assert call(g_=_g(lib, storage="fp32")) == UNSUPPORTED
+    assert call(B=0, q=None, out=None, ws=None, cu=None) == OK

@@ -13,6 +13,8 @@ longest sequence and four more, each at three heads.
     re-encoded by the oracle from the same inputs and compared with the stored latents.
   * prefill: the rho = 2 workload's prompts (4 x 8192 tokens), sampled rows checked as pass-2
     decodes of their causal prefixes.
+  * RoPE decode: the headline batch through lla_decode_attn_rope, sampled rows against the
+    oracle's RoPE decode on the stored latents.
 """
 import numpy as np
 import pytest
@@ -100,6 +102,45 @@ def test_full_size_decode_and_encode_sampled(wname, loop):
             assert_parity(c_k[positions], ek, "bf16", f"{wname} c_k b{b} h{h}")
             assert_parity(c_v[positions], ev, "bf16", f"{wname} c_v b{b} h{h}")
     assert_parity(np.stack(got_rows), np.stack(ref_rows), "bf16", f"{wname} decode loop {loop}")
+
+
+@pytest.mark.parametrize("pairing", [0, 1])
+def test_full_size_rope_decode_sampled(pairing):
+    """The RoPE decode (lla_decode_attn_rope, base 10^4) on the headline batch as bench.py runs
+    it: sampled (sequence, head) rows against oracle.decode_rope fed the stored latents."""
+    ensure_library()
+    import bench
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+
+    dev = torch.device(DEV, 0)
+    db = bench.DecodeBench("ouro14_rho4", dev, layers=1)
+    w = db.w
+    loop = 1
+    lla.lla_clear_device_error()
+    lla.lla_decode_attn_rope(db.geom, db.codecs[0], db.caches[0], 10000.0, pairing, db.ctx,
+                             db.max_ctx, loop, db.q[0, loop], db.cur_k[0, loop],
+                             db.cur_v[0, loop], db.out[0, loop], db.ws)
+    torch.cuda.synchronize()
+    assert lla.lla_get_device_error() == 0
+    out = f64(db.out[0, loop])
+    cod = {k: (None if v is None else f64(v)) for k, v in
+           W.codec_tensors(w.T, w.H, w.d, w.r_k, w.r_v, w.seed, 0, dtype=torch.bfloat16).items()}
+    q, ck, cv = f64(db.q[0, loop]), f64(db.cur_k[0, loop]), f64(db.cur_v[0, loop])
+    bb = lla.lla_cache_block_bytes(db.geom)
+    scale = 1.0 / np.sqrt(w.d)
+    got_rows, ref_rows = [], []
+    for b in _sample_sequences(db.lens):
+        L = db.lens[b]
+        pages, table = _compact_pages(db.pools[0], db.pt.block_table[b], L, bb)
+        for h in (0, w.H // 2, w.H - 1):
+            c_k, c_v = unpack_head(pages, w.H, w.r_k, w.r_v, w.storage, table, L, h)
+            ref = oracle.decode_rope(loop, c_k, c_v, cod["w_up_k"][h], cod["w_up_v"][h], None,
+                                     None, q[b, h], ck[b, h], cv[b, h], scale, 10000.0, pairing)
+            got_rows.append(out[b, h])
+            ref_rows.append(ref)
+    assert_parity(np.stack(got_rows), np.stack(ref_rows), "bf16", "rope decode, full size",
+                  output_rounding=True)
 
 
 def test_full_size_prefill_sampled_rows():
