@@ -707,6 +707,38 @@ __global__ void __launch_bounds__(kGThreads) prefill_generic_kernel(const GParam
 // written as a bf16 page in the K-plane layout (granule g of 8 dimensions at g*1024 + token*16),
 // and the page's queries are rotated and scaled by scale * log2 e into a bf16 copy of q.
 
+// 32 consecutive elements (bf16 or fp32, 16-byte aligned) as floats, loads issued together.
+__device__ __forceinline__ void load32(const void *src, int is_bf16, float (&v)[32]) {
+    if (is_bf16) {
+        uint4 u[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) u[i] = reinterpret_cast<const uint4 *>(src)[i];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 a = bf2_to_f2(u[i].x), b = bf2_to_f2(u[i].y), c = bf2_to_f2(u[i].z), d = bf2_to_f2(u[i].w);
+            v[8 * i] = a.x; v[8 * i + 1] = a.y; v[8 * i + 2] = b.x; v[8 * i + 3] = b.y;
+            v[8 * i + 4] = c.x; v[8 * i + 5] = c.y; v[8 * i + 6] = d.x; v[8 * i + 7] = d.y;
+        }
+    } else {
+        float4 f[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) f[i] = reinterpret_cast<const float4 *>(src)[i];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            v[4 * i] = f[i].x; v[4 * i + 1] = f[i].y; v[4 * i + 2] = f[i].z; v[4 * i + 3] = f[i].w;
+        }
+    }
+}
+
+// 32 floats as bf16 (round to nearest even) with 16-byte stores.
+__device__ __forceinline__ void store32_bf16(void *dst, const float (&v)[32]) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        reinterpret_cast<uint4 *>(dst)[i] =
+            make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                       pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+}
+
 struct RParams {
     int T, H, loop, io_bf16, kpps, pairing;
     float scale_log2;
@@ -795,27 +827,28 @@ __global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant
     const int c = lane & 3;
     const int tok0 = 16 * warp + (lane >> 2);
     const uint32_t tq = tmem + (static_cast<uint32_t>(32 * warp) << 16);
-    for (int h = 0; h < p.H; ++h) {
+    // W_up,t^K of head h (B: row e = dimension, K-major) and the page's K-plane of head h (A, as
+    // stored), by cp.async; the (mu_hi, mu_lo) granule of head h before W
+    auto stage = [&](int h) {
         const int64_t hl = (static_cast<int64_t>(h) * p.T + p.loop) * D;
-        // B: W_up,t^K of head h (row e = dimension, K-major), the (mu_hi, mu_lo) granule before it
         const char *W = static_cast<const char *>(p.w_up_k) + hl * RK * 2;
         for (int i = tid; i < D * Z::NG; i += 128) {
             const int e = i / Z::NG, g = i - e * Z::NG;
             cp_async16(sm + Z::oW + g * (D * 16) + e * 16, W + (static_cast<int64_t>(e) * RK + g * 8) * 2);
         }
-        // A: the page's K-plane of head h, as stored
         const char *K = p.pool + (static_cast<int64_t>(blk) * p.H + h) * p.head_page_bytes;
         for (int i = tid; i < Z::NG * 64; i += 128) cp_async16(sm + Z::oA + i * 16, K + i * 16);
         cp_async_commit();
-        {
-            const float mu = p.mu_k ? p.mu_k[hl + tid] : 0.f;
-            const __nv_bfloat16 hi = __float2bfloat16_rn(mu);
-            const __nv_bfloat16 lo = __float2bfloat16_rn(mu - __bfloat162float(hi));
-            *reinterpret_cast<uint4 *>(sm + Z::oB + tid * 16) =
-                make_uint4(static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
-                               (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16),
-                           0u, 0u, 0u);
-        }
+        const float mu = p.mu_k ? p.mu_k[hl + tid] : 0.f;
+        const __nv_bfloat16 hi = __float2bfloat16_rn(mu);
+        const __nv_bfloat16 lo = __float2bfloat16_rn(mu - __bfloat162float(hi));
+        *reinterpret_cast<uint4 *>(sm + Z::oB + tid * 16) =
+            make_uint4(static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
+                           (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16),
+                       0u, 0u, 0u);
+    };
+    stage(0);
+    for (int h = 0; h < p.H; ++h) {
         cp_async_wait_all();
         fence_proxy_async_smem();
         tc_fence_before();
@@ -837,6 +870,8 @@ __global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant
             mbar_wait(bar, h & 1, &never, p.err);
         }
         tc_fence_after();
+        // the MMA has read its operands: the next head's travel while this one's epilogue runs
+        if (h + 1 < p.H) stage(h + 1);
         uint32_t r0[32], r1[32];  // dimensions 0..63 (k = 0..7) and 64..127 (k = 8..15)
         tmem_ld16x256_x8_nowait(tq, r0);
         tmem_ld16x256_x8_nowait(tq + 64, r1);
@@ -879,20 +914,42 @@ __global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant
                 *reinterpret_cast<uint32_t *>(kout + k * 1024 + t * 16 + c * 4) =
                     ok ? pack_bf16x2(y[2 * k], y[2 * k + 1]) : 0u;
         }
-        // the page's queries of head h: rotated at their positions, scaled into the exp2 domain
+        // the page's queries of head h: rotated at their positions, scaled into the exp2 domain;
+        // thread (r, hf) rotates pairs 32 hf .. 32 hf + 31 of query r
         {
             const int r = tid >> 1, hf = tid & 1;
             if (r < nvalid) {
                 const int64_t qrow = (static_cast<int64_t>(q0) + pg * kPT + r) * p.H + h;
-                const float2 *tr = tab + r * 65;
-                __nv_bfloat16 *qo = static_cast<__nv_bfloat16 *>(p.qrot) + qrow * D;
-                for (int jj = 32 * hf; jj < 32 * hf + 32; ++jj) {
-                    const int ia = p.pairing ? 2 * jj : jj, ib = p.pairing ? 2 * jj + 1 : jj + 64;
-                    const float xa = load_elem(p.q, qrow * D + ia, p.io_bf16);
-                    const float xb = load_elem(p.q, qrow * D + ib, p.io_bf16);
-                    const float2 cs = tr[jj];
-                    qo[ia] = __float2bfloat16_rn((xa * cs.x - xb * cs.y) * p.scale_log2);
-                    qo[ib] = __float2bfloat16_rn((xa * cs.y + xb * cs.x) * p.scale_log2);
+                const float2 *tr = tab + r * 65 + 32 * hf;
+                const int es = p.io_bf16 ? 2 : 4;
+                const char *qs = static_cast<const char *>(p.q) + qrow * D * es;
+                char *qo = static_cast<char *>(p.qrot) + qrow * D * 2;
+                float xa[32], xb[32];
+                if (p.pairing == 0) {  // pairs (j, j + 64): two runs of 32
+                    load32(qs + 32 * hf * es, p.io_bf16, xa);
+                    load32(qs + (64 + 32 * hf) * es, p.io_bf16, xb);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const float2 cs = tr[i];
+                        const float a = xa[i], bb = xb[i];
+                        xa[i] = (a * cs.x - bb * cs.y) * p.scale_log2;
+                        xb[i] = (a * cs.y + bb * cs.x) * p.scale_log2;
+                    }
+                    store32_bf16(qo + 32 * hf * 2, xa);
+                    store32_bf16(qo + (64 + 32 * hf) * 2, xb);
+                } else {  // pairs (2j, 2j + 1): one run of 64
+                    load32(qs + 64 * hf * es, p.io_bf16, xa);
+                    load32(qs + (64 * hf + 32) * es, p.io_bf16, xb);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const float2 cs = tr[i];
+                        float *pr = i < 16 ? xa + 2 * i : xb + 2 * (i - 16);
+                        const float a = pr[0], bb = pr[1];
+                        pr[0] = (a * cs.x - bb * cs.y) * p.scale_log2;
+                        pr[1] = (a * cs.y + bb * cs.x) * p.scale_log2;
+                    }
+                    store32_bf16(qo + 64 * hf * 2, xa);
+                    store32_bf16(qo + (64 * hf + 32) * 2, xb);
                 }
             }
         }

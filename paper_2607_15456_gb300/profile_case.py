@@ -13,6 +13,12 @@ rope: the same decode calls through lla_decode_attn_rope (RoPE after reconstruct
     ncu --set full --clock-control none -k regex:decode_rope_kernel -s 6 -c 1 \\
         python -m paper_2607_15456_gb300.profile_case --case rope --workload ouro14_rho4 --layers 2 --calls 10
 
+rope_prefill: the same prompts through lla_prefill_attn_rope (key rebuild, then attention):
+
+    ncu --set full --clock-control none -k regex:"rope_rebuild_kernel|prefill_tc_kernel" -c 2 \\
+        python -m paper_2607_15456_gb300.profile_case --case rope_prefill --workload ouro14_rho2 \\
+        --prompts 4 --len 8192 --calls 1
+
 prefill: encodes `--prompts` prompts of `--len` tokens of a workload's ranks (tensor-core encode,
 one launch per axis), then runs `--calls` causal prefill calls over them:
 
@@ -86,8 +92,16 @@ def prefill_case(args):
     q = W.normal((N, H, d), w.seed, 302, device=dev)
     out = torch.empty_like(q)
     cu = torch.tensor([i * args.len for i in range(args.prompts + 1)], dtype=torch.int32, device=dev)
+    ws = None
+    if args.case == "rope_prefill":
+        ws = torch.empty(lla.lla_prefill_rope_workspace_size(geom, args.prompts, args.len),
+                         dtype=torch.uint8, device=dev)
     for _ in range(args.calls):
-        lla.lla_prefill_attn(geom, codec, cache, cu, args.len, 1, q, out)
+        if ws is not None:
+            lla.lla_prefill_attn_rope(geom, codec, cache, 10000.0, lla.LLA_ROPE_HALF, cu, args.len, 1,
+                                      q, out, ws)
+        else:
+            lla.lla_prefill_attn(geom, codec, cache, cu, args.len, 1, q, out)
     torch.cuda.synchronize()
     err = lla.lla_get_device_error()
     if err:
@@ -99,7 +113,7 @@ def prefill_case(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--case", choices=["decode", "rope", "prefill"], default="decode")
+    ap.add_argument("--case", choices=["decode", "rope", "prefill", "rope_prefill"], default="decode")
     ap.add_argument("--workload", default="ouro14_rho4")
     ap.add_argument("--layers", type=int, default=2)
     ap.add_argument("--calls", type=int, default=10)
