@@ -231,6 +231,15 @@ class DecodeBench:
                                          self.q[l, t], self.cur_k[l, t], self.cur_v[l, t],
                                          self.out[l, t], self.ws)
 
+    def decode_calls_loops(self, ws):
+        """The same T x D pass-1 calls as D calls that each take all T loops of a layer in one
+        pass over its latents (lla_decode_attn_loops)."""
+        lla = self.lla
+        for l in range(self.w.D):
+            lla.lla_decode_attn_loops(self.geom, self.codecs[l], self.caches[l], self.ctx,
+                                      self.max_ctx, self.q[l], self.cur_k[l], self.cur_v[l],
+                                      self.out[l], ws)
+
     def encode_calls(self):
         # the completed token of every sequence, in every layer: its stacked loop-t keys and
         # values (one lla_encode_layers launch for all layers)
@@ -368,6 +377,7 @@ def run_ours(args, rank, world, local_rank):
         result["cpu_baseline"] = cpu_baseline(bench.w, bench.lens, args.cpu_seconds)
     if not args.no_extras and rank == 0:
         result.update(run_rope_extra(bench))
+        result.update(run_loops_extra(bench))
         del bench
         torch.cuda.empty_cache()
         result.update(run_extras(device))
@@ -413,6 +423,32 @@ def run_rope_extra(bench):
         "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
         "bytes_per_launch": nbytes, "key_rebuild_TFLOP_s": rebuild_flops / per_launch_s / 1e12,
         "tokens_per_s_decode_only": bench.B / (ms / 1e3)}}
+
+
+def run_loops_extra(bench):
+    """Multi-query decode against the shared latent (the next row after full RoPE): the step's
+    T x D pass-1 calls as D calls of lla_decode_attn_loops, each reading a layer's latents once
+    for all T loops.  Reported beside the headline, never as it: the paper's loops run one after
+    the other, so this is the regime of loops computed together."""
+    import torch
+    w, lla = bench.w, bench.lla
+    peak, _ = measured_peaks()
+    ws = torch.zeros(lla.lla_decode_loops_workspace_size(bench.geom, bench.B), dtype=torch.uint8,
+                     device=bench.device)
+    ms = _time_ms(lambda: bench.decode_calls_loops(ws), reps=3, warm=1)
+    per_launch_s = ms / 1e3 / w.D
+    lat = sum(bench.lens) * w.H * (w.r_k + w.r_v) * 2
+    nbytes = lat + w.T * (w.H * w.d * (w.r_k + w.r_v) * 2 + 4 * bench.B * w.H * w.d * 2)
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the multi-loop decode measurement")
+    return {"loops_decode": {
+        "workload": f"{w.name} batch, all {w.T} loops of a layer per call (shared latent), "
+                    f"{w.D} calls per step",
+        "kernel": "decode_loops_kernel (lla_decode_attn_loops)", "bound": "hbm",
+        "ms_per_sweep": ms, "avg_launch_us": per_launch_s * 1e6,
+        "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
+        "bytes_per_launch": nbytes, "tokens_per_s_decode_only": bench.B / (ms / 1e3),
+        "note": "the layer's latents cross HBM once for its T loop calls"}}
 
 
 def run_extras(device):

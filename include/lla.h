@@ -14,6 +14,7 @@
  *   lla_decode_attn_rope the same with rotary positions applied after reconstruction (Sec. 3,
  *                        "RoPE and reconstruction"), keys rebuilt on the tensor cores
  *   lla_prefill_attn_rope  causal prefill with rotary positions after reconstruction
+ *   lla_decode_attn_loops  the decode calls of all T loops in one pass over the latents
  *   lla_prefill_attn     causal pass-2 prefill attention over the latents of a prompt
  *   lla_dense_*          the uncompressed loop-t KV decode in the same kernel style (the
  *                        "teacher" column of Table absorbed_latency, App. J), for comparison
@@ -175,6 +176,28 @@ lla_status lla_decode_attn(const lla_geometry *g, const lla_codec *codec, const 
                            const void *q, const void *cur_k, const void *cur_v,
                            lla_dtype io_dtype, void *out, void *workspace,
                            size_t workspace_bytes, void *stream);
+
+/* Workspace bytes lla_decode_attn_loops needs for a batch of B sequences on the current device. */
+lla_status lla_decode_loops_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes);
+
+/*
+ * The decode calls of all T loops of one layer in one pass over the latents: T queries of each
+ * (sequence, head) against the shared latent (the latent of a token is one code for every loop,
+ * Sec. 3 Eq. encode; App. J absorbed attention per loop).  For loops computed in parallel or
+ * speculatively, or a verification of several loop outputs; the layer's latents are read once
+ * instead of T times.  The result of loop t equals lla_decode_attn at loop t.
+ *   q, cur_k, cur_v, out  device [T][B][H][d] io_dtype (loop-major): loop t's query, pass-1 exact
+ *                         current key and value (both NULL: pass 2), and output
+ *   workspace             >= lla_decode_loops_workspace_size bytes, zero-filled before first use;
+ *                         every completed call leaves it zero-filled again
+ * Other arguments and the error behaviour are those of lla_decode_attn.  Storage LLA_BF16, d = 128,
+ * T = 4 and (r_k, r_v) one of (96, 160), (128, 128); LLA_ERR_UNSUPPORTED otherwise.
+ */
+lla_status lla_decode_attn_loops(const lla_geometry *g, const lla_codec *codec,
+                                 const lla_cache *cache, const int32_t *context_lens, int32_t B,
+                                 int32_t max_ctx, const void *q, const void *cur_k,
+                                 const void *cur_v, lla_dtype io_dtype, void *out, void *workspace,
+                                 size_t workspace_bytes, void *stream);
 
 /* Rotary position embedding (RoFormer) applied after reconstruction (Sec. 3 "RoPE and
  * reconstruction"): pair j of a d-vector at position p is turned by the angle p * base^(-2j/d). */

@@ -183,7 +183,7 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
                          const int32_t *context_lens, int32_t B, int32_t max_ctx, int32_t loop,
                          const void *q, const void *cur_k, const void *cur_v, lla_dtype io_dtype,
                          void *out, void *workspace, size_t workspace_bytes, void *stream,
-                         bool absorbed, const lla_rope *rope = nullptr) {
+                         bool absorbed, const lla_rope *rope = nullptr, bool loops = false) {
     lla_status st = check_geometry(g);
     if (st != LLA_OK) return st;
     if ((st = check_cache(cache, true)) != LLA_OK) return st;
@@ -213,6 +213,8 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
             (cur_v && !aligned(cur_v, 16)) || (out && !aligned(out, 16)))
             return LLA_ERR_INVALID_ARG;
         if ((st = decode_rope_fits(g->r_k, g->r_v, es, g->d, B)) != LLA_OK) return st;
+    } else if (loops) {
+        if ((st = decode_loops_fits(g->r_k, g->r_v, es, g->d, g->T, B)) != LLA_OK) return st;
     } else if ((st = decode_fits(g->r_k, g->r_v, es, g->d)) != LLA_OK) {
         return st;
     }
@@ -237,6 +239,7 @@ lla_status decode_common(const lla_geometry *g, const lla_codec *codec, const ll
     if (rope)
         return launch_decode_rope(a, rope->base, rope->pairing == LLA_ROPE_ADJACENT ? 1 : 0,
                                   static_cast<cudaStream_t>(stream));
+    if (loops) return launch_decode_loops(a, static_cast<cudaStream_t>(stream));
     return launch_decode(a, static_cast<cudaStream_t>(stream));
 }
 
@@ -260,6 +263,25 @@ lla_status lla_decode_attn_rope(const lla_geometry *g, const lla_codec *codec,
     if (!rope) return LLA_ERR_INVALID_ARG;
     return decode_common(g, codec, cache, context_lens, B, max_ctx, loop, q, cur_k, cur_v,
                          io_dtype, out, workspace, workspace_bytes, stream, true, rope);
+}
+
+lla_status lla_decode_loops_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
+    const int grid = num_sms();
+    if (grid <= 0) return LLA_ERR_CUDA;
+    *bytes = decode_loops_workspace_bytes(g->r_v, B, g->H, g->T, grid);
+    return LLA_OK;
+}
+
+lla_status lla_decode_attn_loops(const lla_geometry *g, const lla_codec *codec,
+                                 const lla_cache *cache, const int32_t *context_lens, int32_t B,
+                                 int32_t max_ctx, const void *q, const void *cur_k,
+                                 const void *cur_v, lla_dtype io_dtype, void *out, void *workspace,
+                                 size_t workspace_bytes, void *stream) {
+    return decode_common(g, codec, cache, context_lens, B, max_ctx, 0, q, cur_k, cur_v, io_dtype,
+                         out, workspace, workspace_bytes, stream, true, nullptr, true);
 }
 
 lla_status lla_dense_decode_attn(const lla_geometry *g, const lla_cache *cache,

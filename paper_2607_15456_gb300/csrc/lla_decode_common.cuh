@@ -1011,8 +1011,9 @@ __device__ __forceinline__ int atom_add_acq_rel_gpu(int *addr, int v) {
 // Management: the run that left its state in slot `slot` -- reduce it, then finish the
 // (sequence, head) in place, or write a partial and merge all of them if this CTA is the last
 // to arrive.  One acquire-release atomic both publishes this CTA's partial and tells the last
-// CTA that every other partial is visible.
-template <int ES, int RK, int RV, int D, int TT, int NTG, int WL = kWstMax>
+// CTA that every other partial is visible.  With RELEASE false the state slot stays taken (a
+// later finish reads more of it and releases it).
+template <int ES, int RK, int RV, int D, int TT, int NTG, int WL = kWstMax, bool RELEASE = true>
 __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t u, const Range &rg,
                          int slot, uint32_t parity, int qs, int mt) {
     constexpr int WST = AsyncSizes<ES, RK, RV, D, WL>::WST;
@@ -1039,7 +1040,7 @@ __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t 
     for (int i = 0; i < TT; ++i) l += lred[i];
     const float m = a.s.misc[kAM + slot];
     m_sync();
-    mbar_arrive(&a.stfree[slot]);  // the run's state slot may take a later run's state
+    if constexpr (RELEASE) mbar_arrive(&a.stfree[slot]);  // the slot may take a later run's state
     if (u == R.seg_start && R.run_end == R.seg_end) {
         m_output<ES, RK, RV, D, WL>(p, a, R.b, R.h, m, l, qs, mt);
         return;

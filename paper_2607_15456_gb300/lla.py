@@ -81,6 +81,8 @@ def library() -> ctypes.CDLL:
             "lla_decode_attn_noalloc": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P]),
             "lla_decode_attn_rope": (I32, [P, P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ,
                                            P]),
+            "lla_decode_loops_workspace_size": (I32, [P, I32, P]),
+            "lla_decode_attn_loops": (I32, [P, P, P, P, I32, I32, P, P, P, I32, P, P, SZ, P]),
             "lla_prefill_attn": (I32, [P, P, P, P, I32, I32, I32, P, I32, P, P]),
             "lla_prefill_rope_workspace_size": (I32, [P, I32, I32, P]),
             "lla_prefill_attn_rope": (I32, [P, P, P, P, P, I32, I32, I32, P, I32, P, P, SZ, P]),
@@ -261,6 +263,26 @@ def lla_decode_attn_rope(geom: Geometry, codec: Codec, cache: Cache, rope_base: 
         _ptr(context_lens), q.shape[0], max_ctx, loop, _ptr(q), _ptr(cur_k), _ptr(cur_v),
         _dtype_code(q), _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
         _stream(stream)))
+
+
+def lla_decode_loops_workspace_size(geom: Geometry, B: int) -> int:
+    g = geom.c()
+    out = ctypes.c_size_t()
+    _check("lla_decode_loops_workspace_size",
+           library().lla_decode_loops_workspace_size(ctypes.byref(g), B, ctypes.byref(out)))
+    return out.value
+
+
+def lla_decode_attn_loops(geom: Geometry, codec: Codec, cache: Cache, context_lens: torch.Tensor,
+                          max_ctx: int, q: torch.Tensor, cur_k: Optional[torch.Tensor],
+                          cur_v: Optional[torch.Tensor], out: torch.Tensor,
+                          workspace: torch.Tensor, stream=None) -> None:
+    """All T loops' decode calls in one pass over the latents: q, cur_k, cur_v, out [T][B][H][d]."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    _check("lla_decode_attn_loops", library().lla_decode_attn_loops(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(context_lens), q.shape[1],
+        max_ctx, _ptr(q), _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def lla_decode_attn_noalloc(geom: Geometry, codec: Codec, cache: Cache,

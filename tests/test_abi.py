@@ -254,3 +254,22 @@ def test_prefill_rope_argument_checks(lib):
     assert call(g_=g72) == UNSUPPORTED
     assert call(g_=_g(lib, storage="fp32")) == UNSUPPORTED
     assert call(B=0, q=None, out=None, ws=None, cu=None) == OK
+
+
+def test_decode_loops_argument_checks(lib):
+    so = lib.library()
+
+    def call(g=None, B=4, max_ctx=128, q=FAKE, ck=FAKE, cv=FAKE, io=0, out=FAKE, ws=FAKE,
+             lens=FAKE):
+        g = g or _g(lib)
+        codec, cache = _codec(lib), _cache(lib)
+        return so.lla_decode_attn_loops(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache),
+                                        lens, B, max_ctx, q, ck, cv, io, out, ws, 1 << 20, None)
+    assert call(ck=None) == INVALID
+    assert call(B=-1) == INVALID
+    assert call(q=None) == INVALID
+    assert call(max_ctx=4 * 64 + 1) == INVALID
+    assert call(g=_g(lib, T=3)) == UNSUPPORTED
+    assert call(g=_g(lib, r_k=72, r_v=120)) == UNSUPPORTED
+    assert call(g=_g(lib, storage="fp32")) == UNSUPPORTED
+    assert call(B=0, q=None, ck=None, cv=None, out=None, ws=None, lens=None) == OK
