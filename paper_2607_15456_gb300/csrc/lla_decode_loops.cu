@@ -22,7 +22,7 @@
 namespace lla {
 namespace {
 
-constexpr int kLoopsWst = 20 * 1024;  // staging buffer of W_up,t rows
+constexpr int kLoopsWst = 40 * 1024;  // staging buffer of W_up,t rows (one pass each)
 constexpr int kNQ = 4;                // loops per call
 
 template <int RK, int RV>
@@ -277,9 +277,9 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_loops_kernel(const Pa
                 mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
                 float sc[kNQ];
                 {
-                    float a0[kNQ], a1[kNQ];
+                    float2 acc[kNQ];  // even and odd latent columns, packed
 #pragma unroll
-                    for (int t = 0; t < kNQ; ++t) a0[t] = a1[t] = 0.f;
+                    for (int t = 0; t < kNQ; ++t) acc[t] = make_float2(0.f, 0.f);
                     if (tt < nvalid) {
                         const char *kp = sb + tt * F::GK + ks * F::NGT * (kBlockTokens * F::GK);
 #pragma unroll
@@ -293,15 +293,14 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_loops_kernel(const Pa
                                 load_qvec<F::KE>(l.qlat + (t * kQSlots + qslot) * Z::QSLOT +
                                                      (ks * F::NGT + g) * F::KE, qv);
 #pragma unroll
-                                for (int e = 0; e < F::KE; e += 2) {
-                                    a0[t] = fmaf(v[e], qv[e], a0[t]);
-                                    a1[t] = fmaf(v[e + 1], qv[e + 1], a1[t]);
-                                }
+                                for (int e = 0; e < F::KE; e += 2)
+                                    acc[t] = __ffma2_rn(make_float2(v[e], v[e + 1]),
+                                                        make_float2(qv[e], qv[e + 1]), acc[t]);
                             }
                         }
                     }
 #pragma unroll
-                    for (int t = 0; t < kNQ; ++t) sc[t] = a0[t] + a1[t];
+                    for (int t = 0; t < kNQ; ++t) sc[t] = acc[t].x + acc[t].y;
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&s.empty[stage]);  // K-plane read
@@ -313,11 +312,19 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_loops_kernel(const Pa
                 const bool valid = tt < nvalid;
                 float x[kNQ];
                 if (ks == 0) {
+                    float lm[kNQ];
 #pragma unroll
                     for (int t = 0; t < kNQ; ++t) {
                         x[t] = valid ? (sc[t] + l.spart[t * 64 + tt] + beta[t]) * p.scale_log2 : -INFINITY;
-                        const float lm = warp_max(x[t]);
-                        if (lane == 0) l.miscl[t * 64 + kAWmax + slot * 8 + warp] = lm;
+                        lm[t] = x[t];
+                    }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1)  // the T warp maxima, interleaved
+#pragma unroll
+                        for (int t = 0; t < kNQ; ++t) lm[t] = fmaxf(lm[t], __shfl_xor_sync(0xffffffffu, lm[t], o));
+                    if (lane == 0) {
+#pragma unroll
+                        for (int t = 0; t < kNQ; ++t) l.miscl[t * 64 + kAWmax + slot * 8 + warp] = lm[t];
                     }
                 }
                 named_bar_sync(kBarTok, F::S_THREADS);
@@ -352,7 +359,7 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_loops_kernel(const Pa
                     }
                     const char *vp = sb + F::KPLANE + tg * F::ROWB + vc * Z::VB;
                     const int cnt = nvalid > tg ? (nvalid - tg + Z::NTG - 1) / Z::NTG : 0;
-#pragma unroll 2
+#pragma unroll 4
                     for (int i = 0; i < cnt; ++i) {
                         const int row = tg + i * Z::NTG;
                         float v[Z::VE];
