@@ -701,8 +701,8 @@ __global__ void __launch_bounds__(kGThreads) prefill_generic_kernel(const GParam
 // ------------------------------------------------- rotary positions: rebuild and rotate keys
 //
 // Sec. 3 "RoPE and reconstruction": keys are rebuilt by Eq. decode and rotated at their
-// positions before attention.  One CTA per (sequence, page of 64 prompt tokens) loops over the
-// heads: Khat (64 tokens x d) = C_k W_up,t^K^T + mu^K_t on tcgen05 (M = 64 tokens, N = d,
+// positions before attention.  One CTA per (sequence, page of 64 prompt tokens, group of heads)
+// loops over its heads: Khat (64 tokens x d) = C_k W_up,t^K^T + mu^K_t on tcgen05 (M = 64 tokens, N = d,
 // K = r_k, plus one K step for mu^K_t), then each token's pairs are rotated in registers and
 // written as a bf16 page in the K-plane layout (granule g of 8 dimensions at g*1024 + token*16),
 // and the page's queries are rotated and scaled by scale * log2 e into a bf16 copy of q.
@@ -786,6 +786,8 @@ __global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + 1);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int pg = blockIdx.x, b = blockIdx.y;
+    const int hpg = (p.H + gridDim.z - 1) / gridDim.z;  // heads of this CTA: [h0, h1)
+    const int h0 = blockIdx.z * hpg, h1 = min(p.H, h0 + hpg);
     pdl_wait();
     const int q0 = p.cu_seqlens[b];
     const int L = p.cu_seqlens[b + 1] - q0;
@@ -793,7 +795,7 @@ __global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant
         if (tid == 0 && pg == 0) atomicOr(p.err, LLA_DEVERR_CONTEXT);
         return;
     }
-    if (pg * kPT >= L) return;  // uniform, before any barrier
+    if (pg * kPT >= L || h0 >= h1) return;  // uniform, before any barrier
     const int nvalid = min(kPT, L - pg * kPT);
     int32_t blk = p.block_table[static_cast<int64_t>(b) * p.max_blocks + pg];
     if (blk < 0 || blk >= p.num_blocks) {
@@ -847,8 +849,8 @@ __global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant
                            (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16),
                        0u, 0u, 0u);
     };
-    stage(0);
-    for (int h = 0; h < p.H; ++h) {
+    stage(h0);
+    for (int h = h0; h < h1; ++h) {
         cp_async_wait_all();
         fence_proxy_async_smem();
         tc_fence_before();
@@ -867,11 +869,11 @@ __global__ void __launch_bounds__(128) rope_rebuild_kernel(const __grid_constant
         }
         {
             volatile int never = 0;
-            mbar_wait(bar, h & 1, &never, p.err);
+            mbar_wait(bar, (h - h0) & 1, &never, p.err);
         }
         tc_fence_after();
         // the MMA has read its operands: the next head's travel while this one's epilogue runs
-        if (h + 1 < p.H) stage(h + 1);
+        if (h + 1 < h1) stage(h + 1);
         uint32_t r0[32], r1[32];  // dimensions 0..63 (k = 0..7) and 64..127 (k = 8..15)
         tmem_ld16x256_x8_nowait(tq, r0);
         tmem_ld16x256_x8_nowait(tq + 64, r1);
@@ -1081,7 +1083,9 @@ lla_status launch_rebuild(const RParams &rp, int kpps, int B, cudaStream_t strea
             return LLA_ERR_CUDA;
         configured[dev] = true;
     }
-    return launch_pf(rope_rebuild_kernel<RK>, dim3(kpps, B), 128, RB<RK>::SMEM, stream, rp);
+    // heads split over a few CTAs per page, so that more CTAs hide each other's load latency
+    const int groups = rp.H >= 8 ? 4 : 1;
+    return launch_pf(rope_rebuild_kernel<RK>, dim3(kpps, B, groups), 128, RB<RK>::SMEM, stream, rp);
 }
 }  // namespace
 
