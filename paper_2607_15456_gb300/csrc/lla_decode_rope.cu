@@ -61,11 +61,14 @@ template <int RK, int RV>
 struct RopeShape {
     using F = Fast<2, RK, RV>;
     static constexpr int KSTEPS = RK / 16;          // MMAs of K = 16 per page
-    // TMEM columns: two 64-column accumulators, then two A slots of W_up,t^K (two bf16 per
-    // column) followed by the mu step's (mu_hi, mu_lo, 0, ...) in 8 more columns
+    // TMEM columns: three 64-column accumulators (the MMA runs up to two pages ahead of the
+    // epilogue), then two A slots of W_up,t^K (two bf16 per column) followed by the mu step's
+    // (mu_hi, mu_lo, 0, ...) in 8 more columns
+    static constexpr int NACC = 3;
+    static constexpr int A_BASE = NACC * 64;
     static constexpr int A_COLS = RK / 2 + 8;
     static constexpr int A_STRIDE = A_COLS <= 64 ? 64 : 96;
-    static constexpr int TMEM_COLS = 128 + 2 * A_STRIDE <= 256 ? 256 : 512;
+    static constexpr int TMEM_COLS = A_BASE + 2 * A_STRIDE <= 256 ? 256 : 512;
     static constexpr uint32_t IDESC = umma_idesc_bf16(kRopeD, 64, 0, 0);
     static_assert(RK % 32 == 0, "whole K steps, W_up,t^K rows in 16-column TMEM stores");
     static_assert(A_COLS <= A_STRIDE, "A slot");
@@ -83,7 +86,7 @@ __host__ __device__ inline RopeLayout rope_layout(int stages, int stage_bytes, i
     int o = (async_layout<2, RK, RV, kRopeD, kRopeWst>(stages, stage_bytes, B).total + 127) & ~127;
     L.ones = o;  o += 2 * 64 * 16;                // B operand of the mu step: (1, 1, 0...) and zeros
     L.red = o;   o += 2 * 4 * 64 * 4;             // per-warp partial scores, two page slots
-    L.bars = o;  o += 8 * 8;                      // aful[2], afree[2], tfull[2], tfree[2]
+    L.bars = o;  o += 10 * 8;                     // aful[2], afree[2], tfull[3], tfree[3]
     L.tmem = o;  o += 16;
     L.total = o;
     return L;
@@ -102,7 +105,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
     char *ones = smem + RL.ones;
     float *red4 = reinterpret_cast<float *>(smem + RL.red);
     uint64_t *aful = reinterpret_cast<uint64_t *>(smem + RL.bars);
-    uint64_t *afree = aful + 2, *tfull = aful + 4, *tfree = aful + 6;
+    uint64_t *afree = aful + 2, *tfull = aful + 4, *tfree = aful + 7;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + RL.tmem);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool pass1 = p.cur_k != nullptr;
@@ -115,6 +118,8 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
             mbar_init(&a.stfree[i], kMThreads);
             mbar_init(&aful[i], 1);
             mbar_init(&afree[i], 1);
+        }
+        for (int i = 0; i < Z::NACC; ++i) {
             mbar_init(&tfull[i], 1);
             mbar_init(&tfree[i], 4);
         }
@@ -153,13 +158,14 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
             const Run R = locate_run(p, s, u, rg.hi[pass]);
             const int as = r & 1;
-            const uint32_t acol = tmem_base + 128 + as * Z::A_STRIDE;
+            const uint32_t acol = tmem_base + Z::A_BASE + as * Z::A_STRIDE;
             if (lane == 0) mbar_wait(&aful[as], (r >> 1) & 1, s.abort_flag, p.err);
             for (int k = 0; k < R.npages; ++k, ++it) {
-                const int b = it & 1;
+                const int b = it % Z::NACC;
                 if (lane == 0) {
                     mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
-                    if (it >= 2) mbar_wait(&tfree[b], ((it - 2) >> 1) & 1, s.abort_flag, p.err);
+                    if (it >= Z::NACC)
+                        mbar_wait(&tfree[b], ((it - Z::NACC) / Z::NACC) & 1, s.abort_flag, p.err);
                     tc_fence_after();
                     const uint32_t d = tmem_base + b * 64;
                     const uint32_t bbase = smem_addr(s.ring + stage * p.stage_bytes);
@@ -183,7 +189,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
         // every MMA has completed before TMEM is released, even after an abort
         if (lane == 0 && it > 0) {
             volatile int never = 0;
-            mbar_wait(&tfull[(it - 1) & 1], ((it - 1) >> 1) & 1, &never, p.err);
+            mbar_wait(&tfull[(it - 1) % Z::NACC], ((it - 1) / Z::NACC) & 1, &never, p.err);
         }
         named_bar_sync(kBarTmem, 128 + 32);  // the epilogue warps have read every buffer
         tc_fence_after();
@@ -230,7 +236,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
                               0u, 0u, 0u, 0u, 0u, 0u, 0u};
             if (r >= 2) mbar_wait(&afree[as], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
             tc_fence_after();
-            const uint32_t acol = tlane + 128 + as * Z::A_STRIDE;
+            const uint32_t acol = tlane + Z::A_BASE + as * Z::A_STRIDE;
 #pragma unroll
             for (int c = 0; c < RK / 32; ++c) {
                 uint32_t part[16];
@@ -298,7 +304,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
             }
             const int P = pass1 ? R.Lb : R.Lb - 1;  // the query's position
             for (int k = 0; k < R.npages; ++k, ++it) {
-                const int b = it & 1, slot = it & 1;
+                const int b = it % Z::NACC, slot = it & 1;
                 const int pg = R.pg0 + k;
                 // exact phase of the page's first token: Delta0 theta_j in turns, mod 1
                 const int delta0 = P - pg * kBlockTokens;  // >= 0: the page holds a cached token
@@ -321,7 +327,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
                     DD[hv] = make_float2(fmaf(er, h2, ei * s2), fmaf(orr, h2, oi * s2));
                 }
                 uint32_t v0[32], v1[32];  // this dimension of tokens 0..31 and 32..63
-                mbar_wait(&tfull[b], (it >> 1) & 1, s.abort_flag, p.err);
+                mbar_wait(&tfull[b], (it / Z::NACC) & 1, s.abort_flag, p.err);
                 tc_fence_after();
                 const uint32_t tcol = tlane + b * 64;
                 tmem_ld32_nowait(tcol, v0);
@@ -356,7 +362,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
                 tmem_wait_ld(v1);
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&tfree[b]);  // the buffer may take page it + 2
+                if (lane == 0) mbar_arrive(&tfree[b]);  // the buffer may take page it + NACC
                 float S[16];  // S[2k + e]: token 8k + 2(lane % 4) + e, summed over 4 dimensions
 #pragma unroll
                 for (int k8 = 0; k8 < 8; ++k8) {
