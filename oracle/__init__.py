@@ -24,6 +24,9 @@ calls it through ctypes.  Citations (paper sections and equations):
                                        reconstruction (Sec. 3, "RoPE and reconstruction")
 * ``decode_rope``, ``prefill_rope`` -- ``decode`` / ``prefill`` with every reconstructed key
                                        and the query rotated at their token positions
+* ``ratio_2d``, ``encode_2d``,      -- the LLA-2D variant (Sec. 3, "The LLA-2D variant (loop x
+  ``decode_2d``                        head)"): one latent per (token, layer) over the
+                                       loop-major (loop, head) stack, every head rebuilt from it
 
 Parity status of every function: pinned (see ``tests/test_oracle_pins.py``).
 """
@@ -75,6 +78,14 @@ def _load():
         lib.lla_oracle_decode_batch.argtypes = [i32, i32, i32, i32, d, i64, p, i32]
         lib.lla_oracle_encode_batch.restype = i32
         lib.lla_oracle_encode_batch.argtypes = [i32, i32, i64, i64, p, i32]
+        lib.lla_oracle_ratio_2d.restype = d
+        lib.lla_oracle_ratio_2d.argtypes = [i32, i32, i32, i32, i32]
+        lib.lla_oracle_encode_2d.restype = None
+        lib.lla_oracle_encode_2d.argtypes = [i32, i32, i32, i32, i64, p, p, p, p]
+        lib.lla_oracle_decode_2d_head.restype = i32
+        lib.lla_oracle_decode_2d_head.argtypes = [i32] * 7 + [i64] + [p] * 9 + [d, p]
+        lib.lla_oracle_decode_2d_batch.restype = i32
+        lib.lla_oracle_decode_2d_batch.argtypes = [i32, i32, i32, i32, i32, d, i64, p, i32]
         lib.lla_oracle_max_threads.restype = i32
         lib.lla_oracle_max_threads.argtypes = []
         _lib = lib
@@ -248,11 +259,81 @@ def prefill_rope(t: int, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, scale: float,
     return out
 
 
+# ---------------------------------------------------------------- LLA-2D (Sec. 3)
+
+def ratio_2d(T: int, H: int, d_head: int, r_k: int, r_v: int) -> float:
+    """rho_2D = 2 T H d / (r_k + r_v): one latent pair per (token, layer)."""
+    return _load().lla_oracle_ratio_2d(T, H, d_head, r_k, r_v)
+
+
+def encode_2d(x, mu, w_down) -> np.ndarray:
+    """LLA-2D encode.  x [T][N][H][d], mu [T*H*d] or None, w_down [T*H*d][r] -> c [N][r]."""
+    x, w_down = _f64(x), _f64(w_down)
+    T, N, H, d = x.shape
+    r = w_down.shape[1]
+    assert w_down.shape[0] == T * H * d
+    mu = None if mu is None else _f64(mu).reshape(T * H * d)
+    c = np.zeros((N, r), dtype=np.float64)
+    _load().lla_oracle_encode_2d(T, H, d, r, N, _ptr(x), _ptr(mu), _ptr(w_down), _ptr(c))
+    return c
+
+
+def _decode_2d_args(w_up_k, w_up_v, mu_k, mu_v):
+    w_up_k, w_up_v = _f64(w_up_k), _f64(w_up_v)
+    T, H, d, r_k = w_up_k.shape
+    r_v = w_up_v.shape[3]
+    assert w_up_v.shape[:3] == (T, H, d)
+    mu_k = None if mu_k is None else _f64(mu_k).reshape(T * H * d)
+    mu_v = None if mu_v is None else _f64(mu_v).reshape(T * H * d)
+    return w_up_k, w_up_v, mu_k, mu_v, T, H, d, r_k, r_v
+
+
+def decode_2d(t: int, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, cur_k, cur_v,
+              scale: float, heads: Optional[Sequence[int]] = None,
+              n_threads: int = 0) -> np.ndarray:
+    """One LLA-2D decode call for one sequence at loop t.
+
+    c_k [L][r_k], c_v [L][r_v] (one latent per token for all heads); w_up_k [T][H][d][r_k];
+    w_up_v [T][H][d][r_v]; mu_* [T*H*d] or None; q [H][d]; cur_k / cur_v [H][d] (pass 1) or
+    None (pass 2).  Returns out [len(heads)][d] for the listed heads (default: all).
+    """
+    w_up_k, w_up_v, mu_k, mu_v, T, H, d, r_k, r_v = _decode_2d_args(w_up_k, w_up_v, mu_k, mu_v)
+    c_k = _f64(c_k).reshape(-1, r_k)
+    c_v = _f64(c_v).reshape(-1, r_v)
+    L = c_k.shape[0]
+    q = _f64(q).reshape(H, d)
+    cur_k = None if cur_k is None else _f64(cur_k).reshape(H, d)
+    cur_v = None if cur_v is None else _f64(cur_v).reshape(H, d)
+    heads = list(range(H)) if heads is None else list(heads)
+    out = np.zeros((len(heads), d), dtype=np.float64)
+    arr = (_Decode2dItem * len(heads))()
+    for k, h in enumerate(heads):
+        it = arr[k]
+        it.t, it.h, it.L = t, h, L
+        it.c_k, it.c_v, it.w_up_k, it.w_up_v = _ptr(c_k), _ptr(c_v), _ptr(w_up_k), _ptr(w_up_v)
+        it.mu_k, it.mu_v = _ptr(mu_k), _ptr(mu_v)
+        it.q = q[h].ctypes.data
+        it.cur_k = None if cur_k is None else cur_k[h].ctypes.data
+        it.cur_v = None if cur_v is None else cur_v[h].ctypes.data
+        it.out = out[k].ctypes.data
+    rc = _load().lla_oracle_decode_2d_batch(T, H, d, r_k, r_v, scale, len(heads),
+                                            ctypes.cast(arr, ctypes.c_void_p), n_threads)
+    if rc:
+        raise ValueError("bad decode arguments")
+    return out
+
+
 # ---------------------------------------------------------------- batched drivers (OpenMP)
 
 class _DecodeItem(ctypes.Structure):
     _fields_ = [("t", ctypes.c_int32), ("rope", ctypes.c_int32), ("L", ctypes.c_int64),
                 ("rope_base", ctypes.c_double)] + [
+        (n, ctypes.c_void_p) for n in
+        ("c_k", "c_v", "w_up_k", "w_up_v", "mu_k", "mu_v", "q", "cur_k", "cur_v", "out")]
+
+
+class _Decode2dItem(ctypes.Structure):
+    _fields_ = [("t", ctypes.c_int32), ("h", ctypes.c_int32), ("L", ctypes.c_int64)] + [
         (n, ctypes.c_void_p) for n in
         ("c_k", "c_v", "w_up_k", "w_up_v", "mu_k", "mu_v", "q", "cur_k", "cur_v", "out")]
 
@@ -321,5 +402,6 @@ def encode_batch(T: int, d: int, items: Sequence[dict], n_threads: int = 0) -> l
 
 __all__ = ["ratio", "teacher_cache_bytes_per_token", "latent_cache_bytes_per_token", "encode",
            "reconstruct", "attention", "decode", "prefill", "rope", "decode_rope",
-           "prefill_rope", "ROPE_HALF", "ROPE_ADJACENT", "decode_batch", "encode_batch",
+           "prefill_rope", "ROPE_HALF", "ROPE_ADJACENT", "ratio_2d", "encode_2d", "decode_2d",
+           "decode_batch", "encode_batch",
            "max_threads", "build_oracle", "library_path"]

@@ -314,6 +314,125 @@ int lla_oracle_prefill_rope(int T, int d, int r_k, int r_v, int t, int64_t N, co
     return rc;
 }
 
+/*
+ * LLA-2D (Sec. 3, "The LLA-2D variant (loop x head)"): one latent per (token, layer) that
+ * covers every head.  The stacked vector runs over loops and heads, loop-major,
+ *   x = [x_{1,1}; ...; x_{1,H}; x_{2,1}; ...; x_{T,H}] in R^{T H d},
+ * is encoded as c = (x - mu) W_down with W_down in R^{THd x r}, and head h at loop t is rebuilt
+ * as xhat_{t,h} = c W_up,t,h^T + mu_{t,h} with W_up,t,h in R^{d x r}, mu_{t,h} the (t, h) slice
+ * of mu.  The cache then holds (r_k + r_v) scalars per token and layer (Sec. 3 and App. J "Per-
+ * head LLA versus LLA-2D at inference"): rho_2D = 2 T H d / (r_k + r_v).
+ */
+double lla_oracle_ratio_2d(int T, int H, int d_head, int r_k, int r_v)
+{
+    return 2.0 * (double)T * (double)H * (double)d_head / (double)(r_k + r_v);
+}
+
+/*
+ * LLA-2D encode of N tokens of one (layer, axis).
+ *   x      [T][N][H][d]  x[t][n][h] is the loop-t vector of head h of token n
+ *   mu     [T*H*d]       mean of the stacked vector, or NULL
+ *   w_down [T*H*d][r]
+ *   c      [N][r]
+ */
+void lla_oracle_encode_2d(int T, int H, int d, int r, int64_t N, const double *x,
+                          const double *mu, const double *w_down, double *c)
+{
+    const int S = T * H * d;
+    double *xs = (double *)malloc(sizeof(double) * (size_t)S);
+    for (int64_t n = 0; n < N; ++n) {
+        /* stack over loops, then heads: entry (t, h, e) at (t H + h) d + e */
+        for (int t = 0; t < T; ++t)
+            for (int h = 0; h < H; ++h)
+                for (int e = 0; e < d; ++e)
+                    xs[((int64_t)t * H + h) * d + e] = x[(((int64_t)t * N + n) * H + h) * d + e];
+        if (mu) /* centre: x - mu */
+            for (int k = 0; k < S; ++k)
+                xs[k] -= mu[k];
+        for (int j = 0; j < r; ++j) {
+            double acc = 0.0;
+            for (int k = 0; k < S; ++k)
+                acc += xs[k] * w_down[(int64_t)k * r + j];
+            c[n * r + j] = acc;
+        }
+    }
+    free(xs);
+}
+
+/*
+ * One LLA-2D decode call for one (sequence, head h) at loop t: every cached token's key and
+ * value of head h are rebuilt from the shared latent with the (t, h) up-projection, then plain
+ * softmax attention as in lla_oracle_decode (pass 1 appends the current token's exact loop-t
+ * key and value of head h).
+ *   c_k [L][r_k], c_v [L][r_v]            the sequence's latents (shared by all heads)
+ *   w_up_k [T][H][d][r_k], w_up_v [T][H][d][r_v]
+ *   mu_k, mu_v [T*H*d] or NULL
+ *   q, cur_k, cur_v, out [d]              head h's vectors (cur_* NULL: pass 2)
+ */
+int lla_oracle_decode_2d_head(int T, int H, int d, int r_k, int r_v, int t, int h, int64_t L,
+                              const double *c_k, const double *c_v, const double *w_up_k,
+                              const double *w_up_v, const double *mu_k, const double *mu_v,
+                              const double *q, const double *cur_k, const double *cur_v,
+                              double scale, double *out)
+{
+    if (t < 0 || t >= T || h < 0 || h >= H || L < 0)
+        return -1;
+    if ((cur_k == NULL) != (cur_v == NULL))
+        return -1;
+    const int pass1 = cur_k != NULL;
+    if (!pass1 && L < 1)
+        return -1;
+    const int64_t th = (int64_t)t * H + h; /* slice (t, h) of the up-projections and of mu */
+    const int64_t n = L + (pass1 ? 1 : 0);
+    double *K = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    double *V = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    lla_oracle_reconstruct(d, r_k, L, c_k, w_up_k + th * d * r_k, mu_k ? mu_k + th * d : NULL, K);
+    lla_oracle_reconstruct(d, r_v, L, c_v, w_up_v + th * d * r_v, mu_v ? mu_v + th * d : NULL, V);
+    if (pass1) /* the current token's exact loop-t key and value of head h */
+        for (int e = 0; e < d; ++e) {
+            K[L * d + e] = cur_k[e];
+            V[L * d + e] = cur_v[e];
+        }
+    int rc = lla_oracle_attention(d, n, q, K, V, scale, out);
+    free(K);
+    free(V);
+    return rc;
+}
+
+/* One (sequence, head) problem for lla_oracle_decode_2d_batch. */
+typedef struct {
+    int32_t t, h;
+    int64_t L;
+    const double *c_k, *c_v, *w_up_k, *w_up_v, *mu_k, *mu_v;
+    const double *q, *cur_k, *cur_v;
+    double *out;
+} lla_oracle_decode_2d_item;
+
+int lla_oracle_decode_2d_batch(int T, int H, int d, int r_k, int r_v, double scale,
+                               int64_t n_items, const lla_oracle_decode_2d_item *items,
+                               int n_threads)
+{
+    int err = 0;
+#ifdef _OPENMP
+    if (n_threads <= 0)
+        n_threads = omp_get_max_threads();
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads)
+#endif
+    for (int64_t i = 0; i < n_items; ++i) {
+        const lla_oracle_decode_2d_item *it = &items[i];
+        int rc = lla_oracle_decode_2d_head(T, H, d, r_k, r_v, it->t, it->h, it->L, it->c_k,
+                                           it->c_v, it->w_up_k, it->w_up_v, it->mu_k, it->mu_v,
+                                           it->q, it->cur_k, it->cur_v, scale, it->out);
+        if (rc != 0) {
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+            err = rc;
+        }
+    }
+    return err;
+}
+
 /* One independent decode problem for lla_oracle_decode_batch. */
 typedef struct {
     int32_t t;

@@ -46,6 +46,20 @@ MUTANTS = [
      "for (int64_t i = 0; i < n; ++i)\n        memcpy(Kr + i * d, K + i * d, sizeof(double) * (size_t)d);"),
     ("prefill_rope_query_position", "lla_oracle_rope(d, pairing, base, pos0 + i, q + i * d, qr);",
      "lla_oracle_rope(d, pairing, base, pos0, q + i * d, qr);"),
+    ("ratio_2d_drops_heads",
+     "return 2.0 * (double)T * (double)H * (double)d_head / (double)(r_k + r_v);",
+     "return 2.0 * (double)T * (double)d_head / (double)(r_k + r_v);"),
+    ("encode_2d_head_major_stack",
+     "xs[((int64_t)t * H + h) * d + e] = x[(((int64_t)t * N + n) * H + h) * d + e];",
+     "xs[((int64_t)h * T + t) * d + e] = x[(((int64_t)t * N + n) * H + h) * d + e];"),
+    ("encode_2d_mu_sign", "xs[k] -= mu[k];", "xs[k] += mu[k];"),
+    ("decode_2d_pass1_value_is_key", "V[L * d + e] = cur_v[e];", "V[L * d + e] = cur_k[e];"),
+    ("decode_2d_head_major_slice", "const int64_t th = (int64_t)t * H + h;",
+     "const int64_t th = (int64_t)h * T + t;"),
+    ("decode_2d_mu_loop_slice", "mu_k ? mu_k + th * d : NULL, K);",
+     "mu_k ? mu_k + (int64_t)t * d : NULL, K);"),
+    ("decode_2d_value_loop_only", "lla_oracle_reconstruct(d, r_v, L, c_v, w_up_v + th * d * r_v,",
+     "lla_oracle_reconstruct(d, r_v, L, c_v, w_up_v + (int64_t)t * d * r_v,"),
 ]
 
 

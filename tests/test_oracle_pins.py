@@ -554,3 +554,207 @@ def test_rope_batched_driver_equals_single_calls():
                                  cod["mu_k"], cod["mu_v"], it["q"], it["cur_k"], it["cur_v"],
                                  0.2, it["rope"][1], it["rope"][0])
         np.testing.assert_array_equal(o, ref)
+
+
+# ------------------------------------------------------------------ LLA-2D (Sec. 3)
+
+def test_ratio_2d_matches_printed_values():
+    """Table isocache prints LLA-2D at rho = 5.33 and 21.33 at the per-head rows' cache budget;
+    rho_2D = 2 T H d / (r_k + r_v), a factor H above per-head LLA at fixed ranks (App. J "Per-
+    head LLA versus LLA-2D at inference")."""
+    g = _gold("ratios.json")["isocache_2d"]
+    T, H, d = g["T"], g["H"], g["d_head"]
+    for r_k, r_v, printed in g["rows"]:
+        rho = oracle.ratio_2d(T, H, d, r_k, r_v)
+        assert abs(rho - printed) <= 0.005 + 1e-12, (r_k, r_v, rho, printed)
+        # matched budget: the 2D latent per token and layer is as large as the H per-head ones
+        assert oracle.latent_cache_bytes_per_token(1, 1, r_k, r_v, 2) == \
+            oracle.latent_cache_bytes_per_token(H, 1, r_k // H, r_v // H, 2)
+        assert rho == oracle.ratio(T, d, r_k // H, r_v // H)
+    assert oracle.ratio_2d(4, 16, 128, 96, 160) == 16 * oracle.ratio(4, 128, 96, 160)
+
+
+def test_encode_2d_matches_loop_major_stack():
+    """The 2D stack runs over loops and heads (loop-major, then head): the latent of token n is
+    the centred [x_{1,1}; ...; x_{1,H}; ...; x_{T,H}] times W_down (numpy matmul)."""
+    T, H, d, N, r = 3, 2, 8, 5, 7
+    g = _rng(60)
+    x = g.standard_normal((T, N, H, d))
+    mu = g.standard_normal(T * H * d)
+    w = g.standard_normal((T * H * d, r))
+    stacked = np.concatenate([x[t, :, h] for t in range(T) for h in range(H)], axis=1)
+    np.testing.assert_allclose(oracle.encode_2d(x, mu, w), (stacked - mu) @ w, rtol=1e-13,
+                               atol=1e-12)
+    np.testing.assert_allclose(oracle.encode_2d(x, None, w), stacked @ w, rtol=1e-13,
+                               atol=1e-12)
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+def test_full_rank_2d_decode_equals_uncompressed_attention(pass1):
+    """r = T H d with W_down = Q orthogonal and W_up,t,h = the (t, h) row block of Q: every
+    head's keys and values come back exactly, so LLA-2D decode is uncompressed loop-t attention
+    of that head (torch SDPA on the raw K/V)."""
+    T, H, d, L = 2, 3, 8, 11
+    g = _rng(61)
+    S = T * H * d
+    Qk, Qv = _orthogonal(S, 62), _orthogonal(S, 63)
+    xk, xv = g.standard_normal((T, L + 1, H, d)), g.standard_normal((T, L + 1, H, d))
+    mu_k, mu_v = g.standard_normal(S), g.standard_normal(S)
+    n_cached = L if pass1 else L + 1
+    c_k = oracle.encode_2d(xk[:, :n_cached], mu_k, Qk)
+    c_v = oracle.encode_2d(xv[:, :n_cached], mu_v, Qv)
+    blk = lambda Q, t, h: Q[(t * H + h) * d:(t * H + h + 1) * d]
+    w_up_k = np.stack([np.stack([blk(Qk, t, h) for h in range(H)]) for t in range(T)])
+    w_up_v = np.stack([np.stack([blk(Qv, t, h) for h in range(H)]) for t in range(T)])
+    scale = 1 / math.sqrt(d)
+    for t in range(T):
+        q = g.standard_normal((H, d))
+        cur_k = xk[t, L] if pass1 else None
+        cur_v = xv[t, L] if pass1 else None
+        out = oracle.decode_2d(t, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, cur_k, cur_v, scale)
+        for h in range(H):
+            ref = _sdpa(q[h], xk[t, :, h], xv[t, :, h], scale)[0]
+            np.testing.assert_allclose(out[h], ref, rtol=0, atol=1e-12)
+
+
+def _block_2d_codec(T, H, d, r_k, r_v, seed):
+    """H per-head codecs arranged as one 2D codec: latent columns h r .. (h+1) r - 1 belong to
+    head h, W_up,t,h is zero outside them."""
+    per = [_random_codec(T, d, r_k, r_v, seed + h) for h in range(H)]
+    g = _rng(seed + 100)
+    down = {}
+    two = {}
+    for ax, r in (("k", r_k), ("v", r_v)):
+        wd = [g.standard_normal((T * d, r)) / math.sqrt(T * d) for _ in range(H)]
+        W = np.zeros((T * H * d, H * r))
+        up = np.zeros((T, H, d, H * r))
+        mu = np.zeros(T * H * d)
+        for h in range(H):
+            for t in range(T):
+                rows = slice((t * H + h) * d, (t * H + h + 1) * d)
+                W[rows, h * r:(h + 1) * r] = wd[h][t * d:(t + 1) * d]
+                up[t, h, :, h * r:(h + 1) * r] = per[h]["w_up_" + ax][t]
+                mu[rows] = per[h]["mu_" + ax][t * d:(t + 1) * d]
+        down[ax] = wd
+        two.update({"w_down_" + ax: W, "w_up_" + ax: up, "mu_" + ax: mu})
+    return per, down, two
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+def test_block_diagonal_2d_codec_equals_per_head_lla(pass1):
+    """A 2D codec that keeps each head in its own block of the latent is H per-head codecs side
+    by side (Sec. 3: per-head LLA is LLA-2D without the cross-head coupling): its encode is the
+    per-head latents concatenated and its decode is per-head decode, head by head."""
+    T, H, d, r_k, r_v, L = 3, 2, 16, 5, 7, 9
+    g = _rng(64)
+    per, down, two = _block_2d_codec(T, H, d, r_k, r_v, 65)
+    xk, xv = g.standard_normal((T, L, H, d)), g.standard_normal((T, L, H, d))
+    c_k = oracle.encode_2d(xk, two["mu_k"], two["w_down_k"])
+    c_v = oracle.encode_2d(xv, two["mu_v"], two["w_down_v"])
+    for h in range(H):
+        np.testing.assert_allclose(c_k[:, h * r_k:(h + 1) * r_k],
+                                   oracle.encode(xk[:, :, h], per[h]["mu_k"], down["k"][h]),
+                                   rtol=0, atol=1e-12)
+        np.testing.assert_allclose(c_v[:, h * r_v:(h + 1) * r_v],
+                                   oracle.encode(xv[:, :, h], per[h]["mu_v"], down["v"][h]),
+                                   rtol=0, atol=1e-12)
+    scale = 1 / math.sqrt(d)
+    q = g.standard_normal((H, d))
+    cur_k = g.standard_normal((H, d)) if pass1 else None
+    cur_v = g.standard_normal((H, d)) if pass1 else None
+    for t in range(T):
+        out = oracle.decode_2d(t, c_k, c_v, two["w_up_k"], two["w_up_v"], two["mu_k"],
+                               two["mu_v"], q, cur_k, cur_v, scale)
+        for h in range(H):
+            ref = oracle.decode(t, c_k[:, h * r_k:(h + 1) * r_k], c_v[:, h * r_v:(h + 1) * r_v],
+                                per[h]["w_up_k"], per[h]["w_up_v"], per[h]["mu_k"],
+                                per[h]["mu_v"], q[h], None if cur_k is None else cur_k[h],
+                                None if cur_v is None else cur_v[h], scale)
+            np.testing.assert_allclose(out[h], ref, rtol=0, atol=1e-12)
+
+
+def test_svd_initialised_2d_codec_meets_eckart_young():
+    """SVD initialisation of the 2D codec over the (loop, head) stack: the squared
+    reconstruction error summed over every loop and head is the sum of the trailing squared
+    singular values of the stacked matrix."""
+    T, H, d, N, r = 2, 3, 8, 200, 9
+    g = _rng(66)
+    S = T * H * d
+    spectrum = np.exp(-np.arange(S) / 5.0)
+    X = (g.standard_normal((N, S)) * spectrum) @ _orthogonal(S, 67)
+    mu = X.mean(axis=0)
+    _, sv, Vt = np.linalg.svd(X - mu, full_matrices=False)
+    w_down = Vt[:r].T
+    x = np.stack([np.stack([X[:, (t * H + h) * d:(t * H + h + 1) * d] for h in range(H)], axis=1)
+                  for t in range(T)])  # [T][N][H][d]
+    c = oracle.encode_2d(x, mu, w_down)
+    err = 0.0
+    for t in range(T):
+        for h in range(H):
+            rows = slice((t * H + h) * d, (t * H + h + 1) * d)
+            xhat = oracle.reconstruct(c, w_down[rows], mu[rows])
+            err += np.sum((x[t, :, h] - xhat) ** 2)
+    expect = np.sum(sv[r:] ** 2)
+    assert abs(err - expect) <= 1e-10 * expect
+
+
+def _absorbed_2d(t, h, c_k, c_v, up_k, up_v, mu_k, mu_v, q, cur_k, cur_v, scale):
+    """App. J "Absorbed attention" for head h of a 2D codec, written independently of the
+    oracle: q~ = W_up,t,h^T q against the shared latent, the value sum kept in latent space."""
+    H, d = up_k.shape[1], q.shape[0]
+    sl = slice((t * H + h) * d, (t * H + h + 1) * d)
+    s = scale * (c_k @ (up_k[t, h].T @ q) + (0.0 if mu_k is None else q @ mu_k[sl]))
+    if cur_k is not None:
+        s = np.append(s, scale * (q @ cur_k))
+    p = np.exp(s - s.max())
+    L = c_k.shape[0]
+    o = up_v[t, h] @ (p[:L] @ c_v) + (0.0 if mu_v is None else p[:L].sum() * mu_v[sl])
+    if cur_k is not None:
+        o = o + p[L] * cur_v
+    return o / p.sum()
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+def test_decode_2d_equals_absorbed_formulation(pass1):
+    T, H, d, r_k, r_v, L = 4, 4, 32, 24, 40, 37
+    g = _rng(68)
+    up_k = g.standard_normal((T, H, d, r_k)) / math.sqrt(r_k)
+    up_v = g.standard_normal((T, H, d, r_v)) / math.sqrt(r_v)
+    mu_k, mu_v = g.standard_normal(T * H * d), g.standard_normal(T * H * d)
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    q = g.standard_normal((H, d))
+    cur_k = g.standard_normal((H, d)) if pass1 else None
+    cur_v = g.standard_normal((H, d)) if pass1 else None
+    scale = 1 / math.sqrt(d)
+    for t in range(T):
+        out = oracle.decode_2d(t, c_k, c_v, up_k, up_v, mu_k, mu_v, q, cur_k, cur_v, scale)
+        for h in range(H):
+            ref = _absorbed_2d(t, h, c_k, c_v, up_k, up_v, mu_k, mu_v, q[h],
+                               None if cur_k is None else cur_k[h],
+                               None if cur_v is None else cur_v[h], scale)
+            np.testing.assert_allclose(out[h], ref, rtol=0, atol=1e-12)
+
+
+def test_decode_2d_special_cases():
+    """One cached token in pass 2 returns its rebuilt value; pass 1 with an empty cache returns
+    the current value; a zero query averages the rebuilt values (uniform softmax)."""
+    T, H, d, r_k, r_v = 2, 3, 8, 6, 10
+    g = _rng(69)
+    up_k = g.standard_normal((T, H, d, r_k))
+    up_v = g.standard_normal((T, H, d, r_v))
+    mu_v = g.standard_normal(T * H * d)
+    c_k, c_v = g.standard_normal((5, r_k)), g.standard_normal((5, r_v))
+    q = g.standard_normal((H, d))
+    for t in range(T):
+        one = oracle.decode_2d(t, c_k[:1], c_v[:1], up_k, up_v, None, mu_v, q, None, None, 0.3)
+        zero = oracle.decode_2d(t, c_k, c_v, up_k, up_v, None, mu_v, np.zeros((H, d)), None,
+                                None, 0.3)
+        cv = g.standard_normal((H, d))
+        empty = oracle.decode_2d(t, c_k[:0], c_v[:0], up_k, up_v, None, mu_v, q,
+                                 g.standard_normal((H, d)), cv, 0.3)
+        for h in range(H):
+            sl = slice((t * H + h) * d, (t * H + h + 1) * d)
+            np.testing.assert_allclose(one[h], up_v[t, h] @ c_v[0] + mu_v[sl], rtol=0, atol=1e-12)
+            np.testing.assert_allclose(zero[h], up_v[t, h] @ c_v.mean(axis=0) + mu_v[sl],
+                                       rtol=0, atol=1e-12)
+        np.testing.assert_allclose(empty, cv, rtol=0, atol=0)
