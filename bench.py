@@ -381,6 +381,8 @@ def run_ours(args, rank, world, local_rank):
         del bench
         torch.cuda.empty_cache()
         result.update(run_extras(device))
+        torch.cuda.empty_cache()
+        result.update(run_2d_extra(device))
     return result
 
 
@@ -449,6 +451,70 @@ def run_loops_extra(bench):
         "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
         "bytes_per_launch": nbytes, "tokens_per_s_decode_only": bench.B / (ms / 1e3),
         "note": "the layer's latents cross HBM once for its T loop calls"}}
+
+
+def run_2d_extra(device):
+    """LLA-2D decode (Sec. 3, "The LLA-2D variant (loop x head)": one latent per (token, layer)
+    for all heads, read by the H absorbed queries of each sequence on the tensor cores) on the
+    stress workload's batch and contexts at the same cache budget, (r_k, r_v) = (288, 480),
+    rho_2D = 21.33: two layers' caches of random bf16 latents, cycled through 2 x T pass-1 calls
+    (every call has the shape and bytes of a call of the 48-layer model), and the same 2D shape on
+    the headline batch of 16 sequences."""
+    import torch
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+    peak, _ = measured_peaks()
+    out = {}
+    for name, wname, B in (("lla2d_decode", "stress2d_rho2133", None),
+                           ("lla2d_decode_b16", "stress2d_rho2133", 16)):
+        w = W.WORKLOADS[wname]
+        if B is not None:  # the headline batch's contexts with the 2D shape
+            lens = W.context_lengths(W.WORKLOADS["ouro14_rho4"])
+        else:
+            lens = W.context_lengths(w)
+        B = len(lens)
+        geom = lla.Geometry(w.T, w.H, w.d, w.r_k, w.r_v, "bf16")
+        pt = W.page_table(lens, w.seed, extra_tokens=1)
+        table = pt.block_table.to(device)
+        Nt = sum(lens)
+        layers = []
+        for l in range(2):
+            ck = W.normal((Nt, w.r_k), w.seed, 400, l, device=device)
+            cv = W.normal((Nt, w.r_v), w.seed, 401, l, device=device)
+            pool = W.pack_latent_pages(ck, cv, pt.block_table, lens, pt.num_blocks)
+            del ck, cv
+            codec = lla.Codec(**W.codec_tensors_2d(w.T, w.H, w.d, w.r_k, w.r_v, w.seed, l,
+                                                   device=device))
+            layers.append((pool, codec, lla.Cache(pool, pt.num_blocks, table, pt.max_blocks)))
+        shape = (2, w.T, B, w.H, w.d)
+        q = W.normal(shape, w.seed, 402, device=device)
+        ck = W.normal(shape, w.seed, 403, device=device)
+        cv = W.normal(shape, w.seed, 404, device=device)
+        o = torch.empty_like(q)
+        ctx = torch.tensor(lens, dtype=torch.int32, device=device)
+        ws = torch.empty(lla.lla_decode_2d_workspace_size(geom, B), dtype=torch.uint8, device=device)
+
+        def sweep():
+            for t in range(w.T):
+                for l in range(2):
+                    lla.lla_decode_attn_2d(geom, layers[l][1], layers[l][2], ctx, max(lens), t,
+                                           q[l, t], ck[l, t], cv[l, t], o[l, t], ws)
+        ms = _time_ms(sweep, reps=5, warm=2)
+        per_launch_s = ms / 1e3 / (2 * w.T)
+        nbytes = Nt * (w.r_k + w.r_v) * 2 + w.H * w.d * (w.r_k + w.r_v) * 2 + 4 * B * w.H * w.d * 2
+        if lla.lla_get_device_error() != 0:
+            raise RuntimeError("device error in the LLA-2D decode measurement")
+        out[name] = {
+            "workload": f"LLA-2D, H={w.H}, (r_k, r_v)=({w.r_k}, {w.r_v}), rho_2D={w.rho:.2f}, "
+                        f"B={B}, sum context {Nt}; 2 layers x {w.T} pass-1 calls",
+            "kernel": "absorb2d_kernel + attn2d_kernel + finish2d_kernel (lla_decode_attn_2d)",
+            "bound": "hbm", "avg_call_us": per_launch_s * 1e6,
+            "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
+            "bytes_per_call": nbytes,
+            "tokens_per_s_decode_only": B / (per_launch_s * w.D * w.T)}
+        del layers, q, ck, cv, o, ws
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_extras(device):

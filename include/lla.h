@@ -16,6 +16,8 @@
  *   lla_prefill_attn_rope  causal prefill with rotary positions after reconstruction
  *   lla_decode_attn_loops  the decode calls of all T loops in one pass over the latents
  *   lla_prefill_attn     causal pass-2 prefill attention over the latents of a prompt
+ *   lla_encode_2d, lla_decode_attn_2d
+ *                        the LLA-2D variant: one latent per (token, layer) for every head
  *   lla_dense_*          the uncompressed loop-t KV decode in the same kernel style (the
  *                        "teacher" column of Table absorbed_latency, App. J), for comparison
  *
@@ -256,6 +258,57 @@ lla_status lla_prefill_attn_rope(const lla_geometry *g, const lla_codec *codec,
                                  const int32_t *cu_seqlens, int32_t B, int32_t max_len,
                                  int32_t loop, const void *q, lla_dtype io_dtype, void *out,
                                  void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * LLA-2D (Sec. 3, "The LLA-2D variant (loop x head)"; App. J "Per-head LLA versus LLA-2D at
+ * inference").  One latent pair per (token, layer) serves all H heads.  A token's stacked
+ * vector runs over loops and heads, loop-major: x = [x_{1,1}; ...; x_{1,H}; x_{2,1}; ...;
+ * x_{T,H}] in R^{T H d}; c = (x - mu) W_down; head h at loop t is rebuilt as
+ * xhat_{t,h} = c W_up,t,h^T + mu_{t,h}.  rho_2D = 2 T H d / (r_k + r_v).
+ *
+ * The geometry is an lla_geometry whose r_k, r_v are the 2D ranks; the codec is an lla_codec with
+ *   w_down_k, w_down_v   [T*H*d][r_k | r_v] storage dtype (rows ordered (t, h, e)), 16-B aligned
+ *   w_up_k, w_up_v       [T][H][d][r_k | r_v] storage dtype, 16-B aligned
+ *   mu_k, mu_v           [T*H*d] fp32 or NULL
+ * and the cache an lla_cache with ONE page per block: pool [num_blocks][K-plane | V-plane], the
+ * planes laid out as in the per-head cache (the K-plane granule-interleaved, the V-plane
+ * row-major), lla_cache_2d_block_bytes bytes per block.
+ */
+
+/* Bytes of one LLA-2D cache block (one page of 64 tokens).  Host only. */
+lla_status lla_cache_2d_block_bytes(const lla_geometry *g, size_t *bytes);
+
+/*
+ * LLA-2D encode of N newly completed tokens of one layer into the cache.
+ *   x_k, x_v      device [T][N][H][d] in x_dtype, 16-byte aligned (pre-RoPE keys / values)
+ *   slot_mapping  device [N] int64 (negative: skip the token; past the pool: LLA_DEVERR_SLOT)
+ * fp32 accumulation, latents rounded to `storage`.  H * d <= 16384 (LLA_ERR_UNSUPPORTED beyond).
+ */
+lla_status lla_encode_2d(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                         const void *x_k, const void *x_v, lla_dtype x_dtype,
+                         const int64_t *slot_mapping, int32_t N, void *stream);
+
+/* Workspace bytes lla_decode_attn_2d needs for B sequences on the current device
+ * (LLA_ERR_UNSUPPORTED for a shape with no kernel). */
+lla_status lla_decode_2d_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes);
+
+/*
+ * One LLA-2D decode call (one layer, loop `loop`, B sequences, all heads), App. A two-pass
+ * decoder with App. J absorbed attention per head against the shared latent:
+ *   q~_h = W_up,t,h^K^T q_h,  s_hi = scale (q~_h . c_k,i + q_h . mu^K_{t,h}),
+ *   o_h = (W_up,t,h^V sum_i p_hi c_v,i + (sum_i p_hi) mu^V_{t,h} + p_h,cur v_cur,h) / sum p.
+ *   q, cur_k, cur_v, out  device [B][H][d] io_dtype (cur_k = cur_v = NULL: pass 2)
+ *   workspace             device, >= lla_decode_2d_workspace_size bytes; overwritten (no zero
+ *                         fill needed); calls that share it must be ordered (one stream)
+ * Other arguments and the error behaviour are those of lla_decode_attn.  Three launches on
+ * `stream`.  Storage LLA_BF16, d = 128, H <= 16, (r_k, r_v) one of (96, 160), (128, 128),
+ * (288, 480); LLA_ERR_UNSUPPORTED otherwise.
+ */
+lla_status lla_decode_attn_2d(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                              const int32_t *context_lens, int32_t B, int32_t max_ctx,
+                              int32_t loop, const void *q, const void *cur_k, const void *cur_v,
+                              lla_dtype io_dtype, void *out, void *workspace,
+                              size_t workspace_bytes, void *stream);
 
 /*
  * lla_decode_attn for callers that cannot allocate device memory (for example a plug-in inside a

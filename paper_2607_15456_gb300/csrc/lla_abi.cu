@@ -284,6 +284,97 @@ lla_status lla_decode_attn_loops(const lla_geometry *g, const lla_codec *codec,
                          out, workspace, workspace_bytes, stream, true, nullptr, true);
 }
 
+lla_status lla_cache_2d_block_bytes(const lla_geometry *g, size_t *bytes) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!bytes) return LLA_ERR_INVALID_ARG;
+    *bytes = head_page_bytes(g->r_k, g->r_v, elem_size(g->storage));  // one page per block
+    return LLA_OK;
+}
+
+lla_status lla_encode_2d(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                         const void *x_k, const void *x_v, lla_dtype x_dtype,
+                         const int64_t *slot_mapping, int32_t N, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!codec || !codec->w_down_k || !codec->w_down_v) return LLA_ERR_INVALID_ARG;
+    if ((st = check_cache(cache, false)) != LLA_OK) return st;
+    if (!valid_dtype(x_dtype) || N < 0) return LLA_ERR_INVALID_ARG;
+    if (N > 0 && (!x_k || !x_v || !slot_mapping)) return LLA_ERR_INVALID_ARG;
+    if (!aligned(codec->w_down_k, 16) || !aligned(codec->w_down_v, 16)) return LLA_ERR_INVALID_ARG;
+    if (N > 0 && (!aligned(x_k, 16) || !aligned(x_v, 16))) return LLA_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(g->H) * g->d > 16384) return LLA_ERR_UNSUPPORTED;
+    if (N == 0) return LLA_OK;
+    // The 2D stack [x_{1,1}; ...; x_{1,H}; ...; x_{T,H}] of a token is the per-head stack of one
+    // head of width H d: x [T][N][H][d] read as [T][N][1][H d], W_down [T H d][r], mu [T H d],
+    // and one page per block.
+    EncodeArgs a = {};
+    a.T = g->T; a.H = 1; a.d = g->H * g->d; a.r_k = g->r_k; a.r_v = g->r_v;
+    a.storage_bf16 = g->storage == LLA_BF16;
+    a.x_bf16 = x_dtype == LLA_BF16;
+    a.w_down_k = codec->w_down_k; a.w_down_v = codec->w_down_v;
+    a.mu_k = codec->mu_k; a.mu_v = codec->mu_v;
+    a.x_k = x_k; a.x_v = x_v;
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.slot_mapping = slot_mapping; a.N = N;
+    a.dense = 0;
+    return launch_encode(a, static_cast<cudaStream_t>(stream));
+}
+
+lla_status lla_decode_2d_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
+    if (!decode_2d_supported(elem_size(g->storage), g->d, g->H, g->r_k, g->r_v))
+        return LLA_ERR_UNSUPPORTED;
+    const size_t n = decode_2d_workspace_bytes(g->r_k, g->r_v, B);
+    if (n == 0) return LLA_ERR_CUDA;
+    *bytes = n;
+    return LLA_OK;
+}
+
+lla_status lla_decode_attn_2d(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                              const int32_t *context_lens, int32_t B, int32_t max_ctx,
+                              int32_t loop, const void *q, const void *cur_k, const void *cur_v,
+                              lla_dtype io_dtype, void *out, void *workspace,
+                              size_t workspace_bytes, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if ((st = check_cache(cache, true)) != LLA_OK) return st;
+    if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;
+    if (!aligned(codec->w_up_k, 16) || !aligned(codec->w_up_v, 16)) return LLA_ERR_INVALID_ARG;
+    if (loop < 0 || loop >= g->T) return LLA_ERR_INVALID_ARG;
+    if (B < 0 || B > LLA_MAX_BATCH || !valid_dtype(io_dtype)) return LLA_ERR_INVALID_ARG;
+    if (max_ctx < 0 || static_cast<int64_t>(max_ctx) >
+                           static_cast<int64_t>(cache->max_blocks_per_seq) * LLA_BLOCK_TOKENS)
+        return LLA_ERR_INVALID_ARG;
+    // the batch's pages are counted in 32 bits inside the kernels
+    if (static_cast<int64_t>(B) * ((static_cast<int64_t>(max_ctx) + LLA_BLOCK_TOKENS - 1) / LLA_BLOCK_TOKENS) >=
+        (int64_t(1) << 31))
+        return LLA_ERR_UNSUPPORTED;
+    if ((cur_k == nullptr) != (cur_v == nullptr)) return LLA_ERR_INVALID_ARG;
+    if (B > 0 && (!context_lens || !q || !out)) return LLA_ERR_INVALID_ARG;
+    if (!decode_2d_supported(elem_size(g->storage), g->d, g->H, g->r_k, g->r_v))
+        return LLA_ERR_UNSUPPORTED;
+    if (B == 0) return LLA_OK;
+    if (!workspace) return LLA_ERR_INVALID_ARG;
+    DecodeArgs a = {};
+    a.T = g->T; a.H = g->H; a.d = g->d; a.r_k = g->r_k; a.r_v = g->r_v;
+    a.loop = loop;
+    a.absorbed = 1;
+    a.storage_bf16 = 1;
+    a.io_bf16 = io_dtype == LLA_BF16;
+    a.scale = g->scale;
+    a.w_up_k = codec->w_up_k; a.w_up_v = codec->w_up_v;
+    a.mu_k = codec->mu_k; a.mu_v = codec->mu_v;
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.block_table = cache->block_table; a.max_blocks = cache->max_blocks_per_seq;
+    a.context_lens = context_lens; a.B = B; a.max_ctx = max_ctx;
+    a.q = q; a.cur_k = cur_k; a.cur_v = cur_v; a.out = out;
+    a.workspace = workspace; a.workspace_bytes = workspace_bytes;
+    return launch_decode_2d(a, static_cast<cudaStream_t>(stream));
+}
+
 lla_status lla_dense_decode_attn(const lla_geometry *g, const lla_cache *cache,
                                  const int32_t *context_lens, int32_t B, int32_t max_ctx,
                                  const void *q, const void *cur_k, const void *cur_v,

@@ -1,0 +1,829 @@
+// lla_decode_2d.cu -- decode over the LLA-2D cache (Sec. 3, "The LLA-2D variant (loop x head)";
+// App. J "Absorbed attention" and "Per-head LLA versus LLA-2D at inference").
+//
+// One latent pair per (token, layer) serves every head: head h at loop t rebuilds its key and
+// value as c W_up,t,h^T + mu_{t,h}.  Absorbed head by head (App. J), the H queries of a sequence
+// read the same latent, so each page of 64 tokens is a small dense contraction:
+//   q~_h = W_up,t,h^K^T q_h,  beta_h = q_h . mu^K_{t,h}                     (absorb kernel)
+//   S^T [64 x 32]   = C_k [64 x r_k] [Q~_hi; Q~_lo]^T     s_hi = scale (q~_h . c_k,i + beta_h)
+//   O^T [r_v x 16] += C_v^T [r_v x 64] P^T                online softmax over tokens per head
+//   o_h = (W_up,t,h^V o~_h + l_h mu^V_{t,h} + p_cur v_cur,h) / (l_h + p_cur)  (finish kernel)
+// Three launches on the caller's stream, chained by programmatic dependent launch:
+//   absorb2d_kernel   q~ (fp32, scaled into the exp2 domain) and beta of every (sequence, head),
+//                     the page prefix sums of the batch and the length checks
+//   attn2d_kernel     one CTA per SM.  The batch's pages, in sequence order, are split evenly
+//                     over the CTAs; a CTA takes its pages as runs (its part of one sequence)
+//                     and writes per run the partial (maximum, sum, O^T) of every head.
+//                       warp 0     producer: the K-plane of a page by one bulk copy, its V-plane
+//                                  by TMA boxes of 64 columns with 128-byte swizzle
+//                       warp 1     MMA issuer and TMEM owner: S^T (M = 64 tokens, N = 32: q~ as
+//                                  a bf16 high part and a bf16 remainder per head, so that the
+//                                  scores see q~ to about 16 significant bits; K = r_k) and O^T
+//                                  (M = 128 latent rows per chunk, N = 16 heads,
+//                                  K = 64 tokens; the swizzled V-plane is an MN-major A operand);
+//                                  the O^T product of a page is issued after the next page's
+//                                  S^T, so the softmax of one page overlaps the next page's scores
+//                       warps 2-5  per page: the scores of 16 tokens per warp, the maxima over
+//                                  the page per head, P^T as a bf16 operand, the lazy O^T rescale;
+//                                  per run: the partial out to the workspace
+//   finish2d_kernel   per (head, 8 sequences): merges the runs of each sequence, adds the pass-1
+//                     current token, and applies W_up,t,h^V once for the 8 sequences
+// Storage bf16, d = 128, H <= 16; accumulators fp32 in TMEM.
+#include <cuda_runtime.h>
+
+#include "lla_device.cuh"
+#include "lla_internal.h"
+#include "lla_tcgen05.cuh"
+#include "lla_tmap.h"
+
+namespace lla {
+namespace {
+
+constexpr int kPT = 64;          // tokens per page
+constexpr int kD = 128;          // head width
+constexpr int kNQ = 16;          // the heads of a sequence, padded
+constexpr int kNS = 2 * kNQ;     // score MMA N: q~ high parts, then remainders
+constexpr int kT2 = 192;         // threads of the attention kernel
+constexpr int kSm0 = 64;         // first softmax thread
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kRescaleLog2 = 8.f;  // rescale O^T only when a head's maximum grows by more
+constexpr int kSmemCap = 227 * 1024;
+constexpr int kFinishSeqs = 8;   // sequences per finish CTA
+constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one sequence fit one finish CTA)
+
+// Shared-memory plan of the attention kernel for ranks (RK, RV).  Offsets from a 1024-byte
+// aligned base (128-byte swizzle atoms of the V stages).
+template <int RK, int RV>
+struct Z2 {
+    static constexpr int NCH = (RV + 127) / 128;        // 128-row chunks of O^T
+    static constexpr int NBOX = (RV + 63) / 64;         // TMA boxes a V-plane loads
+    static constexpr int BOX = kPT * 128;               // one box: 64 rows x 128 bytes
+    static constexpr int KPAGE = kPT * RK * 2;
+    static constexpr int VPAGE = NCH * 2 * BOX;         // two boxes per chunk, loaded or zero
+    static constexpr int VBYTES = NBOX * BOX;
+    static constexpr int QB = kNS * RK * 2;             // [Q~_hi; Q~_lo] operand
+    static constexpr int PBUF = kPT * kNQ * 2;          // P^T operand (one of two)
+    static constexpr int RED = 1024;                    // maxima, sums, beta
+    static constexpr int NBAR = 32;
+    static constexpr int FIXED = QB + 2 * PBUF + RED + NBAR * 8;
+    static constexpr int ST0 = (kSmemCap - 1024 - FIXED) / (KPAGE + VPAGE);
+    static constexpr int ST = ST0 > 4 ? 4 : ST0;
+    static constexpr int oV = 0;
+    static constexpr int oK = oV + ST * VPAGE;
+    static constexpr int oQ = oK + ST * KPAGE;
+    static constexpr int oP = oQ + QB;
+    static constexpr int oRed = oP + 2 * PBUF;
+    static constexpr int oBar = oRed + RED;
+    static constexpr int SMEM = 1024 + oBar + NBAR * 8;
+    // TMEM columns: S^T double buffer [0, 64), O^T chunks [64, 64 + 16 NCH)
+    static constexpr uint32_t TM_S = 0, TM_O = 2 * kNS, TM_COLS = 128;
+    static constexpr uint32_t IDESC_S = umma_idesc_bf16(64, kNS, 0, 0);
+    static constexpr uint32_t IDESC_O = umma_idesc_bf16(128, kNQ, 1, 0);
+    static constexpr int PSTRIDE = kNQ * RV + 2 * kNQ;  // floats per run partial
+    static_assert(RK % 16 == 0 && RV % 32 == 0 && NCH <= 4, "ranks");
+    static_assert(ST >= 2, "pipeline depth");
+    static_assert(SMEM <= kSmemCap, "shared memory");
+    static_assert(TM_O + NCH * kNQ <= TM_COLS, "TMEM columns");
+};
+
+// barrier indices
+enum {
+    bKfull = 0 /* [4] */, bKempty = 4, bVfull = 8, bVempty = 12,
+    bSfull = 16 /* [2] */, bSfree = 18, bPfull = 20, bPfree = 22,
+    bOfree = 25, bQready = 26, bQfree = 27, bAbort = 28, bTslot = 29
+};
+
+struct A2Params {
+    int T, H, loop, io_bf16, pass1, B, max_ctx, max_blocks, rk;
+    float scale_log2;
+    const void *w_up_k;  // [T][H][d][r_k] bf16
+    const float *mu_k;   // [T*H*d] or NULL
+    const void *q;       // [B][H][d]
+    const int32_t *context_lens;
+    float *qt;           // [B][16][r_k]: q~ * scale * log2 e (rows >= H unused)
+    float *beta;         // [B][16]: beta * scale * log2 e
+    int *pstart;         // [B + 1]: first global page of each sequence
+    unsigned *err;
+};
+
+struct T2Params {
+    int H, B;
+    const char *pool;
+    int64_t num_blocks, page_bytes;
+    const int32_t *block_table;
+    int max_blocks;
+    const int32_t *context_lens;
+    const float *qt;
+    const float *beta;
+    const int *pstart;
+    float *part;  // [B + grid][PSTRIDE]: run (sequence b, CTA c) at slot b + c
+    unsigned *err;
+};
+
+struct F2Params {
+    int T, H, loop, io_bf16, B, grid;
+    float scale_log2;
+    const void *w_up_v;  // [T][H][d][r_v] bf16
+    const float *mu_v;   // [T*H*d] or NULL
+    const void *q, *cur_k, *cur_v;
+    void *out;
+    const int *pstart;
+    const float *part;
+};
+
+// CTA c of `grid` holds the global pages [page_lo(c), page_lo(c + 1)) of the np pages; with
+// fewer pages than CTAs some CTAs hold none.
+__host__ __device__ __forceinline__ int page_lo(int c, int np, int grid) {
+    return static_cast<int>(static_cast<int64_t>(c) * np / grid);
+}
+
+// The CTA that holds global page g (the last c with page_lo(c) <= g).
+__host__ __device__ __forceinline__ int cta_of(int g, int np, int grid) {
+    return static_cast<int>((static_cast<int64_t>(g + 1) * grid + np - 1) / np) - 1;
+}
+
+// ------------------------------------------------------------------------- absorb kernel
+
+// One CTA: the page prefix sums of the batch (B <= 1024) with the length checks; an invalid
+// length counts as an empty sequence.
+__device__ void page_prefix(const A2Params &p) {
+    __shared__ int wsum[8];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    int cnt[4], tot = 0;
+    const int limit = min(p.max_ctx, p.max_blocks * kPT);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int b = tid * 4 + k;
+        int c = 0;
+        if (b < p.B) {
+            const int L = p.context_lens[b];
+            if (L < 0 || L > limit) {
+                atomicOr(p.err, LLA_DEVERR_CONTEXT);
+            } else {
+                if (!p.pass1 && L == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
+                c = (L + kPT - 1) / kPT;
+            }
+        }
+        cnt[k] = c;
+        tot += c;
+    }
+    int x = tot;  // inclusive scan over the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) wsum[warp] = x;
+    __syncthreads();
+    int pre = 0;
+    for (int w = 0; w < warp; ++w) pre += wsum[w];
+    int ex = pre + x - tot;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int b = tid * 4 + k;
+        if (b < p.B) p.pstart[b] = ex;
+        ex += cnt[k];
+    }
+    if (tid == blockDim.x - 1) p.pstart[p.B] = pre + x;
+}
+
+// Grid (H, ceil(B / 16)), 256 threads: q~ and beta of head h for 16 sequences.
+template <int RK>
+__global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
+    __shared__ float qs[16][kD];
+    const int h = blockIdx.x, b0 = blockIdx.y * 16, tid = threadIdx.x;
+    const int nb = min(16, p.B - b0);
+    pdl_wait();  // the workspace is free once the previous call has finished
+    if (blockIdx.x == 0 && blockIdx.y == 0) page_prefix(p);
+    for (int i = tid; i < 16 * kD; i += 256) {
+        const int bi = i >> 7, e = i & (kD - 1);
+        qs[bi][e] = bi < nb ? load_elem(p.q, (static_cast<int64_t>(b0 + bi) * p.H + h) * kD + e, p.io_bf16)
+                            : 0.f;
+    }
+    __syncthreads();
+    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
+    const uint16_t *W = static_cast<const uint16_t *>(p.w_up_k) + th * kD * RK;
+    for (int j = tid; j < RK; j += 256) {
+        float acc[16];
+#pragma unroll
+        for (int bi = 0; bi < 16; ++bi) acc[bi] = 0.f;
+#pragma unroll 4
+        for (int e = 0; e < kD; ++e) {
+            const float w = bf_to_f(W[e * RK + j]);
+#pragma unroll
+            for (int bi = 0; bi < 16; ++bi) acc[bi] = fmaf(w, qs[bi][e], acc[bi]);
+        }
+#pragma unroll
+        for (int bi = 0; bi < 16; ++bi)
+            if (bi < nb) p.qt[(static_cast<int64_t>(b0 + bi) * kNQ + h) * RK + j] = acc[bi] * p.scale_log2;
+    }
+    // beta_h = q_h . mu^K_{t,h}: warp w takes sequences w and w + 8
+    const int warp = tid >> 5, lane = tid & 31;
+    for (int bi = warp; bi < nb; bi += 8) {
+        float s = 0.f;
+        if (p.mu_k)
+            for (int e = lane; e < kD; e += 32) s = fmaf(qs[bi][e], p.mu_k[th * kD + e], s);
+        s = warp_sum(s);
+        if (lane == 0) p.beta[static_cast<int64_t>(b0 + bi) * kNQ + h] = s * p.scale_log2;
+    }
+    __syncthreads();
+    pdl_trigger();
+}
+
+// ------------------------------------------------------------------------- attention kernel
+
+// First sequence with pages at or after global page g0: the last b with pstart[b] <= g0.
+__device__ __forceinline__ int first_seq(const int *pstart, int B, int g0) {
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (pstart[mid] <= g0) lo = mid;
+        else hi = mid - 1;
+    }
+    return lo;
+}
+
+template <int RK, int RV>
+__global__ void __launch_bounds__(kT2, 1)
+    attn2d_kernel(const __grid_constant__ CUtensorMap tv, const T2Params p) {
+    using Z = Z2<RK, RV>;
+    extern __shared__ __align__(1024) char sm_raw[];
+    char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + Z::oBar);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar + bAbort);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + bTslot);
+    float *red = reinterpret_cast<float *>(sm + Z::oRed);  // [2 pages][4 warps][16] maxima
+    float *lsum = red + 128;                                // [4 warps][16] run sums
+    float *betas = lsum + 64;                               // [16]
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int G = gridDim.x, c = blockIdx.x;
+
+    if (tid == 0) {
+        for (int s = 0; s < Z::ST; ++s) {
+            mbar_init(&bar[bKfull + s], 1);
+            mbar_init(&bar[bKempty + s], 1);
+            mbar_init(&bar[bVfull + s], 1);
+            mbar_init(&bar[bVempty + s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&bar[bSfull + s], 1);
+            mbar_init(&bar[bSfree + s], 128);
+            mbar_init(&bar[bPfull + s], 128);
+            mbar_init(&bar[bPfree + s], 1);
+        }
+        mbar_init(&bar[bOfree], 128);
+        mbar_init(&bar[bQready], 128);
+        mbar_init(&bar[bQfree], 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) tmem_alloc(tslot, Z::TM_COLS);
+    // V boxes that no load writes (the second box of a last chunk past r_v) stay zero
+    if constexpr (Z::NCH * 2 > Z::NBOX) {
+        for (int s = 0; s < Z::ST; ++s)
+            for (int a = Z::NBOX; a < Z::NCH * 2; ++a)
+                for (int i = tid; i < Z::BOX / 16; i += kT2)
+                    reinterpret_cast<uint4 *>(sm + Z::oV + s * Z::VPAGE + a * Z::BOX)[i] = make_uint4(0, 0, 0, 0);
+        fence_proxy_async_smem();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+    pdl_wait();  // q~, beta and the page prefix sums come from the absorb kernel
+
+    const int NP = p.pstart[p.B];
+    const int g0 = page_lo(c, NP, G), g1 = page_lo(c + 1, NP, G);
+    const int bfirst = g0 < g1 ? first_seq(p.pstart, p.B, g0) : p.B;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------------------- producer
+        if (lane == 0) {
+            const uint64_t pol = policy_evict_first();
+            int it = 0;
+            for (int b = bfirst; b < p.B; ++b) {
+                const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+                if (s0 >= g1) break;
+                const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
+                const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks;
+                for (int pg = pa; pg < pe; ++pg, ++it) {
+                    const int st = it % Z::ST;
+                    const uint32_t ph = (it / Z::ST) & 1;
+                    int32_t blk = bt[pg];
+                    if (blk < 0 || blk >= p.num_blocks) {
+                        atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                        blk = 0;
+                    }
+                    mbar_wait(&bar[bKempty + st], ph ^ 1u, abort_flag, p.err);
+                    mbar_arrive_expect_tx(&bar[bKfull + st], Z::KPAGE);
+                    bulk_g2s(sm + Z::oK + st * Z::KPAGE, p.pool + blk * p.page_bytes, Z::KPAGE,
+                             &bar[bKfull + st], pol);
+                    mbar_wait(&bar[bVempty + st], ph ^ 1u, abort_flag, p.err);
+                    mbar_arrive_expect_tx(&bar[bVfull + st], Z::VBYTES);
+                    char *vs = sm + Z::oV + st * Z::VPAGE;
+#pragma unroll
+                    for (int a = 0; a < Z::NBOX; ++a)
+                        tma_load_3d(vs + a * Z::BOX, &tv, a * 64, 0, blk, &bar[bVfull + st]);
+                }
+            }
+            // every copy has landed before the CTA can exit, even after an abort
+            volatile int never = 0;
+            for (int j = max(0, it - Z::ST); j < it; ++j) {
+                mbar_wait(&bar[bKfull + j % Z::ST], (j / Z::ST) & 1, &never, p.err);
+                mbar_wait(&bar[bVfull + j % Z::ST], (j / Z::ST) & 1, &never, p.err);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t base = smem_addr(sm);
+            const uint64_t dq = umma_desc(base + Z::oQ, kNS * 16, 128);
+            const uint64_t dk0 = umma_desc(base + Z::oK, kPT * 16, 128);
+            const uint64_t dp0 = umma_desc(base + Z::oP, kNQ * 16, 128);
+            const uint64_t dv0 = umma_desc_sw128_mn(base + Z::oV, Z::BOX);
+            int it = 0, r = 0;
+            // O^T += C_v^T P^T for page j (first: the first page of run rr zeroes O^T)
+            auto issue_pv = [&](int j, bool first, int rr) {
+                const int s = j & 1, st = j % Z::ST;
+                mbar_wait(&bar[bPfull + s], (j >> 1) & 1, abort_flag, p.err);
+                mbar_wait(&bar[bVfull + st], (j / Z::ST) & 1, abort_flag, p.err);
+                if (first && rr > 0) mbar_wait(&bar[bOfree], (rr - 1) & 1, abort_flag, p.err);
+                tc_fence_after();
+                const uint64_t dv = dv0 + static_cast<uint64_t>((st * Z::VPAGE) >> 4);
+                const uint64_t dp = dp0 + static_cast<uint64_t>((s * Z::PBUF) >> 4);
+#pragma unroll
+                for (int ch = 0; ch < Z::NCH; ++ch)
+#pragma unroll
+                    for (int ks = 0; ks < kPT / 16; ++ks)
+                        umma_bf16(tmem + Z::TM_O + ch * kNQ, dv + ((ch * 2 * Z::BOX + ks * 2048) >> 4),
+                                  dp + ks * ((2 * kNQ * 16) >> 4), Z::IDESC_O, !first || ks > 0);
+                umma_commit(&bar[bVempty + st]);
+                umma_commit(&bar[bPfree + s]);  // also: O^T holds pages up to j
+            };
+            for (int b = bfirst; b < p.B; ++b) {
+                const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+                if (s0 >= g1) break;
+                const int n = min(g1, s1) - max(g0, s0);
+                if (n <= 0) continue;
+                mbar_wait(&bar[bQready], r & 1, abort_flag, p.err);
+                tc_fence_after();
+                for (int k = 0; k < n; ++k, ++it) {
+                    const int s = it & 1, st = it % Z::ST;
+                    mbar_wait(&bar[bKfull + st], (it / Z::ST) & 1, abort_flag, p.err);
+                    if (it >= 2) mbar_wait(&bar[bSfree + s], ((it - 2) >> 1) & 1, abort_flag, p.err);
+                    tc_fence_after();
+                    const uint64_t dk = dk0 + static_cast<uint64_t>((st * Z::KPAGE) >> 4);
+#pragma unroll
+                    for (int ks = 0; ks < RK / 16; ++ks)
+                        umma_bf16(tmem + Z::TM_S + s * kNS, dk + ks * ((2 * kPT * 16) >> 4),
+                                  dq + ks * ((2 * kNS * 16) >> 4), Z::IDESC_S, ks > 0);
+                    umma_commit(&bar[bSfull + s]);
+                    umma_commit(&bar[bKempty + st]);
+                    if (k == n - 1) umma_commit(&bar[bQfree]);
+                    if (k > 0) issue_pv(it - 1, k == 1, r);
+                }
+                issue_pv(it - 1, n == 1, r);
+                ++r;
+            }
+            // every MMA has completed before TMEM is released, even after an abort (the last
+            // product's completion on its P buffer; the one before on the other buffer had
+            // completed before the softmax released the last page)
+            if (it > 0) {
+                volatile int never = 0;
+                mbar_wait(&bar[bPfree + ((it - 1) & 1)], ((it - 1) >> 1) & 1, &never, p.err);
+            }
+        }
+        __syncwarp();
+    } else {
+        // --------------------------------------------------------------- softmax warps 2-5
+        const int q4 = warp & 3;  // TMEM lane quarter
+        const uint32_t tl = tmem + (static_cast<uint32_t>(32 * q4) << 16);
+        const int st_tid = tid - kSm0;
+        const int tok = 16 * q4 + lane;  // the token of this lane in the M = 64 layout (lane < 16)
+        int it = 0, r = 0;
+        for (int b = bfirst; b < p.B; ++b) {
+            const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+            if (s0 >= g1) break;
+            const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
+            if (pe <= pa) continue;
+            const int L = p.context_lens[b];
+            // q~ of the sequence as a K-major operand of 32 rows: row n = bf16(q~_n), row 16 + n =
+            // bf16(q~_n - row n), granule g of row n at g*512 + n*16; and beta
+            if (r > 0) mbar_wait(&bar[bQfree], (r - 1) & 1, abort_flag, p.err);
+            {
+                const float4 *src = reinterpret_cast<const float4 *>(p.qt + static_cast<int64_t>(b) * kNQ * RK);
+                for (int i = st_tid; i < kNQ * (RK / 8); i += 128) {
+                    const int n = i / (RK / 8), g = i - n * (RK / 8);
+                    uint4 hi = make_uint4(0, 0, 0, 0), lo = hi;
+                    if (n < p.H) {
+                        const float4 a = src[2 * i], c4 = src[2 * i + 1];
+                        const float v[8] = {a.x, a.y, a.z, a.w, c4.x, c4.y, c4.z, c4.w};
+                        float r8[8];
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) r8[u] = v[u] - __bfloat162float(__float2bfloat16_rn(v[u]));
+                        hi = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                        pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+                        lo = make_uint4(pack_bf16x2(r8[0], r8[1]), pack_bf16x2(r8[2], r8[3]),
+                                        pack_bf16x2(r8[4], r8[5]), pack_bf16x2(r8[6], r8[7]));
+                    }
+                    char *dq = sm + Z::oQ + g * (kNS * 16);
+                    *reinterpret_cast<uint4 *>(dq + n * 16) = hi;
+                    *reinterpret_cast<uint4 *>(dq + (kNQ + n) * 16) = lo;
+                }
+                if (st_tid < kNQ) betas[st_tid] = st_tid < p.H ? p.beta[static_cast<int64_t>(b) * kNQ + st_tid] : 0.f;
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(&bar[bQready]);
+            named_bar_sync(1, 128);  // beta is visible
+            float m[kNQ], acc[kNQ];
+#pragma unroll
+            for (int n = 0; n < kNQ; ++n) {
+                m[n] = -INFINITY;
+                acc[n] = 0.f;
+            }
+            const int nps = pe - pa;
+            for (int k = 0; k < nps; ++k, ++it) {
+                const int s = it & 1, st = it % Z::ST;
+                const int tok0 = (pa + k) * kPT;
+                mbar_wait(&bar[bSfull + s], (it >> 1) & 1, abort_flag, p.err);
+                tc_fence_after();
+                float x2[kNS], x[kNQ];
+                tmem_ld32(tl + Z::TM_S + s * kNS, x2);
+                tc_fence_before();
+                mbar_arrive(&bar[bSfree + s]);
+                const bool valid = lane < 16 && tok0 + tok < L;
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) x[n] = valid ? (x2[n] + x2[kNQ + n]) + betas[n] : -INFINITY;
+                // per-head maxima over the page: 16 tokens per warp, then the 4 warps
+                float mx[kNQ];
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) mx[n] = x[n];
+#pragma unroll
+                for (int o = 8; o >= 1; o >>= 1)
+#pragma unroll
+                    for (int n = 0; n < kNQ; ++n) mx[n] = fmaxf(mx[n], __shfl_xor_sync(0xffffffffu, mx[n], o));
+                float *rp = red + s * 64;
+                if (lane == 0) {
+#pragma unroll
+                    for (int n = 0; n < kNQ; n += 4)
+                        *reinterpret_cast<float4 *>(rp + q4 * 16 + n) = make_float4(mx[n], mx[n + 1], mx[n + 2], mx[n + 3]);
+                }
+                named_bar_sync(1, 128);
+                bool any = false;
+                float f[kNQ];
+#pragma unroll
+                for (int n = 0; n < kNQ; n += 4) {
+                    float4 a = *reinterpret_cast<const float4 *>(rp + n);
+#pragma unroll
+                    for (int w = 1; w < 4; ++w) {
+                        const float4 bb = *reinterpret_cast<const float4 *>(rp + w * 16 + n);
+                        a = make_float4(fmaxf(a.x, bb.x), fmaxf(a.y, bb.y), fmaxf(a.z, bb.z), fmaxf(a.w, bb.w));
+                    }
+                    const float pm[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const float mn = fmaxf(m[n + u], pm[u]);
+                        const bool need = mn > m[n + u] + kRescaleLog2;  // also the first page
+                        f[n + u] = need ? ex2_approx(m[n + u] - mn) : 1.f;
+                        if (need) {
+                            acc[n + u] *= f[n + u];
+                            m[n + u] = mn;
+                            any = true;
+                        }
+                    }
+                }
+                if (any && k > 0) {
+                    // O^T holds pages up to it - 1 of this run (the product of page it - 1 has
+                    // released its P buffer; the one of page it - 2 had released the other before
+                    // this warp wrote page it - 1, so the parity test cannot pass a phase early):
+                    // scale head n's column by f[n]
+                    mbar_wait(&bar[bPfree + ((it - 1) & 1)], ((it - 1) >> 1) & 1, abort_flag, p.err);
+                    tc_fence_after();
+#pragma unroll
+                    for (int ch = 0; ch < Z::NCH; ++ch) {
+                        float o[kNQ];
+                        tmem_ld16(tl + Z::TM_O + ch * kNQ, o);
+#pragma unroll
+                        for (int n = 0; n < kNQ; ++n) o[n] *= f[n];
+                        tmem_st16(tl + Z::TM_O + ch * kNQ, o);
+                    }
+                }
+                float pv[kNQ];
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) {
+                    pv[n] = ex2_approx(x[n] - m[n]);
+                    acc[n] += pv[n];
+                }
+                if (it >= 2) mbar_wait(&bar[bPfree + s], ((it - 2) >> 1) & 1, abort_flag, p.err);
+                if (lane < 16) {
+                    // P^T as a K-major operand: head n, tokens 8g .. 8g + 7 at g*256 + n*16
+                    char *pp = sm + Z::oP + s * Z::PBUF + (tok >> 3) * (kNQ * 16) + (tok & 7) * 2;
+#pragma unroll
+                    for (int n = 0; n < kNQ; ++n)
+                        *reinterpret_cast<uint16_t *>(pp + n * 16) = __bfloat16_as_ushort(__float2bfloat16_rn(pv[n]));
+                }
+                if (k == nps - 1 && tok0 + kPT > L) {
+                    // V rows past the sequence hold no latents: zero them (0 * NaN would poison O)
+                    mbar_wait(&bar[bVfull + st], (it / Z::ST) & 1, abort_flag, p.err);
+                    char *vs = sm + Z::oV + st * Z::VPAGE;
+                    const int nv = L - tok0;
+                    const int nz = (kPT - nv) * Z::NBOX * 8;
+                    for (int w = st_tid; w < nz; w += 128) {
+                        const int cc = w & 7, r2 = w >> 3;
+                        const int a = r2 % Z::NBOX, row = nv + r2 / Z::NBOX;
+                        *reinterpret_cast<uint4 *>(vs + a * Z::BOX + row * 128 + cc * 16) = make_uint4(0, 0, 0, 0);
+                    }
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                mbar_arrive(&bar[bPfull + s]);
+            }
+            // the run's partial: maxima, sums over its tokens, and O^T (complete once the last
+            // page's product has released its P buffer)
+            mbar_wait(&bar[bPfree + ((it - 1) & 1)], ((it - 1) >> 1) & 1, abort_flag, p.err);
+            tc_fence_after();
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1)
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) acc[n] += __shfl_xor_sync(0xffffffffu, acc[n], o);
+            if (lane == 0) {
+#pragma unroll
+                for (int n = 0; n < kNQ; n += 4)
+                    *reinterpret_cast<float4 *>(lsum + q4 * 16 + n) = make_float4(acc[n], acc[n + 1], acc[n + 2], acc[n + 3]);
+            }
+            float *dst = p.part + static_cast<int64_t>(b + c) * Z::PSTRIDE;
+#pragma unroll
+            for (int ch = 0; ch < Z::NCH; ++ch) {
+                float o[kNQ];
+                tmem_ld16(tl + Z::TM_O + ch * kNQ, o);
+                const int j = ch * 128 + 32 * q4 + lane;
+                if (j < RV) {
+#pragma unroll
+                    for (int n = 0; n < kNQ; ++n)
+                        if (n < p.H) dst[n * RV + j] = o[n];
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&bar[bOfree]);
+            named_bar_sync(1, 128);  // the run sums are visible
+            if (st_tid < kNQ) {
+                float mine = 0.f;
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n)
+                    if (st_tid == n) mine = m[n];
+                dst[kNQ * RV + st_tid] = mine;
+                dst[kNQ * RV + kNQ + st_tid] = (lsum[st_tid] + lsum[16 + st_tid]) + (lsum[32 + st_tid] + lsum[48 + st_tid]);
+            }
+            named_bar_sync(1, 128);  // lsum and red are free for the next run
+            ++r;
+        }
+    }
+    pdl_trigger();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, Z::TM_COLS);
+    }
+}
+
+// ------------------------------------------------------------------------- finish kernel
+
+// Grid (H, ceil(B / 8)), 128 threads (thread e = output element e of head h).
+template <int RV>
+__global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
+    constexpr int PS = kNQ * RV + 2 * kNQ;
+    __shared__ __align__(16) float ob[kFinishSeqs][RV];
+    __shared__ float wts[kMaxGrid];
+    __shared__ float coef[kFinishSeqs][3];
+    __shared__ float redm[4], reds[4];
+    const int h = blockIdx.x, b0 = blockIdx.y * kFinishSeqs, tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int nb = min(kFinishSeqs, p.B - b0);
+    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
+    pdl_wait();
+    const int NP = p.pstart[p.B];
+    for (int bi = 0; bi < kFinishSeqs; ++bi) {
+        if (bi >= nb) {
+            for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
+            continue;
+        }
+        const int b = b0 + bi;
+        const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+        float M = -INFINITY, l = 0.f;
+        if (s1 > s0) {
+            // the runs of sequence b: the CTAs c0 .. c1 that hold pages (a CTA between them may
+            // hold none and writes nothing), partials at slots b + c
+            const int c0 = cta_of(s0, NP, p.grid), c1 = cta_of(s1 - 1, NP, p.grid);
+            const int nr = c1 - c0 + 1;
+            float mm = -INFINITY;
+            for (int i = tid; i < nr; i += 128)
+                if (page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid))
+                    mm = fmaxf(mm, p.part[static_cast<int64_t>(b + c0 + i) * PS + kNQ * RV + h]);
+            mm = warp_max(mm);
+            if (lane == 0) redm[warp] = mm;
+            __syncthreads();
+            M = fmaxf(fmaxf(redm[0], redm[1]), fmaxf(redm[2], redm[3]));
+            float ls = 0.f;
+            for (int i = tid; i < nr; i += 128) {
+                float w = 0.f;  // no run: weight 0, and its slot is never read
+                if (page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid)) {
+                    const float *pr = p.part + static_cast<int64_t>(b + c0 + i) * PS + kNQ * RV;
+                    w = ex2_approx(pr[h] - M);
+                    ls = fmaf(w, pr[kNQ + h], ls);
+                }
+                wts[i] = w;
+            }
+            ls = warp_sum(ls);
+            if (lane == 0) reds[warp] = ls;
+            __syncthreads();
+            l = (reds[0] + reds[1]) + (reds[2] + reds[3]);
+            for (int j = tid; j < RV; j += 128) {
+                float a = 0.f;
+                for (int i = 0; i < nr; ++i)
+                    if (wts[i] > 0.f) a = fmaf(wts[i], p.part[static_cast<int64_t>(b + c0 + i) * PS + h * RV + j], a);
+                ob[bi][j] = a;
+            }
+        } else {
+            for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
+        }
+        // pass 1: the current token's score against its exact key
+        float sc = -INFINITY;
+        if (p.cur_k) {
+            const int64_t row = (static_cast<int64_t>(b) * p.H + h) * kD;
+            float v = load_elem(p.q, row + tid, p.io_bf16) * load_elem(p.cur_k, row + tid, p.io_bf16);
+            v = warp_sum(v);
+            __syncthreads();  // redm / reds are free
+            if (lane == 0) reds[warp] = v;
+            __syncthreads();
+            sc = ((reds[0] + reds[1]) + (reds[2] + reds[3])) * p.scale_log2;
+        }
+        if (tid == 0) {
+            const float Mx = fmaxf(M, sc);
+            const float al = M == -INFINITY ? 0.f : ex2_approx(M - Mx);
+            const float pc = p.cur_k ? ex2_approx(sc - Mx) : 0.f;
+            const float den = al * l + pc;
+            const float inv = den > 0.f ? 1.f / den : 0.f;
+            coef[bi][0] = al * inv;
+            coef[bi][1] = al * l * inv;
+            coef[bi][2] = pc * inv;
+        }
+        __syncthreads();  // redm, reds and wts are free for the next sequence
+    }
+    // out_b[e] = coef0 (W_up,t,h^V o~_b)[e] + coef1 mu^V[e] + coef2 v_cur,b[e]
+    const int e = tid;
+    const uint4 *W = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.w_up_v) + (th * kD + e) * RV);
+    float acc[kFinishSeqs];
+#pragma unroll
+    for (int bi = 0; bi < kFinishSeqs; ++bi) acc[bi] = 0.f;
+#pragma unroll 2
+    for (int j8 = 0; j8 < RV / 8; ++j8) {
+        const uint4 w4 = W[j8];
+        const float2 w0 = bf2_to_f2(w4.x), w1 = bf2_to_f2(w4.y), w2 = bf2_to_f2(w4.z), w3 = bf2_to_f2(w4.w);
+#pragma unroll
+        for (int bi = 0; bi < kFinishSeqs; ++bi) {
+            const float4 o0 = *reinterpret_cast<const float4 *>(&ob[bi][j8 * 8]);
+            const float4 o1 = *reinterpret_cast<const float4 *>(&ob[bi][j8 * 8 + 4]);
+            float a = acc[bi];
+            a = fmaf(w0.x, o0.x, a); a = fmaf(w0.y, o0.y, a); a = fmaf(w1.x, o0.z, a); a = fmaf(w1.y, o0.w, a);
+            a = fmaf(w2.x, o1.x, a); a = fmaf(w2.y, o1.y, a); a = fmaf(w3.x, o1.z, a); a = fmaf(w3.y, o1.w, a);
+            acc[bi] = a;
+        }
+    }
+    const float muv = p.mu_v ? p.mu_v[th * kD + e] : 0.f;
+#pragma unroll
+    for (int bi = 0; bi < kFinishSeqs; ++bi) {
+        if (bi >= nb) break;
+        const int64_t idx = (static_cast<int64_t>(b0 + bi) * p.H + h) * kD + e;
+        float v = acc[bi] * coef[bi][0] + coef[bi][1] * muv;
+        if (p.cur_v) v = fmaf(coef[bi][2], load_elem(p.cur_v, idx, p.io_bf16), v);
+        store_elem(p.out, idx, v, p.io_bf16);
+    }
+    __syncthreads();
+    pdl_trigger();
+}
+
+// ------------------------------------------------------------------------- host side
+
+template <typename K, typename... Args>
+lla_status launch_ex(K kern, dim3 grid, int threads, int smem, cudaStream_t stream, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, kern, args...) != cudaSuccess) return LLA_ERR_CUDA;
+    return LLA_OK;
+}
+
+struct WS2 {
+    size_t part, qt, beta, pstart, total;
+};
+
+inline size_t al256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+WS2 ws2_layout(int r_k, int r_v, int B, int grid) {
+    WS2 w;
+    w.part = 0;
+    w.qt = al256(static_cast<size_t>(B + grid) * (kNQ * r_v + 2 * kNQ) * sizeof(float));
+    w.beta = w.qt + al256(static_cast<size_t>(B) * kNQ * r_k * sizeof(float));
+    w.pstart = w.beta + al256(static_cast<size_t>(B) * kNQ * sizeof(float));
+    w.total = w.pstart + al256(static_cast<size_t>(B + 1) * sizeof(int));
+    return w;
+}
+
+template <int RK, int RV>
+lla_status launch_2d(const DecodeArgs &a, cudaStream_t stream) {
+    using Z = Z2<RK, RV>;
+    lla_status st = LLA_OK;
+    unsigned *err = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    const int grid = num_sms();
+    if (grid <= 0 || grid > kMaxGrid) return LLA_ERR_UNSUPPORTED;
+    const WS2 w = ws2_layout(RK, RV, a.B, grid);
+    if (a.workspace_bytes < w.total) return LLA_ERR_WORKSPACE;
+    char *ws = static_cast<char *>(a.workspace);
+    static bool configured[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
+    if (dev < 64 && !configured[dev]) {
+        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
+            cudaSuccess)
+            return LLA_ERR_CUDA;
+        configured[dev] = true;
+    }
+    const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
+    // the V-planes of every page: [num_blocks][64 tokens][r_v] bf16
+    CUtensorMap tv;
+    const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT),
+                              static_cast<uint64_t>(a.num_blocks)};
+    const uint64_t strides[2] = {static_cast<uint64_t>(RV) * 2, static_cast<uint64_t>(page_bytes)};
+    const uint32_t box[3] = {64, kPT, 1};
+    if (!encode_tmap_bf16(&tv, static_cast<const char *>(a.pool) + kPT * RK * 2, 3, dims, strides, box, true))
+        return LLA_ERR_CUDA;
+
+    A2Params ap = {};
+    ap.T = a.T; ap.H = a.H; ap.loop = a.loop; ap.io_bf16 = a.io_bf16; ap.pass1 = a.cur_k != nullptr;
+    ap.B = a.B; ap.max_ctx = a.max_ctx; ap.max_blocks = a.max_blocks; ap.rk = RK;
+    ap.scale_log2 = a.scale * kLog2e;
+    ap.w_up_k = a.w_up_k; ap.mu_k = a.mu_k; ap.q = a.q; ap.context_lens = a.context_lens;
+    ap.qt = reinterpret_cast<float *>(ws + w.qt);
+    ap.beta = reinterpret_cast<float *>(ws + w.beta);
+    ap.pstart = reinterpret_cast<int *>(ws + w.pstart);
+    ap.err = err;
+    if ((st = launch_ex(absorb2d_kernel<RK>, dim3(a.H, (a.B + 15) / 16), 256, 0, stream, ap)) != LLA_OK)
+        return st;
+
+    T2Params tp = {};
+    tp.H = a.H; tp.B = a.B;
+    tp.pool = static_cast<const char *>(a.pool);
+    tp.num_blocks = a.num_blocks; tp.page_bytes = page_bytes;
+    tp.block_table = a.block_table; tp.max_blocks = a.max_blocks;
+    tp.context_lens = a.context_lens;
+    tp.qt = ap.qt; tp.beta = ap.beta; tp.pstart = ap.pstart;
+    tp.part = reinterpret_cast<float *>(ws + w.part);
+    tp.err = err;
+    if ((st = launch_ex(attn2d_kernel<RK, RV>, dim3(grid), kT2, Z::SMEM, stream, tv, tp)) != LLA_OK)
+        return st;
+
+    F2Params fp = {};
+    fp.T = a.T; fp.H = a.H; fp.loop = a.loop; fp.io_bf16 = a.io_bf16; fp.B = a.B; fp.grid = grid;
+    fp.scale_log2 = ap.scale_log2;
+    fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
+    fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
+    fp.pstart = ap.pstart; fp.part = tp.part;
+    return launch_ex(finish2d_kernel<RV>, dim3(a.H, (a.B + kFinishSeqs - 1) / kFinishSeqs), 128, 0, stream, fp);
+}
+
+}  // namespace
+
+bool decode_2d_supported(int es, int d, int H, int r_k, int r_v) {
+    return es == 2 && d == kD && H >= 1 && H <= kNQ &&
+           ((r_k == 96 && r_v == 160) || (r_k == 128 && r_v == 128) || (r_k == 288 && r_v == 480));
+}
+
+size_t decode_2d_workspace_bytes(int r_k, int r_v, int B) {
+    const int grid = num_sms();
+    if (grid <= 0) return 0;
+    return ws2_layout(r_k, r_v, B, grid).total;
+}
+
+lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream) {
+    if (a.B == 0) return LLA_OK;
+    if (a.num_blocks >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // 32-bit TMA coordinate
+#define LLA_2D(K, V) \
+    if (a.r_k == K && a.r_v == V) return launch_2d<K, V>(a, stream);
+    LLA_2D(96, 160)
+    LLA_2D(128, 128)
+    LLA_2D(288, 480)
+#undef LLA_2D
+    return LLA_ERR_UNSUPPORTED;
+}
+
+}  // namespace lla

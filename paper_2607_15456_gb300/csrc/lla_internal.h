@@ -96,6 +96,12 @@ bool prefill_rope_supported(int es, int d, int r_k, int r_v);
 lla_status launch_prefill_rope(const PrefillArgs &a, double base, int pairing, void *workspace,
                                size_t workspace_bytes, cudaStream_t stream);
 
+// LLA-2D decode (one latent per token and layer; w_up_* [T][H][d][r], mu_* [T*H*d]): the
+// shapes with a kernel, the workspace for B sequences (0 if the device is unknown), launch.
+bool decode_2d_supported(int es, int d, int H, int r_k, int r_v);
+size_t decode_2d_workspace_bytes(int r_k, int r_v, int B);
+lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream);
+
 int num_sms();  // SM count of the current device (cached), 0 on failure
 
 }  // namespace lla

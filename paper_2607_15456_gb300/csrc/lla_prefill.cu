@@ -125,7 +125,7 @@ struct PF {
 
 // barrier indices
 enum {
-    kBSetup = 0, kBQt, kBQs, kBOa, kBWv, kBOut, kBOdone, kBOfin,
+    kBSetup = 0, kBQt, kBQs, kBOa, kBWv, kBOut, kBUnused, kBOfin,
     kBSfull = 8 /* [2] */, kBSfree = 10, kBPfull = 12, kBPfree = 14,
     kBOa2 = 16, kBOut1 = 17,
     kBKfull = 18 /* [4] */, kBKempty = 22, kBVfull = 26, kBVempty = 30,
@@ -172,7 +172,6 @@ __global__ void __launch_bounds__(kPThreads, 1)
         mbar_init(&bar[kBWv], 32);
         mbar_init(&bar[kBOut1], 1);
         mbar_init(&bar[kBOut], 1);
-        mbar_init(&bar[kBOdone], 1);
         mbar_init(&bar[kBOfin], 1);
         for (int s = 0; s < F::STK; ++s) {
             mbar_init(&bar[kBKfull + s], 1);
@@ -329,7 +328,6 @@ __global__ void __launch_bounds__(kPThreads, 1)
                 }
                 umma_commit(&bar[kBVempty + sv]);
                 umma_commit(&bar[kBPfree + s]);
-                umma_commit(&bar[kBOdone]);
             }
             umma_commit(&bar[kBOfin]);  // every PV MMA (and, before them, every S MMA) has completed
             // out = (O / l) W_up,t^V^T, with O / l = hi + lo as two bf16 operands in turn, so
@@ -461,8 +459,11 @@ __global__ void __launch_bounds__(kPThreads, 1)
                 m = m_new;
             }
             if (__any_sync(0xffffffffu, need && j > 0)) {
-                // O holds pages 0..j-1: wait for the last of them, then rescale this half
-                mbar_wait(&bar[kBOdone], (j - 1) & 1, abort_flag, p.err);
+                // O holds pages 0..j-1: wait for the last of them, then rescale this half.  The
+                // product of page j - 1 releases P buffer (j - 1) & 1; the one of page j - 3 had
+                // released it before this row wrote page j - 1, so the parity test cannot pass a
+                // phase early (a barrier committed once per page could be two phases behind)
+                mbar_wait(&bar[kBPfree + ((j - 1) & 1)], ((j - 1) >> 1) & 1, abort_flag, p.err);
                 tc_fence_after();
 #pragma unroll 1
                 for (int c0 = half * (RV / 2); c0 < (half + 1) * (RV / 2); c0 += 16) {

@@ -88,6 +88,10 @@ def library() -> ctypes.CDLL:
             "lla_prefill_attn_rope": (I32, [P, P, P, P, P, I32, I32, I32, P, I32, P, P, SZ, P]),
             "lla_dense_store": (I32, [P, P, P, P, I32, P, I32, P]),
             "lla_dense_decode_attn": (I32, [P, P, P, I32, I32, P, P, P, I32, P, P, SZ, P]),
+            "lla_cache_2d_block_bytes": (I32, [P, P]),
+            "lla_encode_2d": (I32, [P, P, P, P, P, I32, P, I32, P]),
+            "lla_decode_2d_workspace_size": (I32, [P, I32, P]),
+            "lla_decode_attn_2d": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ, P]),
             "lla_get_device_error": (I32, [P, P]),
             "lla_clear_device_error": (I32, [P]),
         }
@@ -330,6 +334,46 @@ def lla_prefill_attn_rope(geom: Geometry, codec: Codec, cache: Cache, rope_base:
         ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), ctypes.byref(rp), _ptr(cu_seqlens), B,
         max_len, loop, _ptr(q), _dtype_code(q), _ptr(out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def lla_cache_2d_block_bytes(geom: Geometry) -> int:
+    """Bytes of one LLA-2D cache block (one page of 64 tokens for all heads)."""
+    out = ctypes.c_size_t(0)
+    g = geom.c()
+    _check("lla_cache_2d_block_bytes",
+           library().lla_cache_2d_block_bytes(ctypes.byref(g), ctypes.byref(out)))
+    return out.value
+
+
+def lla_encode_2d(geom: Geometry, codec: Codec, cache: Cache, x_k: torch.Tensor,
+                  x_v: torch.Tensor, slot_mapping: torch.Tensor, stream=None) -> None:
+    """LLA-2D encode.  x_k, x_v [T][N][H][d]; codec w_down_* [T*H*d][r], mu_* [T*H*d];
+    cache with one page per block."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    N = x_k.shape[1] if x_k.dim() == 4 else 0
+    _check("lla_encode_2d", library().lla_encode_2d(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(x_k), _ptr(x_v),
+        _dtype_code(x_k), _ptr(slot_mapping), N, _stream(stream)))
+
+
+def lla_decode_2d_workspace_size(geom: Geometry, B: int) -> int:
+    out = ctypes.c_size_t(0)
+    g = geom.c()
+    _check("lla_decode_2d_workspace_size",
+           library().lla_decode_2d_workspace_size(ctypes.byref(g), B, ctypes.byref(out)))
+    return out.value
+
+
+def lla_decode_attn_2d(geom: Geometry, codec: Codec, cache: Cache, context_lens: torch.Tensor,
+                       max_ctx: int, loop: int, q: torch.Tensor, cur_k: Optional[torch.Tensor],
+                       cur_v: Optional[torch.Tensor], out: torch.Tensor, workspace: torch.Tensor,
+                       stream=None) -> None:
+    """LLA-2D decode call; codec w_up_* [T][H][d][r]; q, cur_k, cur_v, out [B][H][d]."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    _check("lla_decode_attn_2d", library().lla_decode_attn_2d(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(context_lens), q.shape[0],
+        max_ctx, loop, _ptr(q), _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out),
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def lla_dense_store(geom: Geometry, cache: Cache, k: torch.Tensor, v: torch.Tensor,

@@ -12,8 +12,15 @@ Workloads (the five shapes the library is measured and checked on; Ouro-shaped p
   ouro26_rho533   D=48, H=16, (72,120)  rho=5.33,  B=64,  context ~ logU[512, 16384]
   stress_rho2133  D=48, H=16, (18,30)   rho=21.33, B=128, context ~ U[8192, 32768]
 
+and the LLA-2D variant (Sec. 3) at the per-head stress workload's cache budget: one latent per
+(token, layer) of H times the per-head width, (r_k, r_v) = 16 x (18, 30) = (288, 480), the same
+rho_2D = 2 T H d / (r_k + r_v) = 21.33 (Table isocache prints LLA-2D at this ratio):
+
+  stress2d_rho2133  D=48, H=16, (288,480)  B=128, context ~ U[8192, 32768]
+
 Recipe: activations, queries and current-token K/V are N(0,1); W_down is N(0, 1/(T d)) and
-W_up,t is N(0, 1/r) (std = 1/sqrt(.)); mu = 0 unless asked for (then N(0,1)); seeds are the
+W_up,t is N(0, 1/r) (std = 1/sqrt(.)); for LLA-2D W_down is N(0, 1/(T H d)) and W_up,t,h
+N(0, 1/r); mu = 0 unless asked for (then N(0,1)); seeds are the
 workload's index (tiny = 0).  Context lengths are integers drawn uniformly (or log-uniformly,
 floor(exp(U[ln lo, ln hi]))) over the inclusive range and are not rounded to the 64-token page
 grid.  Physical blocks come from a shuffled free list, so every sequence's pages are scattered
@@ -46,10 +53,11 @@ class Workload:
     io: str = "bf16"
     prefill: Optional[Tuple[int, int]] = None  # (sequences, tokens each)
     decode_steps: int = 1
+    lla2d: bool = False  # one latent per (token, layer) for all heads (Sec. 3, LLA-2D)
 
     @property
     def rho(self) -> float:
-        return 2 * self.T * self.d / (self.r_k + self.r_v)
+        return 2 * self.T * self.d * (self.H if self.lla2d else 1) / (self.r_k + self.r_v)
 
 
 WORKLOADS = {
@@ -63,6 +71,8 @@ WORKLOADS = {
                               lens=("loguniform", 512, 16384), seed=3),
     "stress_rho2133": Workload("stress_rho2133", D=48, H=16, d=128, T=4, r_k=18, r_v=30, B=128,
                                lens=("uniform", 8192, 32768), seed=4),
+    "stress2d_rho2133": Workload("stress2d_rho2133", D=48, H=16, d=128, T=4, r_k=288, r_v=480,
+                                 B=128, lens=("uniform", 8192, 32768), seed=4, lla2d=True),
 }
 
 
@@ -117,6 +127,29 @@ def codec_tensors(T: int, H: int, d: int, r_k: int, r_v: int, seed: int, layer: 
     return out
 
 
+def codec_tensors_2d(T: int, H: int, d: int, r_k: int, r_v: int, seed: int, layer: int,
+                     dtype=torch.bfloat16, device="cpu", with_mu: bool = False, mu_seed: int = 1):
+    """LLA-2D codec of one layer: W_down [T*H*d][r] ~ N(0, 1/(T H d)) (rows ordered (t, h, e)),
+    W_up [T][H][d][r] ~ N(0, 1/r), axis K then V, W_down then W_up,t,h in (t, h) order.
+    mu [T*H*d] ~ N(0, 1) fp32 when asked for."""
+    g = _gen(seed, 6, layer)
+    S = T * H * d
+    out = dict(mu_k=None, mu_v=None)
+    for ax, r in (("k", r_k), ("v", r_v)):
+        out["w_down_" + ax] = torch.randn(S, r, generator=g) / math.sqrt(S)
+        out["w_up_" + ax] = torch.randn(T, H, d, r, generator=g) / math.sqrt(r)
+    if with_mu:
+        gm = _gen(seed, 7, layer, mu_seed)
+        out["mu_k"] = torch.randn(S, generator=gm)
+        out["mu_v"] = torch.randn(S, generator=gm)
+    for k in ("w_down_k", "w_down_v", "w_up_k", "w_up_v"):
+        out[k] = out[k].to(dtype).to(device).contiguous()
+    for k in ("mu_k", "mu_v"):
+        if out[k] is not None:
+            out[k] = out[k].to(torch.float32).to(device).contiguous()
+    return out
+
+
 def normal(shape, seed: int, *key: int, dtype=torch.bfloat16, device="cpu") -> torch.Tensor:
     """N(0,1) tensor; drawn on `device` with a generator of that device."""
     s = _gen(seed, 4, *key).initial_seed()
@@ -152,3 +185,31 @@ def page_table(lens: List[int], seed: int, extra_tokens: int = 1, spare_blocks: 
         table[b, :n] = perm[o:o + n]
         o += n
     return PageTable(table, total, mb, [n * BLOCK for n in need])
+
+
+def pack_latent_pages(c_k: torch.Tensor, c_v: torch.Tensor, table: torch.Tensor, lens: List[int],
+                      num_blocks: int) -> torch.Tensor:
+    """A one-page-per-block cache pool (uint8, on c_k's device) holding given bf16 latents:
+    c_k [N][r_k], c_v [N][r_v] of the sequences back to back, token p of sequence b in block
+    table[b][p // 64], row p % 64.  Layout of include/lla.h: the K-plane in 16-byte granules of
+    8 columns (granule g of row i at g*1024 + i*16), the V-plane row-major; rows past a
+    sequence are zero."""
+    r_k, r_v = c_k.shape[1], c_v.shape[1]
+    dev = c_k.device
+    page = BLOCK * (r_k + r_v) * 2
+    pool = torch.zeros((num_blocks, page), dtype=torch.uint8, device=dev)
+    off = 0
+    for b, L in enumerate(lens):
+        n = -(-L // BLOCK)
+        if n == 0:
+            continue
+        kp = torch.zeros((n * BLOCK, r_k), dtype=torch.bfloat16, device=dev)
+        vp = torch.zeros((n * BLOCK, r_v), dtype=torch.bfloat16, device=dev)
+        kp[:L] = c_k[off:off + L]
+        vp[:L] = c_v[off:off + L]
+        kg = kp.view(n, BLOCK, r_k // 8, 8).permute(0, 2, 1, 3).contiguous().view(n, -1)
+        blocks = table[b, :n].to(torch.int64).to(dev)
+        pool[blocks, :BLOCK * r_k * 2] = kg.view(torch.uint8)
+        pool[blocks, BLOCK * r_k * 2:] = vp.view(n, -1).view(torch.uint8)
+        off += L
+    return pool.view(-1)

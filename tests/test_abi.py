@@ -273,3 +273,56 @@ def test_decode_loops_argument_checks(lib):
     assert call(g=_g(lib, r_k=72, r_v=120)) == UNSUPPORTED
     assert call(g=_g(lib, storage="fp32")) == UNSUPPORTED
     assert call(B=0, q=None, ck=None, cv=None, out=None, ws=None, lens=None) == OK
+
+
+def test_2d_block_bytes_and_workspace_shapes(lib):
+    so = lib.library()
+    n = ctypes.c_size_t(0)
+    g = _g(lib, r_k=288, r_v=480)
+    assert so.lla_cache_2d_block_bytes(ctypes.byref(g), ctypes.byref(n)) == OK
+    assert n.value == 64 * (288 + 480) * 2  # one page of 64 tokens for all heads
+    for bad in (_g(lib, r_k=72, r_v=120), _g(lib, d=64), _g(lib, H=17, r_k=288, r_v=480),
+                _g(lib, r_k=288, r_v=480, storage="fp32")):
+        assert so.lla_decode_2d_workspace_size(ctypes.byref(bad), 4, ctypes.byref(n)) == UNSUPPORTED
+    assert so.lla_decode_2d_workspace_size(ctypes.byref(g), -1, ctypes.byref(n)) == INVALID
+
+
+def test_decode_2d_argument_checks(lib):
+    so = lib.library()
+
+    def call(g=None, B=4, max_ctx=128, loop=0, q=FAKE, ck=FAKE, cv=FAKE, io=0, out=FAKE, ws=FAKE,
+             lens=FAKE, codec=None):
+        g = g or _g(lib, r_k=288, r_v=480)
+        codec, cache = codec or _codec(lib), _cache(lib)
+        return so.lla_decode_attn_2d(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache),
+                                     lens, B, max_ctx, loop, q, ck, cv, io, out, ws, 1 << 20, None)
+    assert call(ck=None) == INVALID
+    assert call(B=-1) == INVALID
+    assert call(B=1025) == INVALID
+    assert call(loop=4) == INVALID
+    assert call(q=None) == INVALID
+    assert call(max_ctx=4 * 64 + 1) == INVALID
+    assert call(codec=_codec(lib, w_up_v=None)) == INVALID
+    assert call(codec=_codec(lib, w_up_k=FAKE + 8)) == INVALID
+    assert call(g=_g(lib, r_k=72, r_v=120)) == UNSUPPORTED
+    assert call(g=_g(lib, H=32, r_k=288, r_v=480)) == UNSUPPORTED
+    assert call(g=_g(lib, r_k=288, r_v=480, storage="fp32")) == UNSUPPORTED
+    assert call(B=0, q=None, ck=None, cv=None, out=None, ws=None, lens=None) == OK
+
+
+def test_encode_2d_argument_checks(lib):
+    so = lib.library()
+
+    def call(g=None, N=8, xk=FAKE, xv=FAKE, slots=FAKE, xdt=0, codec=None):
+        g = g or _g(lib, r_k=288, r_v=480)
+        codec, cache = codec or _codec(lib), _cache(lib)
+        return so.lla_encode_2d(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache), xk, xv,
+                                xdt, slots, N, None)
+    assert call(N=-1) == INVALID
+    assert call(xk=None) == INVALID
+    assert call(slots=None) == INVALID
+    assert call(xdt=7) == INVALID
+    assert call(xv=FAKE + 4) == INVALID
+    assert call(codec=_codec(lib, w_down_k=None)) == INVALID
+    assert call(g=_g(lib, H=4096, d=128)) == UNSUPPORTED  # H d past the stack the encode takes
+    assert call(N=0, xk=None, xv=None, slots=None) == OK
