@@ -26,10 +26,12 @@
 //                       warps 2-5  per page: the scores of 16 tokens per warp, the maxima over
 //                                  the page per head, P^T as a bf16 operand, the lazy O^T rescale;
 //                                  per run: the partial out to the workspace
-//   finish2d_kernel   per (head, 8 sequences): merges the runs of each sequence, adds the pass-1
-//                     current token, and applies W_up,t,h^V once for the 8 sequences
+//   finish2d_kernel   per (head, up to 8 sequences): merges the runs of each sequence, adds the
+//                     pass-1 current token, and applies W_up,t,h^V once for those sequences
 // Storage bf16, d = 128, H <= 16; accumulators fp32 in TMEM.
 #include <cuda_runtime.h>
+
+#include <algorithm>
 
 #include "lla_device.cuh"
 #include "lla_internal.h"
@@ -48,7 +50,7 @@ constexpr int kSm0 = 64;         // first softmax thread
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;  // rescale O^T only when a head's maximum grows by more
 constexpr int kSmemCap = 227 * 1024;
-constexpr int kFinishSeqs = 8;   // sequences per finish CTA
+constexpr int kFinishSeqs = 8;   // most sequences per finish CTA
 constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one sequence fit one finish CTA)
 
 // Shared-memory plan of the attention kernel for ranks (RK, RV).  Offsets from a 1024-byte
@@ -122,6 +124,7 @@ struct T2Params {
 
 struct F2Params {
     int T, H, loop, io_bf16, B, grid;
+    int spb;  // sequences per CTA (1 .. 8)
     float scale_log2;
     const void *w_up_v;  // [T][H][d][r_v] bf16
     const float *mu_v;   // [T*H*d] or NULL
@@ -187,44 +190,56 @@ __device__ void page_prefix(const A2Params &p) {
     if (tid == blockDim.x - 1) p.pstart[p.B] = pre + x;
 }
 
-// Grid (H, ceil(B / 16)), 256 threads: q~ and beta of head h for 16 sequences.
+// Grid (H, RK / 32, ceil(B / 16)), 256 threads = 32 columns x 8 slices of 16 rows of the head:
+// q~ of 32 columns of head h for 16 sequences, every weight load of a thread in flight at once;
+// beta of head h by the CTAs of the first column chunk.
 template <int RK>
 __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
+    static_assert(RK % 32 == 0, "column chunks");
     __shared__ float qs[16][kD];
-    const int h = blockIdx.x, b0 = blockIdx.y * 16, tid = threadIdx.x;
+    __shared__ float red[8][16][33];
+    const int h = blockIdx.x, j0 = blockIdx.y * 32, b0 = blockIdx.z * 16, tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(16, p.B - b0);
-    pdl_wait();  // the workspace is free once the previous call has finished
-    if (blockIdx.x == 0 && blockIdx.y == 0) page_prefix(p);
+    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
+    pdl_wait();  // inputs may come from the previous kernel; the workspace is free after it
+    // this thread's 16 weights (column j0 + lane, rows 16 warp .. 16 warp + 15), in flight while
+    // the queries load
+    const uint16_t *W = static_cast<const uint16_t *>(p.w_up_k) + th * kD * RK + j0 + lane;
+    float w[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u) w[u] = bf_to_f(W[(warp * 16 + u) * RK]);
+    if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) page_prefix(p);
     for (int i = tid; i < 16 * kD; i += 256) {
         const int bi = i >> 7, e = i & (kD - 1);
         qs[bi][e] = bi < nb ? load_elem(p.q, (static_cast<int64_t>(b0 + bi) * p.H + h) * kD + e, p.io_bf16)
                             : 0.f;
     }
     __syncthreads();
-    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
-    const uint16_t *W = static_cast<const uint16_t *>(p.w_up_k) + th * kD * RK;
-    for (int j = tid; j < RK; j += 256) {
-        float acc[16];
 #pragma unroll
-        for (int bi = 0; bi < 16; ++bi) acc[bi] = 0.f;
-#pragma unroll 4
-        for (int e = 0; e < kD; ++e) {
-            const float w = bf_to_f(W[e * RK + j]);
+    for (int bi = 0; bi < 16; ++bi) {
+        float a = 0.f;
 #pragma unroll
-            for (int bi = 0; bi < 16; ++bi) acc[bi] = fmaf(w, qs[bi][e], acc[bi]);
-        }
+        for (int u = 0; u < 16; ++u) a = fmaf(w[u], qs[bi][warp * 16 + u], a);
+        red[warp][bi][lane] = a;
+    }
+    __syncthreads();
+    for (int o = tid; o < 16 * 32; o += 256) {
+        const int bi = o >> 5, c = o & 31;
+        float a = 0.f;
 #pragma unroll
-        for (int bi = 0; bi < 16; ++bi)
-            if (bi < nb) p.qt[(static_cast<int64_t>(b0 + bi) * kNQ + h) * RK + j] = acc[bi] * p.scale_log2;
+        for (int sl = 0; sl < 8; ++sl) a += red[sl][bi][c];
+        if (bi < nb) p.qt[(static_cast<int64_t>(b0 + bi) * kNQ + h) * RK + j0 + c] = a * p.scale_log2;
     }
     // beta_h = q_h . mu^K_{t,h}: warp w takes sequences w and w + 8
-    const int warp = tid >> 5, lane = tid & 31;
-    for (int bi = warp; bi < nb; bi += 8) {
-        float s = 0.f;
-        if (p.mu_k)
-            for (int e = lane; e < kD; e += 32) s = fmaf(qs[bi][e], p.mu_k[th * kD + e], s);
-        s = warp_sum(s);
-        if (lane == 0) p.beta[static_cast<int64_t>(b0 + bi) * kNQ + h] = s * p.scale_log2;
+    if (blockIdx.y == 0) {
+        for (int bi = warp; bi < nb; bi += 8) {
+            float s = 0.f;
+            if (p.mu_k)
+                for (int e = lane; e < kD; e += 32) s = fmaf(qs[bi][e], p.mu_k[th * kD + e], s);
+            s = warp_sum(s);
+            if (lane == 0) p.beta[static_cast<int64_t>(b0 + bi) * kNQ + h] = s * p.scale_log2;
+        }
     }
     __syncthreads();
     pdl_trigger();
@@ -590,7 +605,8 @@ __global__ void __launch_bounds__(kT2, 1)
 
 // ------------------------------------------------------------------------- finish kernel
 
-// Grid (H, ceil(B / 8)), 128 threads (thread e = output element e of head h).
+// Grid (H, ceil(B / spb)), 128 threads (thread e = output element e of head h).  spb (at most 8)
+// sequences share one pass over W_up,t,h^V; small batches take fewer per CTA to use more SMs.
 template <int RV>
 __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     constexpr int PS = kNQ * RV + 2 * kNQ;
@@ -598,9 +614,9 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     __shared__ float wts[kMaxGrid];
     __shared__ float coef[kFinishSeqs][3];
     __shared__ float redm[4], reds[4];
-    const int h = blockIdx.x, b0 = blockIdx.y * kFinishSeqs, tid = threadIdx.x;
+    const int h = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
-    const int nb = min(kFinishSeqs, p.B - b0);
+    const int nb = min(p.spb, p.B - b0);
     const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
     pdl_wait();
     const int NP = p.pstart[p.B];
@@ -639,10 +655,19 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
             if (lane == 0) reds[warp] = ls;
             __syncthreads();
             l = (reds[0] + reds[1]) + (reds[2] + reds[3]);
+            const float *pj = p.part + static_cast<int64_t>(b + c0) * PS + h * RV;
             for (int j = tid; j < RV; j += 128) {
                 float a = 0.f;
-                for (int i = 0; i < nr; ++i)
-                    if (wts[i] > 0.f) a = fmaf(wts[i], p.part[static_cast<int64_t>(b + c0 + i) * PS + h * RV + j], a);
+                int i = 0;
+                for (; i + 8 <= nr; i += 8) {  // eight partials in flight
+                    float v[8];
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) v[u] = wts[i + u] > 0.f ? pj[static_cast<int64_t>(i + u) * PS + j] : 0.f;
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) a = fmaf(wts[i + u], v[u], a);
+                }
+                for (; i < nr; ++i)
+                    if (wts[i] > 0.f) a = fmaf(wts[i], pj[static_cast<int64_t>(i) * PS + j], a);
                 ob[bi][j] = a;
             }
         } else {
@@ -677,7 +702,7 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     float acc[kFinishSeqs];
 #pragma unroll
     for (int bi = 0; bi < kFinishSeqs; ++bi) acc[bi] = 0.f;
-#pragma unroll 2
+#pragma unroll 4
     for (int j8 = 0; j8 < RV / 8; ++j8) {
         const uint4 w4 = W[j8];
         const float2 w0 = bf2_to_f2(w4.x), w1 = bf2_to_f2(w4.y), w2 = bf2_to_f2(w4.z), w3 = bf2_to_f2(w4.w);
@@ -777,7 +802,8 @@ lla_status launch_2d(const DecodeArgs &a, cudaStream_t stream) {
     ap.beta = reinterpret_cast<float *>(ws + w.beta);
     ap.pstart = reinterpret_cast<int *>(ws + w.pstart);
     ap.err = err;
-    if ((st = launch_ex(absorb2d_kernel<RK>, dim3(a.H, (a.B + 15) / 16), 256, 0, stream, ap)) != LLA_OK)
+    if ((st = launch_ex(absorb2d_kernel<RK>, dim3(a.H, RK / 32, (a.B + 15) / 16), 256, 0, stream, ap)) !=
+        LLA_OK)
         return st;
 
     T2Params tp = {};
@@ -798,7 +824,10 @@ lla_status launch_2d(const DecodeArgs &a, cudaStream_t stream) {
     fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
     fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
     fp.pstart = ap.pstart; fp.part = tp.part;
-    return launch_ex(finish2d_kernel<RV>, dim3(a.H, (a.B + kFinishSeqs - 1) / kFinishSeqs), 128, 0, stream, fp);
+    // about two finish CTAs per SM: fewer sequences per CTA for small batches
+    const int64_t want = static_cast<int64_t>(a.B) * a.H;
+    fp.spb = static_cast<int>(std::min<int64_t>(kFinishSeqs, std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
+    return launch_ex(finish2d_kernel<RV>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
 }
 
 }  // namespace
