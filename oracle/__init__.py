@@ -24,6 +24,9 @@ calls it through ctypes.  Citations (paper sections and equations):
                                        reconstruction (Sec. 3, "RoPE and reconstruction")
 * ``decode_rope``, ``prefill_rope`` -- ``decode`` / ``prefill`` with every reconstructed key
                                        and the query rotated at their token positions
+* ``decode_decoupled``              -- the decoupled rotary branch (App. J "Absorbed attention"):
+                                       content key by Eq. decode (no rotation) joined with one
+                                       rotary key per token, shared by every loop
 * ``ratio_2d``, ``encode_2d``,      -- the LLA-2D variant (Sec. 3, "The LLA-2D variant (loop x
   ``decode_2d``                        head)"): one latent per (token, layer) over the
                                        loop-major (loop, head) stack, every head rebuilt from it
@@ -78,6 +81,9 @@ def _load():
         lib.lla_oracle_decode_batch.argtypes = [i32, i32, i32, i32, d, i64, p, i32]
         lib.lla_oracle_encode_batch.restype = i32
         lib.lla_oracle_encode_batch.argtypes = [i32, i32, i64, i64, p, i32]
+        lib.lla_oracle_decode_decoupled.restype = i32
+        lib.lla_oracle_decode_decoupled.argtypes = ([i32] * 6 + [i64] + [p] * 12 +
+                                                    [d, i32, d, i64, p])
         lib.lla_oracle_ratio_2d.restype = d
         lib.lla_oracle_ratio_2d.argtypes = [i32, i32, i32, i32, i32]
         lib.lla_oracle_encode_2d.restype = None
@@ -259,6 +265,40 @@ def prefill_rope(t: int, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, q, scale: float,
     return out
 
 
+# ---------------------------------------------------------------- decoupled rotary branch
+
+def decode_decoupled(t: int, c_k, c_v, k_rope, w_up_k, w_up_v, mu_k, mu_v, q, q_rope, cur_k,
+                     cur_v, cur_k_rope, scale: float, base: float = 10000.0,
+                     pairing: int = ROPE_HALF, pos0: int = 0) -> np.ndarray:
+    """One decode call for one (sequence, head) at loop t with the decoupled rotary branch:
+    s_i = scale (q . khat_t,i + rot(q^R, P) . rot(k^R_i, p_i)).  k_rope [L][d_rope] (one rotary
+    key per token, every loop), q_rope [d_rope]; cur_k_rope [d_rope] with cur_k / cur_v in
+    pass 1, None in pass 2.  Other arguments as ``decode``."""
+    w_up_k, w_up_v = _f64(w_up_k), _f64(w_up_v)
+    T, d, r_k = w_up_k.shape
+    r_v = w_up_v.shape[2]
+    c_k = _f64(c_k).reshape(-1, r_k)
+    c_v = _f64(c_v).reshape(-1, r_v)
+    L = c_k.shape[0]
+    q_rope = _f64(q_rope).reshape(-1)
+    d_rope = q_rope.shape[0]
+    k_rope = _f64(k_rope).reshape(L, d_rope)
+    mu_k = None if mu_k is None else _f64(mu_k).reshape(T * d)
+    mu_v = None if mu_v is None else _f64(mu_v).reshape(T * d)
+    q = _f64(q).reshape(d)
+    cur_k = None if cur_k is None else _f64(cur_k).reshape(d)
+    cur_v = None if cur_v is None else _f64(cur_v).reshape(d)
+    cur_k_rope = None if cur_k_rope is None else _f64(cur_k_rope).reshape(d_rope)
+    out = np.zeros(d, dtype=np.float64)
+    rc = _load().lla_oracle_decode_decoupled(
+        T, d, d_rope, r_k, r_v, t, L, _ptr(c_k), _ptr(c_v), _ptr(k_rope), _ptr(w_up_k),
+        _ptr(w_up_v), _ptr(mu_k), _ptr(mu_v), _ptr(q), _ptr(q_rope), _ptr(cur_k), _ptr(cur_v),
+        _ptr(cur_k_rope), scale, pairing, base, pos0, _ptr(out))
+    if rc:
+        raise ValueError("bad decode arguments")
+    return out
+
+
 # ---------------------------------------------------------------- LLA-2D (Sec. 3)
 
 def ratio_2d(T: int, H: int, d_head: int, r_k: int, r_v: int) -> float:
@@ -402,6 +442,7 @@ def encode_batch(T: int, d: int, items: Sequence[dict], n_threads: int = 0) -> l
 
 __all__ = ["ratio", "teacher_cache_bytes_per_token", "latent_cache_bytes_per_token", "encode",
            "reconstruct", "attention", "decode", "prefill", "rope", "decode_rope",
-           "prefill_rope", "ROPE_HALF", "ROPE_ADJACENT", "ratio_2d", "encode_2d", "decode_2d",
+           "prefill_rope", "ROPE_HALF", "ROPE_ADJACENT", "decode_decoupled", "ratio_2d",
+           "encode_2d", "decode_2d",
            "decode_batch", "encode_batch",
            "max_threads", "build_oracle", "library_path"]

@@ -315,6 +315,84 @@ int lla_oracle_prefill_rope(int T, int d, int r_k, int r_v, int t, int64_t N, co
 }
 
 /*
+ * Decoupled rotary branch (App. J "Absorbed attention": an MLA-style NoPE content path plus a
+ * small explicit rotary branch shared across recurrence steps for each token; DeepSeek-V2).
+ * Loop t's key of cached token i is the pair (khat_t,i, k^R_i): the content key khat_t,i of
+ * Eq. decode (no rotation) and a rotary key k^R_i of d_rope dims, one per token for every loop,
+ * rotated at the token's position.  The query is the pair (q, q^R), q^R rotated at the current
+ * token's position.  The score adds the two dot products under one scale:
+ *   s_i = scale (q . khat_t,i + rot(q^R, P) . rot(k^R_i, p_i))
+ * and the value is Eq. decode's vhat_t,i.  Cached token i sits at position pos0 + i; the
+ * current token (the query) at pos0 + L in pass 1, where it attends with its exact loop-t key
+ * and value and its own rotary key, and at pos0 + L - 1 in pass 2.
+ *   k_rope [L][d_rope]      pre-rotation rotary keys of the cached tokens
+ *   q_rope [d_rope]         pre-rotation rotary query
+ *   cur_k_rope [d_rope]     pass 1: the current token's rotary key (NULL in pass 2)
+ * Other arguments as lla_oracle_decode.
+ */
+int lla_oracle_decode_decoupled(int T, int d, int d_rope, int r_k, int r_v, int t, int64_t L,
+                                const double *c_k, const double *c_v, const double *k_rope,
+                                const double *w_up_k, const double *w_up_v, const double *mu_k,
+                                const double *mu_v, const double *q, const double *q_rope,
+                                const double *cur_k, const double *cur_v,
+                                const double *cur_k_rope, double scale, int pairing, double base,
+                                int64_t pos0, double *out)
+{
+    if (t < 0 || t >= T || L < 0 || d_rope < 2 || d_rope % 2 != 0 || base <= 0.0)
+        return -1;
+    if ((cur_k == NULL) != (cur_v == NULL) || (cur_k == NULL) != (cur_k_rope == NULL))
+        return -1;
+    const int pass1 = cur_k != NULL;
+    if (!pass1 && L < 1)
+        return -1;
+    const int64_t n = L + (pass1 ? 1 : 0);
+    const int w = d + d_rope; /* width of a joined key [khat; rot(k^R)] */
+    double *K = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    double *V = (double *)malloc(sizeof(double) * (size_t)(n * d));
+    double *J = (double *)malloc(sizeof(double) * (size_t)(n * w));
+    double *qj = (double *)malloc(sizeof(double) * (size_t)w);
+    /* content keys and values of loop t (Eq. decode; pass 1 appends the exact current pair) */
+    loop_keys_values(d, r_k, r_v, t, L, c_k, c_v, w_up_k, w_up_v, mu_k, mu_v, cur_k, cur_v, K, V);
+    /* joined keys: the content key, then the rotary key turned at the token's position */
+    for (int64_t i = 0; i < n; ++i) {
+        memcpy(J + i * w, K + i * d, sizeof(double) * (size_t)d);
+        const double *kr = i < L ? k_rope + i * d_rope : cur_k_rope;
+        lla_oracle_rope(d_rope, pairing, base, pos0 + i, kr, J + i * w + d);
+    }
+    /* joined query: content query, then the rotary query at the current token's position */
+    memcpy(qj, q, sizeof(double) * (size_t)d);
+    lla_oracle_rope(d_rope, pairing, base, pos0 + n - 1, q_rope, qj + d);
+    /* softmax over the joined dot products, values of width d */
+    double *sj = (double *)malloc(sizeof(double) * (size_t)n);
+    double m = -INFINITY;
+    for (int64_t i = 0; i < n; ++i) {
+        double dot = 0.0;
+        for (int e = 0; e < w; ++e)
+            dot += qj[e] * J[i * w + e];
+        sj[i] = dot * scale;
+        if (sj[i] > m)
+            m = sj[i];
+    }
+    double z = 0.0;
+    for (int64_t i = 0; i < n; ++i) {
+        sj[i] = exp(sj[i] - m);
+        z += sj[i];
+    }
+    for (int e = 0; e < d; ++e) {
+        double acc = 0.0;
+        for (int64_t i = 0; i < n; ++i)
+            acc += sj[i] * V[i * d + e];
+        out[e] = acc / z;
+    }
+    free(sj);
+    free(K);
+    free(V);
+    free(J);
+    free(qj);
+    return 0;
+}
+
+/*
  * LLA-2D (Sec. 3, "The LLA-2D variant (loop x head)"): one latent per (token, layer) that
  * covers every head.  The stacked vector runs over loops and heads, loop-major,
  *   x = [x_{1,1}; ...; x_{1,H}; x_{2,1}; ...; x_{T,H}] in R^{T H d},

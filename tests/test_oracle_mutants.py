@@ -46,6 +46,17 @@ MUTANTS = [
      "for (int64_t i = 0; i < n; ++i)\n        memcpy(Kr + i * d, K + i * d, sizeof(double) * (size_t)d);"),
     ("prefill_rope_query_position", "lla_oracle_rope(d, pairing, base, pos0 + i, q + i * d, qr);",
      "lla_oracle_rope(d, pairing, base, pos0, q + i * d, qr);"),
+    ("decoupled_query_position",
+     "lla_oracle_rope(d_rope, pairing, base, pos0 + n - 1, q_rope, qj + d);",
+     "lla_oracle_rope(d_rope, pairing, base, pos0 + L, q_rope, qj + d);"),
+    ("decoupled_key_position",
+     "lla_oracle_rope(d_rope, pairing, base, pos0 + i, kr, J + i * w + d);",
+     "lla_oracle_rope(d_rope, pairing, base, pos0, kr, J + i * w + d);"),
+    ("decoupled_rotary_dropped", "for (int e = 0; e < w; ++e)\n            dot += qj[e] * J[i * w + e];",
+     "for (int e = 0; e < d; ++e)\n            dot += qj[e] * J[i * w + e];"),
+    ("decoupled_current_rotary_key", "const double *kr = i < L ? k_rope + i * d_rope : cur_k_rope;",
+     "const double *kr = i < L ? k_rope + i * d_rope : k_rope;"),
+    ("decoupled_drops_scale", "sj[i] = dot * scale;", "sj[i] = dot;"),
     ("ratio_2d_drops_heads",
      "return 2.0 * (double)T * (double)H * (double)d_head / (double)(r_k + r_v);",
      "return 2.0 * (double)T * (double)d_head / (double)(r_k + r_v);"),
@@ -72,7 +83,8 @@ def _run_mutant(name, old, new, tmp):
         f.write(src.replace(old, new))
     subprocess.run(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-fopenmp", path_c, "-o",
                     path_so, "-lm"], check=True)
-    env = dict(os.environ, LLA_ORACLE_LIB=path_so)
+    # one OpenMP thread per mutant: the mutants already run side by side
+    env = dict(os.environ, LLA_ORACLE_LIB=path_so, OMP_NUM_THREADS="1")
     res = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
                           os.path.join(ROOT, "tests", "test_oracle_pins.py")],
                          cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)

@@ -758,3 +758,92 @@ def test_decode_2d_special_cases():
             np.testing.assert_allclose(zero[h], up_v[t, h] @ c_v.mean(axis=0) + mu_v[sl],
                                        rtol=0, atol=1e-12)
         np.testing.assert_allclose(empty, cv, rtol=0, atol=0)
+
+
+# ------------------------------------------------------------------ decoupled rotary branch (App. J)
+
+@pytest.mark.parametrize("pass1", [False, True])
+@pytest.mark.parametrize("pairing", [oracle.ROPE_HALF, oracle.ROPE_ADJACENT])
+def test_decoupled_full_rank_equals_sdpa_on_joined_keys(pass1, pairing):
+    """Lossless full-rank codec: the decoupled decode is softmax attention whose keys are the raw
+    loop-t key joined with the token's rotary key turned at its position, and whose query is q
+    joined with the rotary query turned at the current position (torch SDPA, complex-form
+    rotation); the values are the raw loop-t values."""
+    T, d, dr, L, base = 2, 32, 16, 19, 500.0
+    g = _rng(90)
+    Qk, Qv = _orthogonal(T * d, 91), _orthogonal(T * d, 92)
+    xk, xv = g.standard_normal((T, L + 1, d)), g.standard_normal((T, L + 1, d))
+    kr = g.standard_normal((L + 1, dr))  # one rotary key per token, every loop
+    mu_k, mu_v = g.standard_normal(T * d), g.standard_normal(T * d)
+    n_cached = L if pass1 else L + 1
+    c_k = oracle.encode(xk[:, :n_cached], mu_k, Qk)
+    c_v = oracle.encode(xv[:, :n_cached], mu_v, Qv)
+    w_up_k = np.stack([Qk[t * d:(t + 1) * d] for t in range(T)])
+    w_up_v = np.stack([Qv[t * d:(t + 1) * d] for t in range(T)])
+    scale = 1 / math.sqrt(d + dr)
+    pos0 = 7
+    for t in range(T):
+        q, qr = g.standard_normal(d), g.standard_normal(dr)
+        out = oracle.decode_decoupled(t, c_k, c_v, kr[:n_cached], w_up_k, w_up_v, mu_k, mu_v, q, qr,
+                                      xk[t, L] if pass1 else None, xv[t, L] if pass1 else None,
+                                      kr[L] if pass1 else None, scale, base, pairing, pos0)
+        J = np.stack([np.concatenate([xk[t, i], _rot_complex(kr[i], pos0 + i, base, pairing)])
+                      for i in range(L + 1)])
+        qj = np.concatenate([q, _rot_complex(qr, pos0 + L, base, pairing)])
+        ref = _sdpa(qj, J, xv[t], scale)[0]
+        np.testing.assert_allclose(out, ref, rtol=0, atol=1e-12)
+
+
+def test_decoupled_without_rotary_parts_is_the_nope_decode():
+    """Zero rotary keys and query leave only the content path: the plain LLA decode (pinned
+    above), in both passes and at every loop."""
+    T, d, dr, r_k, r_v, L = 4, 32, 8, 12, 20, 23
+    g = _rng(93)
+    cod = _random_codec(T, d, r_k, r_v, 94)
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    q = g.standard_normal(d)
+    ck, cv = g.standard_normal(d), g.standard_normal(d)
+    for t in range(T):
+        for pass1 in (False, True):
+            a = oracle.decode_decoupled(t, c_k, c_v, np.zeros((L, dr)), cod["w_up_k"], cod["w_up_v"],
+                                        cod["mu_k"], cod["mu_v"], q, np.zeros(dr),
+                                        ck if pass1 else None, cv if pass1 else None,
+                                        np.zeros(dr) if pass1 else None, 0.2)
+            b = oracle.decode(t, c_k, c_v, cod["w_up_k"], cod["w_up_v"], cod["mu_k"], cod["mu_v"], q,
+                              ck if pass1 else None, cv if pass1 else None, 0.2)
+            np.testing.assert_allclose(a, b, rtol=0, atol=1e-13)
+
+
+@pytest.mark.parametrize("pass1", [False, True])
+def test_decoupled_absorbed_form_and_relative_positions(pass1):
+    """App. J absorbed form written independently: the content score moves W_up,t^K to the query
+    (q~ = W_up,t^K^T q, plus q . mu^K_t) and the rotary score is rot(q^R, P - p) . k^R (RoFormer's
+    relative form, complex multiplication); shifting every position leaves the output unchanged."""
+    T, d, dr, r_k, r_v, L, base = 4, 64, 32, 24, 40, 30, 10000.0
+    g = _rng(95)
+    cod = _random_codec(T, d, r_k, r_v, 96)
+    c_k, c_v = g.standard_normal((L, r_k)), g.standard_normal((L, r_v))
+    kr = g.standard_normal((L, dr))
+    q, qr = g.standard_normal(d), g.standard_normal(dr)
+    ck = g.standard_normal(d) if pass1 else None
+    cv = g.standard_normal(d) if pass1 else None
+    ckr = g.standard_normal(dr) if pass1 else None
+    scale = 1 / math.sqrt(d + dr)
+    for t in range(T):
+        out = oracle.decode_decoupled(t, c_k, c_v, kr, cod["w_up_k"], cod["w_up_v"], cod["mu_k"],
+                                      cod["mu_v"], q, qr, ck, cv, ckr, scale, base, 0, 11)
+        shifted = oracle.decode_decoupled(t, c_k, c_v, kr, cod["w_up_k"], cod["w_up_v"], cod["mu_k"],
+                                          cod["mu_v"], q, qr, ck, cv, ckr, scale, base, 0, 5011)
+        np.testing.assert_allclose(out, shifted, rtol=0, atol=1e-10)
+        Wk, Wv = cod["w_up_k"][t], cod["w_up_v"][t]
+        mk, mv = cod["mu_k"][t * d:(t + 1) * d], cod["mu_v"][t * d:(t + 1) * d]
+        P = L if pass1 else L - 1  # the current token's index
+        s = scale * (c_k @ (Wk.T @ q) + q @ mk +
+                     np.array([_rot_complex(qr, P - i, base, 0) @ kr[i] for i in range(L)]))
+        if pass1:
+            s = np.append(s, scale * (q @ ck + qr @ ckr))
+        p = np.exp(s - s.max())
+        o = Wv @ (p[:L] @ c_v) + p[:L].sum() * mv
+        if pass1:
+            o = o + p[L] * cv
+        np.testing.assert_allclose(out, o / p.sum(), rtol=0, atol=1e-12)
