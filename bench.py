@@ -378,6 +378,7 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_extras and rank == 0:
         result.update(run_rope_extra(bench))
         result.update(run_loops_extra(bench))
+        result.update(run_decoupled_extra(bench))
         del bench
         torch.cuda.empty_cache()
         result.update(run_extras(device))
@@ -451,6 +452,53 @@ def run_loops_extra(bench):
         "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
         "bytes_per_launch": nbytes, "tokens_per_s_decode_only": bench.B / (ms / 1e3),
         "note": "the layer's latents cross HBM once for its T loop calls"}}
+
+
+def run_decoupled_extra(bench, d_rope=64):
+    """Per-head LLA with the decoupled rotary branch (App. J "Absorbed attention"; d_rope = 64 as
+    in Table decoupled_char) on the headline batch: one rotary key per token and layer stored
+    turned at its position, then the step's D x T pass-1 calls through lla_decode_attn_decoupled.
+    Algorithmic bytes: the latents, the rotary planes once, this loop's W_up,t and the inputs and
+    outputs."""
+    import torch
+    w, lla, W = bench.w, bench.lla, bench.W
+    peak, _ = measured_peaks()
+    plane = lla.lla_rope_plane_bytes(d_rope)
+    Nt = sum(bench.lens)
+    pos = torch.cat([torch.arange(L, dtype=torch.int32) for L in bench.lens]).to(bench.device)
+    slots = torch.cat([bench.pt.slots(b, range(L)) for b, L in enumerate(bench.lens)]).to(bench.device)
+    pools = []
+    for l in range(w.D):
+        pool = torch.empty(bench.pt.num_blocks * plane, dtype=torch.uint8, device=bench.device)
+        k = W.normal((Nt, d_rope), w.seed, 500, l, device=bench.device)
+        lla.lla_encode_rope_keys(d_rope, ROPE_BASE, lla.LLA_ROPE_HALF, pool, bench.pt.num_blocks, k, pos, slots)
+        pools.append(pool)
+        del k
+    qr = W.normal((w.D, w.T, bench.B, w.H, d_rope), w.seed, 501, device=bench.device)
+    ckr = W.normal((w.D, w.T, bench.B, d_rope), w.seed, 502, device=bench.device)
+    ws = torch.empty(lla.lla_decode_decoupled_workspace_size(bench.geom, d_rope, bench.B), dtype=torch.uint8,
+                     device=bench.device)
+
+    def sweep():
+        for t in range(w.T):
+            for l in range(w.D):
+                lla.lla_decode_attn_decoupled(bench.geom, bench.codecs[l], bench.caches[l], pools[l], d_rope,
+                                              ROPE_BASE, lla.LLA_ROPE_HALF, bench.ctx, bench.max_ctx, t,
+                                              bench.q[l, t], qr[l, t], bench.cur_k[l, t], bench.cur_v[l, t],
+                                              ckr[l, t], bench.out[l, t], ws)
+    ms = _time_ms(sweep, reps=3, warm=1)
+    per_launch_s = ms / 1e3 / (w.D * w.T)
+    nbytes = (bench.decode_bytes_per_launch() + Nt * d_rope * 2
+              + bench.B * w.H * d_rope * 2 + bench.B * d_rope * 2)
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the decoupled decode measurement")
+    return {"decoupled_decode": {
+        "workload": f"{w.name} batch, decoupled rotary branch d_rope={d_rope} (base {ROPE_BASE:g}), "
+                    f"{w.D}x{w.T} pass-1 calls",
+        "kernel": "absorb2d_kernel + attn2d_kernel<96,160,64> + finish2d_kernel (lla_decode_attn_decoupled)",
+        "bound": "hbm", "ms_per_sweep": ms, "avg_call_us": per_launch_s * 1e6,
+        "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
+        "bytes_per_call": nbytes, "tokens_per_s_decode_only": bench.B / (ms / 1e3)}}
 
 
 def run_2d_extra(device):

@@ -18,6 +18,8 @@
  *   lla_prefill_attn     causal pass-2 prefill attention over the latents of a prompt
  *   lla_encode_2d, lla_decode_attn_2d
  *                        the LLA-2D variant: one latent per (token, layer) for every head
+ *   lla_encode_rope_keys, lla_decode_attn_decoupled
+ *                        per-head LLA with a decoupled rotary branch (one rotary key per token)
  *   lla_dense_*          the uncompressed loop-t KV decode in the same kernel style (the
  *                        "teacher" column of Table absorbed_latency, App. J), for comparison
  *
@@ -309,6 +311,60 @@ lla_status lla_decode_attn_2d(const lla_geometry *g, const lla_codec *codec, con
                               int32_t loop, const void *q, const void *cur_k, const void *cur_v,
                               lla_dtype io_dtype, void *out, void *workspace,
                               size_t workspace_bytes, void *stream);
+
+/*
+ * Decoupled rotary branch (App. J "Absorbed attention": an MLA-style NoPE content path plus a
+ * small explicit rotary branch shared across recurrence steps for each token, as in DeepSeek-V2).
+ * Loop t's key of cached token i is its content key khat_t,i (Eq. decode, not rotated) joined
+ * with one rotary key k^R_i of d_rope dims per token and layer, shared by every loop and head and
+ * turned at the token's position; the query of head h is q_h joined with its rotary query q^R_h
+ * turned at the current token's position:
+ *   s_i = scale (q_h . khat_t,i + rot(q^R_h, P) . rot(k^R_i, p_i)),  o = softmax(s) Vhat_t.
+ * The rotary keys live in rotary planes, one per cache block: [num_blocks][64 x d_rope] bf16 in
+ * the granule layout of a K-plane (element (row i, column j) at (j/8)*1024 + i*16 + (j%8)*2),
+ * lla_rope_plane_bytes bytes each, addressed through the cache's block table.
+ */
+
+/* Bytes of one rotary plane (64 tokens x d_rope, bf16); d_rope a multiple of 16 in 16..96. */
+lla_status lla_rope_plane_bytes(int32_t d_rope, size_t *bytes);
+
+/*
+ * Writes the rotary keys of N tokens, each turned at its position, into the rotary planes.
+ *   rope_pool     device [num_blocks][rotary plane], 16-byte aligned
+ *   k_rope        device [N][d_rope] x_dtype: pre-rotation rotary keys
+ *   positions     device [N] int32: the token's position in its sequence (< 0 sets
+ *                 LLA_DEVERR_CONTEXT and skips the token)
+ *   slot_mapping  device [N] int64: block * 64 + row (negative: skip; past the pool:
+ *                 LLA_DEVERR_SLOT)
+ */
+lla_status lla_encode_rope_keys(int32_t d_rope, const lla_rope *rope, void *rope_pool, int64_t num_blocks,
+                                const void *k_rope, lla_dtype x_dtype, const int32_t *positions,
+                                const int64_t *slot_mapping, int32_t N, void *stream);
+
+/* Workspace bytes lla_decode_attn_decoupled needs for B sequences on the current device
+ * (LLA_ERR_UNSUPPORTED for a shape with no kernel). */
+lla_status lla_decode_decoupled_workspace_size(const lla_geometry *g, int32_t d_rope, int32_t B,
+                                               size_t *bytes);
+
+/*
+ * One decode call of per-head LLA (the codec and cache of lla_decode_attn) with the decoupled
+ * rotary branch.  Cached token i of sequence b sits at position i; the current token at
+ * context_lens[b] in pass 1 and context_lens[b] - 1 in pass 2.
+ *   rope_pool    device rotary planes written by lla_encode_rope_keys (same block table)
+ *   q_rope       device [B][H][d_rope] io_dtype: pre-rotation rotary queries
+ *   cur_k_rope   device [B][d_rope] io_dtype, pass 1 (with cur_k, cur_v): the current token's
+ *                pre-rotation rotary key; NULL in pass 2
+ *   workspace    >= lla_decode_decoupled_workspace_size bytes; overwritten (no zero fill)
+ * Other arguments and the error behaviour are those of lla_decode_attn; three launches on
+ * `stream`.  Storage LLA_BF16, d = 128, H <= 64, (r_k, r_v) = (96, 160), d_rope 32 or 64;
+ * LLA_ERR_UNSUPPORTED otherwise.
+ */
+lla_status lla_decode_attn_decoupled(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                                     const void *rope_pool, int32_t d_rope, const lla_rope *rope,
+                                     const int32_t *context_lens, int32_t B, int32_t max_ctx, int32_t loop,
+                                     const void *q, const void *q_rope, const void *cur_k, const void *cur_v,
+                                     const void *cur_k_rope, lla_dtype io_dtype, void *out, void *workspace,
+                                     size_t workspace_bytes, void *stream);
 
 /*
  * lla_decode_attn for callers that cannot allocate device memory (for example a plug-in inside a

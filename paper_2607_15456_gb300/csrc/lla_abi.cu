@@ -375,6 +375,90 @@ lla_status lla_decode_attn_2d(const lla_geometry *g, const lla_codec *codec, con
     return launch_decode_2d(a, static_cast<cudaStream_t>(stream));
 }
 
+lla_status lla_rope_plane_bytes(int32_t d_rope, size_t *bytes) {
+    if (!bytes || d_rope < 16 || d_rope > 96 || d_rope % 16 != 0) return LLA_ERR_INVALID_ARG;
+    *bytes = static_cast<size_t>(LLA_BLOCK_TOKENS) * d_rope * 2;
+    return LLA_OK;
+}
+
+namespace {
+bool valid_rope(const lla_rope *rope) {
+    return rope && rope->base > 1.0 && rope->base < 1e300 &&
+           (rope->pairing == LLA_ROPE_HALF || rope->pairing == LLA_ROPE_ADJACENT);
+}
+}  // namespace
+
+lla_status lla_encode_rope_keys(int32_t d_rope, const lla_rope *rope, void *rope_pool, int64_t num_blocks,
+                                const void *k_rope, lla_dtype x_dtype, const int32_t *positions,
+                                const int64_t *slot_mapping, int32_t N, void *stream) {
+    if (d_rope < 16 || d_rope > 96 || d_rope % 16 != 0 || !valid_rope(rope)) return LLA_ERR_INVALID_ARG;
+    if (!rope_pool || num_blocks < 1 || !aligned(rope_pool, 16) || !valid_dtype(x_dtype) || N < 0)
+        return LLA_ERR_INVALID_ARG;
+    if (N > 0 && (!k_rope || !positions || !slot_mapping)) return LLA_ERR_INVALID_ARG;
+    return launch_rope_key_store(d_rope, rope->base, rope->pairing == LLA_ROPE_ADJACENT ? 1 : 0, rope_pool,
+                                 num_blocks, k_rope, x_dtype == LLA_BF16, positions, slot_mapping, N,
+                                 static_cast<cudaStream_t>(stream));
+}
+
+lla_status lla_decode_decoupled_workspace_size(const lla_geometry *g, int32_t d_rope, int32_t B,
+                                               size_t *bytes) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
+    if (!decode_decoupled_supported(elem_size(g->storage), g->d, g->H, g->r_k, g->r_v, d_rope))
+        return LLA_ERR_UNSUPPORTED;
+    const size_t n = decode_decoupled_workspace_bytes(g->r_k, g->r_v, d_rope, B, g->H);
+    if (n == 0) return LLA_ERR_CUDA;
+    *bytes = n;
+    return LLA_OK;
+}
+
+lla_status lla_decode_attn_decoupled(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
+                                     const void *rope_pool, int32_t d_rope, const lla_rope *rope,
+                                     const int32_t *context_lens, int32_t B, int32_t max_ctx, int32_t loop,
+                                     const void *q, const void *q_rope, const void *cur_k, const void *cur_v,
+                                     const void *cur_k_rope, lla_dtype io_dtype, void *out, void *workspace,
+                                     size_t workspace_bytes, void *stream) {
+    lla_status st = check_geometry(g);
+    if (st != LLA_OK) return st;
+    if ((st = check_cache(cache, true)) != LLA_OK) return st;
+    if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;
+    if (!aligned(codec->w_up_k, 16) || !aligned(codec->w_up_v, 16)) return LLA_ERR_INVALID_ARG;
+    if (loop < 0 || loop >= g->T) return LLA_ERR_INVALID_ARG;
+    if (!valid_rope(rope) || !rope_pool || !aligned(rope_pool, 16)) return LLA_ERR_INVALID_ARG;
+    if (B < 0 || B > LLA_MAX_BATCH || !valid_dtype(io_dtype)) return LLA_ERR_INVALID_ARG;
+    if (max_ctx < 0 || static_cast<int64_t>(max_ctx) >
+                           static_cast<int64_t>(cache->max_blocks_per_seq) * LLA_BLOCK_TOKENS)
+        return LLA_ERR_INVALID_ARG;
+    if ((cur_k == nullptr) != (cur_v == nullptr) || (cur_k == nullptr) != (cur_k_rope == nullptr))
+        return LLA_ERR_INVALID_ARG;
+    if (B > 0 && (!context_lens || !q || !q_rope || !out)) return LLA_ERR_INVALID_ARG;
+    if (!decode_decoupled_supported(elem_size(g->storage), g->d, g->H, g->r_k, g->r_v, d_rope))
+        return LLA_ERR_UNSUPPORTED;
+    // the pages of every (sequence, head) are counted in 32 bits inside the kernels
+    if (static_cast<int64_t>(B) * g->H *
+            ((static_cast<int64_t>(max_ctx) + LLA_BLOCK_TOKENS - 1) / LLA_BLOCK_TOKENS) >= (int64_t(1) << 31))
+        return LLA_ERR_UNSUPPORTED;
+    if (B == 0) return LLA_OK;
+    if (!workspace) return LLA_ERR_INVALID_ARG;
+    DecodeArgs a = {};
+    a.T = g->T; a.H = g->H; a.d = g->d; a.r_k = g->r_k; a.r_v = g->r_v;
+    a.loop = loop;
+    a.absorbed = 1;
+    a.storage_bf16 = 1;
+    a.io_bf16 = io_dtype == LLA_BF16;
+    a.scale = g->scale;
+    a.w_up_k = codec->w_up_k; a.w_up_v = codec->w_up_v;
+    a.mu_k = codec->mu_k; a.mu_v = codec->mu_v;
+    a.pool = cache->pool; a.num_blocks = cache->num_blocks;
+    a.block_table = cache->block_table; a.max_blocks = cache->max_blocks_per_seq;
+    a.context_lens = context_lens; a.B = B; a.max_ctx = max_ctx;
+    a.q = q; a.cur_k = cur_k; a.cur_v = cur_v; a.out = out;
+    a.workspace = workspace; a.workspace_bytes = workspace_bytes;
+    return launch_decode_decoupled(a, rope_pool, d_rope, rope->base, rope->pairing == LLA_ROPE_ADJACENT ? 1 : 0,
+                                   q_rope, cur_k_rope, static_cast<cudaStream_t>(stream));
+}
+
 lla_status lla_dense_decode_attn(const lla_geometry *g, const lla_cache *cache,
                                  const int32_t *context_lens, int32_t B, int32_t max_ctx,
                                  const void *q, const void *cur_k, const void *cur_v,

@@ -29,9 +29,18 @@
 //   finish2d_kernel   per (head, up to 8 sequences): merges the runs of each sequence, adds the
 //                     pass-1 current token, and applies W_up,t,h^V once for those sequences
 // Storage bf16, d = 128, H <= 16; accumulators fp32 in TMEM.
+//
+// The same kernels take the decoupled rotary branch of per-head LLA (App. J "Absorbed
+// attention": an MLA-style NoPE content path plus a small explicit rotary branch shared across
+// recurrence steps for each token).  A unit is then one (sequence, head) with one query: its
+// pages are the head's latent pages, and its score operand is the head's K-plane followed by the
+// block's rotary plane (64 rotary keys of d_rope dims, turned at their positions when stored),
+// against [q~; rot(q^R, P)].  rope_key_store_kernel writes the rotary planes.
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
+#include <cstring>
 
 #include "lla_device.cuh"
 #include "lla_internal.h"
@@ -55,15 +64,18 @@ constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one sequence fit
 
 // Shared-memory plan of the attention kernel for ranks (RK, RV).  Offsets from a 1024-byte
 // aligned base (128-byte swizzle atoms of the V stages).
-template <int RK, int RV>
+template <int RK, int RV, int DR = 0>
 struct Z2 {
+    static constexpr int RKX = RK + DR;                 // score contraction: latent, then rotary key
+    static constexpr int NQM = DR > 0 ? 1 : kNQ;        // queries of a unit (LLA-2D: the heads)
     static constexpr int NCH = (RV + 127) / 128;        // 128-row chunks of O^T
     static constexpr int NBOX = (RV + 63) / 64;         // TMA boxes a V-plane loads
     static constexpr int BOX = kPT * 128;               // one box: 64 rows x 128 bytes
-    static constexpr int KPAGE = kPT * RK * 2;
+    static constexpr int KPLANE = kPT * RK * 2;
+    static constexpr int KPAGE = kPT * RKX * 2;         // K-plane, then the rotary plane
     static constexpr int VPAGE = NCH * 2 * BOX;         // two boxes per chunk, loaded or zero
     static constexpr int VBYTES = NBOX * BOX;
-    static constexpr int QB = kNS * RK * 2;             // [Q~_hi; Q~_lo] operand
+    static constexpr int QB = kNS * RKX * 2;            // [Q~_hi; Q~_lo] operand
     static constexpr int PBUF = kPT * kNQ * 2;          // P^T operand (one of two)
     static constexpr int RED = 1024;                    // maxima, sums, beta
     static constexpr int NBAR = 32;
@@ -81,8 +93,10 @@ struct Z2 {
     static constexpr uint32_t TM_S = 0, TM_O = 2 * kNS, TM_COLS = 128;
     static constexpr uint32_t IDESC_S = umma_idesc_bf16(64, kNS, 0, 0);
     static constexpr uint32_t IDESC_O = umma_idesc_bf16(128, kNQ, 1, 0);
-    static constexpr int PSTRIDE = kNQ * RV + 2 * kNQ;  // floats per run partial
-    static_assert(RK % 16 == 0 && RV % 32 == 0 && NCH <= 4, "ranks");
+    // a run partial: O^T of each query ([NQM][RV]), then 16 maxima and 16 sums
+    static constexpr int PSTRIDE = NQM * RV + 2 * kNQ;
+    static constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
+    static_assert(RK % 16 == 0 && DR % 16 == 0 && RV % 32 == 0 && NCH <= 4, "ranks");
     static_assert(ST >= 2, "pipeline depth");
     static_assert(SMEM <= kSmemCap, "shared memory");
     static_assert(TM_O + NCH * kNQ <= TM_COLS, "TMEM columns");
@@ -96,22 +110,31 @@ enum {
 };
 
 struct A2Params {
-    int T, H, loop, io_bf16, pass1, B, max_ctx, max_blocks, rk;
+    int T, H, loop, io_bf16, pass1, B, max_ctx, max_blocks;
+    int upr;         // units per sequence: 1 (LLA-2D) or H (decoupled: one unit per head)
+    int decoupled;   // per-head codec [H][T][d][r] with a rotary branch, else LLA-2D [T][H][d][r]
     float scale_log2;
-    const void *w_up_k;  // [T][H][d][r_k] bf16
-    const float *mu_k;   // [T*H*d] or NULL
+    const void *w_up_k;
+    const float *mu_k;   // LLA-2D [T*H*d], decoupled [H][T*d], or NULL
     const void *q;       // [B][H][d]
+    const void *q_rope;  // decoupled: [B][H][d_rope]
+    int d_rope, pairing;
+    unsigned long long phi[48];  // decoupled: theta_j in 64-bit fixed-point turns
     const int32_t *context_lens;
-    float *qt;           // [B][16][r_k]: q~ * scale * log2 e (rows >= H unused)
-    float *beta;         // [B][16]: beta * scale * log2 e
-    int *pstart;         // [B + 1]: first global page of each sequence
+    float *qt;           // [units][NQM][RK + DR]: q~ (and rot(q^R)) * scale * log2 e
+    float *beta;         // [units][NQM]: beta * scale * log2 e
+    int *pstart;         // [units + 1]: first global page of each unit
     unsigned *err;
 };
 
 struct T2Params {
-    int H, B;
+    int nq;   // queries of a unit: H (LLA-2D) or 1 (decoupled)
+    int upr;  // units per sequence; unit u is head u % upr of sequence u / upr
+    int B;    // units
     const char *pool;
     int64_t num_blocks, page_bytes;
+    const char *rope_pool;  // decoupled: [num_blocks][rotary plane]
+    int64_t rope_page_bytes;
     const int32_t *block_table;
     int max_blocks;
     const int32_t *context_lens;
@@ -125,14 +148,24 @@ struct T2Params {
 struct F2Params {
     int T, H, loop, io_bf16, B, grid;
     int spb;  // sequences per CTA (1 .. 8)
+    int upr, decoupled, d_rope;
     float scale_log2;
     const void *w_up_v;  // [T][H][d][r_v] bf16
     const float *mu_v;   // [T*H*d] or NULL
     const void *q, *cur_k, *cur_v;
+    const void *q_rope, *cur_k_rope;  // decoupled: [B][H][d_rope], [B][d_rope]
     void *out;
     const int *pstart;
     const float *part;
 };
+
+// (cos, sin) of pos turns of phi / 2^64 (phi = theta / 2 pi in 64-bit fixed point): the product
+// wraps modulo one turn exactly, and 32 bits of the fraction reach sincospif.
+__device__ __forceinline__ void turn_sincos(long long pos, unsigned long long phi, float *sn, float *cs) {
+    const unsigned long long turns = static_cast<unsigned long long>(pos) * phi;
+    const float tf = __uint2float_rn(static_cast<uint32_t>(turns >> 32)) * 2.3283064365386963e-10f;
+    sincospif(2.f * tf, sn, cs);
+}
 
 // CTA c of `grid` holds the global pages [page_lo(c), page_lo(c + 1)) of the np pages; with
 // fewer pages than CTAs some CTAs hold none.
@@ -147,29 +180,25 @@ __host__ __device__ __forceinline__ int cta_of(int g, int np, int grid) {
 
 // ------------------------------------------------------------------------- absorb kernel
 
-// One CTA: the page prefix sums of the batch (B <= 1024) with the length checks; an invalid
-// length counts as an empty sequence.
+// One CTA: the page prefix sums of the batch's units (unit u is head u % upr of sequence
+// u / upr) with the length checks; an invalid length counts as an empty sequence.
 __device__ void page_prefix(const A2Params &p) {
     __shared__ int wsum[8];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    int cnt[4], tot = 0;
+    const int U = p.B * p.upr;
+    const int per = (U + 255) / 256;  // units of this thread: [tid per, (tid + 1) per)
     const int limit = min(p.max_ctx, p.max_blocks * kPT);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int b = tid * 4 + k;
-        int c = 0;
-        if (b < p.B) {
-            const int L = p.context_lens[b];
-            if (L < 0 || L > limit) {
-                atomicOr(p.err, LLA_DEVERR_CONTEXT);
-            } else {
-                if (!p.pass1 && L == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
-                c = (L + kPT - 1) / kPT;
-            }
+    auto pages = [&](int u, bool flag) {
+        const int L = p.context_lens[u / p.upr];
+        if (L < 0 || L > limit) {
+            if (flag) atomicOr(p.err, LLA_DEVERR_CONTEXT);
+            return 0;
         }
-        cnt[k] = c;
-        tot += c;
-    }
+        if (flag && !p.pass1 && L == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
+        return (L + kPT - 1) / kPT;
+    };
+    int tot = 0;
+    for (int u = tid * per; u < min(U, (tid + 1) * per); ++u) tot += pages(u, u % p.upr == 0);
     int x = tot;  // inclusive scan over the warp
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -181,27 +210,34 @@ __device__ void page_prefix(const A2Params &p) {
     int pre = 0;
     for (int w = 0; w < warp; ++w) pre += wsum[w];
     int ex = pre + x - tot;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int b = tid * 4 + k;
-        if (b < p.B) p.pstart[b] = ex;
-        ex += cnt[k];
+    for (int u = tid * per; u < min(U, (tid + 1) * per); ++u) {
+        p.pstart[u] = ex;
+        ex += pages(u, false);
     }
-    if (tid == blockDim.x - 1) p.pstart[p.B] = pre + x;
+    if (tid == blockDim.x - 1) p.pstart[U] = pre + x;
 }
 
 // Grid (H, RK / 32, ceil(B / 16)), 256 threads = 32 columns x 8 slices of 16 rows of the head:
 // q~ of 32 columns of head h for 16 sequences, every weight load of a thread in flight at once;
-// beta of head h by the CTAs of the first column chunk.
-template <int RK>
+// beta of head h (and, with the rotary branch, rot(q^R, P)) by the CTAs of the first column
+// chunk.  The weight slice of (loop t, head h) is (t, h) of [T][H] for LLA-2D and (h, t) of
+// [H][T] for the per-head codec of the rotary branch.
+template <int RK, int DR>
 __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
     static_assert(RK % 32 == 0, "column chunks");
+    constexpr int RKX = RK + DR;
+    constexpr int NQM = DR > 0 ? 1 : kNQ;
     __shared__ float qs[16][kD];
     __shared__ float red[8][16][33];
     const int h = blockIdx.x, j0 = blockIdx.y * 32, b0 = blockIdx.z * 16, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(16, p.B - b0);
-    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
+    const int64_t th = p.decoupled ? static_cast<int64_t>(h) * p.T + p.loop
+                                   : static_cast<int64_t>(p.loop) * p.H + h;
+    // the output row of (sequence b, head h): query h of unit b, or query 0 of unit b H + h
+    auto row = [&](int b) {
+        return p.decoupled ? static_cast<int64_t>(b) * p.H + h : static_cast<int64_t>(b) * NQM + h;
+    };
     pdl_wait();  // inputs may come from the previous kernel; the workspace is free after it
     // this thread's 16 weights (column j0 + lane, rows 16 warp .. 16 warp + 15), in flight while
     // the queries load
@@ -229,16 +265,36 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
         float a = 0.f;
 #pragma unroll
         for (int sl = 0; sl < 8; ++sl) a += red[sl][bi][c];
-        if (bi < nb) p.qt[(static_cast<int64_t>(b0 + bi) * kNQ + h) * RK + j0 + c] = a * p.scale_log2;
+        if (bi < nb) p.qt[row(b0 + bi) * RKX + j0 + c] = a * p.scale_log2;
     }
-    // beta_h = q_h . mu^K_{t,h}: warp w takes sequences w and w + 8
     if (blockIdx.y == 0) {
+        // beta_h = q_h . mu^K_{t,h}: warp w takes sequences w and w + 8
         for (int bi = warp; bi < nb; bi += 8) {
             float s = 0.f;
             if (p.mu_k)
                 for (int e = lane; e < kD; e += 32) s = fmaf(qs[bi][e], p.mu_k[th * kD + e], s);
             s = warp_sum(s);
-            if (lane == 0) p.beta[static_cast<int64_t>(b0 + bi) * kNQ + h] = s * p.scale_log2;
+            if (lane == 0) p.beta[row(b0 + bi)] = s * p.scale_log2;
+        }
+        if constexpr (DR > 0) {
+            // the rotary query turned at the current token's position: context_lens[b] in
+            // pass 1, context_lens[b] - 1 in pass 2
+            constexpr int HP = DR / 2;
+            for (int i = tid; i < nb * HP; i += 256) {
+                const int bi = i / HP, j = i - bi * HP;
+                const int b = b0 + bi;
+                const int L = p.context_lens[b];
+                const long long P = max(0, p.pass1 ? L : L - 1);
+                float sn, cs;
+                turn_sincos(P, p.phi[j], &sn, &cs);
+                const int a = p.pairing ? 2 * j : j, c = p.pairing ? 2 * j + 1 : j + HP;
+                const int64_t src = (static_cast<int64_t>(b) * p.H + h) * DR;
+                const float x = load_elem(p.q_rope, src + a, p.io_bf16);
+                const float y = load_elem(p.q_rope, src + c, p.io_bf16);
+                float *dst = p.qt + row(b) * RKX + RK;
+                dst[a] = (x * cs - y * sn) * p.scale_log2;
+                dst[c] = (x * sn + y * cs) * p.scale_log2;
+            }
         }
     }
     __syncthreads();
@@ -258,10 +314,10 @@ __device__ __forceinline__ int first_seq(const int *pstart, int B, int g0) {
     return lo;
 }
 
-template <int RK, int RV>
+template <int RK, int RV, int DR>
 __global__ void __launch_bounds__(kT2, 1)
     attn2d_kernel(const __grid_constant__ CUtensorMap tv, const T2Params p) {
-    using Z = Z2<RK, RV>;
+    using Z = Z2<RK, RV, DR>;
     extern __shared__ __align__(1024) char sm_raw[];
     char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + Z::oBar);
@@ -320,7 +376,8 @@ __global__ void __launch_bounds__(kT2, 1)
                 const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
                 if (s0 >= g1) break;
                 const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
-                const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks;
+                const int32_t *bt = p.block_table + static_cast<int64_t>(b / p.upr) * p.max_blocks;
+                const int head = b % p.upr;
                 for (int pg = pa; pg < pe; ++pg, ++it) {
                     const int st = it % Z::ST;
                     const uint32_t ph = (it / Z::ST) & 1;
@@ -329,16 +386,20 @@ __global__ void __launch_bounds__(kT2, 1)
                         atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
                         blk = 0;
                     }
+                    const int64_t page = static_cast<int64_t>(blk) * p.upr + head;  // head page
                     mbar_wait(&bar[bKempty + st], ph ^ 1u, abort_flag, p.err);
                     mbar_arrive_expect_tx(&bar[bKfull + st], Z::KPAGE);
-                    bulk_g2s(sm + Z::oK + st * Z::KPAGE, p.pool + blk * p.page_bytes, Z::KPAGE,
-                             &bar[bKfull + st], pol);
+                    char *ks = sm + Z::oK + st * Z::KPAGE;
+                    bulk_g2s(ks, p.pool + page * p.page_bytes, Z::KPLANE, &bar[bKfull + st], pol);
+                    if constexpr (DR > 0)  // the block's rotary plane continues the K-plane
+                        bulk_g2s(ks + Z::KPLANE, p.rope_pool + blk * p.rope_page_bytes, Z::KPAGE - Z::KPLANE,
+                                 &bar[bKfull + st], pol);
                     mbar_wait(&bar[bVempty + st], ph ^ 1u, abort_flag, p.err);
                     mbar_arrive_expect_tx(&bar[bVfull + st], Z::VBYTES);
                     char *vs = sm + Z::oV + st * Z::VPAGE;
 #pragma unroll
                     for (int a = 0; a < Z::NBOX; ++a)
-                        tma_load_3d(vs + a * Z::BOX, &tv, a * 64, 0, blk, &bar[bVfull + st]);
+                        tma_load_3d(vs + a * Z::BOX, &tv, a * 64, 0, static_cast<int>(page), &bar[bVfull + st]);
                 }
             }
             // every copy has landed before the CTA can exit, even after an abort
@@ -390,7 +451,7 @@ __global__ void __launch_bounds__(kT2, 1)
                     tc_fence_after();
                     const uint64_t dk = dk0 + static_cast<uint64_t>((st * Z::KPAGE) >> 4);
 #pragma unroll
-                    for (int ks = 0; ks < RK / 16; ++ks)
+                    for (int ks = 0; ks < Z::RKX / 16; ++ks)
                         umma_bf16(tmem + Z::TM_S + s * kNS, dk + ks * ((2 * kPT * 16) >> 4),
                                   dq + ks * ((2 * kNS * 16) >> 4), Z::IDESC_S, ks > 0);
                     umma_commit(&bar[bSfull + s]);
@@ -422,16 +483,16 @@ __global__ void __launch_bounds__(kT2, 1)
             if (s0 >= g1) break;
             const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
             if (pe <= pa) continue;
-            const int L = p.context_lens[b];
-            // q~ of the sequence as a K-major operand of 32 rows: row n = bf16(q~_n), row 16 + n =
+            const int L = p.context_lens[b / p.upr];
+            // q~ of the unit as a K-major operand of 32 rows: row n = bf16(q~_n), row 16 + n =
             // bf16(q~_n - row n), granule g of row n at g*512 + n*16; and beta
             if (r > 0) mbar_wait(&bar[bQfree], (r - 1) & 1, abort_flag, p.err);
             {
-                const float4 *src = reinterpret_cast<const float4 *>(p.qt + static_cast<int64_t>(b) * kNQ * RK);
-                for (int i = st_tid; i < kNQ * (RK / 8); i += 128) {
-                    const int n = i / (RK / 8), g = i - n * (RK / 8);
+                const float4 *src = reinterpret_cast<const float4 *>(p.qt + static_cast<int64_t>(b) * Z::NQM * Z::RKX);
+                for (int i = st_tid; i < kNQ * (Z::RKX / 8); i += 128) {
+                    const int n = i / (Z::RKX / 8), g = i - n * (Z::RKX / 8);
                     uint4 hi = make_uint4(0, 0, 0, 0), lo = hi;
-                    if (n < p.H) {
+                    if (n < p.nq) {
                         const float4 a = src[2 * i], c4 = src[2 * i + 1];
                         const float v[8] = {a.x, a.y, a.z, a.w, c4.x, c4.y, c4.z, c4.w};
                         float r8[8];
@@ -446,7 +507,7 @@ __global__ void __launch_bounds__(kT2, 1)
                     *reinterpret_cast<uint4 *>(dq + n * 16) = hi;
                     *reinterpret_cast<uint4 *>(dq + (kNQ + n) * 16) = lo;
                 }
-                if (st_tid < kNQ) betas[st_tid] = st_tid < p.H ? p.beta[static_cast<int64_t>(b) * kNQ + st_tid] : 0.f;
+                if (st_tid < kNQ) betas[st_tid] = st_tid < p.nq ? p.beta[static_cast<int64_t>(b) * Z::NQM + st_tid] : 0.f;
             }
             fence_proxy_async_smem();
             mbar_arrive(&bar[bQready]);
@@ -575,8 +636,8 @@ __global__ void __launch_bounds__(kT2, 1)
                 const int j = ch * 128 + 32 * q4 + lane;
                 if (j < RV) {
 #pragma unroll
-                    for (int n = 0; n < kNQ; ++n)
-                        if (n < p.H) dst[n * RV + j] = o[n];
+                    for (int n = 0; n < Z::NQM; ++n)
+                        if (n < p.nq) dst[n * RV + j] = o[n];
                 }
             }
             tc_fence_before();
@@ -587,8 +648,8 @@ __global__ void __launch_bounds__(kT2, 1)
 #pragma unroll
                 for (int n = 0; n < kNQ; ++n)
                     if (st_tid == n) mine = m[n];
-                dst[kNQ * RV + st_tid] = mine;
-                dst[kNQ * RV + kNQ + st_tid] = (lsum[st_tid] + lsum[16 + st_tid]) + (lsum[32 + st_tid] + lsum[48 + st_tid]);
+                dst[Z::PO_M + st_tid] = mine;
+                dst[Z::PO_L + st_tid] = (lsum[st_tid] + lsum[16 + st_tid]) + (lsum[32 + st_tid] + lsum[48 + st_tid]);
             }
             named_bar_sync(1, 128);  // lsum and red are free for the next run
             ++r;
@@ -607,9 +668,11 @@ __global__ void __launch_bounds__(kT2, 1)
 
 // Grid (H, ceil(B / spb)), 128 threads (thread e = output element e of head h).  spb (at most 8)
 // sequences share one pass over W_up,t,h^V; small batches take fewer per CTA to use more SMs.
-template <int RV>
+// (Sequence b, head h) is query h of unit b (LLA-2D) or query 0 of unit b H + h (decoupled).
+template <int RV, int NQM>
 __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
-    constexpr int PS = kNQ * RV + 2 * kNQ;
+    constexpr int PS = NQM * RV + 2 * kNQ;
+    constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
     __shared__ __align__(16) float ob[kFinishSeqs][RV];
     __shared__ float wts[kMaxGrid];
     __shared__ float coef[kFinishSeqs][3];
@@ -617,26 +680,29 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     const int h = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(p.spb, p.B - b0);
-    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
+    const int64_t th = p.decoupled ? static_cast<int64_t>(h) * p.T + p.loop
+                                   : static_cast<int64_t>(p.loop) * p.H + h;
+    const int qn = p.decoupled ? 0 : h;  // the query of (b, h) within its unit
     pdl_wait();
-    const int NP = p.pstart[p.B];
+    const int NP = p.pstart[p.B * p.upr];
     for (int bi = 0; bi < kFinishSeqs; ++bi) {
         if (bi >= nb) {
             for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
             continue;
         }
         const int b = b0 + bi;
-        const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+        const int u = p.decoupled ? b * p.upr + h : b;  // the unit of (b, h)
+        const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
         float M = -INFINITY, l = 0.f;
         if (s1 > s0) {
-            // the runs of sequence b: the CTAs c0 .. c1 that hold pages (a CTA between them may
-            // hold none and writes nothing), partials at slots b + c
+            // the runs of unit u: the CTAs c0 .. c1 that hold pages (a CTA between them may
+            // hold none and writes nothing), partials at slots u + c
             const int c0 = cta_of(s0, NP, p.grid), c1 = cta_of(s1 - 1, NP, p.grid);
             const int nr = c1 - c0 + 1;
             float mm = -INFINITY;
             for (int i = tid; i < nr; i += 128)
                 if (page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid))
-                    mm = fmaxf(mm, p.part[static_cast<int64_t>(b + c0 + i) * PS + kNQ * RV + h]);
+                    mm = fmaxf(mm, p.part[static_cast<int64_t>(u + c0 + i) * PS + PO_M + qn]);
             mm = warp_max(mm);
             if (lane == 0) redm[warp] = mm;
             __syncthreads();
@@ -645,9 +711,9 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
             for (int i = tid; i < nr; i += 128) {
                 float w = 0.f;  // no run: weight 0, and its slot is never read
                 if (page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid)) {
-                    const float *pr = p.part + static_cast<int64_t>(b + c0 + i) * PS + kNQ * RV;
-                    w = ex2_approx(pr[h] - M);
-                    ls = fmaf(w, pr[kNQ + h], ls);
+                    const float *pr = p.part + static_cast<int64_t>(u + c0 + i) * PS;
+                    w = ex2_approx(pr[PO_M + qn] - M);
+                    ls = fmaf(w, pr[PO_L + qn], ls);
                 }
                 wts[i] = w;
             }
@@ -655,7 +721,7 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
             if (lane == 0) reds[warp] = ls;
             __syncthreads();
             l = (reds[0] + reds[1]) + (reds[2] + reds[3]);
-            const float *pj = p.part + static_cast<int64_t>(b + c0) * PS + h * RV;
+            const float *pj = p.part + static_cast<int64_t>(u + c0) * PS + qn * RV;
             for (int j = tid; j < RV; j += 128) {
                 float a = 0.f;
                 int i = 0;
@@ -673,11 +739,15 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
         } else {
             for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
         }
-        // pass 1: the current token's score against its exact key
+        // pass 1: the current token's score against its exact key (with the rotary branch, also
+        // q^R . k^R_cur: both turn at the current position, so the rotation cancels)
         float sc = -INFINITY;
         if (p.cur_k) {
             const int64_t row = (static_cast<int64_t>(b) * p.H + h) * kD;
             float v = load_elem(p.q, row + tid, p.io_bf16) * load_elem(p.cur_k, row + tid, p.io_bf16);
+            if (p.decoupled && tid < p.d_rope)
+                v = fmaf(load_elem(p.q_rope, (static_cast<int64_t>(b) * p.H + h) * p.d_rope + tid, p.io_bf16),
+                         load_elem(p.cur_k_rope, static_cast<int64_t>(b) * p.d_rope + tid, p.io_bf16), v);
             v = warp_sum(v);
             __syncthreads();  // redm / reds are free
             if (lane == 0) reds[warp] = v;
@@ -753,41 +823,60 @@ struct WS2 {
 
 inline size_t al256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
-WS2 ws2_layout(int r_k, int r_v, int B, int grid) {
+// Workspace of U units: run partials, q~ rows, beta, page prefix sums.
+WS2 ws2_layout(int rkx, int r_v, int nqm, int U, int grid) {
     WS2 w;
     w.part = 0;
-    w.qt = al256(static_cast<size_t>(B + grid) * (kNQ * r_v + 2 * kNQ) * sizeof(float));
-    w.beta = w.qt + al256(static_cast<size_t>(B) * kNQ * r_k * sizeof(float));
-    w.pstart = w.beta + al256(static_cast<size_t>(B) * kNQ * sizeof(float));
-    w.total = w.pstart + al256(static_cast<size_t>(B + 1) * sizeof(int));
+    w.qt = al256(static_cast<size_t>(U + grid) * (nqm * r_v + 2 * kNQ) * sizeof(float));
+    w.beta = w.qt + al256(static_cast<size_t>(U) * nqm * rkx * sizeof(float));
+    w.pstart = w.beta + al256(static_cast<size_t>(U) * nqm * sizeof(float));
+    w.total = w.pstart + al256(static_cast<size_t>(U + 1) * sizeof(int));
     return w;
 }
 
-template <int RK, int RV>
-lla_status launch_2d(const DecodeArgs &a, cudaStream_t stream) {
-    using Z = Z2<RK, RV>;
+// The rotary branch of a decoupled call (unused by LLA-2D).
+struct Rotary {
+    const char *pool;  // [num_blocks][64 x d_rope] rotary planes
+    const void *q_rope, *cur_k_rope;
+    unsigned long long phi[48];
+    int pairing;
+};
+
+// theta_j = base^(-2j/d_rope) in 64-bit fixed-point turns (theta_j <= 1 rad < 1 turn).
+void rotary_phases(int d_rope, double base, unsigned long long *phi) {
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int j = 0; j < d_rope / 2; ++j)
+        phi[j] = static_cast<unsigned long long>(ldexp(pow(base, -2.0 * j / d_rope) / two_pi, 64));
+}
+
+template <int RK, int RV, int DR>
+lla_status launch_units(const DecodeArgs &a, const Rotary *rot, cudaStream_t stream) {
+    using Z = Z2<RK, RV, DR>;
+    constexpr bool kDec = DR > 0;
     lla_status st = LLA_OK;
     unsigned *err = device_error_word(&st);
     if (st != LLA_OK) return st;
     const int grid = num_sms();
     if (grid <= 0 || grid > kMaxGrid) return LLA_ERR_UNSUPPORTED;
-    const WS2 w = ws2_layout(RK, RV, a.B, grid);
+    const int upr = kDec ? a.H : 1;
+    const int U = a.B * upr;
+    const WS2 w = ws2_layout(Z::RKX, RV, Z::NQM, U, grid);
     if (a.workspace_bytes < w.total) return LLA_ERR_WORKSPACE;
     char *ws = static_cast<char *>(a.workspace);
     static bool configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
+        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV, DR>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
             cudaSuccess)
             return LLA_ERR_CUDA;
         configured[dev] = true;
     }
     const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
-    // the V-planes of every page: [num_blocks][64 tokens][r_v] bf16
+    // the V-planes of every head page: [num_blocks * upr][64 tokens][r_v] bf16
     CUtensorMap tv;
     const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT),
-                              static_cast<uint64_t>(a.num_blocks)};
+                              static_cast<uint64_t>(a.num_blocks) * upr};
     const uint64_t strides[2] = {static_cast<uint64_t>(RV) * 2, static_cast<uint64_t>(page_bytes)};
     const uint32_t box[3] = {64, kPT, 1};
     if (!encode_tmap_bf16(&tv, static_cast<const char *>(a.pool) + kPT * RK * 2, 3, dims, strides, box, true))
@@ -795,39 +884,103 @@ lla_status launch_2d(const DecodeArgs &a, cudaStream_t stream) {
 
     A2Params ap = {};
     ap.T = a.T; ap.H = a.H; ap.loop = a.loop; ap.io_bf16 = a.io_bf16; ap.pass1 = a.cur_k != nullptr;
-    ap.B = a.B; ap.max_ctx = a.max_ctx; ap.max_blocks = a.max_blocks; ap.rk = RK;
+    ap.B = a.B; ap.max_ctx = a.max_ctx; ap.max_blocks = a.max_blocks;
+    ap.upr = upr; ap.decoupled = kDec ? 1 : 0;
     ap.scale_log2 = a.scale * kLog2e;
     ap.w_up_k = a.w_up_k; ap.mu_k = a.mu_k; ap.q = a.q; ap.context_lens = a.context_lens;
+    if (kDec) {
+        ap.q_rope = rot->q_rope;
+        ap.d_rope = DR;
+        ap.pairing = rot->pairing;
+        memcpy(ap.phi, rot->phi, sizeof(ap.phi));
+    }
     ap.qt = reinterpret_cast<float *>(ws + w.qt);
     ap.beta = reinterpret_cast<float *>(ws + w.beta);
     ap.pstart = reinterpret_cast<int *>(ws + w.pstart);
     ap.err = err;
-    if ((st = launch_ex(absorb2d_kernel<RK>, dim3(a.H, RK / 32, (a.B + 15) / 16), 256, 0, stream, ap)) !=
+    if ((st = launch_ex(absorb2d_kernel<RK, DR>, dim3(a.H, RK / 32, (a.B + 15) / 16), 256, 0, stream, ap)) !=
         LLA_OK)
         return st;
 
     T2Params tp = {};
-    tp.H = a.H; tp.B = a.B;
+    tp.nq = kDec ? 1 : a.H; tp.upr = upr; tp.B = U;
     tp.pool = static_cast<const char *>(a.pool);
     tp.num_blocks = a.num_blocks; tp.page_bytes = page_bytes;
+    if (kDec) {
+        tp.rope_pool = rot->pool;
+        tp.rope_page_bytes = static_cast<int64_t>(kPT) * DR * 2;
+    }
     tp.block_table = a.block_table; tp.max_blocks = a.max_blocks;
     tp.context_lens = a.context_lens;
     tp.qt = ap.qt; tp.beta = ap.beta; tp.pstart = ap.pstart;
     tp.part = reinterpret_cast<float *>(ws + w.part);
     tp.err = err;
-    if ((st = launch_ex(attn2d_kernel<RK, RV>, dim3(grid), kT2, Z::SMEM, stream, tv, tp)) != LLA_OK)
+    if ((st = launch_ex(attn2d_kernel<RK, RV, DR>, dim3(grid), kT2, Z::SMEM, stream, tv, tp)) != LLA_OK)
         return st;
 
     F2Params fp = {};
     fp.T = a.T; fp.H = a.H; fp.loop = a.loop; fp.io_bf16 = a.io_bf16; fp.B = a.B; fp.grid = grid;
+    fp.upr = upr; fp.decoupled = kDec ? 1 : 0; fp.d_rope = DR;
     fp.scale_log2 = ap.scale_log2;
     fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
     fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
+    if (kDec) {
+        fp.q_rope = rot->q_rope;
+        fp.cur_k_rope = rot->cur_k_rope;
+    }
     fp.pstart = ap.pstart; fp.part = tp.part;
     // about two finish CTAs per SM: fewer sequences per CTA for small batches
     const int64_t want = static_cast<int64_t>(a.B) * a.H;
     fp.spb = static_cast<int>(std::min<int64_t>(kFinishSeqs, std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
-    return launch_ex(finish2d_kernel<RV>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
+    return launch_ex(finish2d_kernel<RV, Z::NQM>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
+}
+
+// ------------------------------------------------------------------------- rotary keys
+
+struct RKParams {
+    int N, d_rope, pairing, x_bf16;
+    char *pool;
+    int64_t num_blocks;
+    const void *k;  // [N][d_rope]
+    const int32_t *positions;
+    const int64_t *slots;
+    unsigned long long phi[48];
+    unsigned *err;
+};
+
+// One thread per (token, pair): k^R of token n turned at positions[n] (pair j by
+// positions[n] theta_j), written as bf16 at row slot % 64 of block slot / 64 in the granule
+// layout of a K-plane (granule g of row i at g*1024 + i*16).
+__global__ void __launch_bounds__(256) rope_key_store_kernel(const RKParams p) {
+    const int hp = p.d_rope / 2;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+    pdl_wait();
+    if (i < static_cast<int64_t>(p.N) * hp) {
+        const int n = static_cast<int>(i / hp), j = static_cast<int>(i - static_cast<int64_t>(n) * hp);
+        const int64_t slot = p.slots[n];
+        const int pos = p.positions[n];
+        if (slot >= 0) {
+            const int64_t blk = slot / kPT;
+            const int row = static_cast<int>(slot - blk * kPT);
+            if (blk >= p.num_blocks) {
+                atomicOr(p.err, LLA_DEVERR_SLOT);
+            } else if (pos < 0) {
+                atomicOr(p.err, LLA_DEVERR_CONTEXT);
+            } else {
+                float sn, cs;
+                turn_sincos(pos, p.phi[j], &sn, &cs);
+                const int a = p.pairing ? 2 * j : j, c = p.pairing ? 2 * j + 1 : j + hp;
+                const float x = load_elem(p.k, static_cast<int64_t>(n) * p.d_rope + a, p.x_bf16);
+                const float y = load_elem(p.k, static_cast<int64_t>(n) * p.d_rope + c, p.x_bf16);
+                char *plane = p.pool + blk * (static_cast<int64_t>(kPT) * p.d_rope * 2);
+                *reinterpret_cast<__nv_bfloat16 *>(plane + (a >> 3) * (kPT * 16) + row * 16 + (a & 7) * 2) =
+                    __float2bfloat16_rn(x * cs - y * sn);
+                *reinterpret_cast<__nv_bfloat16 *>(plane + (c >> 3) * (kPT * 16) + row * 16 + (c & 7) * 2) =
+                    __float2bfloat16_rn(x * sn + y * cs);
+            }
+        }
+    }
+    pdl_trigger();
 }
 
 }  // namespace
@@ -840,14 +993,58 @@ bool decode_2d_supported(int es, int d, int H, int r_k, int r_v) {
 size_t decode_2d_workspace_bytes(int r_k, int r_v, int B) {
     const int grid = num_sms();
     if (grid <= 0) return 0;
-    return ws2_layout(r_k, r_v, B, grid).total;
+    return ws2_layout(r_k, r_v, kNQ, B, grid).total;
+}
+
+bool decode_decoupled_supported(int es, int d, int H, int r_k, int r_v, int d_rope) {
+    return es == 2 && d == kD && H >= 1 && H <= 64 && r_k == 96 && r_v == 160 &&
+           (d_rope == 32 || d_rope == 64);
+}
+
+size_t decode_decoupled_workspace_bytes(int r_k, int r_v, int d_rope, int B, int H) {
+    const int grid = num_sms();
+    if (grid <= 0) return 0;
+    return ws2_layout(r_k + d_rope, r_v, 1, B * H, grid).total;
+}
+
+lla_status launch_decode_decoupled(const DecodeArgs &a, const void *rope_pool, int d_rope, double base,
+                                   int pairing, const void *q_rope, const void *cur_k_rope,
+                                   cudaStream_t stream) {
+    if (a.B == 0) return LLA_OK;
+    if (a.num_blocks * a.H >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // 32-bit TMA coordinate
+    Rotary rot = {};
+    rot.pool = static_cast<const char *>(rope_pool);
+    rot.q_rope = q_rope;
+    rot.cur_k_rope = cur_k_rope;
+    rot.pairing = pairing;
+    rotary_phases(d_rope, base, rot.phi);
+    if (a.r_k == 96 && a.r_v == 160 && d_rope == 32) return launch_units<96, 160, 32>(a, &rot, stream);
+    if (a.r_k == 96 && a.r_v == 160 && d_rope == 64) return launch_units<96, 160, 64>(a, &rot, stream);
+    return LLA_ERR_UNSUPPORTED;
+}
+
+lla_status launch_rope_key_store(int d_rope, double base, int pairing, void *rope_pool, int64_t num_blocks,
+                                 const void *k, int x_bf16, const int32_t *positions, const int64_t *slots,
+                                 int N, cudaStream_t stream) {
+    if (N == 0) return LLA_OK;
+    lla_status st = LLA_OK;
+    unsigned *err = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    RKParams rp = {};
+    rp.N = N; rp.d_rope = d_rope; rp.pairing = pairing; rp.x_bf16 = x_bf16;
+    rp.pool = static_cast<char *>(rope_pool); rp.num_blocks = num_blocks;
+    rp.k = k; rp.positions = positions; rp.slots = slots; rp.err = err;
+    rotary_phases(d_rope, base, rp.phi);
+    const int64_t total = static_cast<int64_t>(N) * (d_rope / 2);
+    if ((total + 255) / 256 > 0x7fffffff) return LLA_ERR_UNSUPPORTED;
+    return launch_ex(rope_key_store_kernel, dim3(static_cast<unsigned>((total + 255) / 256)), 256, 0, stream, rp);
 }
 
 lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream) {
     if (a.B == 0) return LLA_OK;
     if (a.num_blocks >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // 32-bit TMA coordinate
 #define LLA_2D(K, V) \
-    if (a.r_k == K && a.r_v == V) return launch_2d<K, V>(a, stream);
+    if (a.r_k == K && a.r_v == V) return launch_units<K, V, 0>(a, nullptr, stream);
     LLA_2D(96, 160)
     LLA_2D(128, 128)
     LLA_2D(288, 480)

@@ -101,6 +101,17 @@ lla_status launch_prefill_rope(const PrefillArgs &a, double base, int pairing, v
 bool decode_2d_supported(int es, int d, int H, int r_k, int r_v);
 size_t decode_2d_workspace_bytes(int r_k, int r_v, int B);
 lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream);
+// Per-head LLA decode with the decoupled rotary branch (App. J): the shapes with a kernel, the
+// workspace for B sequences of H heads, launch (rope_pool [num_blocks][64 x d_rope] rotary planes,
+// q_rope [B][H][d_rope], cur_k_rope [B][d_rope] in pass 1); and the rotary-key store.
+bool decode_decoupled_supported(int es, int d, int H, int r_k, int r_v, int d_rope);
+size_t decode_decoupled_workspace_bytes(int r_k, int r_v, int d_rope, int B, int H);
+lla_status launch_decode_decoupled(const DecodeArgs &a, const void *rope_pool, int d_rope, double base,
+                                   int pairing, const void *q_rope, const void *cur_k_rope,
+                                   cudaStream_t stream);
+lla_status launch_rope_key_store(int d_rope, double base, int pairing, void *rope_pool, int64_t num_blocks,
+                                 const void *k, int x_bf16, const int32_t *positions, const int64_t *slots,
+                                 int N, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached), 0 on failure
 

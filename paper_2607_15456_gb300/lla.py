@@ -92,6 +92,11 @@ def library() -> ctypes.CDLL:
             "lla_encode_2d": (I32, [P, P, P, P, P, I32, P, I32, P]),
             "lla_decode_2d_workspace_size": (I32, [P, I32, P]),
             "lla_decode_attn_2d": (I32, [P, P, P, P, I32, I32, I32, P, P, P, I32, P, P, SZ, P]),
+            "lla_rope_plane_bytes": (I32, [I32, P]),
+            "lla_encode_rope_keys": (I32, [I32, P, P, I64, P, I32, P, P, I32, P]),
+            "lla_decode_decoupled_workspace_size": (I32, [P, I32, I32, P]),
+            "lla_decode_attn_decoupled": (I32, [P, P, P, P, I32, P, P, I32, I32, I32, P, P, P, P, P, I32,
+                                                P, P, SZ, P]),
             "lla_get_device_error": (I32, [P, P]),
             "lla_clear_device_error": (I32, [P]),
         }
@@ -374,6 +379,48 @@ def lla_decode_attn_2d(geom: Geometry, codec: Codec, cache: Cache, context_lens:
         ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(context_lens), q.shape[0],
         max_ctx, loop, _ptr(q), _ptr(cur_k), _ptr(cur_v), _dtype_code(q), _ptr(out),
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def lla_rope_plane_bytes(d_rope: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check("lla_rope_plane_bytes", library().lla_rope_plane_bytes(d_rope, ctypes.byref(out)))
+    return out.value
+
+
+def lla_encode_rope_keys(d_rope: int, rope_base: float, rope_pairing: int, rope_pool: torch.Tensor,
+                         num_blocks: int, k_rope: torch.Tensor, positions: torch.Tensor,
+                         slot_mapping: torch.Tensor, stream=None) -> None:
+    """Rotary keys k_rope [N][d_rope], turned at positions [N] int32, into the rotary planes."""
+    rp = lla_rope(float(rope_base), int(rope_pairing))
+    N = k_rope.shape[0] if k_rope.dim() == 2 else 0
+    _check("lla_encode_rope_keys", library().lla_encode_rope_keys(
+        d_rope, ctypes.byref(rp), _ptr(rope_pool), num_blocks, _ptr(k_rope), _dtype_code(k_rope),
+        _ptr(positions), _ptr(slot_mapping), N, _stream(stream)))
+
+
+def lla_decode_decoupled_workspace_size(geom: Geometry, d_rope: int, B: int) -> int:
+    out = ctypes.c_size_t(0)
+    g = geom.c()
+    _check("lla_decode_decoupled_workspace_size", library().lla_decode_decoupled_workspace_size(
+        ctypes.byref(g), d_rope, B, ctypes.byref(out)))
+    return out.value
+
+
+def lla_decode_attn_decoupled(geom: Geometry, codec: Codec, cache: Cache, rope_pool: torch.Tensor,
+                              d_rope: int, rope_base: float, rope_pairing: int,
+                              context_lens: torch.Tensor, max_ctx: int, loop: int, q: torch.Tensor,
+                              q_rope: torch.Tensor, cur_k: Optional[torch.Tensor],
+                              cur_v: Optional[torch.Tensor], cur_k_rope: Optional[torch.Tensor],
+                              out: torch.Tensor, workspace: torch.Tensor, stream=None) -> None:
+    """Per-head LLA decode with the decoupled rotary branch; q, cur_k, cur_v, out [B][H][d],
+    q_rope [B][H][d_rope], cur_k_rope [B][d_rope] (pass 1) or None."""
+    g, cd, ch = geom.c(), codec.c(), cache.c()
+    rp = lla_rope(float(rope_base), int(rope_pairing))
+    _check("lla_decode_attn_decoupled", library().lla_decode_attn_decoupled(
+        ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), _ptr(rope_pool), d_rope, ctypes.byref(rp),
+        _ptr(context_lens), q.shape[0], max_ctx, loop, _ptr(q), _ptr(q_rope), _ptr(cur_k), _ptr(cur_v),
+        _ptr(cur_k_rope), _dtype_code(q), _ptr(out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def lla_dense_store(geom: Geometry, cache: Cache, k: torch.Tensor, v: torch.Tensor,

@@ -326,3 +326,44 @@ def test_encode_2d_argument_checks(lib):
     assert call(codec=_codec(lib, w_down_k=None)) == INVALID
     assert call(g=_g(lib, H=4096, d=128)) == UNSUPPORTED  # H d past the stack the encode takes
     assert call(N=0, xk=None, xv=None, slots=None) == OK
+
+
+def test_decoupled_argument_checks(lib):
+    so = lib.library()
+    n = ctypes.c_size_t(0)
+    assert so.lla_rope_plane_bytes(64, ctypes.byref(n)) == OK and n.value == 64 * 64 * 2
+    assert so.lla_rope_plane_bytes(40, ctypes.byref(n)) == INVALID
+    g = _g(lib)
+    for bad in (_g(lib, r_k=72, r_v=120), _g(lib, d=64), _g(lib, H=65), _g(lib, storage="fp32")):
+        assert so.lla_decode_decoupled_workspace_size(ctypes.byref(bad), 64, 4, ctypes.byref(n)) == UNSUPPORTED
+    assert so.lla_decode_decoupled_workspace_size(ctypes.byref(g), 48, 4, ctypes.byref(n)) == UNSUPPORTED
+
+    def call(g=None, B=4, max_ctx=128, loop=0, q=FAKE, qr=FAKE, ck=FAKE, cv=FAKE, ckr=FAKE, io=0,
+             out=FAKE, ws=FAKE, lens=FAKE, rope_pool=FAKE, d_rope=64, rope=None):
+        g = g or _g(lib)
+        codec, cache = _codec(lib), _cache(lib)
+        rope = rope or lib.lla_rope(10000.0, 0)
+        return so.lla_decode_attn_decoupled(ctypes.byref(g), ctypes.byref(codec), ctypes.byref(cache),
+                                            rope_pool, d_rope, ctypes.byref(rope), lens, B, max_ctx, loop,
+                                            q, qr, ck, cv, ckr, io, out, ws, 1 << 20, None)
+    assert call(ckr=None) == INVALID          # pass 1 needs the current rotary key
+    assert call(ck=None, cv=None) == INVALID  # pass 2 takes none
+    assert call(qr=None) == INVALID
+    assert call(rope_pool=None) == INVALID
+    assert call(rope=lib.lla_rope(1.0, 0)) == INVALID
+    assert call(rope=lib.lla_rope(10000.0, 5)) == INVALID
+    assert call(loop=4) == INVALID
+    assert call(max_ctx=4 * 64 + 1) == INVALID
+    assert call(d_rope=48) == UNSUPPORTED
+    assert call(g=_g(lib, r_k=128, r_v=128)) == UNSUPPORTED
+    assert call(B=0, q=None, qr=None, ck=None, cv=None, ckr=None, out=None, ws=None, lens=None) == OK
+
+    def enc(d_rope=64, N=8, k=FAKE, pos=FAKE, slots=FAKE, pool=FAKE, xdt=0, rope=None):
+        rope = rope or lib.lla_rope(10000.0, 1)
+        return so.lla_encode_rope_keys(d_rope, ctypes.byref(rope), pool, 10, k, xdt, pos, slots, N, None)
+    assert enc(d_rope=40) == INVALID
+    assert enc(pos=None) == INVALID
+    assert enc(pool=FAKE + 8) == INVALID
+    assert enc(N=-1) == INVALID
+    assert enc(rope=lib.lla_rope(0.5, 0)) == INVALID
+    assert enc(N=0, k=None, pos=None, slots=None) == OK
