@@ -32,10 +32,11 @@
 //
 // The same kernels take the decoupled rotary branch of per-head LLA (App. J "Absorbed
 // attention": an MLA-style NoPE content path plus a small explicit rotary branch shared across
-// recurrence steps for each token).  A unit is then one (sequence, head) with one query: its
-// pages are the head's latent pages, and its score operand is the head's K-plane followed by the
-// block's rotary plane (64 rotary keys of d_rope dims, turned at their positions when stored),
-// against [q~; rot(q^R, P)].  rope_key_store_kernel writes the rotary planes.
+// recurrence steps for each token).  The attention kernel's unit of work is then one (sequence,
+// head) with one query instead of one sequence with H queries: a unit's pages are the head's
+// latent pages, and its score operand is the head's K-plane followed by the block's rotary plane
+// (64 rotary keys of d_rope dims, turned at their positions when stored), against
+// [q~; rot(q^R, P)]; H up to 64.  rope_key_store_kernel writes the rotary planes.
 #include <cuda_runtime.h>
 
 #include <algorithm>
