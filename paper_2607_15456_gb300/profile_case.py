@@ -19,6 +19,18 @@ rope_prefill: the same prompts through lla_prefill_attn_rope (key rebuild, then 
         python -m paper_2607_15456_gb300.profile_case --case rope_prefill --workload ouro14_rho2 \\
         --prompts 4 --len 8192 --calls 1
 
+loops / decoupled: the same cache through lla_decode_attn_loops (all T loops of a layer per call)
+or lla_decode_attn_decoupled (rotary planes of d_rope = 64 stored first, one per layer):
+
+    ncu --set full --clock-control none -k regex:attn2d_kernel -s 2 -c 1 \\
+        python -m paper_2607_15456_gb300.profile_case --case decoupled --workload ouro14_rho4 --layers 2 --calls 10
+
+2d: LLA-2D on the stress2d workload's shape with `--batch` sequences (random latents written into
+two layers' pages; --batch 32 keeps a layer near 1 GB, above L2):
+
+    ncu --set full --clock-control none -k regex:attn2d_kernel -s 2 -c 1 \\
+        python -m paper_2607_15456_gb300.profile_case --case 2d --batch 32 --calls 8
+
 prefill: encodes `--prompts` prompts of `--len` tokens of a workload's ranks (tensor-core encode,
 one launch per axis), then runs `--calls` causal prefill calls over them:
 
@@ -47,9 +59,37 @@ def decode_case(args):
     torch.cuda.set_device(dev)
     bench = DecodeBench(args.workload, dev, layers=args.layers)
     w = bench.w
+    if args.case == "decoupled":
+        from paper_2607_15456_gb300 import workloads as W
+        d_rope = 64
+        plane = lla.lla_rope_plane_bytes(d_rope)
+        pos = torch.cat([torch.arange(L, dtype=torch.int32) for L in bench.lens]).to(dev)
+        slots = torch.cat([bench.pt.slots(b, range(L)) for b, L in enumerate(bench.lens)]).to(dev)
+        pools = []
+        for l in range(w.D):
+            pool = torch.empty(bench.pt.num_blocks * plane, dtype=torch.uint8, device=dev)
+            k = W.normal((sum(bench.lens), d_rope), w.seed, 500, l, device=dev)
+            lla.lla_encode_rope_keys(d_rope, 10000.0, lla.LLA_ROPE_HALF, pool, bench.pt.num_blocks, k, pos,
+                                     slots)
+            pools.append(pool)
+        qr = W.normal((bench.B, w.H, d_rope), w.seed, 501, device=dev)
+        ckr = W.normal((bench.B, d_rope), w.seed, 502, device=dev)
+        dws = torch.empty(lla.lla_decode_decoupled_workspace_size(bench.geom, d_rope, bench.B),
+                          dtype=torch.uint8, device=dev)
+    if args.case == "loops":
+        lws = torch.zeros(lla.lla_decode_loops_workspace_size(bench.geom, bench.B), dtype=torch.uint8,
+                          device=dev)
     for i in range(args.calls):
         l, t = i % w.D, (i // w.D) % w.T
-        if args.case == "rope":
+        if args.case == "decoupled":
+            lla.lla_decode_attn_decoupled(bench.geom, bench.codecs[l], bench.caches[l], pools[l], d_rope,
+                                          10000.0, lla.LLA_ROPE_HALF, bench.ctx, bench.max_ctx, t,
+                                          bench.q[l, t], qr, bench.cur_k[l, t], bench.cur_v[l, t], ckr,
+                                          bench.out[l, t], dws)
+        elif args.case == "loops":
+            lla.lla_decode_attn_loops(bench.geom, bench.codecs[l], bench.caches[l], bench.ctx, bench.max_ctx,
+                                      bench.q[l], bench.cur_k[l], bench.cur_v[l], bench.out[l], lws)
+        elif args.case == "rope":
             lla.lla_decode_attn_rope(bench.geom, bench.codecs[l], bench.caches[l], 10000.0,
                                      lla.LLA_ROPE_HALF, bench.ctx, bench.max_ctx, t, bench.q[l, t],
                                      bench.cur_k[l, t], bench.cur_v[l, t], bench.out[l, t],
@@ -65,6 +105,43 @@ def decode_case(args):
         raise SystemExit(f"device error word {err:#x}")
     print(f"profile case done: {args.workload}, {w.D} layers, {args.calls} decode calls, "
           f"{bench.decode_bytes_per_launch()} algorithmic bytes per decode launch")
+
+
+def case_2d(args):
+    import torch
+
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = W.WORKLOADS["stress2d_rho2133"]
+    lens = W.context_lengths(w, B=args.batch)
+    pt = W.page_table(lens, w.seed, extra_tokens=1)
+    table = pt.block_table.to(dev)
+    geom = lla.Geometry(w.T, w.H, w.d, w.r_k, w.r_v, "bf16")
+    layers = []
+    for l in range(2):
+        ck = W.normal((sum(lens), w.r_k), w.seed, 400, l, device=dev)
+        cv = W.normal((sum(lens), w.r_v), w.seed, 401, l, device=dev)
+        pool = W.pack_latent_pages(ck, cv, pt.block_table, lens, pt.num_blocks)
+        del ck, cv
+        codec = lla.Codec(**W.codec_tensors_2d(w.T, w.H, w.d, w.r_k, w.r_v, w.seed, l, device=dev))
+        layers.append((pool, codec, lla.Cache(pool, pt.num_blocks, table, pt.max_blocks)))
+    shape = (len(lens), w.H, w.d)
+    q, k, v = (W.normal(shape, w.seed, 402 + i, device=dev) for i in range(3))
+    out = torch.empty_like(q)
+    ctx = torch.tensor(lens, dtype=torch.int32, device=dev)
+    ws = torch.empty(lla.lla_decode_2d_workspace_size(geom, len(lens)), dtype=torch.uint8, device=dev)
+    for i in range(args.calls):
+        l, t = i % 2, (i // 2) % w.T
+        lla.lla_decode_attn_2d(geom, layers[l][1], layers[l][2], ctx, max(lens), t, q, k, v, out, ws)
+    torch.cuda.synchronize()
+    err = lla.lla_get_device_error()
+    if err:
+        raise SystemExit(f"device error word {err:#x}")
+    nbytes = sum(lens) * (w.r_k + w.r_v) * 2 + w.H * w.d * (w.r_k + w.r_v) * 2 + 4 * len(lens) * w.H * w.d * 2
+    print(f"profile case done: LLA-2D, B={len(lens)}, {args.calls} calls, {nbytes} algorithmic bytes per call")
 
 
 def prefill_case(args):
@@ -113,15 +190,19 @@ def prefill_case(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--case", choices=["decode", "rope", "prefill", "rope_prefill"], default="decode")
+    ap.add_argument("--case", choices=["decode", "rope", "loops", "decoupled", "2d", "prefill", "rope_prefill"],
+                    default="decode")
     ap.add_argument("--workload", default="ouro14_rho4")
     ap.add_argument("--layers", type=int, default=2)
     ap.add_argument("--calls", type=int, default=10)
     ap.add_argument("--prompts", type=int, default=4)
     ap.add_argument("--len", type=int, default=8192)
+    ap.add_argument("--batch", type=int, default=32)
     args = ap.parse_args()
-    if args.case in ("decode", "rope"):
+    if args.case in ("decode", "rope", "loops", "decoupled"):
         decode_case(args)
+    elif args.case == "2d":
+        case_2d(args)
     else:
         prefill_case(args)
 
