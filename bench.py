@@ -268,6 +268,24 @@ class DecodeBench:
                 + self.B * w.H * (w.r_k + w.r_v) * 2)
 
 
+def max_over_ranks(values, world, device):
+    """Each value's maximum over the ranks (the slowest rank sets the whole job's time); with
+    one rank, the values themselves."""
+    if world <= 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_tokens_per_s(world, batch_per_rank, ms_per_step):
+    """Whole-job throughput: every rank decodes its own batch of `batch_per_rank` sequences
+    (replicas, weak scaling), one token each per step."""
+    return world * batch_per_rank / (ms_per_step / 1e3)
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -315,16 +333,13 @@ def run_ours(args, rank, world, local_rank):
     clocks = sampler.stop()
     total_ms = t_start.elapsed_time(t_end)
     dec_ms = sum(a.elapsed_time(b) for a, b in ev)
-    if world > 1:
-        t = torch.tensor([total_ms, dec_ms], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, dec_ms = float(t[0]), float(t[1])
+    total_ms, dec_ms = max_over_ranks([total_ms, dec_ms], world, device)
     err = lla.lla_get_device_error()
     if err != 0:
         raise RuntimeError(f"device error word {err:#x} after the timed region")
 
     ms_per_step = total_ms / K
-    value = world * bench.B / (ms_per_step / 1e3)
+    value = job_tokens_per_s(world, bench.B, ms_per_step)
     launches_dec = w.D * w.T
     dec_launch_s = dec_ms / 1e3 / (K * launches_dec)
     bytes_launch = bench.decode_bytes_per_launch()
@@ -765,13 +780,9 @@ def run_e2e(bench, args, world):
     b.record(main)
     torch.cuda.synchronize()
     bench.q, bench.cur_k, bench.cur_v, bench.out = bufs[0]
-    ms = a.elapsed_time(b)
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=bench.device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t[0])
+    ms = max_over_ranks([a.elapsed_time(b)], world, bench.device)[0]
     nbytes = lambda t: t.numel() * t.element_size()
-    return {"value": world * bench.B / (ms / K / 1e3), "unit": "tokens/s",
+    return {"value": job_tokens_per_s(world, bench.B, ms / K), "unit": "tokens/s",
             "h2d_bytes_per_step": nbytes(q_h) + nbytes(k_h) + nbytes(v_h),
             "d2h_bytes_per_step": nbytes(o_h[0]), "ms_per_step": ms / K,
             "copies": "double-buffered; inputs and outputs on their own streams, overlapping the "
