@@ -119,6 +119,9 @@ def _ptr(t: Optional[torch.Tensor]):
         return t
     if not t.is_contiguous():
         raise ValueError("tensors passed to liblla must be contiguous")
+    if not t.is_cuda:
+        # every buffer of the ABI is a device buffer: a host address would fault the kernel
+        raise ValueError("tensors passed to liblla must be CUDA tensors")
     return t.data_ptr()
 
 

@@ -367,3 +367,14 @@ def test_decoupled_argument_checks(lib):
     assert enc(N=-1) == INVALID
     assert enc(rope=lib.lla_rope(0.5, 0)) == INVALID
     assert enc(N=0, k=None, pos=None, slots=None) == OK
+
+
+def test_binding_rejects_host_tensors_before_any_launch(lib):
+    """A host tensor's address handed to a kernel would be an illegal device address: the binding
+    refuses it while marshalling."""
+    import torch
+    with pytest.raises(ValueError, match="CUDA tensors"):
+        lib._ptr(torch.zeros(4))
+    with pytest.raises(ValueError, match="contiguous"):
+        lib._ptr(torch.zeros(4, 4).t())
+    assert lib._ptr(None) is None and lib._ptr(FAKE) == FAKE
