@@ -83,6 +83,10 @@ typedef enum { LLA_BF16 = 0, LLA_F32 = 1 } lla_dtype;
 #define LLA_DEVERR_TIMEOUT 0x8u     /* a bounded wait expired */
 #define LLA_DEVERR_SLOT 0x10u       /* an encode slot outside the pool */
 
+/* Every wait of a kernel on its own pipeline (an mbarrier phase) gives up after this much global
+ * time, sets LLA_DEVERR_TIMEOUT and lets the launch finish with undefined outputs. */
+#define LLA_DEFAULT_WAIT_LIMIT_NS 2000000000ull
+
 /* Shape of the codec and the cache (Sec. 3; App. A "Models"). */
 typedef struct {
     int32_t T;          /* loops (recurrence steps), 1..16 */
@@ -375,10 +379,13 @@ lla_status lla_decode_attn_decoupled(const lla_geometry *g, const lla_codec *cod
  * counterpart; this is a deployment convenience.
  *   - Returns LLA_ERR_WORKSPACE (and enqueues nothing) when lla_decode_workspace_size for this
  *     geometry and B exceeds 1 MiB.
- *   - Every call shares the array and clears the part it uses (cudaMemsetAsync on `stream`);
- *     calls that can overlap on the GPU race on it: order them on one stream.
- *   - The first call on a device looks up the array's address with that device current; make
- *     that first call before any stream capture.
+ *   - Every call shares the array and clears the arrival counters in the part it uses
+ *     (cudaMemsetAsync on `stream`); the rest keeps the last call's bytes, which are always
+ *     overwritten before they are read.  Calls that can overlap on the GPU race on the array:
+ *     order them on one stream.
+ *   - The first call on a device looks up the array's address with that device current and
+ *     keeps it; make that first call before any stream capture.  After cudaDeviceReset the kept
+ *     address is stale: do not call this entry point on that device again.
  *   - Allocates nothing (no cudaMalloc, no cudaFree).
  */
 lla_status lla_decode_attn_noalloc(const lla_geometry *g, const lla_codec *codec,
@@ -422,6 +429,19 @@ lla_status lla_get_device_error(void *stream, uint32_t *word);
 
 /* Clears the device error word of the current device (enqueued on `stream`). */
 lla_status lla_clear_device_error(void *stream);
+
+/*
+ * Limit of each pipeline wait (a host helper; the paper has no counterpart) in
+ * the lla_decode_attn and lla_dense_decode_attn launches enqueued after this call, process-wide;
+ * 0 restores LLA_DEFAULT_WAIT_LIMIT_NS.  A wait that runs out sets LLA_DEVERR_TIMEOUT and the
+ * launch ends with undefined outputs: its producer issues no further copy and waits, with the
+ * default limit, for the copies it has in flight, and every other wait of that CTA returns at
+ * once.  The split-KV arrival counters still return to zero, so the workspace stays usable.
+ * Meant for watchdogs and for tests of the timeout path; a limit below the time a page takes to
+ * arrive makes every launch fail.  lla_get_wait_limit_ns returns the limit in force.
+ */
+lla_status lla_set_wait_limit_ns(uint64_t nanoseconds);
+uint64_t lla_get_wait_limit_ns(void);
 
 #ifdef __cplusplus
 }

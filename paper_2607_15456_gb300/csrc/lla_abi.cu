@@ -5,6 +5,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "lla_internal.h"
 
 namespace lla {
@@ -42,36 +44,46 @@ lla_status check_cache(const lla_cache *c, bool need_table) {
 
 }  // namespace
 
+// Per-device caches below are filled on first use; host threads may race to fill one, so each
+// entry is atomic (both racers store the same value).
 unsigned *device_error_word(lla_status *st) {
-    static unsigned *addr[kMaxDevices] = {};
+    static std::atomic<unsigned *> addr[kMaxDevices];
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev >= kMaxDevices) {
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
         *st = LLA_ERR_CUDA;
         return nullptr;
     }
-    if (!addr[dev]) {
+    unsigned *a = addr[dev].load(std::memory_order_acquire);
+    if (!a) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) {
             *st = LLA_ERR_CUDA;
             return nullptr;
         }
-        addr[dev] = static_cast<unsigned *>(p);
+        a = static_cast<unsigned *>(p);
+        addr[dev].store(a, std::memory_order_release);
     }
     *st = LLA_OK;
-    return addr[dev];
+    return a;
 }
 
 int num_sms() {
-    static int cached[kMaxDevices] = {};
+    static std::atomic<int> cached[kMaxDevices];
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev >= kMaxDevices) return 0;
-    if (!cached[dev]) {
-        int n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+    int n = cached[dev].load(std::memory_order_relaxed);
+    if (!n) {
         if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-        cached[dev] = n;
+        cached[dev].store(n, std::memory_order_relaxed);
     }
-    return cached[dev];
+    return n;
 }
+
+namespace {
+std::atomic<uint64_t> g_wait_limit_ns{0};  // 0: LLA_DEFAULT_WAIT_LIMIT_NS
+}  // namespace
+
+uint64_t pipeline_wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
 
 }  // namespace lla
 
@@ -579,6 +591,16 @@ lla_status lla_get_device_error(void *stream, uint32_t *word) {
     *word = host;
     if (host == 0) return LLA_OK;
     return (host & LLA_DEVERR_TIMEOUT) ? LLA_ERR_TIMEOUT : LLA_ERR_DEVICE_CHECK;
+}
+
+lla_status lla_set_wait_limit_ns(uint64_t nanoseconds) {
+    g_wait_limit_ns.store(nanoseconds, std::memory_order_relaxed);
+    return LLA_OK;
+}
+
+uint64_t lla_get_wait_limit_ns(void) {
+    const uint64_t v = g_wait_limit_ns.load(std::memory_order_relaxed);
+    return v ? v : LLA_DEFAULT_WAIT_LIMIT_NS;
 }
 
 lla_status lla_clear_device_error(void *stream) {

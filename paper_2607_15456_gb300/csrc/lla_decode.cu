@@ -75,7 +75,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
         for (int k = 0; k < VE; ++k) accv[k] = 0.f;
 
         for (int k = 0; k < R.npages; k += p.pps) {
-            mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+            mbar_wait(&s.full[stage], ph, s.abort_flag, p.err, wait_limit(p));
             const char *sb = s.ring + stage * p.stage_bytes;
             const int n = min(p.pps, R.npages - k);
             const int tok0 = (R.pg0 + k) * kBlockTokens;  // sequence position of row 0
@@ -255,7 +255,7 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
         float beta = 0.f;
         const float *qq = a.qlat + qslot * a.qslot + ks * F::NGT * F::KE;
         if (is_s) {
-            mbar_wait(&a.qready[qslot], (r / kQSlots) & 1, s.abort_flag, p.err);
+            mbar_wait(&a.qready[qslot], (r / kQSlots) & 1, s.abort_flag, p.err, wait_limit(p));
             beta = m_part(a, qslot, 1);
         }
         float m_run = -INFINITY, l_part = 0.f;
@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
             float *pring = s.psm + slot * kComputeThreads;
 
             if (is_s) {
-                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
+                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err, wait_limit(p));
                 float sc[F::TPT];
 #pragma unroll
                 for (int i = 0; i < F::TPT; ++i) {
@@ -333,7 +333,7 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
                 const float alpha = exp2f(m_run - m_new);
                 m_run = m_new;
                 if (ks == 0) {
-                    mbar_wait(&s.pempty[slot], pph ^ 1u, s.abort_flag, p.err);
+                    mbar_wait(&s.pempty[slot], pph ^ 1u, s.abort_flag, p.err, wait_limit(p));
                     float lsum = 0.f;
 #pragma unroll
                     for (int i = 0; i < F::TPT; ++i) {
@@ -346,8 +346,8 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
                 }
                 mbar_arrive(&s.pfull[slot]);
             } else {
-                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err);
-                mbar_wait(&s.pfull[slot], pph, s.abort_flag, p.err);
+                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err, wait_limit(p));
+                mbar_wait(&s.pfull[slot], pph, s.abort_flag, p.err, wait_limit(p));
                 if (vwork) value_step<ES, RK, RV>(accv, sb, pring, s.misc[kAPAlpha + slot], nvalid, vc, tg);
                 mbar_arrive(&s.pempty[slot]);
                 __syncwarp();
@@ -361,7 +361,7 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
 
         // leave the run's softmax state in slot rslot for the management warps, once the run
         // that used the slot before (r - 2) has been read
-        if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err);
+        if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err, wait_limit(p));
         if (is_s && ks == 0) a.lred[rslot * kLredSlot + tt] = l_part;
         if (tid == 0) s.misc[kAM + rslot] = m_run;
         if (vwork) value_store<ES, RK, RV>(a.red + rslot * a.redslot, accv, vc, tg);
@@ -415,10 +415,13 @@ FastEntry fast_entry(int es, int r_k, int r_v) {
 
 }  // namespace
 
-size_t decode_workspace_bytes(int r_v, int B, int H, int grid) {
+size_t decode_counters_offset(int r_v, int grid) {
     const size_t part = static_cast<size_t>(grid) * 2 * (r_v + 2) * sizeof(float);
-    const size_t part_al = (part + 255) & ~static_cast<size_t>(255);
-    return part_al + static_cast<size_t>(B) * H * sizeof(int);
+    return (part + 255) & ~static_cast<size_t>(255);
+}
+
+size_t decode_workspace_bytes(int r_v, int B, int H, int grid) {
+    return decode_counters_offset(r_v, grid) + static_cast<size_t>(B) * H * sizeof(int);
 }
 
 lla_status decode_fits(int r_k, int r_v, int es, int d) {
@@ -465,12 +468,12 @@ lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream) {
     p.block_table = a.block_table; p.max_blocks = a.max_blocks;
     p.context_lens = a.context_lens; p.B = a.B; p.max_ctx = a.max_ctx;
     p.q = a.q; p.cur_k = a.cur_k; p.cur_v = a.cur_v; p.out = a.out;
-    const size_t part = static_cast<size_t>(grid) * 2 * (a.r_v + 2) * sizeof(float);
-    const size_t part_al = (part + 255) & ~static_cast<size_t>(255);
     p.partials = static_cast<float *>(a.workspace);
-    p.counters = reinterpret_cast<int *>(static_cast<char *>(a.workspace) + part_al);
+    p.counters = reinterpret_cast<int *>(static_cast<char *>(a.workspace) +
+                                         decode_counters_offset(a.r_v, grid));
     p.pps = pps; p.stages = stages; p.stage_bytes = stage_bytes;
     p.err = err;
+    p.wait_ns = pipeline_wait_limit_ns();
 
     if (fe.launch) return fe.launch(p, grid, smem, stream);
 

@@ -371,15 +371,20 @@ __global__ void __launch_bounds__(kT2, 1)
     if (warp == 0) {
         // ------------------------------------------------------------------------- producer
         if (lane == 0) {
+            // after a failed wait (or once the abort flag is up) no further copy is issued, so no
+            // full barrier receives a second arrival in one phase; itk / itv count the K and V
+            // rounds issued, and the last ST of each are awaited below
             const uint64_t pol = policy_evict_first();
-            int it = 0;
-            for (int b = bfirst; b < p.B; ++b) {
+            int itk = 0, itv = 0;
+            bool stop = false;
+            for (int b = bfirst; b < p.B && !stop; ++b) {
                 const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
                 if (s0 >= g1) break;
                 const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
                 const int32_t *bt = p.block_table + static_cast<int64_t>(b / p.upr) * p.max_blocks;
                 const int head = b % p.upr;
-                for (int pg = pa; pg < pe; ++pg, ++it) {
+                for (int pg = pa; pg < pe; ++pg) {
+                    const int it = itk;
                     const int st = it % Z::ST;
                     const uint32_t ph = (it / Z::ST) & 1;
                     int32_t blk = bt[pg];
@@ -388,27 +393,35 @@ __global__ void __launch_bounds__(kT2, 1)
                         blk = 0;
                     }
                     const int64_t page = static_cast<int64_t>(blk) * p.upr + head;  // head page
-                    mbar_wait(&bar[bKempty + st], ph ^ 1u, abort_flag, p.err);
+                    if (!mbar_wait(&bar[bKempty + st], ph ^ 1u, abort_flag, p.err) || *abort_flag) {
+                        stop = true;
+                        break;
+                    }
                     mbar_arrive_expect_tx(&bar[bKfull + st], Z::KPAGE);
                     char *ks = sm + Z::oK + st * Z::KPAGE;
                     bulk_g2s(ks, p.pool + page * p.page_bytes, Z::KPLANE, &bar[bKfull + st], pol);
                     if constexpr (DR > 0)  // the block's rotary plane continues the K-plane
                         bulk_g2s(ks + Z::KPLANE, p.rope_pool + blk * p.rope_page_bytes, Z::KPAGE - Z::KPLANE,
                                  &bar[bKfull + st], pol);
-                    mbar_wait(&bar[bVempty + st], ph ^ 1u, abort_flag, p.err);
+                    ++itk;
+                    if (!mbar_wait(&bar[bVempty + st], ph ^ 1u, abort_flag, p.err) || *abort_flag) {
+                        stop = true;
+                        break;
+                    }
                     mbar_arrive_expect_tx(&bar[bVfull + st], Z::VBYTES);
                     char *vs = sm + Z::oV + st * Z::VPAGE;
 #pragma unroll
                     for (int a = 0; a < Z::NBOX; ++a)
                         tma_load_3d(vs + a * Z::BOX, &tv, a * 64, 0, static_cast<int>(page), &bar[bVfull + st]);
+                    ++itv;
                 }
             }
             // every copy has landed before the CTA can exit, even after an abort
             volatile int never = 0;
-            for (int j = max(0, it - Z::ST); j < it; ++j) {
+            for (int j = max(0, itk - Z::ST); j < itk; ++j)
                 mbar_wait(&bar[bKfull + j % Z::ST], (j / Z::ST) & 1, &never, p.err);
+            for (int j = max(0, itv - Z::ST); j < itv; ++j)
                 mbar_wait(&bar[bVfull + j % Z::ST], (j / Z::ST) & 1, &never, p.err);
-            }
         }
         __syncwarp();
     } else if (warp == 1) {

@@ -43,7 +43,12 @@ struct Params {
     int *counters;    // [B * H]
     int pps, stages, stage_bytes;
     unsigned *err;
+    uint64_t wait_ns;  // limit of each pipeline wait; 0 = kWaitLimitNs
 };
+
+__device__ __forceinline__ uint64_t wait_limit(const Params &p) {
+    return p.wait_ns ? p.wait_ns : kWaitLimitNs;
+}
 
 struct Layout {
     int ring, full, empty, pfull, pempty, prefix, lens, qlat, qfull, spart, psm, tmp, red, lred,
@@ -291,57 +296,73 @@ __device__ __forceinline__ void order_runs(const Params &p, const Smem &s, Range
 // Producer: the whole warp walks the CTA's range.  Block ids are fetched 32 pages at a time
 // (one per lane) so the copies of consecutive steps are issued back to back instead of each
 // waiting for its own block-table load; lane 0 issues the bulk copies.
+//
+// After a failed wait (or once another thread raised the abort flag) no further copy is issued:
+// a new round on a stage whose previous copies have not landed would arrive twice on one phase
+// of its full barrier.  Every round issued before that found its stage released by all consumer
+// warps with the flag still down, so its previous round had landed; the last `stages` issued
+// rounds are then awaited with the full limit, so no copy outlives the CTA.
 __device__ void producer(const Params &p, const Smem &s, const Range &rg) {
     const int lane = threadIdx.x & 31;
     const int hpb = p.head_page_bytes;
     const uint64_t pol = policy_evict_first();
-    int it = 0, st = 0;
+    int it = 0, st = 0;  // it: rounds issued
     uint32_t sph = 0;
-    for (int pass = 0; pass < 3; ++pass)
-    for (int64_t u = rg.lo[pass]; u < rg.hi[pass];) {
+    bool stop = false;
+    for (int pass = 0; pass < 3 && !stop; ++pass)
+    for (int64_t u = rg.lo[pass]; u < rg.hi[pass] && !stop;) {
         const Run R = locate_run(p, s, u, rg.hi[pass]);
         const int32_t *bt = p.block_table + static_cast<int64_t>(R.b) * p.max_blocks + R.pg0;
-        for (int k0 = 0; k0 < R.npages; k0 += 32) {
+        for (int k0 = 0; k0 < R.npages && !stop; k0 += 32) {
             const int32_t blk_lane = (k0 + lane < R.npages) ? bt[k0 + lane] : -1;
             const int kend = min(R.npages, k0 + 32);
-            for (int k = k0; k < kend; k += p.pps, ++it) {
+            for (int k = k0; k < kend; k += p.pps) {
                 const int stage = st;
                 const uint32_t ph = sph;
-                if (++st == p.stages) {
-                    st = 0;
-                    sph ^= 1u;
-                }
                 int32_t blk[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
                     blk[i] = __shfl_sync(0xffffffffu, blk_lane, (k - k0 + i) & 31);
+                int halt = 0;
                 if (lane == 0) {
-                    mbar_wait(&s.empty[stage], ph ^ 1u, s.abort_flag, p.err);
-                    const int n = min(p.pps, R.npages - k);
-                    uint32_t bytes = 0;
-                    for (int i = 0; i < n; ++i) {
-                        if (blk[i] < 0 || blk[i] >= p.num_blocks) {
-                            atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
-                            blk[i] = -1;
-                        } else {
-                            bytes += hpb;
+                    halt = !mbar_wait(&s.empty[stage], ph ^ 1u, s.abort_flag, p.err, wait_limit(p)) ||
+                           *s.abort_flag;
+                    if (!halt) {
+                        const int n = min(p.pps, R.npages - k);
+                        uint32_t bytes = 0;
+                        for (int i = 0; i < n; ++i) {
+                            if (blk[i] < 0 || blk[i] >= p.num_blocks) {
+                                atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                                blk[i] = -1;
+                            } else {
+                                bytes += hpb;
+                            }
                         }
+                        mbar_arrive_expect_tx(&s.full[stage], bytes);
+                        char *dst = s.ring + stage * p.stage_bytes;
+                        for (int i = 0; i < n; ++i)
+                            if (blk[i] >= 0)
+                                bulk_g2s(dst + i * hpb,
+                                         p.pool + blk[i] * p.block_bytes + static_cast<int64_t>(R.h) * hpb,
+                                         hpb, &s.full[stage], pol);
                     }
-                    mbar_arrive_expect_tx(&s.full[stage], bytes);
-                    char *dst = s.ring + stage * p.stage_bytes;
-                    for (int i = 0; i < n; ++i)
-                        if (blk[i] >= 0)
-                            bulk_g2s(dst + i * hpb,
-                                     p.pool + blk[i] * p.block_bytes + static_cast<int64_t>(R.h) * hpb,
-                                     hpb, &s.full[stage], pol);
                 }
-                __syncwarp();
+                if (__shfl_sync(0xffffffffu, halt, 0)) {
+                    stop = true;
+                    break;
+                }
+                ++it;
+                if (++st == p.stages) {
+                    st = 0;
+                    sph ^= 1u;
+                }
             }
         }
         u = R.run_end;
     }
     if (lane == 0 && *s.abort_flag) {
-        // let the copies still in flight land before the CTA exits
+        // let the copies still in flight land before the CTA exits (full limit, whatever the
+        // pipeline's limit was)
         volatile int never = 0;
         const int first = it > p.stages ? it - p.stages : 0;
         for (int j = first; j < it; ++j)
@@ -1027,7 +1048,7 @@ __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t 
                                          (static_cast<int64_t>(R.h) * p.T + p.loop) * D * RV * ES,
                                   0, mt);
     }
-    mbar_wait(&a.stfull[slot], parity, a.s.abort_flag, p.err);
+    mbar_wait(&a.stfull[slot], parity, a.s.abort_flag, p.err, wait_limit(p));
     const float *red = a.red + slot * a.redslot;
     const float *lred = a.lred + slot * kLredSlot;
     for (int j = mt; j < RV; j += kMThreads) {  // fixed order: bitwise-reproducible sums

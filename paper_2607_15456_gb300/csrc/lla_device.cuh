@@ -1,9 +1,11 @@
 // lla_device.cuh -- device helpers shared by the liblla kernels (sm_103a, inline PTX).
 //
-// mbarrier waits are bounded: a wait that has not completed within kWaitLimitNs of global
-// time sets LLA_DEVERR_TIMEOUT in the error word and reports failure, so no kernel here can
-// spin forever.  Callers keep going after a failed wait (with undefined results) so that
-// every CTA still reaches every barrier and exits.
+// mbarrier waits are bounded: a wait that has not completed within its limit (kWaitLimitNs of
+// global time unless the launch passes a shorter one) sets LLA_DEVERR_TIMEOUT in the error word
+// and reports failure, so no kernel here can spin forever.  Callers keep going after a failed
+// wait (with undefined results) so that every CTA still reaches every barrier and exits; a
+// producer stops issuing copies once a wait has failed and waits, with the full limit, for the
+// copies it has in flight before its CTA exits.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -14,7 +16,7 @@
 namespace lla {
 
 constexpr int kBlockTokens = LLA_BLOCK_TOKENS;
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s of global time per wait
+constexpr uint64_t kWaitLimitNs = LLA_DEFAULT_WAIT_LIMIT_NS;  // 2 s of global time per wait
 
 __device__ __forceinline__ uint64_t global_ns() {
     uint64_t t;
@@ -48,14 +50,15 @@ __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
 // for up to kSuspendNs (it does not spin and take issue slots from other warps).
 constexpr uint32_t kSuspendNs = 1000000;  // 1 ms
 
-__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity,
+                                              uint32_t suspend_ns = kSuspendNs) {
     uint32_t done;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(done)
-        : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
+        : "r"(smem_addr(bar)), "r"(parity), "r"(suspend_ns)
         : "memory");
     return done != 0;
 }
@@ -74,16 +77,20 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t *bar, uint32_t parity) {
 }
 
 // Bounded wait on phase `parity` of `bar`.  Returns false (and flags the error word) when the
-// wait expired or when `abort_flag` (shared) was already raised by another thread.
+// wait expired after `limit_ns` of global time, or at once when `abort_flag` (shared) was
+// already raised by another thread.  The flag is written before the caller's next arrival on
+// any barrier, so a thread that completes a phase those arrivals end sees it raised.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort_flag,
-                                          unsigned *err) {
+                                          unsigned *err, uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_test_wait(bar, parity)) return true;  // already complete: no suspension
-    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    const uint32_t hint = limit_ns < kSuspendNs ? static_cast<uint32_t>(limit_ns) : kSuspendNs;
+    if (mbar_try_wait(bar, parity, hint)) return true;
     const uint64_t t0 = global_ns();
     for (;;) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait(bar, parity, hint)) return true;
         if (*abort_flag) return false;
-        if (global_ns() - t0 > kWaitLimitNs) {
+        if (global_ns() - t0 > limit_ns) {
             *abort_flag = 1;
             atomicOr(err, LLA_DEVERR_TIMEOUT);
             return false;

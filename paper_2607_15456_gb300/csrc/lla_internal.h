@@ -66,7 +66,10 @@ inline size_t head_page_bytes(int r_k, int r_v, int es) {
     return static_cast<size_t>(LLA_BLOCK_TOKENS) * (r_k + r_v) * es;
 }
 
-// Decode: workspace bytes for `grid` CTAs and B sequences; launch.
+// Decode: workspace bytes for `grid` CTAs and B sequences (split-KV partial records, then the
+// B*H arrival counters from decode_counters_offset on, the only part that must start at zero);
+// launch.
+size_t decode_counters_offset(int r_v, int grid);
 size_t decode_workspace_bytes(int r_v, int B, int H, int grid);
 lla_status decode_fits(int r_k, int r_v, int es, int d);  // UNSUPPORTED if no kernel shape fits
 lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream);
@@ -114,5 +117,9 @@ lla_status launch_rope_key_store(int d_rope, double base, int pairing, void *rop
                                  int N, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached), 0 on failure
+
+// The limit of each pipeline wait in lla_decode_attn / lla_dense_decode_attn launches, as set by
+// lla_set_wait_limit_ns (0: the kernels' own 2 s).
+uint64_t pipeline_wait_limit_ns();
 
 }  // namespace lla

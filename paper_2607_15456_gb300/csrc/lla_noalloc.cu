@@ -16,13 +16,19 @@
 //     Calls that can overlap on the GPU (unordered streams, several host threads) race on it and
 //     produce wrong results: order them on one stream.
 //   * The first call on a device looks up the array's device address with cudaGetSymbolAddress,
-//     with that device current.  Make that first call before any stream capture.
-//   * Every call clears the part of the array it uses (cudaMemsetAsync on the caller's stream),
-//     because the arrival counters must start at zero.  That clear is enqueued before
+//     with that device current, and keeps it for later calls.  Make that first call before any
+//     stream capture.  The kept address belongs to the device's current context: after
+//     cudaDeviceReset it is stale, and the library must not be called on that device again.
+//   * Every call clears the arrival counters (the B*H integers at the end of its part of the
+//     array, cudaMemsetAsync on the caller's stream), because they must start at zero.  The
+//     split-KV partial records before them are always written before they are read, so stale
+//     bytes there from an earlier call are never seen.  The clear is enqueued before
 //     lla_decode_attn checks its remaining arguments, so a call rejected there leaves only the
 //     clear of this library-owned array behind.
 //   * Nothing here calls cudaMalloc, cudaFree or any allocating library routine.
 #include <cuda_runtime.h>
+
+#include <atomic>
 
 #include "lla_internal.h"
 
@@ -35,16 +41,19 @@ constexpr int kMaxDevices = 64;
 // stand-in symbol.  scratch_address() returns the real device address.
 static __device__ __align__(256) unsigned char g_decode_scratch[kScratchBytes];
 
+// Host threads may make their first calls at the same time: every entry is atomic, and two
+// threads that both look the address up store the same value.
+std::atomic<void *> g_scratch_addr[kMaxDevices];
+
 lla_status scratch_address(void **out) {
-    static void *addr[kMaxDevices] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return LLA_ERR_CUDA;
-    if (!addr[dev]) {
-        void *p = nullptr;
+    void *p = g_scratch_addr[dev].load(std::memory_order_acquire);
+    if (!p) {
         if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess || !p) return LLA_ERR_CUDA;
-        addr[dev] = p;
+        g_scratch_addr[dev].store(p, std::memory_order_release);
     }
-    *out = addr[dev];
+    *out = p;
     return LLA_OK;
 }
 
@@ -61,7 +70,12 @@ extern "C" lla_status lla_decode_attn_noalloc(const lla_geometry *g, const lla_c
     if (need > kScratchBytes) return LLA_ERR_WORKSPACE;
     void *scratch = nullptr;
     if ((st = scratch_address(&scratch)) != LLA_OK) return st;
-    if (B > 0 && cudaMemsetAsync(scratch, 0, need, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    const int sms = lla::num_sms();
+    if (sms <= 0) return LLA_ERR_CUDA;
+    const size_t counters = lla::decode_counters_offset(g->r_v, sms);  // the counters start here
+    if (B > 0 && need > counters &&
+        cudaMemsetAsync(static_cast<char *>(scratch) + counters, 0, need - counters,
+                        static_cast<cudaStream_t>(stream)) != cudaSuccess)
         return LLA_ERR_CUDA;
     return lla_decode_attn(g, codec, cache, context_lens, B, max_ctx, loop, q, cur_k, cur_v,
                            io_dtype, out, scratch, kScratchBytes, stream);

@@ -99,6 +99,8 @@ def library() -> ctypes.CDLL:
                                                 P, P, SZ, P]),
             "lla_get_device_error": (I32, [P, P]),
             "lla_clear_device_error": (I32, [P]),
+            "lla_set_wait_limit_ns": (I32, [ctypes.c_uint64]),
+            "lla_get_wait_limit_ns": (ctypes.c_uint64, []),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -457,3 +459,11 @@ def lla_get_device_error(stream=None) -> int:
 
 def lla_clear_device_error(stream=None) -> None:
     _check("lla_clear_device_error", library().lla_clear_device_error(_stream(stream)))
+
+
+def lla_set_wait_limit_ns(nanoseconds: int) -> None:
+    _check("lla_set_wait_limit_ns", library().lla_set_wait_limit_ns(int(nanoseconds)))
+
+
+def lla_get_wait_limit_ns() -> int:
+    return int(library().lla_get_wait_limit_ns())

@@ -41,6 +41,17 @@ def test_library_exports_every_declared_symbol(lib):
     assert not missing, missing
 
 
+def test_wait_limit_is_a_host_setting(lib):
+    """The pipeline wait limit is kept on the host (no GPU call): 0 means the 2 s default."""
+    assert lib.lla_get_wait_limit_ns() == 2_000_000_000
+    lib.lla_set_wait_limit_ns(12345)
+    try:
+        assert lib.lla_get_wait_limit_ns() == 12345
+    finally:
+        lib.lla_set_wait_limit_ns(0)
+    assert lib.lla_get_wait_limit_ns() == 2_000_000_000
+
+
 def test_status_strings_and_version(lib):
     assert lib.lla_version() >= 100
     assert lib.lla_status_string(0) == "ok"

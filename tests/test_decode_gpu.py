@@ -313,3 +313,35 @@ def test_dense_comparator_matches_uncompressed_attention(lla, storage):
         off += L
     assert_parity(f64(out), ref, "bf16", "dense decode")
     assert lla.lla_get_device_error() == 0
+
+
+def test_a_wait_that_runs_out_is_reported_and_the_next_call_is_exact(lla):
+    """Failure detection without a GPU fault: with the pipeline wait limit set far below the
+    time a latent page takes to arrive from HBM, a wait of the decode launch runs out.  The
+    kernel sets LLA_DEVERR_TIMEOUT, its producer stops issuing copies and lets those in flight
+    land (with the default limit), every other wait returns at once, and the launch ends.  The
+    host reads the timeout; with the limit restored and the word cleared, the split-KV counters
+    are back at zero and the next call matches the oracle."""
+    sc = Scene(lla, H=16, lens=[4000, 3100, 2049, 700], io="bf16", seed=14)
+    lla.lla_clear_device_error()
+    word = 0
+    try:
+        lla.lla_set_wait_limit_ns(1)
+        assert lla.lla_get_wait_limit_ns() == 1
+        for _ in range(5):  # one launch nearly always suffices; the expiry depends on timing
+            sc.decode(0, pass1=True)
+            word = lla.lla_get_device_error()
+            if word & lla.LLA_DEVERR_TIMEOUT:
+                break
+    finally:
+        lla.lla_set_wait_limit_ns(0)
+    assert word & lla.LLA_DEVERR_TIMEOUT, hex(word)
+    assert word & ~lla.LLA_DEVERR_TIMEOUT == 0, hex(word)
+    assert lla.lla_get_wait_limit_ns() == 2_000_000_000
+    from paper_2607_15456_gb300 import lla as m
+    size = m.lla_decode_workspace_size(sc.geom, sc.B)
+    counters = sc.ws[size - sc.B * sc.H * 4:size].view(torch.int32)
+    assert int(counters.abs().sum()) == 0
+    lla.lla_clear_device_error()
+    _check_decode(sc, 1, pass1=True)
+    assert lla.lla_get_device_error() == 0
