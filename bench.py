@@ -49,6 +49,9 @@ def parse_args():
                    help="target CPU time of the oracle sample")
     p.add_argument("--no-extras", action="store_true",
                    help="skip the prefill, prefill-size encode and comparator measurements")
+    p.add_argument("--no-workloads", action="store_true",
+                   help="skip the other workloads' decode rows, the rho = 2 workload as written and "
+                        "the long prompt")
     return p.parse_args()
 
 
@@ -161,7 +164,13 @@ class ClockSampler:
 # ------------------------------------------------------------------------------- our arm
 
 class DecodeBench:
-    def __init__(self, wname: str, device, layers=None):
+    """One workload's model: D layers of codecs and paged latent caches, and the decode step's
+    inputs.  fill="encode" writes every cached token through lla_encode from N(0,1) stacked loop
+    vectors; fill="random" writes N(0,1) bf16 latents straight into the pages (the decode reads
+    the same bytes either way; used where encoding millions of tokens per layer would only add
+    set-up time).  extra_tokens reserves room for the tokens later steps append."""
+
+    def __init__(self, wname: str, device, layers=None, fill="encode", extra_tokens=1):
         import torch
         from paper_2607_15456_gb300 import lla
         from paper_2607_15456_gb300 import workloads as W
@@ -173,29 +182,35 @@ class DecodeBench:
             w = replace(w, D=layers)
         self.w = w
         self.device = device
+        self.fill = fill
         self.geom = lla.Geometry(w.T, w.H, w.d, w.r_k, w.r_v, w.storage)
         self.lens = W.context_lengths(w)
         self.B = len(self.lens)
-        # one page table for all layers (the next token's page is allocated too)
-        self.pt = W.page_table(self.lens, w.seed, extra_tokens=1)
+        # one page table for all layers (the pages of the tokens still to come are allocated too)
+        self.pt = W.page_table(self.lens, w.seed, extra_tokens=extra_tokens)
         self.table = self.pt.block_table.to(device)
         bb = lla.lla_cache_block_bytes(self.geom)
         self.codecs, self.caches, self.pools = [], [], []
-        slots_all = torch.cat([self.pt.slots(b, range(L)) for b, L in enumerate(self.lens)])
+        if fill == "encode":
+            slots_all = torch.cat([self.pt.slots(b, range(L)) for b, L in enumerate(self.lens)])
+            N = slots_all.numel()
         chunk = 1 << 17
-        N = slots_all.numel()
         for l in range(w.D):
             cod = W.codec_tensors(w.T, w.H, w.d, w.r_k, w.r_v, w.seed, l, dtype=torch.bfloat16,
                                   device=device)
             codec = lla.Codec(**cod)
-            pool = torch.empty(self.pt.num_blocks * bb, dtype=torch.uint8, device=device)
+            if fill == "random":
+                pool = W.random_pool(self.pt.num_blocks * bb, w.seed, 120, l, device=device)
+            else:
+                pool = torch.empty(self.pt.num_blocks * bb, dtype=torch.uint8, device=device)
             cache = lla.Cache(pool, self.pt.num_blocks, self.table, self.pt.max_blocks)
-            for ci, n0 in enumerate(range(0, N, chunk)):
-                n1 = min(N, n0 + chunk)
-                xk = W.normal((w.T, n1 - n0, w.H, w.d), w.seed, 100, l, ci, device=device)
-                xv = W.normal((w.T, n1 - n0, w.H, w.d), w.seed, 101, l, ci, device=device)
-                lla.lla_encode(self.geom, codec, cache, xk, xv, slots_all[n0:n1].to(device))
-                del xk, xv
+            if fill == "encode":
+                for ci, n0 in enumerate(range(0, N, chunk)):
+                    n1 = min(N, n0 + chunk)
+                    xk = W.normal((w.T, n1 - n0, w.H, w.d), w.seed, 100, l, ci, device=device)
+                    xv = W.normal((w.T, n1 - n0, w.H, w.d), w.seed, 101, l, ci, device=device)
+                    lla.lla_encode(self.geom, codec, cache, xk, xv, slots_all[n0:n1].to(device))
+                    del xk, xv
             self.codecs.append(codec)
             self.caches.append(cache)
             self.pools.append(pool)
@@ -266,6 +281,26 @@ class DecodeBench:
         w = self.w
         return (w.H * w.T * w.d * (w.r_k + w.r_v) * 2 + 2 * w.T * self.B * w.H * w.d * 2
                 + self.B * w.H * (w.r_k + w.r_v) * 2)
+
+
+def latent_cache_bytes(w, lens, extra_tokens=1) -> int:
+    """Bytes of the whole model's paged latent cache (D layers, every block of every sequence)."""
+    blocks = sum(max(1, -(-(L + extra_tokens) // 64)) for L in lens)
+    return w.D * blocks * w.H * 64 * (w.r_k + w.r_v) * 2
+
+
+def config_dict(w, lens, world) -> dict:
+    """The workload's description, printed identically by both arms of the benchmark."""
+    return {
+        "workload": w.name, "D": w.D, "H": w.H, "d_head": w.d, "T": w.T, "r_k": w.r_k,
+        "r_v": w.r_v, "rho": round(w.rho, 4), "batch_per_gpu": len(lens),
+        "context": list(w.lens), "sum_context": sum(lens), "block_tokens": 64,
+        "storage": "bf16 latents and codec weights, fp32 accumulation",
+        "step": f"{w.T}x{w.D} pass-1 lla_decode_attn calls + one lla_encode_layers call "
+                f"encoding the {len(lens)} completed tokens in all {w.D} layers",
+        "l2": "no flush: latent cache (%.1f GB) far larger than L2" % (latent_cache_bytes(w, lens) / 1e9),
+        "parallelism": f"replicas x{world} (independent batches)",
+    }
 
 
 def max_over_ranks(values, world, device):
@@ -360,17 +395,7 @@ def run_ours(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
-        "config": {
-            "workload": w.name, "D": w.D, "H": w.H, "d_head": w.d, "T": w.T, "r_k": w.r_k,
-            "r_v": w.r_v, "rho": round(w.rho, 4), "batch_per_gpu": bench.B,
-            "context": list(w.lens), "sum_context": sum(bench.lens), "block_tokens": 64,
-            "storage": "bf16 latents and codec weights, fp32 accumulation",
-            "step": f"{w.T}x{w.D} pass-1 lla_decode_attn calls + one lla_encode_layers call "
-                    f"encoding the {bench.B} completed tokens in all {w.D} layers",
-            "l2": "no flush: latent cache (%.1f GB) far larger than L2" %
-                  (len(bench.pools) * bench.pools[0].numel() / 1e9),
-            "parallelism": f"replicas x{world} (independent batches)",
-        },
+        "config": config_dict(w, bench.lens, world),
         "roofline": {
             "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
             "frac": achieved / peak, "traffic": ncu_traffic(w.name),
@@ -399,6 +424,15 @@ def run_ours(args, rank, world, local_rank):
         _extra(result, "prefill_encode_comparator", run_extras, device)
         torch.cuda.empty_cache()
         _extra(result, "lla2d_decode", run_2d_extra, device)
+        torch.cuda.empty_cache()
+    if not args.no_workloads and rank == 0:
+        _extra(result, "workloads", run_workload_rows, device, ("ouro14_rho2", "ouro26_rho533", "stress_rho2133"),
+               5, 2, 3.0, world == 1 and not args.no_cpu_baseline)
+        torch.cuda.empty_cache()
+        _extra(result, "rho2_as_written", run_rho2_as_written, device)
+        torch.cuda.empty_cache()
+        _extra(result, "long_prompt", run_long_prompt, device, 65536, False)
+        _extra(result, "long_prompt_rope", run_long_prompt, device, 65536, True)
     return result
 
 
@@ -718,6 +752,269 @@ def run_extras(device):
     return out
 
 
+def _dense_comparator(w, lens, device, reps=2):
+    """The uncompressed loop-t decode (same kernel, no codec) at the workload's full batch: the T
+    loop caches of one layer (N(0,1) bf16 keys and values, d = 128) resident, read by D x T
+    calls per step.  A whole model's teacher cache (D x T such caches) does not fit the GPU for
+    the larger workloads; every call still reads its whole cache from HBM (each is far larger
+    than L2), so the per-call time is that of a resident model."""
+    import torch
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+    peak, _ = measured_peaks()
+    B = len(lens)
+    dgeom = lla.Geometry(1, w.H, w.d, w.d, w.d, "bf16")
+    pt = W.page_table(lens, w.seed, extra_tokens=1)
+    table = pt.block_table.to(device)
+    bb = lla.lla_cache_block_bytes(dgeom)
+    caches = [lla.Cache(W.random_pool(pt.num_blocks * bb, w.seed, 130, t, device=device), pt.num_blocks,
+                        table, pt.max_blocks) for t in range(w.T)]
+    ctx = torch.tensor(lens, dtype=torch.int32, device=device)
+    qs = W.normal((w.T, B, w.H, w.d), w.seed, 131, device=device)
+    out = torch.empty_like(qs)
+    ws = torch.zeros(lla.lla_decode_workspace_size(dgeom, B), dtype=torch.uint8, device=device)
+
+    def sweep():
+        for _ in range(w.D):
+            for t in range(w.T):
+                lla.lla_dense_decode_attn(dgeom, caches[t], ctx, max(lens), qs[t], qs[t], qs[t], out[t], ws)
+    ms = _time_ms(sweep, reps=reps, warm=1)
+    per_launch_s = ms / 1e3 / (w.D * w.T)
+    nbytes = sum(lens) * w.H * 2 * w.d * 2 + 4 * B * w.H * w.d * 2
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the comparator measurement")
+    whole = w.D * w.T * sum(max(1, -(-(L + 1) // 64)) for L in lens) * bb
+    res = {"kernel": "decode_async_kernel<2,128,128> (lla_dense_decode_attn)",
+           "ms_per_step_decode_only": ms, "tokens_per_s_decode_only": B / (ms / 1e3),
+           "avg_launch_us": per_launch_s * 1e6, "GB_s": nbytes / per_launch_s / 1e9,
+           "hbm_frac": nbytes / per_launch_s / 1e9 / peak, "bytes_per_launch": nbytes,
+           "teacher_cache_GB": whole / 1e9,
+           "note": "one layer's T loop caches resident at full batch, read D x T times per step"}
+    del caches, qs, out, ws
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho2133"), steps=5,
+                      warmup=2, cpu_seconds=3.0, cpu=True):
+    """Decode throughput of the other Ouro-shaped workloads at full depth: D layers of latent
+    caches resident (N(0,1) bf16 latents written into the pages), one step = T x D pass-1
+    lla_decode_attn calls + one lla_encode_layers call, timed as the headline; beside it the
+    uncompressed comparator at the same batch and the oracle on a bounded sample of the step."""
+    import torch
+    from paper_2607_15456_gb300 import lla
+    peak, _ = measured_peaks()
+    out = {}
+    for name in names:
+        bench = DecodeBench(name, device, fill="random")
+        w = bench.w
+        for _ in range(warmup):
+            bench.step()
+        torch.cuda.synchronize()
+        stream = torch.cuda.current_stream()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for k in range(steps):
+            ev[k][0].record(stream)
+            bench.decode_calls()
+            ev[k][1].record(stream)
+            bench.encode_calls()
+        t1.record(stream)
+        torch.cuda.synchronize()
+        if lla.lla_get_device_error() != 0:
+            raise RuntimeError(f"device error in the {name} decode measurement")
+        ms = t0.elapsed_time(t1) / steps
+        dec_s = sum(a.elapsed_time(b) for a, b in ev) / 1e3 / (steps * w.D * w.T)
+        nbytes = bench.decode_bytes_per_launch()
+        row = {"config": config_dict(w, bench.lens, 1), "steps": steps, "warmup": warmup,
+               "kernel": "decode_async_kernel (lla_decode_attn)", "bound": "hbm",
+               "ms_per_step": ms, "tokens_per_s": bench.B / (ms / 1e3),
+               "avg_launch_us": dec_s * 1e6, "GB_s": nbytes / dec_s / 1e9,
+               "hbm_frac": nbytes / dec_s / 1e9 / peak, "frac_of_nominal_8tbs": nbytes / dec_s / 1e9 / NOMINAL_HBM_GBS,
+               "bytes_per_launch": nbytes, "latent_cache_GB": latent_cache_bytes(w, bench.lens) / 1e9,
+               "fill": "N(0,1) bf16 latents written into every page (the decode reads the same bytes "
+                       "as for encoded ones)"}
+        lens = bench.lens
+        del bench
+        torch.cuda.empty_cache()
+        row["comparator"] = _dense_comparator(w, lens, device, reps=1 if w.B >= 128 else 2)
+        if cpu:
+            row["cpu_baseline"] = cpu_baseline(w, lens, cpu_seconds)
+        out["decode_" + name] = row
+    return out
+
+
+def run_rho2_as_written(device, steps=None):
+    """The rho = 2 workload as it is written: a causal prefill of 4 prompts of 8192 tokens
+    through all 24 layers (lla_prefill_two_pass: each layer's pass-1 keys and values encoded, then
+    the loop-major pass-2 attention over the latents), then 256 decode steps at batch 32 whose
+    contexts grow from 8192 to 8447 (each step: T x D pass-1 calls, then the encode of the 32
+    completed tokens in every layer).  The 4 prefilled prompts are sequences 0..3 of the batch;
+    the other 28 hold N(0,1) latents.  Pass-1 captures are N(0,1) draws made before the timed
+    region (one per layer); pass-2 queries are one N(0,1) draw per loop, handed to every layer."""
+    import torch
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+    peak, _ = measured_peaks()
+    w = W.WORKLOADS["ouro14_rho2"]
+    nseq, Lp = w.prefill
+    steps = w.decode_steps if steps is None else steps
+    bench = DecodeBench("ouro14_rho2", device, fill="random", extra_tokens=steps + 1)
+    geom, pt = bench.geom, bench.pt
+    N = nseq * Lp
+    slots = torch.cat([pt.slots(b, range(Lp)) for b in range(nseq)]).to(device)
+    cu = torch.tensor([i * Lp for i in range(nseq + 1)], dtype=torch.int32, device=device)
+    caps = [(W.normal((w.T, N, w.H, w.d), w.seed, 140, l, device=device),
+             W.normal((w.T, N, w.H, w.d), w.seed, 141, l, device=device)) for l in range(w.D)]
+    qp = [W.normal((N, w.H, w.d), w.seed, 142, t, device=device) for t in range(w.T)]
+    op = torch.empty_like(qp[0])
+    # prefill tables: the 4 prompts' rows of the batch's block table
+    pcaches = [lla.Cache(c.pool, c.num_blocks, bench.table[:nseq].contiguous(), c.max_blocks_per_seq)
+               for c in bench.caches]
+    marks = {}
+
+    def capture(l):
+        return caps[l]
+
+    def query(l, t):
+        if l == 0 and t == 0:  # phase 1 (every layer encoded) ends here
+            marks["encoded"] = torch.cuda.Event(enable_timing=True)
+            marks["encoded"].record()
+        return qp[t], op
+
+    def prefill():
+        lla.lla_prefill_two_pass(geom, bench.codecs, pcaches, slots, cu, Lp, capture, query)
+
+    prefill()  # warm-up (rewrites the same latents)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    prefill()
+    b.record()
+    torch.cuda.synchronize()
+    pf_ms = a.elapsed_time(b)
+    enc_ms = a.elapsed_time(marks["encoded"])
+    del caps
+    torch.cuda.empty_cache()
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the rho = 2 prefill")
+    pairs = nseq * w.H * Lp * (Lp + 1) / 2
+    attn_flops = w.D * w.T * (pairs * 2 * (w.r_k + w.r_v) + N * w.H * 2 * w.d * (w.r_k + w.r_v))
+    enc_bytes = w.D * (2 * w.T * N * w.H * w.d * 2 + w.H * w.T * w.d * (w.r_k + w.r_v) * 2
+                       + N * w.H * (w.r_k + w.r_v) * 2)
+
+    # 256 decode steps, contexts L + s, the completed token of step s written at position L + s
+    base = torch.tensor(bench.lens, dtype=torch.int32)
+    ctx_all = torch.stack([base + s for s in range(steps)]).to(device)
+    slots_all = torch.stack([torch.stack([pt.slots(bb, [L + s])[0] for bb, L in enumerate(bench.lens)])
+                             for s in range(steps)]).to(device)
+
+    def run_steps(n, ev=None):
+        for s in range(n):
+            bench.ctx, bench.max_ctx, bench.next_slots = ctx_all[s], max(bench.lens) + s, slots_all[s]
+            if ev is not None:
+                ev[s][0].record()
+            bench.decode_calls()
+            if ev is not None:
+                ev[s][1].record()
+            bench.encode_calls()
+
+    run_steps(2)  # warm-up (the first two steps, repeated below with the same inputs)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    a.record()
+    run_steps(steps, ev)
+    b.record()
+    torch.cuda.synchronize()
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the rho = 2 decode steps")
+    dec_total_ms = a.elapsed_time(b)
+    dec_kernel_s = sum(x.elapsed_time(y) for x, y in ev) / 1e3
+    lat = sum((L + s) for s in range(steps) for L in bench.lens) * w.H * (w.r_k + w.r_v) * 2
+    dec_bytes = w.D * w.T * (lat + steps * (w.H * w.d * (w.r_k + w.r_v) * 2 + 4 * bench.B * w.H * w.d * 2))
+    B = bench.B
+    del bench, pcaches, qp, op
+    torch.cuda.empty_cache()
+    return {"rho2_as_written": {
+        "workload": f"{w.name}: prefill {nseq}x{Lp} through {w.D} layers (two-pass, streamed layer by "
+                    f"layer), then {steps} decode steps at B={B}, contexts {Lp} -> {Lp + steps - 1}",
+        "prefill_ms": pf_ms, "prefill_tokens_per_s": N / (pf_ms / 1e3),
+        "prefill_encode_phase_ms": enc_ms, "prefill_attention_phase_ms": pf_ms - enc_ms,
+        "prefill_attention_TFLOP_s": attn_flops / ((pf_ms - enc_ms) / 1e3) / 1e12,
+        "prefill_encode_GB_s": enc_bytes / (enc_ms / 1e3) / 1e9,
+        "decode_steps": steps, "decode_ms_per_step": dec_total_ms / steps,
+        "decode_tokens_per_s": B * steps / (dec_total_ms / 1e3),
+        "decode_kernel_GB_s": dec_bytes / dec_kernel_s / 1e9,
+        "decode_kernel_hbm_frac": dec_bytes / dec_kernel_s / 1e9 / peak,
+        "total_s": (pf_ms + dec_total_ms) / 1e3,
+        "kernels": "encode_tc_kernel + prefill_tc_kernel (lla_prefill_two_pass); decode_async_kernel + "
+                   "encode_layers_kernel (decode steps)"}}
+
+
+def run_long_prompt(device, L=65536, rope=False):
+    """One long prompt through the streamed two-pass prefill of the rho = 2 Ouro-1.4B geometry
+    (24 layers): the regime the layer-by-layer streaming exists for (App. J reaches 64k prompts
+    this way).  One layer's capture is live at a time; the same N(0,1) capture tensors stand in
+    for every layer's pass-1 keys and values, one N(0,1) query draw per loop for every layer."""
+    import torch
+    from paper_2607_15456_gb300 import lla
+    from paper_2607_15456_gb300 import workloads as W
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except Exception:
+        pass
+    tc_peak = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    w = W.WORKLOADS["ouro14_rho2"]
+    geom = lla.Geometry(w.T, w.H, w.d, w.r_k, w.r_v, "bf16")
+    pt = W.page_table([L], w.seed, extra_tokens=0)
+    table = pt.block_table.to(device)
+    bb = lla.lla_cache_block_bytes(geom)
+    codecs = [lla.Codec(**W.codec_tensors(w.T, w.H, w.d, w.r_k, w.r_v, w.seed, l, device=device))
+              for l in range(w.D)]
+    caches = [lla.Cache(torch.empty(pt.num_blocks * bb, dtype=torch.uint8, device=device), pt.num_blocks,
+                        table, pt.max_blocks) for _ in range(w.D)]
+    slots = pt.slots(0, range(L)).to(device)
+    cu = torch.tensor([0, L], dtype=torch.int32, device=device)
+    cap = (W.normal((w.T, L, w.H, w.d), w.seed, 150, device=device),
+           W.normal((w.T, L, w.H, w.d), w.seed, 151, device=device))
+    qp = [W.normal((L, w.H, w.d), w.seed, 152, t, device=device) for t in range(w.T)]
+    op = torch.empty_like(qp[0])
+    ws = None
+    if rope:
+        ws = torch.empty(lla.lla_prefill_rope_workspace_size(geom, 1, L), dtype=torch.uint8, device=device)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    lla.lla_prefill_two_pass(geom, codecs, caches, slots, cu, L, lambda l: cap, lambda l, t: (qp[t], op),
+                             rope_base=ROPE_BASE if rope else None, workspace=ws)
+    b.record()
+    torch.cuda.synchronize()
+    if lla.lla_get_device_error() != 0:
+        raise RuntimeError("device error in the long-prompt prefill")
+    ms = a.elapsed_time(b)
+    pairs = w.H * L * (L + 1) / 2
+    if rope:
+        flops = w.D * w.T * (pairs * 2 * (w.d + w.r_v) + L * w.H * 2 * w.d * (w.r_k + w.r_v))
+    else:
+        flops = w.D * w.T * (pairs * 2 * (w.r_k + w.r_v) + L * w.H * 2 * w.d * (w.r_k + w.r_v))
+    cap_gb = 2 * cap[0].numel() * 2 / 1e9
+    res = {"workload": f"one {L}-token prompt, {w.name} geometry ({w.D} layers, (r_k, r_v)=({w.r_k}, {w.r_v}))"
+                       + (", RoPE after reconstruction" if rope else ""),
+           "kernels": ("rope_rebuild_kernel + prefill_tc_kernel<ROPE>" if rope else "prefill_tc_kernel")
+                      + " + encode_tc_kernel (lla_prefill_two_pass)",
+           "ms": ms, "tokens_per_s": L / (ms / 1e3), "TFLOP_s": flops / (ms / 1e3) / 1e12,
+           "tensor_frac": flops / (ms / 1e3) / 1e12 / tc_peak,
+           "capture_live_GB": cap_gb, "captures_of_all_layers_GB_bf16": cap_gb * w.D,
+           "latent_cache_GB": w.D * pt.num_blocks * bb / 1e9,
+           "note": "TFLOP/s over the whole call (the encodes included) against sustained bf16"}
+    del caches, cap, qp, op, ws
+    torch.cuda.empty_cache()
+    return {("long_prompt_rope" if rope else "long_prompt"): res}
+
+
 def run_e2e(bench, args, world):
     """Same step with the step's inputs (q, k_cur, v_cur of every call) copied from pinned
     host memory and the outputs copied back, inside the timed region.  Inputs and outputs are
@@ -791,12 +1088,13 @@ def run_e2e(bench, args, world):
 
 # ----------------------------------------------------------------- oracle (CPU) timing
 
-def oracle_step_time(w, lens, target_s: float):
+def oracle_step_time(w, lens, target_s: float, detail: bool = False):
     """Times the CPU oracle on a bounded sample of one decode step and extrapolates to the
     whole step.  The sample is layer 0: pass-1 decode items (loop, sequence, head) in order
     until about target_s of work, plus the encode of the B completed tokens of layer 0.  The
     oracle's time depends on shapes only, so latents and activations are N(0,1) draws.
-    Returns (seconds per full step, sample description, threads)."""
+    Returns (seconds per full step, sample description, threads), and with detail also the
+    sample's own seconds and its share of the full step's work."""
     import numpy as np
 
     import oracle
@@ -843,6 +1141,10 @@ def oracle_step_time(w, lens, target_s: float):
               f"layer's decode work, plus the layer's encode of {len(lens)} tokens; extrapolated "
               f"linearly to the full step (work is linear in context length x heads x loops x "
               f"layers)")
+    if detail:
+        sample_s = secs + enc_s
+        frac = sample_s / step_s  # the sample's share of the full step's (linear) work
+        return step_s, sample, threads, sample_s, frac
     return step_s, sample, threads
 
 
@@ -853,27 +1155,35 @@ def cpu_baseline(w, lens, target_s):
 
 
 def run_reference(args, rank, world):
+    """The oracle as it stands on the host cores.  Each step is one bounded sample of the
+    workload's decode step (see oracle_step_time); ms_per_step is the sample's own time and
+    value the throughput that sample ran at (tokens of the full step x the sample's share of the
+    step's work / the sample's time), so steps x ms_per_step is the time actually measured."""
     from paper_2607_15456_gb300 import workloads as W
     w = W.WORKLOADS[args.workload]
     lens = W.context_lengths(w)
     per_step = max(2.0, min(args.cpu_seconds, 150.0 / max(1, args.steps + args.warmup)))
     for _ in range(args.warmup):
         oracle_step_time(w, lens, per_step)
-    times, sample, threads = [], "", 1
+    full, sample_s, share, sample, threads = [], [], [], "", 1
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        s, sample, threads = oracle_step_time(w, lens, per_step)
-        times.append(s)
+        s_full, sample, threads, secs, frac = oracle_step_time(w, lens, per_step, detail=True)
+        full.append(s_full)
+        sample_s.append(secs)
+        share.append(frac)
     wall = time.perf_counter() - t0
-    step_s = statistics.mean(times)
-    value = len(lens) / step_s
+    value = len(lens) * sum(share) / sum(sample_s)
     return {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name, "D": w.D, "H": w.H, "d_head": w.d, "T": w.T,
-                   "r_k": w.r_k, "r_v": w.r_v, "batch_per_gpu": len(lens)},
+        "ms_per_step": statistics.mean(sample_s) * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_dict(w, lens, world),
+        "extrapolated": True,
+        "step_definition": "one bounded sample of the decode step per timed step; value = tokens "
+                           "of the step x the sample's share of its work / the sample's time",
+        "full_step_seconds_extrapolated": statistics.mean(full),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,

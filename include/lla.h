@@ -16,6 +16,8 @@
  *   lla_prefill_attn_rope  causal prefill with rotary positions after reconstruction
  *   lla_decode_attn_loops  the decode calls of all T loops in one pass over the latents
  *   lla_prefill_attn     causal pass-2 prefill attention over the latents of a prompt
+ *   lla_prefill_two_pass the two-pass prefill of a batch of prompts through all layers, streamed
+ *                        layer by layer (encode, then the loop-major re-forward's attention)
  *   lla_encode_2d, lla_decode_attn_2d
  *                        the LLA-2D variant: one latent per (token, layer) for every head
  *   lla_encode_rope_keys, lla_decode_attn_decoupled
@@ -360,7 +362,7 @@ lla_status lla_decode_decoupled_workspace_size(const lla_geometry *g, int32_t d_
  *                pre-rotation rotary key; NULL in pass 2
  *   workspace    >= lla_decode_decoupled_workspace_size bytes; overwritten (no zero fill)
  * Other arguments and the error behaviour are those of lla_decode_attn; three launches on
- * `stream`.  Storage LLA_BF16, d = 128, H <= 64, (r_k, r_v) = (96, 160), d_rope 32 or 64;
+ * `stream`.  Storage LLA_BF16, d = 128, H <= 64, (r_k, r_v) = (96, 160), d_rope 32, 64 or 96;
  * LLA_ERR_UNSUPPORTED otherwise.
  */
 lla_status lla_decode_attn_decoupled(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
@@ -405,6 +407,50 @@ lla_status lla_decode_attn_noalloc(const lla_geometry *g, const lla_codec *codec
 lla_status lla_prefill_attn(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
                             const int32_t *cu_seqlens, int32_t B, int32_t max_len, int32_t loop,
                             const void *q, lla_dtype io_dtype, void *out, void *stream);
+
+/*
+ * Callbacks of lla_prefill_two_pass, called on the calling host thread in the order given there.
+ * Each enqueues its own work on `stream` (the stream passed to lla_prefill_two_pass) and returns
+ * LLA_OK, or another status to stop the prefill (lla_prefill_two_pass then returns it).
+ *   lla_capture_fn  sets *x_k, *x_v to device [T][N][H][d] arrays (x_dtype, 16-byte aligned) with
+ *                   layer `layer`'s pass-1 pre-RoPE keys and values of the N prompt tokens, stacked
+ *                   over the loops as Eq. encode takes them.
+ *   lla_query_fn    sets *q to device [N][H][d] pass-2 queries (io_dtype) of layer `layer` at loop
+ *                   `loop` and *out to where their attention output goes (same shape).
+ */
+typedef lla_status (*lla_capture_fn)(int32_t layer, const void **x_k, const void **x_v, void *stream,
+                                     void *user);
+typedef lla_status (*lla_query_fn)(int32_t layer, int32_t loop, const void **q, void **out, void *stream,
+                                   void *user);
+
+/*
+ * The capacity decoder's two-pass prefill of B prompts through all D layers, streamed layer by
+ * layer (App. A "Decoding and caching"; App. J "Eviction and long-context prefill").  Host
+ * orchestration of this library's kernels on `stream`, in this order:
+ *   phase 1, for l = 0 .. D-1:  capture(l); lla_encode of the N tokens into caches[l]
+ *   phase 2, for t = 0 .. T-1, for l = 0 .. D-1:  query(l, t); causal attention at loop t over
+ *            caches[l] (lla_prefill_attn, or lla_prefill_attn_rope when rope is not NULL)
+ * Only one layer's capture is needed at a time: the arrays capture(l) handed over may be reused
+ * or freed, in stream order, once capture(l + 1) has been called (the last once the call has
+ * returned).  With rope, the rebuilt keys of one (layer, loop) occupy the workspace and the next
+ * overwrites them.
+ *   codecs, caches  host arrays of D per-layer codecs and caches (their block tables give the
+ *                   positions attention reads, slot_mapping the slots encode writes: the caller
+ *                   keeps them consistent, token i of prompt b at row i of its pages)
+ *   slot_mapping    device [N] int64, N = cu_seqlens[B] prompt tokens in prompt order
+ *   cu_seqlens, B, max_len   as lla_prefill_attn
+ *   rope            NULL (positions-free content path) or the rotation of lla_prefill_attn_rope
+ *   workspace       with rope: >= lla_prefill_rope_workspace_size(g, B, max_len) bytes (device);
+ *                   else unused (may be NULL)
+ * Returns the first non-OK status of a callback or of a call it makes (the work enqueued before
+ * it stays enqueued); the error behaviour of each step is that of its call.
+ */
+lla_status lla_prefill_two_pass(const lla_geometry *g, int32_t D, const lla_codec *codecs,
+                                const lla_cache *caches, lla_dtype x_dtype,
+                                const int64_t *slot_mapping, int32_t N, const int32_t *cu_seqlens,
+                                int32_t B, int32_t max_len, lla_dtype io_dtype, const lla_rope *rope,
+                                lla_capture_fn capture, lla_query_fn query, void *user,
+                                void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * Comparator: the uncompressed loop-indexed cache ("Teacher cache", Sec. 3) decoded by the same

@@ -1012,7 +1012,7 @@ size_t decode_2d_workspace_bytes(int r_k, int r_v, int B) {
 
 bool decode_decoupled_supported(int es, int d, int H, int r_k, int r_v, int d_rope) {
     return es == 2 && d == kD && H >= 1 && H <= 64 && r_k == 96 && r_v == 160 &&
-           (d_rope == 32 || d_rope == 64);
+           (d_rope == 32 || d_rope == 64 || d_rope == 96);
 }
 
 size_t decode_decoupled_workspace_bytes(int r_k, int r_v, int d_rope, int B, int H) {
@@ -1034,6 +1034,7 @@ lla_status launch_decode_decoupled(const DecodeArgs &a, const void *rope_pool, i
     rotary_phases(d_rope, base, rot.phi);
     if (a.r_k == 96 && a.r_v == 160 && d_rope == 32) return launch_units<96, 160, 32>(a, &rot, stream);
     if (a.r_k == 96 && a.r_v == 160 && d_rope == 64) return launch_units<96, 160, 64>(a, &rot, stream);
+    if (a.r_k == 96 && a.r_v == 160 && d_rope == 96) return launch_units<96, 160, 96>(a, &rot, stream);
     return LLA_ERR_UNSUPPORTED;
 }
 

@@ -57,6 +57,13 @@ class lla_cache(ctypes.Structure):
                 ("block_table", ctypes.c_void_p), ("max_blocks_per_seq", ctypes.c_int32)]
 
 
+# lla_capture_fn and lla_query_fn of include/lla.h
+CAPTURE_FN = ctypes.CFUNCTYPE(ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p),
+                              ctypes.POINTER(ctypes.c_void_p), ctypes.c_void_p, ctypes.c_void_p)
+QUERY_FN = ctypes.CFUNCTYPE(ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                            ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(ctypes.c_void_p),
+                            ctypes.c_void_p, ctypes.c_void_p)
+
 _lib = None
 
 
@@ -99,6 +106,8 @@ def library() -> ctypes.CDLL:
                                                 P, P, SZ, P]),
             "lla_get_device_error": (I32, [P, P]),
             "lla_clear_device_error": (I32, [P]),
+            "lla_prefill_two_pass": (I32, [P, I32, P, P, I32, P, I32, P, I32, I32, I32, P, CAPTURE_FN,
+                                           QUERY_FN, P, P, SZ, P]),
             "lla_set_wait_limit_ns": (I32, [ctypes.c_uint64]),
             "lla_get_wait_limit_ns": (ctypes.c_uint64, []),
         }
@@ -344,6 +353,59 @@ def lla_prefill_attn_rope(geom: Geometry, codec: Codec, cache: Cache, rope_base:
         ctypes.byref(g), ctypes.byref(cd), ctypes.byref(ch), ctypes.byref(rp), _ptr(cu_seqlens), B,
         max_len, loop, _ptr(q), _dtype_code(q), _ptr(out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def lla_prefill_two_pass(geom: Geometry, codecs, caches, slot_mapping: torch.Tensor,
+                         cu_seqlens: torch.Tensor, max_len: int, capture, query,
+                         x_dtype=torch.bfloat16, io_dtype=torch.bfloat16, rope_base=None,
+                         rope_pairing: int = LLA_ROPE_HALF, workspace: Optional[torch.Tensor] = None,
+                         stream=None) -> None:
+    """Two-pass prefill of len(cu_seqlens) - 1 prompts through len(codecs) layers, streamed layer
+    by layer.  capture(layer) returns layer's pass-1 (x_k, x_v) [T][N][H][d]; query(layer, loop)
+    returns (q, out) [N][H][d].  Both are called from inside the C call, in its order; the
+    tensors they return are kept alive until it returns (stream order covers the rest).
+    rope_base None: positions-free content path; else RoPE after reconstruction (workspace of
+    lla_prefill_rope_workspace_size bytes)."""
+    D = len(codecs)
+    if len(caches) != D:
+        raise ValueError("one cache per codec")
+    cds = (lla_codec * max(D, 1))(*[c.c() for c in codecs])
+    chs = (lla_cache * max(D, 1))(*[c.c() for c in caches])
+    g = geom.c()
+    keep, errors = [], []
+
+    def _capture(layer, pk, pv, _stream_, _user):
+        try:
+            xk, xv = capture(layer)
+            keep.append((xk, xv))
+            pk[0], pv[0] = _ptr(xk), _ptr(xv)
+            return 0
+        except Exception as e:  # reported after the C call returns
+            errors.append(e)
+            return 1
+
+    def _query(layer, loop, pq, po, _stream_, _user):
+        try:
+            q, out = query(layer, loop)
+            keep.append((q, out))
+            pq[0], po[0] = _ptr(q), _ptr(out)
+            return 0
+        except Exception as e:
+            errors.append(e)
+            return 1
+
+    cb_c, cb_q = CAPTURE_FN(_capture), QUERY_FN(_query)
+    rp = None if rope_base is None else lla_rope(float(rope_base), int(rope_pairing))
+    xd = LLA_BF16 if x_dtype == torch.bfloat16 else LLA_F32
+    iod = LLA_BF16 if io_dtype == torch.bfloat16 else LLA_F32
+    B = cu_seqlens.shape[0] - 1
+    st = library().lla_prefill_two_pass(
+        ctypes.byref(g), D, cds, chs, xd, _ptr(slot_mapping), slot_mapping.numel(), _ptr(cu_seqlens),
+        B, max_len, iod, None if rp is None else ctypes.byref(rp), cb_c, cb_q, None, _ptr(workspace),
+        0 if workspace is None else workspace.numel() * workspace.element_size(), _stream(stream))
+    if errors:
+        raise errors[0]
+    _check("lla_prefill_two_pass", st)
 
 
 def lla_cache_2d_block_bytes(geom: Geometry) -> int:

@@ -213,3 +213,17 @@ def pack_latent_pages(c_k: torch.Tensor, c_v: torch.Tensor, table: torch.Tensor,
         pool[blocks, BLOCK * r_k * 2:] = vp.view(n, -1).view(torch.uint8)
         off += L
     return pool.view(-1)
+
+
+def random_pool(num_bytes: int, seed: int, *key: int, device="cpu", chunk: int = 1 << 30) -> torch.Tensor:
+    """A cache pool (uint8, num_bytes a multiple of 2) whose every bf16 element is an N(0,1)
+    draw: valid latents in every position of every page, whatever the layout, for timing decode
+    over a full-size cache without encoding it.  Drawn in chunks of `chunk` elements."""
+    pool = torch.empty(num_bytes, dtype=torch.uint8, device=device)
+    flat = pool.view(torch.bfloat16)
+    s = _gen(seed, 8, *key).initial_seed()
+    g = torch.Generator(device=device).manual_seed(s)
+    for o in range(0, flat.numel(), chunk):
+        n = min(chunk, flat.numel() - o)
+        flat[o:o + n] = torch.randn(n, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+    return pool

@@ -25,6 +25,7 @@ def lib():
 def declared_functions():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    text = re.sub(r"typedef[^;]*;", "", text)  # callback types, structs and enums
     return sorted(set(re.findall(r"\b(lla_[a-z_0-9]+)\s*\(", text)))
 
 
@@ -389,3 +390,47 @@ def test_binding_rejects_host_tensors_before_any_launch(lib):
     with pytest.raises(ValueError, match="contiguous"):
         lib._ptr(torch.zeros(4, 4).t())
     assert lib._ptr(None) is None and lib._ptr(FAKE) == FAKE
+
+
+def test_two_pass_prefill_order_and_checks(lib):
+    """lla_prefill_two_pass with empty prompts (N = 0, B = 0: nothing reaches the GPU): every
+    layer's capture in layer order, then the queries loop by loop and layer by layer; a callback's
+    status stops it and is returned; missing callbacks and bad dtypes are rejected."""
+    so = lib.library()
+    D, T = 3, 4
+    g = _g(lib, T=T)
+    cds = (lib.lla_codec * D)(*[lib.lla_codec(FAKE, FAKE, FAKE, FAKE, None, None) for _ in range(D)])
+    chs = (lib.lla_cache * D)(*[lib.lla_cache(FAKE, 10, FAKE, 4) for _ in range(D)])
+    order = []
+
+    def cap(layer, pk, pv, stream, user):
+        order.append(("c", layer))
+        pk[0] = pv[0] = FAKE
+        return 0
+
+    def qry(layer, loop, pq, po, stream, user):
+        order.append(("q", layer, loop))
+        pq[0] = po[0] = FAKE
+        return 0
+
+    c, q = lib.CAPTURE_FN(cap), lib.QUERY_FN(qry)
+
+    def call(capture=c, query=q, xdt=0, iodt=0, D=D):
+        return so.lla_prefill_two_pass(ctypes.byref(g), D, cds, chs, xdt, FAKE, 0, FAKE, 0, 0, iodt, None,
+                                       capture, query, None, None, 0, None)
+
+    assert call() == OK
+    assert order == [("c", l) for l in range(D)] + [("q", l, t) for t in range(T) for l in range(D)]
+    assert call(xdt=7) == INVALID
+    assert call(iodt=7) == INVALID
+    assert call(capture=lib.CAPTURE_FN()) == INVALID
+    assert call(D=0, capture=lib.CAPTURE_FN(), query=lib.QUERY_FN()) == OK
+
+    def failing(layer, pk, pv, stream, user):
+        order.append(("c", layer))
+        pk[0] = pv[0] = FAKE
+        return UNSUPPORTED if layer == 1 else OK
+
+    order.clear()
+    assert call(capture=lib.CAPTURE_FN(failing)) == UNSUPPORTED
+    assert order == [("c", 0), ("c", 1)]

@@ -111,7 +111,7 @@ def test_tiny_workload_two_pass_decode(lla, pairing, with_mu):
     assert lla.lla_get_device_error() == 0
 
 
-@pytest.mark.parametrize("d_rope", [32, 64])
+@pytest.mark.parametrize("d_rope", [32, 64, 96])
 def test_ragged_batch(lla, d_rope):
     """Empty (pass 1 only), one token, page-aligned, ragged tails and several pages, H=16, bf16
     inputs and outputs, with mu."""
