@@ -254,9 +254,23 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
         const int qslot = r % kQSlots;   // query slot
         float beta = 0.f;
         const float *qq = a.qlat + qslot * a.qslot + ks * F::NGT * F::KE;
+        // q~ of this thread's granules stays in registers for the whole run when it is small
+        // enough (up to 48 floats); else it is re-read from shared memory (a broadcast) per token
+        constexpr bool kQreg = F::NGT * F::KE <= 48;
+        float qr[kQreg ? F::NGT * F::KE : 1];
         if (is_s) {
             mbar_wait(&a.qready[qslot], (r / kQSlots) & 1, s.abort_flag, p.err, wait_limit(p));
             beta = m_part(a, qslot, 1);
+            if constexpr (kQreg) {
+#pragma unroll
+                for (int g = 0; g < F::NGT; ++g) {
+                    if (F::NGK % F::KSPLIT != 0 && ks * F::NGT + g >= F::NGK) break;
+                    float t[F::KE];
+                    load_qvec<F::KE>(qq + g * F::KE, t);
+#pragma unroll
+                    for (int e = 0; e < F::KE; ++e) qr[g * F::KE + e] = t[e];
+                }
+            }
         }
         float m_run = -INFINITY, l_part = 0.f;
         float accv[AV];
@@ -287,7 +301,12 @@ __global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Pa
                             if (F::NGK % F::KSPLIT != 0 && ks * F::NGT + g >= F::NGK) break;
                             float v[F::KE], qv[F::KE];
                             load_gran<ES, F::GK>(kp + g * (kBlockTokens * F::GK), v);
-                            load_qvec<F::KE>(qq + g * F::KE, qv);  // broadcast read
+                            if constexpr (kQreg) {
+#pragma unroll
+                                for (int e = 0; e < F::KE; ++e) qv[e] = qr[g * F::KE + e];
+                            } else {
+                                load_qvec<F::KE>(qq + g * F::KE, qv);  // broadcast read
+                            }
 #pragma unroll
                             for (int e = 0; e < F::KE; ++e) {
                                 if ((e & 3) == 0) a0 = fmaf(v[e], qv[e], a0);

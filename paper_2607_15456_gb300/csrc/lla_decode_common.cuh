@@ -21,7 +21,7 @@ constexpr int kComputeThreads = kComputeWarps * 32;
 constexpr int kThreads = kComputeThreads + 32;  // + one producer warp
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
-constexpr int kStepTargetBytes = 32 * 1024;
+constexpr int kStepTargetBytes = 48 * 1024;  // most data per pipeline step (whole head pages)
 constexpr int kBarAll = 1;  // named barrier over the 256 consumer threads
 constexpr int kBarTok = 2;  // named barrier over the score threads
 
@@ -295,7 +295,9 @@ __device__ __forceinline__ void order_runs(const Params &p, const Smem &s, Range
 
 // Producer: the whole warp walks the CTA's range.  Block ids are fetched 32 pages at a time
 // (one per lane) so the copies of consecutive steps are issued back to back instead of each
-// waiting for its own block-table load; lane 0 issues the bulk copies.
+// waiting for its own block-table load.  Lane 0 issues a one-page step's bulk copy; when a step
+// holds several small pages, lanes 0 .. n-1 issue one copy each in the same instruction (issued
+// one after another from one lane, the copies of 6 KB pages paced the whole kernel).
 //
 // After a failed wait (or once another thread raised the abort flag) no further copy is issued:
 // a new round on a stage whose previous copies have not landed would arrive twice on one phase
@@ -319,37 +321,46 @@ __device__ void producer(const Params &p, const Smem &s, const Range &rg) {
             for (int k = k0; k < kend; k += p.pps) {
                 const int stage = st;
                 const uint32_t ph = sph;
-                int32_t blk[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    blk[i] = __shfl_sync(0xffffffffu, blk_lane, (k - k0 + i) & 31);
                 int halt = 0;
-                if (lane == 0) {
-                    halt = !mbar_wait(&s.empty[stage], ph ^ 1u, s.abort_flag, p.err, wait_limit(p)) ||
-                           *s.abort_flag;
-                    if (!halt) {
-                        const int n = min(p.pps, R.npages - k);
-                        uint32_t bytes = 0;
-                        for (int i = 0; i < n; ++i) {
-                            if (blk[i] < 0 || blk[i] >= p.num_blocks) {
-                                atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
-                                blk[i] = -1;
-                            } else {
-                                bytes += hpb;
-                            }
+                if (p.pps == 1) {
+                    const int32_t b0 = __shfl_sync(0xffffffffu, blk_lane, (k - k0) & 31);
+                    if (lane == 0) {
+                        halt = !mbar_wait(&s.empty[stage], ph ^ 1u, s.abort_flag, p.err, wait_limit(p)) ||
+                               *s.abort_flag;
+                        if (!halt) {
+                            const bool ok = b0 >= 0 && b0 < p.num_blocks;
+                            if (!ok) atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                            mbar_arrive_expect_tx(&s.full[stage], ok ? hpb : 0);
+                            if (ok)
+                                bulk_g2s(s.ring + stage * p.stage_bytes,
+                                         p.pool + b0 * p.block_bytes + static_cast<int64_t>(R.h) * hpb, hpb,
+                                         &s.full[stage], pol);
                         }
-                        mbar_arrive_expect_tx(&s.full[stage], bytes);
-                        char *dst = s.ring + stage * p.stage_bytes;
-                        for (int i = 0; i < n; ++i)
-                            if (blk[i] >= 0)
-                                bulk_g2s(dst + i * hpb,
-                                         p.pool + blk[i] * p.block_bytes + static_cast<int64_t>(R.h) * hpb,
-                                         hpb, &s.full[stage], pol);
                     }
-                }
-                if (__shfl_sync(0xffffffffu, halt, 0)) {
-                    stop = true;
-                    break;
+                    if (__shfl_sync(0xffffffffu, halt, 0)) {
+                        stop = true;
+                        break;
+                    }
+                } else {
+                    // several pages per step: lanes 0 .. n-1 issue one bulk copy each, together
+                    if (lane == 0)
+                        halt = !mbar_wait(&s.empty[stage], ph ^ 1u, s.abort_flag, p.err, wait_limit(p)) ||
+                               *s.abort_flag;
+                    if (__shfl_sync(0xffffffffu, halt, 0)) {
+                        stop = true;
+                        break;
+                    }
+                    const int n = min(p.pps, R.npages - k);
+                    const int32_t mine = __shfl_sync(0xffffffffu, blk_lane, (k - k0 + lane) & 31);
+                    const bool valid = lane < n && mine >= 0 && mine < p.num_blocks;
+                    if (lane < n && !valid) atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                    const unsigned vm = __ballot_sync(0xffffffffu, valid);
+                    if (lane == 0) mbar_arrive_expect_tx(&s.full[stage], __popc(vm) * hpb);
+                    __syncwarp();
+                    if (valid)
+                        bulk_g2s(s.ring + stage * p.stage_bytes + lane * hpb,
+                                 p.pool + mine * p.block_bytes + static_cast<int64_t>(R.h) * hpb, hpb,
+                                 &s.full[stage], pol);
                 }
                 ++it;
                 if (++st == p.stages) {
@@ -629,6 +640,52 @@ __device__ __forceinline__ void value_step(float (&accv)[Fast<ES, RK, RV>::UPT *
 #pragma unroll
     for (int e = 0; e < AV; ++e) accv[e] *= alpha;
     const char *vbase = sb + F::KPLANE + vc * F::VB + tg * F::ROWB;
+    if constexpr (kBlockTokens % F::NTG == 0 && F::VE % 2 == 0) {
+        // A full step (the common case): every thread owns RPT rows of each page, known at
+        // compile time, so the loads of G rows go out together and two accumulator sets halve
+        // the dependent chains (the loop below ran latency-bound on 4-byte units).
+        if (nvalid == F::TOK) {
+            constexpr int RPT = kBlockTokens / F::NTG;
+            constexpr int G = RPT >= 4 ? 4 : RPT;  // rows whose loads go out together
+            float acc2[AV];
+#pragma unroll
+            for (int e = 0; e < AV; ++e) acc2[e] = 0.f;
+#pragma unroll
+            for (int pi = 0; pi < F::PPS; ++pi) {
+                const char *vp = vbase + pi * F::HPB;
+                const float *pp = pring + pi * kBlockTokens + tg;
+#pragma unroll
+                for (int i0 = 0; i0 < RPT; i0 += G) {
+                    float pv[G];
+                    float v[G][F::UPT][F::VE];
+#pragma unroll
+                    for (int i = 0; i < G; ++i) {
+                        pv[i] = pp[(i0 + i) * F::NTG];
+#pragma unroll
+                        for (int uu = 0; uu < F::UPT; ++uu)
+                            load_gran<ES, F::VB>(vp + (i0 + i) * (F::NTG * F::ROWB) + uu * (F::VC * F::VB), v[i][uu]);
+                    }
+#pragma unroll
+                    for (int i = 0; i < G; ++i) {
+                        float *acc = (i & 1) ? acc2 : accv;
+                        const float2 p2 = make_float2(pv[i], pv[i]);
+#pragma unroll
+                        for (int uu = 0; uu < F::UPT; ++uu)
+#pragma unroll
+                            for (int e = 0; e < F::VE; e += 2) {
+                                const float2 r = __ffma2_rn(p2, make_float2(v[i][uu][e], v[i][uu][e + 1]),
+                                                            make_float2(acc[uu * F::VE + e], acc[uu * F::VE + e + 1]));
+                                acc[uu * F::VE + e] = r.x;
+                                acc[uu * F::VE + e + 1] = r.y;
+                            }
+                    }
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < AV; ++e) accv[e] += acc2[e];
+            return;
+        }
+    }
 #pragma unroll
     for (int pi = 0; pi < F::PPS; ++pi) {
         // rows tg, tg + NTG, ... of page pi that hold valid tokens

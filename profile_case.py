@@ -2,40 +2,41 @@
 
 decode (default): builds a workload's latent cache for a few layers only (same batch, context
 lengths, heads and ranks, so every decode launch has exactly the shape and bytes of a launch in
-the full benchmark), then runs `--calls` pass-1 decode calls (and one encode call per layer), so
-that a profiler can skip the warm-up launches and capture one to three of them:
+the full benchmark; `--fill random` writes N(0,1) latents instead of encoding them), then runs
+`--calls` pass-1 decode calls (and one encode call per layer), so that a profiler can skip the
+warm-up launches and capture one to three of them:
 
     ncu --set full --clock-control none -k regex:decode_async_kernel -s 6 -c 1 \\
-        python -m paper_2607_15456_gb300.profile_case --workload ouro14_rho4 --layers 2 --calls 10
+        python profile_case.py --workload ouro14_rho4 --layers 2 --calls 10
 
 rope: the same decode calls through lla_decode_attn_rope (RoPE after reconstruction, base 10^4):
 
     ncu --set full --clock-control none -k regex:decode_rope_kernel -s 6 -c 1 \\
-        python -m paper_2607_15456_gb300.profile_case --case rope --workload ouro14_rho4 --layers 2 --calls 10
+        python profile_case.py --case rope --workload ouro14_rho4 --layers 2 --calls 10
 
 rope_prefill: the same prompts through lla_prefill_attn_rope (key rebuild, then attention):
 
     ncu --set full --clock-control none -k regex:"rope_rebuild_kernel|prefill_tc_kernel" -c 2 \\
-        python -m paper_2607_15456_gb300.profile_case --case rope_prefill --workload ouro14_rho2 \\
+        python profile_case.py --case rope_prefill --workload ouro14_rho2 \\
         --prompts 4 --len 8192 --calls 1
 
 loops / decoupled: the same cache through lla_decode_attn_loops (all T loops of a layer per call)
 or lla_decode_attn_decoupled (rotary planes of d_rope = 64 stored first, one per layer):
 
     ncu --set full --clock-control none -k regex:attn2d_kernel -s 2 -c 1 \\
-        python -m paper_2607_15456_gb300.profile_case --case decoupled --workload ouro14_rho4 --layers 2 --calls 10
+        python profile_case.py --case decoupled --workload ouro14_rho4 --layers 2 --calls 10
 
 2d: LLA-2D on the stress2d workload's shape with `--batch` sequences (random latents written into
 two layers' pages; --batch 32 keeps a layer near 1 GB, above L2):
 
     ncu --set full --clock-control none -k regex:attn2d_kernel -s 2 -c 1 \\
-        python -m paper_2607_15456_gb300.profile_case --case 2d --batch 32 --calls 8
+        python profile_case.py --case 2d --batch 32 --calls 8
 
 prefill: encodes `--prompts` prompts of `--len` tokens of a workload's ranks (tensor-core encode,
 one launch per axis), then runs `--calls` causal prefill calls over them:
 
     ncu --set full --clock-control none -k regex:"encode_tc_kernel|prefill_tc_kernel" -c 3 \\
-        python -m paper_2607_15456_gb300.profile_case --case prefill --workload ouro14_rho2 \\
+        python profile_case.py --case prefill --workload ouro14_rho2 \\
         --prompts 4 --len 8192 --calls 1
 """
 from __future__ import annotations
@@ -44,7 +45,7 @@ import argparse
 import os
 import sys
 
-ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
@@ -57,7 +58,7 @@ def decode_case(args):
 
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    bench = DecodeBench(args.workload, dev, layers=args.layers)
+    bench = DecodeBench(args.workload, dev, layers=args.layers, fill=args.fill)
     w = bench.w
     if args.case == "decoupled":
         from paper_2607_15456_gb300 import workloads as W
@@ -198,6 +199,8 @@ def main():
     ap.add_argument("--prompts", type=int, default=4)
     ap.add_argument("--len", type=int, default=8192)
     ap.add_argument("--batch", type=int, default=32)
+    ap.add_argument("--fill", choices=["encode", "random"], default="encode",
+                    help="decode cases: latents through lla_encode, or N(0,1) bf16 written into the pages")
     args = ap.parse_args()
     if args.case in ("decode", "rope", "loops", "decoupled"):
         decode_case(args)
