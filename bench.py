@@ -832,7 +832,8 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
                "ms_per_step": ms, "tokens_per_s": bench.B / (ms / 1e3),
                "avg_launch_us": dec_s * 1e6, "GB_s": nbytes / dec_s / 1e9,
                "hbm_frac": nbytes / dec_s / 1e9 / peak, "frac_of_nominal_8tbs": nbytes / dec_s / 1e9 / NOMINAL_HBM_GBS,
-               "bytes_per_launch": nbytes, "latent_cache_GB": latent_cache_bytes(w, bench.lens) / 1e9,
+               "bytes_per_launch": nbytes, "traffic": ncu_traffic(name),
+               "latent_cache_GB": latent_cache_bytes(w, bench.lens) / 1e9,
                "fill": "N(0,1) bf16 latents written into every page (the decode reads the same bytes "
                        "as for encoded ones)"}
         lens = bench.lens
