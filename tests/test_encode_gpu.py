@@ -92,6 +92,15 @@ def test_encode_prompt_on_tensor_cores(lla, r_k, r_v, with_mu):
     _encode_and_compare(lla, 4, 3, 128, r_k, r_v, "bf16", "bf16", [130, 101, 69], with_mu, 7)
 
 
+@pytest.mark.parametrize("r_k,r_v", [(192, 320), (96, 160)])
+def test_encode_prompt_many_units_per_cta(lla, r_k, r_v):
+    # 4200 tokens (33 tiles, the last ragged) of 8 heads with mu: every CTA of the persistent
+    # kernel takes several (head, tile, column group) units, alternates its two accumulator
+    # slots and crosses a head boundary (the bias mu W_down is recomputed there); at (192, 320)
+    # the two column groups of the V axis read the same x tile one after the other
+    _encode_and_compare(lla, 4, 8, 128, r_k, r_v, "bf16", "bf16", [2000, 1500, 700], True, 10)
+
+
 def test_encode_prompt_long_reduction_on_tensor_cores(lla):
     # T*d = 16 * 256 = 4096: 64 slabs of the reduction axis through the stage ring
     _encode_and_compare(lla, 16, 2, 256, 96, 160, "bf16", "bf16", [150], True, 8)

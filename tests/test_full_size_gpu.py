@@ -104,10 +104,12 @@ def test_full_size_decode_and_encode_sampled(wname, loop):
     assert_parity(np.stack(got_rows), np.stack(ref_rows), "bf16", f"{wname} decode loop {loop}")
 
 
-@pytest.mark.parametrize("pairing", [0, 1])
-def test_full_size_rope_decode_sampled(pairing):
+@pytest.mark.parametrize("pairing,io", [(0, "bf16"), (1, "bf16"), (0, "fp32")])
+def test_full_size_rope_decode_sampled(pairing, io):
     """The RoPE decode (lla_decode_attn_rope, base 10^4) on the headline batch as bench.py runs
-    it: sampled (sequence, head) rows against oracle.decode_rope fed the stored latents."""
+    it: sampled (sequence, head) rows against oracle.decode_rope fed the stored latents.  With
+    fp32 inputs and outputs the plain bound holds (max abs <= 2e-2, relative L2 <= 5e-3, no
+    allowance for an output's own rounding)."""
     ensure_library()
     import bench
     from paper_2607_15456_gb300 import lla
@@ -117,16 +119,18 @@ def test_full_size_rope_decode_sampled(pairing):
     db = bench.DecodeBench("ouro14_rho4", dev, layers=1)
     w = db.w
     loop = 1
+    dt = torch.float32 if io == "fp32" else torch.bfloat16
+    qi, cki, cvi = (t[0, loop].to(dt).contiguous() for t in (db.q, db.cur_k, db.cur_v))
+    o = torch.empty_like(qi)
     lla.lla_clear_device_error()
     lla.lla_decode_attn_rope(db.geom, db.codecs[0], db.caches[0], 10000.0, pairing, db.ctx,
-                             db.max_ctx, loop, db.q[0, loop], db.cur_k[0, loop],
-                             db.cur_v[0, loop], db.out[0, loop], db.ws)
+                             db.max_ctx, loop, qi, cki, cvi, o, db.ws)
     torch.cuda.synchronize()
     assert lla.lla_get_device_error() == 0
-    out = f64(db.out[0, loop])
+    out = f64(o)
     cod = {k: (None if v is None else f64(v)) for k, v in
            W.codec_tensors(w.T, w.H, w.d, w.r_k, w.r_v, w.seed, 0, dtype=torch.bfloat16).items()}
-    q, ck, cv = f64(db.q[0, loop]), f64(db.cur_k[0, loop]), f64(db.cur_v[0, loop])
+    q, ck, cv = f64(qi), f64(cki), f64(cvi)
     bb = lla.lla_cache_block_bytes(db.geom)
     scale = 1.0 / np.sqrt(w.d)
     got_rows, ref_rows = [], []
@@ -139,16 +143,18 @@ def test_full_size_rope_decode_sampled(pairing):
                                      None, q[b, h], ck[b, h], cv[b, h], scale, 10000.0, pairing)
             got_rows.append(out[b, h])
             ref_rows.append(ref)
-    assert_parity(np.stack(got_rows), np.stack(ref_rows), "bf16", "rope decode, full size",
-                  output_rounding=True)
+    assert_parity(np.stack(got_rows), np.stack(ref_rows), "bf16", f"rope decode, full size, {io} io",
+                  io=io, output_rounding=io == "bf16")
 
 
-def test_full_size_prefill_sampled_rows():
+@pytest.mark.parametrize("io", ["bf16", "fp32"])
+def test_full_size_prefill_sampled_rows(io):
     """Causal prefill at the benchmark's prompt size (Ouro-1.4B at rho = 2: 4 prompts of 8192
     tokens, 16 heads), in the launch configuration bench.py times.  Row i of a prompt is the
     pass-2 decode of query i over keys 0..i, so sampled rows are checked with the oracle's decode
     on the latents the GPU stored (first and last rows, rows on tile and page boundaries, and
-    random rows), against the bf16 bound taken before the output's own rounding."""
+    random rows).  bf16 queries and outputs: the bf16 bound taken before the output's own
+    rounding; fp32 queries and outputs: the plain bound (max abs <= 2e-2, relative L2 <= 5e-3)."""
     ensure_library()
     from paper_2607_15456_gb300 import lla
     from paper_2607_15456_gb300 import workloads as W
@@ -169,7 +175,7 @@ def test_full_size_prefill_sampled_rows():
     slots = torch.cat([pt.slots(b, range(L)) for b in range(nseq)]).to(dev)
     lla.lla_encode(geom, codec, cache, W.normal((T, N, H, d), w.seed, 300, device=dev),
                    W.normal((T, N, H, d), w.seed, 301, device=dev), slots)
-    q = W.normal((N, H, d), w.seed, 302, device=dev)
+    q = W.normal((N, H, d), w.seed, 302, device=dev, dtype=torch.float32 if io == "fp32" else torch.bfloat16)
     out = torch.empty_like(q)
     cu = torch.tensor([i * L for i in range(nseq + 1)], dtype=torch.int32, device=dev)
     lla.lla_clear_device_error()
@@ -192,5 +198,5 @@ def test_full_size_prefill_sampled_rows():
             ref.append(oracle.decode(loop, c_k[:i + 1], c_v[:i + 1], w64["w_up_k"][h], w64["w_up_v"][h],
                                      None, None, qb[i], None, None, scale))
             got.append(ob[i])
-    assert_parity(np.stack(got), np.stack(ref), "bf16", "full-size prefill rows", io="bf16",
-                  output_rounding=True)
+    assert_parity(np.stack(got), np.stack(ref), "bf16", f"full-size prefill rows, {io} io", io=io,
+                  output_rounding=io == "bf16")
