@@ -10,10 +10,13 @@
 // the second read of a tile's x_v hits L2, and a CTA meets few heads (the bias mu W_down is
 // computed once per head it meets).  bf16 operands, fp32 accumulation in TMEM, latents rounded
 // to bf16 and scattered to each token's slot.  Warp roles:
-//   warp 0     producer: per slab of 64 reduction rows, TMA tensor loads with 128-byte swizzle of
-//              the x tile (one box of 128 tokens x 64 elements: a K-major operand) and of W_down
-//              (boxes of 64 rows x 64 columns: an MN-major operand) into a ring of stages that
-//              runs on across units
+//   warp 0     x producer: per slab of 64 reduction rows, a TMA tensor load with 128-byte swizzle
+//              of the x tile (one box of 128 tokens x 64 elements: a K-major operand) into its
+//              own ring, which runs on across units
+//   warp 6     W producer: the slab's W_down (boxes of 64 rows x 64 columns: an MN-major
+//              operand) into a second ring; the two rings let the x stream from HBM run ahead
+//              of the W_down stream from L2 (one shared ring of 40 KB stages gave x only 16 of
+//              every 40 bytes in flight)
 //   warp 1     MMA issuer and TMEM owner: 4 MMAs (K = 16) per slab, M = 128, N = R, into one of
 //              two accumulator slots, so a unit's epilogue overlaps the next unit's products
 //   warps 2-5  epilogue: one token row per thread, TMEM -> bias -> bf16 -> the paged cache
@@ -30,18 +33,20 @@ namespace {
 
 constexpr int kEM = 128;             // tokens per tile
 constexpr int kES = 64;              // reduction rows per slab
-constexpr int kEThreads = 192;
+constexpr int kEThreads = 224;
 constexpr int kMaxGroup = 192;       // columns of a group
 constexpr int kMaxGroups = 6;        // groups of both axes (ranks up to 512: at most 3 each)
 constexpr int kASlab = kEM * kES * 2;   // x slab (16 KB)
 constexpr int kBAtom = kES * 128;       // one W_down atom of 64 columns (8 KB)
-constexpr int kStage = kASlab + 3 * kBAtom;  // 40 KB
-constexpr int kStages = 5;
+constexpr int kWStage = 3 * kBAtom;          // 24 KB
+constexpr int kXStages = 5;                 // x slabs in flight (from HBM)
+constexpr int kWStages = 5;                 // W_down slabs in flight (from L2)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kSlotCols = 256;  // accumulator slot s at column s * 256
-constexpr int oBias = kStages * kStage;
+constexpr int oW = kXStages * kASlab;
+constexpr int oBias = oW + kWStages * kWStage;
 constexpr int oBar = oBias + kMaxGroups * kMaxGroup * 4;
-constexpr int kNumBars = 2 * kStages + 4 + 1;  // full, empty, accfull[2], accempty[2], done
+constexpr int kNumBars = 2 * kXStages + 2 * kWStages + 4 + 1;
 constexpr int kSmem = 1024 + oBar + kNumBars * 8 + 16;  // + alignment slack, abort flag, TMEM slot
 static_assert(kSmem <= 227 * 1024, "shared memory");
 
@@ -89,8 +94,10 @@ __global__ void __launch_bounds__(kEThreads, 1)
     char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     float *bias = reinterpret_cast<float *>(sm + oBias);  // [group][192] of the current head
     uint64_t *full = reinterpret_cast<uint64_t *>(sm + oBar);
-    uint64_t *empty = full + kStages;
-    uint64_t *accfull = empty + kStages;  // [2]
+    uint64_t *empty = full + kXStages;
+    uint64_t *wfull = empty + kXStages;
+    uint64_t *wempty = wfull + kWStages;
+    uint64_t *accfull = wempty + kWStages;  // [2]
     uint64_t *accempty = accfull + 2;     // [2]
     uint64_t *done = accempty + 2;
     volatile int *abort_flag = reinterpret_cast<volatile int *>(done + 1);
@@ -102,9 +109,13 @@ __global__ void __launch_bounds__(kEThreads, 1)
     const int NS = Td / kES;
 
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kXStages; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
+        }
+        for (int s = 0; s < kWStages; ++s) {
+            mbar_init(&wfull[s], 1);
+            mbar_init(&wempty[s], 1);
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&accfull[s], 1);
@@ -121,10 +132,12 @@ __global__ void __launch_bounds__(kEThreads, 1)
     const uint32_t tmem = *tslot;
     pdl_wait();  // x, slots and the pool may come from the previous kernel
 
-    if (warp == 0) {
-        // ------------------------------------------------------------------------- producer
-        // After a failed wait no further copy is issued (a second arrival on an incomplete phase
-        // of a full barrier); the copies in flight are awaited below with the full limit.
+    if (warp == 0 || warp == 6) {
+        // ------------------------------------------------------------ producers: x (0), W (6)
+        const bool isx = warp == 0;
+        const int NST = isx ? kXStages : kWStages;
+        uint64_t *F = isx ? full : wfull;
+        uint64_t *E = isx ? empty : wempty;
         int q = 0;  // slabs issued
         bool stop = false;
         for (int64_t u = u0; u < u1 && !stop; ++u) {
@@ -133,30 +146,31 @@ __global__ void __launch_bounds__(kEThreads, 1)
             const CUtensorMap *tx = U.axis ? &txv : &txk;
             const CUtensorMap *tw = U.axis ? &twv : &twk;
             for (int s = 0; s < NS; ++s) {
-                const int st = q % kStages;
-                const uint32_t ph = (q / kStages) & 1;
+                const int st = q % NST;
+                const uint32_t ph = (q / NST) & 1;
                 int halt = 0;
                 if (lane == 0) {
-                    halt = !mbar_wait(&empty[st], ph ^ 1u, abort_flag, p.err) || *abort_flag;
-                    if (!halt) mbar_arrive_expect_tx(&full[st], kASlab + atoms * kBAtom);
+                    halt = !mbar_wait(&E[st], ph ^ 1u, abort_flag, p.err) || *abort_flag;
+                    if (!halt) mbar_arrive_expect_tx(&F[st], isx ? kASlab : atoms * kBAtom);
                 }
                 if (__shfl_sync(0xffffffffu, halt, 0)) {
                     stop = true;
                     break;
                 }
                 __syncwarp();
-                char *a = sm + st * kStage;
-                char *b = a + kASlab;
                 const int k0 = s * kES, t = k0 / p.d, e0 = k0 - t * p.d;
-                if (lane == 0) tma_load_4d(a, tx, e0, U.h, U.n0, t, &full[st]);
-                if (lane < atoms) tma_load_3d(b + lane * kBAtom, tw, U.col0 + lane * 64, k0, U.h, &full[st]);
+                if (isx) {
+                    if (lane == 0) tma_load_4d(sm + st * kASlab, tx, e0, U.h, U.n0, t, &F[st]);
+                } else {
+                    if (lane < atoms) tma_load_3d(sm + oW + st * kWStage + lane * kBAtom, tw, U.col0 + lane * 64, k0, U.h, &F[st]);
+                }
                 ++q;
             }
         }
         if (lane == 0 && *abort_flag) {
             volatile int never = 0;
-            for (int j = q > kStages ? q - kStages : 0; j < q; ++j)
-                mbar_wait(&full[j % kStages], (j / kStages) & 1, &never, p.err);
+            for (int j = q > NST ? q - NST : 0; j < q; ++j)
+                mbar_wait(&F[j % NST], (j / NST) & 1, &never, p.err);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------------------ MMA issuer
@@ -174,18 +188,20 @@ __global__ void __launch_bounds__(kEThreads, 1)
                 bool ok = true;
 #pragma unroll 1
                 for (int s = 0; s < NS; ++s, ++q) {
-                    const int st = q % kStages;
-                    if (!mbar_wait(&full[st], (q / kStages) & 1, abort_flag, p.err)) {
+                    const int st = q % kXStages, sw = q % kWStages;
+                    if (!mbar_wait(&full[st], (q / kXStages) & 1, abort_flag, p.err) ||
+                        !mbar_wait(&wfull[sw], (q / kWStages) & 1, abort_flag, p.err)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a = base + st * kStage, b = a + kASlab;
+                    const uint32_t a = base + st * kASlab, b = base + oW + sw * kWStage;
 #pragma unroll
                     for (int ks = 0; ks < kES / 16; ++ks)
                         umma_bf16(d, umma_desc_sw128_k(a + ks * 32), umma_desc_sw128_mn(b + ks * 2048, kBAtom),
                                   idesc, s > 0 || ks > 0);
                     umma_commit(&empty[st]);
+                    umma_commit(&wempty[sw]);
                 }
                 if (!ok) break;
                 umma_commit(&accfull[slot]);
@@ -196,7 +212,7 @@ __global__ void __launch_bounds__(kEThreads, 1)
             mbar_wait(done, 0, &never, p.err);
         }
         __syncwarp();
-    } else {
+    } else if (warp <= 5) {
         // --------------------------------------------------------------------------- epilogue
         const int et = tid - 64;  // 0..127
         const int quarter = warp & 3;
