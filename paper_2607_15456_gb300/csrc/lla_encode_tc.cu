@@ -19,7 +19,8 @@
 //              every 40 bytes in flight)
 //   warp 1     MMA issuer and TMEM owner: 4 MMAs (K = 16) per slab, M = 128, N = R, into one of
 //              two accumulator slots, so a unit's epilogue overlaps the next unit's products
-//   warps 2-5  epilogue: one token row per thread, TMEM -> bias -> bf16 -> the paged cache
+//   warps 2-5  epilogue: one token row per thread, TMEM -> bias -> bf16 -> the paged cache (V-plane
+//              rows pass through a per-warp staging buffer, so a store writes 8 rows of 64 bytes)
 // Tokens past N read as zeros (tensor-map fill) and are not stored.
 #include <cuda_runtime.h>
 
@@ -45,7 +46,8 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kSlotCols = 256;  // accumulator slot s at column s * 256
 constexpr int oW = kXStages * kASlab;
 constexpr int oBias = oW + kWStages * kWStage;
-constexpr int oBar = oBias + kMaxGroups * kMaxGroup * 4;
+constexpr int oStg = oBias + kMaxGroups * kMaxGroup * 4;   // V-plane store staging: 4 warps x 32 rows x 80 B
+constexpr int oBar = oStg + 4 * 32 * 80;
 constexpr int kNumBars = 2 * kXStages + 2 * kWStages + 4 + 1;
 constexpr int kSmem = 1024 + oBar + kNumBars * 8 + 16;  // + alignment slack, abort flag, TMEM slot
 static_assert(kSmem <= 227 * 1024, "shared memory");
@@ -276,11 +278,36 @@ __global__ void __launch_bounds__(kEThreads, 1)
             mbar_wait(&accfull[slot], (j >> 1) & 1, abort_flag, p.err);
             tc_fence_after();
             const uint32_t tl = tmem + slot * kSlotCols + (static_cast<uint32_t>(quarter * 32) << 16);
+            char *stg = sm + oStg + quarter * (32 * 80);
 #pragma unroll 1
             for (int c0 = 0; c0 < U.R; c0 += 32) {
                 float v[32];
                 tmem_ld32(tl + c0, v);  // warp-collective: every lane loads, valid rows store
-                if (dst) {
+                if (U.axis == 1) {
+                    // V-plane rows are r_v * 2 bytes apart: stage the warp's 32 rows x 64 bytes and
+                    // store 8 rows of 64 contiguous bytes per instruction
+#pragma unroll
+                    for (int k = 0; k < 32; k += 8) {
+                        const int c = c0 + k;
+                        float b8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                        if (use_bias) {
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) b8[i] = bs[c + i];
+                        }
+                        *reinterpret_cast<uint4 *>(stg + lane * 80 + (k / 8) * 16) =
+                            make_uint4(pack_bf16(v[k] - b8[0], v[k + 1] - b8[1]), pack_bf16(v[k + 2] - b8[2], v[k + 3] - b8[3]),
+                                       pack_bf16(v[k + 4] - b8[4], v[k + 5] - b8[5]), pack_bf16(v[k + 6] - b8[6], v[k + 7] - b8[7]));
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int rr = 8 * i + (lane >> 2), cc = lane & 3;
+                        char *d = reinterpret_cast<char *>(__shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(dst), rr));
+                        const uint4 val = *reinterpret_cast<const uint4 *>(stg + rr * 80 + cc * 16);
+                        if (d) *reinterpret_cast<uint4 *>(d + (U.col0 + c0 + cc * 8) * 2) = val;
+                    }
+                    __syncwarp();
+                } else if (dst) {
 #pragma unroll
                     for (int k = 0; k < 32; k += 8) {
                         const int c = c0 + k, jc = U.col0 + c;  // column in the group, in the axis
