@@ -827,6 +827,21 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
         ms = t0.elapsed_time(t1) / steps
         dec_s = sum(a.elapsed_time(b) for a, b in ev) / 1e3 / (steps * w.D * w.T)
         nbytes = bench.decode_bytes_per_launch()
+        rope = None
+        try:  # shapes without a tensor-core key rebuild are refused before anything is enqueued
+            bench.decode_calls_rope()
+        except lla.LLAError as e:
+            if e.status != 2:  # LLA_ERR_UNSUPPORTED
+                raise
+        else:
+            # the same sweep with rotary positions after reconstruction (keys rebuilt on tcgen05)
+            rms = _time_ms(bench.decode_calls_rope, reps=2, warm=1)
+            rs = rms / 1e3 / (w.D * w.T)
+            rope = {"kernel": "decode_rope_kernel (lla_decode_attn_rope)", "ms_per_sweep": rms,
+                    "avg_launch_us": rs * 1e6, "GB_s": nbytes / rs / 1e9, "hbm_frac": nbytes / rs / 1e9 / peak,
+                    "tokens_per_s_decode_only": bench.B / (rms / 1e3)}
+            if lla.lla_get_device_error() != 0:
+                raise RuntimeError(f"device error in the {name} RoPE decode measurement")
         row = {"config": config_dict(w, bench.lens, 1), "steps": steps, "warmup": warmup,
                "kernel": "decode_async_kernel (lla_decode_attn)", "bound": "hbm",
                "ms_per_step": ms, "tokens_per_s": bench.B / (ms / 1e3),
@@ -836,6 +851,8 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
                "latent_cache_GB": latent_cache_bytes(w, bench.lens) / 1e9,
                "fill": "N(0,1) bf16 latents written into every page (the decode reads the same bytes "
                        "as for encoded ones)"}
+        if rope is not None:
+            row["rope_decode"] = rope
         lens = bench.lens
         del bench
         torch.cuda.empty_cache()

@@ -232,7 +232,7 @@ typedef struct {
  *   q, cur_k      pre-RoPE: the call rotates them
  * Every other argument, the workspace (lla_decode_workspace_size) and the error behaviour are
  * those of lla_decode_attn.  Keys are rebuilt on the tensor cores: storage must be LLA_BF16,
- * d = 128 and (r_k, r_v) one of (96, 160), (128, 128), else LLA_ERR_UNSUPPORTED.  q, cur_k,
+ * d = 128 and (r_k, r_v) one of (96, 160), (128, 128), (192, 320), else LLA_ERR_UNSUPPORTED.  q, cur_k,
  * cur_v and out must be 16-byte aligned.
  */
 lla_status lla_decode_attn_rope(const lla_geometry *g, const lla_codec *codec,

@@ -67,7 +67,7 @@ struct RopeShape {
     static constexpr int NACC = 3;
     static constexpr int A_BASE = NACC * 64;
     static constexpr int A_COLS = RK / 2 + 8;
-    static constexpr int A_STRIDE = A_COLS <= 64 ? 64 : 96;
+    static constexpr int A_STRIDE = A_COLS <= 64 ? 64 : A_COLS <= 96 ? 96 : 128;
     static constexpr int TMEM_COLS = A_BASE + 2 * A_STRIDE <= 256 ? 256 : 512;
     static constexpr uint32_t IDESC = umma_idesc_bf16(kRopeD, 64, 0, 0);
     static_assert(RK % 32 == 0, "whole K steps, W_up,t^K rows in 16-column TMEM stores");
@@ -487,6 +487,7 @@ RopeEntry rope_entry(int es, int d, int r_k, int r_v) {
     if (es != 2 || d != kRopeD) return RopeEntry{nullptr, nullptr};
     if (r_k == 96 && r_v == 160) return RopeEntry{launch_rope<96, 160>, rope_layout_bytes<96, 160>};
     if (r_k == 128 && r_v == 128) return RopeEntry{launch_rope<128, 128>, rope_layout_bytes<128, 128>};
+    if (r_k == 192 && r_v == 320) return RopeEntry{launch_rope<192, 320>, rope_layout_bytes<192, 320>};
     return RopeEntry{nullptr, nullptr};
 }
 

@@ -75,7 +75,7 @@ def test_tiny_workload_two_pass_decode(lla, pairing, with_mu):
     assert lla.lla_get_device_error() == 0
 
 
-@pytest.mark.parametrize("rk,rv", [(96, 160), (128, 128)])
+@pytest.mark.parametrize("rk,rv", [(96, 160), (128, 128), (192, 320)])
 @pytest.mark.parametrize("base", [10000.0, 1e6])
 def test_ragged_batch(lla, rk, rv, base):
     """Empty (pass 1 only), one token, page-aligned, ragged tails and several pages in one
@@ -97,6 +97,15 @@ def test_long_sequences_split_across_many_ctas(lla):
         _check(sc, t, pass1=True)
     sc.append_token()
     _check(sc, 3, pass1=False, pairing=ADJ)
+
+
+def test_long_sequences_split_across_many_ctas_rho2(lla):
+    """The rho = 2 rank shape (192, 320): 64 KB head pages, two ring stages, W_up,t^K of 96
+    TMEM columns per A slot; long sequences split over CTAs, both passes."""
+    sc = Scene(lla, H=16, r_k=192, r_v=320, lens=[3000, 2100, 70], io="bf16", seed=48, with_mu=True)
+    _check(sc, 1, pass1=True)
+    sc.append_token()
+    _check(sc, 2, pass1=False, pairing=ADJ)
 
 
 def test_far_positions_keep_their_phase(lla):
