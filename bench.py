@@ -542,7 +542,7 @@ def run_decoupled_extra(bench, d_rope=64):
         del k
     qr = W.normal((w.D, w.T, bench.B, w.H, d_rope), w.seed, 501, device=bench.device)
     ckr = W.normal((w.D, w.T, bench.B, d_rope), w.seed, 502, device=bench.device)
-    ws = torch.empty(lla.lla_decode_decoupled_workspace_size(bench.geom, d_rope, bench.B), dtype=torch.uint8,
+    ws = torch.zeros(lla.lla_decode_decoupled_workspace_size(bench.geom, d_rope, bench.B), dtype=torch.uint8,
                      device=bench.device)
 
     def sweep():

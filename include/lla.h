@@ -360,10 +360,13 @@ lla_status lla_decode_decoupled_workspace_size(const lla_geometry *g, int32_t d_
  *   q_rope       device [B][H][d_rope] io_dtype: pre-rotation rotary queries
  *   cur_k_rope   device [B][d_rope] io_dtype, pass 1 (with cur_k, cur_v): the current token's
  *                pre-rotation rotary key; NULL in pass 2
- *   workspace    >= lla_decode_decoupled_workspace_size bytes; overwritten (no zero fill)
- * Other arguments and the error behaviour are those of lla_decode_attn; three launches on
- * `stream`.  Storage LLA_BF16, d = 128, H <= 64, (r_k, r_v) = (96, 160), d_rope 32, 64 or 96;
- * LLA_ERR_UNSUPPORTED otherwise.
+ *   workspace    >= lla_decode_decoupled_workspace_size bytes, zero-filled once before the first
+ *                call (lla_decode_workspace_init); as for lla_decode_attn, its split-KV counters
+ *                return to zero after every call
+ * Other arguments and the error behaviour are those of lla_decode_attn; one launch on `stream`
+ * (the absorbed decode kernel with the block's rotary plane streamed beside each head page).
+ * Storage LLA_BF16, d = 128, (r_k, r_v) = (96, 160), d_rope 32, 64 or 96; LLA_ERR_UNSUPPORTED
+ * otherwise.
  */
 lla_status lla_decode_attn_decoupled(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
                                      const void *rope_pool, int32_t d_rope, const lla_rope *rope,

@@ -27,7 +27,7 @@
 //   * A range that covers a (sequence, head) completely finishes it in place; ranges that split
 //     one write (m, l, o_latent) partials, and the last CTA to arrive (atomic counter) merges
 //     them by log-sum-exp, adds the current token and applies W_up,t^V, mu^V_t and 1/l.
-#include "lla_decode_common.cuh"
+#include "lla_decode_async.cuh"
 
 namespace lla {
 namespace {
@@ -167,228 +167,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
     empty_sequences(p, s);
 }
 
-template <int ES, int RK, int RV, int D>
-__global__ void __launch_bounds__(kAsyncThreads, 1) decode_async_kernel(const Params p) {
-    using F = Fast<ES, RK, RV>;
-    extern __shared__ __align__(128) char smem[];
-    const ASmem a = carve_async<ES, RK, RV, D>(smem, p);
-    const Smem &s = a.s;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-    pdl_wait();  // inputs may come from the previous kernel in the stream
-    if (tid == 0) {
-        for (int i = 0; i < kQSlots; ++i) mbar_init(&a.qready[i], kMThreads);
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(&a.stfull[i], kComputeThreads);
-            mbar_init(&a.stfree[i], kMThreads);
-        }
-    }
-    Range rg = prologue(p, s, F::S_THREADS, F::V_THREADS);  // fences the inits above too
-    order_runs(p, s, rg);
-    pdl_trigger();
-
-    if (warp == kComputeWarps) {
-        if (rg.A0 < rg.A1) named_bar_sync(kBarStart, kMThreads + 32);
-        producer(p, s, rg);
-        return;
-    }
-
-    if (tid >= kMBase) {
-        // ---------------------------------------------------------------- management warps
-        const int mt = tid - kMBase;
-        // set-ups run two runs ahead of finishes: set-up(r), then finish(r - 2), so that a short
-        // run is never followed by a wait for the next run's q~ behind a merge
-        auto finish = [&](const Run &R, int64_t u, int k) {
-            m_finish<ES, RK, RV, D, F::TT, F::NTG>(p, a, R, u, rg, k & 1, (k >> 1) & 1, k % kQSlots, mt);
-        };
-        int r = 0;
-        Run q0{}, q1{};  // runs r - 2 and r - 1, awaiting their finish
-        int64_t u0 = 0, u1 = 0;
-        for (int pass = 0; pass < 3; ++pass)
-        for (int64_t u = rg.lo[pass]; u < rg.hi[pass];) {
-            const Run R = locate_run(p, s, u, rg.hi[pass]);
-            const int slot = r % kQSlots;
-            m_setup<ES, RK, RV, D>(p, a, R.b, R.h, slot, mt, r == 0);
-            mbar_arrive(&a.qready[slot]);
-            if (r >= 2) finish(q0, u0, r - 2);
-            q0 = q1;
-            u0 = u1;
-            q1 = R;
-            u1 = u;
-            ++r;
-            u = R.run_end;
-        }
-        if (r >= 2) finish(q0, u0, r - 2);
-        if (r >= 1) finish(q1, u1, r - 1);
-        // sequences with no cached token: pass 1 attends to the current token only
-        const bool pass1 = p.cur_k != nullptr;
-        for (int b = 0; b < p.B; ++b) {
-            if (s.lens[b] != 0) continue;
-            for (int h = 0; h < p.H; ++h) {
-                if ((b * p.H + h) % gridDim.x != blockIdx.x) continue;
-                const int64_t row = (static_cast<int64_t>(b) * p.H + h) * D;
-                if (!pass1 && mt == 0) atomicOr(p.err, LLA_DEVERR_EMPTY_PASS2);
-                for (int e = mt; e < D; e += kMThreads)
-                    store_elem(p.out, row + e, pass1 ? load_elem(p.cur_v, row + e, p.io_bf16) : 0.f,
-                               p.io_bf16);
-            }
-        }
-        cp_async_wait_all();  // no copy into shared memory outlives the CTA
-        return;
-    }
-
-    // ------------------------------------------------------------------ score and value warps
-    const bool is_s = warp < F::S_WARPS;
-    const int ks = tid / F::TT, tt = tid % F::TT;  // score threads
-    const int vt = tid - F::S_THREADS;              // value threads
-    const int vc = vt % F::VC, tg = vt / F::VC;
-    const bool vwork = !is_s && tg < F::NTG;
-    constexpr int AV = F::UPT * F::VE;
-
-    int it = 0, stage = 0, r = 0;
-    uint32_t ph = 0;
-    for (int pass = 0; pass < 3; ++pass)
-    for (int64_t u = rg.lo[pass]; u < rg.hi[pass]; ++r) {
-        const Run R = locate_run(p, s, u, rg.hi[pass]);
-        const int rslot = r & 1;         // state slot
-        const int qslot = r % kQSlots;   // query slot
-        float beta = 0.f;
-        const float *qq = a.qlat + qslot * a.qslot + ks * F::NGT * F::KE;
-        // q~ of this thread's granules stays in registers for the whole run when it is small
-        // enough (up to 48 floats); else it is re-read from shared memory (a broadcast) per token
-        constexpr bool kQreg = F::NGT * F::KE <= 48;
-        float qr[kQreg ? F::NGT * F::KE : 1];
-        if (is_s) {
-            mbar_wait(&a.qready[qslot], (r / kQSlots) & 1, s.abort_flag, p.err, wait_limit(p));
-            beta = m_part(a, qslot, 1);
-            if constexpr (kQreg) {
-#pragma unroll
-                for (int g = 0; g < F::NGT; ++g) {
-                    if (F::NGK % F::KSPLIT != 0 && ks * F::NGT + g >= F::NGK) break;
-                    float t[F::KE];
-                    load_qvec<F::KE>(qq + g * F::KE, t);
-#pragma unroll
-                    for (int e = 0; e < F::KE; ++e) qr[g * F::KE + e] = t[e];
-                }
-            }
-        }
-        float m_run = -INFINITY, l_part = 0.f;
-        float accv[AV];
-#pragma unroll
-        for (int e = 0; e < AV; ++e) accv[e] = 0.f;
-
-        for (int k = 0; k < R.npages; k += F::PPS, ++it) {
-            const int slot = it & 1;
-            const uint32_t pph = (it >> 1) & 1;
-            const char *sb = s.ring + stage * p.stage_bytes;
-            const int n = min(F::PPS, R.npages - k);
-            const int tok0 = (R.pg0 + k) * kBlockTokens;
-            const int nvalid = min(n * kBlockTokens, R.Lb - tok0);
-            float *pring = s.psm + slot * kComputeThreads;
-
-            if (is_s) {
-                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err, wait_limit(p));
-                float sc[F::TPT];
-#pragma unroll
-                for (int i = 0; i < F::TPT; ++i) {
-                    const int tok = tt + i * F::TT;
-                    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-                    if (tok < nvalid) {
-                        const char *kp = sb + (tok >> 6) * F::HPB + (tok & 63) * F::GK +
-                                         ks * F::NGT * (kBlockTokens * F::GK);
-#pragma unroll
-                        for (int g = 0; g < F::NGT; ++g) {
-                            if (F::NGK % F::KSPLIT != 0 && ks * F::NGT + g >= F::NGK) break;
-                            float v[F::KE], qv[F::KE];
-                            load_gran<ES, F::GK>(kp + g * (kBlockTokens * F::GK), v);
-                            if constexpr (kQreg) {
-#pragma unroll
-                                for (int e = 0; e < F::KE; ++e) qv[e] = qr[g * F::KE + e];
-                            } else {
-                                load_qvec<F::KE>(qq + g * F::KE, qv);  // broadcast read
-                            }
-#pragma unroll
-                            for (int e = 0; e < F::KE; ++e) {
-                                if ((e & 3) == 0) a0 = fmaf(v[e], qv[e], a0);
-                                else if ((e & 3) == 1) a1 = fmaf(v[e], qv[e], a1);
-                                else if ((e & 3) == 2) a2 = fmaf(v[e], qv[e], a2);
-                                else a3 = fmaf(v[e], qv[e], a3);
-                            }
-                        }
-                    }
-                    sc[i] = (a0 + a1) + (a2 + a3);
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&s.empty[stage]);  // K-plane read
-                if constexpr (F::KSPLIT == 2) {
-                    if (ks == 1) {
-#pragma unroll
-                        for (int i = 0; i < F::TPT; ++i) s.spart[tt + i * F::TT] = sc[i];
-                    }
-                    named_bar_sync(kBarTok, F::S_THREADS);
-                    if (ks == 0) {
-#pragma unroll
-                        for (int i = 0; i < F::TPT; ++i) sc[i] += s.spart[tt + i * F::TT];
-                    }
-                }
-                float x[F::TPT];
-                float lm = -INFINITY;
-#pragma unroll
-                for (int i = 0; i < F::TPT; ++i) {
-                    const bool valid = tt + i * F::TT < nvalid;
-                    x[i] = valid ? (sc[i] + beta) * p.scale_log2 : -INFINITY;
-                    lm = fmaxf(lm, x[i]);
-                }
-                float *wmax = s.misc + kAWmax + slot * 8;
-                if (ks == 0) {
-                    lm = warp_max(lm);
-                    if (lane == 0) wmax[warp] = lm;
-                }
-                named_bar_sync(kBarTok, F::S_THREADS);
-                float ms = wmax[0];
-#pragma unroll
-                for (int w = 1; w < F::TT / 32; ++w) ms = fmaxf(ms, wmax[w]);
-                const float m_new = fmaxf(m_run, ms);
-                const float alpha = exp2f(m_run - m_new);
-                m_run = m_new;
-                if (ks == 0) {
-                    mbar_wait(&s.pempty[slot], pph ^ 1u, s.abort_flag, p.err, wait_limit(p));
-                    float lsum = 0.f;
-#pragma unroll
-                    for (int i = 0; i < F::TPT; ++i) {
-                        const float pv = (tt + i * F::TT < nvalid) ? exp2f(x[i] - m_new) : 0.f;
-                        pring[tt + i * F::TT] = pv;
-                        lsum += pv;
-                    }
-                    l_part = fmaf(l_part, alpha, lsum);
-                    if (tid == 0) s.misc[kAPAlpha + slot] = alpha;
-                }
-                mbar_arrive(&s.pfull[slot]);
-            } else {
-                mbar_wait(&s.full[stage], ph, s.abort_flag, p.err, wait_limit(p));
-                mbar_wait(&s.pfull[slot], pph, s.abort_flag, p.err, wait_limit(p));
-                if (vwork) value_step<ES, RK, RV>(accv, sb, pring, s.misc[kAPAlpha + slot], nvalid, vc, tg);
-                mbar_arrive(&s.pempty[slot]);
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&s.empty[stage]);  // V-plane read
-            }
-            if (++stage == p.stages) {
-                stage = 0;
-                ph ^= 1u;
-            }
-        }
-
-        // leave the run's softmax state in slot rslot for the management warps, once the run
-        // that used the slot before (r - 2) has been read
-        if (r >= 2) mbar_wait(&a.stfree[rslot], ((r - 2) >> 1) & 1, s.abort_flag, p.err, wait_limit(p));
-        if (is_s && ks == 0) a.lred[rslot * kLredSlot + tt] = l_part;
-        if (tid == 0) s.misc[kAM + rslot] = m_run;
-        if (vwork) value_store<ES, RK, RV>(a.red + rslot * a.redslot, accv, vc, tg);
-        mbar_arrive(&a.stfull[rslot]);
-        u = R.run_end;
-    }
-}
-
 template <int ES, int GK, int VB>
 lla_status launch_generic(const Params &prm, int grid, int smem, cudaStream_t stream) {
     static bool configured[64] = {};
@@ -398,7 +176,7 @@ lla_status launch_generic(const Params &prm, int grid, int smem, cudaStream_t st
 template <int ES, int RK, int RV>
 lla_status launch_fast(const Params &prm, int grid, int smem, cudaStream_t stream) {
     static bool configured[64] = {};
-    return launch_kernel(decode_async_kernel<ES, RK, RV, 128>, configured, prm, grid, smem, stream,
+    return launch_kernel(decode_async_kernel<ES, RK, RV, 128, 0>, configured, prm, grid, smem, stream,
                          kAsyncThreads);
 }
 

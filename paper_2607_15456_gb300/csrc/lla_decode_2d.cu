@@ -160,14 +160,6 @@ struct F2Params {
     const float *part;
 };
 
-// (cos, sin) of pos turns of phi / 2^64 (phi = theta / 2 pi in 64-bit fixed point): the product
-// wraps modulo one turn exactly, and 32 bits of the fraction reach sincospif.
-__device__ __forceinline__ void turn_sincos(long long pos, unsigned long long phi, float *sn, float *cs) {
-    const unsigned long long turns = static_cast<unsigned long long>(pos) * phi;
-    const float tf = __uint2float_rn(static_cast<uint32_t>(turns >> 32)) * 2.3283064365386963e-10f;
-    sincospif(2.f * tf, sn, cs);
-}
-
 // CTA c of `grid` holds the global pages [page_lo(c), page_lo(c + 1)) of the np pages; with
 // fewer pages than CTAs some CTAs hold none.
 __host__ __device__ __forceinline__ int page_lo(int c, int np, int grid) {
@@ -856,13 +848,6 @@ struct Rotary {
     int pairing;
 };
 
-// theta_j = base^(-2j/d_rope) in 64-bit fixed-point turns (theta_j <= 1 rad < 1 turn).
-void rotary_phases(int d_rope, double base, unsigned long long *phi) {
-    const double two_pi = 6.283185307179586476925286766559;
-    for (int j = 0; j < d_rope / 2; ++j)
-        phi[j] = static_cast<unsigned long long>(ldexp(pow(base, -2.0 * j / d_rope) / two_pi, 64));
-}
-
 template <int RK, int RV, int DR>
 lla_status launch_units(const DecodeArgs &a, const Rotary *rot, cudaStream_t stream) {
     using Z = Z2<RK, RV, DR>;
@@ -999,6 +984,13 @@ __global__ void __launch_bounds__(256) rope_key_store_kernel(const RKParams p) {
 
 }  // namespace
 
+// theta_j = base^(-2j/d_rope) in 64-bit fixed-point turns (theta_j <= 1 rad < 1 turn).
+void rotary_phases(int d_rope, double base, unsigned long long *phi) {
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int j = 0; j < d_rope / 2; ++j)
+        phi[j] = static_cast<unsigned long long>(ldexp(pow(base, -2.0 * j / d_rope) / two_pi, 64));
+}
+
 bool decode_2d_supported(int es, int d, int H, int r_k, int r_v) {
     return es == 2 && d == kD && H >= 1 && H <= kNQ &&
            ((r_k == 96 && r_v == 160) || (r_k == 128 && r_v == 128) || (r_k == 288 && r_v == 480));
@@ -1008,34 +1000,6 @@ size_t decode_2d_workspace_bytes(int r_k, int r_v, int B) {
     const int grid = num_sms();
     if (grid <= 0) return 0;
     return ws2_layout(r_k, r_v, kNQ, B, grid).total;
-}
-
-bool decode_decoupled_supported(int es, int d, int H, int r_k, int r_v, int d_rope) {
-    return es == 2 && d == kD && H >= 1 && H <= 64 && r_k == 96 && r_v == 160 &&
-           (d_rope == 32 || d_rope == 64 || d_rope == 96);
-}
-
-size_t decode_decoupled_workspace_bytes(int r_k, int r_v, int d_rope, int B, int H) {
-    const int grid = num_sms();
-    if (grid <= 0) return 0;
-    return ws2_layout(r_k + d_rope, r_v, 1, B * H, grid).total;
-}
-
-lla_status launch_decode_decoupled(const DecodeArgs &a, const void *rope_pool, int d_rope, double base,
-                                   int pairing, const void *q_rope, const void *cur_k_rope,
-                                   cudaStream_t stream) {
-    if (a.B == 0) return LLA_OK;
-    if (a.num_blocks * a.H >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // 32-bit TMA coordinate
-    Rotary rot = {};
-    rot.pool = static_cast<const char *>(rope_pool);
-    rot.q_rope = q_rope;
-    rot.cur_k_rope = cur_k_rope;
-    rot.pairing = pairing;
-    rotary_phases(d_rope, base, rot.phi);
-    if (a.r_k == 96 && a.r_v == 160 && d_rope == 32) return launch_units<96, 160, 32>(a, &rot, stream);
-    if (a.r_k == 96 && a.r_v == 160 && d_rope == 64) return launch_units<96, 160, 64>(a, &rot, stream);
-    if (a.r_k == 96 && a.r_v == 160 && d_rope == 96) return launch_units<96, 160, 96>(a, &rot, stream);
-    return LLA_ERR_UNSUPPORTED;
 }
 
 lla_status launch_rope_key_store(int d_rope, double base, int pairing, void *rope_pool, int64_t num_blocks,

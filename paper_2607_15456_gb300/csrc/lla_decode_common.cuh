@@ -304,7 +304,10 @@ __device__ __forceinline__ void order_runs(const Params &p, const Smem &s, Range
 // of its full barrier.  Every round issued before that found its stage released by all consumer
 // warps with the flag still down, so its previous round had landed; the last `stages` issued
 // rounds are then awaited with the full limit, so no copy outlives the CTA.
-__device__ void producer(const Params &p, const Smem &s, const Range &rg) {
+// With a rotary pool (the decoupled rotary branch, one page per step) the block's rotary plane of
+// `rope_bytes` lands right after the head page, on the same barrier.
+__device__ void producer(const Params &p, const Smem &s, const Range &rg, const char *rope_pool = nullptr,
+                         int rope_bytes = 0) {
     const int lane = threadIdx.x & 31;
     const int hpb = p.head_page_bytes;
     const uint64_t pol = policy_evict_first();
@@ -330,11 +333,15 @@ __device__ void producer(const Params &p, const Smem &s, const Range &rg) {
                         if (!halt) {
                             const bool ok = b0 >= 0 && b0 < p.num_blocks;
                             if (!ok) atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
-                            mbar_arrive_expect_tx(&s.full[stage], ok ? hpb : 0);
-                            if (ok)
-                                bulk_g2s(s.ring + stage * p.stage_bytes,
-                                         p.pool + b0 * p.block_bytes + static_cast<int64_t>(R.h) * hpb, hpb,
+                            mbar_arrive_expect_tx(&s.full[stage], ok ? hpb + rope_bytes : 0);
+                            if (ok) {
+                                char *dst = s.ring + stage * p.stage_bytes;
+                                bulk_g2s(dst, p.pool + b0 * p.block_bytes + static_cast<int64_t>(R.h) * hpb, hpb,
                                          &s.full[stage], pol);
+                                if (rope_pool)  // shared by the block's heads: read again from L2
+                                    bulk_g2s(dst + hpb, rope_pool + static_cast<int64_t>(b0) * rope_bytes,
+                                             rope_bytes, &s.full[stage], pol);
+                            }
                         }
                     }
                     if (__shfl_sync(0xffffffffu, halt, 0)) {

@@ -181,6 +181,14 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
+// (cos, sin) of pos turns of phi / 2^64 (phi = theta / 2 pi in 64-bit fixed point): the product
+// wraps modulo one turn exactly, and 32 bits of the fraction reach sincospif.
+__device__ __forceinline__ void turn_sincos(long long pos, unsigned long long phi, float *sn, float *cs) {
+    const unsigned long long turns = static_cast<unsigned long long>(pos) * phi;
+    const float tf = __uint2float_rn(static_cast<uint32_t>(turns >> 32)) * 2.3283064365386963e-10f;
+    sincospif(2.f * tf, sn, cs);
+}
+
 // Byte offset of element (row i, column j) inside a K-plane (see lla.h).
 __host__ __device__ __forceinline__ int64_t kplane_offset(int i, int j, int es, int gk) {
     const int byte = j * es;

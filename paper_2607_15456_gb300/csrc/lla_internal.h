@@ -104,8 +104,11 @@ lla_status launch_prefill_rope(const PrefillArgs &a, double base, int pairing, v
 bool decode_2d_supported(int es, int d, int H, int r_k, int r_v);
 size_t decode_2d_workspace_bytes(int r_k, int r_v, int B);
 lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream);
-// Per-head LLA decode with the decoupled rotary branch (App. J): the shapes with a kernel, the
-// workspace for B sequences of H heads, launch (rope_pool [num_blocks][64 x d_rope] rotary planes,
+// theta_j = base^(-2j/d_rope) of each rotation pair in 64-bit fixed-point turns.
+void rotary_phases(int d_rope, double base, unsigned long long *phi);
+// Per-head LLA decode with the decoupled rotary branch (App. J) on the absorbed decode kernel: the
+// shapes with a kernel, the workspace for B sequences of H heads (the absorbed decode's: zeroed
+// once, its counters return to zero), launch (rope_pool [num_blocks][64 x d_rope] rotary planes,
 // q_rope [B][H][d_rope], cur_k_rope [B][d_rope] in pass 1); and the rotary-key store.
 bool decode_decoupled_supported(int es, int d, int H, int r_k, int r_v, int d_rope);
 size_t decode_decoupled_workspace_bytes(int r_k, int r_v, int d_rope, int B, int H);

@@ -75,7 +75,7 @@ def decode_case(args):
             pools.append(pool)
         qr = W.normal((bench.B, w.H, d_rope), w.seed, 501, device=dev)
         ckr = W.normal((bench.B, d_rope), w.seed, 502, device=dev)
-        dws = torch.empty(lla.lla_decode_decoupled_workspace_size(bench.geom, d_rope, bench.B),
+        dws = torch.zeros(lla.lla_decode_decoupled_workspace_size(bench.geom, d_rope, bench.B),
                           dtype=torch.uint8, device=dev)
     if args.case == "loops":
         lws = torch.zeros(lla.lla_decode_loops_workspace_size(bench.geom, bench.B), dtype=torch.uint8,

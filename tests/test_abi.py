@@ -346,7 +346,7 @@ def test_decoupled_argument_checks(lib):
     assert so.lla_rope_plane_bytes(64, ctypes.byref(n)) == OK and n.value == 64 * 64 * 2
     assert so.lla_rope_plane_bytes(40, ctypes.byref(n)) == INVALID
     g = _g(lib)
-    for bad in (_g(lib, r_k=72, r_v=120), _g(lib, d=64), _g(lib, H=65), _g(lib, storage="fp32")):
+    for bad in (_g(lib, r_k=72, r_v=120), _g(lib, d=64), _g(lib, storage="fp32")):
         assert so.lla_decode_decoupled_workspace_size(ctypes.byref(bad), 64, 4, ctypes.byref(n)) == UNSUPPORTED
     assert so.lla_decode_decoupled_workspace_size(ctypes.byref(g), 48, 4, ctypes.byref(n)) == UNSUPPORTED
 

@@ -5,9 +5,9 @@ decoupled rotary branch, App. J "Absorbed attention") against the CPU float64 or
 The latent cache comes from lla_encode as in test_decode_gpu.py; one rotary key per token (shared
 by every loop and head) is stored turned at the token's position.  The oracle rebuilds every
 content key by Eq. decode, joins it with the rotary key turned at its position, and runs plain
-softmax attention; the GPU reads the head's K-plane and the block's rotary plane as one score
-operand on the tensor cores.  Tolerances: bf16 storage, max abs <= 2e-2 (before the final
-rounding of bf16 outputs) and relative L2 <= 5e-3.
+softmax attention; the GPU streams the block's rotary plane beside each head page and extends
+every token's absorbed score over the rotary dimensions.  Tolerances: bf16 storage, max abs
+<= 2e-2 (before the final rounding of bf16 outputs) and relative L2 <= 5e-3.
 """
 import numpy as np
 import pytest
@@ -42,7 +42,7 @@ class Rotary:
             pos = torch.cat([torch.arange(L, dtype=torch.int32) for L in sc.lens]).to(DEV)
             lla.lla_encode_rope_keys(d_rope, base, pairing, self.pool, sc.pt.num_blocks, self.k, pos,
                                      sc.slots)
-        self.ws = torch.empty(lla.lla_decode_decoupled_workspace_size(sc.geom, d_rope, sc.B),
+        self.ws = torch.zeros(lla.lla_decode_decoupled_workspace_size(sc.geom, d_rope, sc.B),
                               dtype=torch.uint8, device=DEV)
 
     def append(self, key=61):
