@@ -29,14 +29,6 @@
 //   finish2d_kernel   per (head, up to 8 sequences): merges the runs of each sequence, adds the
 //                     pass-1 current token, and applies W_up,t,h^V once for those sequences
 // Storage bf16, d = 128, H <= 16; accumulators fp32 in TMEM.
-//
-// The same kernels take the decoupled rotary branch of per-head LLA (App. J "Absorbed
-// attention": an MLA-style NoPE content path plus a small explicit rotary branch shared across
-// recurrence steps for each token).  The attention kernel's unit of work is then one (sequence,
-// head) with one query instead of one sequence with H queries: a unit's pages are the head's
-// latent pages, and its score operand is the head's K-plane followed by the block's rotary plane
-// (64 rotary keys of d_rope dims, turned at their positions when stored), against
-// [q~; rot(q^R, P)]; H up to 64.  rope_key_store_kernel writes the rotary planes.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -65,15 +57,15 @@ constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one sequence fit
 
 // Shared-memory plan of the attention kernel for ranks (RK, RV).  Offsets from a 1024-byte
 // aligned base (128-byte swizzle atoms of the V stages).
-template <int RK, int RV, int DR = 0>
+template <int RK, int RV>
 struct Z2 {
-    static constexpr int RKX = RK + DR;                 // score contraction: latent, then rotary key
-    static constexpr int NQM = DR > 0 ? 1 : kNQ;        // queries of a unit (LLA-2D: the heads)
+    static constexpr int RKX = RK;                      // score contraction
+    static constexpr int NQM = kNQ;                     // queries of a sequence (its heads, padded)
     static constexpr int NCH = (RV + 127) / 128;        // 128-row chunks of O^T
     static constexpr int NBOX = (RV + 63) / 64;         // TMA boxes a V-plane loads
     static constexpr int BOX = kPT * 128;               // one box: 64 rows x 128 bytes
     static constexpr int KPLANE = kPT * RK * 2;
-    static constexpr int KPAGE = kPT * RKX * 2;         // K-plane, then the rotary plane
+    static constexpr int KPAGE = kPT * RKX * 2;         // K-plane
     static constexpr int VPAGE = NCH * 2 * BOX;         // two boxes per chunk, loaded or zero
     static constexpr int VBYTES = NBOX * BOX;
     static constexpr int QB = kNS * RKX * 2;            // [Q~_hi; Q~_lo] operand
@@ -97,7 +89,7 @@ struct Z2 {
     // a run partial: O^T of each query ([NQM][RV]), then 16 maxima and 16 sums
     static constexpr int PSTRIDE = NQM * RV + 2 * kNQ;
     static constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
-    static_assert(RK % 16 == 0 && DR % 16 == 0 && RV % 32 == 0 && NCH <= 4, "ranks");
+    static_assert(RK % 16 == 0 && RV % 32 == 0 && NCH <= 4, "ranks");
     static_assert(ST >= 2, "pipeline depth");
     static_assert(SMEM <= kSmemCap, "shared memory");
     static_assert(TM_O + NCH * kNQ <= TM_COLS, "TMEM columns");
@@ -112,30 +104,22 @@ enum {
 
 struct A2Params {
     int T, H, loop, io_bf16, pass1, B, max_ctx, max_blocks;
-    int upr;         // units per sequence: 1 (LLA-2D) or H (decoupled: one unit per head)
-    int decoupled;   // per-head codec [H][T][d][r] with a rotary branch, else LLA-2D [T][H][d][r]
     float scale_log2;
-    const void *w_up_k;
-    const float *mu_k;   // LLA-2D [T*H*d], decoupled [H][T*d], or NULL
+    const void *w_up_k;  // [T][H][d][r_k]
+    const float *mu_k;   // [T*H*d] or NULL
     const void *q;       // [B][H][d]
-    const void *q_rope;  // decoupled: [B][H][d_rope]
-    int d_rope, pairing;
-    unsigned long long phi[48];  // decoupled: theta_j in 64-bit fixed-point turns
     const int32_t *context_lens;
-    float *qt;           // [units][NQM][RK + DR]: q~ (and rot(q^R)) * scale * log2 e
-    float *beta;         // [units][NQM]: beta * scale * log2 e
-    int *pstart;         // [units + 1]: first global page of each unit
+    float *qt;           // [B][16][RK]: q~ * scale * log2 e
+    float *beta;         // [B][16]: beta * scale * log2 e
+    int *pstart;         // [B + 1]: first global page of each sequence
     unsigned *err;
 };
 
 struct T2Params {
-    int nq;   // queries of a unit: H (LLA-2D) or 1 (decoupled)
-    int upr;  // units per sequence; unit u is head u % upr of sequence u / upr
-    int B;    // units
+    int nq;   // queries of a sequence: H
+    int B;
     const char *pool;
     int64_t num_blocks, page_bytes;
-    const char *rope_pool;  // decoupled: [num_blocks][rotary plane]
-    int64_t rope_page_bytes;
     const int32_t *block_table;
     int max_blocks;
     const int32_t *context_lens;
@@ -149,12 +133,10 @@ struct T2Params {
 struct F2Params {
     int T, H, loop, io_bf16, B, grid;
     int spb;  // sequences per CTA (1 .. 8)
-    int upr, decoupled, d_rope;
     float scale_log2;
     const void *w_up_v;  // [T][H][d][r_v] bf16
     const float *mu_v;   // [T*H*d] or NULL
     const void *q, *cur_k, *cur_v;
-    const void *q_rope, *cur_k_rope;  // decoupled: [B][H][d_rope], [B][d_rope]
     void *out;
     const int *pstart;
     const float *part;
@@ -173,16 +155,16 @@ __host__ __device__ __forceinline__ int cta_of(int g, int np, int grid) {
 
 // ------------------------------------------------------------------------- absorb kernel
 
-// One CTA: the page prefix sums of the batch's units (unit u is head u % upr of sequence
-// u / upr) with the length checks; an invalid length counts as an empty sequence.
+// One CTA: the page prefix sums of the batch's sequences with the length checks; an invalid
+// length counts as an empty sequence.
 __device__ void page_prefix(const A2Params &p) {
     __shared__ int wsum[8];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int U = p.B * p.upr;
-    const int per = (U + 255) / 256;  // units of this thread: [tid per, (tid + 1) per)
+    const int U = p.B;
+    const int per = (U + 255) / 256;  // sequences of this thread: [tid per, (tid + 1) per)
     const int limit = min(p.max_ctx, p.max_blocks * kPT);
     auto pages = [&](int u, bool flag) {
-        const int L = p.context_lens[u / p.upr];
+        const int L = p.context_lens[u];
         if (L < 0 || L > limit) {
             if (flag) atomicOr(p.err, LLA_DEVERR_CONTEXT);
             return 0;
@@ -191,7 +173,7 @@ __device__ void page_prefix(const A2Params &p) {
         return (L + kPT - 1) / kPT;
     };
     int tot = 0;
-    for (int u = tid * per; u < min(U, (tid + 1) * per); ++u) tot += pages(u, u % p.upr == 0);
+    for (int u = tid * per; u < min(U, (tid + 1) * per); ++u) tot += pages(u, true);
     int x = tot;  // inclusive scan over the warp
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -212,25 +194,19 @@ __device__ void page_prefix(const A2Params &p) {
 
 // Grid (H, RK / 32, ceil(B / 16)), 256 threads = 32 columns x 8 slices of 16 rows of the head:
 // q~ of 32 columns of head h for 16 sequences, every weight load of a thread in flight at once;
-// beta of head h (and, with the rotary branch, rot(q^R, P)) by the CTAs of the first column
-// chunk.  The weight slice of (loop t, head h) is (t, h) of [T][H] for LLA-2D and (h, t) of
-// [H][T] for the per-head codec of the rotary branch.
-template <int RK, int DR>
+// beta of head h by the CTAs of the first column chunk.  The weight slice of (loop t, head h) is
+// (t, h) of [T][H].
+template <int RK>
 __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
     static_assert(RK % 32 == 0, "column chunks");
-    constexpr int RKX = RK + DR;
-    constexpr int NQM = DR > 0 ? 1 : kNQ;
     __shared__ float qs[16][kD];
     __shared__ float red[8][16][33];
     const int h = blockIdx.x, j0 = blockIdx.y * 32, b0 = blockIdx.z * 16, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(16, p.B - b0);
-    const int64_t th = p.decoupled ? static_cast<int64_t>(h) * p.T + p.loop
-                                   : static_cast<int64_t>(p.loop) * p.H + h;
-    // the output row of (sequence b, head h): query h of unit b, or query 0 of unit b H + h
-    auto row = [&](int b) {
-        return p.decoupled ? static_cast<int64_t>(b) * p.H + h : static_cast<int64_t>(b) * NQM + h;
-    };
+    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
+    // the output row of (sequence b, head h): query h of sequence b
+    auto row = [&](int b) { return static_cast<int64_t>(b) * kNQ + h; };
     pdl_wait();  // inputs may come from the previous kernel; the workspace is free after it
     // this thread's 16 weights (column j0 + lane, rows 16 warp .. 16 warp + 15), in flight while
     // the queries load
@@ -258,7 +234,7 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
         float a = 0.f;
 #pragma unroll
         for (int sl = 0; sl < 8; ++sl) a += red[sl][bi][c];
-        if (bi < nb) p.qt[row(b0 + bi) * RKX + j0 + c] = a * p.scale_log2;
+        if (bi < nb) p.qt[row(b0 + bi) * RK + j0 + c] = a * p.scale_log2;
     }
     if (blockIdx.y == 0) {
         // beta_h = q_h . mu^K_{t,h}: warp w takes sequences w and w + 8
@@ -268,26 +244,6 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
                 for (int e = lane; e < kD; e += 32) s = fmaf(qs[bi][e], p.mu_k[th * kD + e], s);
             s = warp_sum(s);
             if (lane == 0) p.beta[row(b0 + bi)] = s * p.scale_log2;
-        }
-        if constexpr (DR > 0) {
-            // the rotary query turned at the current token's position: context_lens[b] in
-            // pass 1, context_lens[b] - 1 in pass 2
-            constexpr int HP = DR / 2;
-            for (int i = tid; i < nb * HP; i += 256) {
-                const int bi = i / HP, j = i - bi * HP;
-                const int b = b0 + bi;
-                const int L = p.context_lens[b];
-                const long long P = max(0, p.pass1 ? L : L - 1);
-                float sn, cs;
-                turn_sincos(P, p.phi[j], &sn, &cs);
-                const int a = p.pairing ? 2 * j : j, c = p.pairing ? 2 * j + 1 : j + HP;
-                const int64_t src = (static_cast<int64_t>(b) * p.H + h) * DR;
-                const float x = load_elem(p.q_rope, src + a, p.io_bf16);
-                const float y = load_elem(p.q_rope, src + c, p.io_bf16);
-                float *dst = p.qt + row(b) * RKX + RK;
-                dst[a] = (x * cs - y * sn) * p.scale_log2;
-                dst[c] = (x * sn + y * cs) * p.scale_log2;
-            }
         }
     }
     __syncthreads();
@@ -307,10 +263,10 @@ __device__ __forceinline__ int first_seq(const int *pstart, int B, int g0) {
     return lo;
 }
 
-template <int RK, int RV, int DR>
+template <int RK, int RV>
 __global__ void __launch_bounds__(kT2, 1)
     attn2d_kernel(const __grid_constant__ CUtensorMap tv, const T2Params p) {
-    using Z = Z2<RK, RV, DR>;
+    using Z = Z2<RK, RV>;
     extern __shared__ __align__(1024) char sm_raw[];
     char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + Z::oBar);
@@ -373,8 +329,7 @@ __global__ void __launch_bounds__(kT2, 1)
                 const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
                 if (s0 >= g1) break;
                 const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
-                const int32_t *bt = p.block_table + static_cast<int64_t>(b / p.upr) * p.max_blocks;
-                const int head = b % p.upr;
+                const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks;
                 for (int pg = pa; pg < pe; ++pg) {
                     const int it = itk;
                     const int st = it % Z::ST;
@@ -384,7 +339,7 @@ __global__ void __launch_bounds__(kT2, 1)
                         atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
                         blk = 0;
                     }
-                    const int64_t page = static_cast<int64_t>(blk) * p.upr + head;  // head page
+                    const int64_t page = blk;
                     if (!mbar_wait(&bar[bKempty + st], ph ^ 1u, abort_flag, p.err) || *abort_flag) {
                         stop = true;
                         break;
@@ -392,9 +347,6 @@ __global__ void __launch_bounds__(kT2, 1)
                     mbar_arrive_expect_tx(&bar[bKfull + st], Z::KPAGE);
                     char *ks = sm + Z::oK + st * Z::KPAGE;
                     bulk_g2s(ks, p.pool + page * p.page_bytes, Z::KPLANE, &bar[bKfull + st], pol);
-                    if constexpr (DR > 0)  // the block's rotary plane continues the K-plane
-                        bulk_g2s(ks + Z::KPLANE, p.rope_pool + blk * p.rope_page_bytes, Z::KPAGE - Z::KPLANE,
-                                 &bar[bKfull + st], pol);
                     ++itk;
                     if (!mbar_wait(&bar[bVempty + st], ph ^ 1u, abort_flag, p.err) || *abort_flag) {
                         stop = true;
@@ -489,8 +441,8 @@ __global__ void __launch_bounds__(kT2, 1)
             if (s0 >= g1) break;
             const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
             if (pe <= pa) continue;
-            const int L = p.context_lens[b / p.upr];
-            // q~ of the unit as a K-major operand of 32 rows: row n = bf16(q~_n), row 16 + n =
+            const int L = p.context_lens[b];
+            // q~ of the sequence as a K-major operand of 32 rows: row n = bf16(q~_n), row 16 + n =
             // bf16(q~_n - row n), granule g of row n at g*512 + n*16; and beta
             if (r > 0) mbar_wait(&bar[bQfree], (r - 1) & 1, abort_flag, p.err);
             {
@@ -674,7 +626,7 @@ __global__ void __launch_bounds__(kT2, 1)
 
 // Grid (H, ceil(B / spb)), 128 threads (thread e = output element e of head h).  spb (at most 8)
 // sequences share one pass over W_up,t,h^V; small batches take fewer per CTA to use more SMs.
-// (Sequence b, head h) is query h of unit b (LLA-2D) or query 0 of unit b H + h (decoupled).
+// (Sequence b, head h) is query h of sequence b.
 template <int RV, int NQM>
 __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     constexpr int PS = NQM * RV + 2 * kNQ;
@@ -686,22 +638,21 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     const int h = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(p.spb, p.B - b0);
-    const int64_t th = p.decoupled ? static_cast<int64_t>(h) * p.T + p.loop
-                                   : static_cast<int64_t>(p.loop) * p.H + h;
-    const int qn = p.decoupled ? 0 : h;  // the query of (b, h) within its unit
+    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
+    const int qn = h;  // the query of (b, h) within its sequence
     pdl_wait();
-    const int NP = p.pstart[p.B * p.upr];
+    const int NP = p.pstart[p.B];
     for (int bi = 0; bi < kFinishSeqs; ++bi) {
         if (bi >= nb) {
             for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
             continue;
         }
         const int b = b0 + bi;
-        const int u = p.decoupled ? b * p.upr + h : b;  // the unit of (b, h)
+        const int u = b;
         const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
         float M = -INFINITY, l = 0.f;
         if (s1 > s0) {
-            // the runs of unit u: the CTAs c0 .. c1 that hold pages (a CTA between them may
+            // the runs of sequence u: the CTAs c0 .. c1 that hold pages (a CTA between them may
             // hold none and writes nothing), partials at slots u + c
             const int c0 = cta_of(s0, NP, p.grid), c1 = cta_of(s1 - 1, NP, p.grid);
             const int nr = c1 - c0 + 1;
@@ -745,15 +696,11 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
         } else {
             for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
         }
-        // pass 1: the current token's score against its exact key (with the rotary branch, also
-        // q^R . k^R_cur: both turn at the current position, so the rotation cancels)
+        // pass 1: the current token's score against its exact key
         float sc = -INFINITY;
         if (p.cur_k) {
             const int64_t row = (static_cast<int64_t>(b) * p.H + h) * kD;
             float v = load_elem(p.q, row + tid, p.io_bf16) * load_elem(p.cur_k, row + tid, p.io_bf16);
-            if (p.decoupled && tid < p.d_rope)
-                v = fmaf(load_elem(p.q_rope, (static_cast<int64_t>(b) * p.H + h) * p.d_rope + tid, p.io_bf16),
-                         load_elem(p.cur_k_rope, static_cast<int64_t>(b) * p.d_rope + tid, p.io_bf16), v);
             v = warp_sum(v);
             __syncthreads();  // redm / reds are free
             if (lane == 0) reds[warp] = v;
@@ -840,42 +787,31 @@ WS2 ws2_layout(int rkx, int r_v, int nqm, int U, int grid) {
     return w;
 }
 
-// The rotary branch of a decoupled call (unused by LLA-2D).
-struct Rotary {
-    const char *pool;  // [num_blocks][64 x d_rope] rotary planes
-    const void *q_rope, *cur_k_rope;
-    unsigned long long phi[48];
-    int pairing;
-};
-
-template <int RK, int RV, int DR>
-lla_status launch_units(const DecodeArgs &a, const Rotary *rot, cudaStream_t stream) {
-    using Z = Z2<RK, RV, DR>;
-    constexpr bool kDec = DR > 0;
+template <int RK, int RV>
+lla_status launch_units(const DecodeArgs &a, cudaStream_t stream) {
+    using Z = Z2<RK, RV>;
     lla_status st = LLA_OK;
     unsigned *err = device_error_word(&st);
     if (st != LLA_OK) return st;
     const int grid = num_sms();
     if (grid <= 0 || grid > kMaxGrid) return LLA_ERR_UNSUPPORTED;
-    const int upr = kDec ? a.H : 1;
-    const int U = a.B * upr;
-    const WS2 w = ws2_layout(Z::RKX, RV, Z::NQM, U, grid);
+    const WS2 w = ws2_layout(Z::RKX, RV, Z::NQM, a.B, grid);
     if (a.workspace_bytes < w.total) return LLA_ERR_WORKSPACE;
     char *ws = static_cast<char *>(a.workspace);
     static bool configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV, DR>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
+        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
             cudaSuccess)
             return LLA_ERR_CUDA;
         configured[dev] = true;
     }
     const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
-    // the V-planes of every head page: [num_blocks * upr][64 tokens][r_v] bf16
+    // the V-planes of every page: [num_blocks][64 tokens][r_v] bf16
     CUtensorMap tv;
     const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT),
-                              static_cast<uint64_t>(a.num_blocks) * upr};
+                              static_cast<uint64_t>(a.num_blocks)};
     const uint64_t strides[2] = {static_cast<uint64_t>(RV) * 2, static_cast<uint64_t>(page_bytes)};
     const uint32_t box[3] = {64, kPT, 1};
     if (!encode_tmap_bf16(&tv, static_cast<const char *>(a.pool) + kPT * RK * 2, 3, dims, strides, box, true))
@@ -884,49 +820,32 @@ lla_status launch_units(const DecodeArgs &a, const Rotary *rot, cudaStream_t str
     A2Params ap = {};
     ap.T = a.T; ap.H = a.H; ap.loop = a.loop; ap.io_bf16 = a.io_bf16; ap.pass1 = a.cur_k != nullptr;
     ap.B = a.B; ap.max_ctx = a.max_ctx; ap.max_blocks = a.max_blocks;
-    ap.upr = upr; ap.decoupled = kDec ? 1 : 0;
     ap.scale_log2 = a.scale * kLog2e;
     ap.w_up_k = a.w_up_k; ap.mu_k = a.mu_k; ap.q = a.q; ap.context_lens = a.context_lens;
-    if (kDec) {
-        ap.q_rope = rot->q_rope;
-        ap.d_rope = DR;
-        ap.pairing = rot->pairing;
-        memcpy(ap.phi, rot->phi, sizeof(ap.phi));
-    }
     ap.qt = reinterpret_cast<float *>(ws + w.qt);
     ap.beta = reinterpret_cast<float *>(ws + w.beta);
     ap.pstart = reinterpret_cast<int *>(ws + w.pstart);
     ap.err = err;
-    if ((st = launch_ex(absorb2d_kernel<RK, DR>, dim3(a.H, RK / 32, (a.B + 15) / 16), 256, 0, stream, ap)) !=
-        LLA_OK)
+    if ((st = launch_ex(absorb2d_kernel<RK>, dim3(a.H, RK / 32, (a.B + 15) / 16), 256, 0, stream, ap)) != LLA_OK)
         return st;
 
     T2Params tp = {};
-    tp.nq = kDec ? 1 : a.H; tp.upr = upr; tp.B = U;
+    tp.nq = a.H; tp.B = a.B;
     tp.pool = static_cast<const char *>(a.pool);
     tp.num_blocks = a.num_blocks; tp.page_bytes = page_bytes;
-    if (kDec) {
-        tp.rope_pool = rot->pool;
-        tp.rope_page_bytes = static_cast<int64_t>(kPT) * DR * 2;
-    }
     tp.block_table = a.block_table; tp.max_blocks = a.max_blocks;
     tp.context_lens = a.context_lens;
     tp.qt = ap.qt; tp.beta = ap.beta; tp.pstart = ap.pstart;
     tp.part = reinterpret_cast<float *>(ws + w.part);
     tp.err = err;
-    if ((st = launch_ex(attn2d_kernel<RK, RV, DR>, dim3(grid), kT2, Z::SMEM, stream, tv, tp)) != LLA_OK)
+    if ((st = launch_ex(attn2d_kernel<RK, RV>, dim3(grid), kT2, Z::SMEM, stream, tv, tp)) != LLA_OK)
         return st;
 
     F2Params fp = {};
     fp.T = a.T; fp.H = a.H; fp.loop = a.loop; fp.io_bf16 = a.io_bf16; fp.B = a.B; fp.grid = grid;
-    fp.upr = upr; fp.decoupled = kDec ? 1 : 0; fp.d_rope = DR;
     fp.scale_log2 = ap.scale_log2;
     fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
     fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
-    if (kDec) {
-        fp.q_rope = rot->q_rope;
-        fp.cur_k_rope = rot->cur_k_rope;
-    }
     fp.pstart = ap.pstart; fp.part = tp.part;
     // about two finish CTAs per SM: fewer sequences per CTA for small batches
     const int64_t want = static_cast<int64_t>(a.B) * a.H;
@@ -1023,7 +942,7 @@ lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream) {
     if (a.B == 0) return LLA_OK;
     if (a.num_blocks >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // 32-bit TMA coordinate
 #define LLA_2D(K, V) \
-    if (a.r_k == K && a.r_v == V) return launch_units<K, V, 0>(a, nullptr, stream);
+    if (a.r_k == K && a.r_v == V) return launch_units<K, V>(a, stream);
     LLA_2D(96, 160)
     LLA_2D(128, 128)
     LLA_2D(288, 480)
