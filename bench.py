@@ -842,6 +842,27 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
                     "tokens_per_s_decode_only": bench.B / (rms / 1e3)}
             if lla.lla_get_device_error() != 0:
                 raise RuntimeError(f"device error in the {name} RoPE decode measurement")
+        loops = None
+        lws = torch.zeros(1, dtype=torch.uint8, device=device)
+        try:  # the T loops of a layer in one pass over its latents, where a kernel shape exists
+            lws = torch.zeros(lla.lla_decode_loops_workspace_size(bench.geom, bench.B), dtype=torch.uint8,
+                              device=device)
+            bench.decode_calls_loops(lws)
+        except lla.LLAError as e:
+            if e.status != 2:  # LLA_ERR_UNSUPPORTED
+                raise
+        else:
+            lms = _time_ms(lambda: bench.decode_calls_loops(lws), reps=2, warm=1)
+            ls_ = lms / 1e3 / w.D
+            lbytes = (sum(bench.lens) * w.H * (w.r_k + w.r_v) * 2
+                      + w.T * (w.H * w.d * (w.r_k + w.r_v) * 2 + 4 * bench.B * w.H * w.d * 2))
+            loops = {"kernel": "decode_loops_kernel (lla_decode_attn_loops)", "ms_per_sweep": lms,
+                     "avg_launch_us": ls_ * 1e6, "GB_s": lbytes / ls_ / 1e9, "hbm_frac": lbytes / ls_ / 1e9 / peak,
+                     "bytes_per_launch": lbytes, "tokens_per_s_decode_only": bench.B / (lms / 1e3),
+                     "note": "all T loops of a layer per call: the layer's latents cross HBM once"}
+            if lla.lla_get_device_error() != 0:
+                raise RuntimeError(f"device error in the {name} multi-loop decode measurement")
+        del lws
         row = {"config": config_dict(w, bench.lens, 1), "steps": steps, "warmup": warmup,
                "kernel": "decode_async_kernel (lla_decode_attn)", "bound": "hbm",
                "ms_per_step": ms, "tokens_per_s": bench.B / (ms / 1e3),
@@ -853,6 +874,8 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
                        "as for encoded ones)"}
         if rope is not None:
             row["rope_decode"] = rope
+        if loops is not None:
+            row["loops_decode"] = loops
         lens = bench.lens
         del bench
         torch.cuda.empty_cache()

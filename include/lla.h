@@ -201,7 +201,7 @@ lla_status lla_decode_loops_workspace_size(const lla_geometry *g, int32_t B, siz
  *   workspace             >= lla_decode_loops_workspace_size bytes, zero-filled before first use;
  *                         every completed call leaves it zero-filled again
  * Other arguments and the error behaviour are those of lla_decode_attn.  Storage LLA_BF16, d = 128,
- * T = 4 and (r_k, r_v) one of (96, 160), (128, 128); LLA_ERR_UNSUPPORTED otherwise.
+ * T = 4 and (r_k, r_v) one of (96, 160), (128, 128), (72, 120); LLA_ERR_UNSUPPORTED otherwise.
  */
 lla_status lla_decode_attn_loops(const lla_geometry *g, const lla_codec *codec,
                                  const lla_cache *cache, const int32_t *context_lens, int32_t B,
@@ -232,7 +232,8 @@ typedef struct {
  *   q, cur_k      pre-RoPE: the call rotates them
  * Every other argument, the workspace (lla_decode_workspace_size) and the error behaviour are
  * those of lla_decode_attn.  Keys are rebuilt on the tensor cores: storage must be LLA_BF16,
- * d = 128 and (r_k, r_v) one of (96, 160), (128, 128), (192, 320), else LLA_ERR_UNSUPPORTED.  q, cur_k,
+ * d = 128 and (r_k, r_v) one of (96, 160), (128, 128), (192, 320), (72, 120), else
+ * LLA_ERR_UNSUPPORTED.  q, cur_k,
  * cur_v and out must be 16-byte aligned.
  */
 lla_status lla_decode_attn_rope(const lla_geometry *g, const lla_codec *codec,

@@ -21,7 +21,12 @@ constexpr int kComputeThreads = kComputeWarps * 32;
 constexpr int kThreads = kComputeThreads + 32;  // + one producer warp
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
-constexpr int kStepTargetBytes = 48 * 1024;  // most data per pipeline step (whole head pages)
+// Most data per pipeline step (whole head pages).  A file whose kernel takes one head page per
+// step defines LLA_DECODE_STEP_BYTES as 32 KB before including this header.
+#ifndef LLA_DECODE_STEP_BYTES
+#define LLA_DECODE_STEP_BYTES (48 * 1024)
+#endif
+constexpr int kStepTargetBytes = LLA_DECODE_STEP_BYTES;
 constexpr int kBarAll = 1;  // named barrier over the 256 consumer threads
 constexpr int kBarTok = 2;  // named barrier over the score threads
 

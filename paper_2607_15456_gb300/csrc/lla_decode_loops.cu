@@ -17,6 +17,8 @@
 // states, the value warps keep T latent sums (one 16-byte unit of 8 latents per thread, so that a
 // run's state stays small), and the management warps set up and finish the T loops of a run one
 // after the other through per-loop views of the run state.
+// one head page per pipeline step at every rank shape this kernel takes
+#define LLA_DECODE_STEP_BYTES (32 * 1024)
 #include "lla_decode_common.cuh"
 
 namespace lla {
@@ -425,6 +427,7 @@ LoopsEntry loops_entry(int es, int d, int T, int r_k, int r_v) {
     if (es != 2 || d != 128 || T != kNQ) return LoopsEntry{nullptr, nullptr};
     if (r_k == 96 && r_v == 160) return LoopsEntry{launch_loops<96, 160>, loops_layout_bytes<96, 160>};
     if (r_k == 128 && r_v == 128) return LoopsEntry{launch_loops<128, 128>, loops_layout_bytes<128, 128>};
+    if (r_k == 72 && r_v == 120) return LoopsEntry{launch_loops<72, 120>, loops_layout_bytes<72, 120>};
     return LoopsEntry{nullptr, nullptr};
 }
 

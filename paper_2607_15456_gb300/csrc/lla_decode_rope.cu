@@ -33,6 +33,8 @@
 //     slot; the merge of split runs and W_up,t^V, mu^V_t, 1/l (shared with lla_decode.cu).
 #include <string.h>
 
+// one head page per pipeline step at every rank shape this kernel takes
+#define LLA_DECODE_STEP_BYTES (32 * 1024)
 #include "lla_decode_common.cuh"
 #include "lla_tcgen05.cuh"
 
@@ -60,17 +62,21 @@ struct RopeParams {
 template <int RK, int RV>
 struct RopeShape {
     using F = Fast<2, RK, RV>;
-    static constexpr int KSTEPS = RK / 16;          // MMAs of K = 16 per page
+    // MMAs of K = 16 per page: a rank that is not a multiple of 16 (72) takes one more step whose
+    // upper half multiplies zero columns of A (its B half lies past the K-plane, in the first
+    // 1 KB of the V-plane: rows below the token's own, so written for every valid token)
+    static constexpr int KSTEPS = (RK + 15) / 16;
+    static constexpr int KPAD = KSTEPS * 16;
     // TMEM columns: three 64-column accumulators (the MMA runs up to two pages ahead of the
     // epilogue), then two A slots of W_up,t^K (two bf16 per column) followed by the mu step's
     // (mu_hi, mu_lo, 0, ...) in 8 more columns
     static constexpr int NACC = 3;
     static constexpr int A_BASE = NACC * 64;
-    static constexpr int A_COLS = RK / 2 + 8;
+    static constexpr int A_COLS = KPAD / 2 + 8;
     static constexpr int A_STRIDE = A_COLS <= 64 ? 64 : A_COLS <= 96 ? 96 : 128;
     static constexpr int TMEM_COLS = A_BASE + 2 * A_STRIDE <= 256 ? 256 : 512;
     static constexpr uint32_t IDESC = umma_idesc_bf16(kRopeD, 64, 0, 0);
-    static_assert(RK % 32 == 0, "whole K steps, W_up,t^K rows in 16-column TMEM stores");
+    static_assert(RK % 8 == 0 && (RK % 32 == 0 || RK % 32 == 8), "W_up,t^K rows in 16- and 8-column TMEM stores");
     static_assert(A_COLS <= A_STRIDE, "A slot");
     static_assert(F::PPS == 1 && F::TT == 64, "one page per pipeline step");
     static_assert(F::S_WARPS == 4 && F::V_WARPS == 4, "four epilogue and four value warps");
@@ -173,7 +179,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
                     for (int st = 0; st < Z::KSTEPS; ++st)
                         umma_bf16_ts(d, acol + st * 8, umma_desc(bbase + st * 2048, 1024, 128),
                                      Z::IDESC, st > 0);
-                    if (has_mu) umma_bf16_ts(d, acol + RK / 2, ones_desc, Z::IDESC, true);
+                    if (has_mu) umma_bf16_ts(d, acol + Z::KPAD / 2, ones_desc, Z::IDESC, true);
                     umma_commit(&tfull[b]);
                     umma_commit(&s.empty[stage]);  // the K-plane has been read
                     if (k == R.npages - 1) umma_commit(&afree[as]);
@@ -244,7 +250,11 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
                 for (int i = 0; i < 16; ++i) part[i] = wv[16 * c + i];
                 tmem_st16u(acol + 16 * c, part);
             }
-            tmem_st8u(acol + RK / 2, mv);
+            if constexpr (RK % 32 == 8) {  // the last 8 K elements, then the zero pad of the step
+                const uint32_t tail[8] = {wv[RK / 2 - 4], wv[RK / 2 - 3], wv[RK / 2 - 2], wv[RK / 2 - 1], 0u, 0u, 0u, 0u};
+                tmem_st8u(acol + (RK / 32) * 16, tail);
+            }
+            tmem_st8u(acol + Z::KPAD / 2, mv);
             tmem_wait_st();
             tc_fence_before();
             m_sync();
@@ -488,6 +498,7 @@ RopeEntry rope_entry(int es, int d, int r_k, int r_v) {
     if (r_k == 96 && r_v == 160) return RopeEntry{launch_rope<96, 160>, rope_layout_bytes<96, 160>};
     if (r_k == 128 && r_v == 128) return RopeEntry{launch_rope<128, 128>, rope_layout_bytes<128, 128>};
     if (r_k == 192 && r_v == 320) return RopeEntry{launch_rope<192, 320>, rope_layout_bytes<192, 320>};
+    if (r_k == 72 && r_v == 120) return RopeEntry{launch_rope<72, 120>, rope_layout_bytes<72, 120>};
     return RopeEntry{nullptr, nullptr};
 }
 

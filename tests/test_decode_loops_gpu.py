@@ -69,7 +69,7 @@ def test_tiny_workload_both_passes(lla, with_mu):
     _check(sc, pass1=False, tight=True)
 
 
-@pytest.mark.parametrize("rk,rv", [(96, 160), (128, 128)])
+@pytest.mark.parametrize("rk,rv", [(96, 160), (128, 128), (72, 120)])
 def test_ragged_batch(lla, rk, rv):
     sc = Scene(lla, r_k=rk, r_v=rv, io="bf16", lens=[0, 1, 63, 64, 65, 200, 513], seed=51,
                with_mu=True)

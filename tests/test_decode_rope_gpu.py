@@ -75,7 +75,7 @@ def test_tiny_workload_two_pass_decode(lla, pairing, with_mu):
     assert lla.lla_get_device_error() == 0
 
 
-@pytest.mark.parametrize("rk,rv", [(96, 160), (128, 128), (192, 320)])
+@pytest.mark.parametrize("rk,rv", [(96, 160), (128, 128), (192, 320), (72, 120)])
 @pytest.mark.parametrize("base", [10000.0, 1e6])
 def test_ragged_batch(lla, rk, rv, base):
     """Empty (pass 1 only), one token, page-aligned, ragged tails and several pages in one
@@ -106,6 +106,15 @@ def test_long_sequences_split_across_many_ctas_rho2(lla):
     _check(sc, 1, pass1=True)
     sc.append_token()
     _check(sc, 2, pass1=False, pairing=ADJ)
+
+
+def test_long_sequences_split_across_many_ctas_rho533(lla):
+    """The Ouro-2.6B rank shape (72, 120): r_k is not a multiple of 16, so the key rebuild takes a
+    fifth K step over zero columns of A; long sequences split over CTAs, both passes, with mu."""
+    sc = Scene(lla, H=16, r_k=72, r_v=120, lens=[5000, 2100, 64, 65], io="bf16", seed=49, with_mu=True)
+    _check(sc, 3, pass1=True, tight=True)
+    sc.append_token()
+    _check(sc, 0, pass1=False, pairing=ADJ)
 
 
 def test_far_positions_keep_their_phase(lla):
