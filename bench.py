@@ -70,6 +70,7 @@ def measured_peaks():
 def decode_source_hash() -> str:
     h = hashlib.sha256()
     for rel in ("paper_2607_15456_gb300/csrc/lla_decode.cu",
+                "paper_2607_15456_gb300/csrc/lla_decode_async.cuh",
                 "paper_2607_15456_gb300/csrc/lla_decode_common.cuh",
                 "paper_2607_15456_gb300/csrc/lla_device.cuh"):
         with open(os.path.join(ROOT, rel), "rb") as f:
