@@ -514,7 +514,8 @@ def run_loops_extra(bench):
     return {"loops_decode": {
         "workload": f"{w.name} batch, all {w.T} loops of a layer per call (shared latent), "
                     f"{w.D} calls per step",
-        "kernel": "decode_loops_kernel (lla_decode_attn_loops)", "bound": "hbm",
+        "kernel": "absorb2d_kernel + attn2d_kernel<r_k, r_v, 4> + finish2d_kernel (lla_decode_attn_loops)",
+        "bound": "hbm",
         "ms_per_sweep": ms, "avg_launch_us": per_launch_s * 1e6,
         "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
         "bytes_per_launch": nbytes, "tokens_per_s_decode_only": bench.B / (ms / 1e3),
@@ -562,7 +563,7 @@ def run_decoupled_extra(bench, d_rope=64):
     return {"decoupled_decode": {
         "workload": f"{w.name} batch, decoupled rotary branch d_rope={d_rope} (base {ROPE_BASE:g}), "
                     f"{w.D}x{w.T} pass-1 calls",
-        "kernel": "absorb2d_kernel + attn2d_kernel<96,160,64> + finish2d_kernel (lla_decode_attn_decoupled)",
+        "kernel": f"decode_async_kernel<2, 96, 160, 128, {d_rope}> (lla_decode_attn_decoupled)",
         "bound": "hbm", "ms_per_sweep": ms, "avg_call_us": per_launch_s * 1e6,
         "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
         "bytes_per_call": nbytes, "tokens_per_s_decode_only": bench.B / (ms / 1e3)}}
@@ -857,7 +858,8 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
             ls_ = lms / 1e3 / w.D
             lbytes = (sum(bench.lens) * w.H * (w.r_k + w.r_v) * 2
                       + w.T * (w.H * w.d * (w.r_k + w.r_v) * 2 + 4 * bench.B * w.H * w.d * 2))
-            loops = {"kernel": "decode_loops_kernel (lla_decode_attn_loops)", "ms_per_sweep": lms,
+            loops = {"kernel": "absorb2d_kernel + attn2d_kernel<r_k, r_v, 4> + finish2d_kernel (lla_decode_attn_loops)",
+                     "ms_per_sweep": lms,
                      "avg_launch_us": ls_ * 1e6, "GB_s": lbytes / ls_ / 1e9, "hbm_frac": lbytes / ls_ / 1e9 / peak,
                      "bytes_per_launch": lbytes, "tokens_per_s_decode_only": bench.B / (lms / 1e3),
                      "note": "all T loops of a layer per call: the layer's latents cross HBM once"}

@@ -198,10 +198,13 @@ lla_status lla_decode_loops_workspace_size(const lla_geometry *g, int32_t B, siz
  * instead of T times.  The result of loop t equals lla_decode_attn at loop t.
  *   q, cur_k, cur_v, out  device [T][B][H][d] io_dtype (loop-major): loop t's query, pass-1 exact
  *                         current key and value (both NULL: pass 2), and output
- *   workspace             >= lla_decode_loops_workspace_size bytes, zero-filled before first use;
- *                         every completed call leaves it zero-filled again
+ *   workspace             >= lla_decode_loops_workspace_size bytes; needs no initialisation (the
+ *                         call writes every workspace byte it reads) and holds no state between
+ *                         calls, so calls on one stream may share it
  * Other arguments and the error behaviour are those of lla_decode_attn.  Storage LLA_BF16, d = 128,
- * T = 4 and (r_k, r_v) one of (96, 160), (128, 128), (72, 120); LLA_ERR_UNSUPPORTED otherwise.
+ * 1 <= T <= 4 and (r_k, r_v) one of (96, 160), (128, 128), (72, 120), (192, 320);
+ * LLA_ERR_UNSUPPORTED otherwise.  Three kernels on the stream (q~ absorption; the page stream on
+ * the tensor cores, q~ and p as sums of three bf16 parts; the merge and output projection).
  */
 lla_status lla_decode_attn_loops(const lla_geometry *g, const lla_codec *codec,
                                  const lla_cache *cache, const int32_t *context_lens, int32_t B,

@@ -283,7 +283,7 @@ lla_status lla_decode_loops_workspace_size(const lla_geometry *g, int32_t B, siz
     if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
     const int grid = num_sms();
     if (grid <= 0) return LLA_ERR_CUDA;
-    *bytes = decode_loops_workspace_bytes(g->r_v, B, g->H, g->T, grid);
+    *bytes = decode_loops_workspace_bytes(g->r_k, g->r_v, B, g->H, grid);
     return LLA_OK;
 }
 

@@ -1,34 +1,40 @@
-// lla_decode_2d.cu -- decode over the LLA-2D cache (Sec. 3, "The LLA-2D variant (loop x head)";
-// App. J "Absorbed attention" and "Per-head LLA versus LLA-2D at inference").
-//
-// One latent pair per (token, layer) serves every head: head h at loop t rebuilds its key and
-// value as c W_up,t,h^T + mu_{t,h}.  Absorbed head by head (App. J), the H queries of a sequence
-// read the same latent, so each page of 64 tokens is a small dense contraction:
-//   q~_h = W_up,t,h^K^T q_h,  beta_h = q_h . mu^K_{t,h}                     (absorb kernel)
-//   S^T [64 x 32]   = C_k [64 x r_k] [Q~_hi; Q~_lo]^T     s_hi = scale (q~_h . c_k,i + beta_h)
-//   O^T [r_v x 16] += C_v^T [r_v x 64] P^T                online softmax over tokens per head
-//   o_h = (W_up,t,h^V o~_h + l_h mu^V_{t,h} + p_cur v_cur,h) / (l_h + p_cur)  (finish kernel)
+// lla_decode_2d.cu -- decode over a latent page that several queries share, on the tensor cores:
+//   * the LLA-2D cache (Sec. 3, "The LLA-2D variant (loop x head)"; App. J "Absorbed attention"
+//     and "Per-head LLA versus LLA-2D at inference"): one latent pair per (token, layer) serves
+//     every head, so the H queries of a sequence read the same page;
+//   * the T loops of a per-head cache (Sec. 3, Eq. encode: one stacked code per (token, layer,
+//     head) serves every loop), so the T loop queries of a (sequence, head) read the same page.
+// A unit is what owns a page stream (a sequence for LLA-2D, a (sequence, head) pair for the
+// loops) and a query is one of its NQ readers (a head, a loop).  Query n of a unit rebuilds its
+// key and value as c W_up,n^T + mu_n.  Absorbed query by query (App. J), each page of 64 tokens
+// is a small dense contraction:
+//   q~_n = W_up,n^K^T q_n,  beta_n = q_n . mu^K_n                            (absorb kernel)
+//   S^T [64 x 2NQ]  = C_k [64 x r_k] [Q~_hi; Q~_lo]^T     s_n,i = scale (q~_n . c_k,i + beta_n)
+//   O^T [r_v x 16] += C_v^T [r_v x 64] P^T                online softmax over tokens per query
+//   o_n = (W_up,n^V o~_n + l_n mu^V_n + p_cur v_cur,n) / (l_n + p_cur)      (finish kernel)
 // Three launches on the caller's stream, chained by programmatic dependent launch:
-//   absorb2d_kernel   q~ (fp32, scaled into the exp2 domain) and beta of every (sequence, head),
-//                     the page prefix sums of the batch and the length checks
-//   attn2d_kernel     one CTA per SM.  The batch's pages, in sequence order, are split evenly
-//                     over the CTAs; a CTA takes its pages as runs (its part of one sequence)
-//                     and writes per run the partial (maximum, sum, O^T) of every head.
+//   absorb2d_kernel   q~ (fp32, scaled into the exp2 domain) and beta of every (unit, query),
+//                     the page prefix sums of the units and the length checks
+//   attn2d_kernel     one CTA per SM.  The units' pages, in unit order, are split evenly over
+//                     the CTAs; a CTA takes its pages as runs (its part of one unit) and writes
+//                     per run the partial (maximum, sum, O^T) of every query.
 //                       warp 0     producer: the K-plane of a page by one bulk copy, its V-plane
 //                                  by TMA boxes of 64 columns with 128-byte swizzle
-//                       warp 1     MMA issuer and TMEM owner: S^T (M = 64 tokens, N = 32: q~ as
-//                                  a bf16 high part and a bf16 remainder per head, so that the
-//                                  scores see q~ to about 16 significant bits; K = r_k) and O^T
-//                                  (M = 128 latent rows per chunk, N = 16 heads,
-//                                  K = 64 tokens; the swizzled V-plane is an MN-major A operand);
-//                                  the O^T product of a page is issued after the next page's
-//                                  S^T, so the softmax of one page overlaps the next page's scores
+//                       warp 1     MMA issuer and TMEM owner: S^T (M = 64 tokens, N = 2 NQ: q~
+//                                  as a bf16 high part and a bf16 remainder per query, so that
+//                                  the scores see q~ to about 16 significant bits; K = r_k, a
+//                                  rank that is not a multiple of 16 padded with zero columns)
+//                                  and O^T (M = 128 latent rows per chunk, N = 16 queries padded
+//                                  with zero rows of P^T, K = 64 tokens; the swizzled V-plane is
+//                                  an MN-major A operand); the O^T product of a page is issued
+//                                  after the next page's S^T, so the softmax of one page overlaps
+//                                  the next page's scores
 //                       warps 2-5  per page: the scores of 16 tokens per warp, the maxima over
-//                                  the page per head, P^T as a bf16 operand, the lazy O^T rescale;
-//                                  per run: the partial out to the workspace
-//   finish2d_kernel   per (head, up to 8 sequences): merges the runs of each sequence, adds the
-//                     pass-1 current token, and applies W_up,t,h^V once for those sequences
-// Storage bf16, d = 128, H <= 16; accumulators fp32 in TMEM.
+//                                  the page per query, P^T as a bf16 operand, the lazy O^T
+//                                  rescale; per run: the partial out to the workspace
+//   finish2d_kernel   per (query slice, up to 8 units): merges the runs of each unit, adds the
+//                     pass-1 current token, and applies W_up,n^V once for those units
+// Storage bf16, d = 128; accumulators fp32 in TMEM.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -45,30 +51,36 @@ namespace {
 
 constexpr int kPT = 64;          // tokens per page
 constexpr int kD = 128;          // head width
-constexpr int kNQ = 16;          // the heads of a sequence, padded
-constexpr int kNS = 2 * kNQ;     // score MMA N: q~ high parts, then remainders
+constexpr int kNQ = 16;          // O^T columns: the queries of a unit, padded
 constexpr int kT2 = 192;         // threads of the attention kernel
 constexpr int kSm0 = 64;         // first softmax thread
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kRescaleLog2 = 8.f;  // rescale O^T only when a head's maximum grows by more
+constexpr float kRescaleLog2 = 8.f;  // rescale O^T only when a query's maximum grows by more
 constexpr int kSmemCap = 227 * 1024;
-constexpr int kFinishSeqs = 8;   // most sequences per finish CTA
-constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one sequence fit one finish CTA)
+constexpr int kFinishSeqs = 8;   // most units per finish CTA
+constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one unit fit one finish CTA)
 
-// Shared-memory plan of the attention kernel for ranks (RK, RV).  Offsets from a 1024-byte
-// aligned base (128-byte swizzle atoms of the V stages).
-template <int RK, int RV>
+// Shared-memory plan of the attention kernel for ranks (RK, RV) and NQ query slots per unit
+// (16: the heads of an LLA-2D sequence; 4: the loops of a per-head (sequence, head)).  Offsets
+// from a 1024-byte aligned base (128-byte swizzle atoms of the V stages).
+template <int RK, int RV, int NQ>
 struct Z2 {
-    static constexpr int RKX = RK;                      // score contraction
-    static constexpr int NQM = kNQ;                     // queries of a sequence (its heads, padded)
+    static constexpr int RKX = (RK + 15) / 16 * 16;     // score contraction, zero-padded
+    // q~ and p as sums of bf16 parts, each the rounding of what the earlier parts leave: with
+    // 16 query slots q~ in two parts (about 16 significant bits) and p in one; with 4 slots the
+    // MMA's padding columns carry three parts of each (24 bits, the precision of fp32)
+    static constexpr int QS = NQ == 4 ? 3 : 2;
+    static constexpr int PSPL = NQ == 4 ? 3 : 1;
+    static constexpr int NS = (QS * NQ + 7) / 8 * 8;    // score MMA N: the q~ parts, padded
+    static constexpr int NQM = NQ;                      // queries of a unit in the workspace
     static constexpr int NCH = (RV + 127) / 128;        // 128-row chunks of O^T
     static constexpr int NBOX = (RV + 63) / 64;         // TMA boxes a V-plane loads
     static constexpr int BOX = kPT * 128;               // one box: 64 rows x 128 bytes
-    static constexpr int KPLANE = kPT * RK * 2;
-    static constexpr int KPAGE = kPT * RKX * 2;         // K-plane
+    static constexpr int KPLANE = kPT * RK * 2;         // bytes of a K-plane copy
+    static constexpr int KPAGE = kPT * RKX * 2;         // K stage: the copy, then zero granules
     static constexpr int VPAGE = NCH * 2 * BOX;         // two boxes per chunk, loaded or zero
     static constexpr int VBYTES = NBOX * BOX;
-    static constexpr int QB = kNS * RKX * 2;            // [Q~_hi; Q~_lo] operand
+    static constexpr int QB = NS * RKX * 2;             // [Q~_hi; Q~_lo] operand
     static constexpr int PBUF = kPT * kNQ * 2;          // P^T operand (one of two)
     static constexpr int RED = 1024;                    // maxima, sums, beta
     static constexpr int NBAR = 32;
@@ -82,14 +94,16 @@ struct Z2 {
     static constexpr int oRed = oP + 2 * PBUF;
     static constexpr int oBar = oRed + RED;
     static constexpr int SMEM = 1024 + oBar + NBAR * 8;
-    // TMEM columns: S^T double buffer [0, 64), O^T chunks [64, 64 + 16 NCH)
-    static constexpr uint32_t TM_S = 0, TM_O = 2 * kNS, TM_COLS = 128;
-    static constexpr uint32_t IDESC_S = umma_idesc_bf16(64, kNS, 0, 0);
+    // TMEM columns: S^T double buffer [0, 2 NS), O^T chunks [2 NS, 2 NS + 16 NCH)
+    static constexpr uint32_t TM_S = 0, TM_O = 2 * NS, TM_COLS = 128;
+    static constexpr uint32_t IDESC_S = umma_idesc_bf16(64, NS, 0, 0);
     static constexpr uint32_t IDESC_O = umma_idesc_bf16(128, kNQ, 1, 0);
     // a run partial: O^T of each query ([NQM][RV]), then 16 maxima and 16 sums
     static constexpr int PSTRIDE = NQM * RV + 2 * kNQ;
     static constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
-    static_assert(RK % 16 == 0 && RV % 32 == 0 && NCH <= 4, "ranks");
+    static_assert(NQ == 4 || NQ == 16, "query slots");
+    static_assert(PSPL * NQ <= kNQ, "p parts in the O^T columns");
+    static_assert(RK % 8 == 0 && RV % 8 == 0 && NCH <= 4, "ranks in 16-byte granules");
     static_assert(ST >= 2, "pipeline depth");
     static_assert(SMEM <= kSmemCap, "shared memory");
     static_assert(TM_O + NCH * kNQ <= TM_COLS, "TMEM columns");
@@ -102,22 +116,31 @@ enum {
     bOfree = 25, bQready = 26, bQfree = 27, bAbort = 28, bTslot = 29
 };
 
+// Unit u of the batch: sequence u / hu, head u % hu of a per-head cache (hu = H for the loops,
+// 1 for LLA-2D, whose one page per block serves every head).  Query n of unit u:
+//   LLA-2D  head n of sequence u at loop `loop`: weights [T][H][d][r] at (loop, n), io row (u H + n)
+//   loops   loop n of (sequence b, head h):      weights [H][T][d][r] at (h, n),
+//                                                io row ((n B + b) H + h)
+// (mu alike: [T*H*d] rows (t, h, e) for LLA-2D, [H][T*d] for the per-head codec).
 struct A2Params {
     int T, H, loop, io_bf16, pass1, B, max_ctx, max_blocks;
+    int loops;           // 0: LLA-2D, 1: the loops of a per-head cache
+    int hu;              // units per sequence
     float scale_log2;
-    const void *w_up_k;  // [T][H][d][r_k]
-    const float *mu_k;   // [T*H*d] or NULL
-    const void *q;       // [B][H][d]
+    const void *w_up_k;  // LLA-2D [T][H][d][r_k], per-head [H][T][d][r_k]
+    const float *mu_k;   // LLA-2D [T*H*d], per-head [H][T*d], or NULL
+    const void *q;       // io rows of d
     const int32_t *context_lens;
-    float *qt;           // [B][16][RK]: q~ * scale * log2 e
-    float *beta;         // [B][16]: beta * scale * log2 e
-    int *pstart;         // [B + 1]: first global page of each sequence
+    float *qt;           // [units][NQM][RKX]: q~ * scale * log2 e, zero past r_k
+    float *beta;         // [units][NQM]: beta * scale * log2 e
+    int *pstart;         // [units + 1]: first global page of each unit
     unsigned *err;
 };
 
 struct T2Params {
-    int nq;   // queries of a sequence: H
-    int B;
+    int nq;   // queries of a unit
+    int U;    // units
+    int hu;   // units per sequence
     const char *pool;
     int64_t num_blocks, page_bytes;
     const int32_t *block_table;
@@ -126,16 +149,17 @@ struct T2Params {
     const float *qt;
     const float *beta;
     const int *pstart;
-    float *part;  // [B + grid][PSTRIDE]: run (sequence b, CTA c) at slot b + c
+    float *part;  // [U + grid][PSTRIDE]: run (unit u, CTA c) at slot u + c
     unsigned *err;
 };
 
 struct F2Params {
     int T, H, loop, io_bf16, B, grid;
-    int spb;  // sequences per CTA (1 .. 8)
+    int loops, hu, U;
+    int spb;  // units per CTA (1 .. 8)
     float scale_log2;
-    const void *w_up_v;  // [T][H][d][r_v] bf16
-    const float *mu_v;   // [T*H*d] or NULL
+    const void *w_up_v;  // LLA-2D [T][H][d][r_v], per-head [H][T][d][r_v], bf16
+    const float *mu_v;   // LLA-2D [T*H*d], per-head [H][T*d], or NULL
     const void *q, *cur_k, *cur_v;
     void *out;
     const int *pstart;
@@ -155,16 +179,17 @@ __host__ __device__ __forceinline__ int cta_of(int g, int np, int grid) {
 
 // ------------------------------------------------------------------------- absorb kernel
 
-// One CTA: the page prefix sums of the batch's sequences with the length checks; an invalid
-// length counts as an empty sequence.
+// One CTA: the page prefix sums of the units with the length checks (once per sequence); an
+// invalid length counts as an empty sequence.
 __device__ void page_prefix(const A2Params &p) {
     __shared__ int wsum[8];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int U = p.B;
-    const int per = (U + 255) / 256;  // sequences of this thread: [tid per, (tid + 1) per)
+    const int U = p.B * p.hu;
+    const int per = (U + 255) / 256;  // units of this thread: [tid per, (tid + 1) per)
     const int limit = min(p.max_ctx, p.max_blocks * kPT);
     auto pages = [&](int u, bool flag) {
-        const int L = p.context_lens[u];
+        const int L = p.context_lens[u / p.hu];
+        flag = flag && u % p.hu == 0;
         if (L < 0 || L > limit) {
             if (flag) atomicOr(p.err, LLA_DEVERR_CONTEXT);
             return 0;
@@ -192,40 +217,43 @@ __device__ void page_prefix(const A2Params &p) {
     if (tid == blockDim.x - 1) p.pstart[U] = pre + x;
 }
 
-// Grid (H, RK / 32, ceil(B / 16)), 256 threads = 32 columns x 8 slices of 16 rows of the head:
-// q~ of 32 columns of head h for 16 sequences, every weight load of a thread in flight at once;
-// beta of head h by the CTAs of the first column chunk.  The weight slice of (loop t, head h) is
-// (t, h) of [T][H].
-template <int RK>
+// Grid (weight slices, RKX / 32, ceil(B / 16)), 256 threads = 32 columns x 8 slices of 16 rows:
+// q~ of 32 columns of one weight slice for 16 sequences, every weight load of a thread in flight
+// at once; beta by the CTAs of the first column chunk.  Slice w is (loop, head w) for LLA-2D and
+// (loop w / H, head w % H) for the loops (th: its row block of d in W_up and mu); columns
+// r_k .. RKX - 1 of q~ are written as zeros.
+template <int RK, int NQ>
 __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
-    static_assert(RK % 32 == 0, "column chunks");
+    constexpr int RKX = (RK + 15) / 16 * 16;
     __shared__ float qs[16][kD];
     __shared__ float red[8][16][33];
-    const int h = blockIdx.x, j0 = blockIdx.y * 32, b0 = blockIdx.z * 16, tid = threadIdx.x;
+    const int w = blockIdx.x, j0 = blockIdx.y * 32, b0 = blockIdx.z * 16, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(16, p.B - b0);
-    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
-    // the output row of (sequence b, head h): query h of sequence b
-    auto row = [&](int b) { return static_cast<int64_t>(b) * kNQ + h; };
+    const int t = p.loops ? w / p.H : p.loop, h = p.loops ? w - t * p.H : w;
+    const int64_t th = p.loops ? static_cast<int64_t>(h) * p.T + t : static_cast<int64_t>(t) * p.H + h;
+    const int n = p.loops ? t : h;  // the query of (sequence b, slice w) within its unit
+    auto unit = [&](int b) { return p.loops ? b * p.H + h : b; };
+    auto iorow = [&](int b) { return ((p.loops ? static_cast<int64_t>(t) * p.B : 0) + b) * p.H + h; };
+    const int col = j0 + lane;
     pdl_wait();  // inputs may come from the previous kernel; the workspace is free after it
     // this thread's 16 weights (column j0 + lane, rows 16 warp .. 16 warp + 15), in flight while
     // the queries load
-    const uint16_t *W = static_cast<const uint16_t *>(p.w_up_k) + th * kD * RK + j0 + lane;
-    float w[16];
+    const uint16_t *W = static_cast<const uint16_t *>(p.w_up_k) + th * kD * RK + col;
+    float wv[16];
 #pragma unroll
-    for (int u = 0; u < 16; ++u) w[u] = bf_to_f(W[(warp * 16 + u) * RK]);
+    for (int u = 0; u < 16; ++u) wv[u] = col < RK ? bf_to_f(W[(warp * 16 + u) * RK]) : 0.f;
     if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) page_prefix(p);
     for (int i = tid; i < 16 * kD; i += 256) {
         const int bi = i >> 7, e = i & (kD - 1);
-        qs[bi][e] = bi < nb ? load_elem(p.q, (static_cast<int64_t>(b0 + bi) * p.H + h) * kD + e, p.io_bf16)
-                            : 0.f;
+        qs[bi][e] = bi < nb ? load_elem(p.q, iorow(b0 + bi) * kD + e, p.io_bf16) : 0.f;
     }
     __syncthreads();
 #pragma unroll
     for (int bi = 0; bi < 16; ++bi) {
         float a = 0.f;
 #pragma unroll
-        for (int u = 0; u < 16; ++u) a = fmaf(w[u], qs[bi][warp * 16 + u], a);
+        for (int u = 0; u < 16; ++u) a = fmaf(wv[u], qs[bi][warp * 16 + u], a);
         red[warp][bi][lane] = a;
     }
     __syncthreads();
@@ -234,16 +262,17 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
         float a = 0.f;
 #pragma unroll
         for (int sl = 0; sl < 8; ++sl) a += red[sl][bi][c];
-        if (bi < nb) p.qt[row(b0 + bi) * RK + j0 + c] = a * p.scale_log2;
+        if (bi < nb && j0 + c < RKX)
+            p.qt[(static_cast<int64_t>(unit(b0 + bi)) * NQ + n) * RKX + j0 + c] = j0 + c < RK ? a * p.scale_log2 : 0.f;
     }
     if (blockIdx.y == 0) {
-        // beta_h = q_h . mu^K_{t,h}: warp w takes sequences w and w + 8
+        // beta_n = q_n . mu^K_n: warp w takes sequences w and w + 8
         for (int bi = warp; bi < nb; bi += 8) {
             float s = 0.f;
             if (p.mu_k)
                 for (int e = lane; e < kD; e += 32) s = fmaf(qs[bi][e], p.mu_k[th * kD + e], s);
             s = warp_sum(s);
-            if (lane == 0) p.beta[row(b0 + bi)] = s * p.scale_log2;
+            if (lane == 0) p.beta[static_cast<int64_t>(unit(b0 + bi)) * NQ + n] = s * p.scale_log2;
         }
     }
     __syncthreads();
@@ -252,9 +281,9 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
 
 // ------------------------------------------------------------------------- attention kernel
 
-// First sequence with pages at or after global page g0: the last b with pstart[b] <= g0.
-__device__ __forceinline__ int first_seq(const int *pstart, int B, int g0) {
-    int lo = 0, hi = B - 1;
+// First unit with pages at or after global page g0: the last u with pstart[u] <= g0.
+__device__ __forceinline__ int first_unit(const int *pstart, int U, int g0) {
+    int lo = 0, hi = U - 1;
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
         if (pstart[mid] <= g0) lo = mid;
@@ -263,10 +292,28 @@ __device__ __forceinline__ int first_seq(const int *pstart, int B, int g0) {
     return lo;
 }
 
-template <int RK, int RV>
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[N]) {
+    static_assert(N == 16 || N == 32, "score columns");
+    if constexpr (N == 16) tmem_ld16(taddr, v);
+    else tmem_ld32(taddr, v);
+}
+
+// The K bf16 parts of v: part 0 = bf16(v), part k = bf16 of what parts 0 .. k-1 leave (each
+// difference is exact in fp32).
+template <int K>
+__device__ __forceinline__ void bf16_parts(float v, float (&part)[K]) {
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+        part[k] = __bfloat162float(__float2bfloat16_rn(v));
+        v -= part[k];
+    }
+}
+
+template <int RK, int RV, int NQ>
 __global__ void __launch_bounds__(kT2, 1)
     attn2d_kernel(const __grid_constant__ CUtensorMap tv, const T2Params p) {
-    using Z = Z2<RK, RV>;
+    using Z = Z2<RK, RV, NQ>;
     extern __shared__ __align__(1024) char sm_raw[];
     char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + Z::oBar);
@@ -298,23 +345,37 @@ __global__ void __launch_bounds__(kT2, 1)
         fence_mbar_init();
     }
     if (warp == 1) tmem_alloc(tslot, Z::TM_COLS);
-    // V boxes that no load writes (the second box of a last chunk past r_v) stay zero
+    // operand bytes that no copy writes stay zero: the V boxes past r_v of a last chunk, the K
+    // granules past r_k (against zero q~ columns), and the P^T rows of absent queries
     if constexpr (Z::NCH * 2 > Z::NBOX) {
         for (int s = 0; s < Z::ST; ++s)
             for (int a = Z::NBOX; a < Z::NCH * 2; ++a)
                 for (int i = tid; i < Z::BOX / 16; i += kT2)
                     reinterpret_cast<uint4 *>(sm + Z::oV + s * Z::VPAGE + a * Z::BOX)[i] = make_uint4(0, 0, 0, 0);
-        fence_proxy_async_smem();
     }
+    if constexpr (Z::KPAGE > Z::KPLANE) {
+        for (int s = 0; s < Z::ST; ++s)
+            for (int i = tid; i < (Z::KPAGE - Z::KPLANE) / 16; i += kT2)
+                reinterpret_cast<uint4 *>(sm + Z::oK + s * Z::KPAGE + Z::KPLANE)[i] = make_uint4(0, 0, 0, 0);
+    }
+    if constexpr (Z::PSPL * NQ < kNQ) {
+        for (int i = tid; i < 2 * Z::PBUF / 16; i += kT2)
+            reinterpret_cast<uint4 *>(sm + Z::oP)[i] = make_uint4(0, 0, 0, 0);
+    }
+    if constexpr (Z::QS * NQ < Z::NS) {  // the padding rows of the q~ operand
+        for (int i = tid; i < Z::QB / 16; i += kT2)
+            reinterpret_cast<uint4 *>(sm + Z::oQ)[i] = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
     pdl_wait();  // q~, beta and the page prefix sums come from the absorb kernel
 
-    const int NP = p.pstart[p.B];
+    const int NP = p.pstart[p.U];
     const int g0 = page_lo(c, NP, G), g1 = page_lo(c + 1, NP, G);
-    const int bfirst = g0 < g1 ? first_seq(p.pstart, p.B, g0) : p.B;
+    const int ufirst = g0 < g1 ? first_unit(p.pstart, p.U, g0) : p.U;
 
     if (warp == 0) {
         // ------------------------------------------------------------------------- producer
@@ -325,10 +386,11 @@ __global__ void __launch_bounds__(kT2, 1)
             const uint64_t pol = policy_evict_first();
             int itk = 0, itv = 0;
             bool stop = false;
-            for (int b = bfirst; b < p.B && !stop; ++b) {
-                const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+            for (int u = ufirst; u < p.U && !stop; ++u) {
+                const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
                 if (s0 >= g1) break;
                 const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
+                const int b = u / p.hu, hh = u - b * p.hu;
                 const int32_t *bt = p.block_table + static_cast<int64_t>(b) * p.max_blocks;
                 for (int pg = pa; pg < pe; ++pg) {
                     const int it = itk;
@@ -339,12 +401,12 @@ __global__ void __launch_bounds__(kT2, 1)
                         atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
                         blk = 0;
                     }
-                    const int64_t page = blk;
+                    const int64_t page = static_cast<int64_t>(blk) * p.hu + hh;
                     if (!mbar_wait(&bar[bKempty + st], ph ^ 1u, abort_flag, p.err) || *abort_flag) {
                         stop = true;
                         break;
                     }
-                    mbar_arrive_expect_tx(&bar[bKfull + st], Z::KPAGE);
+                    mbar_arrive_expect_tx(&bar[bKfull + st], Z::KPLANE);
                     char *ks = sm + Z::oK + st * Z::KPAGE;
                     bulk_g2s(ks, p.pool + page * p.page_bytes, Z::KPLANE, &bar[bKfull + st], pol);
                     ++itk;
@@ -372,7 +434,7 @@ __global__ void __launch_bounds__(kT2, 1)
         // ------------------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const uint32_t base = smem_addr(sm);
-            const uint64_t dq = umma_desc(base + Z::oQ, kNS * 16, 128);
+            const uint64_t dq = umma_desc(base + Z::oQ, Z::NS * 16, 128);
             const uint64_t dk0 = umma_desc(base + Z::oK, kPT * 16, 128);
             const uint64_t dp0 = umma_desc(base + Z::oP, kNQ * 16, 128);
             const uint64_t dv0 = umma_desc_sw128_mn(base + Z::oV, Z::BOX);
@@ -395,8 +457,8 @@ __global__ void __launch_bounds__(kT2, 1)
                 umma_commit(&bar[bVempty + st]);
                 umma_commit(&bar[bPfree + s]);  // also: O^T holds pages up to j
             };
-            for (int b = bfirst; b < p.B; ++b) {
-                const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+            for (int u = ufirst; u < p.U; ++u) {
+                const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
                 if (s0 >= g1) break;
                 const int n = min(g1, s1) - max(g0, s0);
                 if (n <= 0) continue;
@@ -410,8 +472,8 @@ __global__ void __launch_bounds__(kT2, 1)
                     const uint64_t dk = dk0 + static_cast<uint64_t>((st * Z::KPAGE) >> 4);
 #pragma unroll
                     for (int ks = 0; ks < Z::RKX / 16; ++ks)
-                        umma_bf16(tmem + Z::TM_S + s * kNS, dk + ks * ((2 * kPT * 16) >> 4),
-                                  dq + ks * ((2 * kNS * 16) >> 4), Z::IDESC_S, ks > 0);
+                        umma_bf16(tmem + Z::TM_S + s * Z::NS, dk + ks * ((2 * kPT * 16) >> 4),
+                                  dq + ks * ((2 * Z::NS * 16) >> 4), Z::IDESC_S, ks > 0);
                     umma_commit(&bar[bSfull + s]);
                     umma_commit(&bar[bKempty + st]);
                     if (k == n - 1) umma_commit(&bar[bQfree]);
@@ -436,43 +498,50 @@ __global__ void __launch_bounds__(kT2, 1)
         const int st_tid = tid - kSm0;
         const int tok = 16 * q4 + lane;  // the token of this lane in the M = 64 layout (lane < 16)
         int it = 0, r = 0;
-        for (int b = bfirst; b < p.B; ++b) {
-            const int s0 = p.pstart[b], s1 = p.pstart[b + 1];
+        for (int u = ufirst; u < p.U; ++u) {
+            const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
             if (s0 >= g1) break;
             const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
             if (pe <= pa) continue;
-            const int L = p.context_lens[b];
-            // q~ of the sequence as a K-major operand of 32 rows: row n = bf16(q~_n), row 16 + n =
-            // bf16(q~_n - row n), granule g of row n at g*512 + n*16; and beta
+            const int L = p.context_lens[u / p.hu];
+            // q~ of the unit as a K-major operand of NS rows: row k NQ + n = bf16 part k of q~_n,
+            // granule g of row n at g*(NS * 16) + n*16 (rows past QS NQ stay zero); and beta
             if (r > 0) mbar_wait(&bar[bQfree], (r - 1) & 1, abort_flag, p.err);
             {
-                const float4 *src = reinterpret_cast<const float4 *>(p.qt + static_cast<int64_t>(b) * Z::NQM * Z::RKX);
-                for (int i = st_tid; i < kNQ * (Z::RKX / 8); i += 128) {
+                const float4 *src = reinterpret_cast<const float4 *>(p.qt + static_cast<int64_t>(u) * Z::NQM * Z::RKX);
+                for (int i = st_tid; i < NQ * (Z::RKX / 8); i += 128) {
                     const int n = i / (Z::RKX / 8), g = i - n * (Z::RKX / 8);
-                    uint4 hi = make_uint4(0, 0, 0, 0), lo = hi;
+                    float pt[Z::QS][8];
+#pragma unroll
+                    for (int k = 0; k < Z::QS; ++k)
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) pt[k][e] = 0.f;
                     if (n < p.nq) {
                         const float4 a = src[2 * i], c4 = src[2 * i + 1];
                         const float v[8] = {a.x, a.y, a.z, a.w, c4.x, c4.y, c4.z, c4.w};
-                        float r8[8];
 #pragma unroll
-                        for (int u = 0; u < 8; ++u) r8[u] = v[u] - __bfloat162float(__float2bfloat16_rn(v[u]));
-                        hi = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                                        pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-                        lo = make_uint4(pack_bf16x2(r8[0], r8[1]), pack_bf16x2(r8[2], r8[3]),
-                                        pack_bf16x2(r8[4], r8[5]), pack_bf16x2(r8[6], r8[7]));
+                        for (int e = 0; e < 8; ++e) {
+                            float pe[Z::QS];
+                            bf16_parts(v[e], pe);
+#pragma unroll
+                            for (int k = 0; k < Z::QS; ++k) pt[k][e] = pe[k];
+                        }
                     }
-                    char *dq = sm + Z::oQ + g * (kNS * 16);
-                    *reinterpret_cast<uint4 *>(dq + n * 16) = hi;
-                    *reinterpret_cast<uint4 *>(dq + (kNQ + n) * 16) = lo;
+                    char *dq = sm + Z::oQ + g * (Z::NS * 16);
+#pragma unroll
+                    for (int k = 0; k < Z::QS; ++k)
+                        *reinterpret_cast<uint4 *>(dq + (k * NQ + n) * 16) =
+                            make_uint4(pack_bf16x2(pt[k][0], pt[k][1]), pack_bf16x2(pt[k][2], pt[k][3]),
+                                       pack_bf16x2(pt[k][4], pt[k][5]), pack_bf16x2(pt[k][6], pt[k][7]));
                 }
-                if (st_tid < kNQ) betas[st_tid] = st_tid < p.nq ? p.beta[static_cast<int64_t>(b) * Z::NQM + st_tid] : 0.f;
+                if (st_tid < NQ) betas[st_tid] = st_tid < p.nq ? p.beta[static_cast<int64_t>(u) * Z::NQM + st_tid] : 0.f;
             }
             fence_proxy_async_smem();
             mbar_arrive(&bar[bQready]);
             named_bar_sync(1, 128);  // beta is visible
-            float m[kNQ], acc[kNQ];
+            float m[NQ], acc[NQ];
 #pragma unroll
-            for (int n = 0; n < kNQ; ++n) {
+            for (int n = 0; n < NQ; ++n) {
                 m[n] = -INFINITY;
                 acc[n] = 0.f;
             }
@@ -482,32 +551,37 @@ __global__ void __launch_bounds__(kT2, 1)
                 const int tok0 = (pa + k) * kPT;
                 mbar_wait(&bar[bSfull + s], (it >> 1) & 1, abort_flag, p.err);
                 tc_fence_after();
-                float x2[kNS], x[kNQ];
-                tmem_ld32(tl + Z::TM_S + s * kNS, x2);
+                float x2[Z::NS], x[NQ];
+                tmem_ld_cols(tl + Z::TM_S + s * Z::NS, x2);
                 tc_fence_before();
                 mbar_arrive(&bar[bSfree + s]);
                 const bool valid = lane < 16 && tok0 + tok < L;
 #pragma unroll
-                for (int n = 0; n < kNQ; ++n) x[n] = valid ? (x2[n] + x2[kNQ + n]) + betas[n] : -INFINITY;
-                // per-head maxima over the page: 16 tokens per warp, then the 4 warps
-                float mx[kNQ];
+                for (int n = 0; n < NQ; ++n) {
+                    float sn = x2[n];
 #pragma unroll
-                for (int n = 0; n < kNQ; ++n) mx[n] = x[n];
+                    for (int k = 1; k < Z::QS; ++k) sn += x2[k * NQ + n];
+                    x[n] = valid ? sn + betas[n] : -INFINITY;
+                }
+                // per-query maxima over the page: 16 tokens per warp, then the 4 warps
+                float mx[NQ];
+#pragma unroll
+                for (int n = 0; n < NQ; ++n) mx[n] = x[n];
 #pragma unroll
                 for (int o = 8; o >= 1; o >>= 1)
 #pragma unroll
-                    for (int n = 0; n < kNQ; ++n) mx[n] = fmaxf(mx[n], __shfl_xor_sync(0xffffffffu, mx[n], o));
+                    for (int n = 0; n < NQ; ++n) mx[n] = fmaxf(mx[n], __shfl_xor_sync(0xffffffffu, mx[n], o));
                 float *rp = red + s * 64;
                 if (lane == 0) {
 #pragma unroll
-                    for (int n = 0; n < kNQ; n += 4)
+                    for (int n = 0; n < NQ; n += 4)
                         *reinterpret_cast<float4 *>(rp + q4 * 16 + n) = make_float4(mx[n], mx[n + 1], mx[n + 2], mx[n + 3]);
                 }
                 named_bar_sync(1, 128);
                 bool any = false;
-                float f[kNQ];
+                float f[NQ];
 #pragma unroll
-                for (int n = 0; n < kNQ; n += 4) {
+                for (int n = 0; n < NQ; n += 4) {
                     float4 a = *reinterpret_cast<const float4 *>(rp + n);
 #pragma unroll
                     for (int w = 1; w < 4; ++w) {
@@ -516,13 +590,13 @@ __global__ void __launch_bounds__(kT2, 1)
                     }
                     const float pm[4] = {a.x, a.y, a.z, a.w};
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const float mn = fmaxf(m[n + u], pm[u]);
-                        const bool need = mn > m[n + u] + kRescaleLog2;  // also the first page
-                        f[n + u] = need ? ex2_approx(m[n + u] - mn) : 1.f;
+                    for (int e = 0; e < 4; ++e) {
+                        const float mn = fmaxf(m[n + e], pm[e]);
+                        const bool need = mn > m[n + e] + kRescaleLog2;  // also the first page
+                        f[n + e] = need ? ex2_approx(m[n + e] - mn) : 1.f;
                         if (need) {
-                            acc[n + u] *= f[n + u];
-                            m[n + u] = mn;
+                            acc[n + e] *= f[n + e];
+                            m[n + e] = mn;
                             any = true;
                         }
                     }
@@ -531,7 +605,7 @@ __global__ void __launch_bounds__(kT2, 1)
                     // O^T holds pages up to it - 1 of this run (the product of page it - 1 has
                     // released its P buffer; the one of page it - 2 had released the other before
                     // this warp wrote page it - 1, so the parity test cannot pass a phase early):
-                    // scale head n's column by f[n]
+                    // scale query n's columns by f[n]
                     mbar_wait(&bar[bPfree + ((it - 1) & 1)], ((it - 1) >> 1) & 1, abort_flag, p.err);
                     tc_fence_after();
 #pragma unroll
@@ -539,23 +613,32 @@ __global__ void __launch_bounds__(kT2, 1)
                         float o[kNQ];
                         tmem_ld16(tl + Z::TM_O + ch * kNQ, o);
 #pragma unroll
-                        for (int n = 0; n < kNQ; ++n) o[n] *= f[n];
+                        for (int k = 0; k < Z::PSPL; ++k)
+#pragma unroll
+                            for (int n = 0; n < NQ; ++n) o[k * NQ + n] *= f[n];
                         tmem_st16(tl + Z::TM_O + ch * kNQ, o);
                     }
                 }
-                float pv[kNQ];
+                float pv[NQ];
 #pragma unroll
-                for (int n = 0; n < kNQ; ++n) {
+                for (int n = 0; n < NQ; ++n) {
                     pv[n] = ex2_approx(x[n] - m[n]);
                     acc[n] += pv[n];
                 }
                 if (it >= 2) mbar_wait(&bar[bPfree + s], ((it - 2) >> 1) & 1, abort_flag, p.err);
                 if (lane < 16) {
-                    // P^T as a K-major operand: head n, tokens 8g .. 8g + 7 at g*256 + n*16
+                    // P^T as a K-major operand: row k NQ + n = bf16 part k of query n's p, tokens
+                    // 8g .. 8g + 7 at g*256 + row*16
                     char *pp = sm + Z::oP + s * Z::PBUF + (tok >> 3) * (kNQ * 16) + (tok & 7) * 2;
 #pragma unroll
-                    for (int n = 0; n < kNQ; ++n)
-                        *reinterpret_cast<uint16_t *>(pp + n * 16) = __bfloat16_as_ushort(__float2bfloat16_rn(pv[n]));
+                    for (int n = 0; n < NQ; ++n) {
+                        float pe[Z::PSPL];
+                        bf16_parts(pv[n], pe);
+#pragma unroll
+                        for (int k = 0; k < Z::PSPL; ++k)
+                            *reinterpret_cast<uint16_t *>(pp + (k * NQ + n) * 16) =
+                                __bfloat16_as_ushort(__float2bfloat16_rn(pe[k]));
+                    }
                 }
                 if (k == nps - 1 && tok0 + kPT > L) {
                     // V rows past the sequence hold no latents: zero them (0 * NaN would poison O)
@@ -580,13 +663,13 @@ __global__ void __launch_bounds__(kT2, 1)
 #pragma unroll
             for (int o = 8; o >= 1; o >>= 1)
 #pragma unroll
-                for (int n = 0; n < kNQ; ++n) acc[n] += __shfl_xor_sync(0xffffffffu, acc[n], o);
+                for (int n = 0; n < NQ; ++n) acc[n] += __shfl_xor_sync(0xffffffffu, acc[n], o);
             if (lane == 0) {
 #pragma unroll
-                for (int n = 0; n < kNQ; n += 4)
+                for (int n = 0; n < NQ; n += 4)
                     *reinterpret_cast<float4 *>(lsum + q4 * 16 + n) = make_float4(acc[n], acc[n + 1], acc[n + 2], acc[n + 3]);
             }
-            float *dst = p.part + static_cast<int64_t>(b + c) * Z::PSTRIDE;
+            float *dst = p.part + static_cast<int64_t>(u + c) * Z::PSTRIDE;
 #pragma unroll
             for (int ch = 0; ch < Z::NCH; ++ch) {
                 float o[kNQ];
@@ -594,17 +677,21 @@ __global__ void __launch_bounds__(kT2, 1)
                 const int j = ch * 128 + 32 * q4 + lane;
                 if (j < RV) {
 #pragma unroll
-                    for (int n = 0; n < Z::NQM; ++n)
-                        if (n < p.nq) dst[n * RV + j] = o[n];
+                    for (int n = 0; n < NQ; ++n) {
+                        float on = o[n];
+#pragma unroll
+                        for (int k = 1; k < Z::PSPL; ++k) on += o[k * NQ + n];
+                        if (n < p.nq) dst[n * RV + j] = on;
+                    }
                 }
             }
             tc_fence_before();
             mbar_arrive(&bar[bOfree]);
             named_bar_sync(1, 128);  // the run sums are visible
-            if (st_tid < kNQ) {
+            if (st_tid < NQ) {
                 float mine = 0.f;
 #pragma unroll
-                for (int n = 0; n < kNQ; ++n)
+                for (int n = 0; n < NQ; ++n)
                     if (st_tid == n) mine = m[n];
                 dst[Z::PO_M + st_tid] = mine;
                 dst[Z::PO_L + st_tid] = (lsum[st_tid] + lsum[16 + st_tid]) + (lsum[32 + st_tid] + lsum[48 + st_tid]);
@@ -624,9 +711,9 @@ __global__ void __launch_bounds__(kT2, 1)
 
 // ------------------------------------------------------------------------- finish kernel
 
-// Grid (H, ceil(B / spb)), 128 threads (thread e = output element e of head h).  spb (at most 8)
-// sequences share one pass over W_up,t,h^V; small batches take fewer per CTA to use more SMs.
-// (Sequence b, head h) is query h of sequence b.
+// Grid (weight slices, ceil(B / spb)), 128 threads (thread e = output element e).  spb (at most
+// 8) sequences share one pass over the slice's W_up^V; small batches take fewer per CTA to use
+// more SMs.  Slice w and sequence b give unit and query as in the absorb kernel.
 template <int RV, int NQM>
 __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     constexpr int PS = NQM * RV + 2 * kNQ;
@@ -635,25 +722,27 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     __shared__ float wts[kMaxGrid];
     __shared__ float coef[kFinishSeqs][3];
     __shared__ float redm[4], reds[4];
-    const int h = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
+    const int w = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(p.spb, p.B - b0);
-    const int64_t th = static_cast<int64_t>(p.loop) * p.H + h;
-    const int qn = h;  // the query of (b, h) within its sequence
+    const int t = p.loops ? w / p.H : p.loop, h = p.loops ? w - t * p.H : w;
+    const int64_t th = p.loops ? static_cast<int64_t>(h) * p.T + t : static_cast<int64_t>(t) * p.H + h;
+    const int qn = p.loops ? t : h;  // the query of (b, w) within its unit
+    auto iorow = [&](int b) { return ((p.loops ? static_cast<int64_t>(t) * p.B : 0) + b) * p.H + h; };
     pdl_wait();
-    const int NP = p.pstart[p.B];
+    const int NP = p.pstart[p.U];
     for (int bi = 0; bi < kFinishSeqs; ++bi) {
         if (bi >= nb) {
             for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
             continue;
         }
         const int b = b0 + bi;
-        const int u = b;
+        const int u = p.loops ? b * p.H + h : b;
         const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
         float M = -INFINITY, l = 0.f;
         if (s1 > s0) {
-            // the runs of sequence u: the CTAs c0 .. c1 that hold pages (a CTA between them may
-            // hold none and writes nothing), partials at slots u + c
+            // the runs of unit u: the CTAs c0 .. c1 that hold pages (a CTA between them may hold
+            // none and writes nothing), partials at slots u + c
             const int c0 = cta_of(s0, NP, p.grid), c1 = cta_of(s1 - 1, NP, p.grid);
             const int nr = c1 - c0 + 1;
             float mm = -INFINITY;
@@ -666,13 +755,13 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
             M = fmaxf(fmaxf(redm[0], redm[1]), fmaxf(redm[2], redm[3]));
             float ls = 0.f;
             for (int i = tid; i < nr; i += 128) {
-                float w = 0.f;  // no run: weight 0, and its slot is never read
+                float wt = 0.f;  // no run: weight 0, and its slot is never read
                 if (page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid)) {
                     const float *pr = p.part + static_cast<int64_t>(u + c0 + i) * PS;
-                    w = ex2_approx(pr[PO_M + qn] - M);
-                    ls = fmaf(w, pr[PO_L + qn], ls);
+                    wt = ex2_approx(pr[PO_M + qn] - M);
+                    ls = fmaf(wt, pr[PO_L + qn], ls);
                 }
-                wts[i] = w;
+                wts[i] = wt;
             }
             ls = warp_sum(ls);
             if (lane == 0) reds[warp] = ls;
@@ -685,9 +774,9 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
                 for (; i + 8 <= nr; i += 8) {  // eight partials in flight
                     float v[8];
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) v[u] = wts[i + u] > 0.f ? pj[static_cast<int64_t>(i + u) * PS + j] : 0.f;
+                    for (int e = 0; e < 8; ++e) v[e] = wts[i + e] > 0.f ? pj[static_cast<int64_t>(i + e) * PS + j] : 0.f;
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) a = fmaf(wts[i + u], v[u], a);
+                    for (int e = 0; e < 8; ++e) a = fmaf(wts[i + e], v[e], a);
                 }
                 for (; i < nr; ++i)
                     if (wts[i] > 0.f) a = fmaf(wts[i], pj[static_cast<int64_t>(i) * PS + j], a);
@@ -699,7 +788,7 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
         // pass 1: the current token's score against its exact key
         float sc = -INFINITY;
         if (p.cur_k) {
-            const int64_t row = (static_cast<int64_t>(b) * p.H + h) * kD;
+            const int64_t row = iorow(b) * kD;
             float v = load_elem(p.q, row + tid, p.io_bf16) * load_elem(p.cur_k, row + tid, p.io_bf16);
             v = warp_sum(v);
             __syncthreads();  // redm / reds are free
@@ -717,9 +806,9 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
             coef[bi][1] = al * l * inv;
             coef[bi][2] = pc * inv;
         }
-        __syncthreads();  // redm, reds and wts are free for the next sequence
+        __syncthreads();  // redm, reds and wts are free for the next unit
     }
-    // out_b[e] = coef0 (W_up,t,h^V o~_b)[e] + coef1 mu^V[e] + coef2 v_cur,b[e]
+    // out_b[e] = coef0 (W_up^V o~_b)[e] + coef1 mu^V[e] + coef2 v_cur,b[e]
     const int e = tid;
     const uint4 *W = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.w_up_v) + (th * kD + e) * RV);
     float acc[kFinishSeqs];
@@ -743,7 +832,7 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
 #pragma unroll
     for (int bi = 0; bi < kFinishSeqs; ++bi) {
         if (bi >= nb) break;
-        const int64_t idx = (static_cast<int64_t>(b0 + bi) * p.H + h) * kD + e;
+        const int64_t idx = iorow(b0 + bi) * kD + e;
         float v = acc[bi] * coef[bi][0] + coef[bi][1] * muv;
         if (p.cur_v) v = fmaf(coef[bi][2], load_elem(p.cur_v, idx, p.io_bf16), v);
         store_elem(p.out, idx, v, p.io_bf16);
@@ -787,31 +876,42 @@ WS2 ws2_layout(int rkx, int r_v, int nqm, int U, int grid) {
     return w;
 }
 
-template <int RK, int RV>
-lla_status launch_units(const DecodeArgs &a, cudaStream_t stream) {
-    using Z = Z2<RK, RV>;
+// The three launches for NQ query slots per unit; loops: the T loops of each (sequence, head)
+// of a per-head cache (hu = H units per sequence), else the H heads of each LLA-2D sequence.
+template <int RK, int RV, int NQ>
+lla_status launch_units(const DecodeArgs &a, bool loops, cudaStream_t stream) {
+    using Z = Z2<RK, RV, NQ>;
     lla_status st = LLA_OK;
     unsigned *err = device_error_word(&st);
     if (st != LLA_OK) return st;
     const int grid = num_sms();
     if (grid <= 0 || grid > kMaxGrid) return LLA_ERR_UNSUPPORTED;
-    const WS2 w = ws2_layout(Z::RKX, RV, Z::NQM, a.B, grid);
+    const int hu = loops ? a.H : 1;
+    const int nq = loops ? a.T : a.H;
+    const int nw = loops ? a.T * a.H : a.H;  // weight slices
+    if (nq < 1 || nq > NQ) return LLA_ERR_UNSUPPORTED;
+    if (static_cast<int64_t>(a.num_blocks) * hu >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // TMA coordinate
+    const int U = a.B * hu;
+    // the units' pages are numbered in 32 bits
+    if (static_cast<int64_t>(U) * ((static_cast<int64_t>(a.max_ctx) + kPT - 1) / kPT) >= (int64_t(1) << 31))
+        return LLA_ERR_UNSUPPORTED;
+    const WS2 w = ws2_layout(Z::RKX, RV, Z::NQM, U, grid);
     if (a.workspace_bytes < w.total) return LLA_ERR_WORKSPACE;
     char *ws = static_cast<char *>(a.workspace);
     static bool configured[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
     if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
+        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
             cudaSuccess)
             return LLA_ERR_CUDA;
         configured[dev] = true;
     }
     const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
-    // the V-planes of every page: [num_blocks][64 tokens][r_v] bf16
+    // the V-planes of every page: [num_blocks * hu][64 tokens][r_v] bf16
     CUtensorMap tv;
     const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT),
-                              static_cast<uint64_t>(a.num_blocks)};
+                              static_cast<uint64_t>(a.num_blocks) * hu};
     const uint64_t strides[2] = {static_cast<uint64_t>(RV) * 2, static_cast<uint64_t>(page_bytes)};
     const uint32_t box[3] = {64, kPT, 1};
     if (!encode_tmap_bf16(&tv, static_cast<const char *>(a.pool) + kPT * RK * 2, 3, dims, strides, box, true))
@@ -820,17 +920,19 @@ lla_status launch_units(const DecodeArgs &a, cudaStream_t stream) {
     A2Params ap = {};
     ap.T = a.T; ap.H = a.H; ap.loop = a.loop; ap.io_bf16 = a.io_bf16; ap.pass1 = a.cur_k != nullptr;
     ap.B = a.B; ap.max_ctx = a.max_ctx; ap.max_blocks = a.max_blocks;
+    ap.loops = loops ? 1 : 0; ap.hu = hu;
     ap.scale_log2 = a.scale * kLog2e;
     ap.w_up_k = a.w_up_k; ap.mu_k = a.mu_k; ap.q = a.q; ap.context_lens = a.context_lens;
     ap.qt = reinterpret_cast<float *>(ws + w.qt);
     ap.beta = reinterpret_cast<float *>(ws + w.beta);
     ap.pstart = reinterpret_cast<int *>(ws + w.pstart);
     ap.err = err;
-    if ((st = launch_ex(absorb2d_kernel<RK>, dim3(a.H, RK / 32, (a.B + 15) / 16), 256, 0, stream, ap)) != LLA_OK)
+    if ((st = launch_ex(absorb2d_kernel<RK, NQ>, dim3(nw, Z::RKX / 32 + (Z::RKX % 32 ? 1 : 0), (a.B + 15) / 16), 256, 0,
+                        stream, ap)) != LLA_OK)
         return st;
 
     T2Params tp = {};
-    tp.nq = a.H; tp.B = a.B;
+    tp.nq = nq; tp.U = U; tp.hu = hu;
     tp.pool = static_cast<const char *>(a.pool);
     tp.num_blocks = a.num_blocks; tp.page_bytes = page_bytes;
     tp.block_table = a.block_table; tp.max_blocks = a.max_blocks;
@@ -838,19 +940,20 @@ lla_status launch_units(const DecodeArgs &a, cudaStream_t stream) {
     tp.qt = ap.qt; tp.beta = ap.beta; tp.pstart = ap.pstart;
     tp.part = reinterpret_cast<float *>(ws + w.part);
     tp.err = err;
-    if ((st = launch_ex(attn2d_kernel<RK, RV>, dim3(grid), kT2, Z::SMEM, stream, tv, tp)) != LLA_OK)
+    if ((st = launch_ex(attn2d_kernel<RK, RV, NQ>, dim3(grid), kT2, Z::SMEM, stream, tv, tp)) != LLA_OK)
         return st;
 
     F2Params fp = {};
     fp.T = a.T; fp.H = a.H; fp.loop = a.loop; fp.io_bf16 = a.io_bf16; fp.B = a.B; fp.grid = grid;
+    fp.loops = ap.loops; fp.hu = hu; fp.U = U;
     fp.scale_log2 = ap.scale_log2;
     fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
     fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
     fp.pstart = ap.pstart; fp.part = tp.part;
     // about two finish CTAs per SM: fewer sequences per CTA for small batches
-    const int64_t want = static_cast<int64_t>(a.B) * a.H;
+    const int64_t want = static_cast<int64_t>(a.B) * nw;
     fp.spb = static_cast<int>(std::min<int64_t>(kFinishSeqs, std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
-    return launch_ex(finish2d_kernel<RV, Z::NQM>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
+    return launch_ex(finish2d_kernel<RV, Z::NQM>, dim3(nw, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
 }
 
 // ------------------------------------------------------------------------- rotary keys
@@ -942,11 +1045,39 @@ lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream) {
     if (a.B == 0) return LLA_OK;
     if (a.num_blocks >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // 32-bit TMA coordinate
 #define LLA_2D(K, V) \
-    if (a.r_k == K && a.r_v == V) return launch_units<K, V>(a, stream);
+    if (a.r_k == K && a.r_v == V) return launch_units<K, V, kNQ>(a, false, stream);
     LLA_2D(96, 160)
     LLA_2D(128, 128)
     LLA_2D(288, 480)
 #undef LLA_2D
+    return LLA_ERR_UNSUPPORTED;
+}
+
+// The T loops of a per-head cache: up to 4 loops per (sequence, head) unit.
+constexpr int kLoopSlots = 4;
+
+lla_status decode_loops_fits(int r_k, int r_v, int es, int d, int T, int B) {
+    (void)B;
+    if (es != 2 || d != kD || T < 1 || T > kLoopSlots) return LLA_ERR_UNSUPPORTED;
+    if ((r_k == 96 && r_v == 160) || (r_k == 128 && r_v == 128) || (r_k == 72 && r_v == 120) ||
+        (r_k == 192 && r_v == 320))
+        return LLA_OK;
+    return LLA_ERR_UNSUPPORTED;
+}
+
+size_t decode_loops_workspace_bytes(int r_k, int r_v, int B, int H, int grid) {
+    return ws2_layout((r_k + 15) / 16 * 16, r_v, kLoopSlots, B * H, grid).total;
+}
+
+lla_status launch_decode_loops(const DecodeArgs &a, cudaStream_t stream) {
+    if (a.B == 0) return LLA_OK;
+#define LLA_LOOPS(K, V) \
+    if (a.r_k == K && a.r_v == V) return launch_units<K, V, kLoopSlots>(a, true, stream);
+    LLA_LOOPS(96, 160)
+    LLA_LOOPS(128, 128)
+    LLA_LOOPS(72, 120)
+    LLA_LOOPS(192, 320)
+#undef LLA_LOOPS
     return LLA_ERR_UNSUPPORTED;
 }
 

@@ -78,9 +78,10 @@ lla_status launch_decode(const DecodeArgs &a, cudaStream_t stream);
 // pairing (0: (j, j + d/2), 1: (2j, 2j + 1)).
 lla_status decode_rope_fits(int r_k, int r_v, int es, int d, int B);
 // The decode calls of all T loops in one pass over the latents (q, cur_k, cur_v, out are
-// [T][B][H][d]): UNSUPPORTED unless a kernel shape exists and fits; its workspace size.
+// [T][B][H][d]; the shared-latent tensor-core kernels of lla_decode_2d.cu with one unit per
+// (sequence, head)): UNSUPPORTED unless a kernel shape exists; its workspace size.
 lla_status decode_loops_fits(int r_k, int r_v, int es, int d, int T, int B);
-size_t decode_loops_workspace_bytes(int r_v, int B, int H, int T, int grid);
+size_t decode_loops_workspace_bytes(int r_k, int r_v, int B, int H, int grid);
 lla_status launch_decode_loops(const DecodeArgs &a, cudaStream_t stream);
 lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cudaStream_t stream);
 

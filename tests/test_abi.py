@@ -233,7 +233,7 @@ def test_decode_rope_argument_checks(lib):
     assert _decode_rope(lib, loop=4) == INVALID
     assert _decode_rope(lib, ws=None) == INVALID
     # shapes without a tensor-core key rebuild
-    assert _decode_rope(lib, g=_g(lib, r_k=72, r_v=120)) == UNSUPPORTED   # r_k not a multiple of 16
+    assert _decode_rope(lib, g=_g(lib, r_k=18, r_v=30)) == UNSUPPORTED    # 4-byte K granules
     assert _decode_rope(lib, g=_g(lib, storage="fp32")) == UNSUPPORTED
     assert _decode_rope(lib, g=_g(lib, d=64)) == UNSUPPORTED
     assert _decode_rope(lib, B=0, lens=None, q=None, out=None, ws=None) == OK
@@ -281,8 +281,8 @@ def test_decode_loops_argument_checks(lib):
     assert call(B=-1) == INVALID
     assert call(q=None) == INVALID
     assert call(max_ctx=4 * 64 + 1) == INVALID
-    assert call(g=_g(lib, T=3)) == UNSUPPORTED
-    assert call(g=_g(lib, r_k=72, r_v=120)) == UNSUPPORTED
+    assert call(g=_g(lib, T=5)) == UNSUPPORTED          # more loops than query slots
+    assert call(g=_g(lib, r_k=18, r_v=30)) == UNSUPPORTED
     assert call(g=_g(lib, storage="fp32")) == UNSUPPORTED
     assert call(B=0, q=None, ck=None, cv=None, out=None, ws=None, lens=None) == OK
 
