@@ -20,15 +20,16 @@
 //                     per run the partial (maximum, sum, O^T) of every query.
 //                       warp 0     producer: the K-plane of a page by one bulk copy, its V-plane
 //                                  by TMA boxes of 64 columns with 128-byte swizzle
-//                       warp 1     MMA issuer and TMEM owner: S^T (M = 64 tokens, N = 2 NQ: q~
-//                                  as a bf16 high part and a bf16 remainder per query, so that
-//                                  the scores see q~ to about 16 significant bits; K = r_k, a
-//                                  rank that is not a multiple of 16 padded with zero columns)
-//                                  and O^T (M = 128 latent rows per chunk, N = 16 queries padded
-//                                  with zero rows of P^T, K = 64 tokens; the swizzled V-plane is
-//                                  an MN-major A operand); the O^T product of a page is issued
-//                                  after the next page's S^T, so the softmax of one page overlaps
-//                                  the next page's scores
+//                       warp 1     S^T issuer and TMEM owner: M = 64 tokens, N = the q~ parts
+//                                  of the NQ queries (q~ as a bf16 high part and remainders, so
+//                                  that the scores see q~ to 16 or 24 significant bits), K = r_k
+//                                  (a rank that is not a multiple of 16 padded with zero
+//                                  columns); it runs up to two pages ahead of the softmax
+//                       warp 6     O^T issuer: M = 128 latent rows per chunk, N = 16 (the p
+//                                  parts of the queries, padded with zero rows of P^T), K = 64
+//                                  tokens; the swizzled V-plane is an MN-major A operand.  Two
+//                                  issuing threads, because an MMA takes its issuing thread tens
+//                                  of cycles
 //                       warps 2-5  per page: the scores of 16 tokens per warp, the maxima over
 //                                  the page per query, P^T as a bf16 operand, the lazy O^T
 //                                  rescale; per run: the partial out to the workspace
@@ -52,8 +53,9 @@ namespace {
 constexpr int kPT = 64;          // tokens per page
 constexpr int kD = 128;          // head width
 constexpr int kNQ = 16;          // O^T columns: the queries of a unit, padded
-constexpr int kT2 = 192;         // threads of the attention kernel
+constexpr int kT2 = 224;         // threads of the attention kernel
 constexpr int kSm0 = 64;         // first softmax thread
+constexpr int kPvWarp = 6;       // issuer of the O^T products
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;  // rescale O^T only when a query's maximum grows by more
 constexpr int kSmemCap = 227 * 1024;
@@ -236,13 +238,13 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
     auto unit = [&](int b) { return p.loops ? b * p.H + h : b; };
     auto iorow = [&](int b) { return ((p.loops ? static_cast<int64_t>(t) * p.B : 0) + b) * p.H + h; };
     const int col = j0 + lane;
-    pdl_wait();  // inputs may come from the previous kernel; the workspace is free after it
-    // this thread's 16 weights (column j0 + lane, rows 16 warp .. 16 warp + 15), in flight while
-    // the queries load
+    // this thread's 16 weights (column j0 + lane, rows 16 warp .. 16 warp + 15): inputs of the
+    // call, loaded before the wait on the previous kernel
     const uint16_t *W = static_cast<const uint16_t *>(p.w_up_k) + th * kD * RK + col;
     float wv[16];
 #pragma unroll
     for (int u = 0; u < 16; ++u) wv[u] = col < RK ? bf_to_f(W[(warp * 16 + u) * RK]) : 0.f;
+    pdl_wait();  // the queries may come from the previous kernel; the workspace is free after it
     if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) page_prefix(p);
     for (int i = tid; i < 16 * kD; i += 256) {
         const int bi = i >> 7, e = i & (kD - 1);
@@ -431,32 +433,14 @@ __global__ void __launch_bounds__(kT2, 1)
         }
         __syncwarp();
     } else if (warp == 1) {
-        // ------------------------------------------------------------------------ MMA issuer
+        // ---------------------------------------------------------------- S^T issuer
+        // (an MMA takes its issuing thread tens of cycles: the score and value products of a
+        // page are issued by two threads, each committing only its own products)
         if (lane == 0) {
             const uint32_t base = smem_addr(sm);
             const uint64_t dq = umma_desc(base + Z::oQ, Z::NS * 16, 128);
             const uint64_t dk0 = umma_desc(base + Z::oK, kPT * 16, 128);
-            const uint64_t dp0 = umma_desc(base + Z::oP, kNQ * 16, 128);
-            const uint64_t dv0 = umma_desc_sw128_mn(base + Z::oV, Z::BOX);
             int it = 0, r = 0;
-            // O^T += C_v^T P^T for page j (first: the first page of run rr zeroes O^T)
-            auto issue_pv = [&](int j, bool first, int rr) {
-                const int s = j & 1, st = j % Z::ST;
-                mbar_wait(&bar[bPfull + s], (j >> 1) & 1, abort_flag, p.err);
-                mbar_wait(&bar[bVfull + st], (j / Z::ST) & 1, abort_flag, p.err);
-                if (first && rr > 0) mbar_wait(&bar[bOfree], (rr - 1) & 1, abort_flag, p.err);
-                tc_fence_after();
-                const uint64_t dv = dv0 + static_cast<uint64_t>((st * Z::VPAGE) >> 4);
-                const uint64_t dp = dp0 + static_cast<uint64_t>((s * Z::PBUF) >> 4);
-#pragma unroll
-                for (int ch = 0; ch < Z::NCH; ++ch)
-#pragma unroll
-                    for (int ks = 0; ks < kPT / 16; ++ks)
-                        umma_bf16(tmem + Z::TM_O + ch * kNQ, dv + ((ch * 2 * Z::BOX + ks * 2048) >> 4),
-                                  dp + ks * ((2 * kNQ * 16) >> 4), Z::IDESC_O, !first || ks > 0);
-                umma_commit(&bar[bVempty + st]);
-                umma_commit(&bar[bPfree + s]);  // also: O^T holds pages up to j
-            };
             for (int u = ufirst; u < p.U; ++u) {
                 const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
                 if (s0 >= g1) break;
@@ -477,12 +461,46 @@ __global__ void __launch_bounds__(kT2, 1)
                     umma_commit(&bar[bSfull + s]);
                     umma_commit(&bar[bKempty + st]);
                     if (k == n - 1) umma_commit(&bar[bQfree]);
-                    if (k > 0) issue_pv(it - 1, k == 1, r);
                 }
-                issue_pv(it - 1, n == 1, r);
                 ++r;
             }
-            // every MMA has completed before TMEM is released, even after an abort (the last
+            // the softmax warps wait for every S^T product (its full barrier) before they finish
+        }
+        __syncwarp();
+    } else if (warp == kPvWarp) {
+        // ---------------------------------------------------------------- O^T issuer
+        if (lane == 0) {
+            const uint32_t base = smem_addr(sm);
+            const uint64_t dp0 = umma_desc(base + Z::oP, kNQ * 16, 128);
+            const uint64_t dv0 = umma_desc_sw128_mn(base + Z::oV, Z::BOX);
+            int it = 0, r = 0;
+            for (int u = ufirst; u < p.U; ++u) {
+                const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
+                if (s0 >= g1) break;
+                const int n = min(g1, s1) - max(g0, s0);
+                if (n <= 0) continue;
+                for (int k = 0; k < n; ++k, ++it) {
+                    // O^T += C_v^T P^T for page it (the first page of run r zeroes O^T, once the
+                    // softmax warps have read run r - 1's)
+                    const int s = it & 1, st = it % Z::ST;
+                    mbar_wait(&bar[bPfull + s], (it >> 1) & 1, abort_flag, p.err);
+                    mbar_wait(&bar[bVfull + st], (it / Z::ST) & 1, abort_flag, p.err);
+                    if (k == 0 && r > 0) mbar_wait(&bar[bOfree], (r - 1) & 1, abort_flag, p.err);
+                    tc_fence_after();
+                    const uint64_t dv = dv0 + static_cast<uint64_t>((st * Z::VPAGE) >> 4);
+                    const uint64_t dp = dp0 + static_cast<uint64_t>((s * Z::PBUF) >> 4);
+#pragma unroll
+                    for (int ch = 0; ch < Z::NCH; ++ch)
+#pragma unroll
+                        for (int ks = 0; ks < kPT / 16; ++ks)
+                            umma_bf16(tmem + Z::TM_O + ch * kNQ, dv + ((ch * 2 * Z::BOX + ks * 2048) >> 4),
+                                      dp + ks * ((2 * kNQ * 16) >> 4), Z::IDESC_O, k > 0 || ks > 0);
+                    umma_commit(&bar[bVempty + st]);
+                    umma_commit(&bar[bPfree + s]);  // also: O^T holds pages up to it
+                }
+                ++r;
+            }
+            // every product has completed before TMEM is released, even after an abort (the last
             // product's completion on its P buffer; the one before on the other buffer had
             // completed before the softmax released the last page)
             if (it > 0) {
@@ -713,15 +731,20 @@ __global__ void __launch_bounds__(kT2, 1)
 
 // Grid (weight slices, ceil(B / spb)), 128 threads (thread e = output element e).  spb (at most
 // 8) sequences share one pass over the slice's W_up^V; small batches take fewer per CTA to use
-// more SMs.  Slice w and sequence b give unit and query as in the absorb kernel.
+// more SMs.  Slice w and sequence b give unit and query as in the absorb kernel.  The runs of a
+// unit are merged by one warp, or by two or four that split its columns when the CTA has fewer
+// than three units (no block barrier between units: each is a chain of dependent loads), then
+// all threads apply W_up^V; rows of W_up^V up to 160 wide are loaded before the wait on the
+// attention kernel.
 template <int RV, int NQM>
-__global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
+__global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     constexpr int PS = NQM * RV + 2 * kNQ;
     constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
+    constexpr bool kPre = RV <= 160;
+    constexpr int NW = kPre ? RV / 8 : 1;
     __shared__ __align__(16) float ob[kFinishSeqs][RV];
-    __shared__ float wts[kMaxGrid];
+    __shared__ float wts[4][kMaxGrid];  // per warp: the run weights of its current unit
     __shared__ float coef[kFinishSeqs][3];
-    __shared__ float redm[4], reds[4];
     const int w = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(p.spb, p.B - b0);
@@ -729,94 +752,104 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
     const int64_t th = p.loops ? static_cast<int64_t>(h) * p.T + t : static_cast<int64_t>(t) * p.H + h;
     const int qn = p.loops ? t : h;  // the query of (b, w) within its unit
     auto iorow = [&](int b) { return ((p.loops ? static_cast<int64_t>(t) * p.B : 0) + b) * p.H + h; };
+    // this thread's row e of W_up^V and mu^V (inputs of the call, not of earlier kernels)
+    const int e = tid;
+    const uint4 *W = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.w_up_v) + (th * kD + e) * RV);
+    uint4 wr[NW];
+    if constexpr (kPre) {
+#pragma unroll
+        for (int j8 = 0; j8 < NW; ++j8) wr[j8] = W[j8];
+    }
+    const float muv = p.mu_v ? p.mu_v[th * kD + e] : 0.f;
     pdl_wait();
     const int NP = p.pstart[p.U];
-    for (int bi = 0; bi < kFinishSeqs; ++bi) {
+    // G warps per unit (all four for one unit, two each for two): warp `sub` of a group takes
+    // the columns j = lane + 32 (sub + G q)
+    const int G = nb == 1 ? 4 : nb == 2 ? 2 : 1;
+    const int grp = warp / G, sub = warp - grp * G;
+    constexpr int NJ = (RV + 31) / 32;
+    float *wt = wts[warp];
+    for (int bi = grp; bi < kFinishSeqs; bi += 4 / G) {
         if (bi >= nb) {
-            for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
+            for (int j = lane + 32 * sub; j < RV; j += 32 * G) ob[bi][j] = 0.f;
             continue;
         }
         const int b = b0 + bi;
         const int u = p.loops ? b * p.H + h : b;
+        // pass 1: the current token's score against its exact key (loads issued first)
+        float qk = 0.f;
+        if (p.cur_k && sub == 0) {
+            const int64_t row = iorow(b) * kD;
+#pragma unroll
+            for (int i = 0; i < kD / 32; ++i)
+                qk = fmaf(load_elem(p.q, row + lane + 32 * i, p.io_bf16), load_elem(p.cur_k, row + lane + 32 * i, p.io_bf16), qk);
+        }
         const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
         float M = -INFINITY, l = 0.f;
+        float acc[NJ];
+#pragma unroll
+        for (int q = 0; q < NJ; ++q) acc[q] = 0.f;
         if (s1 > s0) {
             // the runs of unit u: the CTAs c0 .. c1 that hold pages (a CTA between them may hold
             // none and writes nothing), partials at slots u + c
             const int c0 = cta_of(s0, NP, p.grid), c1 = cta_of(s1 - 1, NP, p.grid);
             const int nr = c1 - c0 + 1;
+            const float *pu = p.part + static_cast<int64_t>(u + c0) * PS;
             float mm = -INFINITY;
-            for (int i = tid; i < nr; i += 128)
-                if (page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid))
-                    mm = fmaxf(mm, p.part[static_cast<int64_t>(u + c0 + i) * PS + PO_M + qn]);
-            mm = warp_max(mm);
-            if (lane == 0) redm[warp] = mm;
-            __syncthreads();
-            M = fmaxf(fmaxf(redm[0], redm[1]), fmaxf(redm[2], redm[3]));
+            for (int i = lane; i < nr; i += 32) {
+                const bool has = page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid);
+                wt[i] = has ? pu[static_cast<int64_t>(i) * PS + PO_M + qn] : -INFINITY;
+                mm = fmaxf(mm, wt[i]);
+            }
+            M = warp_max(mm);
             float ls = 0.f;
-            for (int i = tid; i < nr; i += 128) {
-                float wt = 0.f;  // no run: weight 0, and its slot is never read
-                if (page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid)) {
-                    const float *pr = p.part + static_cast<int64_t>(u + c0 + i) * PS;
-                    wt = ex2_approx(pr[PO_M + qn] - M);
-                    ls = fmaf(wt, pr[PO_L + qn], ls);
-                }
-                wts[i] = wt;
+            for (int i = lane; i < nr; i += 32) {
+                const float w8 = wt[i] == -INFINITY ? 0.f : ex2_approx(wt[i] - M);  // no run: 0
+                if (w8 > 0.f) ls = fmaf(w8, pu[static_cast<int64_t>(i) * PS + PO_L + qn], ls);
+                wt[i] = w8;
             }
-            ls = warp_sum(ls);
-            if (lane == 0) reds[warp] = ls;
-            __syncthreads();
-            l = (reds[0] + reds[1]) + (reds[2] + reds[3]);
-            const float *pj = p.part + static_cast<int64_t>(u + c0) * PS + qn * RV;
-            for (int j = tid; j < RV; j += 128) {
-                float a = 0.f;
-                int i = 0;
-                for (; i + 8 <= nr; i += 8) {  // eight partials in flight
-                    float v[8];
+            l = warp_sum(ls);
+            __syncwarp();
+            // every column load of a run in flight at once, runs four at a time
+#pragma unroll 4
+            for (int i = 0; i < nr; ++i) {
+                const float w8 = wt[i];
+                if (w8 > 0.f) {  // warp-uniform; a slot without a run is never read
+                    const float *pr = pu + static_cast<int64_t>(i) * PS + qn * RV;
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) v[e] = wts[i + e] > 0.f ? pj[static_cast<int64_t>(i + e) * PS + j] : 0.f;
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) a = fmaf(wts[i + e], v[e], a);
+                    for (int q = 0; q < NJ; ++q) {
+                        const int j = lane + 32 * (sub + G * q);
+                        if (j < RV) acc[q] = fmaf(w8, pr[j], acc[q]);
+                    }
                 }
-                for (; i < nr; ++i)
-                    if (wts[i] > 0.f) a = fmaf(wts[i], pj[static_cast<int64_t>(i) * PS + j], a);
-                ob[bi][j] = a;
             }
-        } else {
-            for (int j = tid; j < RV; j += 128) ob[bi][j] = 0.f;
+            __syncwarp();  // wt is free for the warp's next unit
         }
-        // pass 1: the current token's score against its exact key
-        float sc = -INFINITY;
-        if (p.cur_k) {
-            const int64_t row = iorow(b) * kD;
-            float v = load_elem(p.q, row + tid, p.io_bf16) * load_elem(p.cur_k, row + tid, p.io_bf16);
-            v = warp_sum(v);
-            __syncthreads();  // redm / reds are free
-            if (lane == 0) reds[warp] = v;
-            __syncthreads();
-            sc = ((reds[0] + reds[1]) + (reds[2] + reds[3])) * p.scale_log2;
+#pragma unroll
+        for (int q = 0; q < NJ; ++q) {
+            const int j = lane + 32 * (sub + G * q);
+            if (j < RV) ob[bi][j] = acc[q];
         }
-        if (tid == 0) {
-            const float Mx = fmaxf(M, sc);
-            const float al = M == -INFINITY ? 0.f : ex2_approx(M - Mx);
-            const float pc = p.cur_k ? ex2_approx(sc - Mx) : 0.f;
-            const float den = al * l + pc;
-            const float inv = den > 0.f ? 1.f / den : 0.f;
-            coef[bi][0] = al * inv;
-            coef[bi][1] = al * l * inv;
-            coef[bi][2] = pc * inv;
+        if (sub == 0) {
+            const float sc = p.cur_k ? warp_sum(qk) * p.scale_log2 : -INFINITY;
+            if (lane == 0) {
+                const float Mx = fmaxf(M, sc);
+                const float al = M == -INFINITY ? 0.f : ex2_approx(M - Mx);
+                const float pc = p.cur_k ? ex2_approx(sc - Mx) : 0.f;
+                const float den = al * l + pc;
+                const float inv = den > 0.f ? 1.f / den : 0.f;
+                coef[bi][0] = al * inv;
+                coef[bi][1] = al * l * inv;
+                coef[bi][2] = pc * inv;
+            }
         }
-        __syncthreads();  // redm, reds and wts are free for the next unit
     }
+    __syncthreads();
     // out_b[e] = coef0 (W_up^V o~_b)[e] + coef1 mu^V[e] + coef2 v_cur,b[e]
-    const int e = tid;
-    const uint4 *W = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.w_up_v) + (th * kD + e) * RV);
     float acc[kFinishSeqs];
 #pragma unroll
     for (int bi = 0; bi < kFinishSeqs; ++bi) acc[bi] = 0.f;
-#pragma unroll 4
-    for (int j8 = 0; j8 < RV / 8; ++j8) {
-        const uint4 w4 = W[j8];
+    auto step = [&](int j8, const uint4 w4) {
         const float2 w0 = bf2_to_f2(w4.x), w1 = bf2_to_f2(w4.y), w2 = bf2_to_f2(w4.z), w3 = bf2_to_f2(w4.w);
 #pragma unroll
         for (int bi = 0; bi < kFinishSeqs; ++bi) {
@@ -827,8 +860,14 @@ __global__ void __launch_bounds__(128) finish2d_kernel(const F2Params p) {
             a = fmaf(w2.x, o1.x, a); a = fmaf(w2.y, o1.y, a); a = fmaf(w3.x, o1.z, a); a = fmaf(w3.y, o1.w, a);
             acc[bi] = a;
         }
+    };
+    if constexpr (kPre) {
+#pragma unroll
+        for (int j8 = 0; j8 < NW; ++j8) step(j8, wr[j8]);  // fully unrolled: wr stays in registers
+    } else {
+#pragma unroll 4
+        for (int j8 = 0; j8 < RV / 8; ++j8) step(j8, W[j8]);
     }
-    const float muv = p.mu_v ? p.mu_v[th * kD + e] : 0.f;
 #pragma unroll
     for (int bi = 0; bi < kFinishSeqs; ++bi) {
         if (bi >= nb) break;
