@@ -5,6 +5,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <algorithm>
 #include <atomic>
 
 #include "lla_internal.h"
@@ -177,7 +178,11 @@ lla_status lla_decode_workspace_size(const lla_geometry *g, int32_t B, size_t *b
     if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
     const int sms = num_sms();
     if (sms <= 0) return LLA_ERR_CUDA;
-    *bytes = decode_workspace_bytes(g->r_v, B, g->H, sms);  // one CTA per SM
+    // one CTA per SM; the full-RoPE decode on the tensor cores keeps a slot per (unit, CTA) run
+    size_t n = decode_workspace_bytes(g->r_v, B, g->H, sms);
+    if (decode_rope_tc_supported(elem_size(g->storage), g->d, g->r_k, g->r_v))
+        n = std::max(n, decode_rope_tc_workspace_bytes(g->r_v, B, g->H, sms));
+    *bytes = n;
     return LLA_OK;
 }
 

@@ -46,6 +46,7 @@
 #include "lla_internal.h"
 #include "lla_tcgen05.cuh"
 #include "lla_tmap.h"
+#include "lla_units.cuh"
 
 namespace lla {
 namespace {
@@ -167,17 +168,6 @@ struct F2Params {
     const int *pstart;
     const float *part;
 };
-
-// CTA c of `grid` holds the global pages [page_lo(c), page_lo(c + 1)) of the np pages; with
-// fewer pages than CTAs some CTAs hold none.
-__host__ __device__ __forceinline__ int page_lo(int c, int np, int grid) {
-    return static_cast<int>(static_cast<int64_t>(c) * np / grid);
-}
-
-// The CTA that holds global page g (the last c with page_lo(c) <= g).
-__host__ __device__ __forceinline__ int cta_of(int g, int np, int grid) {
-    return static_cast<int>((static_cast<int64_t>(g + 1) * grid + np - 1) / np) - 1;
-}
 
 // ------------------------------------------------------------------------- absorb kernel
 
@@ -881,22 +871,6 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
 }
 
 // ------------------------------------------------------------------------- host side
-
-template <typename K, typename... Args>
-lla_status launch_ex(K kern, dim3 grid, int threads, int smem, cudaStream_t stream, Args... args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = dim3(threads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, kern, args...) != cudaSuccess) return LLA_ERR_CUDA;
-    return LLA_OK;
-}
 
 struct WS2 {
     size_t part, qt, beta, pstart, total;

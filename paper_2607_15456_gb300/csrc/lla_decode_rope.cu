@@ -512,14 +512,45 @@ int rope_stages(const RopeEntry &e, int stage_bytes, int B) {
 }  // namespace
 
 lla_status decode_rope_fits(int r_k, int r_v, int es, int d, int B) {
+    if (decode_rope_tc_supported(es, d, r_k, r_v)) return LLA_OK;
     const RopeEntry e = rope_entry(es, d, r_k, r_v);
     if (!e.launch) return LLA_ERR_UNSUPPORTED;
     const int hpb = static_cast<int>(head_page_bytes(r_k, r_v, es));
     return rope_stages(e, hpb, B) >= 2 ? LLA_OK : LLA_ERR_UNSUPPORTED;
 }
 
+void rope_tables(double base, int d, RopeTables *t) {
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int j = 0; j < kRopePairs; ++j) {
+        const double theta = pow(base, -2.0 * j / d);
+        const double turns = theta / two_pi;  // < 1: theta_j <= 1
+        t->phi[j] = static_cast<unsigned long long>(ldexp(turns, 64));
+        t->c1[j] = static_cast<float>(cos(theta));
+        t->s1[j] = static_cast<float>(sin(theta));
+        t->c32[j] = static_cast<float>(cos(32.0 * theta));
+        t->s32[j] = static_cast<float>(sin(32.0 * theta));
+        t->s2[j] = static_cast<float>(sin(2.0 * theta));
+        const double sh = sin(theta);
+        t->h2[j] = static_cast<float>(2.0 * sh * sh);  // 1 - cos 2 theta, without cancellation
+    }
+}
+
 lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cudaStream_t stream) {
     const int es = a.storage_bf16 ? 2 : 4;
+    // the rotation tables of this base (kept for the next call with the same base and width)
+    struct TableCache {
+        double base = 0.0;
+        int d = 0;
+        RopeTables t;
+    };
+    static thread_local TableCache cache;
+    if (!(cache.base == base && cache.d == a.d)) {
+        rope_tables(base, a.d, &cache.t);
+        cache.base = base;
+        cache.d = a.d;
+    }
+    const RopeTables &t = cache.t;
+    if (decode_rope_tc_supported(es, a.d, a.r_k, a.r_v)) return launch_decode_rope_tc(a, t, pairing, stream);
     const RopeEntry e = rope_entry(es, a.d, a.r_k, a.r_v);
     if (!e.launch) return LLA_ERR_UNSUPPORTED;
     const int hpb = static_cast<int>(head_page_bytes(a.r_k, a.r_v, es));
@@ -553,43 +584,14 @@ lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cud
     p.counters = reinterpret_cast<int *>(static_cast<char *>(a.workspace) + part_al);
     p.pps = 1; p.stages = stages; p.stage_bytes = hpb;
     p.err = err;
-    // theta_j = base^(-2j/d): its phase step in 64-bit fixed-point turns and the per-pair
-    // constants of the recurrence, in double precision (kept for the next call with the same
-    // base and head width)
-    struct TableCache {
-        double base = 0.0;
-        int d = 0;
-        RopeParams rp;
-    };
-    static thread_local TableCache cache;
-    if (cache.base == base && cache.d == a.d) {
-        memcpy(rp.phi, cache.rp.phi, sizeof(rp.phi));
-        memcpy(rp.c1, cache.rp.c1, sizeof(rp.c1));
-        memcpy(rp.s1, cache.rp.s1, sizeof(rp.s1));
-        memcpy(rp.c32, cache.rp.c32, sizeof(rp.c32));
-        memcpy(rp.s32, cache.rp.s32, sizeof(rp.s32));
-        memcpy(rp.s2, cache.rp.s2, sizeof(rp.s2));
-        memcpy(rp.h2, cache.rp.h2, sizeof(rp.h2));
-        rp.pairing = pairing;
-        return e.launch(rp, grid, smem, stream);
-    }
-    const double two_pi = 6.283185307179586476925286766559;
-    for (int j = 0; j < kRopePairs; ++j) {
-        const double theta = pow(base, -2.0 * j / a.d);
-        const double turns = theta / two_pi;  // < 1: theta_j <= 1
-        rp.phi[j] = static_cast<unsigned long long>(ldexp(turns, 64));
-        rp.c1[j] = static_cast<float>(cos(theta));
-        rp.s1[j] = static_cast<float>(sin(theta));
-        rp.c32[j] = static_cast<float>(cos(32.0 * theta));
-        rp.s32[j] = static_cast<float>(sin(32.0 * theta));
-        rp.s2[j] = static_cast<float>(sin(2.0 * theta));
-        const double sh = sin(theta);
-        rp.h2[j] = static_cast<float>(2.0 * sh * sh);  // 1 - cos 2 theta, without cancellation
-    }
+    memcpy(rp.phi, t.phi, sizeof(rp.phi));
+    memcpy(rp.c1, t.c1, sizeof(rp.c1));
+    memcpy(rp.s1, t.s1, sizeof(rp.s1));
+    memcpy(rp.c32, t.c32, sizeof(rp.c32));
+    memcpy(rp.s32, t.s32, sizeof(rp.s32));
+    memcpy(rp.s2, t.s2, sizeof(rp.s2));
+    memcpy(rp.h2, t.h2, sizeof(rp.h2));
     rp.pairing = pairing;
-    cache.base = base;
-    cache.d = a.d;
-    cache.rp = rp;
     return e.launch(rp, grid, smem, stream);
 }
 

@@ -84,6 +84,20 @@ lla_status decode_loops_fits(int r_k, int r_v, int es, int d, int T, int B);
 size_t decode_loops_workspace_bytes(int r_k, int r_v, int B, int H, int grid);
 lla_status launch_decode_loops(const DecodeArgs &a, cudaStream_t stream);
 lla_status launch_decode_rope(const DecodeArgs &a, double base, int pairing, cudaStream_t stream);
+// Per rotation pair j of a 128-wide head: theta_j = base^(-2j/128) as 64-bit fixed-point turns,
+// and cos / sin of theta_j and of 32 theta_j, sin 2 theta_j and 1 - cos 2 theta_j (computed in
+// double precision; the last without cancellation).
+struct RopeTables {
+    unsigned long long phi[64];
+    float c1[64], s1[64], c32[64], s32[64], s2[64], h2[64];
+};
+void rope_tables(double base, int d, RopeTables *t);
+// The full-RoPE decode with the latent value sum on the tensor cores (units of one (sequence,
+// head) each, a separate merge kernel): the shapes with a kernel, its workspace, launch.  Its
+// workspace slots return to zero when a call completes.
+bool decode_rope_tc_supported(int es, int d, int r_k, int r_v);
+size_t decode_rope_tc_workspace_bytes(int r_v, int B, int H, int grid);
+lla_status launch_decode_rope_tc(const DecodeArgs &a, const RopeTables &t, int pairing, cudaStream_t stream);
 
 lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream);
 // The same encode for L layers (one launch for decode batches).
