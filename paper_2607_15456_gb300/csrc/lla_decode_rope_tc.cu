@@ -13,14 +13,15 @@
 //
 // Units are (sequence, head) pairs; their pages, in unit order, are cut into equal ranges, one per
 // CTA (lla_units.cuh), and a CTA takes its range as runs (its part of one unit).  Per CTA, 15 warps:
-//   warp 0       producer: per run, W_up,t^K of the run's head into an A slot (TMA boxes of 8
-//                columns x 128 rows, the no-swizzle K-major operand layout; the columns past r_k
-//                read as zero); per page, the K-plane by one bulk copy and the V-plane by TMA boxes
-//                with 128-byte swizzle
+//   warp 0       producer: per run, W_up,t^K of the run's head into the A slot once the previous
+//                run's key products have read it (TMA boxes of 8 columns x 128 rows, the
+//                no-swizzle K-major operand layout; the columns past r_k read as zero); per page,
+//                the K-plane by one bulk copy and the V-plane by TMA boxes with 128-byte swizzle
 //   warp 1       key issuer and TMEM owner: Khat^T (128 x 64) = W_up,t^K C_k^T per page into one of
 //                four 64-column accumulators (lane = key dimension, column = token)
 //   warp 2       value issuer: O^T (r_v x 16) += C_v^T P^T, with p as three bf16 parts (rows 0-2
-//                of P^T, 24 significant bits)
+//                of P^T, 24 significant bits); M = 128 latent rows per chunk, M = 64 for a last
+//                chunk of at most 64 rows (one V box fewer per stage)
 //   warps 3-6    rotation group 0 (even pages of the CTA), warps 7-10 group 1 (odd pages): lane m
 //                of a warp's TMEM quarter multiplies (khat_m,i + mu_m) by element m of
 //                rot(q, P - p_i), a sinusoid in i that starts from an exact phase per page (64-bit
@@ -68,11 +69,13 @@ struct ZR {
     static constexpr int RKX = (RK + 15) / 16 * 16;     // key contraction, zero-padded
     static constexpr int NG = RKX / 8;                  // 16-byte granules of a W_up row
     static constexpr int NCH = (RV + 127) / 128;        // 128-row chunks of O^T
+    // a last chunk of at most 64 latent rows is one box and an M = 64 product
+    static constexpr bool HALF = RV % 128 != 0 && RV % 128 <= 64;
     static constexpr int NBOX = (RV + 63) / 64;         // TMA boxes a V-plane loads
     static constexpr int BOX = kPT * 128;
     static constexpr int KPLANE = kPT * RK * 2;         // bytes of a K-plane copy
     static constexpr int KPAGE = kPT * RKX * 2;         // K stage: the copy, then zero granules
-    static constexpr int VPAGE = NCH * 2 * BOX;
+    static constexpr int VPAGE = (HALF ? 2 * NCH - 1 : 2 * NCH) * BOX;
     static constexpr int VBYTES = NBOX * BOX;
     static constexpr int ASLOT = 128 * RKX * 2;         // granule g of W_up row m at g*2048 + m*16
     static constexpr int PBUF = kPT * kNO * 2;
@@ -81,13 +84,13 @@ struct ZR {
     static constexpr int MISC = 64 * 4;                 // softmax maxima and sums
     static constexpr int PREF = (LLA_MAX_BATCH + 1 + 3) / 4 * 16;  // page prefix of the sequences
     static constexpr int NBAR = 56;
-    static constexpr int FIXED = 2 * ASLOT + 2 * PBUF + RED + 2 * QSLOT + MISC + PREF + NBAR * 8;
+    static constexpr int FIXED = ASLOT + 2 * PBUF + RED + 2 * QSLOT + MISC + PREF + NBAR * 8;
     static constexpr int ST0 = (kSmemCap - 1024 - FIXED) / (KPAGE + VPAGE);
     static constexpr int ST = ST0 > kMaxSt ? kMaxSt : ST0;
     static constexpr int oV = 0;
     static constexpr int oK = oV + ST * VPAGE;
     static constexpr int oA = oK + ST * KPAGE;
-    static constexpr int oP = oA + 2 * ASLOT;
+    static constexpr int oP = oA + ASLOT;
     static constexpr int oRed = oP + 2 * PBUF;
     static constexpr int oQ = oRed + RED;
     static constexpr int oMisc = oQ + 2 * QSLOT;
@@ -97,6 +100,7 @@ struct ZR {
     static constexpr uint32_t TM_O = kNAcc * 64, TM_COLS = 512;
     static constexpr uint32_t IDESC_K = umma_idesc_bf16(128, 64, 0, 0);
     static constexpr uint32_t IDESC_O = umma_idesc_bf16(128, kNO, 1, 0);
+    static constexpr uint32_t IDESC_O64 = umma_idesc_bf16(64, kNO, 1, 0);
     // a run partial: O^T ([RV]), the run maximum at RV and its sum at RV + 16
     static constexpr int PSTRIDE = RV + 32;
     static constexpr int PO_M = RV, PO_L = RV + 16;
@@ -109,7 +113,7 @@ struct ZR {
 
 // barrier indices
 enum {
-    bKfull = 0 /* [6] */, bKempty = 6, bVfull = 12, bVempty = 18, bAfull = 24 /* [2] */, bAfree = 26,
+    bKfull = 0 /* [6] */, bKempty = 6, bVfull = 12, bVempty = 18, bAfull = 24, bAfree = 26,
     bTfull = 28 /* [4] */, bTfree = 32, bSfull = 36 /* [4] */, bSfree = 40, bPfull = 44 /* [2] */,
     bPfree = 46, bOfree = 48, bQready = 49 /* [2] */, bQfree = 51, bAbort = 53, bTslot = 54
 };
@@ -238,9 +242,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&bar[bVfull + s], 1);
             mbar_init(&bar[bVempty + s], 1);
         }
+        mbar_init(&bar[bAfull], 1);
+        mbar_init(&bar[bAfree], 1);
         for (int s = 0; s < 2; ++s) {
-            mbar_init(&bar[bAfull + s], 1);
-            mbar_init(&bar[bAfree + s], 1);
             mbar_init(&bar[bPfull + s], 128);
             mbar_init(&bar[bPfree + s], 1);
             mbar_init(&bar[bQready + s], 128);
@@ -261,9 +265,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kWKey) tmem_alloc(tslot, Z::TM_COLS);
     // operand bytes that no copy writes stay zero: the V boxes past r_v of a last chunk, the K
     // granules past r_k, and the P^T rows past the three p parts
-    if constexpr (Z::NCH * 2 > Z::NBOX) {
+    if constexpr (Z::VPAGE > Z::VBYTES) {
         for (int s = 0; s < Z::ST; ++s)
-            for (int a = Z::NBOX; a < Z::NCH * 2; ++a)
+            for (int a = Z::NBOX; a < Z::VPAGE / Z::BOX; ++a)
                 for (int i = tid; i < Z::BOX / 16; i += kThreads)
                     reinterpret_cast<uint4 *>(sm + Z::oV + s * Z::VPAGE + a * Z::BOX)[i] = make_uint4(0, 0, 0, 0);
     }
@@ -295,13 +299,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             int itk = 0, itv = 0, ita = 0;
             bool stop = false;
             while (!stop && runs.next(rb, rh, pa, pe)) {
-                const int as = ita & 1;
-                if (!mbar_wait(&bar[bAfree + as], ((ita >> 1) & 1) ^ 1u, abort_flag, p.err) || *abort_flag) break;
-                mbar_arrive_expect_tx(&bar[bAfull + as], Z::ASLOT);
-                char *asl = sm + Z::oA + as * Z::ASLOT;
-                const int wrow = rh * p.T + p.loop;  // W_up,t^K of head rh: [H][T][d][r_k]
+                // W_up,t^K of head rh ([H][T][d][r_k]) once the previous run's key products have
+                // read the slot (the key accumulators keep the rotation groups busy meanwhile)
+                if (!mbar_wait(&bar[bAfree], (ita & 1) ^ 1u, abort_flag, p.err) || *abort_flag) break;
+                mbar_arrive_expect_tx(&bar[bAfull], Z::ASLOT);
+                const int wrow = rh * p.T + p.loop;
 #pragma unroll 1
-                for (int g = 0; g < Z::NG; ++g) tma_load_3d(asl + g * 2048, &tw, 8 * g, 0, wrow, &bar[bAfull + as]);
+                for (int g = 0; g < Z::NG; ++g) tma_load_3d(sm + Z::oA + g * 2048, &tw, 8 * g, 0, wrow, &bar[bAfull]);
                 ++ita;
                 const int32_t *bt = p.block_table + static_cast<int64_t>(rb) * p.max_blocks;
                 for (int pg = pa; pg < pe; ++pg) {
@@ -338,8 +342,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_wait(&bar[bKfull + j % Z::ST], (j / Z::ST) & 1, &never, p.err);
             for (int j = max(0, itv - Z::ST); j < itv; ++j)
                 mbar_wait(&bar[bVfull + j % Z::ST], (j / Z::ST) & 1, &never, p.err);
-            for (int j = max(0, ita - 2); j < ita; ++j)
-                mbar_wait(&bar[bAfull + (j & 1)], (j >> 1) & 1, &never, p.err);
+            if (ita > 0) mbar_wait(&bar[bAfull], (ita - 1) & 1, &never, p.err);
         }
         __syncwarp();
     } else if (warp == kWKey) {
@@ -347,10 +350,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             const uint32_t base = smem_addr(sm);
             int it = 0, r = 0;
+            const uint64_t da = umma_desc(base + Z::oA, 2048, 128);
             while (runs.next(rb, rh, pa, pe)) {
-                const int as = r & 1;
-                mbar_wait(&bar[bAfull + as], (r >> 1) & 1, abort_flag, p.err);
-                const uint64_t da = umma_desc(base + Z::oA + as * Z::ASLOT, 2048, 128);
+                mbar_wait(&bar[bAfull], r & 1, abort_flag, p.err);
                 for (int k = pa; k < pe; ++k, ++it) {
                     const int b = it % kNAcc, st = it % Z::ST;
                     mbar_wait(&bar[bKfull + st], (it / Z::ST) & 1, abort_flag, p.err);
@@ -363,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     umma_commit(&bar[bTfull + b]);
                     umma_commit(&bar[bKempty + st]);  // the K-plane has been read
                 }
-                umma_commit(&bar[bAfree + as]);
+                umma_commit(&bar[bAfree]);
                 ++r;
             }
             // the rotation groups wait for every key product before they finish
@@ -392,7 +394,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                         for (int ks = 0; ks < kPT / 16; ++ks)
                             umma_bf16(tmem + Z::TM_O + ch * kNO, dv + ((ch * 2 * Z::BOX + ks * 2048) >> 4),
-                                      dp + ks * ((2 * kNO * 16) >> 4), Z::IDESC_O, k > pa || ks > 0);
+                                      dp + ks * ((2 * kNO * 16) >> 4),
+                                      Z::HALF && ch == Z::NCH - 1 ? Z::IDESC_O64 : Z::IDESC_O, k > pa || ks > 0);
                     umma_commit(&bar[bVempty + st]);
                     umma_commit(&bar[bPfree + s]);  // also: O^T holds pages up to it
                 }
@@ -620,7 +623,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int ch = 0; ch < Z::NCH; ++ch) {
                 float o[kNO];
                 tmem_ld16(tlo + ch * kNO, o);
-                const int jj = ch * 128 + 32 * quarter + lane;
+                // an M = 128 chunk: row 32 quarter + lane; an M = 64 one: row 16 quarter + lane
+                // in lanes 0-15 of each quarter
+                const bool half = Z::HALF && ch == Z::NCH - 1;
+                const int jj = ch * 128 + (half ? (lane < 16 ? 16 * quarter + lane : RV) : 32 * quarter + lane);
                 if (jj < RV) dst[jj] = (o[0] + o[1]) + o[2];
             }
             tc_fence_before();
