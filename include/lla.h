@@ -236,8 +236,9 @@ typedef struct {
  * Every other argument, the workspace (lla_decode_workspace_size) and the error behaviour are
  * those of lla_decode_attn.  Keys are rebuilt on the tensor cores: storage must be LLA_BF16,
  * d = 128 and (r_k, r_v) one of (96, 160), (128, 128), (192, 320), (72, 120), else
- * LLA_ERR_UNSUPPORTED.  q, cur_k,
- * cur_v and out must be 16-byte aligned.
+ * LLA_ERR_UNSUPPORTED.  q, cur_k, cur_v and out must be 16-byte aligned.  For (96, 160),
+ * (128, 128) and (72, 120) the latent value sum also runs on the tensor cores (p as three bf16
+ * parts) and a second kernel on the stream merges the split runs; (192, 320) is one kernel.
  */
 lla_status lla_decode_attn_rope(const lla_geometry *g, const lla_codec *codec,
                                 const lla_cache *cache, const lla_rope *rope,

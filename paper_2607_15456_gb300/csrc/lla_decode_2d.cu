@@ -733,8 +733,8 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     constexpr bool kPre = RV <= 160;
     constexpr int NW = kPre ? RV / 8 : 1;
     __shared__ __align__(16) float ob[kFinishSeqs][RV];
-    __shared__ float wts[4][kMaxGrid];  // per warp: the run weights of its current unit
-    __shared__ float coef[kFinishSeqs][3];
+    __shared__ float wts[4][kMaxGrid], wls[4][kMaxGrid];  // per warp: run weights and sums
+    __shared__ float coef[kFinishSeqs][3], scs[kFinishSeqs];
     const int w = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(p.spb, p.B - b0);
@@ -751,6 +751,24 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
         for (int j8 = 0; j8 < NW; ++j8) wr[j8] = W[j8];
     }
     const float muv = p.mu_v ? p.mu_v[th * kD + e] : 0.f;
+    // the call's own inputs (not outputs of the earlier kernels) before the wait: each unit's
+    // current-token score and value element e
+    float cv[kFinishSeqs];
+#pragma unroll
+    for (int bi = 0; bi < kFinishSeqs; ++bi)
+        cv[bi] = p.cur_v && bi < nb ? load_elem(p.cur_v, iorow(b0 + bi) * kD + e, p.io_bf16) : 0.f;
+    if (p.cur_k) {
+        for (int bi = warp; bi < nb; bi += 4) {
+            const int64_t row = iorow(b0 + bi) * kD;
+            float qk = 0.f;
+#pragma unroll
+            for (int i = 0; i < kD / 32; ++i)
+                qk = fmaf(load_elem(p.q, row + lane + 32 * i, p.io_bf16), load_elem(p.cur_k, row + lane + 32 * i, p.io_bf16), qk);
+            qk = warp_sum(qk);
+            if (lane == 0) scs[bi] = qk * p.scale_log2;
+        }
+    }
+    __syncthreads();
     pdl_wait();
     const int NP = p.pstart[p.U];
     // G warps per unit (all four for one unit, two each for two): warp `sub` of a group takes
@@ -759,6 +777,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     const int grp = warp / G, sub = warp - grp * G;
     constexpr int NJ = (RV + 31) / 32;
     float *wt = wts[warp];
+    float *wl = wls[warp];
     for (int bi = grp; bi < kFinishSeqs; bi += 4 / G) {
         if (bi >= nb) {
             for (int j = lane + 32 * sub; j < RV; j += 32 * G) ob[bi][j] = 0.f;
@@ -766,14 +785,6 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
         }
         const int b = b0 + bi;
         const int u = p.loops ? b * p.H + h : b;
-        // pass 1: the current token's score against its exact key (loads issued first)
-        float qk = 0.f;
-        if (p.cur_k && sub == 0) {
-            const int64_t row = iorow(b) * kD;
-#pragma unroll
-            for (int i = 0; i < kD / 32; ++i)
-                qk = fmaf(load_elem(p.q, row + lane + 32 * i, p.io_bf16), load_elem(p.cur_k, row + lane + 32 * i, p.io_bf16), qk);
-        }
         const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
         float M = -INFINITY, l = 0.f;
         float acc[NJ];
@@ -785,17 +796,19 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
             const int c0 = cta_of(s0, NP, p.grid), c1 = cta_of(s1 - 1, NP, p.grid);
             const int nr = c1 - c0 + 1;
             const float *pu = p.part + static_cast<int64_t>(u + c0) * PS;
+            // the run maxima and sums in one round of loads
             float mm = -INFINITY;
             for (int i = lane; i < nr; i += 32) {
                 const bool has = page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid);
                 wt[i] = has ? pu[static_cast<int64_t>(i) * PS + PO_M + qn] : -INFINITY;
+                wl[i] = has ? pu[static_cast<int64_t>(i) * PS + PO_L + qn] : 0.f;
                 mm = fmaxf(mm, wt[i]);
             }
             M = warp_max(mm);
             float ls = 0.f;
             for (int i = lane; i < nr; i += 32) {
                 const float w8 = wt[i] == -INFINITY ? 0.f : ex2_approx(wt[i] - M);  // no run: 0
-                if (w8 > 0.f) ls = fmaf(w8, pu[static_cast<int64_t>(i) * PS + PO_L + qn], ls);
+                ls = fmaf(w8, wl[i], ls);
                 wt[i] = w8;
             }
             l = warp_sum(ls);
@@ -821,7 +834,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
             if (j < RV) ob[bi][j] = acc[q];
         }
         if (sub == 0) {
-            const float sc = p.cur_k ? warp_sum(qk) * p.scale_log2 : -INFINITY;
+            const float sc = p.cur_k ? scs[bi] : -INFINITY;
             if (lane == 0) {
                 const float Mx = fmaxf(M, sc);
                 const float al = M == -INFINITY ? 0.f : ex2_approx(M - Mx);
@@ -863,7 +876,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
         if (bi >= nb) break;
         const int64_t idx = iorow(b0 + bi) * kD + e;
         float v = acc[bi] * coef[bi][0] + coef[bi][1] * muv;
-        if (p.cur_v) v = fmaf(coef[bi][2], load_elem(p.cur_v, idx, p.io_bf16), v);
+        if (p.cur_v) v = fmaf(coef[bi][2], cv[bi], v);
         store_elem(p.out, idx, v, p.io_bf16);
     }
     __syncthreads();

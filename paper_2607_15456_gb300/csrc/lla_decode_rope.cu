@@ -12,6 +12,9 @@
 // rotation, so the value side stays in latent space as in lla_decode.cu:
 //   o = (W_up,t^V sum_i p_i c_v,i + (sum_i p_i) mu^V_t + p_cur v_cur) / (sum_i p_i + p_cur).
 //
+// This kernel serves (r_k, r_v) = (192, 320), whose 64 KB head pages and 48 KB W_up rows leave
+// no room for the tensor-core value path of lla_decode_rope_tc.cu (which serves the other shapes).
+//
 // GB300 mapping (one CTA per SM; the persistent split of (sequence, head, page) units over the
 // CTAs, the TMA ring, the split-KV merge and the output projection are shared with lla_decode.cu
 // through lla_decode_common.cuh):
@@ -495,10 +498,8 @@ struct RopeEntry {
 };
 RopeEntry rope_entry(int es, int d, int r_k, int r_v) {
     if (es != 2 || d != kRopeD) return RopeEntry{nullptr, nullptr};
-    if (r_k == 96 && r_v == 160) return RopeEntry{launch_rope<96, 160>, rope_layout_bytes<96, 160>};
-    if (r_k == 128 && r_v == 128) return RopeEntry{launch_rope<128, 128>, rope_layout_bytes<128, 128>};
+    // the other shapes run on the tensor-core value path (lla_decode_rope_tc.cu)
     if (r_k == 192 && r_v == 320) return RopeEntry{launch_rope<192, 320>, rope_layout_bytes<192, 320>};
-    if (r_k == 72 && r_v == 120) return RopeEntry{launch_rope<72, 120>, rope_layout_bytes<72, 120>};
     return RopeEntry{nullptr, nullptr};
 }
 

@@ -650,7 +650,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // Grid (H, ceil(B / spb)), 128 threads (thread e = output element e of head h).  spb (at most 8)
-// sequences share one pass over W_up,t^V of head h.  The runs of a unit are merged by one warp, or
+// sequences share one pass over W_up,t^V of head h.  Everything that is an input of the call (the
+// weights, the context lengths, q, k_cur and v_cur) is read before the wait on the attention
+// kernel, which launches this one ahead of its end.  The runs of a unit are merged by one warp, or
 // by two or four that split its columns when the CTA has fewer than three units; the merged slots
 // are then zeroed (each slot belongs to one unit, so to this CTA alone).
 template <int RV>
@@ -660,8 +662,8 @@ __global__ void __launch_bounds__(128, 1) rope_finish_kernel(const RFParams p) {
     constexpr int NW = kPre ? RV / 8 : 1;
     constexpr int NJ = (RV + 31) / 32;
     __shared__ __align__(16) float ob[kFinishSeqs][RV];
-    __shared__ float wts[4][kMaxGrid];
-    __shared__ float coef[kFinishSeqs][3];
+    __shared__ float wts[4][kMaxGrid], wls[4][kMaxGrid];  // per warp: run weights and sums
+    __shared__ float coef[kFinishSeqs][3], scs[kFinishSeqs];
     __shared__ int PB[LLA_MAX_BATCH + 1];
     const int h = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
@@ -675,12 +677,31 @@ __global__ void __launch_bounds__(128, 1) rope_finish_kernel(const RFParams p) {
         for (int j8 = 0; j8 < NW; ++j8) wr[j8] = W[j8];
     }
     const float muv = p.mu_v ? p.mu_v[th * kD + e] : 0.f;
-    pdl_wait();
+    // the call's own inputs (not outputs of the attention kernel) before the wait on it: the page
+    // prefix of the sequences, each unit's current-token score and value element e
     seq_prefix(p.context_lens, p.B, p.max_ctx, p.max_blocks, p.pass1, false, nullptr, PB);
+    float cv[kFinishSeqs];
+#pragma unroll
+    for (int bi = 0; bi < kFinishSeqs; ++bi)
+        cv[bi] = p.cur_v && bi < nb ? load_elem(p.cur_v, (static_cast<int64_t>(b0 + bi) * p.H + h) * kD + e, p.io_bf16) : 0.f;
+    if (p.cur_k) {
+        for (int bi = warp; bi < nb; bi += 4) {
+            const int64_t row = (static_cast<int64_t>(b0 + bi) * p.H + h) * kD;
+            float qk = 0.f;
+#pragma unroll
+            for (int i = 0; i < kD / 32; ++i)
+                qk = fmaf(load_elem(p.q, row + lane + 32 * i, p.io_bf16), load_elem(p.cur_k, row + lane + 32 * i, p.io_bf16), qk);
+            qk = warp_sum(qk);
+            if (lane == 0) scs[bi] = qk * p.scale_log2;
+        }
+    }
+    __syncthreads();
+    pdl_wait();
     const int NP = p.H * PB[p.B];
     const int G = nb == 1 ? 4 : nb == 2 ? 2 : 1;
     const int grp = warp / G, sub = warp - grp * G;
     float *wt = wts[warp];
+    float *wl = wls[warp];
     for (int bi = grp; bi < kFinishSeqs; bi += 4 / G) {
         if (bi >= nb) {
             for (int j = lane + 32 * sub; j < RV; j += 32 * G) ob[bi][j] = 0.f;
@@ -688,13 +709,6 @@ __global__ void __launch_bounds__(128, 1) rope_finish_kernel(const RFParams p) {
         }
         const int b = b0 + bi;
         const int64_t u = static_cast<int64_t>(b) * p.H + h;
-        float qk = 0.f;
-        if (p.cur_k && sub == 0) {
-            const int64_t row = u * kD;
-#pragma unroll
-            for (int i = 0; i < kD / 32; ++i)
-                qk = fmaf(load_elem(p.q, row + lane + 32 * i, p.io_bf16), load_elem(p.cur_k, row + lane + 32 * i, p.io_bf16), qk);
-        }
         const int P = PB[b + 1] - PB[b];
         const int s0 = p.H * PB[b] + h * P, s1 = s0 + P;
         float M = -INFINITY, l = 0.f;
@@ -705,17 +719,19 @@ __global__ void __launch_bounds__(128, 1) rope_finish_kernel(const RFParams p) {
             const int c0 = cta_of(s0, NP, p.grid), c1 = cta_of(s1 - 1, NP, p.grid);
             const int nr = c1 - c0 + 1;
             const float *pu = p.part + (u + c0) * PS;
+            // the run maxima and sums in one round of loads
             float mm = -INFINITY;
             for (int i = lane; i < nr; i += 32) {
                 const bool has = page_lo(c0 + i + 1, NP, p.grid) > page_lo(c0 + i, NP, p.grid);
                 wt[i] = has ? pu[static_cast<int64_t>(i) * PS + PO_M] : -INFINITY;
+                wl[i] = has ? pu[static_cast<int64_t>(i) * PS + PO_L] : 0.f;
                 mm = fmaxf(mm, wt[i]);
             }
             M = warp_max(mm);
             float ls = 0.f;
             for (int i = lane; i < nr; i += 32) {
                 const float w8 = wt[i] == -INFINITY ? 0.f : ex2_approx(wt[i] - M);
-                if (w8 > 0.f) ls = fmaf(w8, pu[static_cast<int64_t>(i) * PS + PO_L], ls);
+                ls = fmaf(w8, wl[i], ls);
                 wt[i] = w8;
             }
             l = warp_sum(ls);
@@ -739,18 +755,16 @@ __global__ void __launch_bounds__(128, 1) rope_finish_kernel(const RFParams p) {
             const int j = lane + 32 * (sub + G * q);
             if (j < RV) ob[bi][j] = acc[q];
         }
-        if (sub == 0) {
-            const float sc = p.cur_k ? warp_sum(qk) * p.scale_log2 : -INFINITY;
-            if (lane == 0) {
-                const float Mx = fmaxf(M, sc);
-                const float al = M == -INFINITY ? 0.f : ex2_approx(M - Mx);
-                const float pc = p.cur_k ? ex2_approx(sc - Mx) : 0.f;
-                const float den = al * l + pc;
-                const float inv = den > 0.f ? 1.f / den : 0.f;
-                coef[bi][0] = al * inv;
-                coef[bi][1] = al * l * inv;
-                coef[bi][2] = pc * inv;
-            }
+        if (sub == 0 && lane == 0) {
+            const float sc = p.cur_k ? scs[bi] : -INFINITY;
+            const float Mx = fmaxf(M, sc);
+            const float al = M == -INFINITY ? 0.f : ex2_approx(M - Mx);
+            const float pc = p.cur_k ? ex2_approx(sc - Mx) : 0.f;
+            const float den = al * l + pc;
+            const float inv = den > 0.f ? 1.f / den : 0.f;
+            coef[bi][0] = al * inv;
+            coef[bi][1] = al * l * inv;
+            coef[bi][2] = pc * inv;
         }
     }
     __syncthreads();  // every partial has been read
@@ -781,7 +795,7 @@ __global__ void __launch_bounds__(128, 1) rope_finish_kernel(const RFParams p) {
         if (bi >= nb) break;
         const int64_t idx = (static_cast<int64_t>(b0 + bi) * p.H + h) * kD + e;
         float v = acc[bi] * coef[bi][0] + coef[bi][1] * muv;
-        if (p.cur_v) v = fmaf(coef[bi][2], load_elem(p.cur_v, idx, p.io_bf16), v);
+        if (p.cur_v) v = fmaf(coef[bi][2], cv[bi], v);
         store_elem(p.out, idx, v, p.io_bf16);
     }
     // the merged slots return to zero
