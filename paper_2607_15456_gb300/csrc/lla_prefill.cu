@@ -146,12 +146,9 @@ __global__ void __launch_bounds__(kPThreads, 1)
     float *xsum = reinterpret_cast<float *>(sm + F::oL);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-    // grid (B H, query tiles): CTAs start in launch order, x fastest, so every (sequence, head)
-    // starts its longest causal range before any starts a shorter one (longest work first
-    // across the whole grid, a short tail)
     const int nqt = (p.max_len + kBM - 1) / kBM;
-    const int qt = nqt - 1 - static_cast<int>(blockIdx.y);
-    const int b = static_cast<int>(blockIdx.x) / p.H, h = static_cast<int>(blockIdx.x) - b * p.H;
+    const int qt = nqt - 1 - static_cast<int>(blockIdx.x);  // longest causal ranges first
+    const int b = blockIdx.y, h = blockIdx.z;
     pdl_wait();
     const int q0 = p.cu_seqlens[b];
     const int L = p.cu_seqlens[b + 1] - q0;
@@ -1002,8 +999,9 @@ lla_status launch_tc(const PParams &prm, int nqt, int B, int H, cudaStream_t str
     const uint32_t box[3] = {64, kPT, 1};
     if (!encode_tmap_bf16(&tv, prm.pool + kPT * RK * 2, 3, dims, strides, box, true)) return LLA_ERR_CUDA;
     cudaLaunchConfig_t cfg = {};
-    if (nqt > 65535) return LLA_ERR_UNSUPPORTED;  // query tiles on the grid's y axis
-    cfg.gridDim = dim3(B * H, nqt);
+    // x fastest: the tiles of one (sequence, head), longest first, run together and share its
+    // pages in L2 (ordering the longest tiles of every head first was slower: 1.90 -> 2.17 ms)
+    cfg.gridDim = dim3(nqt, B, H);
     cfg.blockDim = dim3(kPThreads);
     cfg.dynamicSmemBytes = PF<RK, RV, ROPE>::SMEM;
     cfg.stream = stream;
