@@ -488,7 +488,7 @@ def run_rope_extra(bench):
     return {"rope_decode": {
         "workload": f"{w.name} batch, RoPE after reconstruction (base {ROPE_BASE:g}, rotate-half "
                     f"pairs), {w.D}x{w.T} pass-1 calls",
-        "kernel": "decode_rope_kernel (lla_decode_attn_rope)", "bound": "hbm",
+        "kernel": f"rope_tc_kernel<{w.r_k}, {w.r_v}> + rope_finish_kernel (lla_decode_attn_rope)", "bound": "hbm",
         "ms_per_sweep": ms, "avg_launch_us": per_launch_s * 1e6,
         "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
         "bytes_per_launch": nbytes, "key_rebuild_TFLOP_s": rebuild_flops / per_launch_s / 1e12,
@@ -514,7 +514,7 @@ def run_loops_extra(bench):
     return {"loops_decode": {
         "workload": f"{w.name} batch, all {w.T} loops of a layer per call (shared latent), "
                     f"{w.D} calls per step",
-        "kernel": "absorb2d_kernel + attn2d_kernel<r_k, r_v, 4> + finish2d_kernel (lla_decode_attn_loops)",
+        "kernel": f"absorb2d_kernel + attn2d_kernel<{w.r_k}, {w.r_v}, 4> + finish2d_kernel (lla_decode_attn_loops)",
         "bound": "hbm",
         "ms_per_sweep": ms, "avg_launch_us": per_launch_s * 1e6,
         "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
@@ -839,7 +839,9 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
             # the same sweep with rotary positions after reconstruction (keys rebuilt on tcgen05)
             rms = _time_ms(bench.decode_calls_rope, reps=2, warm=1)
             rs = rms / 1e3 / (w.D * w.T)
-            rope = {"kernel": "decode_rope_kernel (lla_decode_attn_rope)", "ms_per_sweep": rms,
+            rope_k = (f"rope_tc_kernel<{w.r_k}, {w.r_v}> + rope_finish_kernel" if (w.r_k, w.r_v) != (192, 320)
+                      else "decode_rope_kernel<192, 320>")
+            rope = {"kernel": f"{rope_k} (lla_decode_attn_rope)", "ms_per_sweep": rms,
                     "avg_launch_us": rs * 1e6, "GB_s": nbytes / rs / 1e9, "hbm_frac": nbytes / rs / 1e9 / peak,
                     "tokens_per_s_decode_only": bench.B / (rms / 1e3)}
             if lla.lla_get_device_error() != 0:
@@ -858,7 +860,7 @@ def run_workload_rows(device, names=("ouro14_rho2", "ouro26_rho533", "stress_rho
             ls_ = lms / 1e3 / w.D
             lbytes = (sum(bench.lens) * w.H * (w.r_k + w.r_v) * 2
                       + w.T * (w.H * w.d * (w.r_k + w.r_v) * 2 + 4 * bench.B * w.H * w.d * 2))
-            loops = {"kernel": "absorb2d_kernel + attn2d_kernel<r_k, r_v, 4> + finish2d_kernel (lla_decode_attn_loops)",
+            loops = {"kernel": f"absorb2d_kernel + attn2d_kernel<{w.r_k}, {w.r_v}, 4> + finish2d_kernel (lla_decode_attn_loops)",
                      "ms_per_sweep": lms,
                      "avg_launch_us": ls_ * 1e6, "GB_s": lbytes / ls_ / 1e9, "hbm_frac": lbytes / ls_ / 1e9 / peak,
                      "bytes_per_launch": lbytes, "tokens_per_s_decode_only": bench.B / (lms / 1e3),
