@@ -530,21 +530,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int st_tid = tid - kWSmx * 32, quarter = warp & 3;
         const uint32_t tlo = tmem + (static_cast<uint32_t>(32 * quarter) << 16) + Z::TM_O;
         const int t = st_tid;  // the token of this thread (st_tid < 64)
-        int it = 0, r = 0;
-        while (runs.next(rb, rh, pa, pe)) {
-            const int qs = r & 1;
-            const int L = p.context_lens[rb];  // valid: the unit has pages
-            // q (scaled into the exp2 domain), mu^K and the query's position for the rotation
-            // groups, once both have left run r - 2
-            if (r >= 2) mbar_wait(&bar[bQfree + qs], ((r - 2) >> 1) & 1, abort_flag, p.err);
-            {
-                float *qv = reinterpret_cast<float *>(sm + Z::oQ + qs * Z::QSLOT);
-                const int64_t row = (static_cast<int64_t>(rb) * p.H + rh) * kD;
-                qv[st_tid] = load_elem(p.q, row + st_tid, p.io_bf16) * p.scale_log2;
-                qv[kD + st_tid] = p.mu_k ? p.mu_k[(static_cast<int64_t>(rh) * p.T + p.loop) * kD + st_tid] : 0.f;
-                if (st_tid == 0) reinterpret_cast<int *>(qv + 2 * kD)[0] = p.pass1 ? L : L - 1;
+        // q (scaled into the exp2 domain), mu^K and the query's position of a run, for the
+        // rotation groups, staged one run ahead so that they never wait for these loads
+        auto stage = [&](int qs, int b_, int h_) {
+            float *qv = reinterpret_cast<float *>(sm + Z::oQ + qs * Z::QSLOT);
+            const int64_t row = (static_cast<int64_t>(b_) * p.H + h_) * kD;
+            qv[st_tid] = load_elem(p.q, row + st_tid, p.io_bf16) * p.scale_log2;
+            qv[kD + st_tid] = p.mu_k ? p.mu_k[(static_cast<int64_t>(h_) * p.T + p.loop) * kD + st_tid] : 0.f;
+            if (st_tid == 0) {
+                const int Lq = p.context_lens[b_];  // the run has pages, so Lq >= 1
+                reinterpret_cast<int *>(qv + 2 * kD)[0] = p.pass1 ? Lq : Lq - 1;
             }
             mbar_arrive(&bar[bQready + qs]);
+        };
+        Runs ahead = runs;  // one run ahead of `runs`
+        int ab, ah, apa, ape;
+        if (ahead.next(ab, ah, apa, ape)) stage(0, ab, ah);
+        int it = 0, r = 0;
+        while (runs.next(rb, rh, pa, pe)) {
+            const int L = p.context_lens[rb];  // valid: the unit has pages
+            if (ahead.next(ab, ah, apa, ape)) {
+                // run r + 1 into the slot of run r - 1, once both rotation groups have left it
+                const int qs1 = (r + 1) & 1;
+                if (r >= 1) mbar_wait(&bar[bQfree + qs1], ((r - 1) >> 1) & 1, abort_flag, p.err);
+                stage(qs1, ab, ah);
+            }
             float m_run = -INFINITY, acc = 0.f;
             const int nps = pe - pa;
             for (int k = 0; k < nps; ++k, ++it) {
