@@ -62,8 +62,6 @@ constexpr float kRescaleLog2 = 8.f;  // rescale O^T only when a query's maximum 
 constexpr int kSmemCap = 227 * 1024;
 constexpr int kFinishSeqs = 8;   // most units per finish CTA
 constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one unit fit one finish CTA)
-constexpr int kSmSmem = 226 * 1024;      // shared memory of an SM, less two CTAs' reserve
-constexpr int kAbsorbSmem = 26 * 1024;   // the absorb kernel's static shared memory, rounded up
 
 // Shared-memory plan of the attention kernel for ranks (RK, RV) and NQ query slots per unit
 // (16: the heads of an LLA-2D sequence; 4: the loops of a per-head (sequence, head)).  Offsets
@@ -131,7 +129,6 @@ struct A2Params {
     int T, H, loop, io_bf16, pass1, B, max_ctx, max_blocks;
     int loops;           // 0: LLA-2D, 1: the loops of a per-head cache
     int hu;              // units per sequence
-    int early;           // trigger the attention kernel's launch right after the dependency wait
     float scale_log2;
     const void *w_up_k;  // LLA-2D [T][H][d][r_k], per-head [H][T][d][r_k]
     const float *mu_k;   // LLA-2D [T*H*d], per-head [H][T*d], or NULL
@@ -238,9 +235,6 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
 #pragma unroll
     for (int u = 0; u < 16; ++u) wv[u] = col < RK ? bf_to_f(W[(warp * 16 + u) * RK]) : 0.f;
     pdl_wait();  // the queries may come from the previous kernel; the workspace is free after it
-    // where an attention CTA fits beside this kernel's on an SM it may start its set-up now (it
-    // waits for this grid before reading q~); where it does not, an early start only staggers it
-    if (p.early) pdl_trigger();
     if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) page_prefix(p);
     for (int i = tid; i < 16 * kD; i += 256) {
         const int bi = i >> 7, e = i & (kD - 1);
@@ -273,10 +267,11 @@ __global__ void __launch_bounds__(256) absorb2d_kernel(const A2Params p) {
             if (lane == 0) p.beta[static_cast<int64_t>(unit(b0 + bi)) * NQ + n] = s * p.scale_log2;
         }
     }
-    if (!p.early) {
-        __syncthreads();
-        pdl_trigger();
-    }
+    // (triggering the attention kernel's launch right after the wait, so that its set-up could
+    // overlap this kernel where their CTAs fit one SM, gained 2 % at rho = 4 and lost 10 % on the
+    // Ouro-2.6B batch)
+    __syncthreads();
+    pdl_trigger();
 }
 
 // ------------------------------------------------------------------------- attention kernel
@@ -955,7 +950,6 @@ lla_status launch_units(const DecodeArgs &a, bool loops, cudaStream_t stream) {
     ap.T = a.T; ap.H = a.H; ap.loop = a.loop; ap.io_bf16 = a.io_bf16; ap.pass1 = a.cur_k != nullptr;
     ap.B = a.B; ap.max_ctx = a.max_ctx; ap.max_blocks = a.max_blocks;
     ap.loops = loops ? 1 : 0; ap.hu = hu;
-    ap.early = Z::SMEM + kAbsorbSmem <= kSmSmem ? 1 : 0;
     ap.scale_log2 = a.scale * kLog2e;
     ap.w_up_k = a.w_up_k; ap.mu_k = a.mu_k; ap.q = a.q; ap.context_lens = a.context_lens;
     ap.qt = reinterpret_cast<float *>(ws + w.qt);
