@@ -574,15 +574,16 @@ def run_2d_extra(device):
     for all heads, read by the H absorbed queries of each sequence on the tensor cores) on the
     stress workload's batch and contexts at the same cache budget, (r_k, r_v) = (288, 480),
     rho_2D = 21.33: two layers' caches of random bf16 latents, cycled through 2 x T pass-1 calls
-    (every call has the shape and bytes of a call of the 48-layer model), and the same 2D shape on
-    the headline batch of 16 sequences."""
+    (every call has the shape and bytes of a call of the 48-layer model), the same 2D shape on
+    the headline batch of 16 sequences, and (1152, 1920), rho_2D = 5.33, on the headline batch."""
     import torch
     from paper_2607_15456_gb300 import lla
     from paper_2607_15456_gb300 import workloads as W
     peak, _ = measured_peaks()
     out = {}
     for name, wname, B in (("lla2d_decode", "stress2d_rho2133", None),
-                           ("lla2d_decode_b16", "stress2d_rho2133", 16)):
+                           ("lla2d_decode_b16", "stress2d_rho2133", 16),
+                           ("lla2d_decode_rho533", "ouro14_2d_rho533", None)):
         w = W.WORKLOADS[wname]
         if B is not None:  # the headline batch's contexts with the 2D shape
             lens = W.context_lengths(W.WORKLOADS["ouro14_rho4"])
@@ -623,7 +624,8 @@ def run_2d_extra(device):
         out[name] = {
             "workload": f"LLA-2D, H={w.H}, (r_k, r_v)=({w.r_k}, {w.r_v}), rho_2D={w.rho:.2f}, "
                         f"B={B}, sum context {Nt}; 2 layers x {w.T} pass-1 calls",
-            "kernel": "absorb2d_kernel + attn2d_kernel + finish2d_kernel (lla_decode_attn_2d)",
+            "kernel": ("absorb2d_kernel + " + ("attn2d_big_kernel" if w.r_k > 512 else "attn2d_kernel")
+                       + " + finish2d_kernel (lla_decode_attn_2d)"),
             "bound": "hbm", "avg_call_us": per_launch_s * 1e6,
             "GB_s": nbytes / per_launch_s / 1e9, "hbm_frac": nbytes / per_launch_s / 1e9 / peak,
             "bytes_per_call": nbytes,

@@ -94,7 +94,8 @@ typedef struct {
     int32_t T;          /* loops (recurrence steps), 1..16 */
     int32_t H;          /* attention heads, >= 1 */
     int32_t d;          /* head width d_head: a multiple of 8, 8..256 */
-    int32_t r_k, r_v;   /* latent ranks, 2..512; even for bf16 storage */
+    int32_t r_k, r_v;   /* latent ranks, 2..512 (LLA-2D entry points: 2..2048 and at most T H d);
+                           even for bf16 storage */
     int32_t block_size; /* tokens per cache block: must be LLA_BLOCK_TOKENS */
     lla_dtype storage;  /* dtype of the latents and of the codec weights */
     float scale;        /* softmax scale applied to q . k (e.g. 1/sqrt(d)) */
@@ -315,7 +316,8 @@ lla_status lla_decode_2d_workspace_size(const lla_geometry *g, int32_t B, size_t
  *                         fill needed); calls that share it must be ordered (one stream)
  * Other arguments and the error behaviour are those of lla_decode_attn.  Three launches on
  * `stream`.  Storage LLA_BF16, d = 128, H <= 16, (r_k, r_v) one of (96, 160), (128, 128),
- * (288, 480); LLA_ERR_UNSUPPORTED otherwise.
+ * (288, 480), (1152, 1920) (rho_2D = 5.33: its 384 KB pages stream through the attention kernel in
+ * column chunks of the K-plane and row chunks of the V-plane); LLA_ERR_UNSUPPORTED otherwise.
  */
 lla_status lla_decode_attn_2d(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
                               const int32_t *context_lens, int32_t B, int32_t max_ctx,

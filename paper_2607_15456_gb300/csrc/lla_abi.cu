@@ -24,11 +24,17 @@ int elem_size(lla_dtype t) { return t == LLA_BF16 ? 2 : 4; }
 
 bool valid_dtype(lla_dtype t) { return t == LLA_BF16 || t == LLA_F32; }
 
-lla_status check_geometry(const lla_geometry *g) {
+// max_rank: 512 for the per-head cache; the LLA-2D entry points take latents as wide as the H
+// per-head latents together (kMaxRank2D, and at most T H d, the width of the stacked vector)
+constexpr int kMaxRank = 512, kMaxRank2D = 2048;
+lla_status check_geometry(const lla_geometry *g, int max_rank = kMaxRank) {
     if (!g) return LLA_ERR_INVALID_ARG;
     if (g->T < 1 || g->T > 16 || g->H < 1 || g->H > 4096) return LLA_ERR_INVALID_ARG;
     if (g->d < 8 || g->d > 256 || (g->d % 8) != 0) return LLA_ERR_INVALID_ARG;
-    if (g->r_k < 2 || g->r_v < 2 || g->r_k > 512 || g->r_v > 512) return LLA_ERR_INVALID_ARG;
+    if (g->r_k < 2 || g->r_v < 2 || g->r_k > max_rank || g->r_v > max_rank) return LLA_ERR_INVALID_ARG;
+    if (max_rank > kMaxRank && (static_cast<int64_t>(g->r_k) > static_cast<int64_t>(g->T) * g->H * g->d ||
+                                static_cast<int64_t>(g->r_v) > static_cast<int64_t>(g->T) * g->H * g->d))
+        return LLA_ERR_INVALID_ARG;
     if ((g->r_k % 2) != 0 || (g->r_v % 2) != 0) return LLA_ERR_INVALID_ARG;
     if (g->block_size != LLA_BLOCK_TOKENS) return LLA_ERR_UNSUPPORTED;
     if (!valid_dtype(g->storage)) return LLA_ERR_INVALID_ARG;
@@ -302,7 +308,7 @@ lla_status lla_decode_attn_loops(const lla_geometry *g, const lla_codec *codec,
 }
 
 lla_status lla_cache_2d_block_bytes(const lla_geometry *g, size_t *bytes) {
-    lla_status st = check_geometry(g);
+    lla_status st = check_geometry(g, kMaxRank2D);
     if (st != LLA_OK) return st;
     if (!bytes) return LLA_ERR_INVALID_ARG;
     *bytes = head_page_bytes(g->r_k, g->r_v, elem_size(g->storage));  // one page per block
@@ -312,7 +318,7 @@ lla_status lla_cache_2d_block_bytes(const lla_geometry *g, size_t *bytes) {
 lla_status lla_encode_2d(const lla_geometry *g, const lla_codec *codec, const lla_cache *cache,
                          const void *x_k, const void *x_v, lla_dtype x_dtype,
                          const int64_t *slot_mapping, int32_t N, void *stream) {
-    lla_status st = check_geometry(g);
+    lla_status st = check_geometry(g, kMaxRank2D);
     if (st != LLA_OK) return st;
     if (!codec || !codec->w_down_k || !codec->w_down_v) return LLA_ERR_INVALID_ARG;
     if ((st = check_cache(cache, false)) != LLA_OK) return st;
@@ -339,7 +345,7 @@ lla_status lla_encode_2d(const lla_geometry *g, const lla_codec *codec, const ll
 }
 
 lla_status lla_decode_2d_workspace_size(const lla_geometry *g, int32_t B, size_t *bytes) {
-    lla_status st = check_geometry(g);
+    lla_status st = check_geometry(g, kMaxRank2D);
     if (st != LLA_OK) return st;
     if (!bytes || B < 0 || B > LLA_MAX_BATCH) return LLA_ERR_INVALID_ARG;
     if (!decode_2d_supported(elem_size(g->storage), g->d, g->H, g->r_k, g->r_v))
@@ -355,7 +361,7 @@ lla_status lla_decode_attn_2d(const lla_geometry *g, const lla_codec *codec, con
                               int32_t loop, const void *q, const void *cur_k, const void *cur_v,
                               lla_dtype io_dtype, void *out, void *workspace,
                               size_t workspace_bytes, void *stream) {
-    lla_status st = check_geometry(g);
+    lla_status st = check_geometry(g, kMaxRank2D);
     if (st != LLA_OK) return st;
     if ((st = check_cache(cache, true)) != LLA_OK) return st;
     if (!codec || !codec->w_up_k || !codec->w_up_v) return LLA_ERR_INVALID_ARG;

@@ -60,8 +60,10 @@ constexpr int kPvWarp = 6;       // issuer of the O^T products
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;  // rescale O^T only when a query's maximum grows by more
 constexpr int kSmemCap = 227 * 1024;
-constexpr int kFinishSeqs = 8;   // most units per finish CTA
-constexpr int kMaxGrid = 1024;   // attention CTAs (the runs of one unit fit one finish CTA)
+constexpr int kFinishSeqs = 8;   // most units per finish CTA (4 for latents wider than 512)
+constexpr int kMaxGrid = 256;    // attention CTAs (the runs of one unit fit one finish CTA)
+
+__host__ __device__ constexpr int finish_seqs(int rv) { return rv > 512 ? 4 : kFinishSeqs; }
 
 // Shared-memory plan of the attention kernel for ranks (RK, RV) and NQ query slots per unit
 // (16: the heads of an LLA-2D sequence; 4: the loops of a per-head (sequence, head)).  Offsets
@@ -720,6 +722,443 @@ __global__ void __launch_bounds__(kT2, 1)
     }
 }
 
+// ---------------------------------------------------------------- attention, large latents
+
+// LLA-2D latents too wide for a whole page per pipeline stage ((1152, 1920): a 384 KB page).  A
+// page streams through two rings: its K-plane as KC column chunks (each a contiguous run of
+// granules, one bulk copy), accumulated into S^T chunk by chunk, and its V-plane as 128-row
+// chunks (two 64-column TMA boxes each), each feeding one 16-column O^T accumulator.  Warps:
+//   0     K producer                    1     S^T issuer and TMEM owner
+//   2-5   softmax (as attn2d_kernel)    6     O^T issuer
+//   7     V producer: it also zeroes, once a chunk of a run's partial last page has landed, the
+//         rows past the sequence (0 * NaN would poison O^T), and only then hands the chunk to the
+//         O^T issuer; the hand-over trails the copies by VST - 1 chunks
+template <int RK, int RV>
+struct ZB {
+    static constexpr int NS = 2 * kNQ;
+    static constexpr int RKC = 288;                    // K chunk columns
+    static constexpr int KC = RK / RKC;
+    static constexpr int KCB = kPT * RKC * 2;          // bytes of a K chunk (36 KB)
+    static constexpr int VC = RV / 128;                // 128-row V chunks
+    static constexpr int BOX = kPT * 128;
+    static constexpr int VCB = 2 * BOX;                // bytes of a V chunk (16 KB)
+    static constexpr int KST = 2, VST = 4;
+    static constexpr int QB = NS * RK * 2;             // [Q~_hi; Q~_lo] operand (72 KB)
+    static constexpr int PBUF = kPT * kNQ * 2;
+    static constexpr int RED = 1024;
+    static constexpr int NBAR = 42;
+    static constexpr int oV = 0;                       // 1024-byte aligned (128-byte swizzle)
+    static constexpr int oK = oV + VST * VCB;
+    static constexpr int oQ = oK + KST * KCB;
+    static constexpr int oP = oQ + QB;
+    static constexpr int oRed = oP + 2 * PBUF;
+    static constexpr int oBar = oRed + RED;
+    static constexpr int SMEM = 1024 + oBar + NBAR * 8;
+    static constexpr uint32_t TM_S = 0, TM_O = 2 * NS, TM_COLS = 512;
+    static constexpr uint32_t IDESC_S = umma_idesc_bf16(64, NS, 0, 0);
+    static constexpr uint32_t IDESC_O = umma_idesc_bf16(128, kNQ, 1, 0);
+    static constexpr int PSTRIDE = kNQ * RV + 2 * kNQ;
+    static constexpr int PO_M = kNQ * RV, PO_L = kNQ * RV + kNQ;
+    static_assert(RK % RKC == 0 && RV % 128 == 0, "chunks");
+    static_assert(SMEM <= kSmemCap, "shared memory");
+    static_assert(TM_O + VC * kNQ <= TM_COLS, "TMEM columns");
+    static_assert(VST >= 2 && KST >= 2 && VST <= 8, "ring depths");
+};
+
+// barrier indices of the large-latent kernel
+enum {
+    cKfull = 0 /* [2] */, cKempty = 2, cVfull = 4 /* [8] */, cVok = 12, cVempty = 20,
+    cSfull = 28 /* [2] */, cSfree = 30, cPfull = 32, cPfree = 34, cOfree = 36, cQready = 37,
+    cQfree = 38, cAbort = 39, cTslot = 40
+};
+
+template <int RK, int RV>
+__global__ void __launch_bounds__(256, 1)
+    attn2d_big_kernel(const __grid_constant__ CUtensorMap tv, const T2Params p) {
+    using Z = ZB<RK, RV>;
+    extern __shared__ __align__(1024) char sm_raw[];
+    char *sm = reinterpret_cast<char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + Z::oBar);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar + cAbort);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + cTslot);
+    float *red = reinterpret_cast<float *>(sm + Z::oRed);  // [2 pages][4 warps][16] maxima
+    float *lsum = red + 128;                                // [4 warps][16] run sums
+    float *betas = lsum + 64;                               // [16]
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int G = gridDim.x, c = blockIdx.x;
+
+    if (tid == 0) {
+        for (int s = 0; s < Z::KST; ++s) {
+            mbar_init(&bar[cKfull + s], 1);
+            mbar_init(&bar[cKempty + s], 1);
+        }
+        for (int s = 0; s < Z::VST; ++s) {
+            mbar_init(&bar[cVfull + s], 1);
+            mbar_init(&bar[cVok + s], 1);
+            mbar_init(&bar[cVempty + s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&bar[cSfull + s], 1);
+            mbar_init(&bar[cSfree + s], 128);
+            mbar_init(&bar[cPfull + s], 128);
+            mbar_init(&bar[cPfree + s], 1);
+        }
+        mbar_init(&bar[cOfree], 128);
+        mbar_init(&bar[cQready], 128);
+        mbar_init(&bar[cQfree], 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) tmem_alloc(tslot, Z::TM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+    pdl_wait();  // q~, beta and the page prefix sums come from the absorb kernel
+
+    const int NP = p.pstart[p.U];
+    const int g0 = page_lo(c, NP, G), g1 = page_lo(c + 1, NP, G);
+    const int ufirst = g0 < g1 ? first_unit(p.pstart, p.U, g0) : p.U;
+
+    if (warp == 0) {
+        // ----------------------------------------------------------------------- K producer
+        if (lane == 0) {
+            const uint64_t pol = policy_evict_first();
+            int itk = 0;
+            bool stop = false;
+            for (int u = ufirst; u < p.U && !stop; ++u) {
+                const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
+                if (s0 >= g1) break;
+                const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
+                const int32_t *bt = p.block_table + static_cast<int64_t>(u) * p.max_blocks;
+                for (int pg = pa; pg < pe && !stop; ++pg) {
+                    int32_t blk = bt[pg];
+                    if (blk < 0 || blk >= p.num_blocks) {
+                        atomicOr(p.err, LLA_DEVERR_BLOCK_ID);
+                        blk = 0;
+                    }
+                    const char *src = p.pool + static_cast<int64_t>(blk) * p.page_bytes;
+                    for (int kc = 0; kc < Z::KC; ++kc) {
+                        const int st = itk % Z::KST;
+                        if (!mbar_wait(&bar[cKempty + st], ((itk / Z::KST) & 1) ^ 1u, abort_flag, p.err) || *abort_flag) {
+                            stop = true;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(&bar[cKfull + st], Z::KCB);
+                        bulk_g2s(sm + Z::oK + st * Z::KCB, src + kc * Z::KCB, Z::KCB, &bar[cKfull + st], pol);
+                        ++itk;
+                    }
+                }
+            }
+            volatile int never = 0;
+            for (int j = max(0, itk - Z::KST); j < itk; ++j)
+                mbar_wait(&bar[cKfull + j % Z::KST], (j / Z::KST) & 1, &never, p.err);
+        }
+        __syncwarp();
+    } else if (warp == 7) {
+        // ---------------------------------------------------------- V producer and hand-over
+        int itv = 0, handed = 0;
+        int nvs[Z::VST];  // per stage: valid rows of its chunk (64: nothing to zero)
+#pragma unroll
+        for (int i = 0; i < Z::VST; ++i) nvs[i] = kPT;
+        // chunk j has landed: zero its rows past the sequence, then pass it to the O^T issuer
+        auto hand_over = [&](int j) {
+            const int st = j % Z::VST;
+            volatile int never = 0;
+            mbar_wait(&bar[cVfull + st], (j / Z::VST) & 1, &never, p.err);
+            int nv = kPT;
+#pragma unroll
+            for (int i = 0; i < Z::VST; ++i)
+                if (i == st) nv = nvs[i];
+            if (nv < kPT) {
+                char *vs = sm + Z::oV + st * Z::VCB;
+                for (int w = lane; w < (kPT - nv) * 2 * 8; w += 32) {
+                    const int cc = w & 7, r2 = w >> 3;
+                    const int a = r2 & 1, row = nv + (r2 >> 1);
+                    *reinterpret_cast<uint4 *>(vs + a * Z::BOX + row * 128 + cc * 16) = make_uint4(0, 0, 0, 0);
+                }
+                fence_proxy_async_smem();
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar[cVok + st]);
+        };
+        bool stop = false;
+        for (int u = ufirst; u < p.U && !stop; ++u) {
+            const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
+            if (s0 >= g1) break;
+            const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
+            const int L = p.context_lens[u];
+            const int32_t *bt = p.block_table + static_cast<int64_t>(u) * p.max_blocks;
+            for (int pg = pa; pg < pe && !stop; ++pg) {
+                int32_t blk = bt[pg];
+                if (blk < 0 || blk >= p.num_blocks) blk = 0;  // flagged by the K producer
+                const int nv = min(kPT, L - pg * kPT);
+                for (int vc = 0; vc < Z::VC; ++vc) {
+                    const int st = itv % Z::VST;
+                    bool ok = true;
+                    if (lane == 0)
+                        ok = mbar_wait(&bar[cVempty + st], ((itv / Z::VST) & 1) ^ 1u, abort_flag, p.err) && !*abort_flag;
+                    ok = __shfl_sync(0xffffffffu, ok, 0);
+                    if (!ok) {
+                        stop = true;
+                        break;
+                    }
+#pragma unroll
+                    for (int i = 0; i < Z::VST; ++i)
+                        if (i == st) nvs[i] = nv;
+                    if (lane == 0) {
+                        mbar_arrive_expect_tx(&bar[cVfull + st], Z::VCB);
+                        char *vs = sm + Z::oV + st * Z::VCB;
+                        tma_load_3d(vs, &tv, (2 * vc) * 64, 0, blk, &bar[cVfull + st]);
+                        tma_load_3d(vs + Z::BOX, &tv, (2 * vc + 1) * 64, 0, blk, &bar[cVfull + st]);
+                    }
+                    ++itv;
+                    if (itv - handed >= Z::VST) hand_over(handed++);
+                }
+            }
+        }
+        while (handed < itv) hand_over(handed++);  // also drains every copy after an abort
+    } else if (warp == 1) {
+        // ----------------------------------------------------------------------- S^T issuer
+        if (lane == 0) {
+            const uint32_t base = smem_addr(sm);
+            const uint64_t dq = umma_desc(base + Z::oQ, Z::NS * 16, 128);
+            int it = 0, itk = 0, r = 0;
+            for (int u = ufirst; u < p.U; ++u) {
+                const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
+                if (s0 >= g1) break;
+                const int n = min(g1, s1) - max(g0, s0);
+                if (n <= 0) continue;
+                mbar_wait(&bar[cQready], r & 1, abort_flag, p.err);
+                tc_fence_after();
+                for (int k = 0; k < n; ++k, ++it) {
+                    const int s = it & 1;
+                    if (it >= 2) mbar_wait(&bar[cSfree + s], ((it - 2) >> 1) & 1, abort_flag, p.err);
+                    for (int kc = 0; kc < Z::KC; ++kc, ++itk) {
+                        const int st = itk % Z::KST;
+                        mbar_wait(&bar[cKfull + st], (itk / Z::KST) & 1, abort_flag, p.err);
+                        tc_fence_after();
+                        const uint64_t dk = umma_desc(base + Z::oK + st * Z::KCB, kPT * 16, 128);
+#pragma unroll 6
+                        for (int ks = 0; ks < Z::RKC / 16; ++ks)
+                            umma_bf16(tmem + Z::TM_S + s * Z::NS, dk + ks * ((2 * kPT * 16) >> 4),
+                                      dq + (kc * (Z::RKC / 8) + 2 * ks) * ((Z::NS * 16) >> 4), Z::IDESC_S,
+                                      kc > 0 || ks > 0);
+                        umma_commit(&bar[cKempty + st]);
+                    }
+                    umma_commit(&bar[cSfull + s]);
+                    if (k == n - 1) umma_commit(&bar[cQfree]);
+                }
+                ++r;
+            }
+        }
+        __syncwarp();
+    } else if (warp == 6) {
+        // ----------------------------------------------------------------------- O^T issuer
+        if (lane == 0) {
+            const uint32_t base = smem_addr(sm);
+            const uint64_t dp0 = umma_desc(base + Z::oP, kNQ * 16, 128);
+            int it = 0, itv = 0, r = 0;
+            for (int u = ufirst; u < p.U; ++u) {
+                const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
+                if (s0 >= g1) break;
+                const int n = min(g1, s1) - max(g0, s0);
+                if (n <= 0) continue;
+                for (int k = 0; k < n; ++k, ++it) {
+                    const int s = it & 1;
+                    mbar_wait(&bar[cPfull + s], (it >> 1) & 1, abort_flag, p.err);
+                    if (k == 0 && r > 0) mbar_wait(&bar[cOfree], (r - 1) & 1, abort_flag, p.err);
+                    const uint64_t dp = dp0 + static_cast<uint64_t>((s * Z::PBUF) >> 4);
+                    for (int vc = 0; vc < Z::VC; ++vc, ++itv) {
+                        const int st = itv % Z::VST;
+                        mbar_wait(&bar[cVok + st], (itv / Z::VST) & 1, abort_flag, p.err);
+                        tc_fence_after();
+                        const uint64_t dv = umma_desc_sw128_mn(base + Z::oV + st * Z::VCB, Z::BOX);
+#pragma unroll
+                        for (int ks = 0; ks < kPT / 16; ++ks)
+                            umma_bf16(tmem + Z::TM_O + vc * kNQ, dv + ((ks * 2048) >> 4),
+                                      dp + ks * ((2 * kNQ * 16) >> 4), Z::IDESC_O, k > 0 || ks > 0);
+                        umma_commit(&bar[cVempty + st]);
+                    }
+                    umma_commit(&bar[cPfree + s]);  // also: O^T holds pages up to it
+                }
+                ++r;
+            }
+            if (it > 0) {
+                volatile int never = 0;
+                mbar_wait(&bar[cPfree + ((it - 1) & 1)], ((it - 1) >> 1) & 1, &never, p.err);
+            }
+        }
+        __syncwarp();
+    } else {
+        // --------------------------------------------------------------- softmax warps 2-5
+        const int q4 = warp & 3;
+        const uint32_t tl = tmem + (static_cast<uint32_t>(32 * q4) << 16);
+        const int st_tid = tid - kSm0;
+        const int tok = 16 * q4 + lane;
+        int it = 0, r = 0;
+        for (int u = ufirst; u < p.U; ++u) {
+            const int s0 = p.pstart[u], s1 = p.pstart[u + 1];
+            if (s0 >= g1) break;
+            const int pa = max(g0, s0) - s0, pe = min(g1, s1) - s0;
+            if (pe <= pa) continue;
+            const int L = p.context_lens[u];
+            if (r > 0) mbar_wait(&bar[cQfree], (r - 1) & 1, abort_flag, p.err);
+            {
+                const float4 *src = reinterpret_cast<const float4 *>(p.qt + static_cast<int64_t>(u) * kNQ * RK);
+                for (int i = st_tid; i < kNQ * (RK / 8); i += 128) {
+                    const int n = i / (RK / 8), g = i - n * (RK / 8);
+                    uint4 hi = make_uint4(0, 0, 0, 0), lo = hi;
+                    if (n < p.nq) {
+                        const float4 a = src[2 * i], c4 = src[2 * i + 1];
+                        const float v[8] = {a.x, a.y, a.z, a.w, c4.x, c4.y, c4.z, c4.w};
+                        float r8[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) r8[e] = v[e] - __bfloat162float(__float2bfloat16_rn(v[e]));
+                        hi = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                        pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+                        lo = make_uint4(pack_bf16x2(r8[0], r8[1]), pack_bf16x2(r8[2], r8[3]),
+                                        pack_bf16x2(r8[4], r8[5]), pack_bf16x2(r8[6], r8[7]));
+                    }
+                    char *dq = sm + Z::oQ + g * (Z::NS * 16);
+                    *reinterpret_cast<uint4 *>(dq + n * 16) = hi;
+                    *reinterpret_cast<uint4 *>(dq + (kNQ + n) * 16) = lo;
+                }
+                if (st_tid < kNQ) betas[st_tid] = st_tid < p.nq ? p.beta[static_cast<int64_t>(u) * kNQ + st_tid] : 0.f;
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(&bar[cQready]);
+            named_bar_sync(1, 128);
+            float m[kNQ], acc[kNQ];
+#pragma unroll
+            for (int n = 0; n < kNQ; ++n) {
+                m[n] = -INFINITY;
+                acc[n] = 0.f;
+            }
+            const int nps = pe - pa;
+            for (int k = 0; k < nps; ++k, ++it) {
+                const int s = it & 1;
+                const int tok0 = (pa + k) * kPT;
+                mbar_wait(&bar[cSfull + s], (it >> 1) & 1, abort_flag, p.err);
+                tc_fence_after();
+                float x2[Z::NS], x[kNQ];
+                tmem_ld32(tl + Z::TM_S + s * Z::NS, x2);
+                tc_fence_before();
+                mbar_arrive(&bar[cSfree + s]);
+                const bool valid = lane < 16 && tok0 + tok < L;
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) x[n] = valid ? (x2[n] + x2[kNQ + n]) + betas[n] : -INFINITY;
+                float mx[kNQ];
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) mx[n] = x[n];
+#pragma unroll
+                for (int o = 8; o >= 1; o >>= 1)
+#pragma unroll
+                    for (int n = 0; n < kNQ; ++n) mx[n] = fmaxf(mx[n], __shfl_xor_sync(0xffffffffu, mx[n], o));
+                float *rp = red + s * 64;
+                if (lane == 0) {
+#pragma unroll
+                    for (int n = 0; n < kNQ; n += 4)
+                        *reinterpret_cast<float4 *>(rp + q4 * 16 + n) = make_float4(mx[n], mx[n + 1], mx[n + 2], mx[n + 3]);
+                }
+                named_bar_sync(1, 128);
+                bool any = false;
+                float f[kNQ];
+#pragma unroll
+                for (int n = 0; n < kNQ; n += 4) {
+                    float4 a = *reinterpret_cast<const float4 *>(rp + n);
+#pragma unroll
+                    for (int w = 1; w < 4; ++w) {
+                        const float4 bb = *reinterpret_cast<const float4 *>(rp + w * 16 + n);
+                        a = make_float4(fmaxf(a.x, bb.x), fmaxf(a.y, bb.y), fmaxf(a.z, bb.z), fmaxf(a.w, bb.w));
+                    }
+                    const float pm[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float mn = fmaxf(m[n + e], pm[e]);
+                        const bool need = mn > m[n + e] + kRescaleLog2;
+                        f[n + e] = need ? ex2_approx(m[n + e] - mn) : 1.f;
+                        if (need) {
+                            acc[n + e] *= f[n + e];
+                            m[n + e] = mn;
+                            any = true;
+                        }
+                    }
+                }
+                if (any && k > 0) {
+                    mbar_wait(&bar[cPfree + ((it - 1) & 1)], ((it - 1) >> 1) & 1, abort_flag, p.err);
+                    tc_fence_after();
+#pragma unroll 1
+                    for (int ch = 0; ch < Z::VC; ++ch) {
+                        float o[kNQ];
+                        tmem_ld16(tl + Z::TM_O + ch * kNQ, o);
+#pragma unroll
+                        for (int n = 0; n < kNQ; ++n) o[n] *= f[n];
+                        tmem_st16(tl + Z::TM_O + ch * kNQ, o);
+                    }
+                }
+                float pv[kNQ];
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) {
+                    pv[n] = ex2_approx(x[n] - m[n]);
+                    acc[n] += pv[n];
+                }
+                if (it >= 2) mbar_wait(&bar[cPfree + s], ((it - 2) >> 1) & 1, abort_flag, p.err);
+                if (lane < 16) {
+                    char *pp = sm + Z::oP + s * Z::PBUF + (tok >> 3) * (kNQ * 16) + (tok & 7) * 2;
+#pragma unroll
+                    for (int n = 0; n < kNQ; ++n)
+                        *reinterpret_cast<uint16_t *>(pp + n * 16) = __bfloat16_as_ushort(__float2bfloat16_rn(pv[n]));
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                mbar_arrive(&bar[cPfull + s]);
+            }
+            mbar_wait(&bar[cPfree + ((it - 1) & 1)], ((it - 1) >> 1) & 1, abort_flag, p.err);
+            tc_fence_after();
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1)
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n) acc[n] += __shfl_xor_sync(0xffffffffu, acc[n], o);
+            if (lane == 0) {
+#pragma unroll
+                for (int n = 0; n < kNQ; n += 4)
+                    *reinterpret_cast<float4 *>(lsum + q4 * 16 + n) = make_float4(acc[n], acc[n + 1], acc[n + 2], acc[n + 3]);
+            }
+            float *dst = p.part + static_cast<int64_t>(u + c) * Z::PSTRIDE;
+#pragma unroll 1
+            for (int ch = 0; ch < Z::VC; ++ch) {
+                float o[kNQ];
+                tmem_ld16(tl + Z::TM_O + ch * kNQ, o);
+                const int j = ch * 128 + 32 * q4 + lane;
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n)
+                    if (n < p.nq) dst[n * RV + j] = o[n];
+            }
+            tc_fence_before();
+            mbar_arrive(&bar[cOfree]);
+            named_bar_sync(1, 128);
+            if (st_tid < kNQ) {
+                float mine = 0.f;
+#pragma unroll
+                for (int n = 0; n < kNQ; ++n)
+                    if (st_tid == n) mine = m[n];
+                dst[Z::PO_M + st_tid] = mine;
+                dst[Z::PO_L + st_tid] = (lsum[st_tid] + lsum[16 + st_tid]) + (lsum[32 + st_tid] + lsum[48 + st_tid]);
+            }
+            named_bar_sync(1, 128);
+            ++r;
+        }
+    }
+    pdl_trigger();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, Z::TM_COLS);
+    }
+}
+
 // ------------------------------------------------------------------------- finish kernel
 
 // Grid (weight slices, ceil(B / spb)), 128 threads (thread e = output element e).  spb (at most
@@ -734,10 +1173,11 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     constexpr int PS = NQM * RV + 2 * kNQ;
     constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
     constexpr bool kPre = RV <= 160;
+    constexpr int SPB = finish_seqs(RV);
     constexpr int NW = kPre ? RV / 8 : 1;
-    __shared__ __align__(16) float ob[kFinishSeqs][RV];
+    __shared__ __align__(16) float ob[SPB][RV];
     __shared__ float wts[4][kMaxGrid], wls[4][kMaxGrid];  // per warp: run weights and sums
-    __shared__ float coef[kFinishSeqs][3], scs[kFinishSeqs];
+    __shared__ float coef[SPB][3], scs[SPB];
     const int w = blockIdx.x, b0 = blockIdx.y * p.spb, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int nb = min(p.spb, p.B - b0);
@@ -756,9 +1196,9 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     const float muv = p.mu_v ? p.mu_v[th * kD + e] : 0.f;
     // the call's own inputs (not outputs of the earlier kernels) before the wait: each unit's
     // current-token score and value element e
-    float cv[kFinishSeqs];
+    float cv[SPB];
 #pragma unroll
-    for (int bi = 0; bi < kFinishSeqs; ++bi)
+    for (int bi = 0; bi < SPB; ++bi)
         cv[bi] = p.cur_v && bi < nb ? load_elem(p.cur_v, iorow(b0 + bi) * kD + e, p.io_bf16) : 0.f;
     if (p.cur_k) {
         for (int bi = warp; bi < nb; bi += 4) {
@@ -781,7 +1221,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     constexpr int NJ = (RV + 31) / 32;
     float *wt = wts[warp];
     float *wl = wls[warp];
-    for (int bi = grp; bi < kFinishSeqs; bi += 4 / G) {
+    for (int bi = grp; bi < SPB; bi += 4 / G) {
         if (bi >= nb) {
             for (int j = lane + 32 * sub; j < RV; j += 32 * G) ob[bi][j] = 0.f;
             continue;
@@ -852,13 +1292,13 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     }
     __syncthreads();
     // out_b[e] = coef0 (W_up^V o~_b)[e] + coef1 mu^V[e] + coef2 v_cur,b[e]
-    float acc[kFinishSeqs];
+    float acc[SPB];
 #pragma unroll
-    for (int bi = 0; bi < kFinishSeqs; ++bi) acc[bi] = 0.f;
+    for (int bi = 0; bi < SPB; ++bi) acc[bi] = 0.f;
     auto step = [&](int j8, const uint4 w4) {
         const float2 w0 = bf2_to_f2(w4.x), w1 = bf2_to_f2(w4.y), w2 = bf2_to_f2(w4.z), w3 = bf2_to_f2(w4.w);
 #pragma unroll
-        for (int bi = 0; bi < kFinishSeqs; ++bi) {
+        for (int bi = 0; bi < SPB; ++bi) {
             const float4 o0 = *reinterpret_cast<const float4 *>(&ob[bi][j8 * 8]);
             const float4 o1 = *reinterpret_cast<const float4 *>(&ob[bi][j8 * 8 + 4]);
             float a = acc[bi];
@@ -875,7 +1315,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
         for (int j8 = 0; j8 < RV / 8; ++j8) step(j8, W[j8]);
     }
 #pragma unroll
-    for (int bi = 0; bi < kFinishSeqs; ++bi) {
+    for (int bi = 0; bi < SPB; ++bi) {
         if (bi >= nb) break;
         const int64_t idx = iorow(b0 + bi) * kD + e;
         float v = acc[bi] * coef[bi][0] + coef[bi][1] * muv;
@@ -981,7 +1421,7 @@ lla_status launch_units(const DecodeArgs &a, bool loops, cudaStream_t stream) {
     fp.pstart = ap.pstart; fp.part = tp.part;
     // about two finish CTAs per SM: fewer sequences per CTA for small batches
     const int64_t want = static_cast<int64_t>(a.B) * nw;
-    fp.spb = static_cast<int>(std::min<int64_t>(kFinishSeqs, std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
+    fp.spb = static_cast<int>(std::min<int64_t>(finish_seqs(RV), std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
     return launch_ex(finish2d_kernel<RV, Z::NQM>, dim3(nw, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
 }
 
@@ -1044,7 +1484,8 @@ void rotary_phases(int d_rope, double base, unsigned long long *phi) {
 
 bool decode_2d_supported(int es, int d, int H, int r_k, int r_v) {
     return es == 2 && d == kD && H >= 1 && H <= kNQ &&
-           ((r_k == 96 && r_v == 160) || (r_k == 128 && r_v == 128) || (r_k == 288 && r_v == 480));
+           ((r_k == 96 && r_v == 160) || (r_k == 128 && r_v == 128) || (r_k == 288 && r_v == 480) ||
+            (r_k == 1152 && r_v == 1920));
 }
 
 size_t decode_2d_workspace_bytes(int r_k, int r_v, int B) {
@@ -1070,6 +1511,78 @@ lla_status launch_rope_key_store(int d_rope, double base, int pairing, void *rop
     return launch_ex(rope_key_store_kernel, dim3(static_cast<unsigned>((total + 255) / 256)), 256, 0, stream, rp);
 }
 
+namespace {
+
+// LLA-2D with latents too wide for whole-page stages: the absorb and finish kernels of
+// launch_units around attn2d_big_kernel.
+template <int RK, int RV>
+lla_status launch_big(const DecodeArgs &a, cudaStream_t stream) {
+    using Z = ZB<RK, RV>;
+    lla_status st = LLA_OK;
+    unsigned *err = device_error_word(&st);
+    if (st != LLA_OK) return st;
+    const int grid = num_sms();
+    if (grid <= 0 || grid > kMaxGrid) return LLA_ERR_UNSUPPORTED;
+    if (a.H < 1 || a.H > kNQ) return LLA_ERR_UNSUPPORTED;
+    if (static_cast<int64_t>(a.B) * ((static_cast<int64_t>(a.max_ctx) + kPT - 1) / kPT) >= (int64_t(1) << 31))
+        return LLA_ERR_UNSUPPORTED;
+    const WS2 w = ws2_layout(RK, RV, kNQ, a.B, grid);
+    if (a.workspace_bytes < w.total) return LLA_ERR_WORKSPACE;
+    char *ws = static_cast<char *>(a.workspace);
+    static bool configured[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
+    if (dev < 64 && !configured[dev]) {
+        if (cudaFuncSetAttribute(attn2d_big_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
+            cudaSuccess)
+            return LLA_ERR_CUDA;
+        configured[dev] = true;
+    }
+    const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
+    CUtensorMap tv;
+    const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT), static_cast<uint64_t>(a.num_blocks)};
+    const uint64_t strides[2] = {static_cast<uint64_t>(RV) * 2, static_cast<uint64_t>(page_bytes)};
+    const uint32_t box[3] = {64, kPT, 1};
+    if (!encode_tmap_bf16(&tv, static_cast<const char *>(a.pool) + kPT * RK * 2, 3, dims, strides, box, true))
+        return LLA_ERR_CUDA;
+
+    A2Params ap = {};
+    ap.T = a.T; ap.H = a.H; ap.loop = a.loop; ap.io_bf16 = a.io_bf16; ap.pass1 = a.cur_k != nullptr;
+    ap.B = a.B; ap.max_ctx = a.max_ctx; ap.max_blocks = a.max_blocks;
+    ap.loops = 0; ap.hu = 1;
+    ap.scale_log2 = a.scale * kLog2e;
+    ap.w_up_k = a.w_up_k; ap.mu_k = a.mu_k; ap.q = a.q; ap.context_lens = a.context_lens;
+    ap.qt = reinterpret_cast<float *>(ws + w.qt);
+    ap.beta = reinterpret_cast<float *>(ws + w.beta);
+    ap.pstart = reinterpret_cast<int *>(ws + w.pstart);
+    ap.err = err;
+    if ((st = launch_ex(absorb2d_kernel<RK, kNQ>, dim3(a.H, RK / 32, (a.B + 15) / 16), 256, 0, stream, ap)) != LLA_OK)
+        return st;
+    T2Params tp = {};
+    tp.nq = a.H; tp.U = a.B; tp.hu = 1;
+    tp.pool = static_cast<const char *>(a.pool);
+    tp.num_blocks = a.num_blocks; tp.page_bytes = page_bytes;
+    tp.block_table = a.block_table; tp.max_blocks = a.max_blocks;
+    tp.context_lens = a.context_lens;
+    tp.qt = ap.qt; tp.beta = ap.beta; tp.pstart = ap.pstart;
+    tp.part = reinterpret_cast<float *>(ws + w.part);
+    tp.err = err;
+    if ((st = launch_ex(attn2d_big_kernel<RK, RV>, dim3(grid), 256, Z::SMEM, stream, tv, tp)) != LLA_OK)
+        return st;
+    F2Params fp = {};
+    fp.T = a.T; fp.H = a.H; fp.loop = a.loop; fp.io_bf16 = a.io_bf16; fp.B = a.B; fp.grid = grid;
+    fp.loops = 0; fp.hu = 1; fp.U = a.B;
+    fp.scale_log2 = ap.scale_log2;
+    fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
+    fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
+    fp.pstart = ap.pstart; fp.part = tp.part;
+    const int64_t want = static_cast<int64_t>(a.B) * a.H;
+    fp.spb = static_cast<int>(std::min<int64_t>(finish_seqs(RV), std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
+    return launch_ex(finish2d_kernel<RV, kNQ>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
+}
+
+}  // namespace
+
 lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream) {
     if (a.B == 0) return LLA_OK;
     if (a.num_blocks >= (int64_t(1) << 31)) return LLA_ERR_UNSUPPORTED;  // 32-bit TMA coordinate
@@ -1079,6 +1592,7 @@ lla_status launch_decode_2d(const DecodeArgs &a, cudaStream_t stream) {
     LLA_2D(128, 128)
     LLA_2D(288, 480)
 #undef LLA_2D
+    if (a.r_k == 1152 && a.r_v == 1920) return launch_big<1152, 1920>(a, stream);
     return LLA_ERR_UNSUPPORTED;
 }
 

@@ -18,6 +18,11 @@ rho_2D = 2 T H d / (r_k + r_v) = 21.33 (Table isocache prints LLA-2D at this rat
 
   stress2d_rho2133  D=48, H=16, (288,480)  B=128, context ~ U[8192, 32768]
 
+and LLA-2D at rho_2D = 5.33 (also printed in Table isocache), (r_k, r_v) = (1152, 1920), on the
+Ouro-1.4B headline batch:
+
+  ouro14_2d_rho533  D=24, H=16, (1152,1920) B=16, context ~ U[2048, 4096]
+
 Recipe: activations, queries and current-token K/V are N(0,1); W_down is N(0, 1/(T d)) and
 W_up,t is N(0, 1/r) (std = 1/sqrt(.)); for LLA-2D W_down is N(0, 1/(T H d)) and W_up,t,h
 N(0, 1/r); mu = 0 unless asked for (then N(0,1)); seeds are the
@@ -73,6 +78,8 @@ WORKLOADS = {
                                lens=("uniform", 8192, 32768), seed=4),
     "stress2d_rho2133": Workload("stress2d_rho2133", D=48, H=16, d=128, T=4, r_k=288, r_v=480,
                                  B=128, lens=("uniform", 8192, 32768), seed=4, lla2d=True),
+    "ouro14_2d_rho533": Workload("ouro14_2d_rho533", D=24, H=16, d=128, T=4, r_k=1152, r_v=1920,
+                                 B=16, lens=("uniform", 2048, 4096), seed=1, lla2d=True),
 }
 
 

@@ -297,6 +297,13 @@ def test_2d_block_bytes_and_workspace_shapes(lib):
                 _g(lib, r_k=288, r_v=480, storage="fp32")):
         assert so.lla_decode_2d_workspace_size(ctypes.byref(bad), 4, ctypes.byref(n)) == UNSUPPORTED
     assert so.lla_decode_2d_workspace_size(ctypes.byref(g), -1, ctypes.byref(n)) == INVALID
+    # rho_2D = 5.33: 2D latents wider than the per-head limit of 512, up to T H d
+    wide = _g(lib, r_k=1152, r_v=1920)
+    assert so.lla_cache_2d_block_bytes(ctypes.byref(wide), ctypes.byref(n)) == OK
+    assert n.value == 64 * (1152 + 1920) * 2
+    assert so.lla_cache_block_bytes(ctypes.byref(wide), ctypes.byref(n)) == INVALID  # per-head: <= 512
+    too_wide = _g(lib, T=1, H=4, r_k=1152, r_v=1920)  # T H d = 512
+    assert so.lla_cache_2d_block_bytes(ctypes.byref(too_wide), ctypes.byref(n)) == INVALID
 
 
 def test_decode_2d_argument_checks(lib):

@@ -266,3 +266,31 @@ def test_full_size_stress2d_sampled(lla):
                                f64(q[b]), f64(ck[b]), f64(cv[b]), 1 / math.sqrt(w.d), heads=heads)
         assert_parity(got[b, heads], ref, "bf16", f"2D stress sequence {b}", io="bf16",
                       output_rounding=True)
+
+
+def test_large_latents_ragged_batch(lla):
+    """(1152, 1920), rho_2D = 5.33 (paper Table isocache): a 384 KB page streams through the
+    kernel in K-plane column chunks and V-plane row chunks; empty, one-token, page-aligned and
+    ragged sequences, with mu, both passes; the stored latents against the oracle's encode."""
+    sc = Scene2D(lla, H=16, r_k=1152, r_v=1920, io="bf16", lens=[0, 1, 63, 64, 65, 200], seed=76,
+                 with_mu=True)
+    for b in (1, 4, 5):
+        gk, gv = sc.gpu_latents(b)
+        assert_parity(gk, sc.ck[b], "bf16", "2D K latents")
+        assert_parity(gv, sc.cv[b], "bf16", "2D V latents")
+    _check(sc, 0, pass1=True)
+    sc.append_token()
+    _check(sc, 3, pass1=False)
+    assert lla.lla_get_device_error() == 0
+
+
+@pytest.mark.parametrize("lens", [[3000, 1100], [9000, 3000, 17]])
+def test_large_latents_split_across_ctas(lla, lens):
+    """Fewer and more pages than CTAs at (1152, 1920): runs of one sequence on many CTAs, merged
+    by the finish kernel; the oracle decodes the stored latents."""
+    sc = Scene2D(lla, H=16, r_k=1152, r_v=1920, io="bf16", lens=lens, seed=77, with_mu=True,
+                 oracle_encode=False)
+    _check(sc, 1, pass1=True)
+    sc.append_token()
+    _check(sc, 2, pass1=False)
+    assert lla.lla_get_device_error() == 0
