@@ -64,6 +64,10 @@ constexpr int kFinishSeqs = 8;   // most units per finish CTA (4 for latents wid
 constexpr int kMaxGrid = 256;    // attention CTAs (the runs of one unit fit one finish CTA)
 
 __host__ __device__ constexpr int finish_seqs(int rv) { return rv > 512 ? 4 : kFinishSeqs; }
+// Row slices of the output projection per finish CTA: wide latents split the d output rows of a
+// head over 4 CTAs, so that each reads a quarter of W_up,t,h^V (four threads per row reading
+// it in 64-byte runs) for all of its sequences, instead of every CTA reading all of it.
+__host__ __device__ constexpr int finish_slices(int rv) { return rv > 512 ? 4 : 1; }
 
 // Shared-memory plan of the attention kernel for ranks (RK, RV) and NQ query slots per unit
 // (16: the heads of an LLA-2D sequence; 4: the loops of a per-head (sequence, head)).  Offsets
@@ -1174,6 +1178,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
     constexpr bool kPre = RV <= 160;
     constexpr int SPB = finish_seqs(RV);
+    constexpr int RS = finish_slices(RV);
     constexpr int NW = kPre ? RV / 8 : 1;
     __shared__ __align__(16) float ob[SPB][RV];
     __shared__ float wts[4][kMaxGrid], wls[4][kMaxGrid];  // per warp: run weights and sums
@@ -1185,8 +1190,10 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     const int64_t th = p.loops ? static_cast<int64_t>(h) * p.T + t : static_cast<int64_t>(t) * p.H + h;
     const int qn = p.loops ? t : h;  // the query of (b, w) within its unit
     auto iorow = [&](int b) { return ((p.loops ? static_cast<int64_t>(t) * p.B : 0) + b) * p.H + h; };
-    // this thread's row e of W_up^V and mu^V (inputs of the call, not of earlier kernels)
-    const int e = tid;
+    // this thread's row e of W_up^V and mu^V (inputs of the call, not of earlier kernels); with
+    // row slices, four threads per row (part q4 of its 16-byte units)
+    const int e = RS == 1 ? tid : static_cast<int>(blockIdx.z) * (kD / RS) + (tid >> 2);
+    const int q4 = RS == 1 ? 0 : (tid & 3);
     const uint4 *W = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.w_up_v) + (th * kD + e) * RV);
     uint4 wr[NW];
     if constexpr (kPre) {
@@ -1310,13 +1317,23 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     if constexpr (kPre) {
 #pragma unroll
         for (int j8 = 0; j8 < NW; ++j8) step(j8, wr[j8]);  // fully unrolled: wr stays in registers
+    } else if constexpr (RS > 1) {
+        // a quarter of the row's 16-byte units (threads 4r .. 4r + 3 read 64 consecutive bytes),
+        // then the four partial sums of the row
+#pragma unroll 12
+        for (int j8 = q4; j8 < RV / 8; j8 += 4) step(j8, W[j8]);
+#pragma unroll
+        for (int bi = 0; bi < SPB; ++bi) {
+            acc[bi] += __shfl_xor_sync(0xffffffffu, acc[bi], 1);
+            acc[bi] += __shfl_xor_sync(0xffffffffu, acc[bi], 2);
+        }
     } else {
 #pragma unroll 4
         for (int j8 = 0; j8 < RV / 8; ++j8) step(j8, W[j8]);
     }
 #pragma unroll
     for (int bi = 0; bi < SPB; ++bi) {
-        if (bi >= nb) break;
+        if (bi >= nb || q4 != 0) break;
         const int64_t idx = iorow(b0 + bi) * kD + e;
         float v = acc[bi] * coef[bi][0] + coef[bi][1] * muv;
         if (p.cur_v) v = fmaf(coef[bi][2], cv[bi], v);
@@ -1576,9 +1593,10 @@ lla_status launch_big(const DecodeArgs &a, cudaStream_t stream) {
     fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
     fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
     fp.pstart = ap.pstart; fp.part = tp.part;
-    const int64_t want = static_cast<int64_t>(a.B) * a.H;
-    fp.spb = static_cast<int>(std::min<int64_t>(finish_seqs(RV), std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
-    return launch_ex(finish2d_kernel<RV, kNQ>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
+    // each CTA takes a quarter of a head's output rows for up to four sequences
+    fp.spb = std::min(finish_seqs(RV), a.B);
+    return launch_ex(finish2d_kernel<RV, kNQ>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb, finish_slices(RV)), 128, 0,
+                     stream, fp);
 }
 
 }  // namespace
