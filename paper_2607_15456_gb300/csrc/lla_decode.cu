@@ -169,13 +169,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const Params p) {
 
 template <int ES, int GK, int VB>
 lla_status launch_generic(const Params &prm, int grid, int smem, cudaStream_t stream) {
-    static bool configured[64] = {};
+    static DeviceOnce configured;
     return launch_kernel(decode_kernel<ES, GK, VB>, configured, prm, grid, smem, stream);
 }
 
 template <int ES, int RK, int RV>
 lla_status launch_fast(const Params &prm, int grid, int smem, cudaStream_t stream) {
-    static bool configured[64] = {};
+    static DeviceOnce configured;
     return launch_kernel(decode_async_kernel<ES, RK, RV, 128, 0>, configured, prm, grid, smem, stream,
                          kAsyncThreads);
 }

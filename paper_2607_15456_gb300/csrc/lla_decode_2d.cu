@@ -64,10 +64,12 @@ constexpr int kFinishSeqs = 8;   // most units per finish CTA (4 for latents wid
 constexpr int kMaxGrid = 256;    // attention CTAs (the runs of one unit fit one finish CTA)
 
 __host__ __device__ constexpr int finish_seqs(int rv) { return rv > 512 ? 4 : kFinishSeqs; }
-// Row slices of the output projection per finish CTA: wide latents split the d output rows of a
-// head over 4 CTAs, so that each reads a quarter of W_up,t,h^V (four threads per row reading
-// it in 64-byte runs) for all of its sequences, instead of every CTA reading all of it.
-__host__ __device__ constexpr int finish_slices(int rv) { return rv > 512 ? 4 : 1; }
+// Row slices of the output projection per finish CTA, for latents wider than 160: the d output
+// rows of a head split over 4 CTAs, so that each reads a quarter of W_up,t,h^V (four threads per
+// row reading it in 64-byte runs) for all of its sequences, instead of every CTA reading all of
+// it.  Latents wider than 512 always take them; narrower ones only when the batch leaves SMs
+// idle (a large batch keeps its finish to one wave of CTAs).
+__host__ __device__ constexpr int finish_slices(int rv) { return rv > 160 ? 4 : 1; }
 
 // Shared-memory plan of the attention kernel for ranks (RK, RV) and NQ query slots per unit
 // (16: the heads of an LLA-2D sequence; 4: the loops of a per-head (sequence, head)).  Offsets
@@ -1165,21 +1167,23 @@ __global__ void __launch_bounds__(256, 1)
 
 // ------------------------------------------------------------------------- finish kernel
 
-// Grid (weight slices, ceil(B / spb)), 128 threads (thread e = output element e).  spb (at most
-// 8) sequences share one pass over the slice's W_up^V; small batches take fewer per CTA to use
-// more SMs.  Slice w and sequence b give unit and query as in the absorb kernel.  The runs of a
-// unit are merged by one warp, or by two or four that split its columns when the CTA has fewer
-// than three units (no block barrier between units: each is a chain of dependent loads), then
-// all threads apply W_up^V; rows of W_up^V up to 160 wide are loaded before the wait on the
-// attention kernel.
-template <int RV, int NQM>
+// Grid (weight slices, ceil(B / spb), row slices), 128 threads (thread e = output element e,
+// or, with four row slices, threads 4r .. 4r + 3 = row r of the CTA's 32).  spb (at most 8)
+// sequences share one pass over the slice's W_up^V; small batches take fewer per CTA to use more
+// SMs.  Slice w and sequence b give unit and query as in the absorb kernel.  The runs of a unit
+// are merged by one warp, or by two or four that split its columns when the CTA has fewer than
+// three units (no block barrier between units: each is a chain of dependent loads), then all
+// threads apply W_up^V; a thread's weights, when they fit 80 registers (latents up to 640 wide),
+// are loaded before the wait on the attention kernel.
+template <int RV, int NQM, int RS>
 __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     constexpr int PS = NQM * RV + 2 * kNQ;
     constexpr int PO_M = NQM * RV, PO_L = NQM * RV + kNQ;
-    constexpr bool kPre = RV <= 160;
     constexpr int SPB = finish_seqs(RV);
-    constexpr int RS = finish_slices(RV);
-    constexpr int NW = kPre ? RV / 8 : 1;
+    static_assert(RS == 1 || RS == 4, "row slices");
+    static_assert(RS == 1 || (RV / 8) % RS == 0, "row slices read whole 16-byte units");
+    constexpr bool kPre = RV / 8 / RS <= 20;  // the thread's weights fit 80 registers
+    constexpr int NW = kPre ? RV / 8 / RS : 1;
     __shared__ __align__(16) float ob[SPB][RV];
     __shared__ float wts[4][kMaxGrid], wls[4][kMaxGrid];  // per warp: run weights and sums
     __shared__ float coef[SPB][3], scs[SPB];
@@ -1198,7 +1202,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     uint4 wr[NW];
     if constexpr (kPre) {
 #pragma unroll
-        for (int j8 = 0; j8 < NW; ++j8) wr[j8] = W[j8];
+        for (int j = 0; j < NW; ++j) wr[j] = W[q4 + RS * j];
     }
     const float muv = p.mu_v ? p.mu_v[th * kD + e] : 0.f;
     // the call's own inputs (not outputs of the earlier kernels) before the wait: each unit's
@@ -1226,6 +1230,7 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
     const int G = nb == 1 ? 4 : nb == 2 ? 2 : 1;
     const int grp = warp / G, sub = warp - grp * G;
     constexpr int NJ = (RV + 31) / 32;
+    constexpr int KR = NJ <= 16 ? 4 : NJ <= 32 ? 2 : 1;  // runs whose loads are in flight together
     float *wt = wts[warp];
     float *wl = wls[warp];
     for (int bi = grp; bi < SPB; bi += 4 / G) {
@@ -1263,16 +1268,26 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
             }
             l = warp_sum(ls);
             __syncwarp();
-            // every column load of a run in flight at once, runs four at a time
-#pragma unroll 4
-            for (int i = 0; i < nr; ++i) {
-                const float w8 = wt[i];
-                if (w8 > 0.f) {  // warp-uniform; a slot without a run is never read
-                    const float *pr = pu + static_cast<int64_t>(i) * PS + qn * RV;
+            // the column loads of KR runs in flight at once, then their sums: a slot between the
+            // unit's first and last CTA that holds no run (weight 0) is read, inside the
+            // workspace, but its values are never used
+            for (int i0 = 0; i0 < nr; i0 += KR) {
+                float v[KR][NJ];
+#pragma unroll
+                for (int k = 0; k < KR; ++k) {
+                    const float *pr = pu + static_cast<int64_t>(min(i0 + k, nr - 1)) * PS + qn * RV;
 #pragma unroll
                     for (int q = 0; q < NJ; ++q) {
                         const int j = lane + 32 * (sub + G * q);
-                        if (j < RV) acc[q] = fmaf(w8, pr[j], acc[q]);
+                        v[k][q] = j < RV ? pr[j] : 0.f;
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < KR; ++k) {
+                    const float w8 = i0 + k < nr ? wt[i0 + k] : 0.f;
+                    if (w8 > 0.f) {  // warp-uniform
+#pragma unroll
+                        for (int q = 0; q < NJ; ++q) acc[q] = fmaf(w8, v[k][q], acc[q]);
                     }
                 }
             }
@@ -1314,22 +1329,21 @@ __global__ void __launch_bounds__(128, 1) finish2d_kernel(const F2Params p) {
             acc[bi] = a;
         }
     };
+    // with row slices, a quarter of the row's 16-byte units (threads 4r .. 4r + 3 read 64
+    // consecutive bytes), then the four partial sums of the row
     if constexpr (kPre) {
 #pragma unroll
-        for (int j8 = 0; j8 < NW; ++j8) step(j8, wr[j8]);  // fully unrolled: wr stays in registers
-    } else if constexpr (RS > 1) {
-        // a quarter of the row's 16-byte units (threads 4r .. 4r + 3 read 64 consecutive bytes),
-        // then the four partial sums of the row
+        for (int j = 0; j < NW; ++j) step(q4 + RS * j, wr[j]);  // fully unrolled: wr stays in registers
+    } else {
 #pragma unroll 12
-        for (int j8 = q4; j8 < RV / 8; j8 += 4) step(j8, W[j8]);
+        for (int j8 = q4; j8 < RV / 8; j8 += RS) step(j8, W[j8]);
+    }
+    if constexpr (RS > 1) {
 #pragma unroll
         for (int bi = 0; bi < SPB; ++bi) {
             acc[bi] += __shfl_xor_sync(0xffffffffu, acc[bi], 1);
             acc[bi] += __shfl_xor_sync(0xffffffffu, acc[bi], 2);
         }
-    } else {
-#pragma unroll 4
-        for (int j8 = 0; j8 < RV / 8; ++j8) step(j8, W[j8]);
     }
 #pragma unroll
     for (int bi = 0; bi < SPB; ++bi) {
@@ -1384,15 +1398,8 @@ lla_status launch_units(const DecodeArgs &a, bool loops, cudaStream_t stream) {
     const WS2 w = ws2_layout(Z::RKX, RV, Z::NQM, U, grid);
     if (a.workspace_bytes < w.total) return LLA_ERR_WORKSPACE;
     char *ws = static_cast<char *>(a.workspace);
-    static bool configured[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(attn2d_kernel<RK, RV, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
-            cudaSuccess)
-            return LLA_ERR_CUDA;
-        configured[dev] = true;
-    }
+    static DeviceOnce configured;
+    if (raise_smem_limit(attn2d_kernel<RK, RV, NQ>, Z::SMEM, configured) != LLA_OK) return LLA_ERR_CUDA;
     const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
     // the V-planes of every page: [num_blocks * hu][64 tokens][r_v] bf16
     CUtensorMap tv;
@@ -1436,10 +1443,17 @@ lla_status launch_units(const DecodeArgs &a, bool loops, cudaStream_t stream) {
     fp.w_up_v = a.w_up_v; fp.mu_v = a.mu_v;
     fp.q = a.q; fp.cur_k = a.cur_k; fp.cur_v = a.cur_v; fp.out = a.out;
     fp.pstart = ap.pstart; fp.part = tp.part;
-    // about two finish CTAs per SM: fewer sequences per CTA for small batches
-    const int64_t want = static_cast<int64_t>(a.B) * nw;
+    // about two finish CTAs per SM: fewer sequences per CTA for small batches, and row slices
+    // when even one sequence per CTA leaves SMs idle
+    const int64_t units = static_cast<int64_t>(a.B) * nw;
+    const int rs = units <= 2 * grid ? finish_slices(RV) : 1;
+    const int64_t want = units * rs;
     fp.spb = static_cast<int>(std::min<int64_t>(finish_seqs(RV), std::max<int64_t>(1, (want + 2 * grid - 1) / (2 * grid))));
-    return launch_ex(finish2d_kernel<RV, Z::NQM>, dim3(nw, (a.B + fp.spb - 1) / fp.spb), 128, 0, stream, fp);
+    const dim3 fg(nw, (a.B + fp.spb - 1) / fp.spb, rs);
+    if constexpr (finish_slices(RV) > 1) {
+        if (rs > 1) return launch_ex(finish2d_kernel<RV, Z::NQM, finish_slices(RV)>, fg, 128, 0, stream, fp);
+    }
+    return launch_ex(finish2d_kernel<RV, Z::NQM, 1>, fg, 128, 0, stream, fp);
 }
 
 // ------------------------------------------------------------------------- rotary keys
@@ -1546,15 +1560,8 @@ lla_status launch_big(const DecodeArgs &a, cudaStream_t stream) {
     const WS2 w = ws2_layout(RK, RV, kNQ, a.B, grid);
     if (a.workspace_bytes < w.total) return LLA_ERR_WORKSPACE;
     char *ws = static_cast<char *>(a.workspace);
-    static bool configured[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(attn2d_big_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
-            cudaSuccess)
-            return LLA_ERR_CUDA;
-        configured[dev] = true;
-    }
+    static DeviceOnce configured;
+    if (raise_smem_limit(attn2d_big_kernel<RK, RV>, Z::SMEM, configured) != LLA_OK) return LLA_ERR_CUDA;
     const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
     CUtensorMap tv;
     const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT), static_cast<uint64_t>(a.num_blocks)};
@@ -1595,7 +1602,7 @@ lla_status launch_big(const DecodeArgs &a, cudaStream_t stream) {
     fp.pstart = ap.pstart; fp.part = tp.part;
     // each CTA takes a quarter of a head's output rows for up to four sequences
     fp.spb = std::min(finish_seqs(RV), a.B);
-    return launch_ex(finish2d_kernel<RV, kNQ>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb, finish_slices(RV)), 128, 0,
+    return launch_ex(finish2d_kernel<RV, kNQ, finish_slices(RV)>, dim3(a.H, (a.B + fp.spb - 1) / fp.spb, finish_slices(RV)), 128, 0,
                      stream, fp);
 }
 

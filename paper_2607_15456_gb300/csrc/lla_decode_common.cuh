@@ -1228,16 +1228,9 @@ __device__ void m_finish(const Params &p, const ASmem &a, const Run &R, int64_t 
 }
 
 template <typename Kern, typename Prm>
-lla_status launch_kernel(Kern kern, bool *configured, const Prm &prm, int grid, int smem,
+lla_status launch_kernel(Kern kern, DeviceOnce &configured, const Prm &prm, int grid, int smem,
                          cudaStream_t stream, int threads = kThreads) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit) !=
-            cudaSuccess)
-            return LLA_ERR_CUDA;
-        configured[dev] = true;
-    }
+    if (raise_smem_limit(kern, kSmemLimit, configured) != LLA_OK) return LLA_ERR_CUDA;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(threads);

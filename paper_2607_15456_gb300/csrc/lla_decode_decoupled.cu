@@ -16,7 +16,7 @@ namespace {
 
 template <int DR>
 lla_status launch_dec(const DecParams &dp, int grid, int smem, cudaStream_t stream) {
-    static bool configured[64] = {};
+    static DeviceOnce configured;
     return launch_kernel(decode_async_kernel<2, 96, 160, 128, DR>, configured, dp, grid, smem, stream,
                          kAsyncThreads);
 }

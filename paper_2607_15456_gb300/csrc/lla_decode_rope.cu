@@ -480,7 +480,7 @@ __global__ void __launch_bounds__(kRopeThreads, 1) decode_rope_kernel(const __gr
 
 template <int RK, int RV>
 lla_status launch_rope(const RopeParams &prm, int grid, int smem, cudaStream_t stream) {
-    static bool configured[64] = {};
+    static DeviceOnce configured;
     return launch_kernel(decode_rope_kernel<RK, RV>, configured, prm, grid, smem, stream,
                          kRopeThreads);
 }

@@ -837,15 +837,8 @@ lla_status launch_tc(const DecodeArgs &a, const RopeTables &tab, int pairing, cu
     if (static_cast<int64_t>(a.B) * a.H * ((static_cast<int64_t>(a.max_ctx) + kPT - 1) / kPT) >= (int64_t(1) << 31))
         return LLA_ERR_UNSUPPORTED;  // the units' pages are numbered in 32 bits
     if (a.workspace_bytes < decode_rope_tc_workspace_bytes(RV, a.B, a.H, grid)) return LLA_ERR_WORKSPACE;
-    static bool configured[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(rope_tc_kernel<RK, RV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Z::SMEM) !=
-            cudaSuccess)
-            return LLA_ERR_CUDA;
-        configured[dev] = true;
-    }
+    static DeviceOnce configured;
+    if (raise_smem_limit(rope_tc_kernel<RK, RV>, Z::SMEM, configured) != LLA_OK) return LLA_ERR_CUDA;
     const int64_t page_bytes = static_cast<int64_t>(head_page_bytes(RK, RV, 2));
     // the V-planes of every head page: [num_blocks * H][64 tokens][r_v] bf16
     CUtensorMap tv, tw;

@@ -310,27 +310,17 @@ lla_status launch(K kern, dim3 grid, dim3 block, int smem, cudaStream_t stream, 
 }
 
 template <int ES>
-lla_status set_smem_layers(int dev) {
-    static bool configured[64] = {};
-    if (dev < 64 && configured[dev]) return LLA_OK;
-    if (cudaFuncSetAttribute(encode_layers_kernel<ES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kXsBudget + 2 * kWBuf + kKSlices * kMaxTileTokens * kColTile * 4) !=
-        cudaSuccess)
-        return LLA_ERR_CUDA;
-    if (dev < 64) configured[dev] = true;
-    return LLA_OK;
+lla_status set_smem_layers() {
+    static DeviceOnce configured;
+    return raise_smem_limit(encode_layers_kernel<ES>, kXsBudget + 2 * kWBuf + kKSlices * kMaxTileTokens * kColTile * 4,
+                            configured);
 }
 
 template <int ES>
-lla_status set_smem(int dev) {
-    static bool configured[64] = {};
-    if (dev < 64 && configured[dev]) return LLA_OK;
-    if (cudaFuncSetAttribute(encode_kernel<ES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kXsBudget + 2 * kWBuf + kKSlices * kMaxTileTokens * kColTile * 4) !=
-        cudaSuccess)
-        return LLA_ERR_CUDA;
-    if (dev < 64) configured[dev] = true;
-    return LLA_OK;
+lla_status set_smem() {
+    static DeviceOnce configured;
+    return raise_smem_limit(encode_kernel<ES>, kXsBudget + 2 * kWBuf + kKSlices * kMaxTileTokens * kColTile * 4,
+                            configured);
 }
 
 }  // namespace
@@ -371,9 +361,7 @@ lla_status launch_encode_layers(const EncodeArgs *a, int L, cudaStream_t stream)
     p.nbuf = Td > (es == 2 ? chunk_rows<2>() : chunk_rows<4>()) ? 2 : 1;
     const int ctiles_v = (a0.r_v + kColTile - 1) / kColTile;
     const int smem = (tile * Td + kKSlices * tile * kColTile) * 4 + p.nbuf * kWBuf;
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    st = es == 2 ? set_smem_layers<2>(dev) : set_smem_layers<4>(dev);
+    st = es == 2 ? set_smem_layers<2>() : set_smem_layers<4>();
     if (st != LLA_OK) return st;
     if (static_cast<int64_t>(a0.H) * L > 65535) return LLA_ERR_UNSUPPORTED;
     const dim3 grid((a0.N + tile - 1) / tile, p.ctiles_k + ctiles_v, a0.H * L), block(kThreads);
@@ -425,9 +413,7 @@ lla_status launch_encode(const EncodeArgs &a, cudaStream_t stream) {
     p.nbuf = Td > (es == 2 ? chunk_rows<2>() : chunk_rows<4>()) ? 2 : 1;
     const int ctiles_v = (a.r_v + kColTile - 1) / kColTile;
     const int smem = (tile * Td + kKSlices * tile * kColTile) * 4 + p.nbuf * kWBuf;
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    st = es == 2 ? set_smem<2>(dev) : set_smem<4>(dev);
+    st = es == 2 ? set_smem<2>() : set_smem<4>();
     if (st != LLA_OK) return st;
     if (a.H > 65535) return LLA_ERR_UNSUPPORTED;
     const dim3 grid((a.N + tile - 1) / tile, p.ctiles_k + ctiles_v, a.H), block(kThreads);

@@ -399,15 +399,8 @@ lla_status launch_encode_tc(const EncodeArgs &a, cudaStream_t stream) {
     p.err = err;
     CUtensorMap txk, txv, twk, twv;
     if (!make_maps(a, 0, &txk, &twk) || !make_maps(a, 1, &txv, &twv)) return LLA_ERR_CUDA;
-    static bool configured[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(encode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem) !=
-            cudaSuccess)
-            return LLA_ERR_CUDA;
-        configured[dev] = true;
-    }
+    static DeviceOnce configured;
+    if (raise_smem_limit(encode_tc_kernel, kSmem, configured) != LLA_OK) return LLA_ERR_CUDA;
     const int sms = num_sms();
     if (sms <= 0) return LLA_ERR_CUDA;
     cudaLaunchConfig_t cfg = {};

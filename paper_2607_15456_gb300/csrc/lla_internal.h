@@ -5,6 +5,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/lla.h"
 
 namespace lla {
@@ -135,6 +137,26 @@ lla_status launch_rope_key_store(int d_rope, double base, int pairing, void *rop
                                  int N, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached), 0 on failure
+
+// Per-device flags of a one-time kernel set-up.  Host threads that race on a first call both
+// make the same set-up call; each flag is atomic.
+struct DeviceOnce {
+    std::atomic<bool> done[64];
+};
+
+// Raises the dynamic shared-memory limit of `kern` to `bytes` on the current device, once per
+// device (a flag in `once`).
+template <typename K>
+inline lla_status raise_smem_limit(K kern, int bytes, DeviceOnce &once) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
+    const bool cached = dev >= 0 && dev < 64;
+    if (cached && once.done[dev].load(std::memory_order_acquire)) return LLA_OK;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+        return LLA_ERR_CUDA;
+    if (cached) once.done[dev].store(true, std::memory_order_release);
+    return LLA_OK;
+}
 
 // The limit of each pipeline wait in lla_decode_attn / lla_dense_decode_attn launches, as set by
 // lla_set_wait_limit_ns (0: the kernels' own 2 s).

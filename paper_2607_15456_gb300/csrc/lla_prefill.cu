@@ -982,15 +982,8 @@ lla_status launch_pf(K kern, dim3 grid, int threads, int smem, cudaStream_t stre
 
 template <int RK, int RV, bool ROPE = false>
 lla_status launch_tc(const PParams &prm, int nqt, int B, int H, cudaStream_t stream) {
-    static bool configured[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(prefill_tc_kernel<RK, RV, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 PF<RK, RV, ROPE>::SMEM) != cudaSuccess)
-            return LLA_ERR_CUDA;
-        configured[dev] = true;
-    }
+    static DeviceOnce configured;
+    if (raise_smem_limit(prefill_tc_kernel<RK, RV, ROPE>, PF<RK, RV, ROPE>::SMEM, configured) != LLA_OK) return LLA_ERR_CUDA;
     // the V-planes of every head page: [pages][64 tokens][r_v] bf16, one page = one head page
     CUtensorMap tv;
     const uint64_t dims[3] = {static_cast<uint64_t>(RV), static_cast<uint64_t>(kPT),
@@ -1077,15 +1070,8 @@ bool prefill_rope_supported(int es, int d, int r_k, int r_v) {
 namespace {
 template <int RK>
 lla_status launch_rebuild(const RParams &rp, int kpps, int B, cudaStream_t stream) {
-    static bool configured[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return LLA_ERR_CUDA;
-    if (dev < 64 && !configured[dev]) {
-        if (cudaFuncSetAttribute(rope_rebuild_kernel<RK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 RB<RK>::SMEM) != cudaSuccess)
-            return LLA_ERR_CUDA;
-        configured[dev] = true;
-    }
+    static DeviceOnce configured;
+    if (raise_smem_limit(rope_rebuild_kernel<RK>, RB<RK>::SMEM, configured) != LLA_OK) return LLA_ERR_CUDA;
     // heads split over a few CTAs per page, so that more CTAs hide each other's load latency
     const int groups = rp.H >= 8 ? 4 : 1;
     return launch_pf(rope_rebuild_kernel<RK>, dim3(kpps, B, groups), 128, RB<RK>::SMEM, stream, rp);

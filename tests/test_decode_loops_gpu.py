@@ -95,10 +95,13 @@ def test_fewer_loops_than_query_slots(lla, T):
     _check(sc, pass1=False, tight=True)
 
 
-def test_many_short_sequences_and_determinism(lla):
+@pytest.mark.parametrize("rk,rv", [(96, 160), (192, 320)])
+def test_many_short_sequences_and_determinism(lla, rk, rv):
+    """200 sequences x 2 heads x 4 loops: many runs per CTA; at (192, 320) a batch this large
+    takes the finish without row slices, the small batches above take it with them."""
     g = torch.Generator().manual_seed(53)
     lens = [int(v) for v in torch.randint(1, 141, (200,), generator=g)]
-    sc = Scene(lla, H=2, lens=lens, io="bf16", seed=53)
+    sc = Scene(lla, H=2, r_k=rk, r_v=rv, lens=lens, io="bf16", seed=53)
     pairs = [(b, h) for b in range(0, 200, 7) for h in range(2)]
     _check(sc, pass1=True, pairs=pairs, single=False)
     a = _run_loops(sc, True)[3].clone()
