@@ -26,11 +26,15 @@ or lla_decode_attn_decoupled (rotary planes of d_rope = 64 stored first, one per
     ncu --set full --clock-control none -k regex:attn2d_kernel -s 2 -c 1 \\
         python profile_case.py --case decoupled --workload ouro14_rho4 --layers 2 --calls 10
 
-2d: LLA-2D on the stress2d workload's shape with `--batch` sequences (random latents written into
-two layers' pages; --batch 32 keeps a layer near 1 GB, above L2):
+2d: LLA-2D on an LLA-2D workload's shape (`--workload2d`, the stress2d workload by default) with
+`--batch` sequences (random latents written into two layers' pages; --batch 32 keeps a stress2d
+layer near 1 GB, above L2; the (1152, 1920) workload's 16 sequences take 351 MB a layer):
 
     ncu --set full --clock-control none -k regex:attn2d_kernel -s 2 -c 1 \\
         python profile_case.py --case 2d --batch 32 --calls 8
+    ncu --section SpeedOfLight --section MemoryWorkloadAnalysis --clock-control none \\
+        -k regex:attn2d_big_kernel -s 2 -c 1 \\
+        python profile_case.py --case 2d --workload2d ouro14_2d_rho533 --batch 16 --calls 6
 
 prefill: encodes `--prompts` prompts of `--len` tokens of a workload's ranks (tensor-core encode,
 one launch per axis), then runs `--calls` causal prefill calls over them:
@@ -116,7 +120,9 @@ def case_2d(args):
 
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    w = W.WORKLOADS["stress2d_rho2133"]
+    w = W.WORKLOADS[args.workload2d]
+    if not w.lla2d:
+        raise SystemExit(f"{args.workload2d} is not an LLA-2D workload")
     lens = W.context_lengths(w, B=args.batch)
     pt = W.page_table(lens, w.seed, extra_tokens=1)
     table = pt.block_table.to(dev)
@@ -194,6 +200,7 @@ def main():
     ap.add_argument("--case", choices=["decode", "rope", "loops", "decoupled", "2d", "prefill", "rope_prefill"],
                     default="decode")
     ap.add_argument("--workload", default="ouro14_rho4")
+    ap.add_argument("--workload2d", default="stress2d_rho2133", help="the LLA-2D workload of --case 2d")
     ap.add_argument("--layers", type=int, default=2)
     ap.add_argument("--calls", type=int, default=10)
     ap.add_argument("--prompts", type=int, default=4)
