@@ -638,8 +638,9 @@ def run_2d_extra(device):
 def run_extras(device):
     """The other rows of the hot path on their own workloads, each against its roofline:
     causal prefill attention and the encode of a prefilled prompt (Ouro-1.4B at rho = 2,
-    4 prompts of 8192 tokens, one layer and loop per call), and the uncompressed loop-t decode
-    comparator on the headline batch (D x T calls over plain K/V pages of d = 128)."""
+    4 prompts of 8192 tokens, one layer and loop per call), the same prompts' prefill at the
+    headline workload's ranks (rho = 4), and the uncompressed loop-t decode comparator on the
+    headline batch (D x T calls over plain K/V pages of d = 128)."""
     import torch
     from paper_2607_15456_gb300 import lla
     from paper_2607_15456_gb300 import workloads as W
@@ -708,7 +709,28 @@ def run_extras(device):
         "frac": rp_flops / (rp_ms / 1e3) / 1e12 / tc_peak, "flops_per_call": rp_flops,
         "note": "flops: 2 (d + r_v) per causal (query, key) pair, the key rebuild 2 d r_k and the "
                 "output projection 2 d r_v per (token, head)"}
-    del q, o, pool, cache, ws
+    del pool, cache, ws
+    # the same prompts at the headline workload's ranks (rho = 4, (96, 160)): encoded, then the
+    # causal prefill over them
+    w4 = W.WORKLOADS["ouro14_rho4"]
+    geom4 = lla.Geometry(T, H, d, w4.r_k, w4.r_v, "bf16")
+    codec4 = lla.Codec(**W.codec_tensors(T, H, d, w4.r_k, w4.r_v, w4.seed, 0, device=device))
+    pool = torch.zeros(pt.num_blocks * lla.lla_cache_block_bytes(geom4), dtype=torch.uint8, device=device)
+    cache = lla.Cache(pool, pt.num_blocks, pt.block_table.to(device), pt.max_blocks)
+    xk = W.normal((T, N, H, d), w4.seed, 300, device=device)
+    xv = W.normal((T, N, H, d), w4.seed, 301, device=device)
+    lla.lla_encode(geom4, codec4, cache, xk, xv, slots)
+    del xk, xv
+    p4_ms = _time_ms(lambda: lla.lla_prefill_attn(geom4, codec4, cache, cu, L, 1, q, o))
+    p4_flops = pairs * 2 * (w4.r_k + w4.r_v) + N * H * 2 * d * (w4.r_k + w4.r_v)
+    out["prefill_rho4"] = {
+        "workload": f"{nseq}x{L}-token prompts at {w4.name}'s ranks (r_k, r_v)=({w4.r_k}, {w4.r_v}), "
+                    f"H={H}, one layer and loop",
+        "kernel": "prefill_tc_kernel (lla_prefill_attn)", "bound": "tensor",
+        "ms_per_call": p4_ms, "tokens_per_s": N / (p4_ms / 1e3),
+        "TFLOP_s": p4_flops / (p4_ms / 1e3) / 1e12, "peak_TFLOP_s": tc_peak,
+        "frac": p4_flops / (p4_ms / 1e3) / 1e12 / tc_peak, "flops_per_call": p4_flops}
+    del q, o, pool, cache
 
     # comparator: plain loop-t K/V of the headline batch, d = 128
     w = W.WORKLOADS["ouro14_rho4"]
