@@ -465,7 +465,11 @@ __global__ void __launch_bounds__(kT2, 1)
                 }
                 ++r;
             }
-            // the softmax warps wait for every S^T product (its full barrier) before they finish
+            // every product has completed before TMEM is released, even after an abort (when the
+            // softmax warps stop waiting for them): the last commit on each S^T buffer
+            volatile int never = 0;
+            for (int j = max(0, it - 2); j < it; ++j)
+                mbar_wait(&bar[bSfull + (j & 1)], (j >> 1) & 1, &never, p.err);
         }
         __syncwarp();
     } else if (warp == kPvWarp) {
@@ -957,6 +961,11 @@ __global__ void __launch_bounds__(256, 1)
                 }
                 ++r;
             }
+            // every product has completed before TMEM is released, even after an abort: the last
+            // commit on each S^T buffer
+            volatile int never = 0;
+            for (int j = max(0, it - 2); j < it; ++j)
+                mbar_wait(&bar[cSfull + (j & 1)], (j >> 1) & 1, &never, p.err);
         }
         __syncwarp();
     } else if (warp == 6) {

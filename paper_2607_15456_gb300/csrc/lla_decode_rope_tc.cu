@@ -368,7 +368,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 umma_commit(&bar[bAfree]);
                 ++r;
             }
-            // the rotation groups wait for every key product before they finish
+            // every key product has completed before TMEM is released, even after an abort (when
+            // the rotation groups stop waiting for them): the last commit on each accumulator
+            volatile int never = 0;
+            for (int j = max(0, it - kNAcc); j < it; ++j)
+                mbar_wait(&bar[bTfull + j % kNAcc], (j / kNAcc) & 1, &never, p.err);
         }
         __syncwarp();
     } else if (warp == kWVal) {

@@ -212,6 +212,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
         mbar_arrive(&bar[kBSetup]);
         if (lane == 0) {  // K-planes: one bulk copy per page
             const uint64_t pol = policy_evict_first();
+            int nk = 0;  // copies issued
             for (int j = 0; j < NP; ++j) {
                 const int s = j % F::STK;
                 const uint32_t ph = (j / F::STK) & 1;
@@ -224,10 +225,16 @@ __global__ void __launch_bounds__(kPThreads, 1)
                 // the latent K-plane of the page, or its rebuilt and rotated keys
                 const char *src = ROPE ? p.krot + ((static_cast<int64_t>(b) * p.kpps + j) * p.H + h) * F::KPAGE
                                        : p.pool + hp * p.head_page_bytes;
-                mbar_wait(&bar[kBKempty + s], ph ^ 1u, abort_flag, p.err);
+                if (!mbar_wait(&bar[kBKempty + s], ph ^ 1u, abort_flag, p.err) || *abort_flag) break;
                 mbar_arrive_expect_tx(&bar[kBKfull + s], F::KPAGE);
                 bulk_g2s(sm + F::oK + s * F::KPAGE, src, F::KPAGE, &bar[kBKfull + s], pol);
+                ++nk;
             }
+            // every copy has landed before the ring is reused or the CTA exits, even after an
+            // abort (no copy is issued once a wait has failed)
+            volatile int never = 0;
+            for (int j = max(0, nk - F::STK); j < nk; ++j)
+                mbar_wait(&bar[kBKfull + j % F::STK], (j / F::STK) & 1, &never, p.err);
         }
         __syncwarp();
         // epilogue operand W_up,t^V [d][r_v] (K-major): (row e, chunk c) at c*(d*16) + e*16,
@@ -247,19 +254,24 @@ __global__ void __launch_bounds__(kPThreads, 1)
         if (lane == 0) {  // V-planes: one TMA tensor load with 128-byte swizzle per 64 columns
             // the V ring aliases the prologue operands: wait until Q~ has been computed
             mbar_wait(&bar[kBQt], 0, abort_flag, p.err);
+            int nv = 0;  // copies issued
             for (int j = 0; j < NP; ++j) {
                 const int s = j % F::STV;
                 const uint32_t ph = (j / F::STV) & 1;
                 int32_t blk = bt[j];
                 if (blk < 0 || blk >= p.num_blocks) blk = 0;  // flagged by the K producer
                 const int64_t hp = static_cast<int64_t>(blk) * p.H + h;
-                mbar_wait(&bar[kBVempty + s], ph ^ 1u, abort_flag, p.err);
+                if (!mbar_wait(&bar[kBVempty + s], ph ^ 1u, abort_flag, p.err) || *abort_flag) break;
                 mbar_arrive_expect_tx(&bar[kBVfull + s], F::VPAGE);
                 char *vs = sm + F::oV + s * F::VPAGE;
 #pragma unroll
                 for (int a = 0; a < F::VATOMS; ++a)
                     tma_load_3d(vs + a * (kPT * 128), &tv, a * 64, 0, static_cast<int>(hp), &bar[kBVfull + s]);
+                ++nv;
             }
+            volatile int never = 0;  // as for the K ring
+            for (int j = max(0, nv - F::STV); j < nv; ++j)
+                mbar_wait(&bar[kBVfull + j % F::STV], (j / F::STV) & 1, &never, p.err);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -299,6 +311,14 @@ __global__ void __launch_bounds__(kPThreads, 1)
                 umma_commit(&bar[kBSfull + s]);
                 umma_commit(&bar[kBKempty + sk]);
             }
+            // every product of this thread has completed before TMEM is released, even after an
+            // abort (when the softmax warps stop waiting for them): a commit tracks all earlier
+            // products of its thread, so the last one suffices
+            volatile int never = 0;
+            if (NP > 0)
+                mbar_wait(&bar[kBSfull + ((NP - 1) & 1)], ((NP - 1) >> 1) & 1, &never, p.err);
+            else if constexpr (!ROPE)
+                mbar_wait(&bar[kBQt], 0, &never, p.err);
         }
         __syncwarp();
     } else if (warp == 3) {
@@ -345,6 +365,8 @@ __global__ void __launch_bounds__(kPThreads, 1)
                     umma_bf16(tmem + 0, doa + ks * (4096 >> 4), dwv + ks * (4096 >> 4), ido, part > 0 || ks > 0);
                 umma_commit(&bar[part ? kBOut : kBOut1]);
             }
+            volatile int never = 0;  // as for the S^T issuer: the last commit of this thread
+            mbar_wait(&bar[kBOut], 0, &never, p.err);
         }
         __syncwarp();
     } else {
