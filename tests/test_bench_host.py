@@ -25,3 +25,30 @@ def test_failing_extra_is_reported_and_the_others_kept():
     assert result["value"] == 1.0
     assert "RuntimeError: device error" in result["extra_errors"]["b"]
     json.dumps(result)  # still one JSON line
+
+
+def test_reference_arm_line_on_the_host_cores():
+    """The reference arm (the oracle on the host cores, one bounded sample per timed step) prints
+    the contract's keys, the same config dict as the GPU arm, no host/device copies, and a step
+    time that is the time it actually measured."""
+    import argparse
+
+    from paper_2607_15456_gb300 import workloads as W
+
+    args = argparse.Namespace(workload="ouro14_rho4", steps=1, warmup=0, cpu_seconds=2.0)
+    line = bench.run_reference(args, 0, 1)
+    json.dumps(line)
+    w = W.WORKLOADS["ouro14_rho4"]
+    lens = W.context_lengths(w)
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC
+    assert line["config"] == bench.config_dict(w, lens, 1)
+    assert line["unit"] == "tokens/s" and line["higher_is_better"] is True
+    assert line["steps"] == 1 and line["warmup"] == 0 and line["extrapolated"] is True
+    assert line["value"] > 0 and line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
+    # steps x ms_per_step is measured time, within the arm's own wall clock
+    assert 0 < line["ms_per_step"] * line["steps"] / 1e3 <= line["wall_seconds"] * 1.01
+    # the extrapolated full step is longer than the sample it came from
+    assert line["full_step_seconds_extrapolated"] > line["ms_per_step"] / 1e3
