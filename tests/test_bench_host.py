@@ -52,3 +52,29 @@ def test_reference_arm_line_on_the_host_cores():
     assert 0 < line["ms_per_step"] * line["steps"] / 1e3 <= line["wall_seconds"] * 1.01
     # the extrapolated full step is longer than the sample it came from
     assert line["full_step_seconds_extrapolated"] > line["ms_per_step"] / 1e3
+
+
+def test_algorithmic_bytes_per_decode_launch():
+    """The roofline's numerator: one decode launch reads every cached token's latents of every
+    head once ((r_k + r_v) bf16 values), this loop's W_up^K and W_up^V, and q, k_cur, v_cur, out.
+    On the headline batch (H = 16, (96, 160), sum of contexts 54987) that is
+    16 * 256 * 2 * 54987 + 16 * 128 * 256 * 2 + 4 * 16 * 16 * 128 * 2 = 451,764,224 bytes; the
+    committed DRAM counters are compared with the same figure for each workload."""
+    from types import SimpleNamespace
+
+    from paper_2607_15456_gb300 import workloads as W
+
+    with open(os.path.join(ROOT, "profiles", "decode_traffic.json")) as f:
+        traffic = json.load(f)
+    w = W.WORKLOADS["ouro14_rho4"]
+    lens = W.context_lengths(w)
+    assert sum(lens) == 54987 and len(lens) == 16
+    head = SimpleNamespace(w=w, lens=lens, B=len(lens))
+    assert bench.DecodeBench.decode_bytes_per_launch(head) == 451_764_224
+    for name, entry in traffic.items():
+        w = W.WORKLOADS[name]
+        lens = W.context_lengths(w)
+        ns = SimpleNamespace(w=w, lens=lens, B=len(lens))
+        assert bench.DecodeBench.decode_bytes_per_launch(ns) == entry["algorithmic_bytes_per_launch"], name
+        # the measured traffic is within a few percent above the algorithmic bytes: no re-reads
+        assert 1.0 <= entry["dram_bytes_per_launch"] / entry["algorithmic_bytes_per_launch"] < 1.05, name
