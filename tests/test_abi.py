@@ -42,6 +42,12 @@ def test_library_exports_every_declared_symbol(lib):
     assert not missing, missing
 
 
+def test_binding_has_every_declared_entry_point(lib):
+    """The Python binding carries the C names: one callable per declared function."""
+    missing = [n for n in declared_functions() if not callable(getattr(lib, n, None))]
+    assert not missing, missing
+
+
 def test_wait_limit_is_a_host_setting(lib):
     """The pipeline wait limit is kept on the host (no GPU call): 0 means the 2 s default."""
     assert lib.lla_get_wait_limit_ns() == 2_000_000_000
