@@ -33,8 +33,11 @@
 //                       warps 2-5  per page: the scores of 16 tokens per warp, the maxima over
 //                                  the page per query, P^T as a bf16 operand, the lazy O^T
 //                                  rescale; per run: the partial out to the workspace
-//   finish2d_kernel   per (query slice, up to 8 units): merges the runs of each unit, adds the
-//                     pass-1 current token, and applies W_up,n^V once for those units
+//   finish2d_kernel   per (query slice, up to 8 units, and for small batches or wide latents a
+//                     quarter of the output rows): merges the runs of each unit, adds the pass-1
+//                     current token, and applies W_up,n^V once for those units
+//   attn2d_big_kernel replaces attn2d_kernel for latents wider than a page stage ((1152, 1920)):
+//                     pages stream as K-plane column chunks and V-plane row chunks
 // Storage bf16, d = 128; accumulators fp32 in TMEM.
 #include <cuda_runtime.h>
 
